@@ -1,0 +1,26 @@
+"""CPU oracle of the counter-causal refresh (arXiv 2607.27600) -- TEST INFRASTRUCTURE.
+
+Plain fp64 numpy restatement of the scoring, keep-set selection and
+compaction the paper defines.  Only tests/, __graft_entry__.smoke() and the
+CPU legs of bench.py may import it.  It shares no code with the CUDA path.
+
+Parity status per function (what pins it, in tests/test_oracle_*.py):
+  rms_norm                 torch rms_norm (library routine)
+  rope                     complex-multiplication identity; relative-position property
+  counter_causal_attention torch SDPA with an explicit mask (library routine);
+                           closed forms (row n-2 -> V[n-1], K = 0 -> mean of later V,
+                           last row -> 0); brute force on tiny inputs
+  causal_attention         torch SDPA is_causal (library routine)
+  swiglu_mlp               hand-computed scalar case
+  score_head               closed form; scipy log_softmax (library routine)
+  score_layer/score_full   closed-form special cases, mask-leakage, prefix-drop,
+                           batch/ragged, GQA-permutation, RoPE-shift and L=1
+                           (full == single-layer) invariants
+  select_keep              brute-force sort on tiny inputs; forced keeps; identity
+  compact                  sequential in-place loop; order preservation
+The paper prints no worked example with score values, so no pin is a
+printed number; every step of the score is pinned by the checks above.
+"""
+from .refresh import (rms_norm, rope, rope_angles, softmax, counter_causal_attention,  # noqa: F401
+                      causal_attention, silu, swiglu_mlp, counter_causal_layer, score_head,
+                      score_layer, score_full, select_keep, compact, causal_forward)

@@ -1,0 +1,109 @@
+"""Pins of the oracle's keep-set selection and compaction (Algorithm
+DoMemRefresh) by brute force and invariants (no GPU)."""
+import numpy as np
+import pytest
+
+import oracle
+
+
+def brute_keep(scores, n, budget, n_sink):
+    """Python sort of (score, slot) descending; NaN -> -inf; sinks -> +inf."""
+    items = []
+    for j in range(n):
+        s = float(scores[j])
+        if s != s:
+            s = float("-inf")
+        if j < n_sink:
+            s = float("inf")
+        items.append((s, j))
+    items.sort(reverse=True)
+    return sorted(j for _, j in items[:min(budget, n)])
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_select_matches_brute_force_with_ties(seed):
+    r = np.random.default_rng(seed)
+    b, cap = 3, 40
+    scores = r.integers(-3, 4, size=(b, cap)).astype(np.float32)   # many ties
+    scores[0, 5] = np.nan
+    scores[1, 7] = np.inf
+    scores[2, 0] = -np.inf
+    lens = [40, 17, 1]
+    budget = [11, 17, 1]
+    n_sink = seed % 3
+    idx, cnt = oracle.select_keep(scores, lens, budget, n_sink)
+    for bi in range(b):
+        want = brute_keep(scores[bi], lens[bi], budget[bi], n_sink)
+        assert cnt[bi] == len(want)
+        assert idx[bi, :cnt[bi]].tolist() == want
+        assert np.all(idx[bi, cnt[bi]:] == -1)
+
+
+def test_select_identity_when_budget_covers_sequence():
+    s = np.random.default_rng(1).normal(size=(2, 9)).astype(np.float32)
+    idx, cnt = oracle.select_keep(s, [9, 5], [9, 100], 0)
+    assert cnt.tolist() == [9, 5]
+    assert idx[0].tolist() == list(range(9)) and idx[1, :5].tolist() == list(range(5))
+
+
+def test_select_ties_prefer_later_slot_and_keep_sinks():
+    s = np.zeros((1, 8), np.float32)
+    idx, cnt = oracle.select_keep(s, [8], [3], n_sink=0)
+    assert idx[0, :3].tolist() == [5, 6, 7]
+    idx, cnt = oracle.select_keep(s, [8], [3], n_sink=2)
+    assert idx[0, :3].tolist() == [0, 1, 7]
+
+
+def test_select_keeps_highest_exactly():
+    s = np.array([[0.5, 3.0, -1.0, 2.0, 2.5, -7.0]], np.float32)
+    idx, cnt = oracle.select_keep(s, [6], [3])
+    assert idx[0, :3].tolist() == [1, 3, 4]
+
+
+def sequential_compact(buf, keep_idx, keep_count):
+    """The ascending in-place loop: dst[k] = src[keep_idx[k]] one slot at a time.
+    Safe in place because keep_idx is ascending, so keep_idx[k] >= k."""
+    out = buf.copy()
+    for b in range(buf.shape[0]):
+        for k in range(int(keep_count[b])):
+            out[b, k] = out[b, keep_idx[b, k]]
+    return out
+
+
+@pytest.mark.parametrize("kind", ["shift1", "all", "last", "random", "sparse_tail", "empty"])
+def test_compact_matches_sequential_in_place_loop(kind):
+    r = np.random.default_rng(3)
+    b, cap = 2, 64
+    buf = r.integers(0, 1 << 30, size=(b, cap, 3)).astype(np.int64)
+    idx = np.full((b, cap), -1, np.int32)
+    cnt = np.zeros(b, np.int32)
+    for bi in range(b):
+        n = cap - 7 * bi
+        if kind == "shift1":
+            k = list(range(1, n))
+        elif kind == "all":
+            k = list(range(n))
+        elif kind == "last":
+            k = [n - 1]
+        elif kind == "random":
+            k = sorted(r.choice(n, size=n // 3, replace=False).tolist())
+        elif kind == "sparse_tail":
+            k = list(range(n - 5, n))
+        else:
+            k = []
+        idx[bi, :len(k)] = k
+        cnt[bi] = len(k)
+    got = oracle.compact(buf, idx, cnt)
+    np.testing.assert_array_equal(got, sequential_compact(buf, idx, cnt))
+    for bi in range(b):
+        kept = got[bi, :cnt[bi]]
+        np.testing.assert_array_equal(kept, buf[bi, idx[bi, :cnt[bi]]])
+        np.testing.assert_array_equal(got[bi, cnt[bi]:], buf[bi, cnt[bi]:])
+
+
+def test_compact_preserves_relative_order():
+    buf = np.arange(20)[None, :, None]          # slot value == original slot
+    idx = np.array([[2, 3, 9, 11, 19] + [-1] * 15], np.int32)
+    out = oracle.compact(buf, idx, np.array([5]))
+    assert out[0, :5, 0].tolist() == [2, 3, 9, 11, 19]
+    assert np.all(np.diff(out[0, :5, 0]) > 0)
