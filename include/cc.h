@@ -1,0 +1,166 @@
+/*
+ * cc.h -- C ABI of the counter-causal KV-cache refresh (arXiv 2607.27600).
+ *
+ * One memory refresh (Algorithm DoMemRefresh) is three calls on one CUDA
+ * stream:
+ *   1. cc_score_layer / cc_score_full: the counter-causal surprise score of
+ *      every cached slot (Sec. 3.1, Eq. 3 and the logit score it uses);
+ *   2. cc_select_keep: the keep-set, the J highest scores (argsort, keep
+ *      sigma[1:J]);
+ *   3. cc_compact_kv: K' <- (K' (+) K)_sigma[1:J], V', X likewise, in place.
+ *
+ * Conventions for every call:
+ *   - The caller owns all memory.  Every tensor argument is a device pointer
+ *     unless documented as host.  The library allocates nothing; scratch
+ *     lives in a caller-provided device workspace `ws` of at least the size
+ *     the matching *_workspace_size call returns (256-byte aligned).
+ *   - Calls are asynchronous on `stream` (a cudaStream_t; NULL = legacy
+ *     default stream).  Errors found on the host (null or misaligned
+ *     pointers, bad sizes, workspace too small, unsupported shapes) are
+ *     returned at once and nothing is enqueued.  Errors found on the device
+ *     (seq_len outside [0, cap], a budget below the forced keeps, an
+ *     internal wait that timed out) are recorded in a per-device status word
+ *     that cc_get_status reads and clears; the offending kernel skips the
+ *     affected work instead of faulting.
+ *   - bf16 means IEEE bfloat16 (2 bytes).  Matrices are row-major.  Weight
+ *     matrices use the nn.Linear layout [out_features][in_features].
+ *   - Row-major device buffers must start on a 16-byte boundary and have
+ *     rows whose byte size is a multiple of 16.
+ */
+#ifndef CC_H_
+#define CC_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  CC_OK = 0,
+  CC_ERR_INVALID_ARG = 1,  /* null/misaligned pointer, bad size or shape          */
+  CC_ERR_CUDA = 2,         /* a CUDA runtime call failed                           */
+  CC_ERR_BUDGET = 3,       /* device: budget < forced keeps (1 + n_sink)           */
+  CC_ERR_WORKSPACE = 4,    /* workspace smaller than *_workspace_size              */
+  CC_ERR_TIMEOUT = 5,      /* device: an internal wait gave up (kernel returned)   */
+  CC_ERR_UNSUPPORTED = 6,  /* shape outside what the kernels implement             */
+  CC_ERR_DEVICE_ARG = 7    /* device: seq_len/keep_count outside [0, cap]          */
+} cc_status;
+
+/* Score definition.  Sec. 3.1 takes the logit of the row's own token x_i as
+ * the score; Eq. 3 defines surprise as 1 - P(x_i | x_{i+1:t}).  Both are
+ * returned with the sign that makes "more surprising" rank higher. */
+typedef enum {
+  CC_SCORE_LOGIT = 0,   /* score_i = -z_i[x_i], z_i = final-norm(h_i) W_U^T      */
+  CC_SCORE_LOGPROB = 1  /* score_i = -log softmax(z_i)[x_i] (same order as Eq. 3) */
+} cc_score_mode;
+
+/* Decoder shape (Llama/Qwen pre-norm block: RMSNorm, GQA attention with
+ * rotate-half RoPE, RMSNorm, SwiGLU MLP; final RMSNorm; untied LM head). */
+typedef struct {
+  int32_t n_layers;
+  int32_t d_model;
+  int32_t n_q_heads;
+  int32_t n_kv_heads;   /* n_q_heads % n_kv_heads == 0; q head t reads KV head t / (Hq/Hkv) */
+  int32_t head_dim;     /* 64 or 128                                                        */
+  int32_t d_ff;
+  int32_t vocab;
+  float rope_theta;     /* inv_freq_k = theta^(-2k/head_dim), angles taken exactly mod 2pi  */
+  float rms_eps;
+} cc_model_cfg;
+
+/* One layer's weights, all bf16 device pointers. */
+typedef struct {
+  const void *attn_norm; /* [d_model]                        */
+  const void *wq;        /* [n_q_heads*head_dim][d_model]    */
+  const void *wo;        /* [d_model][n_q_heads*head_dim]    */
+  const void *mlp_norm;  /* [d_model]                        */
+  const void *w_gate;    /* [d_ff][d_model]                  */
+  const void *w_up;      /* [d_ff][d_model]                  */
+  const void *w_down;    /* [d_model][d_ff]                  */
+} cc_layer_weights;
+
+typedef struct {
+  const void *embed;                /* bf16 [vocab][d_model] (full pass only)       */
+  const void *final_norm;           /* bf16 [d_model]                               */
+  const void *lm_head;              /* bf16 [vocab][d_model]                        */
+  const cc_layer_weights *layers;   /* HOST array [n_layers]; the fast pass reads
+                                       only layers[n_layers-1]                      */
+} cc_model_weights;
+
+/* A batch of cached sequences in slot-major buffers of `cap` slots each.
+ * Sequence b holds seq_len[b] valid slots [0, seq_len[b]); slots past that
+ * are ignored (they may hold any bits).  K is stored post-RoPE (Sec. 3.1). */
+typedef struct {
+  int32_t batch;
+  int32_t cap;
+  int32_t *seq_len;  /* device int32 [batch]; cc_compact_kv sets it to keep_count     */
+  void *const *k;    /* HOST array [n_layers] of device bf16 [batch][cap][Hkv][head_dim];
+                        an entry may be NULL where a call does not need that layer     */
+  void *const *v;    /* same layout as k                                               */
+  int32_t *tokens;   /* device int32 [batch][cap]: the token buffer X                  */
+  int32_t *pos;      /* device int32 [batch][cap]: original position ids (>= 0)        */
+  void *h_last;      /* device bf16 [batch][cap][d_model]: H^(L-1), the input of the
+                        last layer recorded by the causal pass (fast mode); may be NULL
+                        for cc_score_full                                               */
+} cc_kv_cache;
+
+/* ---- scoring (Sec. 3.1) ---------------------------------------------------
+ * Writes scores[b*cap + i] (fp32, device [batch][cap]) for every slot
+ * i < seq_len[b]; slot seq_len[b]-1 gets +inf (the last token has no future
+ * context and is always retained); slots >= seq_len[b] get -inf.
+ *
+ * cc_score_layer -- fast single-layer approximation: queries from h_last
+ * with RoPE at pos, counter-causal attention (row i attends slots j with
+ * i < j < seq_len[b]) over k[n_layers-1], v[n_layers-1], then the rest of
+ * the last layer, the final norm and the head.
+ * cc_score_full -- full pass: embedding of tokens, every layer l with fresh
+ * queries over k[l], v[l] (reused, not recomputed), final norm, head.
+ */
+size_t cc_score_workspace_size(const cc_model_cfg *cfg, int32_t batch, int32_t cap,
+                               cc_score_mode mode);
+cc_status cc_score_layer(const cc_model_cfg *cfg, const cc_model_weights *w,
+                         const cc_kv_cache *cache, cc_score_mode mode, float *scores,
+                         void *ws, size_t ws_bytes, void *stream);
+cc_status cc_score_full(const cc_model_cfg *cfg, const cc_model_weights *w,
+                        const cc_kv_cache *cache, cc_score_mode mode, float *scores,
+                        void *ws, size_t ws_bytes, void *stream);
+
+/* ---- keep-set (Algorithm DoMemRefresh: sigma = argsort, keep sigma[1:J]) ---
+ * For each sequence b keeps J_b = min(budget[b], seq_len[b]) slots: the
+ * highest scores, ties broken toward the later slot, NaN ranked as -inf,
+ * slots [0, n_sink) forced (frozen system-prompt slots, Sec. 3.2).
+ * Writes keep_idx[b*cap + k], k < J_b, in ascending slot order, and
+ * keep_count[b] = J_b.  Entries of keep_idx past J_b are not written.
+ * scores, seq_len, budget: device; keep_idx [batch][cap], keep_count [batch]:
+ * device.  A budget below min(seq_len, 1 + n_sink) sets CC_ERR_BUDGET on the
+ * device and keeps the forced slots plus the last slot. */
+size_t cc_select_workspace_size(int32_t batch, int32_t cap);
+cc_status cc_select_keep(const float *scores, const int32_t *seq_len, int32_t batch,
+                         int32_t cap, const int32_t *budget, int32_t n_sink,
+                         int32_t *keep_idx, int32_t *keep_count, void *ws, size_t ws_bytes,
+                         void *stream);
+
+/* ---- compaction (Algorithm DoMemRefresh: K' <- (K' (+) K)_sigma[1:J]) ------
+ * In place, for every sequence b and k < keep_count[b]: slot k of every
+ * non-NULL k[l], v[l] (l < cfg->n_layers), of tokens, pos and (if non-NULL)
+ * h_last receives old slot keep_idx[b*cap + k].  keep_idx must be strictly
+ * ascending per sequence (as cc_select_keep writes it).  Slots >=
+ * keep_count[b] keep their old contents.  Then seq_len[b] = keep_count[b]. */
+size_t cc_compact_workspace_size(const cc_model_cfg *cfg, const cc_kv_cache *cache);
+cc_status cc_compact_kv(const cc_model_cfg *cfg, const cc_kv_cache *cache,
+                        const int32_t *keep_idx, const int32_t *keep_count, void *ws,
+                        size_t ws_bytes, void *stream);
+
+/* ---- status ---------------------------------------------------------------
+ * Synchronises `stream`, returns the first device-side error recorded since
+ * the last call (CC_OK if none) on the current device and clears it.
+ * Returns CC_ERR_CUDA if the stream itself reports a CUDA error. */
+cc_status cc_get_status(void *stream);
+const char *cc_status_str(cc_status s);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* CC_H_ */

@@ -1,0 +1,264 @@
+"""Python binding of the counter-causal refresh C ABI (include/cc.h,
+include/cc_kernels.h).
+
+Argument marshalling only: every function here passes device pointers of
+torch CUDA tensors and the current CUDA stream to the library, whose CUDA
+kernels do all the work.  A non-OK status raises CCError.  There is no
+fallback: if libcc.so is missing, every call raises.
+"""
+import ctypes
+import os
+
+import torch
+
+from . import build as _build
+
+CC_OK = 0
+CC_ERR_INVALID_ARG = 1
+CC_ERR_CUDA = 2
+CC_ERR_BUDGET = 3
+CC_ERR_WORKSPACE = 4
+CC_ERR_TIMEOUT = 5
+CC_ERR_UNSUPPORTED = 6
+CC_ERR_DEVICE_ARG = 7
+STATUS_NAMES = {0: "CC_OK", 1: "CC_ERR_INVALID_ARG", 2: "CC_ERR_CUDA", 3: "CC_ERR_BUDGET",
+                4: "CC_ERR_WORKSPACE", 5: "CC_ERR_TIMEOUT", 6: "CC_ERR_UNSUPPORTED",
+                7: "CC_ERR_DEVICE_ARG"}
+SCORE_LOGIT = 0
+SCORE_LOGPROB = 1
+
+
+class CCError(RuntimeError):
+    def __init__(self, code: int, where: str):
+        self.code = code
+        super().__init__(f"{where}: {STATUS_NAMES.get(code, code)} ({cc_status_str(code)})")
+
+
+class cc_model_cfg(ctypes.Structure):
+    _fields_ = [("n_layers", ctypes.c_int32), ("d_model", ctypes.c_int32),
+                ("n_q_heads", ctypes.c_int32), ("n_kv_heads", ctypes.c_int32),
+                ("head_dim", ctypes.c_int32), ("d_ff", ctypes.c_int32), ("vocab", ctypes.c_int32),
+                ("rope_theta", ctypes.c_float), ("rms_eps", ctypes.c_float)]
+
+
+class cc_layer_weights(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_void_p) for n in
+                ("attn_norm", "wq", "wo", "mlp_norm", "w_gate", "w_up", "w_down")]
+
+
+class cc_model_weights(ctypes.Structure):
+    _fields_ = [("embed", ctypes.c_void_p), ("final_norm", ctypes.c_void_p),
+                ("lm_head", ctypes.c_void_p), ("layers", ctypes.POINTER(cc_layer_weights))]
+
+
+class cc_kv_cache(ctypes.Structure):
+    _fields_ = [("batch", ctypes.c_int32), ("cap", ctypes.c_int32),
+                ("seq_len", ctypes.c_void_p), ("k", ctypes.POINTER(ctypes.c_void_p)),
+                ("v", ctypes.POINTER(ctypes.c_void_p)), ("tokens", ctypes.c_void_p),
+                ("pos", ctypes.c_void_p), ("h_last", ctypes.c_void_p)]
+
+
+_LIB = None
+_SIGS = {
+    "cc_score_workspace_size": (ctypes.c_size_t, [ctypes.POINTER(cc_model_cfg), ctypes.c_int32,
+                                                  ctypes.c_int32, ctypes.c_int]),
+    "cc_score_layer": (ctypes.c_int, [ctypes.POINTER(cc_model_cfg), ctypes.POINTER(cc_model_weights),
+                                      ctypes.POINTER(cc_kv_cache), ctypes.c_int, ctypes.c_void_p,
+                                      ctypes.c_void_p, ctypes.c_size_t, ctypes.c_void_p]),
+    "cc_score_full": (ctypes.c_int, [ctypes.POINTER(cc_model_cfg), ctypes.POINTER(cc_model_weights),
+                                     ctypes.POINTER(cc_kv_cache), ctypes.c_int, ctypes.c_void_p,
+                                     ctypes.c_void_p, ctypes.c_size_t, ctypes.c_void_p]),
+    "cc_select_workspace_size": (ctypes.c_size_t, [ctypes.c_int32, ctypes.c_int32]),
+    "cc_select_keep": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int32,
+                                      ctypes.c_int32, ctypes.c_void_p, ctypes.c_int32,
+                                      ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,
+                                      ctypes.c_size_t, ctypes.c_void_p]),
+    "cc_compact_workspace_size": (ctypes.c_size_t, [ctypes.POINTER(cc_model_cfg),
+                                                    ctypes.POINTER(cc_kv_cache)]),
+    "cc_compact_kv": (ctypes.c_int, [ctypes.POINTER(cc_model_cfg), ctypes.POINTER(cc_kv_cache),
+                                     ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,
+                                     ctypes.c_size_t, ctypes.c_void_p]),
+    "cc_get_status": (ctypes.c_int, [ctypes.c_void_p]),
+    "cc_status_str": (ctypes.c_char_p, [ctypes.c_int]),
+    "cc_linear_f32": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,
+                                     ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,
+                                     ctypes.c_void_p]),
+    "cc_counter_causal_attention": (ctypes.c_int, [ctypes.c_void_p] * 5 + [ctypes.c_int32] * 5
+                                    + [ctypes.c_void_p]),
+}
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def load_library(path: str = None) -> ctypes.CDLL:
+    """Loads libcc.so (built by paper_2607_27600_gb300.build); raises if absent."""
+    global _LIB
+    if _LIB is None:
+        path = path or library_path()
+        if not os.path.exists(path):
+            raise ImportError(f"{path} not found: build it first "
+                              "(python -m paper_2607_27600_gb300.build)")
+        lib = ctypes.CDLL(path)
+        for name, (res, args) in _SIGS.items():
+            fn = getattr(lib, name)
+            fn.restype, fn.argtypes = res, args
+        _LIB = lib
+    return _LIB
+
+
+def exported_symbols():
+    return sorted(_SIGS)
+
+
+# ---------------------------------------------------------------------------
+# marshalling helpers
+# ---------------------------------------------------------------------------
+
+def _dev_ptr(t, name):
+    if t is None:
+        return None
+    if not isinstance(t, torch.Tensor) or not t.is_cuda:
+        raise TypeError(f"{name} must be a CUDA tensor")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    return t.data_ptr()
+
+
+def _stream(stream):
+    if stream is None:
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, torch.cuda.Stream):
+        return stream.cuda_stream
+    return int(stream)
+
+
+def _check(code, where):
+    if code != CC_OK:
+        raise CCError(code, where)
+
+
+def model_cfg(shape) -> cc_model_cfg:
+    """cc_model_cfg from any object with the ModelShape fields."""
+    return cc_model_cfg(shape.n_layers, shape.d_model, shape.n_q_heads, shape.n_kv_heads,
+                        shape.head_dim, shape.d_ff, shape.vocab, float(shape.rope_theta),
+                        float(shape.rms_eps))
+
+
+class Weights:
+    """cc_model_weights over a dict of CUDA bf16 tensors (embed, final_norm,
+    lm_head, layers[l] = {attn_norm, wq, wo, mlp_norm, w_gate, w_up, w_down});
+    keeps the tensors alive."""
+
+    def __init__(self, w: dict):
+        self.w = w
+        layers = w["layers"]
+        self._layers = (cc_layer_weights * len(layers))()
+        for l, lw in enumerate(layers):
+            if lw is None:
+                continue
+            for f in ("attn_norm", "wq", "wo", "mlp_norm", "w_gate", "w_up", "w_down"):
+                setattr(self._layers[l], f, _dev_ptr(lw[f], f"layers[{l}].{f}"))
+        self.c = cc_model_weights(_dev_ptr(w.get("embed"), "embed"),
+                                  _dev_ptr(w["final_norm"], "final_norm"),
+                                  _dev_ptr(w["lm_head"], "lm_head"), self._layers)
+
+
+class Cache:
+    """cc_kv_cache over a dict of CUDA tensors (k[l], v[l] bf16 [B, cap, Hkv, dh];
+    tokens, pos int32 [B, cap]; seq_len int32 [B]; h_last bf16 [B, cap, d] or
+    None); keeps the tensors alive."""
+
+    def __init__(self, c: dict):
+        self.d = c
+        b, cap = c["tokens"].shape
+        ks, vs = c["k"], c["v"]
+        self._k = (ctypes.c_void_p * len(ks))(*[_dev_ptr(x, "k") for x in ks])
+        self._v = (ctypes.c_void_p * len(vs))(*[_dev_ptr(x, "v") for x in vs])
+        self.c = cc_kv_cache(b, cap, _dev_ptr(c["seq_len"], "seq_len"), self._k, self._v,
+                             _dev_ptr(c["tokens"], "tokens"), _dev_ptr(c["pos"], "pos"),
+                             _dev_ptr(c.get("h_last"), "h_last"))
+
+
+def _cfg(cfg):
+    return cfg if isinstance(cfg, cc_model_cfg) else model_cfg(cfg)
+
+
+# ---------------------------------------------------------------------------
+# the C ABI, one Python function per entry point
+# ---------------------------------------------------------------------------
+
+def cc_status_str(code: int) -> str:
+    return load_library().cc_status_str(int(code)).decode()
+
+
+def cc_score_workspace_size(cfg, batch: int, cap: int, mode: int = SCORE_LOGIT) -> int:
+    return int(load_library().cc_score_workspace_size(ctypes.byref(_cfg(cfg)), batch, cap, mode))
+
+
+def _score(fn, cfg, weights: Weights, cache: Cache, mode, scores, ws, stream):
+    c = _cfg(cfg)
+    code = getattr(load_library(), fn)(ctypes.byref(c), ctypes.byref(weights.c),
+                                       ctypes.byref(cache.c), int(mode),
+                                       _dev_ptr(scores, "scores"), _dev_ptr(ws, "ws"),
+                                       ws.numel() * ws.element_size(), _stream(stream))
+    _check(code, fn)
+
+
+def cc_score_layer(cfg, weights, cache, mode, scores, ws, stream=None):
+    _score("cc_score_layer", cfg, weights, cache, mode, scores, ws, stream)
+
+
+def cc_score_full(cfg, weights, cache, mode, scores, ws, stream=None):
+    _score("cc_score_full", cfg, weights, cache, mode, scores, ws, stream)
+
+
+def cc_select_workspace_size(batch: int, cap: int) -> int:
+    return int(load_library().cc_select_workspace_size(batch, cap))
+
+
+def cc_select_keep(scores, seq_len, batch, cap, budget, n_sink, keep_idx, keep_count, ws=None,
+                   stream=None):
+    nbytes = 0 if ws is None else ws.numel() * ws.element_size()
+    code = load_library().cc_select_keep(
+        _dev_ptr(scores, "scores"), _dev_ptr(seq_len, "seq_len"), batch, cap,
+        _dev_ptr(budget, "budget"), n_sink, _dev_ptr(keep_idx, "keep_idx"),
+        _dev_ptr(keep_count, "keep_count"), _dev_ptr(ws, "ws"), nbytes, _stream(stream))
+    _check(code, "cc_select_keep")
+
+
+def cc_compact_workspace_size(cfg, cache: Cache) -> int:
+    return int(load_library().cc_compact_workspace_size(ctypes.byref(_cfg(cfg)),
+                                                        ctypes.byref(cache.c)))
+
+
+def cc_compact_kv(cfg, cache: Cache, keep_idx, keep_count, ws, stream=None):
+    code = load_library().cc_compact_kv(ctypes.byref(_cfg(cfg)), ctypes.byref(cache.c),
+                                        _dev_ptr(keep_idx, "keep_idx"),
+                                        _dev_ptr(keep_count, "keep_count"), _dev_ptr(ws, "ws"),
+                                        ws.numel() * ws.element_size(), _stream(stream))
+    _check(code, "cc_compact_kv")
+
+
+def cc_get_status(stream=None) -> int:
+    return int(load_library().cc_get_status(_stream(stream)))
+
+
+def cc_linear_f32(x, w, y, stream=None):
+    code = load_library().cc_linear_f32(_dev_ptr(x, "x"), _dev_ptr(w, "w"), _dev_ptr(y, "y"),
+                                        x.shape[0], w.shape[0], x.shape[1], _stream(stream))
+    _check(code, "cc_linear_f32")
+
+
+def cc_counter_causal_attention(q, k, v, seq_len, out, batch, cap, n_q_heads, n_kv_heads,
+                                head_dim, stream=None):
+    code = load_library().cc_counter_causal_attention(
+        _dev_ptr(q, "q"), _dev_ptr(k, "k"), _dev_ptr(v, "v"), _dev_ptr(seq_len, "seq_len"),
+        _dev_ptr(out, "out"), batch, cap, n_q_heads, n_kv_heads, head_dim, _stream(stream))
+    _check(code, "cc_counter_causal_attention")
+
+
+def alloc_workspace(nbytes: int, device="cuda") -> torch.Tensor:
+    """A caller-owned device workspace of at least nbytes (256-byte aligned by torch)."""
+    return torch.empty(max(int(nbytes), 256), dtype=torch.uint8, device=device)

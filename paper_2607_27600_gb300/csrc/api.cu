@@ -1,0 +1,541 @@
+// api.cu -- the C ABI (include/cc.h, include/cc_kernels.h): argument checks,
+// workspace layout, TMA tensor maps and the launch sequence of one refresh.
+//
+// Scoring pass per layer (Sec. 3.1, the standard pre-norm layer re-run under
+// the counter-causal mask), on rows b*cap + i of a ragged batch:
+//   xn = RMSNorm(h) ; Q = RoPE(xn Wq^T, pos)                 [rmsnorm, GEMM+RoPE]
+//   O  = counter-causal attention(Q, K_l, V_l)               [attention]
+//   h  = h + O Wo^T                                          [GEMM+residual]
+//   xn = RMSNorm(h) ; A = silu(xn Wg^T) * (xn Wu^T)          [rmsnorm, GEMM+SwiGLU]
+//   h  = h + A Wd^T                                          [GEMM+residual]
+// then the head: -(final-norm(h) . W_U[x_i])  (logit mode, a gather-dot) or
+// logsumexp(final-norm(h) W_U^T) - z[x_i]      (log-prob mode, GEMM+LSE).
+#include <math.h>
+#include <stdio.h>
+
+#include <mutex>
+
+#include "attn.cuh"
+#include "compact.cuh"
+#include "gemm.cuh"
+#include "rowops.cuh"
+#include "select.cuh"
+#include "../../include/cc_kernels.h"
+
+namespace cc {
+__device__ unsigned g_status_word;   // first device-side error since the last cc_get_status
+}
+
+namespace {
+
+using namespace cc;
+
+constexpr int kMaxDevices = 64;
+
+// ---------------------------------------------------------------------------
+// per-device state: status-word address, SM count
+// ---------------------------------------------------------------------------
+struct DevState {
+  unsigned *status = nullptr;
+  int sms = 0;
+  bool ready = false;
+};
+DevState g_dev[kMaxDevices];
+std::mutex g_mu;
+
+bool dev_state(DevState **out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return false;
+  std::lock_guard<std::mutex> lk(g_mu);
+  DevState &d = g_dev[dev];
+  if (!d.ready) {
+    void *p = nullptr;
+    if (cudaGetSymbolAddress(&p, cc::g_status_word) != cudaSuccess) return false;
+    if (cudaDeviceGetAttribute(&d.sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+      return false;
+    d.status = reinterpret_cast<unsigned *>(p);
+    d.ready = true;
+  }
+  *out = &d;
+  return true;
+}
+
+// ---------------------------------------------------------------------------
+// TMA tensor maps (driver entry point fetched through the runtime)
+// ---------------------------------------------------------------------------
+typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
+                                  const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
+                                  const cuuint32_t *, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void *p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  });
+  return fn;
+}
+
+// bf16 tensor of `rank` dims (dims[0] contiguous), strides in bytes for dims 1.., 128B swizzle.
+bool make_tmap(CUtensorMap *m, const void *base, int rank, const uint64_t *dims,
+               const uint64_t *strides, const uint32_t *box) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t d[5], s[4];
+  cuuint32_t bx[5], es[5];
+  for (int i = 0; i < rank; ++i) {
+    d[i] = dims[i];
+    bx[i] = box[i];
+    es[i] = 1;
+    if (i > 0) s[i - 1] = strides[i - 1];
+  }
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, rank, const_cast<void *>(base), d, s, bx, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// rows x cols bf16 matrix (row pitch = cols), box 64 x box_rows
+bool tmap_rows(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols, uint32_t box_rows) {
+  const uint64_t dims[2] = {cols, rows};
+  const uint64_t strides[1] = {cols * 2};
+  const uint32_t box[2] = {64, box_rows};
+  return make_tmap(m, base, 2, dims, strides, box);
+}
+
+// ---------------------------------------------------------------------------
+// checks
+// ---------------------------------------------------------------------------
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+cc_status check_cfg(const cc_model_cfg *c) {
+  if (!c) return CC_ERR_INVALID_ARG;
+  if (c->n_layers < 1 || c->d_model < 1 || c->n_q_heads < 1 || c->n_kv_heads < 1 ||
+      c->d_ff < 1 || c->vocab < 1 || !(c->rms_eps >= 0.f) || !(c->rope_theta > 0.f))
+    return CC_ERR_INVALID_ARG;
+  if (c->n_q_heads % c->n_kv_heads) return CC_ERR_INVALID_ARG;
+  if (c->head_dim != 64 && c->head_dim != 128) return CC_ERR_UNSUPPORTED;
+  if (c->d_model % 32 || c->d_ff % 32) return CC_ERR_UNSUPPORTED;
+  if (c->n_q_heads / c->n_kv_heads > 256) return CC_ERR_UNSUPPORTED;
+  return CC_OK;
+}
+
+size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+struct ScoreWs {
+  size_t xn, q, o, h, act, part, ztgt, total;
+  int n_vtiles;
+};
+
+ScoreWs score_layout(const cc_model_cfg *c, int batch, int cap, cc_score_mode mode) {
+  ScoreWs w{};
+  const size_t R = (size_t)batch * cap;
+  const size_t d = c->d_model, qd = (size_t)c->n_q_heads * c->head_dim, f = c->d_ff;
+  size_t off = 0;
+  auto take = [&](size_t bytes) { size_t o = off; off = align256(off + bytes); return o; };
+  w.xn = take(R * d * 2);
+  w.q = take(R * qd * 2);
+  w.o = take(R * qd * 2);
+  w.h = take(R * d * 4);
+  w.act = take(R * f * 2);
+  w.n_vtiles = (c->vocab + 255) / 256;
+  if (mode == CC_SCORE_LOGPROB) {
+    w.part = take(R * w.n_vtiles * 8);
+    w.ztgt = take(R * 4);
+  }
+  w.total = off;
+  return w;
+}
+
+// RoPE: inv_freq_k / (2 pi) as 0.64 fixed point (angles reduced exactly on the device).
+void rope_turns(const cc_model_cfg *c, unsigned long long *turns) {
+  const int half = c->head_dim / 2;
+  for (int k = 0; k < half; ++k) {
+    const double inv_freq = pow((double)c->rope_theta, -2.0 * k / c->head_dim);
+    const double t = inv_freq / (2.0 * M_PI);   // < 1
+    turns[k] = (unsigned long long)ldexp(t, 64);
+  }
+}
+
+#define CC_TRY(expr)                                         \
+  do {                                                       \
+    cudaError_t e_ = (expr);                                 \
+    if (e_ != cudaSuccess) return CC_ERR_CUDA;               \
+  } while (0)
+
+struct Gemm {
+  CUtensorMap a, b, b2;
+  GemmParams p;
+};
+
+// One GEMM over the cache rows: A [R][K] (bf16 workspace) x W [N][K]^T.
+cc_status gemm_setup(Gemm &g, int epi, const void *A, int K, const void *W, const void *W2, int N,
+                     int batch, int cap, const int32_t *seq_len, unsigned *status) {
+  const uint64_t R = (uint64_t)batch * cap;
+  const int bn = gemm_block_n(epi);
+  if (!tmap_rows(&g.a, A, R, K, 128)) return CC_ERR_CUDA;
+  if (!tmap_rows(&g.b, W, N, K, epi == EPI_SWIGLU ? 128 : 256)) return CC_ERR_CUDA;
+  if (epi == EPI_SWIGLU) {
+    if (!tmap_rows(&g.b2, W2, N, K, 128)) return CC_ERR_CUDA;
+  } else {
+    g.b2 = g.b;
+  }
+  memset(&g.p, 0, sizeof(g.p));
+  g.p.batch = batch;
+  g.p.cap = cap;
+  g.p.seq_len = seq_len;
+  g.p.N = N;
+  g.p.K = K;
+  g.p.n_tiles = (N + bn - 1) / bn;
+  g.p.status = status;
+  return CC_OK;
+}
+
+cc_status run_gemm(Gemm &g, int epi, int sms, cudaStream_t st) {
+  CC_TRY(launch_gemm(epi, g.a, g.b, g.b2, g.p, sms, st));
+  return CC_OK;
+}
+
+cc_status run_attention(const cc_model_cfg *c, const void *q, const void *k, const void *v,
+                        void *out, const int32_t *seq_len, int batch, int cap, unsigned *status,
+                        cudaStream_t st) {
+  const int G = c->n_q_heads / c->n_kv_heads, dh = c->head_dim;
+  const int P = attn_positions_per_unit(G);
+  const uint64_t R = (uint64_t)batch * cap;
+  CUtensorMap tq, tk, tv;
+  {
+    const uint64_t dims[3] = {(uint64_t)dh, (uint64_t)c->n_q_heads, R};
+    const uint64_t strides[2] = {(uint64_t)dh * 2, (uint64_t)c->n_q_heads * dh * 2};
+    const uint32_t box[3] = {64, (uint32_t)G, (uint32_t)P};
+    if (!make_tmap(&tq, q, 3, dims, strides, box)) return CC_ERR_CUDA;
+  }
+  {
+    const uint64_t dims[3] = {(uint64_t)dh, (uint64_t)c->n_kv_heads, R};
+    const uint64_t strides[2] = {(uint64_t)dh * 2, (uint64_t)c->n_kv_heads * dh * 2};
+    const uint32_t box[3] = {64, 1, 128};
+    if (!make_tmap(&tk, k, 3, dims, strides, box)) return CC_ERR_CUDA;
+    if (!make_tmap(&tv, v, 3, dims, strides, box)) return CC_ERR_CUDA;
+  }
+  AttnParams p{};
+  p.batch = batch;
+  p.cap = cap;
+  p.n_q_heads = c->n_q_heads;
+  p.n_kv_heads = c->n_kv_heads;
+  p.head_dim = dh;
+  p.group = G;
+  p.P = P;
+  p.seq_len = seq_len;
+  p.out = reinterpret_cast<__nv_bfloat16 *>(out);
+  p.scale_log2 = (float)(1.4426950408889634 / sqrt((double)dh));
+  p.status = status;
+  CC_TRY(launch_attention(tq, tk, tv, p, st));
+  return CC_OK;
+}
+
+cc_status check_score_args(const cc_model_cfg *c, const cc_model_weights *w, const cc_kv_cache *kv,
+                           cc_score_mode mode, const float *scores, void *ws, size_t ws_bytes,
+                           bool full) {
+  cc_status s = check_cfg(c);
+  if (s != CC_OK) return s;
+  if (!w || !kv || !scores || !w->layers || !w->final_norm || !w->lm_head || !kv->k || !kv->v)
+    return CC_ERR_INVALID_ARG;
+  if (mode != CC_SCORE_LOGIT && mode != CC_SCORE_LOGPROB) return CC_ERR_INVALID_ARG;
+  if (kv->batch < 1 || kv->cap < 1 || !kv->seq_len || !kv->tokens || !kv->pos)
+    return CC_ERR_INVALID_ARG;
+  if (kv->batch > gemm_max_batch()) return CC_ERR_UNSUPPORTED;
+  if ((uint64_t)kv->batch * kv->cap >= (1ull << 31)) return CC_ERR_UNSUPPORTED;
+  if (full && !w->embed) return CC_ERR_INVALID_ARG;
+  if (!full && !kv->h_last) return CC_ERR_INVALID_ARG;
+  const int l0 = full ? 0 : c->n_layers - 1;
+  for (int l = l0; l < c->n_layers; ++l) {
+    const cc_layer_weights &lw = w->layers[l];
+    const void *ptrs[] = {lw.attn_norm, lw.wq, lw.wo, lw.mlp_norm, lw.w_gate, lw.w_up, lw.w_down,
+                          kv->k[l], kv->v[l]};
+    for (const void *p : ptrs)
+      if (!p || !aligned16(p)) return CC_ERR_INVALID_ARG;
+  }
+  const void *ptrs[] = {w->final_norm, w->lm_head, ws, kv->h_last, full ? w->embed : nullptr};
+  for (const void *p : ptrs)
+    if (p && !aligned16(p)) return CC_ERR_INVALID_ARG;
+  if (!ws || ws_bytes < score_layout(c, kv->batch, kv->cap, mode).total) return CC_ERR_WORKSPACE;
+  return CC_OK;
+}
+
+cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_kv_cache *kv,
+                    cc_score_mode mode, float *scores, void *ws, size_t ws_bytes, void *stream,
+                    bool full) {
+  cc_status s = check_score_args(c, w, kv, mode, scores, ws, ws_bytes, full);
+  if (s != CC_OK) return s;
+  DevState *dev;
+  if (!dev_state(&dev)) return CC_ERR_CUDA;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  const int batch = kv->batch, cap = kv->cap, rows = batch * cap;
+  const int d = c->d_model, qd = c->n_q_heads * c->head_dim, f = c->d_ff;
+  const ScoreWs L = score_layout(c, batch, cap, mode);
+  uint8_t *wsb = reinterpret_cast<uint8_t *>(ws);
+  void *xn = wsb + L.xn, *q = wsb + L.q, *o = wsb + L.o, *act = wsb + L.act;
+  float *h = reinterpret_cast<float *>(wsb + L.h);
+  const int32_t *sl = kv->seq_len;
+  unsigned *status = dev->status;
+
+  if (full) CC_TRY(launch_embed(w->embed, kv->tokens, h, d, c->vocab, sl, cap, rows, status, st));
+  const int l0 = full ? 0 : c->n_layers - 1;
+  for (int l = l0; l < c->n_layers; ++l) {
+    const cc_layer_weights &lw = w->layers[l];
+    const bool first_from_bf16 = !full;   // fast mode: the layer input is H^(L-1) (bf16)
+    // xn = RMSNorm(h)
+    CC_TRY(launch_rmsnorm(first_from_bf16 ? kv->h_last : (const void *)h, !first_from_bf16,
+                          lw.attn_norm, xn, d, c->rms_eps, sl, cap, rows, st));
+    // Q = RoPE(xn Wq^T)
+    Gemm gq;
+    if ((s = gemm_setup(gq, EPI_QROPE, xn, d, lw.wq, nullptr, qd, batch, cap, sl, status)) != CC_OK)
+      return s;
+    gq.p.out = q;
+    gq.p.ldo = qd;
+    gq.p.pos = kv->pos;
+    gq.p.head_dim = c->head_dim;
+    rope_turns(c, gq.p.turns);
+    if ((s = run_gemm(gq, EPI_QROPE, dev->sms, st)) != CC_OK) return s;
+    // O = counter-causal attention
+    if ((s = run_attention(c, q, kv->k[l], kv->v[l], o, sl, batch, cap, status, st)) != CC_OK)
+      return s;
+    // h = h + O Wo^T  (fast mode: h = H^(L-1) + O Wo^T)
+    Gemm go;
+    const int epi_o = first_from_bf16 ? EPI_RESID_BF16 : EPI_RESID_F32;
+    if ((s = gemm_setup(go, epi_o, o, qd, lw.wo, nullptr, d, batch, cap, sl, status)) != CC_OK)
+      return s;
+    go.p.out = h;
+    go.p.ldo = d;
+    go.p.resid = kv->h_last;
+    go.p.ld_resid = d;
+    if ((s = run_gemm(go, epi_o, dev->sms, st)) != CC_OK) return s;
+    // xn = RMSNorm(h); act = silu(xn Wg^T) * (xn Wu^T)
+    CC_TRY(launch_rmsnorm(h, true, lw.mlp_norm, xn, d, c->rms_eps, sl, cap, rows, st));
+    Gemm gu;
+    if ((s = gemm_setup(gu, EPI_SWIGLU, xn, d, lw.w_gate, lw.w_up, f, batch, cap, sl, status)) !=
+        CC_OK)
+      return s;
+    gu.p.out = act;
+    gu.p.ldo = f;
+    if ((s = run_gemm(gu, EPI_SWIGLU, dev->sms, st)) != CC_OK) return s;
+    // h = h + act Wd^T
+    Gemm gd;
+    if ((s = gemm_setup(gd, EPI_RESID_F32, act, f, lw.w_down, nullptr, d, batch, cap, sl,
+                        status)) != CC_OK)
+      return s;
+    gd.p.out = h;
+    gd.p.ldo = d;
+    if ((s = run_gemm(gd, EPI_RESID_F32, dev->sms, st)) != CC_OK) return s;
+  }
+  // head
+  if (mode == CC_SCORE_LOGIT) {
+    CC_TRY(launch_head_logit(h, w->final_norm, w->lm_head, kv->tokens, scores, d, c->vocab,
+                             c->rms_eps, sl, cap, rows, status, st));
+  } else {
+    CC_TRY(launch_rmsnorm(h, true, w->final_norm, xn, d, c->rms_eps, sl, cap, rows, st));
+    Gemm gl;
+    if ((s = gemm_setup(gl, EPI_LSE, xn, d, w->lm_head, nullptr, c->vocab, batch, cap, sl,
+                        status)) != CC_OK)
+      return s;
+    float2 *part = reinterpret_cast<float2 *>(wsb + L.part);
+    float *zt = reinterpret_cast<float *>(wsb + L.ztgt);
+    gl.p.out = part;
+    gl.p.ldo = L.n_vtiles;
+    gl.p.tokens = kv->tokens;
+    gl.p.z_target = zt;
+    if ((s = run_gemm(gl, EPI_LSE, dev->sms, st)) != CC_OK) return s;
+    CC_TRY(launch_lse_combine(part, L.n_vtiles, zt, scores, sl, cap, rows, st));
+  }
+  return CC_OK;
+}
+
+// compaction plan: arrays and unit counts
+struct CompactPlan {
+  CompactParams p;
+  size_t ws_bytes;
+};
+
+cc_status compact_plan(const cc_model_cfg *c, const cc_kv_cache *kv, CompactPlan &plan) {
+  cc_status s = check_cfg(c);
+  if (s != CC_OK) return s;
+  if (!kv || kv->batch < 1 || kv->cap < 1 || !kv->k || !kv->v || !kv->tokens || !kv->pos ||
+      !kv->seq_len)
+    return CC_ERR_INVALID_ARG;
+  CompactParams &p = plan.p;
+  memset(&p, 0, sizeof(p));
+  p.batch = kv->batch;
+  p.cap = kv->cap;
+  int n = 0, units = 0;
+  auto add = [&](void *base, int row_bytes, bool bulk) -> bool {
+    if (!base) return true;
+    if (n >= kMaxCompactArrays || !aligned16(base)) return false;
+    CompactArray &A = p.arr[n++];
+    A.base = base;
+    A.row_bytes = row_bytes;
+    A.bulk = bulk ? 1 : 0;
+    A.rows_per_chunk = bulk ? (row_bytes <= kStageBytes ? kStageBytes / row_bytes : 0) : 4096;
+    if (A.rows_per_chunk < 1) return false;
+    A.n_chunks = (kv->cap + A.rows_per_chunk - 1) / A.rows_per_chunk;
+    A.unit_base = units;
+    units += kv->batch * A.n_chunks;
+    return true;
+  };
+  const int kv_row = c->n_kv_heads * c->head_dim * 2;
+  for (int l = 0; l < c->n_layers; ++l) {
+    if (!add(kv->k[l], kv_row, true) || !add(kv->v[l], kv_row, true)) return CC_ERR_UNSUPPORTED;
+  }
+  if (!add(kv->h_last, c->d_model * 2, true)) return CC_ERR_UNSUPPORTED;
+  if (!add(kv->tokens, 4, false) || !add(kv->pos, 4, false)) return CC_ERR_INVALID_ARG;
+  p.n_arrays = n;
+  p.total_units = units;
+  plan.ws_bytes = 256 + align256((size_t)units * 4);
+  return CC_OK;
+}
+
+}  // namespace
+
+// ===========================================================================
+// C ABI
+// ===========================================================================
+extern "C" {
+
+size_t cc_score_workspace_size(const cc_model_cfg *cfg, int32_t batch, int32_t cap,
+                               cc_score_mode mode) {
+  if (check_cfg(cfg) != CC_OK || batch < 1 || cap < 1) return 0;
+  return score_layout(cfg, batch, cap, mode).total;
+}
+
+cc_status cc_score_layer(const cc_model_cfg *cfg, const cc_model_weights *w,
+                         const cc_kv_cache *cache, cc_score_mode mode, float *scores, void *ws,
+                         size_t ws_bytes, void *stream) {
+  return run_score(cfg, w, cache, mode, scores, ws, ws_bytes, stream, false);
+}
+
+cc_status cc_score_full(const cc_model_cfg *cfg, const cc_model_weights *w,
+                        const cc_kv_cache *cache, cc_score_mode mode, float *scores, void *ws,
+                        size_t ws_bytes, void *stream) {
+  return run_score(cfg, w, cache, mode, scores, ws, ws_bytes, stream, true);
+}
+
+size_t cc_select_workspace_size(int32_t batch, int32_t cap) {
+  (void)batch;
+  (void)cap;
+  return 0;   // one CTA per sequence keeps its histograms in shared memory
+}
+
+cc_status cc_select_keep(const float *scores, const int32_t *seq_len, int32_t batch, int32_t cap,
+                         const int32_t *budget, int32_t n_sink, int32_t *keep_idx,
+                         int32_t *keep_count, void *ws, size_t ws_bytes, void *stream) {
+  (void)ws;
+  (void)ws_bytes;
+  if (!scores || !seq_len || !budget || !keep_idx || !keep_count || batch < 1 || cap < 1 ||
+      n_sink < 0)
+    return CC_ERR_INVALID_ARG;
+  DevState *dev;
+  if (!dev_state(&dev)) return CC_ERR_CUDA;
+  CC_TRY(launch_select(scores, seq_len, batch, cap, budget, n_sink, keep_idx, keep_count,
+                       dev->status, reinterpret_cast<cudaStream_t>(stream)));
+  return CC_OK;
+}
+
+size_t cc_compact_workspace_size(const cc_model_cfg *cfg, const cc_kv_cache *cache) {
+  CompactPlan plan;
+  if (compact_plan(cfg, cache, plan) != CC_OK) return 0;
+  return plan.ws_bytes;
+}
+
+cc_status cc_compact_kv(const cc_model_cfg *cfg, const cc_kv_cache *cache,
+                        const int32_t *keep_idx, const int32_t *keep_count, void *ws,
+                        size_t ws_bytes, void *stream) {
+  static CompactPlan plan;   // large (kernel parameter block); guarded below
+  static std::mutex mu;
+  std::lock_guard<std::mutex> lk(mu);
+  cc_status s = compact_plan(cfg, cache, plan);
+  if (s != CC_OK) return s;
+  if (!keep_idx || !keep_count) return CC_ERR_INVALID_ARG;
+  if (!ws || !aligned16(ws) || ws_bytes < plan.ws_bytes) return CC_ERR_WORKSPACE;
+  DevState *dev;
+  if (!dev_state(&dev)) return CC_ERR_CUDA;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  CC_TRY(cudaMemsetAsync(ws, 0, plan.ws_bytes, st));
+  plan.p.keep_idx = keep_idx;
+  plan.p.keep_count = keep_count;
+  plan.p.seq_len = cache->seq_len;
+  plan.p.ticket = reinterpret_cast<unsigned *>(ws);
+  plan.p.flags = reinterpret_cast<unsigned *>(reinterpret_cast<uint8_t *>(ws) + 256);
+  plan.p.status = dev->status;
+  CC_TRY(launch_compact(plan.p, dev->sms * 3, st));
+  return CC_OK;
+}
+
+cc_status cc_get_status(void *stream) {
+  DevState *dev;
+  if (!dev_state(&dev)) return CC_ERR_CUDA;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  if (cudaStreamSynchronize(st) != cudaSuccess) return CC_ERR_CUDA;
+  unsigned v = 0;
+  if (cudaMemcpy(&v, dev->status, sizeof(v), cudaMemcpyDeviceToHost) != cudaSuccess)
+    return CC_ERR_CUDA;
+  const unsigned zero = 0;
+  if (cudaMemcpy(dev->status, &zero, sizeof(zero), cudaMemcpyHostToDevice) != cudaSuccess)
+    return CC_ERR_CUDA;
+  return static_cast<cc_status>(v);
+}
+
+const char *cc_status_str(cc_status s) {
+  switch (s) {
+    case CC_OK: return "ok";
+    case CC_ERR_INVALID_ARG: return "invalid argument";
+    case CC_ERR_CUDA: return "CUDA error";
+    case CC_ERR_BUDGET: return "budget below the forced keeps";
+    case CC_ERR_WORKSPACE: return "workspace too small";
+    case CC_ERR_TIMEOUT: return "device wait timed out";
+    case CC_ERR_UNSUPPORTED: return "unsupported shape";
+    case CC_ERR_DEVICE_ARG: return "device-side argument out of range";
+  }
+  return "unknown status";
+}
+
+// ---- kernel-level entry points (include/cc_kernels.h) ----------------------
+
+cc_status cc_linear_f32(const void *x, const void *w, float *y, int32_t rows, int32_t n,
+                        int32_t k, void *stream) {
+  if (!x || !w || !y || rows < 1 || n < 1 || k < 1 || n % 32 || k % 8) return CC_ERR_INVALID_ARG;
+  if (!aligned16(x) || !aligned16(w) || !aligned16(y)) return CC_ERR_INVALID_ARG;
+  DevState *dev;
+  if (!dev_state(&dev)) return CC_ERR_CUDA;
+  Gemm g;
+  cc_status s = gemm_setup(g, EPI_F32, x, k, w, nullptr, n, 1, rows, nullptr, dev->status);
+  if (s != CC_OK) return s;
+  g.p.out = y;
+  g.p.ldo = n;
+  return run_gemm(g, EPI_F32, dev->sms, reinterpret_cast<cudaStream_t>(stream));
+}
+
+cc_status cc_counter_causal_attention(const void *q, const void *k, const void *v,
+                                      const int32_t *seq_len, void *out, int32_t batch,
+                                      int32_t cap, int32_t n_q_heads, int32_t n_kv_heads,
+                                      int32_t head_dim, void *stream) {
+  if (!q || !k || !v || !seq_len || !out || batch < 1 || cap < 1 || n_q_heads < 1 ||
+      n_kv_heads < 1 || n_q_heads % n_kv_heads)
+    return CC_ERR_INVALID_ARG;
+  if (head_dim != 64 && head_dim != 128) return CC_ERR_UNSUPPORTED;
+  if (n_q_heads / n_kv_heads > 256) return CC_ERR_UNSUPPORTED;
+  if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(out)) return CC_ERR_INVALID_ARG;
+  if ((uint64_t)batch * cap >= (1ull << 31)) return CC_ERR_UNSUPPORTED;
+  DevState *dev;
+  if (!dev_state(&dev)) return CC_ERR_CUDA;
+  cc_model_cfg c{};
+  c.n_q_heads = n_q_heads;
+  c.n_kv_heads = n_kv_heads;
+  c.head_dim = head_dim;
+  return run_attention(&c, q, k, v, out, seq_len, batch, cap, dev->status,
+                       reinterpret_cast<cudaStream_t>(stream));
+}
+
+}  // extern "C"

@@ -1,0 +1,381 @@
+// attn.cu -- counter-causal flash attention on tcgen05 (Sec. 3.1: fresh
+// queries, cached post-RoPE K/V reused, row i attends only slots j with
+// i < j < n).
+//
+// One CTA = one work unit (sequence b, KV head g, block of P positions).
+// The unit's query rows are the G = Hq/Hkv heads of group g at P
+// consecutive positions, row r = position * G + head, so that P*G <= 256
+// rows form two M=128 MMA tiles that share every K/V tile loaded (a GQA
+// group is served by one K/V stream).  Key tiles of 128 slots run from the
+// one holding slot p0+1 to the one holding slot n-1: whole tiles at or
+// below the diagonal are never loaded.
+//
+//   warps 0..3, 4..7  softmax of M-half 0 / 1 (one row per thread): S from
+//                     TMEM, mask, online softmax (log2 domain, lazy rescale),
+//                     P (bf16) written back over S in TMEM, final O / l
+//   warp 8            TMA producer (Q once; K and V tiles, 2 stages each);
+//                     zeroes V rows past the sequence end in the last tile
+//   warp 9            TMEM owner + tcgen05.mma issuer:
+//                     S_h = Q_h K^T (SS),  O_h += P_h V (TS, P from TMEM)
+//
+// TMEM columns: S0 [0,128)  S1 [128,256)  O0 [256,256+DH)  O1 [256+DH, 256+2DH)
+#include "attn.cuh"
+
+namespace cc {
+
+namespace {
+
+constexpr int BKV = 128;        // keys per tile
+constexpr int KST = 2;          // K and V pipeline stages
+constexpr int kThreads = 320;
+
+// 2^x by the PTX ex2.approx instruction (2 ulp; 2^-inf = 0).
+CC_DEV float fast_exp2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+template <int DH>
+struct AttnSmem {
+  static constexpr int NH = DH / 64;                 // 64-element (128-byte) column halves
+  static constexpr int Q_BYTES = NH * 256 * 128;     // 256 rows
+  static constexpr int KV_BYTES = NH * BKV * 128;    // one K (or V) tile
+  static constexpr int OFF_Q = 0;
+  static constexpr int OFF_K = OFF_Q + Q_BYTES;
+  static constexpr int OFF_V = OFF_K + KST * KV_BYTES;
+  static constexpr int OFF_BAR = OFF_V + KST * KV_BYTES;
+  static constexpr int BYTES = OFF_BAR + 256 + 1024;   // barriers + alignment slack
+};
+
+template <int DH>
+__global__ void __launch_bounds__(kThreads, 1)
+    attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                const __grid_constant__ CUtensorMap tmV, const __grid_constant__ AttnParams p) {
+  using L = AttnSmem<DH>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                              ~uintptr_t(1023));
+  uint64_t *bars = reinterpret_cast<uint64_t *>(smem + L::OFF_BAR);
+  uint64_t *q_full = bars + 0;
+  uint64_t *k_full = bars + 1;             // [KST]
+  uint64_t *k_empty = k_full + KST;        // [KST]
+  uint64_t *v_full = k_empty + KST;        // [KST]
+  uint64_t *v_empty = v_full + KST;        // [KST]
+  uint64_t *v_fixed = v_empty + KST;       // tail tile: V rows past n zeroed
+  uint64_t *s_ready = v_fixed + 1;         // [2]
+  uint64_t *p_ready = s_ready + 2;         // [2]
+  uint64_t *o_done = p_ready + 2;          // [2]
+  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(o_done + 2);
+  volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int G = p.group, P = p.P;
+  const int units_per_pb = p.batch * p.n_kv_heads;
+  const int pb = blockIdx.x / units_per_pb;
+  const int rem = blockIdx.x - pb * units_per_pb;
+  const int b = rem / p.n_kv_heads, g = rem - b * p.n_kv_heads;
+  int n = p.seq_len[b];
+  if (n < 0 || n > p.cap) {
+    if (threadIdx.x == 0) set_status(p.status, CC_ERR_DEVICE_ARG);
+    return;
+  }
+  const int p0 = pb * P;
+  if (p0 >= n) return;                       // the whole block lies past the sequence end
+  const int p_last = min(p0 + P, n) - 1;     // last valid position of the block
+  const int t0 = (p0 + 1) / BKV, t1 = (n - 1) / BKV;
+  const int ntiles = t1 - t0 + 1;
+  const size_t row_base = (size_t)b * p.cap;
+
+  if (ntiles <= 0) {   // no slot after the block: every row attends nothing -> 0
+    for (int idx = threadIdx.x; idx < (p_last - p0 + 1) * G; idx += blockDim.x) {
+      int pos = p0 + idx / G, hl = idx % G;
+      uint4 *dst = reinterpret_cast<uint4 *>(p.out + ((row_base + pos) * p.n_q_heads + g * G + hl) * DH);
+      for (int v = 0; v < DH / 8; ++v) dst[v] = make_uint4(0, 0, 0, 0);
+    }
+    return;
+  }
+
+  if (threadIdx.x == 0) {
+    mbar_init(q_full, 1);
+    for (int s = 0; s < KST; ++s) {
+      mbar_init(&k_full[s], 1);
+      mbar_init(&k_empty[s], 1);
+      mbar_init(&v_full[s], 1);
+      mbar_init(&v_empty[s], 1);
+    }
+    mbar_init(v_fixed, 1);
+    for (int h = 0; h < 2; ++h) {
+      mbar_init(&s_ready[h], 1);
+      mbar_init(&p_ready[h], 128);
+      mbar_init(&o_done[h], 1);
+    }
+    *abort_flag = 0;
+    fence_barrier_init();
+  }
+  if (warp == 9) tmem_alloc(tmem_slot, 512);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 8) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      tma_prefetch_desc(&tmQ);
+      tma_prefetch_desc(&tmK);
+      tma_prefetch_desc(&tmV);
+      mbar_arrive_expect_tx(q_full, L::NH * 128 * G * P);
+      for (int hh = 0; hh < L::NH; ++hh)
+        tma_load_3d(smem + L::OFF_Q + hh * 256 * 128, &tmQ, q_full, hh * 64, g * G,
+                    (int)row_base + p0);
+    }
+    for (int it = 0; it < ntiles; ++it) {
+      const int t = t0 + it, s = it % KST;
+      const uint32_t ph = (it / KST) & 1;
+      const int krow = (int)row_base + t * BKV;
+      int ok = 1;
+      if (lane == 0) {
+        ok = mbar_wait(&k_empty[s], ph ^ 1, abort_flag, p.status);
+        if (ok) {
+          mbar_arrive_expect_tx(&k_full[s], L::KV_BYTES);
+          for (int hh = 0; hh < L::NH; ++hh)
+            tma_load_3d(smem + L::OFF_K + s * L::KV_BYTES + hh * BKV * 128, &tmK, &k_full[s],
+                        hh * 64, g, krow);
+          ok = mbar_wait(&v_empty[s], ph ^ 1, abort_flag, p.status);
+        }
+        if (ok) {
+          mbar_arrive_expect_tx(&v_full[s], L::KV_BYTES);
+          for (int hh = 0; hh < L::NH; ++hh)
+            tma_load_3d(smem + L::OFF_V + s * L::KV_BYTES + hh * BKV * 128, &tmV, &v_full[s],
+                        hh * 64, g, krow);
+        }
+      }
+      ok = __shfl_sync(0xFFFFFFFFu, ok, 0);
+      if (!ok) break;
+      if (t == t1 && n - t * BKV < BKV) {
+        // rows past the sequence end may hold any bits; P is 0 there, but
+        // 0 * NaN would still poison O, so zero them before the PV product
+        if (!mbar_wait(&v_full[s], ph, abort_flag, p.status)) break;
+        const int first = n - t * BKV;
+        uint8_t *vs = smem + L::OFF_V + s * L::KV_BYTES;
+        for (int hh = 0; hh < L::NH; ++hh)
+          for (int idx = first * 8 + lane; idx < BKV * 8; idx += 32)
+            reinterpret_cast<uint4 *>(vs + hh * BKV * 128)[idx] = make_uint4(0, 0, 0, 0);
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(v_fixed);
+      }
+    }
+  } else if (warp == 9) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t idesc_qk = make_idesc_bf16(128, BKV, 0, 0);
+      constexpr uint32_t idesc_pv = make_idesc_bf16(128, DH, 0, 1);
+      const uint32_t q_s = smem_u32(smem + L::OFF_Q);
+      auto issue_qk = [&](int it, int h) {
+        const int s = it % KST;
+        const uint32_t k_s = smem_u32(smem + L::OFF_K + s * L::KV_BYTES);
+#pragma unroll
+        for (int kk = 0; kk < DH / 16; ++kk) {
+          const int hh = kk >> 2, ko = (kk & 3) * 32;
+          uint64_t ad = make_sdesc_sw128(q_s + hh * 256 * 128 + h * 128 * 128 + ko, 16, 1024);
+          uint64_t bd = make_sdesc_sw128(k_s + hh * BKV * 128 + ko, 16, 1024);
+          umma_ss(tmem + h * 128, ad, bd, idesc_qk, kk > 0);
+        }
+      };
+      bool ok = mbar_wait(q_full, 0, abort_flag, p.status);
+      if (ok) ok = mbar_wait(&k_full[0], 0, abort_flag, p.status);
+      if (ok) {
+        tc_fence_after();
+        issue_qk(0, 0);
+        umma_commit(&s_ready[0]);
+        issue_qk(0, 1);
+        umma_commit(&s_ready[1]);
+        umma_commit(&k_empty[0]);
+      }
+      for (int it = 0; ok && it < ntiles; ++it) {
+        const int t = t0 + it, s = it % KST;
+        const uint32_t ph = (it / KST) & 1;
+        if (!(ok = mbar_wait(&v_full[s], ph, abort_flag, p.status))) break;
+        if (t == t1 && n - t * BKV < BKV)
+          if (!(ok = mbar_wait(v_fixed, 0, abort_flag, p.status))) break;
+        const uint32_t v_s = smem_u32(smem + L::OFF_V + s * L::KV_BYTES);
+        for (int h = 0; h < 2; ++h) {
+          if (!(ok = mbar_wait(&p_ready[h], it & 1, abort_flag, p.status))) break;
+          tc_fence_after();
+#pragma unroll
+          for (int kk = 0; kk < BKV / 16; ++kk) {
+            // B = V tile, MN-major: 64-column halves 16 KB apart (LBO),
+            // 8-key groups 1024 B apart (SBO); A = P_h, bf16 pairs in TMEM.
+            uint64_t bd = make_sdesc_sw128(v_s + kk * 16 * 128, BKV * 128, 1024);
+            umma_ts(tmem + 256 + h * DH, tmem + h * 128 + kk * 8, bd, idesc_pv,
+                    (it > 0 || kk > 0) ? 1u : 0u);
+          }
+          if (h == 1) umma_commit(&v_empty[s]);
+          if (it + 1 < ntiles) {
+            const int s2 = (it + 1) % KST;
+            if (h == 0)
+              if (!(ok = mbar_wait(&k_full[s2], ((it + 1) / KST) & 1, abort_flag, p.status))) break;
+            tc_fence_after();
+            issue_qk(it + 1, h);
+            umma_commit(&s_ready[h]);
+            if (h == 1) umma_commit(&k_empty[s2]);
+          } else {
+            umma_commit(&o_done[h]);
+          }
+        }
+      }
+    }
+  } else {
+    // ------------------------------------------------------------ softmax
+    const int h = warp >> 2, q = warp & 3;
+    const int R = h * 128 + q * 32 + lane;              // unit row
+    const bool row_used = R < P * G;
+    const int pos = row_used ? p0 + R / G : 0x7FFFFFFF; // slot index of this row
+    const int hl = row_used ? R % G : 0;
+    const uint32_t lane_off = uint32_t(q * 32) << 16;
+    const uint32_t s_t = tmem + lane_off + h * 128;
+    const uint32_t o_t = tmem + lane_off + 256 + h * DH;
+    const float sl2 = p.scale_log2;
+    float m_used = -INFINITY, l = 0.f;
+    bool ok = true;
+    for (int it = 0; it < ntiles; ++it) {
+      const int j0 = (t0 + it) * BKV;
+      if (!(ok = mbar_wait(&s_ready[h], it & 1, abort_flag, p.status))) break;
+      tc_fence_after();
+      uint32_t sr[128];
+      tmem_ld32(s_t + 0, *reinterpret_cast<uint32_t(*)[32]>(&sr[0]));
+      tmem_ld32(s_t + 32, *reinterpret_cast<uint32_t(*)[32]>(&sr[32]));
+      tmem_ld32(s_t + 64, *reinterpret_cast<uint32_t(*)[32]>(&sr[64]));
+      tmem_ld32(s_t + 96, *reinterpret_cast<uint32_t(*)[32]>(&sr[96]));
+      tmem_ld_wait();
+      float mt = -INFINITY;
+      const bool need_mask = (j0 <= p0 + P - 1) || (j0 + BKV > n) || !row_used;
+      if (need_mask) {
+        // key j kept iff pos < j < n
+        const int lo = pos - j0;       // keep c > lo
+        const int hi = n - j0;         // keep c < hi
+#pragma unroll
+        for (int c = 0; c < 128; ++c) {
+          float x = (c > lo && c < hi) ? __uint_as_float(sr[c]) * sl2 : -INFINITY;
+          sr[c] = __float_as_uint(x);
+          mt = fmaxf(mt, x);
+        }
+      } else {
+#pragma unroll
+        for (int c = 0; c < 128; ++c) {
+          float x = __uint_as_float(sr[c]) * sl2;
+          sr[c] = __float_as_uint(x);
+          mt = fmaxf(mt, x);
+        }
+      }
+      // lazy rescaling: move the reference max only when it grows by more
+      // than 2^8, so exp2 stays <= 256 and O is rarely touched
+      const float m_new = fmaxf(m_used, mt);
+      const bool bump = m_new > m_used + 8.0f;        // also true for -inf -> finite
+      const bool rescale_o = bump && it > 0 && l > 0.f;
+      float factor = 1.f;
+      if (bump) {
+        factor = fast_exp2(m_used - m_new);           // 0 when m_used = -inf
+        l *= factor;
+        m_used = m_new;
+      }
+      if (__any_sync(0xFFFFFFFFu, rescale_o)) {
+        // O still holds the previous tiles' sum (S_ready implies the last PV is done)
+        const float f = rescale_o ? factor : 1.f;
+#pragma unroll 1
+        for (int c = 0; c < DH; c += 32) {
+          uint32_t o[32];
+          tmem_ld32(o_t + c, o);
+          tmem_ld_wait();
+#pragma unroll
+          for (int k = 0; k < 32; ++k) o[k] = __float_as_uint(__uint_as_float(o[k]) * f);
+          tmem_st32(o_t + c, o);
+        }
+      }
+      const float mref = (m_used == -INFINITY) ? 0.f : m_used;
+      float lsum = 0.f;
+#pragma unroll
+      for (int c0 = 0; c0 < 128; c0 += 32) {
+        uint32_t pk[16];
+#pragma unroll
+        for (int k = 0; k < 32; k += 2) {
+          float e0 = fast_exp2(__uint_as_float(sr[c0 + k]) - mref);
+          float e1 = fast_exp2(__uint_as_float(sr[c0 + k + 1]) - mref);
+          __nv_bfloat162 v2 = __floats2bfloat162_rn(e0, e1);
+          lsum += __low2float(v2) + __high2float(v2);
+          pk[k / 2] = *reinterpret_cast<uint32_t *>(&v2);
+        }
+        tmem_st16(s_t + c0 / 2, pk);
+      }
+      l += lsum;
+      tmem_st_wait();
+      tc_fence_before();
+      mbar_arrive(&p_ready[h]);
+    }
+    // ---- epilogue: O / l -> bf16 -> out[row_base + pos][g*G + hl][:]
+    if (ok) ok = mbar_wait(&o_done[h], 0, abort_flag, p.status);
+    if (ok) {
+      tc_fence_after();
+      const bool store = row_used && pos <= p_last;
+      const float inv = l > 0.f ? 1.f / l : 0.f;
+      __nv_bfloat16 *dst = p.out + ((row_base + (store ? pos : 0)) * p.n_q_heads + g * G + hl) * DH;
+#pragma unroll 1
+      for (int c = 0; c < DH; c += 32) {
+        uint32_t o[32];
+        tmem_ld32(o_t + c, o);
+        tmem_ld_wait();
+        uint32_t pk[16];
+#pragma unroll
+        for (int k = 0; k < 32; k += 2)
+          pk[k / 2] = pack_bf16x2(__uint_as_float(o[k]) * inv, __uint_as_float(o[k + 1]) * inv);
+        if (store) {
+          uint4 *d = reinterpret_cast<uint4 *>(dst + c);
+#pragma unroll
+          for (int v = 0; v < 4; ++v) d[v] = make_uint4(pk[v * 4], pk[v * 4 + 1], pk[v * 4 + 2], pk[v * 4 + 3]);
+        }
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (*abort_flag) __nanosleep(1000000);   // let copies still in flight land
+  if (warp == 9) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
+template <int DH>
+cudaError_t launch_dh(const CUtensorMap &q, const CUtensorMap &k, const CUtensorMap &v,
+                      const AttnParams &p, cudaStream_t stream) {
+  auto kern = attn_kernel<DH>;
+  static bool attr_set[64] = {};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev < 64 && !attr_set[dev]) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         AttnSmem<DH>::BYTES);
+    if (e != cudaSuccess) return e;
+    attr_set[dev] = true;
+  }
+  const long long units = (long long)p.batch * p.n_kv_heads * ((p.cap + p.P - 1) / p.P);
+  if (units <= 0) return cudaSuccess;
+  kern<<<(unsigned)units, kThreads, AttnSmem<DH>::BYTES, stream>>>(q, k, v, p);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+int attn_positions_per_unit(int group) { return 256 / group; }
+
+cudaError_t launch_attention(const CUtensorMap &q, const CUtensorMap &k, const CUtensorMap &v,
+                             const AttnParams &p, cudaStream_t stream) {
+  if (p.head_dim == 128) return launch_dh<128>(q, k, v, p, stream);
+  if (p.head_dim == 64) return launch_dh<64>(q, k, v, p, stream);
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace cc

@@ -1,0 +1,23 @@
+// attn.cuh -- interface of the counter-causal attention kernel.
+#pragma once
+#include "cc_common.cuh"
+
+namespace cc {
+
+struct AttnParams {
+  int batch, cap;
+  int n_q_heads, n_kv_heads, head_dim, group;
+  int P;                    // positions per work unit (attn_positions_per_unit(group))
+  const int32_t *seq_len;   // device [batch]
+  __nv_bfloat16 *out;       // [batch*cap][n_q_heads][head_dim]
+  float scale_log2;         // log2(e) / sqrt(head_dim)
+  unsigned *status;
+};
+
+int attn_positions_per_unit(int group);
+// q: 3-D map over Q [rows][Hq][dh], box {64, group, P}; k, v: 3-D maps over
+// the cache [batch*cap][Hkv][dh], box {64, 1, 128}; all 128-byte swizzled.
+cudaError_t launch_attention(const CUtensorMap &q, const CUtensorMap &k, const CUtensorMap &v,
+                             const AttnParams &p, cudaStream_t stream);
+
+}  // namespace cc

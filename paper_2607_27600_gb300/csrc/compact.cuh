@@ -1,0 +1,33 @@
+// compact.cuh -- in-place cache compaction kernel.
+#pragma once
+#include "cc_common.cuh"
+
+namespace cc {
+
+constexpr int kStageBytes = 64 * 1024;   // shared-memory staging per unit
+constexpr int kMaxCompactArrays = 2 * 128 + 3;
+
+struct CompactArray {
+  void *base;          // [batch][cap][row_bytes]
+  int row_bytes;       // bulk arrays: multiple of 16; otherwise 4
+  int bulk;            // rows moved by TMA bulk copies
+  int rows_per_chunk;  // destination slots per unit
+  int n_chunks;        // units per sequence = ceil(cap / rows_per_chunk)
+  int unit_base;       // first ticket of this array
+};
+
+struct CompactParams {
+  int batch, cap, n_arrays, total_units;
+  const int32_t *keep_idx;    // [batch][cap]
+  const int32_t *keep_count;  // [batch]
+  int32_t *seq_len;           // [batch], set to keep_count
+  unsigned *ticket;           // zeroed before launch
+  unsigned *flags;            // [total_units], zeroed before launch
+  unsigned *status;
+  CompactArray arr[kMaxCompactArrays];
+};
+
+size_t compact_stage_bytes();
+cudaError_t launch_compact(const CompactParams &p, int grid, cudaStream_t st);
+
+}  // namespace cc

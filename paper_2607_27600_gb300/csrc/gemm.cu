@@ -1,0 +1,342 @@
+// gemm.cu -- persistent tcgen05 GEMM  D[rows, N] = A[rows, K] * B[N, K]^T
+// (bf16 operands, fp32 accumulation in TMEM) with the epilogues the
+// counter-causal layer needs (Sec. 3.1, the "standard" layer re-run over the
+// cache): RoPE'd query projection, residual adds, SwiGLU, LM-head
+// log-sum-exp partials.
+//
+// Rows are the cache slots of a ragged batch: sequence b owns rows
+// b*cap + [0, seq_len[b]).  Only row tiles that hold valid slots are visited
+// (seq_len is read on the device).
+//
+// CTA = 6 warps, one CTA per SM, persistent over (row tile, column tile):
+//   warp 0      TMA producer (A 128x64 and B 256x64 bf16 tiles, 128B swizzle)
+//   warp 1      TMEM owner + single-thread tcgen05.mma issuer (M=128, N=256, K=16)
+//   warps 2..5  epilogue: tcgen05.ld of the accumulator (one row per thread)
+// Two 256-column accumulators in TMEM let the epilogue of one tile overlap
+// the main loop of the next.
+#include "gemm.cuh"
+
+namespace cc {
+
+namespace {
+
+constexpr int BM = 128, BN = 256, BK = 64, ST = 4;
+constexpr int A_BYTES = BM * BK * 2;   // 16 KB
+constexpr int B_BYTES = BN * BK * 2;   // 32 KB
+constexpr int kThreads = 192;
+constexpr int kMaxBatch = 1024;
+constexpr size_t kSmemBytes = 1024 /*align slack*/ + ST * (A_BYTES + B_BYTES) + 256 +
+                              (kMaxBatch + 1) * sizeof(int);
+
+CC_DEV float silu(float x) { return x / (1.0f + __expf(-x)); }
+
+// cos/sin of pos * inv_freq, with the angle reduced exactly: turns is
+// inv_freq / (2 pi) in 0.64 fixed point, so pos * turns mod 2^64 is the
+// fractional number of turns; its top 32 bits, read as a signed fraction of
+// a turn, give the angle in [-pi, pi).
+CC_DEV void rope_cs(uint32_t pos, unsigned long long turns, float &c, float &s) {
+  unsigned long long frac = (unsigned long long)pos * turns;
+  int32_t t32 = (int32_t)(frac >> 32);
+  float ang = (float)t32 * 1.4629180792671596e-09f;   // 2 pi / 2^32
+  __sincosf(ang, &s, &c);
+}
+
+template <int EPI>
+CC_DEV void epilogue_tile(const GemmParams &p, uint32_t tacc, int grow, bool valid, int nt,
+                          int tile_n0) {
+  if constexpr (EPI == EPI_F32 || EPI == EPI_RESID_BF16 || EPI == EPI_RESID_F32) {
+    float *out = reinterpret_cast<float *>(p.out) + (size_t)grow * p.ldo;
+#pragma unroll 1
+    for (int c = 0; c < BN / 32; ++c) {
+      uint32_t r[32];
+      tmem_ld32(tacc + c * 32, r);
+      tmem_ld_wait();
+      int col = tile_n0 + c * 32;
+      if (!valid || col >= p.N) continue;
+      float4 *dst = reinterpret_cast<float4 *>(out + col);
+      if constexpr (EPI == EPI_RESID_BF16) {
+        const uint4 *res = reinterpret_cast<const uint4 *>(
+            reinterpret_cast<const __nv_bfloat16 *>(p.resid) + (size_t)grow * p.ld_resid + col);
+#pragma unroll
+        for (int v = 0; v < 4; ++v) {
+          uint4 h = res[v];
+          uint32_t hw[4] = {h.x, h.y, h.z, h.w};
+#pragma unroll
+          for (int j = 0; j < 2; ++j) {
+            float4 o;
+            o.x = __uint_as_float(r[v * 8 + j * 4 + 0]) + bf16_lo(hw[j * 2 + 0]);
+            o.y = __uint_as_float(r[v * 8 + j * 4 + 1]) + bf16_hi(hw[j * 2 + 0]);
+            o.z = __uint_as_float(r[v * 8 + j * 4 + 2]) + bf16_lo(hw[j * 2 + 1]);
+            o.w = __uint_as_float(r[v * 8 + j * 4 + 3]) + bf16_hi(hw[j * 2 + 1]);
+            dst[v * 2 + j] = o;
+          }
+        }
+      } else {
+#pragma unroll
+        for (int v = 0; v < 8; ++v) {
+          float4 o = make_float4(__uint_as_float(r[v * 4 + 0]), __uint_as_float(r[v * 4 + 1]),
+                                 __uint_as_float(r[v * 4 + 2]), __uint_as_float(r[v * 4 + 3]));
+          if constexpr (EPI == EPI_RESID_F32) {
+            float4 h = dst[v];
+            o.x += h.x; o.y += h.y; o.z += h.z; o.w += h.w;
+          }
+          dst[v] = o;
+        }
+      }
+    }
+  } else if constexpr (EPI == EPI_QROPE) {
+    // Tile columns = BN / head_dim whole heads; rotate-half pairs (k, k+dh/2).
+    const int half = p.head_dim >> 1;
+    const uint32_t pos = valid ? (uint32_t)p.pos[grow] : 0u;
+    __nv_bfloat16 *out = reinterpret_cast<__nv_bfloat16 *>(p.out) + (size_t)grow * p.ldo;
+#pragma unroll 1
+    for (int hb = 0; hb < BN; hb += p.head_dim) {
+#pragma unroll 1
+      for (int c0 = 0; c0 < half; c0 += 32) {
+        uint32_t x1[32], x2[32];
+        tmem_ld32(tacc + hb + c0, x1);
+        tmem_ld32(tacc + hb + half + c0, x2);
+        tmem_ld_wait();
+        int col = tile_n0 + hb + c0;
+        if (!valid || col >= p.N) continue;
+        uint32_t o1[16], o2[16];
+#pragma unroll
+        for (int k = 0; k < 32; k += 2) {
+          float c_a, s_a, c_b, s_b;
+          rope_cs(pos, p.turns[c0 + k], c_a, s_a);
+          rope_cs(pos, p.turns[c0 + k + 1], c_b, s_b);
+          float a1 = __uint_as_float(x1[k]), a2 = __uint_as_float(x2[k]);
+          float b1 = __uint_as_float(x1[k + 1]), b2 = __uint_as_float(x2[k + 1]);
+          o1[k / 2] = pack_bf16x2(a1 * c_a - a2 * s_a, b1 * c_b - b2 * s_b);
+          o2[k / 2] = pack_bf16x2(a2 * c_a + a1 * s_a, b2 * c_b + b1 * s_b);
+        }
+        uint4 *d1 = reinterpret_cast<uint4 *>(out + col);
+        uint4 *d2 = reinterpret_cast<uint4 *>(out + col + half);
+#pragma unroll
+        for (int v = 0; v < 4; ++v) {
+          d1[v] = make_uint4(o1[v * 4], o1[v * 4 + 1], o1[v * 4 + 2], o1[v * 4 + 3]);
+          d2[v] = make_uint4(o2[v * 4], o2[v * 4 + 1], o2[v * 4 + 2], o2[v * 4 + 3]);
+        }
+      }
+    }
+  } else if constexpr (EPI == EPI_SWIGLU) {
+    // columns [0,128) = gate rows nt*128.., [128,256) = up rows nt*128..
+    __nv_bfloat16 *out = reinterpret_cast<__nv_bfloat16 *>(p.out) + (size_t)grow * p.ldo;
+#pragma unroll 1
+    for (int c0 = 0; c0 < 128; c0 += 32) {
+      uint32_t g[32], u[32];
+      tmem_ld32(tacc + c0, g);
+      tmem_ld32(tacc + 128 + c0, u);
+      tmem_ld_wait();
+      int col = nt * 128 + c0;
+      if (!valid || col >= p.N) continue;
+      uint32_t o[16];
+#pragma unroll
+      for (int k = 0; k < 32; k += 2)
+        o[k / 2] = pack_bf16x2(silu(__uint_as_float(g[k])) * __uint_as_float(u[k]),
+                               silu(__uint_as_float(g[k + 1])) * __uint_as_float(u[k + 1]));
+      uint4 *d = reinterpret_cast<uint4 *>(out + col);
+#pragma unroll
+      for (int v = 0; v < 4; ++v) d[v] = make_uint4(o[v * 4], o[v * 4 + 1], o[v * 4 + 2], o[v * 4 + 3]);
+    }
+  } else if constexpr (EPI == EPI_LSE) {
+    // per row: (max, sum exp(z - max)) over this tile's vocab columns, and the
+    // target logit when the row's token falls in the tile.
+    const int tok = valid ? p.tokens[grow] : -1;
+    float m = -INFINITY, s = 0.f, zt = 0.f;
+    bool has_t = false;
+#pragma unroll 1
+    for (int c = 0; c < BN / 32; ++c) {
+      uint32_t r[32];
+      tmem_ld32(tacc + c * 32, r);
+      tmem_ld_wait();
+      const int col = tile_n0 + c * 32;
+      float cm = -INFINITY;
+#pragma unroll
+      for (int k = 0; k < 32; ++k)
+        if (col + k < p.N) cm = fmaxf(cm, __uint_as_float(r[k]));
+      if (cm == -INFINITY) continue;
+      if (cm > m) {
+        s *= __expf(m - cm);
+        m = cm;
+      }
+#pragma unroll
+      for (int k = 0; k < 32; ++k)
+        if (col + k < p.N) s += __expf(__uint_as_float(r[k]) - m);
+      if (tok >= col && tok < col + 32) {
+#pragma unroll
+        for (int k = 0; k < 32; ++k)
+          if (k == tok - col) zt = __uint_as_float(r[k]);
+        has_t = true;
+      }
+    }
+    if (valid) {
+      reinterpret_cast<float2 *>(p.out)[(size_t)grow * p.ldo + nt] = make_float2(m, s);
+      if (has_t) p.z_target[grow] = zt;
+    }
+  }
+}
+
+template <int EPI>
+__global__ void __launch_bounds__(kThreads, 1)
+    gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                const __grid_constant__ CUtensorMap tmB2, const __grid_constant__ GemmParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                              ~uintptr_t(1023));
+  uint8_t *sA = smem;
+  uint8_t *sB = smem + ST * A_BYTES;
+  uint64_t *full = reinterpret_cast<uint64_t *>(sB + ST * B_BYTES);
+  uint64_t *empty = full + ST;
+  uint64_t *tfull = empty + ST;
+  uint64_t *tempty = tfull + 2;
+  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(tempty + 2);
+  volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
+  int *prefix = reinterpret_cast<int *>(smem + ST * (A_BYTES + B_BYTES) + 256);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < ST; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&tfull[a], 1);
+      mbar_init(&tempty[a], 4);
+    }
+    *abort_flag = 0;
+    build_tile_prefix(p.seq_len, p.batch, p.cap, BM, prefix, p.status);
+    fence_barrier_init();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmA);
+    tma_prefetch_desc(&tmB);
+    if (EPI == EPI_SWIGLU) tma_prefetch_desc(&tmB2);
+  }
+  if (warp == 1) tmem_alloc(tmem_slot, 512);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  const int num_m = prefix[p.batch];
+  const int total = num_m * p.n_tiles;
+  const int nk = (p.K + BK - 1) / BK;
+
+  if (warp == 0) {
+    if (lane == 0) {  // ---------------- TMA producer
+      int stage = 0;
+      uint32_t phase = 0;
+      for (int tile = blockIdx.x; tile < total; tile += gridDim.x) {
+        const int nt = tile / num_m, mt = tile - nt * num_m;
+        const int b = find_seq(prefix, p.batch, mt);
+        const int row0 = b * p.cap + (mt - prefix[b]) * BM;
+        for (int kb = 0; kb < nk; ++kb) {
+          if (!mbar_wait(&empty[stage], phase ^ 1, abort_flag, p.status)) goto producer_done;
+          mbar_arrive_expect_tx(&full[stage], A_BYTES + B_BYTES);
+          tma_load_2d(sA + stage * A_BYTES, &tmA, &full[stage], kb * BK, row0);
+          if constexpr (EPI == EPI_SWIGLU) {
+            tma_load_2d(sB + stage * B_BYTES, &tmB, &full[stage], kb * BK, nt * 128);
+            tma_load_2d(sB + stage * B_BYTES + B_BYTES / 2, &tmB2, &full[stage], kb * BK,
+                        nt * 128);
+          } else {
+            tma_load_2d(sB + stage * B_BYTES, &tmB, &full[stage], kb * BK, nt * BN);
+          }
+          if (++stage == ST) { stage = 0; phase ^= 1; }
+        }
+      }
+    producer_done:;
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {  // ---------------- MMA issuer
+      constexpr uint32_t idesc = make_idesc_bf16(BM, BN, 0, 0);
+      int stage = 0, acc = 0;
+      uint32_t phase = 0, acc_phase = 0;
+      for (int tile = blockIdx.x; tile < total; tile += gridDim.x) {
+        if (!mbar_wait(&tempty[acc], acc_phase ^ 1, abort_flag, p.status)) break;
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + acc * BN;
+        for (int kb = 0; kb < nk; ++kb) {
+          if (!mbar_wait(&full[stage], phase, abort_flag, p.status)) goto mma_done;
+          tc_fence_after();
+          const uint32_t a0 = smem_u32(sA + stage * A_BYTES);
+          const uint32_t b0 = smem_u32(sB + stage * B_BYTES);
+#pragma unroll
+          for (int k = 0; k < BK / 16; ++k) {
+            umma_ss(d_tmem, make_sdesc_sw128(a0 + k * 32, 16, 1024),
+                    make_sdesc_sw128(b0 + k * 32, 16, 1024), idesc, (kb | k) != 0);
+          }
+          umma_commit(&empty[stage]);
+          if (++stage == ST) { stage = 0; phase ^= 1; }
+        }
+        umma_commit(&tfull[acc]);
+        if (++acc == 2) { acc = 0; acc_phase ^= 1; }
+      }
+    mma_done:;
+    }
+  } else {  // ------------------------------ epilogue warps 2..5
+    const int q = warp & 3;        // TMEM lane quarter this warp may access
+    const int r = q * 32 + lane;   // accumulator row of this thread
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    for (int tile = blockIdx.x; tile < total; tile += gridDim.x) {
+      const int nt = tile / num_m, mt = tile - nt * num_m;
+      const int b = find_seq(prefix, p.batch, mt);
+      const int i = (mt - prefix[b]) * BM + r;
+      const bool valid = i < (p.seq_len ? p.seq_len[b] : p.cap);
+      const int grow = b * p.cap + i;
+      if (!mbar_wait(&tfull[acc], acc_phase, abort_flag, p.status)) break;
+      tc_fence_after();
+      const uint32_t tacc = tmem_base + acc * BN + (uint32_t(q * 32) << 16);
+      epilogue_tile<EPI>(p, tacc, grow, valid, nt, nt * BN);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&tempty[acc]);
+      if (++acc == 2) { acc = 0; acc_phase ^= 1; }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (*abort_flag) __nanosleep(1000000);   // let copies still in flight land
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, 512);
+  }
+}
+
+template <int EPI>
+cudaError_t launch(const CUtensorMap &a, const CUtensorMap &b, const CUtensorMap &b2,
+                   const GemmParams &p, int grid, cudaStream_t stream) {
+  auto kern = gemm_kernel<EPI>;
+  static bool attr_set[64] = {};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev < 64 && !attr_set[dev]) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)kSmemBytes);
+    if (e != cudaSuccess) return e;
+    attr_set[dev] = true;
+  }
+  kern<<<grid, kThreads, kSmemBytes, stream>>>(a, b, b2, p);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+int gemm_block_n(int epi) { return epi == EPI_SWIGLU ? 128 : BN; }
+int gemm_max_batch() { return kMaxBatch; }
+
+cudaError_t launch_gemm(int epi, const CUtensorMap &a, const CUtensorMap &b, const CUtensorMap &b2,
+                        const GemmParams &p, int grid, cudaStream_t stream) {
+  switch (epi) {
+    case EPI_F32: return launch<EPI_F32>(a, b, b2, p, grid, stream);
+    case EPI_QROPE: return launch<EPI_QROPE>(a, b, b2, p, grid, stream);
+    case EPI_RESID_BF16: return launch<EPI_RESID_BF16>(a, b, b2, p, grid, stream);
+    case EPI_RESID_F32: return launch<EPI_RESID_F32>(a, b, b2, p, grid, stream);
+    case EPI_SWIGLU: return launch<EPI_SWIGLU>(a, b, b2, p, grid, stream);
+    case EPI_LSE: return launch<EPI_LSE>(a, b, b2, p, grid, stream);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+}  // namespace cc

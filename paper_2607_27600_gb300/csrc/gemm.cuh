@@ -1,0 +1,41 @@
+// gemm.cuh -- interface of the tcgen05 GEMM with fused epilogues.
+#pragma once
+#include "cc_common.cuh"
+
+namespace cc {
+
+enum GemmEpi : int {
+  EPI_F32 = 0,        // out fp32 [rows][ldo] = acc
+  EPI_QROPE = 1,      // out bf16 [rows][ldo] = RoPE(acc) at pos[row], per head
+  EPI_RESID_BF16 = 2, // out fp32 [rows][ldo] = acc + resid bf16 [rows][ld_resid]
+  EPI_RESID_F32 = 3,  // out fp32 [rows][ldo] += acc
+  EPI_SWIGLU = 4,     // out bf16 [rows][ldo] = silu(A Wg^T) * (A Wu^T)   (B = Wg, B2 = Wu)
+  EPI_LSE = 5         // out float2 [rows][ldo = n_tiles] = (max, sum exp) per vocab tile,
+                      // z_target[row] = logit of tokens[row]
+};
+
+struct GemmParams {
+  int batch, cap;
+  const int32_t *seq_len;  // device [batch]
+  int N, K;
+  int n_tiles;             // column tiles (of gemm_block_n(epi) columns)
+  void *out;
+  int ldo;
+  const void *resid;
+  int ld_resid;
+  const int32_t *pos;      // EPI_QROPE
+  int head_dim;            // EPI_QROPE
+  const int32_t *tokens;   // EPI_LSE
+  float *z_target;         // EPI_LSE
+  unsigned *status;
+  unsigned long long turns[64];  // EPI_QROPE: inv_freq_k / (2 pi) in 0.64 fixed point
+};
+
+int gemm_block_n(int epi);
+int gemm_max_batch();
+// a: A rows x K (box 64 x 128); b (and b2 for SwiGLU): weights N x K (box 64 x 256,
+// or 64 x 128 for SwiGLU).  grid: persistent CTAs (one per SM).
+cudaError_t launch_gemm(int epi, const CUtensorMap &a, const CUtensorMap &b, const CUtensorMap &b2,
+                        const GemmParams &p, int grid, cudaStream_t stream);
+
+}  // namespace cc

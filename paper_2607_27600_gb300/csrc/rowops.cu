@@ -1,0 +1,214 @@
+// rowops.cu -- per-row kernels of the scoring pass: RMSNorm, embedding
+// gather (full pass), the target-logit head and the log-sum-exp combine
+// (Sec. 3.1: the score of row i is read off the logit of its own token x_i).
+//
+// One warp per cache row, rows = b*cap + i; rows with i >= seq_len[b] are
+// skipped (the heads write -inf there).  All are HBM-bound streams with
+// 16-byte vector accesses.
+#include "rowops.cuh"
+
+namespace cc {
+
+namespace {
+
+constexpr int kWarps = 8;  // warps (rows) per block
+
+CC_DEV bool row_valid(const int32_t *seq_len, int cap, int row, int &i, int &n) {
+  const int b = row / cap;
+  i = row - b * cap;
+  n = seq_len[b];
+  return i < n && n <= cap;
+}
+
+// 8 bf16 of a uint4 -> float
+CC_DEV void unpack8(const uint4 &v, float *f) {
+  f[0] = bf16_lo(v.x); f[1] = bf16_hi(v.x); f[2] = bf16_lo(v.y); f[3] = bf16_hi(v.y);
+  f[4] = bf16_lo(v.z); f[5] = bf16_hi(v.z); f[6] = bf16_lo(v.w); f[7] = bf16_hi(v.w);
+}
+
+// Loads elements [e, e+8) of a row as float (bf16 or fp32 source).
+template <bool IN_F32>
+CC_DEV void load8(const void *row, int e, float *f) {
+  if constexpr (IN_F32) {
+    const float4 *p = reinterpret_cast<const float4 *>(reinterpret_cast<const float *>(row) + e);
+    float4 a = p[0], b = p[1];
+    f[0] = a.x; f[1] = a.y; f[2] = a.z; f[3] = a.w; f[4] = b.x; f[5] = b.y; f[6] = b.z; f[7] = b.w;
+  } else {
+    unpack8(*reinterpret_cast<const uint4 *>(reinterpret_cast<const __nv_bfloat16 *>(row) + e), f);
+  }
+}
+
+template <bool IN_F32>
+CC_DEV float row_inv_rms(const void *row, int d, float eps, int lane) {
+  float ss = 0.f;
+  for (int e = lane * 8; e < d; e += 256) {
+    float f[8];
+    load8<IN_F32>(row, e, f);
+#pragma unroll
+    for (int k = 0; k < 8; ++k) ss = fmaf(f[k], f[k], ss);
+  }
+  ss = warp_sum(ss);
+  return rsqrtf(ss / (float)d + eps);
+}
+
+// out (bf16) = x * gain / rms(x)
+template <bool IN_F32>
+__global__ void __launch_bounds__(kWarps * 32)
+    rmsnorm_kernel(const void *x, const __nv_bfloat16 *gain, __nv_bfloat16 *out, int d, float eps,
+                   const int32_t *seq_len, int cap, int rows) {
+  const int lane = threadIdx.x & 31;
+  const int row = blockIdx.x * kWarps + (threadIdx.x >> 5);
+  int i, n;
+  if (row >= rows || !row_valid(seq_len, cap, row, i, n)) return;
+  const size_t es = IN_F32 ? 4 : 2;
+  const void *xr = reinterpret_cast<const uint8_t *>(x) + (size_t)row * d * es;
+  const float inv = row_inv_rms<IN_F32>(xr, d, eps, lane);
+  __nv_bfloat16 *o = out + (size_t)row * d;
+  for (int e = lane * 8; e < d; e += 256) {
+    float f[8], gf[8];
+    load8<IN_F32>(xr, e, f);
+    unpack8(*reinterpret_cast<const uint4 *>(gain + e), gf);
+    uint4 v;
+    v.x = pack_bf16x2(f[0] * inv * gf[0], f[1] * inv * gf[1]);
+    v.y = pack_bf16x2(f[2] * inv * gf[2], f[3] * inv * gf[3]);
+    v.z = pack_bf16x2(f[4] * inv * gf[4], f[5] * inv * gf[5]);
+    v.w = pack_bf16x2(f[6] * inv * gf[6], f[7] * inv * gf[7]);
+    *reinterpret_cast<uint4 *>(o + e) = v;
+  }
+}
+
+// h (fp32) = embed[tokens[row]]
+__global__ void __launch_bounds__(kWarps * 32)
+    embed_kernel(const __nv_bfloat16 *embed, const int32_t *tokens, float *h, int d, int vocab,
+                 const int32_t *seq_len, int cap, int rows, unsigned *status) {
+  const int lane = threadIdx.x & 31;
+  const int row = blockIdx.x * kWarps + (threadIdx.x >> 5);
+  int i, n;
+  if (row >= rows || !row_valid(seq_len, cap, row, i, n)) return;
+  int tok = tokens[row];
+  if (tok < 0 || tok >= vocab) {
+    if (lane == 0) set_status(status, CC_ERR_DEVICE_ARG);
+    tok = 0;
+  }
+  const __nv_bfloat16 *src = embed + (size_t)tok * d;
+  float *dst = h + (size_t)row * d;
+  for (int e = lane * 8; e < d; e += 256) {
+    float f[8];
+    unpack8(*reinterpret_cast<const uint4 *>(src + e), f);
+    reinterpret_cast<float4 *>(dst + e)[0] = make_float4(f[0], f[1], f[2], f[3]);
+    reinterpret_cast<float4 *>(dst + e)[1] = make_float4(f[4], f[5], f[6], f[7]);
+  }
+}
+
+// score = -(RMSNorm(h) * g) . W_U[x_i]; last valid slot +inf; past the end -inf.
+__global__ void __launch_bounds__(kWarps * 32)
+    head_logit_kernel(const float *h, const __nv_bfloat16 *gain, const __nv_bfloat16 *lm_head,
+                      const int32_t *tokens, float *scores, int d, int vocab, float eps,
+                      const int32_t *seq_len, int cap, int rows, unsigned *status) {
+  const int lane = threadIdx.x & 31;
+  const int row = blockIdx.x * kWarps + (threadIdx.x >> 5);
+  if (row >= rows) return;
+  int i, n;
+  if (!row_valid(seq_len, cap, row, i, n)) {
+    if (lane == 0) scores[row] = -INFINITY;
+    return;
+  }
+  if (i == n - 1) {   // no future context: maximum surprise, always retained
+    if (lane == 0) scores[row] = INFINITY;
+    return;
+  }
+  int tok = tokens[row];
+  if (tok < 0 || tok >= vocab) {
+    if (lane == 0) set_status(status, CC_ERR_DEVICE_ARG);
+    tok = 0;
+  }
+  const float *hr = h + (size_t)row * d;
+  const float inv = row_inv_rms<true>(hr, d, eps, lane);
+  const __nv_bfloat16 *w = lm_head + (size_t)tok * d;
+  float z = 0.f;
+  for (int e = lane * 8; e < d; e += 256) {
+    float f[8], gf[8], wf[8];
+    load8<true>(hr, e, f);
+    unpack8(*reinterpret_cast<const uint4 *>(gain + e), gf);
+    unpack8(*reinterpret_cast<const uint4 *>(w + e), wf);
+#pragma unroll
+    for (int k = 0; k < 8; ++k) z = fmaf(f[k] * gf[k], wf[k], z);
+  }
+  z = warp_sum(z) * inv;
+  if (lane == 0) scores[row] = -z;
+}
+
+// score = -(z_target - logsumexp) from per-tile (max, sum exp) partials.
+__global__ void __launch_bounds__(kWarps * 32)
+    lse_combine_kernel(const float2 *part, int n_tiles, const float *z_target, float *scores,
+                       const int32_t *seq_len, int cap, int rows) {
+  const int lane = threadIdx.x & 31;
+  const int row = blockIdx.x * kWarps + (threadIdx.x >> 5);
+  if (row >= rows) return;
+  int i, n;
+  if (!row_valid(seq_len, cap, row, i, n)) {
+    if (lane == 0) scores[row] = -INFINITY;
+    return;
+  }
+  if (i == n - 1) {
+    if (lane == 0) scores[row] = INFINITY;
+    return;
+  }
+  const float2 *pr = part + (size_t)row * n_tiles;
+  float m = -INFINITY;
+  for (int t = lane; t < n_tiles; t += 32) m = fmaxf(m, pr[t].x);
+  m = warp_max(m);
+  float s = 0.f;
+  for (int t = lane; t < n_tiles; t += 32) s += pr[t].y * __expf(pr[t].x - m);
+  s = warp_sum(s);
+  if (lane == 0) scores[row] = (m + __logf(s)) - z_target[row];
+}
+
+unsigned blocks_for(int rows) { return (unsigned)((rows + kWarps - 1) / kWarps); }
+
+}  // namespace
+
+cudaError_t launch_rmsnorm(const void *x, bool x_f32, const void *gain, void *out, int d, float eps,
+                           const int32_t *seq_len, int cap, int rows, cudaStream_t st) {
+  if (rows <= 0) return cudaSuccess;
+  auto *g = reinterpret_cast<const __nv_bfloat16 *>(gain);
+  auto *o = reinterpret_cast<__nv_bfloat16 *>(out);
+  if (x_f32)
+    rmsnorm_kernel<true><<<blocks_for(rows), kWarps * 32, 0, st>>>(x, g, o, d, eps, seq_len, cap, rows);
+  else
+    rmsnorm_kernel<false><<<blocks_for(rows), kWarps * 32, 0, st>>>(x, g, o, d, eps, seq_len, cap, rows);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_embed(const void *embed, const int32_t *tokens, float *h, int d, int vocab,
+                         const int32_t *seq_len, int cap, int rows, unsigned *status,
+                         cudaStream_t st) {
+  if (rows <= 0) return cudaSuccess;
+  embed_kernel<<<blocks_for(rows), kWarps * 32, 0, st>>>(
+      reinterpret_cast<const __nv_bfloat16 *>(embed), tokens, h, d, vocab, seq_len, cap, rows,
+      status);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_head_logit(const float *h, const void *gain, const void *lm_head,
+                              const int32_t *tokens, float *scores, int d, int vocab, float eps,
+                              const int32_t *seq_len, int cap, int rows, unsigned *status,
+                              cudaStream_t st) {
+  if (rows <= 0) return cudaSuccess;
+  head_logit_kernel<<<blocks_for(rows), kWarps * 32, 0, st>>>(
+      h, reinterpret_cast<const __nv_bfloat16 *>(gain),
+      reinterpret_cast<const __nv_bfloat16 *>(lm_head), tokens, scores, d, vocab, eps, seq_len,
+      cap, rows, status);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_lse_combine(const float2 *part, int n_tiles, const float *z_target,
+                               float *scores, const int32_t *seq_len, int cap, int rows,
+                               cudaStream_t st) {
+  if (rows <= 0) return cudaSuccess;
+  lse_combine_kernel<<<blocks_for(rows), kWarps * 32, 0, st>>>(part, n_tiles, z_target, scores,
+                                                              seq_len, cap, rows);
+  return cudaGetLastError();
+}
+
+}  // namespace cc

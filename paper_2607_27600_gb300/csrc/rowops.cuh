@@ -1,0 +1,24 @@
+// rowops.cuh -- per-row kernels of the scoring pass.
+#pragma once
+#include "cc_common.cuh"
+
+namespace cc {
+
+// out bf16 [rows][d] = x * gain / sqrt(mean(x^2) + eps); x bf16 or fp32 [rows][d]
+cudaError_t launch_rmsnorm(const void *x, bool x_f32, const void *gain, void *out, int d, float eps,
+                           const int32_t *seq_len, int cap, int rows, cudaStream_t st);
+// h fp32 [rows][d] = embed[tokens[row]]
+cudaError_t launch_embed(const void *embed, const int32_t *tokens, float *h, int d, int vocab,
+                         const int32_t *seq_len, int cap, int rows, unsigned *status,
+                         cudaStream_t st);
+// scores[row] = -(final-norm(h) . lm_head[tokens[row]]), +inf at the last slot
+cudaError_t launch_head_logit(const float *h, const void *gain, const void *lm_head,
+                              const int32_t *tokens, float *scores, int d, int vocab, float eps,
+                              const int32_t *seq_len, int cap, int rows, unsigned *status,
+                              cudaStream_t st);
+// scores[row] = logsumexp - z_target, +inf at the last slot
+cudaError_t launch_lse_combine(const float2 *part, int n_tiles, const float *z_target,
+                               float *scores, const int32_t *seq_len, int cap, int rows,
+                               cudaStream_t st);
+
+}  // namespace cc

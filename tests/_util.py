@@ -72,3 +72,43 @@ def rel_err(got, want):
     g, o = got[fin], want[fin]
     rms = np.sqrt(np.mean(o * o))
     return float(np.max(np.abs(g - o) / np.maximum(np.abs(o), rms)))
+
+
+def to_device(x, device="cuda"):
+    """numpy tree -> torch tree on `device`: floats as bf16, integers as int32."""
+    if x is None:
+        return None
+    if isinstance(x, dict):
+        return {k: to_device(v, device) for k, v in x.items()}
+    if isinstance(x, (list, tuple)):
+        return [to_device(v, device) for v in x]
+    a = np.ascontiguousarray(x)
+    t = torch.from_numpy(a)
+    t = t.to(torch.bfloat16) if a.dtype.kind == "f" else t.to(torch.int32)
+    return t.to(device)
+
+
+def keep_set_ok(got_idx, got_cnt, want_idx, want_cnt, oracle_scores, seq_lens, budgets, tol=2e-2):
+    """Keep-set criterion: identical where the oracle's score gap at the
+    budget boundary exceeds `tol` (relative to the scores' rms), otherwise
+    >= 99.5 % overlap.  Returns (ok, details)."""
+    details = []
+    ok = True
+    for b, (n, j) in enumerate(zip(seq_lens, budgets)):
+        jj = min(j, n)
+        g = set(np.asarray(got_idx[b, :got_cnt[b]]).tolist())
+        w = set(np.asarray(want_idx[b, :want_cnt[b]]).tolist())
+        if got_cnt[b] != want_cnt[b]:
+            return False, f"count {got_cnt[b]} != {want_cnt[b]}"
+        s = np.asarray(oracle_scores[b, :n], np.float64)
+        fin = s[np.isfinite(s)]
+        rms = np.sqrt(np.mean(fin * fin)) if fin.size else 1.0
+        srt = np.sort(s)[::-1]
+        gap = (srt[jj - 1] - srt[jj]) / rms if jj < n else np.inf
+        overlap = len(g & w) / max(1, len(w))
+        if gap > tol:
+            ok &= g == w
+        else:
+            ok &= overlap >= 0.995
+        details.append((b, gap, overlap))
+    return bool(ok), details

@@ -1,0 +1,66 @@
+"""The C ABI library builds, loads without a GPU and exports every entry
+point the public headers declare; host-side argument checks answer without
+touching the device (no GPU)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def declared_functions():
+    names = set()
+    for h in os.listdir(os.path.join(ROOT, "include")):
+        if h.endswith(".h"):
+            src = open(os.path.join(ROOT, "include", h)).read()
+            src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+            names |= set(re.findall(r"\b(cc_[a-z0-9_]+)\s*\(", src))
+    return names
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2607_27600_gb300 import build, cc
+    build.build_library()
+    return cc.load_library()
+
+
+def test_every_declared_symbol_is_exported(lib):
+    names = declared_functions()
+    assert {"cc_score_layer", "cc_score_full", "cc_select_keep", "cc_compact_kv"} <= names
+    for n in sorted(names):
+        assert hasattr(lib, n), n
+
+
+def test_binding_covers_every_declared_symbol(lib):
+    from paper_2607_27600_gb300 import cc
+    assert declared_functions() == set(cc.exported_symbols())
+
+
+def test_status_strings(lib):
+    from paper_2607_27600_gb300 import cc
+    assert cc.cc_status_str(cc.CC_OK) == "ok"
+    assert "workspace" in cc.cc_status_str(cc.CC_ERR_WORKSPACE)
+
+
+def test_host_side_validation_without_device(lib):
+    from paper_2607_27600_gb300 import cc
+    # null arguments are rejected before anything reaches the device
+    assert lib.cc_select_keep(None, None, 1, 1, None, 0, None, None, None, 0, None) == \
+        cc.CC_ERR_INVALID_ARG
+    assert lib.cc_score_layer(None, None, None, 0, None, None, 0, None) == cc.CC_ERR_INVALID_ARG
+    bad = cc.cc_model_cfg(1, 100, 8, 3, 128, 256, 10, 1e4, 1e-5)   # Hq % Hkv != 0
+    assert lib.cc_score_workspace_size(ctypes.byref(bad), 1, 16, 0) == 0
+    odd = cc.cc_model_cfg(1, 256, 8, 2, 96, 256, 10, 1e4, 1e-5)    # head_dim 96
+    assert lib.cc_score_workspace_size(ctypes.byref(odd), 1, 16, 0) == 0
+
+
+def test_workspace_size_formula(lib):
+    from paper_2607_27600_gb300 import cc
+    from synth.configs import LLAMA3_8B
+    n = cc.cc_score_workspace_size(LLAMA3_8B, 1, 8192, cc.SCORE_LOGIT)
+    rows, d, q, f = 8192, 4096, 4096, 14336
+    assert n >= rows * (2 * d + 2 * q * 2 + 4 * d + 2 * f)
+    assert cc.cc_score_workspace_size(LLAMA3_8B, 1, 8192, cc.SCORE_LOGPROB) > n

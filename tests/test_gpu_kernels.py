@@ -1,0 +1,108 @@
+"""GPU unit tests of single kernels through the C ABI: the tcgen05 GEMM and
+the counter-causal attention (Sec. 3.1), against the CPU oracle / fp64
+reference on seeded inputs."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def cc():
+    from paper_2607_27600_gb300 import cc as mod
+    mod.load_library()
+    return mod
+
+
+@pytest.mark.parametrize("rows,n,k", [(128, 256, 64), (300, 96, 200), (1000, 512, 4096),
+                                      (129, 32, 8), (2048, 4096, 1408)])
+def test_linear_matches_fp64(cc, rows, n, k):
+    x = synth.normal((rows, k), 1.0, 1, f"x{rows}.{n}.{k}")
+    w = synth.normal((n, k), 0.05, 1, f"w{rows}.{n}.{k}")
+    y = torch.empty(rows, n, dtype=torch.float32, device="cuda")
+    cc.cc_linear_f32(x.cuda(), w.cuda(), y)
+    torch.cuda.synchronize()
+    want = x.double() @ w.double().T
+    err = (y.cpu().double() - want).abs().max().item()
+    scale = want.abs().max().item()
+    assert err <= 1e-4 * scale + 1e-5, (err, scale)
+
+
+def _attn_case(cc, batch, cap, seq, hq, hkv, dh, seed, kscale=1.0):
+    q = synth.normal((batch * cap, hq, dh), 1.0, seed, "q")
+    k = synth.normal((batch, cap, hkv, dh), kscale, seed, "k")
+    v = synth.normal((batch, cap, hkv, dh), 1.0, seed, "v")
+    sl = torch.tensor(seq, dtype=torch.int32)
+    out = torch.full((batch * cap, hq, dh), float("nan"), dtype=torch.bfloat16, device="cuda")
+    cc.cc_counter_causal_attention(q.cuda(), k.cuda(), v.cuda(), sl.cuda(), out, batch, cap, hq,
+                                   hkv, dh)
+    assert cc.cc_get_status() == cc.CC_OK
+    got = out.float().cpu().numpy().reshape(batch, cap, hq, dh)
+    qn = q.float().numpy().reshape(batch, cap, hq, dh)
+    kn, vn = k.float().numpy(), v.float().numpy()
+    for b, n in enumerate(seq):
+        want = oracle.counter_causal_attention(qn[b, :n], kn[b], vn[b], np.arange(n), n)
+        g = got[b, :n]
+        assert np.all(np.isfinite(g))
+        err = np.abs(g - want).max() if n else 0.0
+        # bf16 output rounding (2^-9 relative) plus bf16 P in the PV product
+        assert err <= 2e-2 * max(1.0, np.abs(want).max()), (b, n, err)
+        if n:
+            np.testing.assert_array_equal(g[n - 1], 0.0)   # last row: nothing to attend
+
+
+@pytest.mark.parametrize("hq,hkv,dh", [(8, 2, 64), (32, 8, 128), (28, 4, 128), (4, 4, 128),
+                                       (8, 1, 64)])
+def test_attention_shapes(cc, hq, hkv, dh):
+    _attn_case(cc, 2, 384, [384, 301], hq, hkv, dh, seed=hq * 7 + dh)
+
+
+@pytest.mark.parametrize("seq", [[1], [2], [3], [129], [127, 128], [256, 1, 5, 200]])
+def test_attention_edge_lengths(cc, seq):
+    _attn_case(cc, len(seq), 256, seq, 8, 2, 128, seed=sum(seq))
+
+
+def test_attention_ragged_large_ragged_tail(cc):
+    _attn_case(cc, 2, 1200, [1200, 777], 32, 8, 128, seed=5, kscale=2.0)
+
+
+def test_attention_ignores_non_finite_stale_slots(cc):
+    """Slots past seq_len may hold any bits (NaN here); outputs must not see them."""
+    batch, cap, hq, hkv, dh = 1, 256, 8, 2, 128
+    seq = [150]
+    q = synth.normal((cap, hq, dh), 1.0, 9, "q").cuda()
+    k = synth.normal((batch, cap, hkv, dh), 1.0, 9, "k").cuda()
+    v = synth.normal((batch, cap, hkv, dh), 1.0, 9, "v").cuda()
+    k2, v2 = k.clone(), v.clone()
+    k2[:, 150:] = float("nan")
+    v2[:, 150:] = float("inf")
+    sl = torch.tensor(seq, dtype=torch.int32, device="cuda")
+    o1 = torch.zeros(cap, hq, dh, dtype=torch.bfloat16, device="cuda")
+    o2 = torch.zeros_like(o1)
+    cc.cc_counter_causal_attention(q, k, v, sl, o1, batch, cap, hq, hkv, dh)
+    cc.cc_counter_causal_attention(q, k2, v2, sl, o2, batch, cap, hq, hkv, dh)
+    torch.cuda.synchronize()
+    assert torch.equal(o1[:150], o2[:150])
+
+
+def test_attention_past_slots_do_not_leak(cc):
+    """Row i is bitwise unchanged when K/V at slots <= i change (masked p = 0)."""
+    batch, cap, hq, hkv, dh = 1, 512, 8, 2, 128
+    q = synth.normal((cap, hq, dh), 1.0, 10, "q").cuda()
+    k = synth.normal((batch, cap, hkv, dh), 1.0, 10, "k").cuda()
+    v = synth.normal((batch, cap, hkv, dh), 1.0, 10, "v").cuda()
+    sl = torch.tensor([512], dtype=torch.int32, device="cuda")
+    o1 = torch.zeros(cap, hq, dh, dtype=torch.bfloat16, device="cuda")
+    o2 = torch.zeros_like(o1)
+    cc.cc_counter_causal_attention(q, k, v, sl, o1, batch, cap, hq, hkv, dh)
+    k2, v2 = k.clone(), v.clone()
+    k2[:, :301] += 3.0
+    v2[:, :301] -= 5.0
+    cc.cc_counter_causal_attention(q, k2, v2, sl, o2, batch, cap, hq, hkv, dh)
+    torch.cuda.synchronize()
+    assert torch.equal(o1[300:], o2[300:])
+    assert not torch.equal(o1[:299], o2[:299])

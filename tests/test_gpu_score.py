@@ -1,0 +1,196 @@
+"""GPU parity of the scoring pass, keep-set and compaction (C ABI) against
+the CPU oracle on small seeded workloads with every row checked."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+from synth.configs import ModelShape
+from tests._util import causal_cache, keep_set_ok, rel_err, to_device, to_np
+
+pytestmark = pytest.mark.gpu
+
+TOL = 2e-2
+# small shape the kernels accept (d, d_ff multiples of 32; head_dim 64), two layers
+SMALL_GPU = ModelShape(n_layers=2, d_model=256, n_q_heads=8, n_kv_heads=2, head_dim=64,
+                       d_ff=384, vocab=1000, rope_theta=1e4, rms_eps=1e-5)
+
+
+@pytest.fixture(scope="module")
+def pkg():
+    import paper_2607_27600_gb300 as p
+    p.load_library()
+    return p
+
+
+def _setup(shape, seq, cap, seed):
+    w_np = to_np(synth.model_weights(shape, seed, with_kv_proj=True))
+    c_np = causal_cache(shape, w_np, seq, cap, seed)
+    return w_np, c_np
+
+
+def _gpu(pkg, w_np, c_np):
+    w, c = to_device(w_np), to_device(c_np)
+    return pkg.Weights(w), pkg.Cache(c)
+
+
+def _run_score(pkg, shape, weights, cache, mode, full):
+    from paper_2607_27600_gb300 import cc
+    b, cap = cache.d["tokens"].shape
+    scores = torch.full((b, cap), float("nan"), dtype=torch.float32, device="cuda")
+    ws = cc.alloc_workspace(cc.cc_score_workspace_size(shape, b, cap, mode))
+    fn = cc.cc_score_full if full else cc.cc_score_layer
+    fn(shape, weights, cache, mode, scores, ws)
+    assert cc.cc_get_status() == cc.CC_OK
+    return scores.cpu().numpy()
+
+
+@pytest.fixture(scope="module")
+def tiny(pkg):
+    wl = synth.WORKLOADS["tiny-512"]
+    w_np, c_np = _setup(wl.shape, wl.seq_lens, wl.cap, wl.seed)
+    return wl, w_np, c_np
+
+
+@pytest.mark.parametrize("mode", ["logit", "logprob"])
+def test_tiny_single_layer_all_rows(pkg, tiny, mode):
+    from paper_2607_27600_gb300 import cc
+    wl, w_np, c_np = tiny
+    want = oracle.score_layer(wl.shape, w_np, c_np, mode=mode)
+    weights, cache = _gpu(pkg, w_np, c_np)
+    m = cc.SCORE_LOGIT if mode == "logit" else cc.SCORE_LOGPROB
+    got = _run_score(pkg, wl.shape, weights, cache, m, full=False)
+    assert rel_err(got, want) < TOL
+    # the fast pass of a 1-layer model is the full pass
+    got_full = _run_score(pkg, wl.shape, weights, cache, m, full=True)
+    assert rel_err(got_full, want) < TOL
+
+
+@pytest.mark.parametrize("mode", ["logit", "logprob"])
+def test_small_two_layer_full_and_fast_ragged(pkg, mode):
+    from paper_2607_27600_gb300 import cc
+    seq, cap = [300, 129, 1, 64], 320
+    w_np, c_np = _setup(SMALL_GPU, seq, cap, seed=21)
+    m = cc.SCORE_LOGIT if mode == "logit" else cc.SCORE_LOGPROB
+    weights, cache = _gpu(pkg, w_np, c_np)
+    for full, fn in ((True, oracle.score_full), (False, oracle.score_layer)):
+        want = fn(SMALL_GPU, w_np, c_np, mode=mode)
+        got = _run_score(pkg, SMALL_GPU, weights, cache, m, full=full)
+        assert rel_err(got, want) < TOL, (full, rel_err(got, want))
+
+
+def test_tiny_refresh_keep_set_and_compaction(pkg, tiny):
+    from paper_2607_27600_gb300 import cc
+    wl, w_np, c_np = tiny
+    want = oracle.score_layer(wl.shape, w_np, c_np)
+    weights, cache = _gpu(pkg, w_np, c_np)
+    got = _run_score(pkg, wl.shape, weights, cache, cc.SCORE_LOGIT, full=False)
+    b, cap = c_np["tokens"].shape
+    budget = torch.tensor(wl.budgets, dtype=torch.int32, device="cuda")
+    keep_idx = torch.full((b, cap), -1, dtype=torch.int32, device="cuda")
+    keep_count = torch.zeros(b, dtype=torch.int32, device="cuda")
+    scores_dev = torch.from_numpy(got).cuda()
+    cc.cc_select_keep(scores_dev, cache.d["seq_len"], b, cap, budget, 0, keep_idx, keep_count)
+    gi, gc = keep_idx.cpu().numpy(), keep_count.cpu().numpy()
+    # exact against the oracle's select on the same fp32 scores
+    oi, oc = oracle.select_keep(got, wl.seq_lens, wl.budgets)
+    assert np.array_equal(gc, oc) and np.array_equal(gi[0, :oc[0]], oi[0, :oc[0]])
+    # keep-set rule against the oracle's own scores
+    wi, wc = oracle.select_keep(want.astype(np.float32), wl.seq_lens, wl.budgets)
+    ok, det = keep_set_ok(gi, gc, wi, wc, want, wl.seq_lens, wl.budgets)
+    assert ok, det
+    # compaction: bit-exact against the oracle given the index list
+    before = {k: (list(v) if isinstance(v, list) else v) for k, v in c_np.items()}
+    cws = cc.alloc_workspace(cc.cc_compact_workspace_size(wl.shape, cache))
+    cc.cc_compact_kv(wl.shape, cache, keep_idx, keep_count, cws)
+    assert cc.cc_get_status() == cc.CC_OK
+    for name in ("tokens", "pos"):
+        np.testing.assert_array_equal(cache.d[name].cpu().numpy(),
+                                      oracle.compact(before[name], gi, gc))
+    for name in ("k", "v"):
+        for l in range(wl.shape.n_layers):
+            np.testing.assert_array_equal(cache.d[name][l].float().cpu().numpy(),
+                                          oracle.compact(before[name][l], gi, gc))
+    np.testing.assert_array_equal(cache.d["h_last"].float().cpu().numpy(),
+                                  oracle.compact(before["h_last"], gi, gc))
+    assert cache.d["seq_len"].cpu().tolist() == gc.tolist()
+
+
+@pytest.mark.parametrize("seq,budget,n_sink", [([512], [128], 0), ([512, 300, 1, 7], [64, 300, 1, 3], 2),
+                                               ([4096, 5000], [1000, 17], 0)])
+def test_select_exact_vs_oracle_on_same_scores(pkg, seq, budget, n_sink):
+    from paper_2607_27600_gb300 import cc
+    cap = max(seq)
+    r = np.random.default_rng(len(seq))
+    s = r.integers(-20, 20, size=(len(seq), cap)).astype(np.float32) * 0.25   # many ties
+    s[0, 3] = np.nan
+    s[0, 10] = np.inf
+    s[-1, 0] = -np.inf
+    idx = torch.full((len(seq), cap), -1, dtype=torch.int32, device="cuda")
+    cnt = torch.zeros(len(seq), dtype=torch.int32, device="cuda")
+    cc.cc_select_keep(torch.from_numpy(s).cuda(), torch.tensor(seq, dtype=torch.int32).cuda(),
+                      len(seq), cap, torch.tensor(budget, dtype=torch.int32).cuda(), n_sink, idx,
+                      cnt)
+    assert cc.cc_get_status() == cc.CC_OK
+    oi, oc = oracle.select_keep(s, seq, budget, n_sink)
+    gi, gc = idx.cpu().numpy(), cnt.cpu().numpy()
+    assert np.array_equal(gc, oc)
+    for b in range(len(seq)):
+        assert np.array_equal(gi[b, :oc[b]], oi[b, :oc[b]]), b
+
+
+def test_select_budget_below_forced_keeps_is_reported(pkg):
+    from paper_2607_27600_gb300 import cc
+    s = torch.zeros(1, 16, device="cuda")
+    idx = torch.zeros(1, 16, dtype=torch.int32, device="cuda")
+    cnt = torch.zeros(1, dtype=torch.int32, device="cuda")
+    cc.cc_select_keep(s, torch.tensor([16], dtype=torch.int32, device="cuda"), 1, 16,
+                      torch.tensor([2], dtype=torch.int32, device="cuda"), 4, idx, cnt)
+    assert cc.cc_get_status() == cc.CC_ERR_BUDGET
+    assert cnt.item() == 5
+    assert cc.cc_get_status() == cc.CC_OK   # cleared
+
+
+@pytest.mark.parametrize("kind", ["shift1", "random", "last", "all", "sparse_tail", "dense_gaps"])
+def test_compaction_adversarial_lists_bit_exact(pkg, kind):
+    from paper_2607_27600_gb300 import cc
+    shape = SMALL_GPU
+    seq, cap = [2000, 1500], 2048
+    c = synth.synthetic_cache(shape, seq, cap, seed=3, device="cuda")
+    before = {"k": [x.float().cpu().numpy() for x in c["k"]],
+              "v": [x.float().cpu().numpy() for x in c["v"]],
+              "h": c["h_last"].float().cpu().numpy(), "tokens": c["tokens"].cpu().numpy(),
+              "pos": c["pos"].cpu().numpy()}
+    r = np.random.default_rng(7)
+    idx = np.full((2, cap), -1, np.int32)
+    cnt = np.zeros(2, np.int32)
+    for b, n in enumerate(seq):
+        if kind == "shift1":
+            k = np.arange(1, n)
+        elif kind == "random":
+            k = np.sort(r.choice(n, size=n // 4, replace=False))
+        elif kind == "last":
+            k = np.array([n - 1])
+        elif kind == "all":
+            k = np.arange(n)
+        elif kind == "sparse_tail":
+            k = np.arange(n - 100, n)
+        else:
+            k = np.sort(r.choice(n, size=n - 37, replace=False))
+        idx[b, :len(k)] = k
+        cnt[b] = len(k)
+    cache = pkg.Cache(c)
+    ws = cc.alloc_workspace(cc.cc_compact_workspace_size(shape, cache))
+    cc.cc_compact_kv(shape, cache, torch.from_numpy(idx).cuda(), torch.from_numpy(cnt).cuda(), ws)
+    assert cc.cc_get_status() == cc.CC_OK
+    for l in range(shape.n_layers):
+        np.testing.assert_array_equal(c["k"][l].float().cpu().numpy(),
+                                      oracle.compact(before["k"][l], idx, cnt))
+        np.testing.assert_array_equal(c["v"][l].float().cpu().numpy(),
+                                      oracle.compact(before["v"][l], idx, cnt))
+    np.testing.assert_array_equal(c["h_last"].float().cpu().numpy(),
+                                  oracle.compact(before["h"], idx, cnt))
+    np.testing.assert_array_equal(c["tokens"].cpu().numpy(), oracle.compact(before["tokens"], idx, cnt))
+    np.testing.assert_array_equal(c["pos"].cpu().numpy(), oracle.compact(before["pos"], idx, cnt))
+    assert c["seq_len"].cpu().tolist() == cnt.tolist()
