@@ -1,0 +1,47 @@
+/*
+ * cc_profile.h -- optional launch timing of the counter-causal refresh
+ * library.  When enabled, every kernel the library launches is bracketed by
+ * two CUDA events recorded on the launch's own stream; cc_timing_collect
+ * waits for the recorded events and returns, per kernel kind, the number of
+ * launches and their summed duration.  Used by benchmarks to attribute a
+ * refresh's time to its kernels; off by default.  Not thread-safe against
+ * concurrent library calls from several host threads while enabled.
+ */
+#ifndef CC_PROFILE_H_
+#define CC_PROFILE_H_
+
+#include "cc.h"
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  CC_KERNEL_RMSNORM = 0,     /* RMSNorm rows -> bf16                              */
+  CC_KERNEL_EMBED = 1,       /* embedding gather (full pass)                      */
+  CC_KERNEL_GEMM_QROPE = 2,  /* query projection + RoPE                           */
+  CC_KERNEL_ATTENTION = 3,   /* counter-causal attention                          */
+  CC_KERNEL_GEMM_OPROJ = 4,  /* output projection + residual                      */
+  CC_KERNEL_GEMM_GATEUP = 5, /* gate/up projection + SwiGLU                       */
+  CC_KERNEL_GEMM_DOWN = 6,   /* down projection + residual                        */
+  CC_KERNEL_HEAD_LOGIT = 7,  /* final norm + target-logit gather-dot              */
+  CC_KERNEL_GEMM_LMHEAD = 8, /* LM-head GEMM + log-sum-exp partials (log-prob)    */
+  CC_KERNEL_LSE_COMBINE = 9, /* log-sum-exp combine (log-prob)                    */
+  CC_KERNEL_SELECT = 10,     /* keep-set radix select                             */
+  CC_KERNEL_COMPACT = 11,    /* in-place compaction                               */
+  CC_KERNEL_OTHER = 12,      /* kernel-level entry points (cc_kernels.h)          */
+  CC_KERNEL_COUNT = 13
+} cc_kernel_kind;
+
+/* on != 0: start recording (also clears earlier records); 0: stop. */
+cc_status cc_timing_enable(int32_t on);
+/* Synchronises the recorded events; writes counts[k] launches and
+ * total_ms[k] summed milliseconds for k < CC_KERNEL_COUNT (host arrays),
+ * then clears the records. */
+cc_status cc_timing_collect(int32_t *counts, double *total_ms);
+const char *cc_kernel_name(int32_t kind);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* CC_PROFILE_H_ */

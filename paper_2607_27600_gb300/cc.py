@@ -85,7 +85,12 @@ _SIGS = {
                                      ctypes.c_void_p]),
     "cc_counter_causal_attention": (ctypes.c_int, [ctypes.c_void_p] * 5 + [ctypes.c_int32] * 5
                                     + [ctypes.c_void_p]),
+    "cc_timing_enable": (ctypes.c_int, [ctypes.c_int32]),
+    "cc_timing_collect": (ctypes.c_int, [ctypes.POINTER(ctypes.c_int32),
+                                         ctypes.POINTER(ctypes.c_double)]),
+    "cc_kernel_name": (ctypes.c_char_p, [ctypes.c_int32]),
 }
+KERNEL_COUNT = 13
 
 
 def library_path() -> str:
@@ -257,6 +262,20 @@ def cc_counter_causal_attention(q, k, v, seq_len, out, batch, cap, n_q_heads, n_
         _dev_ptr(q, "q"), _dev_ptr(k, "k"), _dev_ptr(v, "v"), _dev_ptr(seq_len, "seq_len"),
         _dev_ptr(out, "out"), batch, cap, n_q_heads, n_kv_heads, head_dim, _stream(stream))
     _check(code, "cc_counter_causal_attention")
+
+
+def cc_timing_enable(on: bool):
+    _check(load_library().cc_timing_enable(1 if on else 0), "cc_timing_enable")
+
+
+def cc_timing_collect() -> dict:
+    """{kernel name: (launches, total ms)} of the launches recorded since enabling."""
+    counts = (ctypes.c_int32 * KERNEL_COUNT)()
+    total = (ctypes.c_double * KERNEL_COUNT)()
+    lib = load_library()
+    _check(lib.cc_timing_collect(counts, total), "cc_timing_collect")
+    return {lib.cc_kernel_name(k).decode(): (int(counts[k]), float(total[k]))
+            for k in range(KERNEL_COUNT) if counts[k]}
 
 
 def alloc_workspace(nbytes: int, device="cuda") -> torch.Tensor:

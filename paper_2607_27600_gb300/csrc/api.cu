@@ -21,6 +21,8 @@
 #include "rowops.cuh"
 #include "select.cuh"
 #include "../../include/cc_kernels.h"
+#include "../../include/cc_profile.h"
+#include <vector>
 
 namespace cc {
 __device__ unsigned g_status_word;   // first device-side error since the last cc_get_status
@@ -59,6 +61,40 @@ bool dev_state(DevState **out) {
   *out = &d;
   return true;
 }
+
+// ---------------------------------------------------------------------------
+// optional launch timing (cc_profile.h)
+// ---------------------------------------------------------------------------
+struct TimingState {
+  bool on = false;
+  struct Rec { int kind; cudaEvent_t a, b; };
+  std::vector<Rec> recs;
+  std::vector<cudaEvent_t> pool;
+  cudaEvent_t get() {
+    if (!pool.empty()) { cudaEvent_t e = pool.back(); pool.pop_back(); return e; }
+    cudaEvent_t e = nullptr;
+    if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+    return e;
+  }
+};
+TimingState g_timing;
+
+// Brackets the launches issued in its scope with events on `st` when timing is on.
+struct TimedScope {
+  int kind;
+  cudaStream_t st;
+  cudaEvent_t a = nullptr;
+  TimedScope(int k, cudaStream_t s) : kind(k), st(s) {
+    if (g_timing.on && (a = g_timing.get())) cudaEventRecord(a, st);
+  }
+  ~TimedScope() {
+    if (!a) return;
+    cudaEvent_t b = g_timing.get();
+    if (!b) { g_timing.pool.push_back(a); return; }
+    cudaEventRecord(b, st);
+    g_timing.recs.push_back({kind, a, b});
+  }
+};
 
 // ---------------------------------------------------------------------------
 // TMA tensor maps (driver entry point fetched through the runtime)
@@ -196,7 +232,8 @@ cc_status gemm_setup(Gemm &g, int epi, const void *A, int K, const void *W, cons
   return CC_OK;
 }
 
-cc_status run_gemm(Gemm &g, int epi, int sms, cudaStream_t st) {
+cc_status run_gemm(Gemm &g, int epi, int kind, int sms, cudaStream_t st) {
+  TimedScope t(kind, st);
   CC_TRY(launch_gemm(epi, g.a, g.b, g.b2, g.p, sms, st));
   return CC_OK;
 }
@@ -233,6 +270,7 @@ cc_status run_attention(const cc_model_cfg *c, const void *q, const void *k, con
   p.out = reinterpret_cast<__nv_bfloat16 *>(out);
   p.scale_log2 = (float)(1.4426950408889634 / sqrt((double)dh));
   p.status = status;
+  TimedScope t(CC_KERNEL_ATTENTION, st);
   CC_TRY(launch_attention(tq, tk, tv, p, st));
   return CC_OK;
 }
@@ -283,14 +321,20 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
   const int32_t *sl = kv->seq_len;
   unsigned *status = dev->status;
 
-  if (full) CC_TRY(launch_embed(w->embed, kv->tokens, h, d, c->vocab, sl, cap, rows, status, st));
+  if (full) {
+    TimedScope t(CC_KERNEL_EMBED, st);
+    CC_TRY(launch_embed(w->embed, kv->tokens, h, d, c->vocab, sl, cap, rows, status, st));
+  }
   const int l0 = full ? 0 : c->n_layers - 1;
   for (int l = l0; l < c->n_layers; ++l) {
     const cc_layer_weights &lw = w->layers[l];
     const bool first_from_bf16 = !full;   // fast mode: the layer input is H^(L-1) (bf16)
     // xn = RMSNorm(h)
-    CC_TRY(launch_rmsnorm(first_from_bf16 ? kv->h_last : (const void *)h, !first_from_bf16,
-                          lw.attn_norm, xn, d, c->rms_eps, sl, cap, rows, st));
+    {
+      TimedScope t(CC_KERNEL_RMSNORM, st);
+      CC_TRY(launch_rmsnorm(first_from_bf16 ? kv->h_last : (const void *)h, !first_from_bf16,
+                            lw.attn_norm, xn, d, c->rms_eps, sl, cap, rows, st));
+    }
     // Q = RoPE(xn Wq^T)
     Gemm gq;
     if ((s = gemm_setup(gq, EPI_QROPE, xn, d, lw.wq, nullptr, qd, batch, cap, sl, status)) != CC_OK)
@@ -300,7 +344,7 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
     gq.p.pos = kv->pos;
     gq.p.head_dim = c->head_dim;
     rope_turns(c, gq.p.turns);
-    if ((s = run_gemm(gq, EPI_QROPE, dev->sms, st)) != CC_OK) return s;
+    if ((s = run_gemm(gq, EPI_QROPE, CC_KERNEL_GEMM_QROPE, dev->sms, st)) != CC_OK) return s;
     // O = counter-causal attention
     if ((s = run_attention(c, q, kv->k[l], kv->v[l], o, sl, batch, cap, status, st)) != CC_OK)
       return s;
@@ -313,16 +357,19 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
     go.p.ldo = d;
     go.p.resid = kv->h_last;
     go.p.ld_resid = d;
-    if ((s = run_gemm(go, epi_o, dev->sms, st)) != CC_OK) return s;
+    if ((s = run_gemm(go, epi_o, CC_KERNEL_GEMM_OPROJ, dev->sms, st)) != CC_OK) return s;
     // xn = RMSNorm(h); act = silu(xn Wg^T) * (xn Wu^T)
-    CC_TRY(launch_rmsnorm(h, true, lw.mlp_norm, xn, d, c->rms_eps, sl, cap, rows, st));
+    {
+      TimedScope t(CC_KERNEL_RMSNORM, st);
+      CC_TRY(launch_rmsnorm(h, true, lw.mlp_norm, xn, d, c->rms_eps, sl, cap, rows, st));
+    }
     Gemm gu;
     if ((s = gemm_setup(gu, EPI_SWIGLU, xn, d, lw.w_gate, lw.w_up, f, batch, cap, sl, status)) !=
         CC_OK)
       return s;
     gu.p.out = act;
     gu.p.ldo = f;
-    if ((s = run_gemm(gu, EPI_SWIGLU, dev->sms, st)) != CC_OK) return s;
+    if ((s = run_gemm(gu, EPI_SWIGLU, CC_KERNEL_GEMM_GATEUP, dev->sms, st)) != CC_OK) return s;
     // h = h + act Wd^T
     Gemm gd;
     if ((s = gemm_setup(gd, EPI_RESID_F32, act, f, lw.w_down, nullptr, d, batch, cap, sl,
@@ -330,14 +377,18 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
       return s;
     gd.p.out = h;
     gd.p.ldo = d;
-    if ((s = run_gemm(gd, EPI_RESID_F32, dev->sms, st)) != CC_OK) return s;
+    if ((s = run_gemm(gd, EPI_RESID_F32, CC_KERNEL_GEMM_DOWN, dev->sms, st)) != CC_OK) return s;
   }
   // head
   if (mode == CC_SCORE_LOGIT) {
+    TimedScope t(CC_KERNEL_HEAD_LOGIT, st);
     CC_TRY(launch_head_logit(h, w->final_norm, w->lm_head, kv->tokens, scores, d, c->vocab,
                              c->rms_eps, sl, cap, rows, status, st));
   } else {
-    CC_TRY(launch_rmsnorm(h, true, w->final_norm, xn, d, c->rms_eps, sl, cap, rows, st));
+    {
+      TimedScope t(CC_KERNEL_RMSNORM, st);
+      CC_TRY(launch_rmsnorm(h, true, w->final_norm, xn, d, c->rms_eps, sl, cap, rows, st));
+    }
     Gemm gl;
     if ((s = gemm_setup(gl, EPI_LSE, xn, d, w->lm_head, nullptr, c->vocab, batch, cap, sl,
                         status)) != CC_OK)
@@ -348,7 +399,8 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
     gl.p.ldo = L.n_vtiles;
     gl.p.tokens = kv->tokens;
     gl.p.z_target = zt;
-    if ((s = run_gemm(gl, EPI_LSE, dev->sms, st)) != CC_OK) return s;
+    if ((s = run_gemm(gl, EPI_LSE, CC_KERNEL_GEMM_LMHEAD, dev->sms, st)) != CC_OK) return s;
+    TimedScope t(CC_KERNEL_LSE_COMBINE, st);
     CC_TRY(launch_lse_combine(part, L.n_vtiles, zt, scores, sl, cap, rows, st));
   }
   return CC_OK;
@@ -438,6 +490,7 @@ cc_status cc_select_keep(const float *scores, const int32_t *seq_len, int32_t ba
     return CC_ERR_INVALID_ARG;
   DevState *dev;
   if (!dev_state(&dev)) return CC_ERR_CUDA;
+  TimedScope t(CC_KERNEL_SELECT, reinterpret_cast<cudaStream_t>(stream));
   CC_TRY(launch_select(scores, seq_len, batch, cap, budget, n_sink, keep_idx, keep_count,
                        dev->status, reinterpret_cast<cudaStream_t>(stream)));
   return CC_OK;
@@ -469,6 +522,7 @@ cc_status cc_compact_kv(const cc_model_cfg *cfg, const cc_kv_cache *cache,
   plan.p.ticket = reinterpret_cast<unsigned *>(ws);
   plan.p.flags = reinterpret_cast<unsigned *>(reinterpret_cast<uint8_t *>(ws) + 256);
   plan.p.status = dev->status;
+  TimedScope t(CC_KERNEL_COMPACT, st);
   CC_TRY(launch_compact(plan.p, dev->sms * 3, st));
   return CC_OK;
 }
@@ -514,7 +568,7 @@ cc_status cc_linear_f32(const void *x, const void *w, float *y, int32_t rows, in
   if (s != CC_OK) return s;
   g.p.out = y;
   g.p.ldo = n;
-  return run_gemm(g, EPI_F32, dev->sms, reinterpret_cast<cudaStream_t>(stream));
+  return run_gemm(g, EPI_F32, CC_KERNEL_OTHER, dev->sms, reinterpret_cast<cudaStream_t>(stream));
 }
 
 cc_status cc_counter_causal_attention(const void *q, const void *k, const void *v,
@@ -536,6 +590,49 @@ cc_status cc_counter_causal_attention(const void *q, const void *k, const void *
   c.head_dim = head_dim;
   return run_attention(&c, q, k, v, out, seq_len, batch, cap, dev->status,
                        reinterpret_cast<cudaStream_t>(stream));
+}
+
+// ---- launch timing (include/cc_profile.h) ----------------------------------
+
+cc_status cc_timing_enable(int32_t on) {
+  std::lock_guard<std::mutex> lk(g_mu);
+  for (auto &r : g_timing.recs) {
+    g_timing.pool.push_back(r.a);
+    g_timing.pool.push_back(r.b);
+  }
+  g_timing.recs.clear();
+  g_timing.on = on != 0;
+  return CC_OK;
+}
+
+cc_status cc_timing_collect(int32_t *counts, double *total_ms) {
+  if (!counts || !total_ms) return CC_ERR_INVALID_ARG;
+  std::lock_guard<std::mutex> lk(g_mu);
+  for (int k = 0; k < CC_KERNEL_COUNT; ++k) {
+    counts[k] = 0;
+    total_ms[k] = 0.0;
+  }
+  cc_status st = CC_OK;
+  for (auto &r : g_timing.recs) {
+    float ms = 0.f;
+    if (cudaEventSynchronize(r.b) != cudaSuccess || cudaEventElapsedTime(&ms, r.a, r.b) != cudaSuccess)
+      st = CC_ERR_CUDA;
+    if (r.kind >= 0 && r.kind < CC_KERNEL_COUNT) {
+      counts[r.kind] += 1;
+      total_ms[r.kind] += ms;
+    }
+    g_timing.pool.push_back(r.a);
+    g_timing.pool.push_back(r.b);
+  }
+  g_timing.recs.clear();
+  return st;
+}
+
+const char *cc_kernel_name(int32_t kind) {
+  static const char *names[CC_KERNEL_COUNT] = {
+      "rmsnorm", "embed", "gemm_qrope", "attention", "gemm_oproj", "gemm_gateup", "gemm_down",
+      "head_logit", "gemm_lmhead", "lse_combine", "select", "compact", "other"};
+  return (kind >= 0 && kind < CC_KERNEL_COUNT) ? names[kind] : "unknown";
 }
 
 }  // extern "C"

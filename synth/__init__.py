@@ -60,7 +60,7 @@ def tokens(shape, vocab: int, seed: int, name: str = "tokens", device="cpu") -> 
 
 
 def model_weights(shape: ModelShape, seed: int, device="cpu", with_kv_proj: bool = False,
-                  layers=None) -> dict:
+                  layers=None, with_embed: bool = True) -> dict:
     """Random-init weights in nn.Linear layout: a [out, in] matrix per projection.
 
     `layers` restricts which layers are drawn (others are None); the fast
@@ -70,7 +70,7 @@ def model_weights(shape: ModelShape, seed: int, device="cpu", with_kv_proj: bool
     d, q, kv, f, v = shape.d_model, shape.q_dim, shape.kv_dim, shape.d_ff, shape.vocab
     ones = torch.ones(d, dtype=torch.bfloat16, device=device)
     want = range(shape.n_layers) if layers is None else layers
-    out = {"embed": normal((v, d), WEIGHT_STD, seed, "embed", device),
+    out = {"embed": normal((v, d), WEIGHT_STD, seed, "embed", device) if with_embed else None,
            "final_norm": ones.clone(),
            "lm_head": normal((v, d), WEIGHT_STD, seed, "lm_head", device),
            "layers": [None] * shape.n_layers}
