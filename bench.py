@@ -1,0 +1,597 @@
+"""Benchmark of one counter-causal memory refresh (arXiv 2607.27600,
+Sec. 3.1 and Algorithm DoMemRefresh) on GB300.
+
+A step = one refresh of one synthetic cache: counter-causal scores of every
+cached position (fast single-layer approximation, or the full L-layer pass),
+keep-set selection at the budget, in-place compaction of every layer's K/V,
+H^(L-1), tokens and positions.  Metric: scored KV positions per second.
+
+    python bench.py [--gpus N --steps K --warmup W] [--workload NAME] [--impl reference]
+
+Our arm times K steps with CUDA events on the launching stream (inputs
+resident in HBM; the cache is restored and 256 MiB written to flush L2
+between steps, outside the timed events), then K end-to-end steps through
+the public API with host inputs (pinned host -> device copies of the step's
+inputs and device -> host read of the keep-set inside the timed region).
+The reference arm (--impl reference) times the CPU oracle on a bounded row
+sample of the same workload.  Under torchrun each rank runs an independent
+replica (no collective on the data path) and rank 0 prints one JSON line.
+"""
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import synth  # noqa: E402
+
+PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+L2_FLUSH_BYTES = 256 << 20
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return d, "measured"
+    return PEAKS_FALLBACK, "fallback"
+
+
+# ---------------------------------------------------------------------------
+# distributed plumbing (one process per GPU, independent replicas)
+# ---------------------------------------------------------------------------
+
+class Dist:
+    def __init__(self):
+        self.world = int(os.environ.get("WORLD_SIZE", "1"))
+        self.rank = int(os.environ.get("RANK", "0"))
+        self.local = int(os.environ.get("LOCAL_RANK", "0"))
+        self.pg = None
+        if self.world > 1:
+            import torch.distributed as dist
+            backend = "nccl" if torch.cuda.is_available() else "gloo"
+            if backend == "nccl":
+                torch.cuda.set_device(self.local)
+            dist.init_process_group(backend)
+            self.pg = dist
+
+    def barrier(self):
+        if self.pg:
+            if torch.cuda.is_available():
+                self.pg.barrier(device_ids=[self.local])
+            else:
+                self.pg.barrier()
+
+    def max(self, x: float) -> float:
+        if not self.pg:
+            return x
+        dev = f"cuda:{self.local}" if torch.cuda.is_available() else "cpu"
+        t = torch.tensor([x], dtype=torch.float64, device=dev)
+        self.pg.all_reduce(t, op=self.pg.ReduceOp.MAX)
+        return float(t.item())
+
+    def close(self):
+        if self.pg:
+            self.pg.destroy_process_group()
+
+
+# ---------------------------------------------------------------------------
+# clocks during the timed region
+# ---------------------------------------------------------------------------
+
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index: int):
+        self.samples = []
+        self.proc = None
+        try:
+            bus = torch.cuda.get_device_properties(device_index).pci_bus_id
+        except Exception:
+            bus = str(device_index)
+        self.cmd = ["nvidia-smi", "-i", str(bus), f"--query-gpu={self.FIELDS}",
+                    "--format=csv,noheader,nounits", "-lms", "100"]
+        self.thread = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(self.cmd, stdout=subprocess.PIPE,
+                                         stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) >= 8:
+                self.samples.append(parts)
+
+    def stop(self) -> dict:
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        if self.thread:
+            self.thread.join(timeout=5)
+
+        def num(x):
+            try:
+                return float(x)
+            except ValueError:
+                return None
+        sm = [num(s[0]) for s in self.samples if num(s[0]) is not None]
+        mx = [num(s[1]) for s in self.samples if num(s[1]) is not None]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for s in self.samples for i in range(4)
+                          if s[4 + i].lower() == "active"})
+        loaded = [v for v in sm if mx and v > 0.5 * max(mx)] or sm
+        return {"sm_mhz": statistics.median(loaded) if loaded else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons,
+                "samples": len(self.samples)}
+
+
+# ---------------------------------------------------------------------------
+# workload setup
+# ---------------------------------------------------------------------------
+
+def make_inputs(wl, device):
+    """Weights and cache of the workload on `device` (seeded synthetic)."""
+    shape = wl.shape
+    fast = wl.mode == "layer"
+    layers = [shape.n_layers - 1] if fast else None
+    w = synth.model_weights(shape, wl.seed, device=device, layers=layers, with_embed=not fast)
+    # the refresh compacts every layer's cache; the fast pass reads only the last layer's
+    cache = synth.synthetic_cache(shape, wl.seq_lens, wl.cap, wl.seed, device=device,
+                                  with_h_last=fast)
+    return w, cache
+
+
+def clone_cache(c):
+    return {k: ([x.clone() if x is not None else None for x in v] if isinstance(v, list)
+                else (v.clone() if v is not None else None)) for k, v in c.items()}
+
+
+def restore_cache(dst, src):
+    for k, v in src.items():
+        if isinstance(v, list):
+            for a, b in zip(dst[k], v):
+                if a is not None:
+                    a.copy_(b, non_blocking=True)
+        elif v is not None:
+            dst[k].copy_(v, non_blocking=True)
+
+
+def algorithmic_work(wl):
+    """Per-launch algorithmic FLOPs / bytes of each kernel kind for one step."""
+    s = wl.shape
+    n_rows = sum(wl.seq_lens)
+    d, qd, f, hq, dh = s.d_model, s.q_dim, s.d_ff, s.n_q_heads, s.head_dim
+    pairs = sum(n * (n - 1) for n in wl.seq_lens)          # 2 x (pairs j > i)
+    kv_row = s.kv_dim * 2
+    moved = sum(max(0, min(b, n)) for b, n in zip(wl.budgets, wl.seq_lens))
+    n_arrays_kv = 2 * s.n_layers
+    h_row = d * 2 if wl.mode == "layer" else 0
+    return {
+        "gemm_qrope": ("tensor", 2.0 * n_rows * d * qd),
+        "attention": ("tensor", 2.0 * dh * hq * pairs),
+        "gemm_oproj": ("tensor", 2.0 * n_rows * qd * d),
+        "gemm_gateup": ("tensor", 4.0 * n_rows * d * f),
+        "gemm_down": ("tensor", 2.0 * n_rows * f * d),
+        # final norm + gather-dot: h (fp32) read twice, W_U row read once, score written
+        "head_logit": ("hbm", n_rows * (8.0 * d + 2.0 * d + 4.0)),
+        "gemm_lmhead": ("tensor", 2.0 * n_rows * d * s.vocab),
+        "rmsnorm": ("hbm", n_rows * (4.0 * d * 2 + 2.0 * d)),
+        # each kept slot: read + write of every layer's K and V row, H row, token, position
+        "compact": ("hbm", 2.0 * moved * (n_arrays_kv * kv_row + h_row + 8)),
+        # 9 passes over the scores (8 radix passes + the emit pass)
+        "select": ("hbm", 9.0 * 4.0 * n_rows),
+    }
+
+
+def step_flops(wl):
+    s = wl.shape
+    w = algorithmic_work(wl)
+    lay = 1 if wl.mode == "layer" else s.n_layers
+    per_layer = sum(w[k][1] for k in ("gemm_qrope", "attention", "gemm_oproj", "gemm_gateup",
+                                      "gemm_down"))
+    return lay * per_layer + 2.0 * sum(wl.seq_lens) * s.d_model
+
+
+# ---------------------------------------------------------------------------
+# our arm
+# ---------------------------------------------------------------------------
+
+def run_ours(args, dist):
+    import paper_2607_27600_gb300 as pkg
+    from paper_2607_27600_gb300 import cc
+    pkg.load_library()
+    dev = torch.device(f"cuda:{dist.local}")
+    torch.cuda.set_device(dev)
+    wl = synth.WORKLOADS[args.workload]
+    shape = wl.shape
+    mode = cc.SCORE_LOGPROB if args.score == "logprob" else cc.SCORE_LOGIT
+    fast = wl.mode == "layer"
+    if wl.cycles > 1 and not args.single_cycle:
+        raise SystemExit("multi-cycle workloads: use --single-cycle (the first refresh is timed)")
+
+    w, pristine = make_inputs(wl, dev)
+    work = clone_cache(pristine)
+    weights, cache = pkg.Weights(w), pkg.Cache(work)
+    b, cap = wl.batch, wl.cap
+    scores = torch.empty(b, cap, dtype=torch.float32, device=dev)
+    keep_idx = torch.empty(b, cap, dtype=torch.int32, device=dev)
+    keep_count = torch.empty(b, dtype=torch.int32, device=dev)
+    budget = torch.tensor(wl.budgets, dtype=torch.int32, device=dev)
+    ws = cc.alloc_workspace(cc.cc_score_workspace_size(shape, b, cap, mode), dev)
+    cws = cc.alloc_workspace(cc.cc_compact_workspace_size(shape, cache), dev)
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    score_fn = cc.cc_score_layer if fast else cc.cc_score_full
+    stream = torch.cuda.current_stream(dev)
+
+    def step():
+        score_fn(shape, weights, cache, mode, scores, ws)
+        cc.cc_select_keep(scores, cache.d["seq_len"], b, cap, budget, wl.n_sink, keep_idx,
+                          keep_count)
+        cc.cc_compact_kv(shape, cache, keep_idx, keep_count, cws)
+
+    def prepare():
+        restore_cache(work, pristine)
+        flush.fill_(1)
+
+    for _ in range(args.warmup):
+        prepare()
+        step()
+    torch.cuda.synchronize(dev)
+    status = cc.cc_get_status()
+    if status != cc.CC_OK:
+        raise SystemExit(f"device status after warm-up: {cc.cc_status_str(status)}")
+
+    clocks = ClockSampler(dist.local)
+    clocks.start()
+    time.sleep(0.3)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    dist.barrier()
+    torch.cuda.synchronize(dev)
+    cc.cc_timing_enable(True)
+    for i in range(args.steps):
+        prepare()
+        ev[i][0].record(stream)
+        step()
+        ev[i][1].record(stream)
+    torch.cuda.synchronize(dev)
+    kernels = cc.cc_timing_collect()
+    cc.cc_timing_enable(False)
+    dist.barrier()
+    step_ms = [a.elapsed_time(bb) for a, bb in ev]
+    ms_local = sum(step_ms) / args.steps
+    ms = dist.max(ms_local)
+    status = cc.cc_get_status()
+    if status != cc.CC_OK:
+        raise SystemExit(f"device status after timing: {cc.cc_status_str(status)}")
+
+    # ---- end to end through the public API with host inputs
+    host = {"h_last": pristine["h_last"].cpu().pin_memory() if fast else None,
+            "k": pristine["k"][-1].cpu().pin_memory(), "v": pristine["v"][-1].cpu().pin_memory(),
+            "tokens": pristine["tokens"].cpu().pin_memory(),
+            "pos": pristine["pos"].cpu().pin_memory(),
+            "seq_len": pristine["seq_len"].cpu().pin_memory()}
+    if not fast:   # the full pass reads every layer's K/V
+        host["k_all"] = [x.cpu().pin_memory() for x in pristine["k"]]
+        host["v_all"] = [x.cpu().pin_memory() for x in pristine["v"]]
+    out_idx = torch.empty(b, cap, dtype=torch.int32).pin_memory()
+    out_cnt = torch.empty(b, dtype=torch.int32).pin_memory()
+    h2d = sum(t.numel() * t.element_size() for k, t in host.items()
+              if isinstance(t, torch.Tensor))
+    if not fast:
+        h2d += sum(t.numel() * t.element_size() for t in host["k_all"] + host["v_all"])
+        h2d -= host["k"].numel() * host["k"].element_size() * 2
+    d2h = out_idx.numel() * 4 + out_cnt.numel() * 4
+
+    def e2e_step():
+        if fast:
+            work["h_last"].copy_(host["h_last"], non_blocking=True)
+            work["k"][-1].copy_(host["k"], non_blocking=True)
+            work["v"][-1].copy_(host["v"], non_blocking=True)
+        else:
+            for dst, src in zip(work["k"], host["k_all"]):
+                dst.copy_(src, non_blocking=True)
+            for dst, src in zip(work["v"], host["v_all"]):
+                dst.copy_(src, non_blocking=True)
+        work["tokens"].copy_(host["tokens"], non_blocking=True)
+        work["pos"].copy_(host["pos"], non_blocking=True)
+        work["seq_len"].copy_(host["seq_len"], non_blocking=True)
+        step()
+        out_idx.copy_(keep_idx, non_blocking=True)
+        out_cnt.copy_(keep_count, non_blocking=True)
+
+    e2e_ms = []
+    for i in range(args.steps):
+        restore_cache(work, pristine)   # the rest of the device-resident cache
+        flush.fill_(1)
+        torch.cuda.synchronize(dev)
+        t0 = torch.cuda.Event(enable_timing=True)
+        t1 = torch.cuda.Event(enable_timing=True)
+        t0.record(stream)
+        e2e_step()
+        t1.record(stream)
+        torch.cuda.synchronize(dev)
+        e2e_ms.append(t0.elapsed_time(t1))
+    clk = clocks.stop()
+    e2e_ms_max = dist.max(sum(e2e_ms) / len(e2e_ms))
+    status = cc.cc_get_status()
+    if status != cc.CC_OK:
+        raise SystemExit(f"device status after e2e: {cc.cc_status_str(status)}")
+    # sanity: the e2e keep-set equals the device-resident one of the last timed step
+    positions = sum(wl.seq_lens)
+
+    # ---- roofline of the dominant kernel (and a per-kernel table)
+    peaks, peak_src = load_peaks()
+    work_tbl = algorithmic_work(wl)
+    table = {}
+    for name, (cnt, tot) in kernels.items():
+        per = tot / cnt
+        entry = {"launches_per_step": cnt / args.steps, "ms_per_launch": round(per, 4),
+                 "share": round(tot / max(1e-9, sum(t for _, t in kernels.values())), 4)}
+        if name in work_tbl:
+            bound, amount = work_tbl[name]
+            if name == "rmsnorm":
+                amount = amount   # per launch, same row count every launch
+            if bound == "tensor":
+                ach = amount / (per * 1e-3) / 1e12
+                entry.update({"bound": "tensor", "achieved": round(ach, 2), "unit": "TFLOP/s",
+                              "frac": round(ach / peaks["bf16_tflops"], 4)})
+            else:
+                ach = amount / (per * 1e-3) / 1e9
+                entry.update({"bound": "hbm", "achieved": round(ach, 1), "unit": "GB/s",
+                              "frac": round(ach / peaks["hbm_gbs"], 4)})
+        table[name] = entry
+    dom = max(kernels.items(), key=lambda kv: kv[1][1])[0]
+    traffic = read_traffic(dom, wl.name)
+    d = table[dom]
+    roof = {"kernel": dom, "bound": d.get("bound"), "achieved": d.get("achieved"),
+            "peak": peaks["bf16_tflops"] if d.get("bound") == "tensor" else peaks["hbm_gbs"],
+            "unit": d.get("unit"), "frac": d.get("frac"), "traffic": traffic,
+            "peak_source": f"{peak_src} ({'bf16 dense burst' if d.get('bound') == 'tensor' else 'HBM copy'})"}
+
+    launches = sum(c for c, _ in kernels.values())
+    value = positions * dist.world / (ms * 1e-3)
+    line = {
+        "metric": "scored KV positions/sec per refresh",
+        "value": round(value, 1), "unit": "positions/s", "n_gpus": dist.world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 4),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded random-init weights N(0,0.02); synthetic KV cache)",
+        "config": {"workload": wl.name, "pass": "fast single-layer" if fast else f"full {shape.n_layers}-layer",
+                   "score": args.score, "batch": wl.batch, "seq_lens": wl.seq_lens,
+                   "budgets": wl.budgets, "cap": wl.cap, "d_model": shape.d_model,
+                   "heads": f"{shape.n_q_heads}/{shape.n_kv_heads}x{shape.head_dim}",
+                   "d_ff": shape.d_ff, "vocab": shape.vocab,
+                   "layers_compacted": shape.n_layers,
+                   "step_tflop": round(step_flops(wl) / 1e12, 3),
+                   "l2": "cache restored + 256 MiB written between steps (outside the timed events)",
+                   "parallelism": f"replicas x{dist.world}"},
+        "e2e": {"value": round(positions * dist.world / (e2e_ms_max * 1e-3), 1),
+                "unit": "positions/s", "h2d_bytes_per_step": int(h2d),
+                "d2h_bytes_per_step": int(d2h), "ms_per_step": round(e2e_ms_max, 4)},
+        "gpu_launches": int(launches),
+        "roofline": roof,
+        "kernels": table,
+        "tflops_per_step_achieved": round(step_flops(wl) / (ms * 1e-3) / 1e12, 1),
+        "clocks": clk,
+    }
+    if dist.world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(wl, w, pristine, scores, args.cpu_rows, args.score)
+    return line
+
+
+def read_traffic(kernel, workload):
+    """DRAM bytes per launch from a committed ncu summary, when it matches the
+    current kernel sources; else None."""
+    p = os.path.join(ROOT, "profiles", "dram_traffic.json")
+    if not os.path.exists(p):
+        return None
+    try:
+        with open(p) as f:
+            tbl = json.load(f)
+        e = tbl.get(workload, {}).get(kernel)
+        if not e or e.get("csrc_sha") != csrc_digest():
+            return None
+        return e.get("bytes_per_launch")
+    except Exception:
+        return None
+
+
+def csrc_digest():
+    import hashlib
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2607_27600_gb300", "csrc")
+    for f in sorted(os.listdir(csrc)):
+        with open(os.path.join(csrc, f), "rb") as fh:
+            h.update(f.encode() + fh.read())
+    return h.hexdigest()[:16]
+
+
+# ---------------------------------------------------------------------------
+# the oracle on the host cores (CPU baseline / reference arm)
+# ---------------------------------------------------------------------------
+
+def host_inputs(wl, w, cache):
+    """numpy copies (bf16 widened to fp32; K/V of the compacted layers kept as raw 16-bit)."""
+    def f32(t):
+        return None if t is None else t.float().cpu().numpy()
+    last = wl.shape.n_layers - 1
+    fast = wl.mode == "layer"
+    lw = [None] * wl.shape.n_layers
+    for l, x in enumerate(w["layers"]):
+        if x is not None:
+            lw[l] = {k: f32(v) for k, v in x.items()}
+    wn = {"embed": f32(w["embed"]), "final_norm": f32(w["final_norm"]),
+          "lm_head": f32(w["lm_head"]), "layers": lw}
+    kf = [f32(cache["k"][l]) if (not fast or l == last) else None for l in range(wl.shape.n_layers)]
+    vf = [f32(cache["v"][l]) if (not fast or l == last) else None for l in range(wl.shape.n_layers)]
+    cn = {"k": kf, "v": vf, "tokens": cache["tokens"].cpu().numpy(), "pos": cache["pos"].cpu().numpy(),
+          "seq_len": cache["seq_len"].cpu().numpy(), "h_last": f32(cache["h_last"])}
+    raw = {"k": [x.view(torch.int16).cpu().numpy() for x in cache["k"]],
+           "v": [x.view(torch.int16).cpu().numpy() for x in cache["v"]],
+           "h": None if cache["h_last"] is None else cache["h_last"].view(torch.int16).cpu().numpy()}
+    return wn, cn, raw
+
+
+def sample_rows(wl, count, seed=0):
+    r = np.random.default_rng(seed)
+    rows = []
+    per = max(2, count // wl.batch)
+    for n in wl.seq_lens:
+        pick = {0, n - 2, n - 1} | set(r.choice(n, size=min(n, per), replace=False).tolist())
+        rows.append(sorted(x for x in pick if 0 <= x < n)[:max(per, 3)])
+    return rows
+
+
+def _oracle_score_time(wl, wn, cn, rows, score_mode):
+    import oracle
+    fn = oracle.score_layer if wl.mode == "layer" else oracle.score_full
+    t0 = time.perf_counter()
+    fn(wl.shape, wn, cn, mode=score_mode, rows=rows)
+    return time.perf_counter() - t0, sum(len(r) for r in rows)
+
+
+def oracle_fixed_cost(wl, wn, cn, score_mode, small, large):
+    """Per-call cost of the oracle's scoring that does not grow with the rows
+    (widening the weights to fp64), from two sample sizes."""
+    t1, n1 = _oracle_score_time(wl, wn, cn, sample_rows(wl, small, seed=11), score_mode)
+    t2, n2 = _oracle_score_time(wl, wn, cn, sample_rows(wl, large, seed=12), score_mode)
+    per_row = max(0.0, (t2 - t1) / max(1, n2 - n1))
+    return max(0.0, t1 - n1 * per_row)
+
+
+def oracle_refresh_time(wl, wn, cn, raw, scores_np, rows, score_mode, fixed):
+    """Seconds the oracle takes for one refresh of the whole workload: its
+    scoring timed on the sampled rows and extrapolated linearly in the row
+    count (rows are independent given the cache; the per-call fixed cost is
+    counted once), plus its select and compaction run in full."""
+    import oracle
+    t_rows, n_sampled = _oracle_score_time(wl, wn, cn, rows, score_mode)
+    per_row = max(0.0, t_rows - fixed) / n_sampled
+    t1 = time.perf_counter()
+    idx, cnt = oracle.select_keep(scores_np, cn["seq_len"], wl.budgets, wl.n_sink)
+    t_sel = time.perf_counter() - t1
+    t2 = time.perf_counter()
+    for arrs in (raw["k"], raw["v"]):
+        for a in arrs:
+            oracle.compact(a, idx, cnt)
+    if raw["h"] is not None:
+        oracle.compact(raw["h"], idx, cnt)
+    oracle.compact(cn["tokens"], idx, cnt)
+    oracle.compact(cn["pos"], idx, cnt)
+    t_cmp = time.perf_counter() - t2
+    positions = sum(wl.seq_lens)
+    total = fixed + per_row * positions + t_sel + t_cmp
+    return total, n_sampled, t_rows, t_sel, t_cmp
+
+
+def cores_used():
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count()
+
+
+def cpu_baseline(wl, w, cache, scores_dev, n_rows, score_mode):
+    wn, cn, raw = host_inputs(wl, w, cache)
+    scores_np = scores_dev.cpu().numpy()
+    fixed = oracle_fixed_cost(wl, wn, cn, score_mode, n_rows // 4, n_rows // 2)
+    rows = sample_rows(wl, n_rows)
+    total, ns, t_rows, t_sel, t_cmp = oracle_refresh_time(wl, wn, cn, raw, scores_np, rows,
+                                                          score_mode, fixed)
+    return {"value": round(sum(wl.seq_lens) / total, 3), "unit": "positions/s",
+            "cores": cores_used(), "kind": "oracle",
+            "sample": (f"{ns} sampled rows scored ({t_rows:.1f} s incl. {fixed:.1f} s per-call "
+                       f"fixed cost), extrapolated linearly to {sum(wl.seq_lens)} rows, + full "
+                       f"select ({t_sel:.2f} s) + full compaction ({t_cmp:.2f} s); numpy fp64, "
+                       f"BLAS threads = cores")}
+
+
+def run_reference(args, dist):
+    if dist.rank != 0:
+        return None
+    wl = synth.WORKLOADS[args.workload]
+    dev = torch.device("cuda:0") if torch.cuda.is_available() else torch.device("cpu")
+    w, cache = make_inputs(wl, dev)
+    wn, cn, raw = host_inputs(wl, w, cache)
+    r = np.random.default_rng(1)
+    scores_np = r.standard_normal(size=cn["tokens"].shape).astype(np.float32)
+    for b, n in enumerate(wl.seq_lens):
+        scores_np[b, n - 1] = np.inf
+    times = []
+    ns = 0
+    fixed = oracle_fixed_cost(wl, wn, cn, args.score, max(2, args.ref_rows // 2),
+                              args.ref_rows * 3 // 2)
+    for i in range(args.warmup + args.steps):
+        rows = sample_rows(wl, args.ref_rows, seed=i)
+        total, ns, *_ = oracle_refresh_time(wl, wn, cn, raw, scores_np, rows, args.score, fixed)
+        if i >= args.warmup:
+            times.append(total)
+    ms = 1e3 * sum(times) / len(times)
+    positions = sum(wl.seq_lens)
+    value = positions / (ms * 1e-3)
+    sample = (f"per step {ns} sampled rows scored by the oracle, extrapolated linearly to "
+              f"{positions} rows (per-call fixed cost {fixed:.1f} s counted once), + full "
+              f"select and compaction")
+    return {"impl": "reference", "metric": "scored KV positions/sec per refresh",
+            "value": round(value, 3), "unit": "positions/s", "n_gpus": dist.world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 2),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": {"workload": wl.name, "score": args.score},
+            "cpu_baseline": {"value": round(value, 3), "unit": "positions/s", "cores": cores_used(),
+                             "kind": "oracle", "sample": sample},
+            "e2e": {"value": round(value, 3), "unit": "positions/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=30)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default=synth.HEADLINE, choices=sorted(synth.WORKLOADS))
+    ap.add_argument("--score", choices=["logit", "logprob"], default="logit")
+    ap.add_argument("--single-cycle", action="store_true",
+                    help="time only the first refresh of a multi-cycle workload")
+    ap.add_argument("--cpu-rows", type=int, default=256)
+    ap.add_argument("--ref-rows", type=int, default=32)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        raise SystemExit("--warmup must be >= 3")
+    dist = Dist()
+    try:
+        line = run_reference(args, dist) if args.impl == "reference" else run_ours(args, dist)
+        if dist.rank == 0 and line is not None:
+            print(json.dumps(line), flush=True)
+    finally:
+        dist.close()
+
+
+if __name__ == "__main__":
+    main()
