@@ -1,0 +1,214 @@
+"""GPU parity at the full workload sizes, in the launch configuration bench.py
+times (one cc_score_* call over the whole cache), checked on sampled rows
+against the CPU oracle (rows are independent given the cache, so a sampled
+row's score is exactly what the oracle computes for it alone).
+
+Every input comes from the seeded generators (synth) and is copied to the
+host for the oracle; no oracle input comes from the CUDA path.  Multi-cycle
+refreshes use seeded keep-sets, compacted independently on each side.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+from tests._util import keep_set_ok, rel_err
+
+pytestmark = pytest.mark.gpu
+
+TOL = 2e-2
+
+
+@pytest.fixture(scope="module")
+def pkg():
+    import paper_2607_27600_gb300 as p
+    p.load_library()
+    return p
+
+
+def f32(t):
+    return None if t is None else t.float().cpu().numpy()
+
+
+class LazyLayers(list):
+    """Layer weights converted to numpy only when the oracle reaches them."""
+
+    def __init__(self, layers):
+        super().__init__(layers)
+
+    def __getitem__(self, i):
+        lw = list.__getitem__(self, i)
+        return None if lw is None else {k: f32(v) for k, v in lw.items()}
+
+
+class LazyTensors(list):
+    def __getitem__(self, i):
+        return f32(list.__getitem__(self, i))
+
+
+def host_view(w, c, lazy=False):
+    layers = LazyLayers(w["layers"]) if lazy else [
+        None if lw is None else {k: f32(v) for k, v in lw.items()} for lw in w["layers"]]
+    wn = {"embed": f32(w["embed"]), "final_norm": f32(w["final_norm"]),
+          "lm_head": f32(w["lm_head"]), "layers": layers}
+    if lazy:
+        kk, vv = LazyTensors(c["k"]), LazyTensors(c["v"])
+    else:
+        kk, vv = [f32(x) for x in c["k"]], [f32(x) for x in c["v"]]
+    cn = {"k": kk, "v": vv, "tokens": c["tokens"].cpu().numpy(), "pos": c["pos"].cpu().numpy(),
+          "seq_len": c["seq_len"].cpu().numpy(), "h_last": f32(c["h_last"])}
+    return wn, cn
+
+
+def sample(seq_lens, per_seq, seed):
+    r = np.random.default_rng(seed)
+    out = []
+    for n in seq_lens:
+        pick = {0, 1, n // 2, n - 3, n - 2, n - 1} | set(r.choice(n, size=per_seq, replace=False).tolist())
+        out.append(sorted(x for x in pick if 0 <= x < n))
+    return out
+
+
+def gpu_scores(pkg, shape, w, c, mode, full):
+    from paper_2607_27600_gb300 import cc
+    b, cap = c["tokens"].shape
+    scores = torch.empty(b, cap, dtype=torch.float32, device="cuda")
+    ws = cc.alloc_workspace(cc.cc_score_workspace_size(shape, b, cap, mode))
+    fn = cc.cc_score_full if full else cc.cc_score_layer
+    fn(shape, pkg.Weights(w), pkg.Cache(c), mode, scores, ws)
+    assert cc.cc_get_status() == cc.CC_OK
+    del ws
+    return scores.cpu().numpy()
+
+
+def check_rows(got, want, rows):
+    errs = []
+    for b, r in enumerate(rows):
+        errs.append(rel_err(got[b, r], want[b, r]))
+    return max(errs)
+
+
+def workload_inputs(wl, layers_only_last=True):
+    shape = wl.shape
+    fast = wl.mode == "layer"
+    layers = [shape.n_layers - 1] if fast else None
+    w = synth.model_weights(shape, wl.seed, device="cuda", layers=layers, with_embed=not fast)
+    c = synth.synthetic_cache(shape, wl.seq_lens, wl.cap, wl.seed, device="cuda",
+                              layers=layers, with_h_last=fast)
+    return w, c
+
+
+@pytest.mark.parametrize("name", ["llama8b-layer-8k", "llama8b-layer-32k-ragged"])
+def test_fast_pass_full_size_sampled_rows(pkg, name):
+    from paper_2607_27600_gb300 import cc
+    wl = synth.WORKLOADS[name]
+    w, c = workload_inputs(wl)
+    got = gpu_scores(pkg, wl.shape, w, c, cc.SCORE_LOGIT, full=False)
+    wn, cn = host_view(w, c)
+    rows = sample(wl.seq_lens, 24, seed=1)
+    want = oracle.score_layer(wl.shape, wn, cn, rows=rows)
+    assert check_rows(got, want, rows) < TOL
+    for b, n in enumerate(wl.seq_lens):    # every slot is written: -inf past the end
+        assert got[b, n - 1] == np.inf and np.all(got[b, n:] == -np.inf)
+        assert np.all(np.isfinite(got[b, :n - 1]))
+
+
+def test_fast_pass_logprob_full_size(pkg):
+    from paper_2607_27600_gb300 import cc
+    wl = synth.WORKLOADS["llama8b-layer-8k"]
+    w, c = workload_inputs(wl)
+    got = gpu_scores(pkg, wl.shape, w, c, cc.SCORE_LOGPROB, full=False)
+    wn, cn = host_view(w, c)
+    rows = sample(wl.seq_lens, 6, seed=2)
+    want = oracle.score_layer(wl.shape, wn, cn, mode="logprob", rows=rows)
+    assert check_rows(got, want, rows) < TOL
+
+
+def test_full_pass_32_layers_sampled_rows(pkg):
+    from paper_2607_27600_gb300 import cc
+    wl = synth.WORKLOADS["llama8b-full-16k"]
+    w, c = workload_inputs(wl)
+    got = gpu_scores(pkg, wl.shape, w, c, cc.SCORE_LOGIT, full=True)
+    wn, cn = host_view(w, c, lazy=True)
+    rows = [[0, 5, 8191, 16381, 16382, 16383]]
+    want = oracle.score_full(wl.shape, wn, cn, rows=rows)
+    assert check_rows(got, want, rows) < TOL
+
+
+def test_headline_keep_set_full_oracle(pkg):
+    """llama8b-layer-8k end to end: every row scored by the oracle; the GPU
+    keep-set is identical where the oracle's boundary gap exceeds the
+    tolerance, else overlaps >= 99.5 %; the GPU select equals the oracle's
+    select on the same fp32 scores exactly."""
+    from paper_2607_27600_gb300 import cc
+    wl = synth.WORKLOADS["llama8b-layer-8k"]
+    w, c = workload_inputs(wl)
+    got = gpu_scores(pkg, wl.shape, w, c, cc.SCORE_LOGIT, full=False)
+    wn, cn = host_view(w, c)
+    want = oracle.score_layer(wl.shape, wn, cn)
+    assert rel_err(got, want) < TOL
+    b, cap = c["tokens"].shape
+    idx = torch.empty(b, cap, dtype=torch.int32, device="cuda")
+    cnt = torch.empty(b, dtype=torch.int32, device="cuda")
+    cc.cc_select_keep(torch.from_numpy(got).cuda(), c["seq_len"], b, cap,
+                      torch.tensor(wl.budgets, dtype=torch.int32, device="cuda"), 0, idx, cnt)
+    gi, gc = idx.cpu().numpy(), cnt.cpu().numpy()
+    oi, oc = oracle.select_keep(got, wl.seq_lens, wl.budgets)
+    assert np.array_equal(gc, oc) and np.array_equal(gi[0, :oc[0]], oi[0, :oc[0]])
+    wi, wc = oracle.select_keep(want.astype(np.float32), wl.seq_lens, wl.budgets)
+    ok, det = keep_set_ok(gi, gc, wi, wc, want, wl.seq_lens, wl.budgets)
+    assert ok, det
+
+
+def seeded_keep(n, budget, seed):
+    """A seeded keep-set of `budget` slots of [0, n), the last slot always in."""
+    r = np.random.default_rng(seed)
+    k = r.choice(n - 1, size=budget - 1, replace=False)
+    return np.sort(np.concatenate([k, [n - 1]])).astype(np.int32)
+
+
+def test_long_context_refresh_cycles(pkg):
+    """Qwen2.5-7B-like last layer at 131072 positions, then refresh cycles of
+    +4096 appended slots: cycle 1 scored in full size; between cycles both
+    sides compact with the same seeded keep-set (bit-exact check) and append
+    the same seeded chunk; each cycle's scores compared on sampled rows."""
+    from paper_2607_27600_gb300 import cc
+    wl = synth.WORKLOADS["qwen7b-layer-128k"]
+    shape = wl.shape
+    w, c = workload_inputs(wl)
+    wn, cn = host_view(w, c)
+    last = shape.n_layers - 1
+    for cycle in range(wl.cycles):
+        n = int(c["seq_len"][0])
+        got = gpu_scores(pkg, shape, w, c, cc.SCORE_LOGIT, full=False)
+        rows = sample([n], 8 if cycle == 0 else 24, seed=10 + cycle)
+        want = oracle.score_layer(shape, wn, cn, rows=rows)
+        assert check_rows(got, want, rows) < TOL, cycle
+        if cycle + 1 == wl.cycles:
+            break
+        keep = seeded_keep(n, wl.budgets[0], seed=100 + cycle)
+        idx = np.full((1, wl.cap), -1, np.int32)
+        idx[0, :len(keep)] = keep
+        cnt = np.array([len(keep)], np.int32)
+        cache = pkg.Cache(c)
+        cws = cc.alloc_workspace(cc.cc_compact_workspace_size(shape, cache))
+        cc.cc_compact_kv(shape, cache, torch.from_numpy(idx).cuda(), torch.from_numpy(cnt).cuda(), cws)
+        assert cc.cc_get_status() == cc.CC_OK
+        for key in ("tokens", "pos"):
+            cn[key] = oracle.compact(cn[key], idx, cnt)
+        cn["h_last"] = oracle.compact(cn["h_last"], idx, cnt)
+        cn["k"][last] = oracle.compact(cn["k"][last], idx, cnt)
+        cn["v"][last] = oracle.compact(cn["v"][last], idx, cnt)
+        cn["seq_len"] = cnt.copy()
+        np.testing.assert_array_equal(f32(c["k"][last])[0, :len(keep)], cn["k"][last][0, :len(keep)])
+        np.testing.assert_array_equal(c["pos"].cpu().numpy()[0, :len(keep)], cn["pos"][0, :len(keep)])
+        # inference cycle: append the next chunk on the device, mirror it on the host
+        synth.append_chunk(shape, c, wl.append, wl.seed, cycle + 1)
+        s0, s1 = len(keep), len(keep) + wl.append
+        for key in ("tokens", "pos"):
+            cn[key][:, s0:s1] = c[key][:, s0:s1].cpu().numpy()
+        cn["h_last"][:, s0:s1] = f32(c["h_last"][:, s0:s1])
+        cn["k"][last][:, s0:s1] = f32(c["k"][last][:, s0:s1])
+        cn["v"][last][:, s0:s1] = f32(c["v"][last][:, s0:s1])
+        cn["seq_len"] = c["seq_len"].cpu().numpy()
