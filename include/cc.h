@@ -153,6 +153,29 @@ cc_status cc_compact_kv(const cc_model_cfg *cfg, const cc_kv_cache *cache,
                         const int32_t *keep_idx, const int32_t *keep_count, void *ws,
                         size_t ws_bytes, void *stream);
 
+/* ---- compaction without a workspace -----------------------------------------
+ * The paper has no counterpart: this is a library convenience.
+ * Same operation, checks and results as cc_compact_kv, for callers that
+ * cannot allocate device memory for a workspace when they compact -- for
+ * example a serving loop that has handed the whole device pool to the KV
+ * cache, or a runtime that forbids device allocation on its refresh path
+ * (cudaMalloc may block and synchronise the device).  Its scratch (a ticket
+ * counter and one flag per work unit) lives in a fixed 1 MiB array in the
+ * library's device memory, which every GPU that loads the library holds
+ * until the process exits.  The call allocates nothing.
+ *   - A cache needing more than 1 MiB of scratch (more than 262080 work
+ *     units; cc_compact_workspace_size() - 256 bytes / 4) is rejected with
+ *     CC_ERR_WORKSPACE before anything is enqueued.
+ *   - The first call on a device looks up the array's device address (with
+ *     that device current); make that first call before any stream capture.
+ *   - All calls on a device share the array and each call clears it first
+ *     (an asynchronous memset on `stream`): calls whose work overlaps on the
+ *     GPU (different streams, no ordering between them) race on it and must
+ *     not be issued. */
+cc_status cc_compact_kv_static(const cc_model_cfg *cfg, const cc_kv_cache *cache,
+                               const int32_t *keep_idx, const int32_t *keep_count,
+                               void *stream);
+
 /* ---- status ---------------------------------------------------------------
  * Synchronises `stream`, returns the first device-side error recorded since
  * the last call (CC_OK if none) on the current device and clears it.

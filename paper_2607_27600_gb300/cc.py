@@ -78,6 +78,9 @@ _SIGS = {
     "cc_compact_kv": (ctypes.c_int, [ctypes.POINTER(cc_model_cfg), ctypes.POINTER(cc_kv_cache),
                                      ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,
                                      ctypes.c_size_t, ctypes.c_void_p]),
+    "cc_compact_kv_static": (ctypes.c_int, [ctypes.POINTER(cc_model_cfg),
+                                            ctypes.POINTER(cc_kv_cache), ctypes.c_void_p,
+                                            ctypes.c_void_p, ctypes.c_void_p]),
     "cc_get_status": (ctypes.c_int, [ctypes.c_void_p]),
     "cc_status_str": (ctypes.c_char_p, [ctypes.c_int]),
     "cc_linear_f32": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,
@@ -244,6 +247,15 @@ def cc_compact_kv(cfg, cache: Cache, keep_idx, keep_count, ws, stream=None):
                                         _dev_ptr(keep_count, "keep_count"), _dev_ptr(ws, "ws"),
                                         ws.numel() * ws.element_size(), _stream(stream))
     _check(code, "cc_compact_kv")
+
+
+def cc_compact_kv_static(cfg, cache: Cache, keep_idx, keep_count, stream=None):
+    """cc_compact_kv without a workspace: the library's fixed 1 MiB device
+    scratch array is used instead (shared by every call on the device)."""
+    code = load_library().cc_compact_kv_static(ctypes.byref(_cfg(cfg)), ctypes.byref(cache.c),
+                                               _dev_ptr(keep_idx, "keep_idx"),
+                                               _dev_ptr(keep_count, "keep_count"), _stream(stream))
+    _check(code, "cc_compact_kv_static")
 
 
 def cc_get_status(stream=None) -> int:

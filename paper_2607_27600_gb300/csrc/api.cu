@@ -636,3 +636,30 @@ const char *cc_kernel_name(int32_t kind) {
 }
 
 }  // extern "C"
+
+// ---- library-internal helpers (internal.h) ----------------------------------
+#include "internal.h"
+
+namespace cc {
+
+cc_status compact_plan_build(const cc_model_cfg *cfg, const cc_kv_cache *cache, CompactParams &p,
+                             size_t &scratch_bytes) {
+  static CompactPlan plan;
+  static std::mutex mu;
+  std::lock_guard<std::mutex> lk(mu);
+  cc_status s = compact_plan(cfg, cache, plan);
+  if (s != CC_OK) return s;
+  p = plan.p;
+  scratch_bytes = plan.ws_bytes;
+  return CC_OK;
+}
+
+bool current_device_info(unsigned **status, int *sms) {
+  DevState *d;
+  if (!dev_state(&d)) return false;
+  *status = d->status;
+  *sms = d->sms;
+  return true;
+}
+
+}  // namespace cc

@@ -1,0 +1,69 @@
+// compact_static.cu -- cc_compact_kv_static: the in-place compaction of
+// cc_compact_kv for callers that cannot allocate device memory.
+//
+// cc_compact_kv takes its scratch (a work-unit ticket counter and one
+// "sources read" flag per unit) from a caller-provided workspace.  This
+// variant takes it from a fixed array in the library's own device memory
+// instead, so the caller passes only the cache, the keep-set and a stream.
+// The array is a file-scope __device__ variable: every GPU that loads the
+// library holds its kStaticScratchBytes until the process exits, and every
+// call on a device shares it.
+#include <mutex>
+
+#include "internal.h"
+
+namespace {
+
+// 1 MiB: a 256-byte ticket slot plus up to 262080 unit flags (4 bytes each).
+constexpr size_t kStaticScratchBytes = size_t(1) << 20;
+__device__ __align__(256) unsigned char g_compact_scratch[kStaticScratchBytes];
+
+constexpr int kMaxDevices = 64;
+// Device address of g_compact_scratch per device.  In host code the symbol
+// name is only a host-side stand-in, never a device address.
+unsigned char *g_scratch_addr[kMaxDevices] = {};
+std::mutex g_scratch_mu;
+
+cc_status scratch_address(unsigned char **out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return CC_ERR_CUDA;
+  std::lock_guard<std::mutex> lk(g_scratch_mu);
+  if (!g_scratch_addr[dev]) {   // set-up, once per device, with that device current
+    void *p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_compact_scratch) != cudaSuccess || !p) return CC_ERR_CUDA;
+    g_scratch_addr[dev] = static_cast<unsigned char *>(p);
+  }
+  *out = g_scratch_addr[dev];
+  return CC_OK;
+}
+
+}  // namespace
+
+extern "C" cc_status cc_compact_kv_static(const cc_model_cfg *cfg, const cc_kv_cache *cache,
+                                          const int32_t *keep_idx, const int32_t *keep_count,
+                                          void *stream) {
+  static cc::CompactParams p;   // large kernel-parameter block; guarded by mu
+  static std::mutex mu;
+  std::lock_guard<std::mutex> lk(mu);
+  size_t need = 0;
+  cc_status s = cc::compact_plan_build(cfg, cache, p, need);
+  if (s != CC_OK) return s;
+  if (!keep_idx || !keep_count) return CC_ERR_INVALID_ARG;
+  if (need > kStaticScratchBytes) return CC_ERR_WORKSPACE;   // too many work units
+  unsigned char *scratch = nullptr;
+  if ((s = scratch_address(&scratch)) != CC_OK) return s;
+  unsigned *status = nullptr;
+  int sms = 0;
+  if (!cc::current_device_info(&status, &sms)) return CC_ERR_CUDA;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  // the ticket and the flags must start at zero; the array keeps the last call's contents
+  if (cudaMemsetAsync(scratch, 0, need, st) != cudaSuccess) return CC_ERR_CUDA;
+  p.keep_idx = keep_idx;
+  p.keep_count = keep_count;
+  p.seq_len = cache->seq_len;
+  p.ticket = reinterpret_cast<unsigned *>(scratch);
+  p.flags = reinterpret_cast<unsigned *>(scratch + 256);
+  p.status = status;
+  if (cc::launch_compact(p, sms * 3, st) != cudaSuccess) return CC_ERR_CUDA;
+  return CC_OK;
+}
