@@ -168,17 +168,20 @@ struct ScoreWs {
   int n_vtiles;
 };
 
-ScoreWs score_layout(const cc_model_cfg *c, int batch, int cap, cc_score_mode mode) {
+// The full pass carries the GEMM activations (normalised inputs, attention
+// output, SwiGLU output) as [hi | lo] bf16 pairs: split = 2 copies per row.
+ScoreWs score_layout(const cc_model_cfg *c, int batch, int cap, cc_score_mode mode, bool full) {
   ScoreWs w{};
   const size_t R = (size_t)batch * cap;
   const size_t d = c->d_model, qd = (size_t)c->n_q_heads * c->head_dim, f = c->d_ff;
+  const size_t split = full ? 2 : 1;
   size_t off = 0;
   auto take = [&](size_t bytes) { size_t o = off; off = align256(off + bytes); return o; };
-  w.xn = take(R * d * 2);
+  w.xn = take(R * d * 2 * split);
   w.q = take(R * qd * 2);
-  w.o = take(R * qd * 2);
+  w.o = take(R * qd * 2 * split);
   w.h = take(R * d * 4);
-  w.act = take(R * f * 2);
+  w.act = take(R * f * 2 * split);
   w.n_vtiles = (c->vocab + 255) / 256;
   if (mode == CC_SCORE_LOGPROB) {
     w.part = take(R * w.n_vtiles * 8);
@@ -210,11 +213,13 @@ struct Gemm {
 };
 
 // One GEMM over the cache rows: A [R][K] (bf16 workspace) x W [N][K]^T.
+// a_split: A rows are [hi | lo] (2K values) and the product is hi W^T + lo W^T.
 cc_status gemm_setup(Gemm &g, int epi, const void *A, int K, const void *W, const void *W2, int N,
-                     int batch, int cap, const int32_t *seq_len, unsigned *status) {
+                     int batch, int cap, const int32_t *seq_len, unsigned *status,
+                     bool a_split = false) {
   const uint64_t R = (uint64_t)batch * cap;
   const int bn = gemm_block_n(epi);
-  if (!tmap_rows(&g.a, A, R, K, 128)) return CC_ERR_CUDA;
+  if (!tmap_rows(&g.a, A, R, a_split ? 2 * K : K, 128)) return CC_ERR_CUDA;
   if (!tmap_rows(&g.b, W, N, K, epi == EPI_SWIGLU ? 128 : 256)) return CC_ERR_CUDA;
   if (epi == EPI_SWIGLU) {
     if (!tmap_rows(&g.b2, W2, N, K, 128)) return CC_ERR_CUDA;
@@ -229,6 +234,7 @@ cc_status gemm_setup(Gemm &g, int epi, const void *A, int K, const void *W, cons
   g.p.K = K;
   g.p.n_tiles = (N + bn - 1) / bn;
   g.p.status = status;
+  g.p.a_split = a_split ? 1 : 0;
   return CC_OK;
 }
 
@@ -238,9 +244,10 @@ cc_status run_gemm(Gemm &g, int epi, int kind, int sms, cudaStream_t st) {
   return CC_OK;
 }
 
+// out: [R][Hq*dh] bf16, or with split [R][2*Hq*dh] = [hi | lo] per row.
 cc_status run_attention(const cc_model_cfg *c, const void *q, const void *k, const void *v,
                         void *out, const int32_t *seq_len, int batch, int cap, unsigned *status,
-                        cudaStream_t st) {
+                        cudaStream_t st, bool split = false) {
   const int G = c->n_q_heads / c->n_kv_heads, dh = c->head_dim;
   const int P = attn_positions_per_unit(G);
   const uint64_t R = (uint64_t)batch * cap;
@@ -268,6 +275,8 @@ cc_status run_attention(const cc_model_cfg *c, const void *q, const void *k, con
   p.P = P;
   p.seq_len = seq_len;
   p.out = reinterpret_cast<__nv_bfloat16 *>(out);
+  p.out_ld = c->n_q_heads * dh * (split ? 2 : 1);
+  p.out_lo = split ? c->n_q_heads * dh : 0;
   p.scale_log2 = (float)(1.4426950408889634 / sqrt((double)dh));
   p.status = status;
   TimedScope t(CC_KERNEL_ATTENTION, st);
@@ -300,7 +309,8 @@ cc_status check_score_args(const cc_model_cfg *c, const cc_model_weights *w, con
   const void *ptrs[] = {w->final_norm, w->lm_head, ws, kv->h_last, full ? w->embed : nullptr};
   for (const void *p : ptrs)
     if (p && !aligned16(p)) return CC_ERR_INVALID_ARG;
-  if (!ws || ws_bytes < score_layout(c, kv->batch, kv->cap, mode).total) return CC_ERR_WORKSPACE;
+  if (!ws || ws_bytes < score_layout(c, kv->batch, kv->cap, mode, full).total)
+    return CC_ERR_WORKSPACE;
   return CC_OK;
 }
 
@@ -314,7 +324,8 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   const int batch = kv->batch, cap = kv->cap, rows = batch * cap;
   const int d = c->d_model, qd = c->n_q_heads * c->head_dim, f = c->d_ff;
-  const ScoreWs L = score_layout(c, batch, cap, mode);
+  const ScoreWs L = score_layout(c, batch, cap, mode, full);
+  const bool split = full;   // [hi | lo] activations in the full pass
   uint8_t *wsb = reinterpret_cast<uint8_t *>(ws);
   void *xn = wsb + L.xn, *q = wsb + L.q, *o = wsb + L.o, *act = wsb + L.act;
   float *h = reinterpret_cast<float *>(wsb + L.h);
@@ -333,11 +344,12 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
     {
       TimedScope t(CC_KERNEL_RMSNORM, st);
       CC_TRY(launch_rmsnorm(first_from_bf16 ? kv->h_last : (const void *)h, !first_from_bf16,
-                            lw.attn_norm, xn, d, c->rms_eps, sl, cap, rows, st));
+                            lw.attn_norm, xn, d, c->rms_eps, sl, cap, rows, split, st));
     }
     // Q = RoPE(xn Wq^T)
     Gemm gq;
-    if ((s = gemm_setup(gq, EPI_QROPE, xn, d, lw.wq, nullptr, qd, batch, cap, sl, status)) != CC_OK)
+    if ((s = gemm_setup(gq, EPI_QROPE, xn, d, lw.wq, nullptr, qd, batch, cap, sl, status,
+                        split)) != CC_OK)
       return s;
     gq.p.out = q;
     gq.p.ldo = qd;
@@ -346,12 +358,14 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
     rope_turns(c, gq.p.turns);
     if ((s = run_gemm(gq, EPI_QROPE, CC_KERNEL_GEMM_QROPE, dev->sms, st)) != CC_OK) return s;
     // O = counter-causal attention
-    if ((s = run_attention(c, q, kv->k[l], kv->v[l], o, sl, batch, cap, status, st)) != CC_OK)
+    if ((s = run_attention(c, q, kv->k[l], kv->v[l], o, sl, batch, cap, status, st, split)) !=
+        CC_OK)
       return s;
     // h = h + O Wo^T  (fast mode: h = H^(L-1) + O Wo^T)
     Gemm go;
     const int epi_o = first_from_bf16 ? EPI_RESID_BF16 : EPI_RESID_F32;
-    if ((s = gemm_setup(go, epi_o, o, qd, lw.wo, nullptr, d, batch, cap, sl, status)) != CC_OK)
+    if ((s = gemm_setup(go, epi_o, o, qd, lw.wo, nullptr, d, batch, cap, sl, status, split)) !=
+        CC_OK)
       return s;
     go.p.out = h;
     go.p.ldo = d;
@@ -361,19 +375,20 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
     // xn = RMSNorm(h); act = silu(xn Wg^T) * (xn Wu^T)
     {
       TimedScope t(CC_KERNEL_RMSNORM, st);
-      CC_TRY(launch_rmsnorm(h, true, lw.mlp_norm, xn, d, c->rms_eps, sl, cap, rows, st));
+      CC_TRY(launch_rmsnorm(h, true, lw.mlp_norm, xn, d, c->rms_eps, sl, cap, rows, split, st));
     }
     Gemm gu;
-    if ((s = gemm_setup(gu, EPI_SWIGLU, xn, d, lw.w_gate, lw.w_up, f, batch, cap, sl, status)) !=
-        CC_OK)
+    if ((s = gemm_setup(gu, EPI_SWIGLU, xn, d, lw.w_gate, lw.w_up, f, batch, cap, sl, status,
+                        split)) != CC_OK)
       return s;
     gu.p.out = act;
-    gu.p.ldo = f;
+    gu.p.ldo = split ? 2 * f : f;
+    gu.p.out_split = split ? 1 : 0;
     if ((s = run_gemm(gu, EPI_SWIGLU, CC_KERNEL_GEMM_GATEUP, dev->sms, st)) != CC_OK) return s;
     // h = h + act Wd^T
     Gemm gd;
     if ((s = gemm_setup(gd, EPI_RESID_F32, act, f, lw.w_down, nullptr, d, batch, cap, sl,
-                        status)) != CC_OK)
+                        status, split)) != CC_OK)
       return s;
     gd.p.out = h;
     gd.p.ldo = d;
@@ -387,11 +402,11 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
   } else {
     {
       TimedScope t(CC_KERNEL_RMSNORM, st);
-      CC_TRY(launch_rmsnorm(h, true, w->final_norm, xn, d, c->rms_eps, sl, cap, rows, st));
+      CC_TRY(launch_rmsnorm(h, true, w->final_norm, xn, d, c->rms_eps, sl, cap, rows, split, st));
     }
     Gemm gl;
     if ((s = gemm_setup(gl, EPI_LSE, xn, d, w->lm_head, nullptr, c->vocab, batch, cap, sl,
-                        status)) != CC_OK)
+                        status, split)) != CC_OK)
       return s;
     float2 *part = reinterpret_cast<float2 *>(wsb + L.part);
     float *zt = reinterpret_cast<float *>(wsb + L.ztgt);
@@ -459,7 +474,7 @@ extern "C" {
 size_t cc_score_workspace_size(const cc_model_cfg *cfg, int32_t batch, int32_t cap,
                                cc_score_mode mode) {
   if (check_cfg(cfg) != CC_OK || batch < 1 || cap < 1) return 0;
-  return score_layout(cfg, batch, cap, mode).total;
+  return score_layout(cfg, batch, cap, mode, true).total;   // enough for either pass
 }
 
 cc_status cc_score_layer(const cc_model_cfg *cfg, const cc_model_weights *w,

@@ -90,8 +90,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (ntiles <= 0) {   // no slot after the block: every row attends nothing -> 0
     for (int idx = threadIdx.x; idx < (p_last - p0 + 1) * G; idx += blockDim.x) {
       int pos = p0 + idx / G, hl = idx % G;
-      uint4 *dst = reinterpret_cast<uint4 *>(p.out + ((row_base + pos) * p.n_q_heads + g * G + hl) * DH);
-      for (int v = 0; v < DH / 8; ++v) dst[v] = make_uint4(0, 0, 0, 0);
+      __nv_bfloat16 *o = p.out + (row_base + pos) * p.out_ld + (size_t)(g * G + hl) * DH;
+      for (int v = 0; v < DH / 8; ++v) reinterpret_cast<uint4 *>(o)[v] = make_uint4(0, 0, 0, 0);
+      if (p.out_lo > 0)
+        for (int v = 0; v < DH / 8; ++v)
+          reinterpret_cast<uint4 *>(o + p.out_lo)[v] = make_uint4(0, 0, 0, 0);
     }
     return;
   }
@@ -320,7 +323,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc_fence_after();
       const bool store = row_used && pos <= p_last;
       const float inv = l > 0.f ? 1.f / l : 0.f;
-      __nv_bfloat16 *dst = p.out + ((row_base + (store ? pos : 0)) * p.n_q_heads + g * G + hl) * DH;
+      __nv_bfloat16 *dst =
+          p.out + (row_base + (store ? pos : 0)) * p.out_ld + (size_t)(g * G + hl) * DH;
 #pragma unroll 1
       for (int c = 0; c < DH; c += 32) {
         uint32_t o[32];
@@ -334,6 +338,17 @@ __global__ void __launch_bounds__(kThreads, 1)
           uint4 *d = reinterpret_cast<uint4 *>(dst + c);
 #pragma unroll
           for (int v = 0; v < 4; ++v) d[v] = make_uint4(pk[v * 4], pk[v * 4 + 1], pk[v * 4 + 2], pk[v * 4 + 3]);
+          if (p.out_lo > 0) {   // lo = bf16(o - hi)
+            uint32_t lo[16];
+#pragma unroll
+            for (int k = 0; k < 32; k += 2)
+              lo[k / 2] = pack_bf16x2(__uint_as_float(o[k]) * inv - bf16_lo(pk[k / 2]),
+                                      __uint_as_float(o[k + 1]) * inv - bf16_hi(pk[k / 2]));
+            uint4 *dl = reinterpret_cast<uint4 *>(dst + p.out_lo + c);
+#pragma unroll
+            for (int v = 0; v < 4; ++v)
+              dl[v] = make_uint4(lo[v * 4], lo[v * 4 + 1], lo[v * 4 + 2], lo[v * 4 + 3]);
+          }
         }
       }
     }

@@ -9,7 +9,9 @@ struct AttnParams {
   int n_q_heads, n_kv_heads, head_dim, group;
   int P;                    // positions per work unit (attn_positions_per_unit(group))
   const int32_t *seq_len;   // device [batch]
-  __nv_bfloat16 *out;       // [batch*cap][n_q_heads][head_dim]
+  __nv_bfloat16 *out;       // row r, head t at out + r*out_ld + t*head_dim
+  int out_ld;               // elements per output row (n_q_heads*head_dim, or twice that)
+  int out_lo;               // > 0: also write lo = bf16(o - hi) at element offset out_lo
   float scale_log2;         // log2(e) / sqrt(head_dim)
   unsigned *status;
 };

@@ -138,6 +138,19 @@ CC_DEV void epilogue_tile(const GemmParams &p, uint32_t tacc, int grow, bool val
       uint4 *d = reinterpret_cast<uint4 *>(out + col);
 #pragma unroll
       for (int v = 0; v < 4; ++v) d[v] = make_uint4(o[v * 4], o[v * 4 + 1], o[v * 4 + 2], o[v * 4 + 3]);
+      if (p.out_split) {   // lo = bf16(y - hi)
+        uint32_t lo[16];
+#pragma unroll
+        for (int k = 0; k < 32; k += 2) {
+          float y0 = silu(__uint_as_float(g[k])) * __uint_as_float(u[k]);
+          float y1 = silu(__uint_as_float(g[k + 1])) * __uint_as_float(u[k + 1]);
+          lo[k / 2] = pack_bf16x2(y0 - bf16_lo(o[k / 2]), y1 - bf16_hi(o[k / 2]));
+        }
+        uint4 *dl = reinterpret_cast<uint4 *>(out + p.N + col);
+#pragma unroll
+        for (int v = 0; v < 4; ++v)
+          dl[v] = make_uint4(lo[v * 4], lo[v * 4 + 1], lo[v * 4 + 2], lo[v * 4 + 3]);
+      }
     }
   } else if constexpr (EPI == EPI_LSE) {
     // per row: (max, sum exp(z - max)) over this tile's vocab columns, and the
@@ -220,7 +233,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem_base = *tmem_slot;
   const int num_m = prefix[p.batch];
   const int total = num_m * p.n_tiles;
-  const int nk = (p.K + BK - 1) / BK;
+  const int nk = (p.K + BK - 1) / BK;           // k-blocks of one operand pass
+  const int nk_total = p.a_split ? 2 * nk : nk;  // split A: the hi pass, then the lo pass
 
   if (warp == 0) {
     if (lane == 0) {  // ---------------- TMA producer
@@ -230,16 +244,18 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int nt = tile / num_m, mt = tile - nt * num_m;
         const int b = find_seq(prefix, p.batch, mt);
         const int row0 = b * p.cap + (mt - prefix[b]) * BM;
-        for (int kb = 0; kb < nk; ++kb) {
+        for (int kb = 0; kb < nk_total; ++kb) {
           if (!mbar_wait(&empty[stage], phase ^ 1, abort_flag, p.status)) goto producer_done;
           mbar_arrive_expect_tx(&full[stage], A_BYTES + B_BYTES);
-          tma_load_2d(sA + stage * A_BYTES, &tmA, &full[stage], kb * BK, row0);
+          // A column block kb of [hi | lo] (hi and lo halves are K apart), B block kb mod nk
+          const int ka = kb < nk ? kb * BK : p.K + (kb - nk) * BK;
+          const int kw = (kb < nk ? kb : kb - nk) * BK;
+          tma_load_2d(sA + stage * A_BYTES, &tmA, &full[stage], ka, row0);
           if constexpr (EPI == EPI_SWIGLU) {
-            tma_load_2d(sB + stage * B_BYTES, &tmB, &full[stage], kb * BK, nt * 128);
-            tma_load_2d(sB + stage * B_BYTES + B_BYTES / 2, &tmB2, &full[stage], kb * BK,
-                        nt * 128);
+            tma_load_2d(sB + stage * B_BYTES, &tmB, &full[stage], kw, nt * 128);
+            tma_load_2d(sB + stage * B_BYTES + B_BYTES / 2, &tmB2, &full[stage], kw, nt * 128);
           } else {
-            tma_load_2d(sB + stage * B_BYTES, &tmB, &full[stage], kb * BK, nt * BN);
+            tma_load_2d(sB + stage * B_BYTES, &tmB, &full[stage], kw, nt * BN);
           }
           if (++stage == ST) { stage = 0; phase ^= 1; }
         }
@@ -255,7 +271,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!mbar_wait(&tempty[acc], acc_phase ^ 1, abort_flag, p.status)) break;
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + acc * BN;
-        for (int kb = 0; kb < nk; ++kb) {
+        for (int kb = 0; kb < nk_total; ++kb) {
           if (!mbar_wait(&full[stage], phase, abort_flag, p.status)) goto mma_done;
           tc_fence_after();
           const uint32_t a0 = smem_u32(sA + stage * A_BYTES);

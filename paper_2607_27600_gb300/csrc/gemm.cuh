@@ -28,6 +28,8 @@ struct GemmParams {
   const int32_t *tokens;   // EPI_LSE
   float *z_target;         // EPI_LSE
   unsigned *status;
+  int a_split;             // A rows are [hi | lo] (2K values): D = hi W^T + lo W^T
+  int out_split;           // EPI_SWIGLU: out rows are [hi | lo], lo at column offset N
   unsigned long long turns[64];  // EPI_QROPE: inv_freq_k / (2 pi) in 0.64 fixed point
 };
 

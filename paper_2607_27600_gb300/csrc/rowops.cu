@@ -51,11 +51,12 @@ CC_DEV float row_inv_rms(const void *row, int d, float eps, int lane) {
   return rsqrtf(ss / (float)d + eps);
 }
 
-// out (bf16) = x * gain / rms(x)
+// out (bf16) = x * gain / rms(x).  split: the row holds [hi | lo] (2d values),
+// hi = bf16(y), lo = bf16(y - hi), so hi + lo carries y to ~2^-17.
 template <bool IN_F32>
 __global__ void __launch_bounds__(kWarps * 32)
     rmsnorm_kernel(const void *x, const __nv_bfloat16 *gain, __nv_bfloat16 *out, int d, float eps,
-                   const int32_t *seq_len, int cap, int rows) {
+                   const int32_t *seq_len, int cap, int rows, int split) {
   const int lane = threadIdx.x & 31;
   const int row = blockIdx.x * kWarps + (threadIdx.x >> 5);
   int i, n;
@@ -63,17 +64,27 @@ __global__ void __launch_bounds__(kWarps * 32)
   const size_t es = IN_F32 ? 4 : 2;
   const void *xr = reinterpret_cast<const uint8_t *>(x) + (size_t)row * d * es;
   const float inv = row_inv_rms<IN_F32>(xr, d, eps, lane);
-  __nv_bfloat16 *o = out + (size_t)row * d;
+  __nv_bfloat16 *o = out + (size_t)row * d * (split ? 2 : 1);
   for (int e = lane * 8; e < d; e += 256) {
     float f[8], gf[8];
     load8<IN_F32>(xr, e, f);
     unpack8(*reinterpret_cast<const uint4 *>(gain + e), gf);
+#pragma unroll
+    for (int k = 0; k < 8; ++k) f[k] = f[k] * inv * gf[k];
     uint4 v;
-    v.x = pack_bf16x2(f[0] * inv * gf[0], f[1] * inv * gf[1]);
-    v.y = pack_bf16x2(f[2] * inv * gf[2], f[3] * inv * gf[3]);
-    v.z = pack_bf16x2(f[4] * inv * gf[4], f[5] * inv * gf[5]);
-    v.w = pack_bf16x2(f[6] * inv * gf[6], f[7] * inv * gf[7]);
+    v.x = pack_bf16x2(f[0], f[1]);
+    v.y = pack_bf16x2(f[2], f[3]);
+    v.z = pack_bf16x2(f[4], f[5]);
+    v.w = pack_bf16x2(f[6], f[7]);
     *reinterpret_cast<uint4 *>(o + e) = v;
+    if (split) {
+      uint4 lo;
+      lo.x = pack_bf16x2(f[0] - bf16_lo(v.x), f[1] - bf16_hi(v.x));
+      lo.y = pack_bf16x2(f[2] - bf16_lo(v.y), f[3] - bf16_hi(v.y));
+      lo.z = pack_bf16x2(f[4] - bf16_lo(v.z), f[5] - bf16_hi(v.z));
+      lo.w = pack_bf16x2(f[6] - bf16_lo(v.w), f[7] - bf16_hi(v.w));
+      *reinterpret_cast<uint4 *>(o + d + e) = lo;
+    }
   }
 }
 
@@ -169,14 +180,16 @@ unsigned blocks_for(int rows) { return (unsigned)((rows + kWarps - 1) / kWarps);
 }  // namespace
 
 cudaError_t launch_rmsnorm(const void *x, bool x_f32, const void *gain, void *out, int d, float eps,
-                           const int32_t *seq_len, int cap, int rows, cudaStream_t st) {
+                           const int32_t *seq_len, int cap, int rows, bool split, cudaStream_t st) {
   if (rows <= 0) return cudaSuccess;
   auto *g = reinterpret_cast<const __nv_bfloat16 *>(gain);
   auto *o = reinterpret_cast<__nv_bfloat16 *>(out);
   if (x_f32)
-    rmsnorm_kernel<true><<<blocks_for(rows), kWarps * 32, 0, st>>>(x, g, o, d, eps, seq_len, cap, rows);
+    rmsnorm_kernel<true><<<blocks_for(rows), kWarps * 32, 0, st>>>(x, g, o, d, eps, seq_len, cap,
+                                                                    rows, split ? 1 : 0);
   else
-    rmsnorm_kernel<false><<<blocks_for(rows), kWarps * 32, 0, st>>>(x, g, o, d, eps, seq_len, cap, rows);
+    rmsnorm_kernel<false><<<blocks_for(rows), kWarps * 32, 0, st>>>(x, g, o, d, eps, seq_len, cap,
+                                                                     rows, split ? 1 : 0);
   return cudaGetLastError();
 }
 

@@ -4,9 +4,10 @@
 
 namespace cc {
 
-// out bf16 [rows][d] = x * gain / sqrt(mean(x^2) + eps); x bf16 or fp32 [rows][d]
+// out bf16 [rows][d] = x * gain / sqrt(mean(x^2) + eps); x bf16 or fp32 [rows][d].
+// split: out rows are [hi | lo] bf16 [rows][2d] with hi + lo ~= the fp32 value.
 cudaError_t launch_rmsnorm(const void *x, bool x_f32, const void *gain, void *out, int d, float eps,
-                           const int32_t *seq_len, int cap, int rows, cudaStream_t st);
+                           const int32_t *seq_len, int cap, int rows, bool split, cudaStream_t st);
 // h fp32 [rows][d] = embed[tokens[row]]
 cudaError_t launch_embed(const void *embed, const int32_t *tokens, float *h, int d, int vocab,
                          const int32_t *seq_len, int cap, int rows, unsigned *status,
