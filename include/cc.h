@@ -4,7 +4,7 @@
  * One memory refresh (Algorithm DoMemRefresh) is three calls on one CUDA
  * stream:
  *   1. cc_score_layer / cc_score_full: the counter-causal surprise score of
- *      every cached slot (Sec. 3.1, Eq. 3 and the logit score it uses);
+ *      every cached slot (Sec. 3.1, Eq. 5 and the logit score it uses);
  *   2. cc_select_keep: the keep-set, the J highest scores (argsort, keep
  *      sigma[1:J]);
  *   3. cc_compact_kv: K' <- (K' (+) K)_sigma[1:J], V', X likewise, in place.
@@ -49,11 +49,11 @@ typedef enum {
 } cc_status;
 
 /* Score definition.  Sec. 3.1 takes the logit of the row's own token x_i as
- * the score; Eq. 3 defines surprise as 1 - P(x_i | x_{i+1:t}).  Both are
+ * the score; Eq. 5 defines surprise as 1 - P(x_i | x_{i+1:t}).  Both are
  * returned with the sign that makes "more surprising" rank higher. */
 typedef enum {
   CC_SCORE_LOGIT = 0,   /* score_i = -z_i[x_i], z_i = final-norm(h_i) W_U^T      */
-  CC_SCORE_LOGPROB = 1  /* score_i = -log softmax(z_i)[x_i] (same order as Eq. 3) */
+  CC_SCORE_LOGPROB = 1  /* score_i = -log softmax(z_i)[x_i] (same order as Eq. 5) */
 } cc_score_mode;
 
 /* Decoder shape (Llama/Qwen pre-norm block: RMSNorm, GQA attention with

@@ -15,7 +15,7 @@ Conventions (readings of the paper where it is silent or ambiguous):
   * the score of row i is -(logit of its own token x_i) in the default
     "logit" mode (Sec. 3.1 takes the logit of x_i as the score; keeping the
     highest-surprise tokens means a low logit must rank high), or
-    -log P(x_i | x_{i+1:t}) in "logprob" mode (Eq. 3 ranks the same as 1 - P);
+    -log P(x_i | x_{i+1:t}) in "logprob" mode (Eq. 5 ranks the same as 1 - P);
   * the last cached slot gets +inf (maximum surprise, Sec. 3.1);
   * a row with no later key (the last one) has attention output 0;
   * layer = Llama/Qwen pre-norm block: RMSNorm -> counter-causal attention ->

@@ -92,6 +92,7 @@ _SIGS = {
     "cc_timing_collect": (ctypes.c_int, [ctypes.POINTER(ctypes.c_int32),
                                          ctypes.POINTER(ctypes.c_double)]),
     "cc_kernel_name": (ctypes.c_char_p, [ctypes.c_int32]),
+    "cc_debug_withhold_compact_unit": (ctypes.c_int, [ctypes.c_int32]),
 }
 KERNEL_COUNT = 13
 
@@ -288,6 +289,12 @@ def cc_timing_collect() -> dict:
     _check(lib.cc_timing_collect(counts, total), "cc_timing_collect")
     return {lib.cc_kernel_name(k).decode(): (int(counts[k]), float(total[k]))
             for k in range(KERNEL_COUNT) if counts[k]}
+
+
+def cc_debug_withhold_compact_unit(unit: int):
+    """Test hook: the next cc_compact_kv runs with `unit` never publishing its flag."""
+    _check(load_library().cc_debug_withhold_compact_unit(int(unit)),
+           "cc_debug_withhold_compact_unit")
 
 
 def alloc_workspace(nbytes: int, device="cuda") -> torch.Tensor:

@@ -427,6 +427,8 @@ struct CompactPlan {
   size_t ws_bytes;
 };
 
+int g_withhold_unit = -1;   // cc_debug_withhold_compact_unit: consumed by the next cc_compact_kv
+
 cc_status compact_plan(const cc_model_cfg *c, const cc_kv_cache *kv, CompactPlan &plan) {
   cc_status s = check_cfg(c);
   if (s != CC_OK) return s;
@@ -435,6 +437,7 @@ cc_status compact_plan(const cc_model_cfg *c, const cc_kv_cache *kv, CompactPlan
     return CC_ERR_INVALID_ARG;
   CompactParams &p = plan.p;
   memset(&p, 0, sizeof(p));
+  p.withhold_unit = -1;
   p.batch = kv->batch;
   p.cap = kv->cap;
   int n = 0, units = 0;
@@ -537,6 +540,8 @@ cc_status cc_compact_kv(const cc_model_cfg *cfg, const cc_kv_cache *cache,
   plan.p.ticket = reinterpret_cast<unsigned *>(ws);
   plan.p.flags = reinterpret_cast<unsigned *>(reinterpret_cast<uint8_t *>(ws) + 256);
   plan.p.status = dev->status;
+  plan.p.withhold_unit = g_withhold_unit;
+  g_withhold_unit = -1;
   TimedScope t(CC_KERNEL_COMPACT, st);
   CC_TRY(launch_compact(plan.p, dev->sms * 3, st));
   return CC_OK;
@@ -641,6 +646,11 @@ cc_status cc_timing_collect(int32_t *counts, double *total_ms) {
   }
   g_timing.recs.clear();
   return st;
+}
+
+cc_status cc_debug_withhold_compact_unit(int32_t unit) {
+  g_withhold_unit = unit;
+  return CC_OK;
 }
 
 const char *cc_kernel_name(int32_t kind) {

@@ -7,8 +7,9 @@
 // consecutive positions, row r = position * G + head, so that P*G <= 256
 // rows form two M=128 MMA tiles that share every K/V tile loaded (a GQA
 // group is served by one K/V stream).  Key tiles of 128 slots run from the
-// one holding slot p0+1 to the one holding slot n-1: whole tiles at or
-// below the diagonal are never loaded.
+// one holding slot n-1 down to the one holding slot p0+1: whole tiles at or
+// below the diagonal are never loaded, and units running at the same time
+// sweep the same keys in step (L2 reuse when K/V exceed L2).
 //
 //   warps 0..3, 4..7  softmax of M-half 0 / 1 (one row per thread): S from
 //                     TMEM, mask, online softmax (log2 domain, lazy rescale),
@@ -49,7 +50,7 @@ struct AttnSmem {
 };
 
 template <int DH>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __maxnreg__(200)
     attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                 const __grid_constant__ CUtensorMap tmV, const __grid_constant__ AttnParams p) {
   using L = AttnSmem<DH>;
@@ -134,7 +135,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     (int)row_base + p0);
     }
     for (int it = 0; it < ntiles; ++it) {
-      const int t = t0 + it, s = it % KST;
+      const int t = t1 - it, s = it % KST;   // key tiles from the sequence end downwards
       const uint32_t ph = (it / KST) & 1;
       const int krow = (int)row_base + t * BKV;
       int ok = 1;
@@ -198,7 +199,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         umma_commit(&k_empty[0]);
       }
       for (int it = 0; ok && it < ntiles; ++it) {
-        const int t = t0 + it, s = it % KST;
+        const int t = t1 - it, s = it % KST;
         const uint32_t ph = (it / KST) & 1;
         if (!(ok = mbar_wait(&v_full[s], ph, abort_flag, p.status))) break;
         if (t == t1 && n - t * BKV < BKV)
@@ -241,10 +242,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t s_t = tmem + lane_off + h * 128;
     const uint32_t o_t = tmem + lane_off + 256 + h * DH;
     const float sl2 = p.scale_log2;
-    float m_used = -INFINITY, l = 0.f;
+    const float thr = 8.0f / sl2;   // lazy-rescale threshold: 2^8 in exp2 space, in raw units
+    const float2 sl2v = make_float2(sl2, sl2);
+    float m_used = -INFINITY, l = 0.f;   // m_used: reference max of the raw scores
     bool ok = true;
     for (int it = 0; it < ntiles; ++it) {
-      const int j0 = (t0 + it) * BKV;
+      const int j0 = (t1 - it) * BKV;
       if (!(ok = mbar_wait(&s_ready[h], it & 1, abort_flag, p.status))) break;
       tc_fence_after();
       uint32_t sr[128];
@@ -261,26 +264,22 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int hi = n - j0;         // keep c < hi
 #pragma unroll
         for (int c = 0; c < 128; ++c) {
-          float x = (c > lo && c < hi) ? __uint_as_float(sr[c]) * sl2 : -INFINITY;
+          float x = (c > lo && c < hi) ? __uint_as_float(sr[c]) : -INFINITY;
           sr[c] = __float_as_uint(x);
           mt = fmaxf(mt, x);
         }
       } else {
 #pragma unroll
-        for (int c = 0; c < 128; ++c) {
-          float x = __uint_as_float(sr[c]) * sl2;
-          sr[c] = __float_as_uint(x);
-          mt = fmaxf(mt, x);
-        }
+        for (int c = 0; c < 128; ++c) mt = fmaxf(mt, __uint_as_float(sr[c]));
       }
       // lazy rescaling: move the reference max only when it grows by more
-      // than 2^8, so exp2 stays <= 256 and O is rarely touched
+      // than 2^8 in exp2 space, so p <= 256 and O is rarely touched
       const float m_new = fmaxf(m_used, mt);
-      const bool bump = m_new > m_used + 8.0f;        // also true for -inf -> finite
+      const bool bump = m_new > m_used + thr;          // also true for -inf -> finite
       const bool rescale_o = bump && it > 0 && l > 0.f;
       float factor = 1.f;
       if (bump) {
-        factor = fast_exp2(m_used - m_new);           // 0 when m_used = -inf
+        factor = fast_exp2((m_used - m_new) * sl2);   // 0 when m_used = -inf
         l *= factor;
         m_used = m_new;
       }
@@ -297,22 +296,25 @@ __global__ void __launch_bounds__(kThreads, 1)
           tmem_st32(o_t + c, o);
         }
       }
-      const float mref = (m_used == -INFINITY) ? 0.f : m_used;
-      float lsum = 0.f;
+      // p = 2^(s*sl2 - m*sl2): one packed FMA per pair, bf16 P into TMEM over S,
+      // the row sum l in fp32
+      const float nm = (m_used == -INFINITY) ? 0.f : -m_used * sl2;
+      const float2 nmv = make_float2(nm, nm);
+      float2 lsum = make_float2(0.f, 0.f);
 #pragma unroll
       for (int c0 = 0; c0 < 128; c0 += 32) {
         uint32_t pk[16];
 #pragma unroll
         for (int k = 0; k < 32; k += 2) {
-          float e0 = fast_exp2(__uint_as_float(sr[c0 + k]) - mref);
-          float e1 = fast_exp2(__uint_as_float(sr[c0 + k + 1]) - mref);
-          __nv_bfloat162 v2 = __floats2bfloat162_rn(e0, e1);
-          lsum += __low2float(v2) + __high2float(v2);
-          pk[k / 2] = *reinterpret_cast<uint32_t *>(&v2);
+          const float2 y = __ffma2_rn(make_float2(__uint_as_float(sr[c0 + k]),
+                                                  __uint_as_float(sr[c0 + k + 1])), sl2v, nmv);
+          const float2 e = make_float2(fast_exp2(y.x), fast_exp2(y.y));
+          pk[k / 2] = pack_bf16x2(e.x, e.y);
+          lsum = __fadd2_rn(lsum, e);
         }
         tmem_st16(s_t + c0 / 2, pk);
       }
-      l += lsum;
+      l += lsum.x + lsum.y;
       tmem_st_wait();
       tc_fence_before();
       mbar_arrive(&p_ready[h]);

@@ -149,7 +149,7 @@ __global__ void __launch_bounds__(kThreads)
     __syncthreads();
     // ---- 2. publish; 3. wait for lower overlapping units
     if (tid == 0) {
-      st_release(&p.flags[t], 1u);
+      if (t != p.withhold_unit) st_release(&p.flags[t], 1u);
       int go = 1;
       if (work && c > 0) {
         // highest lower chunk whose first source lies below our last destination

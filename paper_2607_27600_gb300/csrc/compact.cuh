@@ -24,6 +24,7 @@ struct CompactParams {
   unsigned *ticket;           // zeroed before launch
   unsigned *flags;            // [total_units], zeroed before launch
   unsigned *status;
+  int withhold_unit;          // test hook: this unit never publishes its flag (-1: none)
   CompactArray arr[kMaxCompactArrays];
 };
 
