@@ -182,6 +182,9 @@ cc_status cc_compact_kv_static(const cc_model_cfg *cfg, const cc_kv_cache *cache
  * Returns CC_ERR_CUDA if the stream itself reports a CUDA error. */
 cc_status cc_get_status(void *stream);
 const char *cc_status_str(cc_status s);
+/* Text of the last CUDA error behind a CC_ERR_CUDA returned on this host
+ * thread (the failing call and the CUDA error name); "" if none. */
+const char *cc_last_error(void);
 
 #ifdef __cplusplus
 }

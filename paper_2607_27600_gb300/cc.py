@@ -31,7 +31,8 @@ SCORE_LOGPROB = 1
 class CCError(RuntimeError):
     def __init__(self, code: int, where: str):
         self.code = code
-        super().__init__(f"{where}: {STATUS_NAMES.get(code, code)} ({cc_status_str(code)})")
+        extra = f" [{cc_last_error()}]" if code == CC_ERR_CUDA else ""
+        super().__init__(f"{where}: {STATUS_NAMES.get(code, code)} ({cc_status_str(code)}){extra}")
 
 
 class cc_model_cfg(ctypes.Structure):
@@ -83,6 +84,7 @@ _SIGS = {
                                             ctypes.c_void_p, ctypes.c_void_p]),
     "cc_get_status": (ctypes.c_int, [ctypes.c_void_p]),
     "cc_status_str": (ctypes.c_char_p, [ctypes.c_int]),
+    "cc_last_error": (ctypes.c_char_p, []),
     "cc_linear_f32": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,
                                      ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,
                                      ctypes.c_void_p]),
@@ -200,6 +202,10 @@ def _cfg(cfg):
 
 def cc_status_str(code: int) -> str:
     return load_library().cc_status_str(int(code)).decode()
+
+
+def cc_last_error() -> str:
+    return load_library().cc_last_error().decode()
 
 
 def cc_score_workspace_size(cfg, batch: int, cap: int, mode: int = SCORE_LOGIT) -> int:

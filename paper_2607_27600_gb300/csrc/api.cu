@@ -201,10 +201,28 @@ void rope_turns(const cc_model_cfg *c, unsigned long long *turns) {
   }
 }
 
+thread_local char g_last_error[256] = "";
+
+cc_status cuda_fail(cudaError_t e, const char *what) {
+  snprintf(g_last_error, sizeof(g_last_error), "%s: %s (%s)", what, cudaGetErrorName(e),
+           cudaGetErrorString(e));
+  return CC_ERR_CUDA;
+}
+
+cc_status tmap_fail() {
+  snprintf(g_last_error, sizeof(g_last_error), "cuTensorMapEncodeTiled failed");
+  return CC_ERR_CUDA;
+}
+
+cc_status device_fail() {
+  cudaError_t e = cudaGetLastError();
+  return cuda_fail(e, "device query (cudaGetDevice / cudaGetSymbolAddress)");
+}
+
 #define CC_TRY(expr)                                         \
   do {                                                       \
     cudaError_t e_ = (expr);                                 \
-    if (e_ != cudaSuccess) return CC_ERR_CUDA;               \
+    if (e_ != cudaSuccess) return cuda_fail(e_, #expr);      \
   } while (0)
 
 struct Gemm {
@@ -219,10 +237,10 @@ cc_status gemm_setup(Gemm &g, int epi, const void *A, int K, const void *W, cons
                      bool a_split = false) {
   const uint64_t R = (uint64_t)batch * cap;
   const int bn = gemm_block_n(epi);
-  if (!tmap_rows(&g.a, A, R, a_split ? 2 * K : K, 128)) return CC_ERR_CUDA;
-  if (!tmap_rows(&g.b, W, N, K, epi == EPI_SWIGLU ? 128 : 256)) return CC_ERR_CUDA;
+  if (!tmap_rows(&g.a, A, R, a_split ? 2 * K : K, 128)) return tmap_fail();
+  if (!tmap_rows(&g.b, W, N, K, epi == EPI_SWIGLU ? 128 : 256)) return tmap_fail();
   if (epi == EPI_SWIGLU) {
-    if (!tmap_rows(&g.b2, W2, N, K, 128)) return CC_ERR_CUDA;
+    if (!tmap_rows(&g.b2, W2, N, K, 128)) return tmap_fail();
   } else {
     g.b2 = g.b;
   }
@@ -256,14 +274,14 @@ cc_status run_attention(const cc_model_cfg *c, const void *q, const void *k, con
     const uint64_t dims[3] = {(uint64_t)dh, (uint64_t)c->n_q_heads, R};
     const uint64_t strides[2] = {(uint64_t)dh * 2, (uint64_t)c->n_q_heads * dh * 2};
     const uint32_t box[3] = {64, (uint32_t)G, (uint32_t)P};
-    if (!make_tmap(&tq, q, 3, dims, strides, box)) return CC_ERR_CUDA;
+    if (!make_tmap(&tq, q, 3, dims, strides, box)) return tmap_fail();
   }
   {
     const uint64_t dims[3] = {(uint64_t)dh, (uint64_t)c->n_kv_heads, R};
     const uint64_t strides[2] = {(uint64_t)dh * 2, (uint64_t)c->n_kv_heads * dh * 2};
     const uint32_t box[3] = {64, 1, 128};
-    if (!make_tmap(&tk, k, 3, dims, strides, box)) return CC_ERR_CUDA;
-    if (!make_tmap(&tv, v, 3, dims, strides, box)) return CC_ERR_CUDA;
+    if (!make_tmap(&tk, k, 3, dims, strides, box)) return tmap_fail();
+    if (!make_tmap(&tv, v, 3, dims, strides, box)) return tmap_fail();
   }
   AttnParams p{};
   p.batch = batch;
@@ -320,7 +338,7 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
   cc_status s = check_score_args(c, w, kv, mode, scores, ws, ws_bytes, full);
   if (s != CC_OK) return s;
   DevState *dev;
-  if (!dev_state(&dev)) return CC_ERR_CUDA;
+  if (!dev_state(&dev)) return device_fail();
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   const int batch = kv->batch, cap = kv->cap, rows = batch * cap;
   const int d = c->d_model, qd = c->n_q_heads * c->head_dim, f = c->d_ff;
@@ -507,7 +525,7 @@ cc_status cc_select_keep(const float *scores, const int32_t *seq_len, int32_t ba
       n_sink < 0)
     return CC_ERR_INVALID_ARG;
   DevState *dev;
-  if (!dev_state(&dev)) return CC_ERR_CUDA;
+  if (!dev_state(&dev)) return device_fail();
   TimedScope t(CC_KERNEL_SELECT, reinterpret_cast<cudaStream_t>(stream));
   CC_TRY(launch_select(scores, seq_len, batch, cap, budget, n_sink, keep_idx, keep_count,
                        dev->status, reinterpret_cast<cudaStream_t>(stream)));
@@ -531,7 +549,7 @@ cc_status cc_compact_kv(const cc_model_cfg *cfg, const cc_kv_cache *cache,
   if (!keep_idx || !keep_count) return CC_ERR_INVALID_ARG;
   if (!ws || !aligned16(ws) || ws_bytes < plan.ws_bytes) return CC_ERR_WORKSPACE;
   DevState *dev;
-  if (!dev_state(&dev)) return CC_ERR_CUDA;
+  if (!dev_state(&dev)) return device_fail();
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   CC_TRY(cudaMemsetAsync(ws, 0, plan.ws_bytes, st));
   plan.p.keep_idx = keep_idx;
@@ -549,7 +567,7 @@ cc_status cc_compact_kv(const cc_model_cfg *cfg, const cc_kv_cache *cache,
 
 cc_status cc_get_status(void *stream) {
   DevState *dev;
-  if (!dev_state(&dev)) return CC_ERR_CUDA;
+  if (!dev_state(&dev)) return device_fail();
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   if (cudaStreamSynchronize(st) != cudaSuccess) return CC_ERR_CUDA;
   unsigned v = 0;
@@ -560,6 +578,8 @@ cc_status cc_get_status(void *stream) {
     return CC_ERR_CUDA;
   return static_cast<cc_status>(v);
 }
+
+const char *cc_last_error(void) { return g_last_error; }
 
 const char *cc_status_str(cc_status s) {
   switch (s) {
@@ -582,7 +602,7 @@ cc_status cc_linear_f32(const void *x, const void *w, float *y, int32_t rows, in
   if (!x || !w || !y || rows < 1 || n < 1 || k < 1 || n % 32 || k % 8) return CC_ERR_INVALID_ARG;
   if (!aligned16(x) || !aligned16(w) || !aligned16(y)) return CC_ERR_INVALID_ARG;
   DevState *dev;
-  if (!dev_state(&dev)) return CC_ERR_CUDA;
+  if (!dev_state(&dev)) return device_fail();
   Gemm g;
   cc_status s = gemm_setup(g, EPI_F32, x, k, w, nullptr, n, 1, rows, nullptr, dev->status);
   if (s != CC_OK) return s;
@@ -603,7 +623,7 @@ cc_status cc_counter_causal_attention(const void *q, const void *k, const void *
   if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(out)) return CC_ERR_INVALID_ARG;
   if ((uint64_t)batch * cap >= (1ull << 31)) return CC_ERR_UNSUPPORTED;
   DevState *dev;
-  if (!dev_state(&dev)) return CC_ERR_CUDA;
+  if (!dev_state(&dev)) return device_fail();
   cc_model_cfg c{};
   c.n_q_heads = n_q_heads;
   c.n_kv_heads = n_kv_heads;
