@@ -53,7 +53,14 @@ typedef enum {
  * returned with the sign that makes "more surprising" rank higher. */
 typedef enum {
   CC_SCORE_LOGIT = 0,   /* score_i = -z_i[x_i], z_i = final-norm(h_i) W_U^T      */
-  CC_SCORE_LOGPROB = 1  /* score_i = -log softmax(z_i)[x_i] (same order as Eq. 5) */
+  CC_SCORE_LOGPROB = 1, /* score_i = -log softmax(z_i)[x_i] (same order as Eq. 5) */
+  /* Flag, OR-ed into the mode, full pass only: carry every GEMM activation
+   * (normalised inputs, attention output, SwiGLU output) as a bf16 pair
+   * hi + lo (~2^-17 relative) instead of one bf16 value; each projection
+   * runs its K loop twice.  Deep random-weight models drift from the exact
+   * result over depth with bf16 activations; this halves that drift at
+   * about 1.7x the cost of the pass.  Queries and P stay bf16. */
+  CC_SCORE_PRECISE = 0x100
 } cc_score_mode;
 
 /* Decoder shape (Llama/Qwen pre-norm block: RMSNorm, GQA attention with
@@ -118,6 +125,8 @@ typedef struct {
  * cc_score_full -- full pass: embedding of tokens, every layer l with fresh
  * queries over k[l], v[l] (reused, not recomputed), final norm, head.
  */
+/* Workspace bytes for either pass in `mode` (with CC_SCORE_PRECISE: the
+ * larger full-pass layout). */
 size_t cc_score_workspace_size(const cc_model_cfg *cfg, int32_t batch, int32_t cap,
                                cc_score_mode mode);
 cc_status cc_score_layer(const cc_model_cfg *cfg, const cc_model_weights *w,

@@ -26,6 +26,7 @@ STATUS_NAMES = {0: "CC_OK", 1: "CC_ERR_INVALID_ARG", 2: "CC_ERR_CUDA", 3: "CC_ER
                 7: "CC_ERR_DEVICE_ARG"}
 SCORE_LOGIT = 0
 SCORE_LOGPROB = 1
+SCORE_PRECISE = 0x100   # flag: hi + lo bf16 GEMM activations in the full pass
 
 
 class CCError(RuntimeError):

@@ -168,8 +168,9 @@ struct ScoreWs {
   int n_vtiles;
 };
 
-// The full pass carries the GEMM activations (normalised inputs, attention
-// output, SwiGLU output) as [hi | lo] bf16 pairs: split = 2 copies per row.
+// With CC_SCORE_PRECISE the full pass carries the GEMM activations
+// (normalised inputs, attention output, SwiGLU output) as [hi | lo] bf16
+// pairs: split = 2 copies per row.
 ScoreWs score_layout(const cc_model_cfg *c, int batch, int cap, cc_score_mode mode, bool full) {
   ScoreWs w{};
   const size_t R = (size_t)batch * cap;
@@ -183,7 +184,7 @@ ScoreWs score_layout(const cc_model_cfg *c, int batch, int cap, cc_score_mode mo
   w.h = take(R * d * 4);
   w.act = take(R * f * 2 * split);
   w.n_vtiles = (c->vocab + 255) / 256;
-  if (mode == CC_SCORE_LOGPROB) {
+  if ((mode & 0xFF) == CC_SCORE_LOGPROB) {
     w.part = take(R * w.n_vtiles * 8);
     w.ztgt = take(R * 4);
   }
@@ -309,7 +310,10 @@ cc_status check_score_args(const cc_model_cfg *c, const cc_model_weights *w, con
   if (s != CC_OK) return s;
   if (!w || !kv || !scores || !w->layers || !w->final_norm || !w->lm_head || !kv->k || !kv->v)
     return CC_ERR_INVALID_ARG;
-  if (mode != CC_SCORE_LOGIT && mode != CC_SCORE_LOGPROB) return CC_ERR_INVALID_ARG;
+  const int base_mode = mode & 0xFF;
+  if ((base_mode != CC_SCORE_LOGIT && base_mode != CC_SCORE_LOGPROB) ||
+      (mode & ~(0xFF | CC_SCORE_PRECISE)))
+    return CC_ERR_INVALID_ARG;
   if (kv->batch < 1 || kv->cap < 1 || !kv->seq_len || !kv->tokens || !kv->pos)
     return CC_ERR_INVALID_ARG;
   if (kv->batch > gemm_max_batch()) return CC_ERR_UNSUPPORTED;
@@ -327,7 +331,7 @@ cc_status check_score_args(const cc_model_cfg *c, const cc_model_weights *w, con
   const void *ptrs[] = {w->final_norm, w->lm_head, ws, kv->h_last, full ? w->embed : nullptr};
   for (const void *p : ptrs)
     if (p && !aligned16(p)) return CC_ERR_INVALID_ARG;
-  if (!ws || ws_bytes < score_layout(c, kv->batch, kv->cap, mode, full).total)
+  if (!ws || ws_bytes < score_layout(c, kv->batch, kv->cap, mode, full && (mode & CC_SCORE_PRECISE)).total)
     return CC_ERR_WORKSPACE;
   return CC_OK;
 }
@@ -342,8 +346,9 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   const int batch = kv->batch, cap = kv->cap, rows = batch * cap;
   const int d = c->d_model, qd = c->n_q_heads * c->head_dim, f = c->d_ff;
-  const ScoreWs L = score_layout(c, batch, cap, mode, full);
-  const bool split = full;   // [hi | lo] activations in the full pass
+  const bool split = full && (mode & CC_SCORE_PRECISE);   // [hi | lo] GEMM activations
+  const ScoreWs L = score_layout(c, batch, cap, mode, split);
+  const bool logit = (mode & 0xFF) == CC_SCORE_LOGIT;
   uint8_t *wsb = reinterpret_cast<uint8_t *>(ws);
   void *xn = wsb + L.xn, *q = wsb + L.q, *o = wsb + L.o, *act = wsb + L.act;
   float *h = reinterpret_cast<float *>(wsb + L.h);
@@ -413,7 +418,7 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
     if ((s = run_gemm(gd, EPI_RESID_F32, CC_KERNEL_GEMM_DOWN, dev->sms, st)) != CC_OK) return s;
   }
   // head
-  if (mode == CC_SCORE_LOGIT) {
+  if (logit) {
     TimedScope t(CC_KERNEL_HEAD_LOGIT, st);
     CC_TRY(launch_head_logit(h, w->final_norm, w->lm_head, kv->tokens, scores, d, c->vocab,
                              c->rms_eps, sl, cap, rows, status, st));
@@ -495,7 +500,7 @@ extern "C" {
 size_t cc_score_workspace_size(const cc_model_cfg *cfg, int32_t batch, int32_t cap,
                                cc_score_mode mode) {
   if (check_cfg(cfg) != CC_OK || batch < 1 || cap < 1) return 0;
-  return score_layout(cfg, batch, cap, mode, true).total;   // enough for either pass
+  return score_layout(cfg, batch, cap, mode, (mode & CC_SCORE_PRECISE) != 0).total;
 }
 
 cc_status cc_score_layer(const cc_model_cfg *cfg, const cc_model_weights *w,

@@ -18,6 +18,7 @@
 //                     zeroes V rows past the sequence end in the last tile
 //   warp 9            TMEM owner + tcgen05.mma issuer:
 //                     S_h = Q_h K^T (SS),  O_h += P_h V (TS, P from TMEM)
+//   warps 10, 11      idle (complete the third warpgroup)
 //
 // TMEM columns: S0 [0,128)  S1 [128,256)  O0 [256,256+DH)  O1 [256+DH, 256+2DH)
 #include "attn.cuh"
@@ -28,7 +29,13 @@ namespace {
 
 constexpr int BKV = 128;        // keys per tile
 constexpr int KST = 2;          // K and V pipeline stages
-constexpr int kThreads = 320;
+constexpr int kThreads = 384;   // 3 warpgroups: softmax 0, softmax 1, producer/MMA
+// Register split after launch (setmaxnreg): the block is launched with 168
+// registers per thread (64512 in all); the producer/MMA warpgroup drops to
+// 64 and the two softmax warpgroups rise to 216: 2*128*216 + 128*64 = 63488.
+constexpr int kRegsLaunch = 168, kRegsSoftmax = 216, kRegsProducer = 64;
+static_assert(2 * 128 * kRegsSoftmax + 128 * kRegsProducer <= kThreads * kRegsLaunch,
+              "register split exceeds the launch allocation");
 
 // 2^x by the PTX ex2.approx instruction (2 ulp; 2^-inf = 0).
 CC_DEV float fast_exp2(float x) {
@@ -122,8 +129,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-
-  if (warp == 8) {
+  if (warp >= 8) {
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegsProducer));
+    if (warp == 8) {
     // ------------------------------------------------------------ producer
     if (lane == 0) {
       tma_prefetch_desc(&tmQ);
@@ -171,7 +179,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) mbar_arrive(v_fixed);
       }
     }
-  } else if (warp == 9) {
+    } else if (warp == 9) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
       constexpr uint32_t idesc_qk = make_idesc_bf16(128, BKV, 0, 0);
@@ -231,7 +239,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
     }
+    }
   } else {
+    asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kRegsSoftmax));
     // ------------------------------------------------------------ softmax
     const int h = warp >> 2, q = warp & 3;
     const int R = h * 128 + q * 32 + lane;              // unit row
@@ -283,19 +293,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         l *= factor;
         m_used = m_new;
       }
-      if (__any_sync(0xFFFFFFFFu, rescale_o)) {
-        // O still holds the previous tiles' sum (S_ready implies the last PV is done)
-        const float f = rescale_o ? factor : 1.f;
-#pragma unroll 1
-        for (int c = 0; c < DH; c += 32) {
-          uint32_t o[32];
-          tmem_ld32(o_t + c, o);
-          tmem_ld_wait();
-#pragma unroll
-          for (int k = 0; k < 32; ++k) o[k] = __float_as_uint(__uint_as_float(o[k]) * f);
-          tmem_st32(o_t + c, o);
-        }
-      }
       // p = 2^(s*sl2 - m*sl2): one packed FMA per pair, bf16 P into TMEM over S,
       // the row sum l in fp32
       const float nm = (m_used == -INFINITY) ? 0.f : -m_used * sl2;
@@ -315,6 +312,20 @@ __global__ void __launch_bounds__(kThreads, 1)
         tmem_st16(s_t + c0 / 2, pk);
       }
       l += lsum.x + lsum.y;
+      // after P is written, so the S registers are free for the O rows
+      if (__any_sync(0xFFFFFFFFu, rescale_o)) {
+        // O still holds the previous tiles' sum (S_ready implies the last PV is done)
+        const float f = rescale_o ? factor : 1.f;
+#pragma unroll 1
+        for (int c = 0; c < DH; c += 32) {
+          uint32_t o[32];
+          tmem_ld32(o_t + c, o);
+          tmem_ld_wait();
+#pragma unroll
+          for (int k = 0; k < 32; ++k) o[k] = __float_as_uint(__uint_as_float(o[k]) * f);
+          tmem_st32(o_t + c, o);
+        }
+      }
       tmem_st_wait();
       tc_fence_before();
       mbar_arrive(&p_ready[h]);
