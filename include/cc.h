@@ -169,12 +169,13 @@ cc_status cc_compact_kv(const cc_model_cfg *cfg, const cc_kv_cache *cache,
  * example a serving loop that has handed the whole device pool to the KV
  * cache, or a runtime that forbids device allocation on its refresh path
  * (cudaMalloc may block and synchronise the device).  Its scratch (a ticket
- * counter and one flag per work unit) lives in a fixed 1 MiB array in the
+ * counter, one flag per work unit and a table of which work units read
+ * each destination chunk) lives in a fixed 1 MiB array in the
  * library's device memory, which every GPU that loads the library holds
  * until the process exits.  The call allocates nothing.
- *   - A cache needing more than 1 MiB of scratch (more than 262080 work
- *     units; cc_compact_workspace_size() - 256 bytes / 4) is rejected with
- *     CC_ERR_WORKSPACE before anything is enqueued.
+ *   - A cache needing more than 1 MiB of scratch (cc_compact_workspace_size()
+ *     above 1 MiB) is rejected with CC_ERR_WORKSPACE before anything is
+ *     enqueued.
  *   - The first call on a device looks up the array's device address (with
  *     that device current); make that first call before any stream capture.
  *   - All calls on a device share the array and each call clears it first

@@ -447,7 +447,8 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
 // compaction plan: arrays and unit counts
 struct CompactPlan {
   CompactParams p;
-  size_t ws_bytes;
+  size_t flags_bytes;   // ticket + flags (zeroed per call)
+  size_t ws_bytes;      // + readers table (filled with -1 per call)
 };
 
 int g_withhold_unit = -1;   // cc_debug_withhold_compact_unit: consumed by the next cc_compact_kv
@@ -464,6 +465,14 @@ cc_status compact_plan(const cc_model_cfg *c, const cc_kv_cache *kv, CompactPlan
   p.batch = kv->batch;
   p.cap = kv->cap;
   int n = 0, units = 0;
+  auto class_of = [&](int rows) -> int {
+    for (int c = 0; c < p.n_classes; ++c)
+      if (p.class_rows[c] == rows) return c;
+    if (p.n_classes >= kMaxDepClasses) return -1;
+    p.class_rows[p.n_classes] = rows;
+    p.class_chunks[p.n_classes] = (kv->cap + rows - 1) / rows;
+    return p.n_classes++;
+  };
   auto add = [&](void *base, int row_bytes, bool bulk) -> bool {
     if (!base) return true;
     if (n >= kMaxCompactArrays || !aligned16(base)) return false;
@@ -471,22 +480,26 @@ cc_status compact_plan(const cc_model_cfg *c, const cc_kv_cache *kv, CompactPlan
     A.base = base;
     A.row_bytes = row_bytes;
     A.bulk = bulk ? 1 : 0;
-    A.rows_per_chunk = bulk ? (row_bytes <= kStageBytes ? kStageBytes / row_bytes : 0) : 4096;
+    A.rows_per_chunk = bulk ? (row_bytes <= kStageBytes ? kStageBytes / row_bytes : 0)
+                            : kStageBytes / 4;
     if (A.rows_per_chunk < 1) return false;
     A.n_chunks = (kv->cap + A.rows_per_chunk - 1) / A.rows_per_chunk;
     A.unit_base = units;
+    A.dep_class = class_of(A.rows_per_chunk);
+    if (A.dep_class < 0) return false;
     units += kv->batch * A.n_chunks;
     return true;
   };
-  const int kv_row = c->n_kv_heads * c->head_dim * 2;
-  for (int l = 0; l < c->n_layers; ++l) {
-    if (!add(kv->k[l], kv_row, true) || !add(kv->v[l], kv_row, true)) return CC_ERR_UNSUPPORTED;
-  }
-  if (!add(kv->h_last, c->d_model * 2, true)) return CC_ERR_UNSUPPORTED;
-  if (!add(kv->tokens, 4, false) || !add(kv->pos, 4, false)) return CC_ERR_INVALID_ARG;
   p.n_arrays = n;
   p.total_units = units;
-  plan.ws_bytes = 256 + align256((size_t)units * 4);
+  // workspace: ticket | flags | readers table
+  size_t deps_entries = 0;
+  for (int c = 0; c < p.n_classes; ++c) {
+    p.class_offset[c] = (long long)deps_entries;
+    deps_entries += (size_t)kv->batch * p.class_chunks[c];
+  }
+  plan.flags_bytes = 256 + align256((size_t)units * 4);
+  plan.ws_bytes = plan.flags_bytes + align256(deps_entries * sizeof(int2));
   return CC_OK;
 }
 
@@ -556,7 +569,10 @@ cc_status cc_compact_kv(const cc_model_cfg *cfg, const cc_kv_cache *cache,
   DevState *dev;
   if (!dev_state(&dev)) return device_fail();
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-  CC_TRY(cudaMemsetAsync(ws, 0, plan.ws_bytes, st));
+  CC_TRY(cudaMemsetAsync(ws, 0, plan.flags_bytes, st));
+  CC_TRY(cudaMemsetAsync(reinterpret_cast<uint8_t *>(ws) + plan.flags_bytes, 0xFF,
+                         plan.ws_bytes - plan.flags_bytes, st));
+  plan.p.deps = reinterpret_cast<int2 *>(reinterpret_cast<uint8_t *>(ws) + plan.flags_bytes);
   plan.p.keep_idx = keep_idx;
   plan.p.keep_count = keep_count;
   plan.p.seq_len = cache->seq_len;
@@ -566,7 +582,7 @@ cc_status cc_compact_kv(const cc_model_cfg *cfg, const cc_kv_cache *cache,
   plan.p.withhold_unit = g_withhold_unit;
   g_withhold_unit = -1;
   TimedScope t(CC_KERNEL_COMPACT, st);
-  CC_TRY(launch_compact(plan.p, dev->sms * 3, st));
+  CC_TRY(launch_compact(plan.p, dev->sms, st));
   return CC_OK;
 }
 
@@ -693,13 +709,14 @@ const char *cc_kernel_name(int32_t kind) {
 namespace cc {
 
 cc_status compact_plan_build(const cc_model_cfg *cfg, const cc_kv_cache *cache, CompactParams &p,
-                             size_t &scratch_bytes) {
+                             size_t &flags_bytes, size_t &scratch_bytes) {
   static CompactPlan plan;
   static std::mutex mu;
   std::lock_guard<std::mutex> lk(mu);
   cc_status s = compact_plan(cfg, cache, plan);
   if (s != CC_OK) return s;
   p = plan.p;
+  flags_bytes = plan.flags_bytes;
   scratch_bytes = plan.ws_bytes;
   return CC_OK;
 }

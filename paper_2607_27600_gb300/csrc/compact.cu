@@ -9,27 +9,31 @@
 // clobber the source of a LOWER destination k' (keep_idx[k'] = k).
 //
 // Work units are chunks of consecutive destination slots of one
-// (array, sequence), numbered so that chunks of an (array, sequence) come in
-// ascending order.  CTAs take unit tickets from an atomic counter (dispatch
-// order).  A unit
+// (array, sequence), numbered so that the chunks of an (array, sequence)
+// come in ascending order.  A unit
 //   1. reads all its source rows into shared memory (TMA bulk copies for
 //      rows of 16-byte multiples; plain loads for 4-byte rows),
 //   2. publishes "sources read" for its ticket (release),
-//   3. waits (acquire, bounded) until every lower unit of the same
-//      (array, sequence) whose source slots overlap its destination slots
-//      has published, and
-//   4. writes its destination rows.
-// A unit only waits on lower tickets, all held by CTAs already running, and
-// publishing never waits, so the scheme cannot deadlock.  Each element is
-// read once and written once; rows with keep_idx[k] == k (always a prefix)
-// are not moved.
+//   3. waits (acquire, bounded) until every lower unit that reads from its
+//      destination slots has published, and
+//   4. writes its destination rows (bulk stores).
+// Which lower units read from a chunk is found once per refresh by a small
+// pre-pass over keep_idx (deps_kernel): chunk u's readers are the chunks
+// holding the first and last k with keep_idx[k] in u.
+//
+// Tickets come from an atomic counter in dispatch order, a unit waits only
+// on lower tickets, and publishing never waits, so nothing can deadlock.
+// Each warp runs its own two-buffer pipeline: the loads of its next unit are
+// in flight while the current unit waits and stores.  Each element is read
+// once and written once; rows with keep_idx[k] == k are not moved.
 #include "compact.cuh"
 
 namespace cc {
 
 namespace {
 
-constexpr int kThreads = 128;
+constexpr int kWarps = 4;
+constexpr int kThreads = kWarps * 32;
 
 CC_DEV void st_release(unsigned *p, unsigned v) {
   asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
@@ -40,12 +44,12 @@ CC_DEV unsigned ld_acquire(const unsigned *p) {
   return v;
 }
 
-// Waits until flags[t] != 0; false after kWaitLimitNs (records CC_ERR_TIMEOUT).
+// Waits until *flag != 0; false after kWaitLimitNs (records CC_ERR_TIMEOUT).
 CC_DEV bool wait_flag(const unsigned *flag, unsigned *status) {
   if (ld_acquire(flag)) return true;
   const uint64_t t0 = globaltimer();
   for (uint32_t it = 1;; ++it) {
-    __nanosleep(64);
+    __nanosleep(32);
     if (ld_acquire(flag)) return true;
     if ((it & 255u) == 0 && globaltimer() - t0 > kWaitLimitNs) {
       set_status(status, CC_ERR_TIMEOUT);
@@ -54,144 +58,180 @@ CC_DEV bool wait_flag(const unsigned *flag, unsigned *status) {
   }
 }
 
+// Pre-pass: for every chunk u of class cls (chunks of class_rows[cls] slots),
+// the first and last chunk whose destinations read sources inside u.
+__global__ void deps_kernel(const __grid_constant__ CompactParams p) {
+  const int cls = blockIdx.z, b = blockIdx.y;
+  const int k = blockIdx.x * blockDim.x + threadIdx.x;
+  int J = p.keep_count[b];
+  if (J < 0 || J > p.cap) J = 0;
+  if (k >= J) return;
+  const int C = p.class_rows[cls];
+  const int32_t *kidx = p.keep_idx + (size_t)b * p.cap;
+  auto src_of = [&](int kk) {
+    int s = kidx[kk];
+    return (s < kk || s >= p.cap) ? kk : s;   // invalid entries are copied onto themselves
+  };
+  const int u = src_of(k) / C;
+  int2 *deps = p.deps + p.class_offset[cls] + (size_t)b * p.class_chunks[cls];
+  if (k == 0 || src_of(k - 1) / C != u) deps[u].x = k / C;
+  if (k == J - 1 || src_of(k + 1) / C != u) deps[u].y = k / C;
+}
+
+struct Unit {
+  int t;          // ticket (>= total: none)
+  int a, b, c;    // array, sequence, chunk
+  int k0, k1;     // destination slots [k0, k1)
+  bool loaded;    // bulk loads issued into the buffer
+};
+
 __global__ void __launch_bounds__(kThreads)
     compact_kernel(const __grid_constant__ CompactParams p) {
   extern __shared__ uint8_t smem_raw[];
-  uint8_t *stage = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 127) &
-                                               ~uintptr_t(127));
-  __shared__ __align__(8) uint64_t bar;
-  __shared__ int s_unit, s_go;
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  if (tid == 0) {
-    mbar_init(&bar, 1);
+  uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 127) &
+                                              ~uintptr_t(127));
+  __shared__ __align__(8) uint64_t bars[kWarps][2];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  uint8_t *buf[2] = {smem + (size_t)(warp * 2 + 0) * kStageBytes,
+                     smem + (size_t)(warp * 2 + 1) * kStageBytes};
+  if (lane == 0) {
+    mbar_init(&bars[warp][0], 1);
+    mbar_init(&bars[warp][1], 1);
     fence_barrier_init();
   }
-  if (blockIdx.x == 0) {   // the new lengths; no unit reads seq_len
-    for (int b = tid; b < p.batch; b += kThreads) {
+  if (blockIdx.x == 0 && warp == 0) {   // the new lengths; no unit reads seq_len
+    for (int b = lane; b < p.batch; b += 32) {
       int j = p.keep_count[b];
       p.seq_len[b] = (j >= 0 && j <= p.cap) ? j : 0;
     }
   }
-  __syncthreads();
-  uint32_t phase = 0;
+  __syncwarp();
+  uint32_t phase[2] = {0, 0};
   volatile int no_abort = 0;
 
-  for (;;) {
-    if (tid == 0) s_unit = (int)atomicAdd(p.ticket, 1u);
-    __syncthreads();
-    const int t = s_unit;
-    __syncthreads();
-    if (t >= p.total_units) break;
-    // ---- locate the unit: array a, sequence b, chunk c
+  auto take = [&]() -> Unit {
+    Unit u;
+    int t = 0;
+    if (lane == 0) t = (int)atomicAdd(p.ticket, 1u);
+    u.t = __shfl_sync(0xFFFFFFFFu, t, 0);
+    u.loaded = false;
+    u.a = u.b = u.c = u.k0 = u.k1 = 0;
+    if (u.t >= p.total_units) return u;
     int a = 0;
-    while (a + 1 < p.n_arrays && p.arr[a + 1].unit_base <= t) ++a;
+    while (a + 1 < p.n_arrays && p.arr[a + 1].unit_base <= u.t) ++a;
     const CompactArray &A = p.arr[a];
-    const int local = t - A.unit_base;
-    const int b = local / A.n_chunks, c = local - b * A.n_chunks;
-    const int C = A.rows_per_chunk;
-    int J = p.keep_count[b];
+    const int local = u.t - A.unit_base;
+    u.a = a;
+    u.b = local / A.n_chunks;
+    u.c = local - u.b * A.n_chunks;
+    int J = p.keep_count[u.b];
     if (J < 0 || J > p.cap) {
-      if (tid == 0) set_status(p.status, CC_ERR_DEVICE_ARG);
+      if (lane == 0) set_status(p.status, CC_ERR_DEVICE_ARG);
       J = 0;
     }
-    const int32_t *kidx = p.keep_idx + (size_t)b * p.cap;
-    const int k0 = c * C, k1 = min(k0 + C, J);
-    // first moving row: identity rows (kidx[k] == k) form a prefix
-    int first = k1;
-    if (k0 < k1) {
-      if (kidx[k1 - 1] == k1 - 1) {
-        first = k1;
-      } else if (kidx[k0] != k0) {
-        first = k0;
-      } else {  // binary search the boundary inside the chunk
-        int lo = k0, hi = k1 - 1;   // kidx[lo] == lo, kidx[hi] != hi
-        while (hi - lo > 1) {
-          int mid = (lo + hi) >> 1;
-          if (kidx[mid] == mid) lo = mid; else hi = mid;
-        }
-        first = hi;
-      }
-    }
-    const size_t seq_off = (size_t)b * p.cap;
-    uint8_t *base = reinterpret_cast<uint8_t *>(A.base);
-    const int rb = A.row_bytes;
-    const bool work = first < k1;
+    u.k0 = u.c * A.rows_per_chunk;
+    u.k1 = min(u.k0 + A.rows_per_chunk, J);
+    return u;
+  };
 
-    // ---- 1. read the sources
-    if (work) {
-      if (A.bulk) {
-        if (warp == 0) {
-          if (lane == 0) mbar_arrive_expect_tx(&bar, (uint32_t)((k1 - first) * rb));
-          __syncwarp();
-          for (int k = first + lane; k < k1; k += 32) {
-            int src = kidx[k];
-            if (src < k || src >= p.cap) {   // not ascending / out of range: copy row onto itself
-              set_status(p.status, CC_ERR_DEVICE_ARG);
-              src = k;
-            }
-            bulk_load(stage + (size_t)(k - k0) * rb, base + (seq_off + src) * rb, rb, &bar);
-          }
-          mbar_wait(&bar, phase, &no_abort, p.status);
-        }
-        phase ^= 1;
-      } else {   // 4-byte rows
-        for (int k = first + tid; k < k1; k += kThreads) {
-          int src = kidx[k];
-          if (src < k || src >= p.cap) {
-            set_status(p.status, CC_ERR_DEVICE_ARG);
-            src = k;
-          }
-          reinterpret_cast<uint32_t *>(stage)[k - k0] =
-              reinterpret_cast<const uint32_t *>(base)[seq_off + src];
-        }
-      }
+  // Source row of destination k; entries that are not ascending or out of
+  // range are copied onto themselves (and reported by `report`).
+  auto source = [&](const int32_t *kidx, int k, bool report) {
+    int s = kidx[k];
+    if (s < k || s >= p.cap) {
+      if (report) set_status(p.status, CC_ERR_DEVICE_ARG);
+      s = k;
     }
-    __syncthreads();
-    // ---- 2. publish; 3. wait for lower overlapping units
-    if (tid == 0) {
-      if (t != p.withhold_unit) st_release(&p.flags[t], 1u);
-      int go = 1;
-      if (work && c > 0) {
-        // highest lower chunk whose first source lies below our last destination
-        int lo = 0, hi = c - 1, cand = -1;
-        while (lo <= hi) {
-          int mid = (lo + hi) >> 1;
-          if (kidx[mid * C] < k1) { cand = mid; lo = mid + 1; } else hi = mid - 1;
-        }
-        for (int c2 = cand; c2 >= 0; --c2) {
-          const int last_src = kidx[min((c2 + 1) * C, J) - 1];
-          if (last_src < first) break;   // this and all lower chunks read below our rows
-          if (!wait_flag(&p.flags[A.unit_base + b * A.n_chunks + c2], p.status)) { go = 0; break; }
-        }
+    return s;
+  };
+
+  // Issues the reads of unit u into buffer slot s.
+  auto load = [&](Unit &u, int s) {
+    if (u.t >= p.total_units || u.k0 >= u.k1) return;
+    const CompactArray &A = p.arr[u.a];
+    const int32_t *kidx = p.keep_idx + (size_t)u.b * p.cap;
+    uint8_t *base = reinterpret_cast<uint8_t *>(A.base);
+    const size_t seq_off = (size_t)u.b * p.cap;
+    if (A.bulk) {
+      int moving = 0;
+      for (int k = u.k0 + lane; k < u.k1; k += 32) moving += (source(kidx, k, false) != k);
+      moving = __reduce_add_sync(0xFFFFFFFFu, moving);
+      if (moving == 0) return;
+      if (lane == 0) mbar_arrive_expect_tx(&bars[warp][s], (uint32_t)(moving * A.row_bytes));
+      __syncwarp();
+      for (int k = u.k0 + lane; k < u.k1; k += 32) {
+        const int src = source(kidx, k, true);
+        if (src != k)
+          bulk_load(buf[s] + (size_t)(k - u.k0) * A.row_bytes,
+                    base + (seq_off + src) * A.row_bytes, A.row_bytes, &bars[warp][s]);
+      }
+      u.loaded = true;
+    } else {   // 4-byte rows: plain loads staged in shared memory
+      uint32_t *st = reinterpret_cast<uint32_t *>(buf[s]);
+      for (int k = u.k0 + lane; k < u.k1; k += 32)
+        st[k - u.k0] = reinterpret_cast<const uint32_t *>(base)[seq_off + source(kidx, k, true)];
+    }
+  };
+
+  Unit cur = take();
+  load(cur, 0);
+  Unit nxt = take();
+  load(nxt, 1);
+  for (int i = 0; cur.t < p.total_units; ++i) {
+    const int s = i & 1;
+    const CompactArray &A = p.arr[cur.a];
+    // ---- 1. sources of `cur` are in shared memory
+    if (cur.loaded) {
+      mbar_wait(&bars[warp][s], phase[s], &no_abort, p.status);
+      phase[s] ^= 1;
+    }
+    __syncwarp();
+    // ---- 2. publish; 3. wait for the lower units that read our destinations
+    bool go = true;
+    if (lane == 0) {
+      if (cur.t != p.withhold_unit) st_release(&p.flags[cur.t], 1u);
+      if (cur.k0 < cur.k1 && cur.c > 0) {
+        const int2 d = p.deps[p.class_offset[A.dep_class] +
+                              (size_t)cur.b * p.class_chunks[A.dep_class] + cur.c];
+        const int hi = min(d.y, cur.c - 1);
+        for (int c2 = max(d.x, 0); c2 <= hi && go; ++c2)
+          go = wait_flag(&p.flags[A.unit_base + cur.b * A.n_chunks + c2], p.status);
       }
       fence_proxy_async_global();
-      s_go = go;
     }
-    __syncthreads();
+    go = __shfl_sync(0xFFFFFFFFu, go ? 1 : 0, 0) != 0;
     // ---- 4. write the destinations
-    if (work && s_go) {
+    if (go && cur.k0 < cur.k1) {
+      const int32_t *kidx = p.keep_idx + (size_t)cur.b * p.cap;
+      uint8_t *base = reinterpret_cast<uint8_t *>(A.base);
+      const size_t seq_off = (size_t)cur.b * p.cap;
       if (A.bulk) {
-        if (warp == 0) {
-          fence_proxy_async_global();
-          for (int k = first + lane; k < k1; k += 32)
-            bulk_store(base + (seq_off + k) * rb, stage + (size_t)(k - k0) * rb, rb);
+        if (cur.loaded) {
+          for (int k = cur.k0 + lane; k < cur.k1; k += 32)
+            if (source(kidx, k, false) != k)
+              bulk_store(base + (seq_off + k) * A.row_bytes,
+                         buf[s] + (size_t)(k - cur.k0) * A.row_bytes, A.row_bytes);
           bulk_commit();
-          bulk_wait_all_read();
         }
       } else {
-        for (int k = first + tid; k < k1; k += kThreads)
-          reinterpret_cast<uint32_t *>(base)[seq_off + k] =
-              reinterpret_cast<const uint32_t *>(stage)[k - k0];
+        const uint32_t *st = reinterpret_cast<const uint32_t *>(buf[s]);
+        for (int k = cur.k0 + lane; k < cur.k1; k += 32)
+          reinterpret_cast<uint32_t *>(base)[seq_off + k] = st[k - cur.k0];
       }
     }
-    __syncthreads();
+    bulk_wait_all_read();   // buffer s may be refilled
+    __syncwarp();
+    Unit nn = take();
+    load(nn, s);
+    cur = nxt;
+    nxt = nn;
   }
-  if (warp == 0) bulk_wait_all();
+  bulk_wait_all();
 }
 
 }  // namespace
 
-size_t compact_stage_bytes() { return kStageBytes + 128; }
+size_t compact_stage_bytes() { return (size_t)kWarps * 2 * kStageBytes + 128; }
 
 cudaError_t launch_compact(const CompactParams &p, int grid, cudaStream_t st) {
   static bool attr_set[64] = {};
@@ -204,6 +244,13 @@ cudaError_t launch_compact(const CompactParams &p, int grid, cudaStream_t st) {
     attr_set[dev] = true;
   }
   if (p.total_units <= 0) return cudaSuccess;
+  for (int cls = 0; cls < p.n_classes; ++cls) {
+    if (p.class_rows[cls] <= 0) return cudaErrorInvalidValue;
+  }
+  const dim3 dgrid((p.cap + 255) / 256, p.batch, p.n_classes);
+  deps_kernel<<<dgrid, 256, 0, st>>>(p);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
   compact_kernel<<<grid, kThreads, compact_stage_bytes(), st>>>(p);
   return cudaGetLastError();
 }

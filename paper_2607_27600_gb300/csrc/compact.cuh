@@ -4,8 +4,9 @@
 
 namespace cc {
 
-constexpr int kStageBytes = 64 * 1024;   // shared-memory staging per unit
+constexpr int kStageBytes = 24 * 1024;   // shared-memory staging per unit (two per warp)
 constexpr int kMaxCompactArrays = 2 * 128 + 3;
+constexpr int kMaxDepClasses = 3;        // distinct chunk sizes (K/V rows, H rows, 4-byte rows)
 
 struct CompactArray {
   void *base;          // [batch][cap][row_bytes]
@@ -14,6 +15,7 @@ struct CompactArray {
   int rows_per_chunk;  // destination slots per unit
   int n_chunks;        // units per sequence = ceil(cap / rows_per_chunk)
   int unit_base;       // first ticket of this array
+  int dep_class;       // chunk-size class (index into the readers table)
 };
 
 struct CompactParams {
@@ -23,6 +25,13 @@ struct CompactParams {
   int32_t *seq_len;           // [batch], set to keep_count
   unsigned *ticket;           // zeroed before launch
   unsigned *flags;            // [total_units], zeroed before launch
+  int2 *deps;                 // readers table, (-1,-1)-filled before launch: per class c,
+                              // [batch][class_chunks[c]] at class_offset[c]: first and
+                              // last chunk reading sources inside each chunk
+  int n_classes;
+  int class_rows[kMaxDepClasses];
+  int class_chunks[kMaxDepClasses];
+  long long class_offset[kMaxDepClasses];
   unsigned *status;
   int withhold_unit;          // test hook: this unit never publishes its flag (-1: none)
   CompactArray arr[kMaxCompactArrays];
