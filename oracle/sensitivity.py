@@ -1,0 +1,92 @@
+"""How far does bf16 arithmetic move the exact counter-causal score of a deep
+random model?  -- TEST INFRASTRUCTURE (a study script over the oracle).
+
+The oracle computes the full counter-causal pass (Sec. 3.1) in fp64.  A GPU
+pass must round some intermediates to bf16 to use the tensor cores.  This
+script re-runs the oracle's layer with bf16 rounding inserted at chosen
+points and reports, per layer, the score's max relative error against the
+exact fp64 pass (the parity metric: |g - o| / max(|o|, rms(o))):
+
+  queries      only the queries entering QK^T are rounded (every other step exact)
+  activations  every GEMM input (normalised inputs, attention output,
+               SwiGLU output) and the queries are rounded
+
+The drift measured here is a property of the arithmetic and of the random
+model, not of any kernel; the 32-layer full-pass tolerances of the parity
+tests are derived from it.  It imports only the oracle and the seeded input
+generators, never the CUDA path.
+
+    python -m oracle.sensitivity --layers 32 --n 16384 --rows 4
+"""
+import argparse
+import sys
+
+import numpy as np
+
+from . import refresh as R
+
+
+def bf16(x):
+    """Round to the nearest bf16 value (ties to even), kept in fp64."""
+    a = np.asarray(x, np.float64).astype(np.float32)
+    u = a.view(np.uint32).astype(np.uint64)
+    u = (u + 0x7FFF + ((u >> 16) & 1)) & 0xFFFF0000
+    return u.astype(np.uint32).view(np.float32).astype(np.float64)
+
+
+def layer(h, rows, pos, lw, k, v, n, shape, round_q, round_act):
+    rq = bf16 if round_q else (lambda x: x)
+    ra = bf16 if round_act else (lambda x: x)
+    a = ra(R.rms_norm(h, lw["attn_norm"], shape.rms_eps))
+    q = (a @ R.f64(lw["wq"]).T).reshape(len(rows), shape.n_q_heads, shape.head_dim)
+    q = rq(R.rope(q, pos, shape.rope_theta))
+    o = ra(R.counter_causal_attention(q, k, v, rows, n))
+    h = h + o.reshape(len(rows), -1) @ R.f64(lw["wo"]).T
+    m = ra(R.rms_norm(h, lw["mlp_norm"], shape.rms_eps))
+    act = ra(R.silu(m @ R.f64(lw["w_gate"]).T) * (m @ R.f64(lw["w_up"]).T))
+    return h + act @ R.f64(lw["w_down"]).T
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--layers", type=int, default=32)
+    ap.add_argument("--n", type=int, default=16384)
+    ap.add_argument("--rows", type=int, default=4)
+    ap.add_argument("--seed", type=int, default=3)
+    args = ap.parse_args(argv)
+    import synth
+    from synth.configs import LLAMA3_8B
+    shape = LLAMA3_8B
+    n, seed = args.n, args.seed
+    rows = np.unique(np.linspace(0, n - 3, args.rows).astype(np.int64))
+    toks = synth.tokens((n,), shape.vocab, seed, "study.tokens").numpy()
+    emb = synth.normal((shape.vocab, shape.d_model), 0.02, seed, "embed").float().numpy()
+    lm = synth.normal((shape.vocab, shape.d_model), 0.02, seed, "lm_head").float().numpy()
+    pos = np.arange(n)[rows]
+    variants = {"exact": (False, False), "queries": (True, False), "activations": (True, True)}
+    hs = {v: R.f64(emb[toks[rows]]) for v in variants}
+    ones = np.ones(shape.d_model)
+    print("layer  queries  activations", flush=True)
+    for l in range(args.layers):
+        lw = {name: synth.normal(shp, 0.02, seed, f"l{l}.{name}").float().numpy() for name, shp in
+              (("wq", (shape.q_dim, shape.d_model)), ("wo", (shape.d_model, shape.q_dim)),
+               ("w_gate", (shape.d_ff, shape.d_model)), ("w_up", (shape.d_ff, shape.d_model)),
+               ("w_down", (shape.d_model, shape.d_ff)))}
+        lw["attn_norm"] = lw["mlp_norm"] = ones
+        std = synth.kv_std(shape)
+        k = synth.normal((n, shape.n_kv_heads, shape.head_dim), std, seed, f"study.k{l}").float().numpy()
+        v = synth.normal((n, shape.n_kv_heads, shape.head_dim), std, seed, f"study.v{l}").float().numpy()
+        for name, (rq, ra) in variants.items():
+            hs[name] = layer(hs[name], rows, pos, lw, k, v, n, shape, rq, ra)
+        sc = {name: R.score_head(hs[name], toks[rows], ones, lm, "logit", shape.rms_eps)
+              for name in variants}
+        ref = sc["exact"]
+        rms = np.sqrt(np.mean(ref * ref))
+        err = {name: float(np.max(np.abs(sc[name] - ref) / np.maximum(np.abs(ref), rms)))
+               for name in ("queries", "activations")}
+        print(f"{l:5d}  {err['queries']:.4f}   {err['activations']:.4f}", flush=True)
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

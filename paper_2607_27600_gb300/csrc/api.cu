@@ -490,8 +490,15 @@ cc_status compact_plan(const cc_model_cfg *c, const cc_kv_cache *kv, CompactPlan
     units += kv->batch * A.n_chunks;
     return true;
   };
+  const int kv_row = c->n_kv_heads * c->head_dim * 2;
+  for (int l = 0; l < c->n_layers; ++l) {
+    if (!add(kv->k[l], kv_row, true) || !add(kv->v[l], kv_row, true)) return CC_ERR_UNSUPPORTED;
+  }
+  if (!add(kv->h_last, c->d_model * 2, true)) return CC_ERR_UNSUPPORTED;
+  if (!add(kv->tokens, 4, false) || !add(kv->pos, 4, false)) return CC_ERR_INVALID_ARG;
   p.n_arrays = n;
   p.total_units = units;
+  if (n < 2 || units < 2) return CC_ERR_INVALID_ARG;   // tokens and pos are always compacted
   // workspace: ticket | flags | readers table
   size_t deps_entries = 0;
   for (int c = 0; c < p.n_classes; ++c) {

@@ -64,3 +64,20 @@ def test_workspace_size_formula(lib):
     rows, d, q, f = 8192, 4096, 4096, 14336
     assert n >= rows * (2 * d + 2 * q * 2 + 4 * d + 2 * f)
     assert cc.cc_score_workspace_size(LLAMA3_8B, 1, 8192, cc.SCORE_LOGPROB) > n
+
+
+def test_compaction_plan_covers_every_array(lib):
+    """The compaction workspace grows with every array the cache holds (a plan
+    that registered no arrays would compact nothing); computed on the host."""
+    import ctypes
+    from paper_2607_27600_gb300 import cc
+    cfg = cc.cc_model_cfg(2, 256, 8, 2, 64, 384, 1000, 1e4, 1e-5)
+    fake = [ctypes.c_void_p(4096 * (i + 1)) for i in range(8)]   # never dereferenced
+    ks = (ctypes.c_void_p * 2)(fake[0], fake[1])
+    vs = (ctypes.c_void_p * 2)(fake[2], fake[3])
+    none = (ctypes.c_void_p * 2)(None, None)
+    full = cc.cc_kv_cache(1, 4096, fake[4], ks, vs, fake[5], fake[6], fake[7])
+    only_x = cc.cc_kv_cache(1, 4096, fake[4], none, none, fake[5], fake[6], None)
+    n_full = lib.cc_compact_workspace_size(ctypes.byref(cfg), ctypes.byref(full))
+    n_x = lib.cc_compact_workspace_size(ctypes.byref(cfg), ctypes.byref(only_x))
+    assert n_x > 256 and n_full > n_x

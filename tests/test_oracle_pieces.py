@@ -170,3 +170,12 @@ def test_score_head_logprob_matches_scipy():
     # logit-mode and log-prob-mode scores differ by exactly the log-normaliser
     lg = oracle.score_head(h, tok, np.ones(10), lm, "logit", 1e-6)
     np.testing.assert_allclose(got - lg, scipy.special.logsumexp(u @ lm.T, axis=-1), rtol=1e-12)
+
+
+def test_sensitivity_bf16_rounding_matches_torch():
+    from oracle.sensitivity import bf16
+    r = rng(21)
+    x = np.concatenate([r.normal(size=1000) * 10.0 ** r.integers(-6, 6, size=1000),
+                        [1.0 + 2.0 ** -8, 1.0 + 3 * 2.0 ** -8, -(1.0 + 2.0 ** -8), 0.0, -0.0]])
+    want = torch.from_numpy(x.astype(np.float32)).to(torch.bfloat16).double().numpy()
+    np.testing.assert_array_equal(bf16(x), want)
