@@ -168,9 +168,9 @@ cc_status cc_compact_kv(const cc_model_cfg *cfg, const cc_kv_cache *cache,
  * cannot allocate device memory for a workspace when they compact -- for
  * example a serving loop that has handed the whole device pool to the KV
  * cache, or a runtime that forbids device allocation on its refresh path
- * (cudaMalloc may block and synchronise the device).  Its scratch (a ticket
- * counter, one flag per work unit and a table of which work units read
- * each destination chunk) lives in a fixed 1 MiB array in the
+ * (cudaMalloc may block and synchronise the device).  Its scratch (a table
+ * of work units, one flag per work unit and a table of which work units
+ * read each destination chunk) lives in a fixed 1 MiB array in the
  * library's device memory, which every GPU that loads the library holds
  * until the process exits.  The call allocates nothing.
  *   - A cache needing more than 1 MiB of scratch (cc_compact_workspace_size()

@@ -42,7 +42,9 @@ cc_status cc_timing_collect(int32_t *counts, double *total_ms);
 const char *cc_kernel_name(int32_t kind);
 
 /* Failure-path test hook.  The next cc_compact_kv call (only that one) runs
- * with work unit `unit` (ticket order) never publishing its "sources read"
+ * with work unit `unit` (units numbered array by array, K_0, V_0, K_1, ...,
+ * then H, tokens, positions; in each, the kept-slot chunks in ascending
+ * order) never publishing its "sources read"
  * flag, as if that unit had stalled: a unit that depends on it waits out its
  * bounded wait (about 2 s), skips its writes and records CC_ERR_TIMEOUT, and
  * the kernel returns normally.  The GPU context stays usable.  -1 disarms. */

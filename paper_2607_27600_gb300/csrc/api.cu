@@ -445,10 +445,10 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
 }
 
 // compaction plan: arrays and unit counts
+// Compaction workspace: unit_base table | flags (zeroed per call) | readers table (-1 per call)
 struct CompactPlan {
   CompactParams p;
-  size_t flags_bytes;   // ticket + flags (zeroed per call)
-  size_t ws_bytes;      // + readers table (filled with -1 per call)
+  size_t base_bytes, flags_bytes, deps_bytes, ws_bytes;
 };
 
 int g_withhold_unit = -1;   // cc_debug_withhold_compact_unit: consumed by the next cc_compact_kv
@@ -484,7 +484,6 @@ cc_status compact_plan(const cc_model_cfg *c, const cc_kv_cache *kv, CompactPlan
                             : kStageBytes / 4;
     if (A.rows_per_chunk < 1) return false;
     A.n_chunks = (kv->cap + A.rows_per_chunk - 1) / A.rows_per_chunk;
-    A.unit_base = units;
     A.dep_class = class_of(A.rows_per_chunk);
     if (A.dep_class < 0) return false;
     units += kv->batch * A.n_chunks;
@@ -499,14 +498,26 @@ cc_status compact_plan(const cc_model_cfg *c, const cc_kv_cache *kv, CompactPlan
   p.n_arrays = n;
   p.total_units = units;
   if (n < 2 || units < 2) return CC_ERR_INVALID_ARG;   // tokens and pos are always compacted
-  // workspace: ticket | flags | readers table
   size_t deps_entries = 0;
   for (int c = 0; c < p.n_classes; ++c) {
     p.class_offset[c] = (long long)deps_entries;
     deps_entries += (size_t)kv->batch * p.class_chunks[c];
   }
-  plan.flags_bytes = 256 + align256((size_t)units * 4);
-  plan.ws_bytes = plan.flags_bytes + align256(deps_entries * sizeof(int2));
+  plan.base_bytes = align256(((size_t)n * kv->batch + 1) * sizeof(int));
+  plan.flags_bytes = align256((size_t)units * 4);
+  plan.deps_bytes = align256(deps_entries * sizeof(int2));
+  plan.ws_bytes = plan.base_bytes + plan.flags_bytes + plan.deps_bytes;
+  return CC_OK;
+}
+
+// Points the plan at workspace `ws` and clears what must start cleared.
+cc_status compact_bind(CompactPlan &plan, void *ws, cudaStream_t st) {
+  uint8_t *w = reinterpret_cast<uint8_t *>(ws);
+  plan.p.unit_base = reinterpret_cast<int *>(w);
+  plan.p.flags = reinterpret_cast<unsigned *>(w + plan.base_bytes);
+  plan.p.deps = reinterpret_cast<int2 *>(w + plan.base_bytes + plan.flags_bytes);
+  CC_TRY(cudaMemsetAsync(plan.p.flags, 0, plan.flags_bytes, st));
+  CC_TRY(cudaMemsetAsync(plan.p.deps, 0xFF, plan.deps_bytes, st));
   return CC_OK;
 }
 
@@ -576,15 +587,10 @@ cc_status cc_compact_kv(const cc_model_cfg *cfg, const cc_kv_cache *cache,
   DevState *dev;
   if (!dev_state(&dev)) return device_fail();
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-  CC_TRY(cudaMemsetAsync(ws, 0, plan.flags_bytes, st));
-  CC_TRY(cudaMemsetAsync(reinterpret_cast<uint8_t *>(ws) + plan.flags_bytes, 0xFF,
-                         plan.ws_bytes - plan.flags_bytes, st));
-  plan.p.deps = reinterpret_cast<int2 *>(reinterpret_cast<uint8_t *>(ws) + plan.flags_bytes);
+  if ((s = compact_bind(plan, ws, st)) != CC_OK) return s;
   plan.p.keep_idx = keep_idx;
   plan.p.keep_count = keep_count;
   plan.p.seq_len = cache->seq_len;
-  plan.p.ticket = reinterpret_cast<unsigned *>(ws);
-  plan.p.flags = reinterpret_cast<unsigned *>(reinterpret_cast<uint8_t *>(ws) + 256);
   plan.p.status = dev->status;
   plan.p.withhold_unit = g_withhold_unit;
   g_withhold_unit = -1;
@@ -716,15 +722,26 @@ const char *cc_kernel_name(int32_t kind) {
 namespace cc {
 
 cc_status compact_plan_build(const cc_model_cfg *cfg, const cc_kv_cache *cache, CompactParams &p,
-                             size_t &flags_bytes, size_t &scratch_bytes) {
+                             size_t &scratch_bytes) {
   static CompactPlan plan;
   static std::mutex mu;
   std::lock_guard<std::mutex> lk(mu);
   cc_status s = compact_plan(cfg, cache, plan);
   if (s != CC_OK) return s;
   p = plan.p;
-  flags_bytes = plan.flags_bytes;
   scratch_bytes = plan.ws_bytes;
+  return CC_OK;
+}
+
+cc_status compact_plan_bind(const cc_model_cfg *cfg, const cc_kv_cache *cache, CompactParams &p,
+                            void *scratch, cudaStream_t st) {
+  static CompactPlan plan;
+  static std::mutex mu;
+  std::lock_guard<std::mutex> lk(mu);
+  cc_status s = compact_plan(cfg, cache, plan);
+  if (s != CC_OK) return s;
+  if ((s = compact_bind(plan, scratch, st)) != CC_OK) return s;
+  p = plan.p;
   return CC_OK;
 }
 

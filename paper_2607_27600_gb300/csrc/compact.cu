@@ -13,7 +13,7 @@
 // come in ascending order.  A unit
 //   1. reads all its source rows into shared memory (TMA bulk copies for
 //      rows of 16-byte multiples; plain loads for 4-byte rows),
-//   2. publishes "sources read" for its ticket (release),
+//   2. publishes "sources read" for its unit (release),
 //   3. waits (acquire, bounded) until every lower unit that reads from its
 //      destination slots has published, and
 //   4. writes its destination rows (bulk stores).
@@ -21,11 +21,14 @@
 // pre-pass over keep_idx (deps_kernel): chunk u's readers are the chunks
 // holding the first and last k with keep_idx[k] in u.
 //
-// Tickets come from an atomic counter in dispatch order, a unit waits only
-// on lower tickets, and publishing never waits, so nothing can deadlock.
-// Each warp runs its own two-buffer pipeline: the loads of its next unit are
-// in flight while the current unit waits and stores.  Each element is read
-// once and written once; rows with keep_idx[k] == k are not moved.
+// A planning pre-pass numbers only the units that hold kept slots.  The
+// kernel is launched cooperatively (every warp resident) and warp w takes
+// units w, w + W, w + 2W, ... in ascending order, no atomics.  A unit waits
+// only on lower units and publishing never waits: the lowest unpublished
+// unit's warp is never blocked, so nothing can deadlock.  Each warp runs its
+// own two-buffer pipeline: the loads of its next unit are in flight while
+// the current unit waits and stores.  Each element is read once and written
+// once; rows with keep_idx[k] == k are not moved.
 #include "compact.cuh"
 
 namespace cc {
@@ -78,8 +81,29 @@ __global__ void deps_kernel(const __grid_constant__ CompactParams p) {
   if (k == J - 1 || src_of(k + 1) / C != u) deps[u].y = k / C;
 }
 
+// Pre-pass: unit_base[a*batch + b] = first unit of (array a, sequence b),
+// counting ceil(keep_count[b] / rows_per_chunk) units each; the last entry
+// is the number of units.
+__global__ void plan_kernel(const __grid_constant__ CompactParams p) {
+  if (threadIdx.x != 0) return;
+  int acc = 0;
+  for (int a = 0; a < p.n_arrays; ++a) {
+    const int C = p.arr[a].rows_per_chunk;
+    for (int b = 0; b < p.batch; ++b) {
+      p.unit_base[a * p.batch + b] = acc;
+      int J = p.keep_count[b];
+      if (J < 0 || J > p.cap) {
+        set_status(p.status, CC_ERR_DEVICE_ARG);
+        J = 0;
+      }
+      acc += (J + C - 1) / C;
+    }
+  }
+  p.unit_base[p.n_arrays * p.batch] = acc;
+}
+
 struct Unit {
-  int t;          // ticket (>= total: none)
+  int t;          // unit number (>= total: none)
   int a, b, c;    // array, sequence, chunk
   int k0, k1;     // destination slots [k0, k1)
   bool loaded;    // bulk loads issued into the buffer
@@ -109,26 +133,28 @@ __global__ void __launch_bounds__(kThreads)
   uint32_t phase[2] = {0, 0};
   volatile int no_abort = 0;
 
+  const int n_pairs = p.n_arrays * p.batch;
+  const int total = p.unit_base[n_pairs];
+  const int stride = gridDim.x * kWarps;
+  int next_t = blockIdx.x * kWarps + warp;
   auto take = [&]() -> Unit {
     Unit u;
-    int t = 0;
-    if (lane == 0) t = (int)atomicAdd(p.ticket, 1u);
-    u.t = __shfl_sync(0xFFFFFFFFu, t, 0);
+    u.t = next_t;
+    next_t += stride;
     u.loaded = false;
     u.a = u.b = u.c = u.k0 = u.k1 = 0;
-    if (u.t >= p.total_units) return u;
-    int a = 0;
-    while (a + 1 < p.n_arrays && p.arr[a + 1].unit_base <= u.t) ++a;
-    const CompactArray &A = p.arr[a];
-    const int local = u.t - A.unit_base;
-    u.a = a;
-    u.b = local / A.n_chunks;
-    u.c = local - u.b * A.n_chunks;
-    int J = p.keep_count[u.b];
-    if (J < 0 || J > p.cap) {
-      if (lane == 0) set_status(p.status, CC_ERR_DEVICE_ARG);
-      J = 0;
+    if (u.t >= total) return u;
+    int lo = 0, hi = n_pairs - 1;   // last pair whose first unit <= t
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (p.unit_base[mid] <= u.t) lo = mid; else hi = mid - 1;
     }
+    u.a = lo / p.batch;
+    u.b = lo - u.a * p.batch;
+    u.c = u.t - p.unit_base[lo];
+    const CompactArray &A = p.arr[u.a];
+    int J = p.keep_count[u.b];
+    if (J < 0 || J > p.cap) J = 0;
     u.k0 = u.c * A.rows_per_chunk;
     u.k1 = min(u.k0 + A.rows_per_chunk, J);
     return u;
@@ -147,7 +173,7 @@ __global__ void __launch_bounds__(kThreads)
 
   // Issues the reads of unit u into buffer slot s.
   auto load = [&](Unit &u, int s) {
-    if (u.t >= p.total_units || u.k0 >= u.k1) return;
+    if (u.t >= total || u.k0 >= u.k1) return;
     const CompactArray &A = p.arr[u.a];
     const int32_t *kidx = p.keep_idx + (size_t)u.b * p.cap;
     uint8_t *base = reinterpret_cast<uint8_t *>(A.base);
@@ -177,7 +203,7 @@ __global__ void __launch_bounds__(kThreads)
   load(cur, 0);
   Unit nxt = take();
   load(nxt, 1);
-  for (int i = 0; cur.t < p.total_units; ++i) {
+  for (int i = 0; cur.t < total; ++i) {
     const int s = i & 1;
     const CompactArray &A = p.arr[cur.a];
     // ---- 1. sources of `cur` are in shared memory
@@ -195,7 +221,7 @@ __global__ void __launch_bounds__(kThreads)
                               (size_t)cur.b * p.class_chunks[A.dep_class] + cur.c];
         const int hi = min(d.y, cur.c - 1);
         for (int c2 = max(d.x, 0); c2 <= hi && go; ++c2)
-          go = wait_flag(&p.flags[A.unit_base + cur.b * A.n_chunks + c2], p.status);
+          go = wait_flag(&p.flags[p.unit_base[cur.a * p.batch + cur.b] + c2], p.status);
       }
       fence_proxy_async_global();
     }
@@ -233,26 +259,37 @@ __global__ void __launch_bounds__(kThreads)
 
 size_t compact_stage_bytes() { return (size_t)kWarps * 2 * kStageBytes + 128; }
 
-cudaError_t launch_compact(const CompactParams &p, int grid, cudaStream_t st) {
-  static bool attr_set[64] = {};
+cudaError_t launch_compact(const CompactParams &p, int sms, cudaStream_t st) {
+  static int blocks_per_sm[64] = {};
   int dev = 0;
   cudaGetDevice(&dev);
-  if (dev < 64 && !attr_set[dev]) {
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  if (!blocks_per_sm[dev]) {
     cudaError_t e = cudaFuncSetAttribute(compact_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)compact_stage_bytes());
     if (e != cudaSuccess) return e;
-    attr_set[dev] = true;
+    int n = 0;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, compact_kernel, kThreads,
+                                                      compact_stage_bytes());
+    if (e != cudaSuccess) return e;
+    if (n < 1) return cudaErrorLaunchOutOfResources;
+    blocks_per_sm[dev] = n;
   }
   if (p.total_units <= 0) return cudaSuccess;
   for (int cls = 0; cls < p.n_classes; ++cls) {
     if (p.class_rows[cls] <= 0) return cudaErrorInvalidValue;
   }
-  const dim3 dgrid((p.cap + 255) / 256, p.batch, p.n_classes);
-  deps_kernel<<<dgrid, 256, 0, st>>>(p);
+  plan_kernel<<<1, 32, 0, st>>>(p);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  compact_kernel<<<grid, kThreads, compact_stage_bytes(), st>>>(p);
-  return cudaGetLastError();
+  const dim3 dgrid((p.cap + 255) / 256, p.batch, p.n_classes);
+  deps_kernel<<<dgrid, 256, 0, st>>>(p);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  // cooperative: every warp resident, so the static unit order cannot deadlock
+  void *args[] = {const_cast<CompactParams *>(&p)};
+  return cudaLaunchCooperativeKernel((const void *)compact_kernel, dim3(sms * blocks_per_sm[dev]),
+                                     dim3(kThreads), args, compact_stage_bytes(), st);
 }
 
 }  // namespace cc

@@ -13,17 +13,18 @@ struct CompactArray {
   int row_bytes;       // bulk arrays: multiple of 16; otherwise 4
   int bulk;            // rows moved by TMA bulk copies
   int rows_per_chunk;  // destination slots per unit
-  int n_chunks;        // units per sequence = ceil(cap / rows_per_chunk)
-  int unit_base;       // first ticket of this array
+  int n_chunks;        // chunks per sequence = ceil(cap / rows_per_chunk) (upper bound of units)
   int dep_class;       // chunk-size class (index into the readers table)
 };
 
 struct CompactParams {
-  int batch, cap, n_arrays, total_units;
+  int batch, cap, n_arrays;
+  int total_units;            // upper bound (every chunk of every array and sequence)
   const int32_t *keep_idx;    // [batch][cap]
   const int32_t *keep_count;  // [batch]
   int32_t *seq_len;           // [batch], set to keep_count
-  unsigned *ticket;           // zeroed before launch
+  int *unit_base;             // [n_arrays*batch + 1] first unit of each (array, sequence),
+                              // written by the planning pre-pass (units past keep_count skipped)
   unsigned *flags;            // [total_units], zeroed before launch
   int2 *deps;                 // readers table, (-1,-1)-filled before launch: per class c,
                               // [batch][class_chunks[c]] at class_offset[c]: first and
@@ -38,6 +39,7 @@ struct CompactParams {
 };
 
 size_t compact_stage_bytes();
-cudaError_t launch_compact(const CompactParams &p, int grid, cudaStream_t st);
+// Launches the pre-passes and the (cooperative) compaction; `sms` = SM count.
+cudaError_t launch_compact(const CompactParams &p, int sms, cudaStream_t st);
 
 }  // namespace cc

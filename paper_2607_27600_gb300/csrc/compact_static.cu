@@ -1,9 +1,9 @@
 // compact_static.cu -- cc_compact_kv_static: the in-place compaction of
 // cc_compact_kv for callers that cannot allocate device memory.
 //
-// cc_compact_kv takes its scratch (a work-unit ticket counter, one "sources
-// read" flag per unit and a table of which units read each destination
-// chunk) from a caller-provided workspace.  This
+// cc_compact_kv takes its scratch (a table of work units, one "sources read"
+// flag per unit and a table of which units read each destination chunk) from
+// a caller-provided workspace.  This
 // variant takes it from a fixed array in the library's own device memory
 // instead, so the caller passes only the cache, the keep-set and a stream.
 // The array is a file-scope __device__ variable: every GPU that loads the
@@ -15,8 +15,8 @@
 
 namespace {
 
-// 1 MiB: a 256-byte ticket slot, one 4-byte flag per work unit and the
-// readers table (8 bytes per destination chunk).
+// 1 MiB: the unit table (4 bytes per array and sequence), one 4-byte flag
+// per work unit and the readers table (8 bytes per destination chunk).
 constexpr size_t kStaticScratchBytes = size_t(1) << 20;
 __device__ __align__(256) unsigned char g_compact_scratch[kStaticScratchBytes];
 
@@ -47,8 +47,8 @@ extern "C" cc_status cc_compact_kv_static(const cc_model_cfg *cfg, const cc_kv_c
   static cc::CompactParams p;   // large kernel-parameter block; guarded by mu
   static std::mutex mu;
   std::lock_guard<std::mutex> lk(mu);
-  size_t need = 0, zeroed = 0;
-  cc_status s = cc::compact_plan_build(cfg, cache, p, zeroed, need);
+  size_t need = 0;
+  cc_status s = cc::compact_plan_build(cfg, cache, p, need);
   if (s != CC_OK) return s;
   if (!keep_idx || !keep_count) return CC_ERR_INVALID_ARG;
   if (need > kStaticScratchBytes) return CC_ERR_WORKSPACE;   // cache too large for the array
@@ -58,16 +58,12 @@ extern "C" cc_status cc_compact_kv_static(const cc_model_cfg *cfg, const cc_kv_c
   int sms = 0;
   if (!cc::current_device_info(&status, &sms)) return CC_ERR_CUDA;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-  // the ticket and the flags start at zero, the readers table at -1; the
-  // array keeps the last call's contents
-  if (cudaMemsetAsync(scratch, 0, zeroed, st) != cudaSuccess) return CC_ERR_CUDA;
-  if (cudaMemsetAsync(scratch + zeroed, 0xFF, need - zeroed, st) != cudaSuccess) return CC_ERR_CUDA;
-  p.deps = reinterpret_cast<int2 *>(scratch + zeroed);
+  // the flags start at zero and the readers table at -1 (cleared on `st`);
+  // the array keeps the last call's contents
+  if ((s = cc::compact_plan_bind(cfg, cache, p, scratch, st)) != CC_OK) return s;
   p.keep_idx = keep_idx;
   p.keep_count = keep_count;
   p.seq_len = cache->seq_len;
-  p.ticket = reinterpret_cast<unsigned *>(scratch);
-  p.flags = reinterpret_cast<unsigned *>(scratch + 256);
   p.status = status;
   if (cc::launch_compact(p, sms, st) != cudaSuccess) return CC_ERR_CUDA;
   return CC_OK;

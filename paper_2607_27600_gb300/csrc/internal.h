@@ -6,10 +6,13 @@
 namespace cc {
 
 // Builds the compaction plan of `cache` (arrays, work units) and the scratch
-// bytes it needs (the first flags_bytes start at zero, the rest at 0xFF);
-// same checks as cc_compact_kv.
+// bytes it needs; same checks as cc_compact_kv.
 cc_status compact_plan_build(const cc_model_cfg *cfg, const cc_kv_cache *cache, CompactParams &p,
-                             size_t &flags_bytes, size_t &scratch_bytes);
+                             size_t &scratch_bytes);
+// Builds the plan with its scratch at `scratch` and enqueues on `st` the
+// clearing of what must start cleared.
+cc_status compact_plan_bind(const cc_model_cfg *cfg, const cc_kv_cache *cache, CompactParams &p,
+                            void *scratch, cudaStream_t st);
 // Status-word address and SM count of the current device.
 bool current_device_info(unsigned **status, int *sms);
 
