@@ -39,8 +39,11 @@ def _headers_mtime():
     return max(os.path.getmtime(h) for h in hs)
 
 
-def build_library(verbose: bool = False, extra_flags=()) -> str:
+def build_library(verbose: bool = False, extra_flags=(), build_dir: str = None) -> str:
+    """Compiles csrc/*.cu and links libcc.so into build_dir (default: _build/)."""
     nvcc = _nvcc()
+    BUILD = build_dir or globals()["BUILD"]
+    LIB = os.path.join(BUILD, "libcc.so")
     os.makedirs(BUILD, exist_ok=True)
     hdr = _headers_mtime()
     jobs = []

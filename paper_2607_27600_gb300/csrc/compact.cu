@@ -35,7 +35,7 @@ namespace cc {
 
 namespace {
 
-constexpr int kWarps = 4;
+constexpr int kWarps = CC_COMPACT_WARPS;   // independent two-buffer pipelines per CTA
 constexpr int kThreads = kWarps * 32;
 
 CC_DEV void st_release(unsigned *p, unsigned v) {

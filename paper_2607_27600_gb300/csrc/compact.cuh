@@ -4,7 +4,13 @@
 
 namespace cc {
 
-constexpr int kStageBytes = 24 * 1024;   // shared-memory staging per unit (two per warp)
+#ifndef CC_COMPACT_STAGE_KB
+#define CC_COMPACT_STAGE_KB 24
+#endif
+#ifndef CC_COMPACT_WARPS
+#define CC_COMPACT_WARPS 4
+#endif
+constexpr int kStageBytes = CC_COMPACT_STAGE_KB * 1024;   // shared-memory staging per unit (two per warp)
 constexpr int kMaxCompactArrays = 2 * 128 + 3;
 constexpr int kMaxDepClasses = 3;        // distinct chunk sizes (K/V rows, H rows, 4-byte rows)
 
