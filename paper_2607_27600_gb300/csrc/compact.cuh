@@ -5,10 +5,10 @@
 namespace cc {
 
 #ifndef CC_COMPACT_STAGE_KB
-#define CC_COMPACT_STAGE_KB 24
+#define CC_COMPACT_STAGE_KB 12
 #endif
 #ifndef CC_COMPACT_WARPS
-#define CC_COMPACT_WARPS 4
+#define CC_COMPACT_WARPS 8
 #endif
 constexpr int kStageBytes = CC_COMPACT_STAGE_KB * 1024;   // shared-memory staging per unit (two per warp)
 constexpr int kMaxCompactArrays = 2 * 128 + 3;
