@@ -266,7 +266,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       tmem_ld32(s_t + 64, *reinterpret_cast<uint32_t(*)[32]>(&sr[64]));
       tmem_ld32(s_t + 96, *reinterpret_cast<uint32_t(*)[32]>(&sr[96]));
       tmem_ld_wait();
-      float mt = -INFINITY;
+      // row max with 8 independent partial maxima (a short dependency chain)
+      float mp[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) mp[u] = -INFINITY;
       const bool need_mask = (j0 <= p0 + P - 1) || (j0 + BKV > n) || !row_used;
       if (need_mask) {
         // key j kept iff pos < j < n
@@ -276,12 +279,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int c = 0; c < 128; ++c) {
           float x = (c > lo && c < hi) ? __uint_as_float(sr[c]) : -INFINITY;
           sr[c] = __float_as_uint(x);
-          mt = fmaxf(mt, x);
+          mp[c & 7] = fmaxf(mp[c & 7], x);
         }
       } else {
 #pragma unroll
-        for (int c = 0; c < 128; ++c) mt = fmaxf(mt, __uint_as_float(sr[c]));
+        for (int c = 0; c < 128; ++c) mp[c & 7] = fmaxf(mp[c & 7], __uint_as_float(sr[c]));
       }
+      const float mt = fmaxf(fmaxf(fmaxf(mp[0], mp[1]), fmaxf(mp[2], mp[3])),
+                             fmaxf(fmaxf(mp[4], mp[5]), fmaxf(mp[6], mp[7])));
       // lazy rescaling: move the reference max only when it grows by more
       // than 2^8 in exp2 space, so p <= 256 and O is rarely touched
       const float m_new = fmaxf(m_used, mt);

@@ -213,17 +213,32 @@ __global__ void __launch_bounds__(kThreads)
     }
     __syncwarp();
     // ---- 2. publish; 3. wait for the lower units that read our destinations
+    // A unit is waited on exactly when one of its source chunks is an active
+    // destination chunk above its own (the readers table lists it there), so
+    // only such units publish (a release store costs a memory barrier).
     bool go = true;
     if (lane == 0) {
-      if (cur.t != p.withhold_unit) st_release(&p.flags[cur.t], 1u);
+      if (cur.k0 < cur.k1) {
+        const int32_t *kidx = p.keep_idx + (size_t)cur.b * p.cap;
+        const int C = A.rows_per_chunk;
+        int J = p.keep_count[cur.b];
+        J = (J < 0 || J > p.cap) ? 0 : J;
+        const int active = (J + C - 1) / C;
+        const int lo_u = max(cur.c + 1, source(kidx, cur.k0, false) / C);
+        const int hi_u = min(active - 1, source(kidx, cur.k1 - 1, false) / C);
+        if (lo_u <= hi_u && cur.t != p.withhold_unit) st_release(&p.flags[cur.t], 1u);
+      }
+      bool waited = false;
       if (cur.k0 < cur.k1 && cur.c > 0) {
         const int2 d = p.deps[p.class_offset[A.dep_class] +
                               (size_t)cur.b * p.class_chunks[A.dep_class] + cur.c];
         const int hi = min(d.y, cur.c - 1);
-        for (int c2 = max(d.x, 0); c2 <= hi && go; ++c2)
+        for (int c2 = max(d.x, 0); c2 <= hi && go; ++c2) {
           go = wait_flag(&p.flags[p.unit_base[cur.a * p.batch + cur.b] + c2], p.status);
+          waited = true;
+        }
       }
-      fence_proxy_async_global();
+      if (waited) fence_proxy_async_global();
     }
     go = __shfl_sync(0xFFFFFFFFu, go ? 1 : 0, 0) != 0;
     // ---- 4. write the destinations
