@@ -13,6 +13,7 @@
 #include <math.h>
 #include <stdio.h>
 
+#include <algorithm>
 #include <mutex>
 
 #include "attn.cuh"
@@ -254,6 +255,19 @@ cc_status gemm_setup(Gemm &g, int epi, const void *A, int K, const void *W, cons
   g.p.n_tiles = (N + bn - 1) / bn;
   g.p.status = status;
   g.p.a_split = a_split ? 1 : 0;
+  // Tile order for L2 reuse: keep a slab of <= ~40 MB of one operand resident
+  // while the other streams, choosing the order that moves fewer bytes.
+  const double budget = 40.0 * (1 << 20);
+  const int num_m = (int)((R + 127) / 128), num_n = g.p.n_tiles;
+  const double k_a = (a_split ? 2.0 : 1.0) * K;
+  const double a_bytes = (double)R * k_a * 2, b_bytes = (double)num_n * 256 * K * 2;
+  const double a_slab = 128.0 * k_a * 2, b_slab = 256.0 * K * 2;
+  const int gn = (int)std::max(1.0, std::min((double)num_n, budget / b_slab));
+  const int gm = (int)std::max(1.0, std::min((double)num_m, budget / a_slab));
+  const double t0 = b_bytes + a_bytes * ((num_n + gn - 1) / gn);
+  const double t1 = a_bytes + b_bytes * ((num_m + gm - 1) / gm);
+  g.p.raster = t0 <= t1 ? 0 : 1;
+  g.p.group = t0 <= t1 ? gn : gm;
   return CC_OK;
 }
 

@@ -105,6 +105,26 @@ CC_DEV void tma_load_3d(void *dst, const CUtensorMap *m, uint64_t *bar, int32_t 
       "l"(reinterpret_cast<uint64_t>(m)), "r"(smem_u32(bar)), "r"(c0), "r"(c1), "r"(c2)
       : "memory");
 }
+// 2-D tile load with an L2 cache policy (from make_policy_*).
+CC_DEV void tma_load_2d_hint(void *dst, const CUtensorMap *m, uint64_t *bar, int32_t c0, int32_t c1,
+                             uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.L2::cache_hint"
+      " [%0], [%1, {%3, %4}], [%2], %5;" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(m)), "r"(smem_u32(bar)), "r"(c0), "r"(c1), "l"(policy)
+      : "memory");
+}
+// L2 policies: keep (evict last) for data read again soon, stream (evict first).
+CC_DEV uint64_t make_policy_evict_last() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+CC_DEV uint64_t make_policy_evict_first() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
 // Contiguous global -> shared copy (16-byte aligned addresses, size % 16 == 0).
 CC_DEV void bulk_load(void *dst, const void *src, uint32_t bytes, uint64_t *bar) {
   asm volatile(

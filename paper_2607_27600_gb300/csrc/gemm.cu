@@ -190,6 +190,26 @@ CC_DEV void epilogue_tile(const GemmParams &p, uint32_t tacc, int grow, bool val
   }
 }
 
+// Tile t -> (row tile m, column tile n) in grouped order: consecutive tiles
+// stay inside one group of `group` resident tiles of one operand while the
+// other operand's tiles stream past (see GemmParams::raster).
+CC_DEV void tile_coords(const GemmParams &p, int t, int num_m, int &m, int &n) {
+  const int num_n = p.n_tiles;
+  if (p.raster == 0) {   // resident column tiles, rows stream
+    const int per = num_m * p.group;
+    const int g = t / per, r = t - g * per;
+    const int gn = min(p.group, num_n - g * p.group);
+    m = r / gn;
+    n = g * p.group + (r - m * gn);
+  } else {               // resident row tiles, columns stream
+    const int per = num_n * p.group;
+    const int g = t / per, r = t - g * per;
+    const int gm = min(p.group, num_m - g * p.group);
+    n = r / gm;
+    m = g * p.group + (r - n * gm);
+  }
+}
+
 template <int EPI>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
@@ -238,10 +258,14 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 0) {
     if (lane == 0) {  // ---------------- TMA producer
+      const uint64_t keep = make_policy_evict_last(), stream = make_policy_evict_first();
+      const uint64_t pol_a = p.raster == 1 ? keep : stream;
+      const uint64_t pol_b = p.raster == 0 ? keep : stream;
       int stage = 0;
       uint32_t phase = 0;
       for (int tile = blockIdx.x; tile < total; tile += gridDim.x) {
-        const int nt = tile / num_m, mt = tile - nt * num_m;
+        int mt, nt;
+        tile_coords(p, tile, num_m, mt, nt);
         const int b = find_seq(prefix, p.batch, mt);
         const int row0 = b * p.cap + (mt - prefix[b]) * BM;
         for (int kb = 0; kb < nk_total; ++kb) {
@@ -250,12 +274,13 @@ __global__ void __launch_bounds__(kThreads, 1)
           // A column block kb of [hi | lo] (hi and lo halves are K apart), B block kb mod nk
           const int ka = kb < nk ? kb * BK : p.K + (kb - nk) * BK;
           const int kw = (kb < nk ? kb : kb - nk) * BK;
-          tma_load_2d(sA + stage * A_BYTES, &tmA, &full[stage], ka, row0);
+          tma_load_2d_hint(sA + stage * A_BYTES, &tmA, &full[stage], ka, row0, pol_a);
           if constexpr (EPI == EPI_SWIGLU) {
-            tma_load_2d(sB + stage * B_BYTES, &tmB, &full[stage], kw, nt * 128);
-            tma_load_2d(sB + stage * B_BYTES + B_BYTES / 2, &tmB2, &full[stage], kw, nt * 128);
+            tma_load_2d_hint(sB + stage * B_BYTES, &tmB, &full[stage], kw, nt * 128, pol_b);
+            tma_load_2d_hint(sB + stage * B_BYTES + B_BYTES / 2, &tmB2, &full[stage], kw, nt * 128,
+                             pol_b);
           } else {
-            tma_load_2d(sB + stage * B_BYTES, &tmB, &full[stage], kw, nt * BN);
+            tma_load_2d_hint(sB + stage * B_BYTES, &tmB, &full[stage], kw, nt * BN, pol_b);
           }
           if (++stage == ST) { stage = 0; phase ^= 1; }
         }
@@ -295,7 +320,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     int acc = 0;
     uint32_t acc_phase = 0;
     for (int tile = blockIdx.x; tile < total; tile += gridDim.x) {
-      const int nt = tile / num_m, mt = tile - nt * num_m;
+      int mt, nt;
+      tile_coords(p, tile, num_m, mt, nt);
       const int b = find_seq(prefix, p.batch, mt);
       const int i = (mt - prefix[b]) * BM + r;
       const bool valid = i < (p.seq_len ? p.seq_len[b] : p.cap);

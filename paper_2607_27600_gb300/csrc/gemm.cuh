@@ -29,6 +29,10 @@ struct GemmParams {
   float *z_target;         // EPI_LSE
   unsigned *status;
   int a_split;             // A rows are [hi | lo] (2K values): D = hi W^T + lo W^T
+  int raster;              // tile order: 0 = groups of `group` column tiles stay resident
+                           // (B kept in L2, A streamed per group); 1 = groups of `group`
+                           // row tiles stay resident (A kept, B streamed per group)
+  int group;
   int out_split;           // EPI_SWIGLU: out rows are [hi | lo], lo at column offset N
   unsigned long long turns[64];  // EPI_QROPE: inv_freq_k / (2 pi) in 0.64 fixed point
 };
