@@ -37,11 +37,38 @@ constexpr int kRegsLaunch = 168, kRegsSoftmax = 216, kRegsProducer = 64;
 static_assert(2 * 128 * kRegsSoftmax + 128 * kRegsProducer <= kThreads * kRegsLaunch,
               "register split exceeds the launch allocation");
 
+#ifndef CC_ATTN_EMU_EVERY
+#define CC_ATTN_EMU_EVERY 0   // every n-th pair of exponentials on the FMA pipe (0: none)
+#endif
+#ifndef CC_ATTN_SPLIT_P
+#define CC_ATTN_SPLIT_P 0     // hand P to the MMA in two 64-key halves
+#endif
+
 // 2^x by the PTX ex2.approx instruction (2 ulp; 2^-inf = 0).
 CC_DEV float fast_exp2(float x) {
   float y;
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
+}
+
+// 2^x for a pair on the FMA pipe, x finite (clamped to >= -125): x = j + f
+// with j = round(x) (adding 1.5*2^23 leaves j in the low mantissa bits) and
+// f in [-1/2, 1/2]; 2^f by a cubic fitted to minimise the relative error on
+// [-1/2, 1/2] (max 7.5e-5, below bf16's half ulp); 2^j added to the exponent
+// field as an integer.  Coefficients re-derived by tests/test_exp2_poly.py.
+CC_DEV float2 exp2_poly2(float2 x) {
+  constexpr float kMagic = 12582912.0f;   // 1.5 * 2^23
+  x.x = fmaxf(x.x, -125.f);
+  x.y = fmaxf(x.y, -125.f);
+  const float2 t = __fadd2_rn(x, make_float2(kMagic, kMagic));
+  const float2 j = __fadd2_rn(t, make_float2(-kMagic, -kMagic));
+  const float2 f = __fadd2_rn(x, make_float2(-j.x, -j.y));
+  float2 p = __ffma2_rn(f, make_float2(0.05517164245247841f, 0.05517164245247841f),
+                        make_float2(0.2426111251115799f, 0.2426111251115799f));
+  p = __ffma2_rn(p, f, make_float2(0.6932609677314758f, 0.6932609677314758f));
+  p = __ffma2_rn(p, f, make_float2(0.9999280571937561f, 0.9999280571937561f));
+  return make_float2(__uint_as_float(__float_as_uint(p.x) + (__float_as_uint(t.x) << 23)),
+                     __uint_as_float(__float_as_uint(p.y) + (__float_as_uint(t.y) << 23)));
 }
 
 template <int DH>
@@ -72,8 +99,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t *v_empty = v_full + KST;        // [KST]
   uint64_t *v_fixed = v_empty + KST;       // tail tile: V rows past n zeroed
   uint64_t *s_ready = v_fixed + 1;         // [2]
-  uint64_t *p_ready = s_ready + 2;         // [2]
-  uint64_t *o_done = p_ready + 2;          // [2]
+  uint64_t *p_ready = s_ready + 2;         // [2] (keys 0..63 of P when split)
+  uint64_t *p_ready_hi = p_ready + 2;      // [2] keys 64..127 of P (split hand-over)
+  uint64_t *o_done = p_ready_hi + 2;       // [2]
   uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(o_done + 2);
   volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
 
@@ -119,6 +147,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int h = 0; h < 2; ++h) {
       mbar_init(&s_ready[h], 1);
       mbar_init(&p_ready[h], 128);
+      mbar_init(&p_ready_hi[h], 128);
       mbar_init(&o_done[h], 1);
     }
     *abort_flag = 0;
@@ -218,12 +247,17 @@ __global__ void __launch_bounds__(kThreads, 1)
           tc_fence_after();
 #pragma unroll
           for (int kk = 0; kk < BKV / 16; ++kk) {
+            if (CC_ATTN_SPLIT_P && kk == BKV / 32) {   // second half of P
+              if (!(ok = mbar_wait(&p_ready_hi[h], it & 1, abort_flag, p.status))) break;
+              tc_fence_after();
+            }
             // B = V tile, MN-major: 64-column halves 16 KB apart (LBO),
             // 8-key groups 1024 B apart (SBO); A = P_h, bf16 pairs in TMEM.
             uint64_t bd = make_sdesc_sw128(v_s + kk * 16 * 128, BKV * 128, 1024);
             umma_ts(tmem + 256 + h * DH, tmem + h * 128 + kk * 8, bd, idesc_pv,
                     (it > 0 || kk > 0) ? 1u : 0u);
           }
+          if (!ok) break;
           if (h == 1) umma_commit(&v_empty[s]);
           if (it + 1 < ntiles) {
             const int s2 = (it + 1) % KST;
@@ -298,6 +332,23 @@ __global__ void __launch_bounds__(kThreads, 1)
         l *= factor;
         m_used = m_new;
       }
+      // O still holds the previous tiles' sum (S_ready implies the last PV is
+      // done); it must be rescaled before any PV of this tile accumulates.
+      auto rescale = [&]() {
+        if (__any_sync(0xFFFFFFFFu, rescale_o)) {
+          const float f = rescale_o ? factor : 1.f;
+#pragma unroll 1
+          for (int c = 0; c < DH; c += 32) {
+            uint32_t o[32];
+            tmem_ld32(o_t + c, o);
+            tmem_ld_wait();
+#pragma unroll
+            for (int k = 0; k < 32; ++k) o[k] = __float_as_uint(__uint_as_float(o[k]) * f);
+            tmem_st32(o_t + c, o);
+          }
+        }
+      };
+      if (CC_ATTN_SPLIT_P) rescale();
       // p = 2^(s*sl2 - m*sl2): one packed FMA per pair, bf16 P into TMEM over S,
       // the row sum l in fp32
       const float nm = (m_used == -INFINITY) ? 0.f : -m_used * sl2;
@@ -310,30 +361,28 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int k = 0; k < 32; k += 2) {
           const float2 y = __ffma2_rn(make_float2(__uint_as_float(sr[c0 + k]),
                                                   __uint_as_float(sr[c0 + k + 1])), sl2v, nmv);
-          const float2 e = make_float2(fast_exp2(y.x), fast_exp2(y.y));
+          float2 e;
+          if (CC_ATTN_EMU_EVERY > 0 && ((c0 + k) / 2) % (CC_ATTN_EMU_EVERY > 0 ? CC_ATTN_EMU_EVERY : 1) ==
+                                           (CC_ATTN_EMU_EVERY > 0 ? CC_ATTN_EMU_EVERY : 1) - 1 &&
+              !need_mask)
+            e = exp2_poly2(y);
+          else
+            e = make_float2(fast_exp2(y.x), fast_exp2(y.y));
           pk[k / 2] = pack_bf16x2(e.x, e.y);
           lsum = __fadd2_rn(lsum, e);
         }
         tmem_st16(s_t + c0 / 2, pk);
-      }
-      l += lsum.x + lsum.y;
-      // after P is written, so the S registers are free for the O rows
-      if (__any_sync(0xFFFFFFFFu, rescale_o)) {
-        // O still holds the previous tiles' sum (S_ready implies the last PV is done)
-        const float f = rescale_o ? factor : 1.f;
-#pragma unroll 1
-        for (int c = 0; c < DH; c += 32) {
-          uint32_t o[32];
-          tmem_ld32(o_t + c, o);
-          tmem_ld_wait();
-#pragma unroll
-          for (int k = 0; k < 32; ++k) o[k] = __float_as_uint(__uint_as_float(o[k]) * f);
-          tmem_st32(o_t + c, o);
+        if (CC_ATTN_SPLIT_P && c0 == 32) {   // keys 0..63 ready: the MMA may start P V
+          tmem_st_wait();
+          tc_fence_before();
+          mbar_arrive(&p_ready[h]);
         }
       }
+      l += lsum.x + lsum.y;
+      if (!CC_ATTN_SPLIT_P) rescale();   // after P is written: S registers free for the O rows
       tmem_st_wait();
       tc_fence_before();
-      mbar_arrive(&p_ready[h]);
+      mbar_arrive(CC_ATTN_SPLIT_P ? &p_ready_hi[h] : &p_ready[h]);
     }
     // ---- epilogue: O / l -> bf16 -> out[row_base + pos][g*G + hl][:]
     if (ok) ok = mbar_wait(&o_done[h], 0, abort_flag, p.status);
