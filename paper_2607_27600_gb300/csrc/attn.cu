@@ -44,6 +44,23 @@ static_assert(2 * 128 * kRegsSoftmax + 128 * kRegsProducer <= kThreads * kRegsLa
 #define CC_ATTN_SPLIT_P 0     // hand P to the MMA in two 64-key halves
 #endif
 
+#ifdef CC_ATTN_TRACE
+// Diagnostic build only: cycle stamps of one CTA's first tiles.
+// slot = (tile * 8 + event); events: 0/1 S ready seen (half 0/1), 2/3 S loaded,
+// 4/5 P stored, 6/7 MMA PV issued (half 0/1).
+__device__ unsigned long long g_attn_trace[64 * 8];
+#define TRACE(cond, it, ev)                                                          \
+  do {                                                                              \
+    if ((cond) && blockIdx.x == CC_ATTN_TRACE && (it) < 64) {                       \
+      unsigned long long c_;                                                        \
+      asm volatile("mov.u64 %0, %%clock64;" : "=l"(c_));                            \
+      g_attn_trace[(it) * 8 + (ev)] = c_;                                           \
+    }                                                                               \
+  } while (0)
+#else
+#define TRACE(cond, it, ev) do { } while (0)
+#endif
+
 // 2^x by the PTX ex2.approx instruction (2 ulp; 2^-inf = 0).
 CC_DEV float fast_exp2(float x) {
   float y;
@@ -244,6 +261,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t v_s = smem_u32(smem + L::OFF_V + s * L::KV_BYTES);
         for (int h = 0; h < 2; ++h) {
           if (!(ok = mbar_wait(&p_ready[h], it & 1, abort_flag, p.status))) break;
+          TRACE(true, it, 6 + h);
           tc_fence_after();
 #pragma unroll
           for (int kk = 0; kk < BKV / 16; ++kk) {
@@ -293,6 +311,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int it = 0; it < ntiles; ++it) {
       const int j0 = (t1 - it) * BKV;
       if (!(ok = mbar_wait(&s_ready[h], it & 1, abort_flag, p.status))) break;
+      TRACE(q == 0 && lane == 0, it, 0 + h);
       tc_fence_after();
       uint32_t sr[128];
       tmem_ld32(s_t + 0, *reinterpret_cast<uint32_t(*)[32]>(&sr[0]));
@@ -300,6 +319,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       tmem_ld32(s_t + 64, *reinterpret_cast<uint32_t(*)[32]>(&sr[64]));
       tmem_ld32(s_t + 96, *reinterpret_cast<uint32_t(*)[32]>(&sr[96]));
       tmem_ld_wait();
+      TRACE(q == 0 && lane == 0, it, 2 + h);
       // row max with 8 independent partial maxima (a short dependency chain)
       float mp[8];
 #pragma unroll
@@ -382,6 +402,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!CC_ATTN_SPLIT_P) rescale();   // after P is written: S registers free for the O rows
       tmem_st_wait();
       tc_fence_before();
+      TRACE(q == 0 && lane == 0, it, 4 + h);
       mbar_arrive(CC_ATTN_SPLIT_P ? &p_ready_hi[h] : &p_ready[h]);
     }
     // ---- epilogue: O / l -> bf16 -> out[row_base + pos][g*G + hl][:]
@@ -452,6 +473,12 @@ cudaError_t launch_dh(const CUtensorMap &q, const CUtensorMap &k, const CUtensor
 }  // namespace
 
 int attn_positions_per_unit(int group) { return 256 / group; }
+
+#ifdef CC_ATTN_TRACE
+extern "C" int cc_debug_attn_trace(unsigned long long *out, int n) {
+  return (int)cudaMemcpyFromSymbol(out, g_attn_trace, sizeof(unsigned long long) * (n < 512 ? n : 512));
+}
+#endif
 
 cudaError_t launch_attention(const CUtensorMap &q, const CUtensorMap &k, const CUtensorMap &v,
                              const AttnParams &p, cudaStream_t stream) {
