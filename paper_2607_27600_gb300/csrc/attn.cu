@@ -46,15 +46,16 @@ static_assert(2 * 128 * kRegsSoftmax + 128 * kRegsProducer <= kThreads * kRegsLa
 
 #ifdef CC_ATTN_TRACE
 // Diagnostic build only: cycle stamps of one CTA's first tiles.
-// slot = (tile * 8 + event); events: 0/1 S ready seen (half 0/1), 2/3 S loaded,
-// 4/5 P stored, 6/7 MMA PV issued (half 0/1).
-__device__ unsigned long long g_attn_trace[64 * 8];
+// slot = (tile * 16 + event); events: 0/1 S ready seen (half 0/1), 2/3 S loaded,
+// 4/5 P stored (warp 0 of the half), 6/7 MMA PV issued, 8..11 P stored by warps
+// 0..3 of half 0, 12/13 MMA thread enters its P wait (half 0/1).
+__device__ unsigned long long g_attn_trace[64 * 16];
 #define TRACE(cond, it, ev)                                                          \
   do {                                                                              \
     if ((cond) && blockIdx.x == CC_ATTN_TRACE && (it) < 64) {                       \
       unsigned long long c_;                                                        \
       asm volatile("mov.u64 %0, %%clock64;" : "=l"(c_));                            \
-      g_attn_trace[(it) * 8 + (ev)] = c_;                                           \
+      g_attn_trace[(it) * 16 + (ev)] = c_;                                           \
     }                                                                               \
   } while (0)
 #else
@@ -230,16 +231,31 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) {
       constexpr uint32_t idesc_qk = make_idesc_bf16(128, BKV, 0, 0);
       constexpr uint32_t idesc_pv = make_idesc_bf16(128, DH, 0, 1);
+      // Shared-memory descriptors built once; a K step only advances the
+      // start-address field (16-byte units): +2 per 16 columns of a 128-byte
+      // row (Q, K), +128 per 16 keys of V.  The issuing thread shares its SM
+      // sub-partition with softmax warps, so each MMA costs a few instructions.
+      uint64_t qd[2][L::NH], kd[KST][L::NH], vd[KST];
       const uint32_t q_s = smem_u32(smem + L::OFF_Q);
+#pragma unroll
+      for (int h = 0; h < 2; ++h)
+#pragma unroll
+        for (int hh = 0; hh < L::NH; ++hh)
+          qd[h][hh] = make_sdesc_sw128(q_s + hh * 256 * 128 + h * 128 * 128, 16, 1024);
+#pragma unroll
+      for (int st = 0; st < KST; ++st) {
+#pragma unroll
+        for (int hh = 0; hh < L::NH; ++hh)
+          kd[st][hh] = make_sdesc_sw128(smem_u32(smem + L::OFF_K + st * L::KV_BYTES) + hh * BKV * 128,
+                                        16, 1024);
+        vd[st] = make_sdesc_sw128(smem_u32(smem + L::OFF_V + st * L::KV_BYTES), BKV * 128, 1024);
+      }
       auto issue_qk = [&](int it, int h) {
-        const int s = it % KST;
-        const uint32_t k_s = smem_u32(smem + L::OFF_K + s * L::KV_BYTES);
+        const int st = it % KST;
 #pragma unroll
         for (int kk = 0; kk < DH / 16; ++kk) {
-          const int hh = kk >> 2, ko = (kk & 3) * 32;
-          uint64_t ad = make_sdesc_sw128(q_s + hh * 256 * 128 + h * 128 * 128 + ko, 16, 1024);
-          uint64_t bd = make_sdesc_sw128(k_s + hh * BKV * 128 + ko, 16, 1024);
-          umma_ss(tmem + h * 128, ad, bd, idesc_qk, kk > 0);
+          const int hh = kk >> 2, ko = (kk & 3) * 2;
+          umma_ss(tmem + h * 128, qd[h][hh] + ko, kd[st][hh] + ko, idesc_qk, kk > 0);
         }
       };
       bool ok = mbar_wait(q_full, 0, abort_flag, p.status);
@@ -255,11 +271,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int it = 0; ok && it < ntiles; ++it) {
         const int t = t1 - it, s = it % KST;
         const uint32_t ph = (it / KST) & 1;
+        TRACE(true, it, 14);
         if (!(ok = mbar_wait(&v_full[s], ph, abort_flag, p.status))) break;
+        TRACE(true, it, 15);
         if (t == t1 && n - t * BKV < BKV)
           if (!(ok = mbar_wait(v_fixed, 0, abort_flag, p.status))) break;
-        const uint32_t v_s = smem_u32(smem + L::OFF_V + s * L::KV_BYTES);
         for (int h = 0; h < 2; ++h) {
+          TRACE(true, it, 12 + h);
           if (!(ok = mbar_wait(&p_ready[h], it & 1, abort_flag, p.status))) break;
           TRACE(true, it, 6 + h);
           tc_fence_after();
@@ -271,8 +289,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             // B = V tile, MN-major: 64-column halves 16 KB apart (LBO),
             // 8-key groups 1024 B apart (SBO); A = P_h, bf16 pairs in TMEM.
-            uint64_t bd = make_sdesc_sw128(v_s + kk * 16 * 128, BKV * 128, 1024);
-            umma_ts(tmem + 256 + h * DH, tmem + h * 128 + kk * 8, bd, idesc_pv,
+            umma_ts(tmem + 256 + h * DH, tmem + h * 128 + kk * 8, vd[s] + kk * 128, idesc_pv,
                     (it > 0 || kk > 0) ? 1u : 0u);
           }
           if (!ok) break;
@@ -282,7 +299,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (h == 0)
               if (!(ok = mbar_wait(&k_full[s2], ((it + 1) / KST) & 1, abort_flag, p.status))) break;
             tc_fence_after();
+            TRACE(h == 0, it, 10);
             issue_qk(it + 1, h);
+            TRACE(h == 0, it, 11);
             umma_commit(&s_ready[h]);
             if (h == 1) umma_commit(&k_empty[s2]);
           } else {
@@ -403,6 +422,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       tmem_st_wait();
       tc_fence_before();
       TRACE(q == 0 && lane == 0, it, 4 + h);
+      TRACE(h == 0 && lane == 0 && q < 2, it, 8 + q);
       mbar_arrive(CC_ATTN_SPLIT_P ? &p_ready_hi[h] : &p_ready[h]);
     }
     // ---- epilogue: O / l -> bf16 -> out[row_base + pos][g*G + hl][:]
@@ -476,7 +496,7 @@ int attn_positions_per_unit(int group) { return 256 / group; }
 
 #ifdef CC_ATTN_TRACE
 extern "C" int cc_debug_attn_trace(unsigned long long *out, int n) {
-  return (int)cudaMemcpyFromSymbol(out, g_attn_trace, sizeof(unsigned long long) * (n < 512 ? n : 512));
+  return (int)cudaMemcpyFromSymbol(out, g_attn_trace, sizeof(unsigned long long) * (n < 1024 ? n : 1024));
 }
 #endif
 

@@ -290,6 +290,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else if (warp == 1) {
     if (lane == 0) {  // ---------------- MMA issuer
       constexpr uint32_t idesc = make_idesc_bf16(BM, BN, 0, 0);
+      const uint64_t a_desc0 = make_sdesc_sw128(smem_u32(sA), 16, 1024);
+      const uint64_t b_desc0 = make_sdesc_sw128(smem_u32(sB), 16, 1024);
       int stage = 0, acc = 0;
       uint32_t phase = 0, acc_phase = 0;
       for (int tile = blockIdx.x; tile < total; tile += gridDim.x) {
@@ -299,13 +301,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int kb = 0; kb < nk_total; ++kb) {
           if (!mbar_wait(&full[stage], phase, abort_flag, p.status)) goto mma_done;
           tc_fence_after();
-          const uint32_t a0 = smem_u32(sA + stage * A_BYTES);
-          const uint32_t b0 = smem_u32(sB + stage * B_BYTES);
+          // descriptors of this stage; a K step of 16 columns advances the
+          // start-address field by 32 bytes (+2 in 16-byte units)
+          const uint64_t ad = a_desc0 + (uint64_t)(stage * (A_BYTES >> 4));
+          const uint64_t bd = b_desc0 + (uint64_t)(stage * (B_BYTES >> 4));
 #pragma unroll
-          for (int k = 0; k < BK / 16; ++k) {
-            umma_ss(d_tmem, make_sdesc_sw128(a0 + k * 32, 16, 1024),
-                    make_sdesc_sw128(b0 + k * 32, 16, 1024), idesc, (kb | k) != 0);
-          }
+          for (int k = 0; k < BK / 16; ++k) umma_ss(d_tmem, ad + 2 * k, bd + 2 * k, idesc, (kb | k) != 0);
           umma_commit(&empty[stage]);
           if (++stage == ST) { stage = 0; phase ^= 1; }
         }
