@@ -113,6 +113,12 @@ def main(argv=None):
                for name in ("queries", "activations", "bf16-pass")}
         print(f"{l:5d}  {err['queries']:.4f}   {err['activations']:.4f}       {err['bf16-pass']:.4f}",
               flush=True)
+    # per-row errors after the last layer: the tail of the drift's distribution
+    print("after the last layer, per-row error quantiles (50 / 90 / 99 / max):")
+    for name in ("queries", "activations", "bf16-pass"):
+        e = np.abs(sc[name] - ref) / np.maximum(np.abs(ref), rms)
+        q = np.quantile(e, [0.5, 0.9, 0.99, 1.0])
+        print(f"  {name:12s} " + "  ".join(f"{x:.4f}" for x in q), flush=True)
     return 0
 
 

