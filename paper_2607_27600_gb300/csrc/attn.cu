@@ -125,10 +125,21 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int G = p.group, P = p.P;
-  const int units_per_pb = p.batch * p.n_kv_heads;
-  const int pb = blockIdx.x / units_per_pb;
-  const int rem = blockIdx.x - pb * units_per_pb;
-  const int b = rem / p.n_kv_heads, g = rem - b * p.n_kv_heads;
+  // Unit order: streams (sequence, KV head) in groups of streams_per_group;
+  // within a group, position blocks outermost (longest units first), the
+  // group's streams innermost.  The group size bounds how far apart in time
+  // two resident units of one stream read the same K/V tile (chosen so the
+  // K/V read in between stays well inside L2).
+  const int blocks_per_stream = (p.cap + P - 1) / P;
+  const int n_streams = p.batch * p.n_kv_heads;
+  const int per_group = p.streams_per_group * blocks_per_stream;
+  const int grp = blockIdx.x / per_group;
+  const int s0 = grp * p.streams_per_group;
+  const int gsz = min(p.streams_per_group, n_streams - s0);
+  const int r = blockIdx.x - grp * per_group;
+  const int pb = r / gsz;
+  const int stream = s0 + (r - pb * gsz);
+  const int b = stream / p.n_kv_heads, g = stream - b * p.n_kv_heads;
   int n = p.seq_len[b];
   if (n < 0 || n > p.cap) {
     if (threadIdx.x == 0) set_status(p.status, CC_ERR_DEVICE_ARG);
@@ -180,6 +191,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegsProducer));
     if (warp == 8) {
     // ------------------------------------------------------------ producer
+    // Rows P*G..255 of the Q tile exist when G does not divide 256: zero
+    // them once so their S rows are exact zeros (finite, never NaN) and the
+    // softmax can treat every row of a tile alike (no per-row mask path).
+    if (G * P < 256) {
+      for (int hh = 0; hh < L::NH; ++hh)
+        for (int idx = G * P * 8 + lane; idx < 256 * 8; idx += 32)
+          reinterpret_cast<uint4 *>(smem + L::OFF_Q + hh * 256 * 128)[idx] = make_uint4(0, 0, 0, 0);
+      fence_proxy_async_smem();
+      __syncwarp();
+    }
     if (lane == 0) {
       tma_prefetch_desc(&tmQ);
       tma_prefetch_desc(&tmK);
@@ -343,7 +364,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       float mp[8];
 #pragma unroll
       for (int u = 0; u < 8; ++u) mp[u] = -INFINITY;
-      const bool need_mask = (j0 <= p0 + P - 1) || (j0 + BKV > n) || !row_used;
+      // uniform over the CTA: rows past P*G have zero queries and need no mask
+      const bool need_mask = (j0 <= p0 + P - 1) || (j0 + BKV > n);
       if (need_mask) {
         // key j kept iff pos < j < n
         const int lo = pos - j0;       // keep c > lo
@@ -486,7 +508,22 @@ cudaError_t launch_dh(const CUtensorMap &q, const CUtensorMap &k, const CUtensor
   }
   const long long units = (long long)p.batch * p.n_kv_heads * ((p.cap + p.P - 1) / p.P);
   if (units <= 0) return cudaSuccess;
-  kern<<<(unsigned)units, kThreads, AttnSmem<DH>::BYTES, stream>>>(q, k, v, p);
+  // Resident units of one stream start about T / (SMs / streams) apart (T a
+  // unit's run time), so between two reads of a K/V tile the resident units
+  // read about streams^2 * cap * (K+V bytes per slot) / SMs bytes.  Pick the
+  // largest stream group keeping that under kReuseBytes.  The bound is set
+  // from timings, far below the L2 size: Llama-3-8B at 8k slots and Qwen2.5
+  // at 32k slots run fastest with all streams in one group (their K/V fit in
+  // L2 whatever the order), four 32k Llama sequences and a 131k Qwen sequence
+  // with groups of a few streams.
+  static int sms[64] = {};
+  if (dev < 64 && !sms[dev]) cudaDeviceGetAttribute(&sms[dev], cudaDevAttrMultiProcessorCount, dev);
+  const double kReuseBytes = 2.0 * (1 << 20);
+  const double per_stream2 = (double)p.cap * 4.0 * DH / (dev < 64 && sms[dev] ? sms[dev] : 148);
+  const int n_streams = p.batch * p.n_kv_heads;
+  AttnParams pp = p;
+  pp.streams_per_group = (int)fmax(1.0, fmin((double)n_streams, floor(sqrt(kReuseBytes / per_stream2))));
+  kern<<<(unsigned)units, kThreads, AttnSmem<DH>::BYTES, stream>>>(q, k, v, pp);
   return cudaGetLastError();
 }
 

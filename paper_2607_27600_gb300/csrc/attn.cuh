@@ -13,6 +13,7 @@ struct AttnParams {
   int out_ld;               // elements per output row (n_q_heads*head_dim, or twice that)
   int out_lo;               // > 0: also write lo = bf16(o - hi) at element offset out_lo
   float scale_log2;         // log2(e) / sqrt(head_dim)
+  int streams_per_group;    // unit order (set by launch_attention): see attn.cu
   unsigned *status;
 };
 

@@ -32,7 +32,7 @@ def test_linear_matches_fp64(cc, rows, n, k):
     assert err <= 1e-4 * scale + 1e-5, (err, scale)
 
 
-def _attn_case(cc, batch, cap, seq, hq, hkv, dh, seed, kscale=1.0):
+def _attn_case(cc, batch, cap, seq, hq, hkv, dh, seed, kscale=1.0, rows=None):
     q = synth.normal((batch * cap, hq, dh), 1.0, seed, "q")
     k = synth.normal((batch, cap, hkv, dh), kscale, seed, "k")
     v = synth.normal((batch, cap, hkv, dh), 1.0, seed, "v")
@@ -45,18 +45,20 @@ def _attn_case(cc, batch, cap, seq, hq, hkv, dh, seed, kscale=1.0):
     qn = q.float().numpy().reshape(batch, cap, hq, dh)
     kn, vn = k.float().numpy(), v.float().numpy()
     for b, n in enumerate(seq):
-        want = oracle.counter_causal_attention(qn[b, :n], kn[b], vn[b], np.arange(n), n)
-        g = got[b, :n]
+        r = np.arange(n) if rows is None else np.unique(np.clip(rows(n), 0, n - 1))
+        want = oracle.counter_causal_attention(qn[b, r], kn[b], vn[b], r, n)
+        g = got[b, r]
         assert np.all(np.isfinite(g))
         err = np.abs(g - want).max() if n else 0.0
         # bf16 output rounding (2^-9 relative) plus bf16 P in the PV product
         assert err <= 2e-2 * max(1.0, np.abs(want).max()), (b, n, err)
-        if n:
-            np.testing.assert_array_equal(g[n - 1], 0.0)   # last row: nothing to attend
+        if n and r[-1] == n - 1:
+            np.testing.assert_array_equal(g[-1], 0.0)   # last row: nothing to attend
 
 
+# group sizes 3, 5, 6, 7 leave 1-4 of a unit's 256 query rows unused
 @pytest.mark.parametrize("hq,hkv,dh", [(8, 2, 64), (32, 8, 128), (28, 4, 128), (4, 4, 128),
-                                       (8, 1, 64)])
+                                       (8, 1, 64), (6, 2, 128), (10, 2, 64), (12, 2, 128)])
 def test_attention_shapes(cc, hq, hkv, dh):
     _attn_case(cc, 2, 384, [384, 301], hq, hkv, dh, seed=hq * 7 + dh)
 
@@ -70,9 +72,19 @@ def test_attention_ragged_large_ragged_tail(cc):
     _attn_case(cc, 2, 1200, [1200, 777], 32, 8, 128, seed=5, kscale=2.0)
 
 
-def test_attention_ignores_non_finite_stale_slots(cc):
+@pytest.mark.parametrize("batch,seq", [(1, [40960]), (2, [40960, 30001])])
+def test_attention_grouped_unit_order(cc, batch, seq):
+    """Caches long enough that units run in groups of a few (sequence, KV
+    head) streams, the last group smaller: sampled rows of every stream."""
+    def rows(n):
+        return np.array([0, 1, 63, 64, 65, 5000, n // 2, n - 130, n - 129, n - 2, n - 1])
+    _attn_case(cc, batch, 40960, seq, 32, 8, 128, seed=41 + batch, rows=rows)
+
+
+@pytest.mark.parametrize("hq,hkv", [(8, 2), (28, 4)])
+def test_attention_ignores_non_finite_stale_slots(cc, hq, hkv):
     """Slots past seq_len may hold any bits (NaN here); outputs must not see them."""
-    batch, cap, hq, hkv, dh = 1, 256, 8, 2, 128
+    batch, cap, dh = 1, 256, 128
     seq = [150]
     q = synth.normal((cap, hq, dh), 1.0, 9, "q").cuda()
     k = synth.normal((batch, cap, hkv, dh), 1.0, 9, "k").cuda()
