@@ -75,6 +75,19 @@ typedef struct {
   int32_t vocab;
   float rope_theta;     /* inv_freq_k = theta^(-2k/head_dim), angles taken exactly mod 2pi  */
   float rms_eps;
+  /* Optional Llama-3.1 RoPE frequency scaling (a property of that model, not
+   * of the paper's method).  0 = off (a zero-initialised struct has it off).
+   * Otherwise, with wavelength w_k = 2 pi / inv_freq_k: w_k below
+   * original_max_pos / high_freq_factor keeps inv_freq_k; above
+   * original_max_pos / low_freq_factor it becomes inv_freq_k / factor; in
+   * between, (1 - a) inv_freq_k / factor + a inv_freq_k with
+   * a = (original_max_pos / w_k - low) / (high - low).
+   * Requires factor >= 1, 0 < low < high, original_max_pos > 0
+   * (else CC_ERR_INVALID_ARG). */
+  float rope_scaling_factor;
+  float rope_low_freq_factor;
+  float rope_high_freq_factor;
+  int32_t rope_original_max_pos;
 } cc_model_cfg;
 
 /* One layer's weights, all bf16 device pointers. */
@@ -86,6 +99,9 @@ typedef struct {
   const void *w_gate;    /* [d_ff][d_model]                  */
   const void *w_up;      /* [d_ff][d_model]                  */
   const void *w_down;    /* [d_model][d_ff]                  */
+  const void *bq;        /* optional [n_q_heads*head_dim] q-projection bias (Qwen2-style
+                            attention), added before RoPE; NULL = none; 16-byte aligned.
+                            K/V biases belong to the cache builder: cached K/V hold them */
 } cc_layer_weights;
 
 typedef struct {

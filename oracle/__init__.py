@@ -7,6 +7,11 @@ CPU legs of bench.py may import it.  It shares no code with the CUDA path.
 Parity status per function (what pins it, in tests/test_oracle_*.py):
   rms_norm                 torch rms_norm (library routine)
   rope                     complex-multiplication identity; relative-position property
+  rope_inv_freq (scaled)   band structure of Llama-3.1 scaling: unchanged short
+                           wavelengths, factor-slowed long ones, an affine blend
+                           between that meets both edges
+  project (q/k/v biases)   closed form with Wq = 0 (queries = rotated bias);
+                           RoPE-shift invariance of a biased, scaled model
   counter_causal_attention torch SDPA with an explicit mask (library routine);
                            closed forms (row n-2 -> V[n-1], K = 0 -> mean of later V,
                            last row -> 0); brute force on tiny inputs
@@ -21,6 +26,7 @@ Parity status per function (what pins it, in tests/test_oracle_*.py):
 The paper prints no worked example with score values, so no pin is a
 printed number; every step of the score is pinned by the checks above.
 """
-from .refresh import (rms_norm, rope, rope_angles, softmax, counter_causal_attention,  # noqa: F401
+from .refresh import (rms_norm, rope, rope_angles, rope_inv_freq, project, softmax,  # noqa: F401
+                      counter_causal_attention,
                       causal_attention, silu, swiglu_mlp, counter_causal_layer, score_head,
                       score_layer, score_full, select_keep, compact, causal_forward)

@@ -20,8 +20,11 @@ Conventions (readings of the paper where it is silent or ambiguous):
   * a row with no later key (the last one) has attention output 0;
   * layer = Llama/Qwen pre-norm block: RMSNorm -> counter-causal attention ->
     residual -> RMSNorm -> SwiGLU MLP -> residual; final RMSNorm; untied LM head;
-  * RoPE: rotate-half pairs (k, k + dh/2), inv_freq_k = theta^(-2k/dh),
-    angles pos * inv_freq_k in fp64; attention scale 1/sqrt(head_dim);
+  * RoPE: rotate-half pairs (k, k + dh/2), inv_freq_k = theta^(-2k/dh)
+    (optionally Llama-3.1 frequency scaling), angles pos * inv_freq_k in
+    fp64; attention scale 1/sqrt(head_dim);
+  * projections: no biases, except the Qwen2-style q/k/v biases where a
+    layer holds them (bq, bk, bv), added before RoPE;
   * GQA: query head t reads KV head t // (Hq / Hkv);
   * keep-set ties are broken toward the later slot; NaN scores rank as -inf;
     sink slots [0, n_sink) are always kept (Sec. 3.2, frozen system prompt);
@@ -52,22 +55,52 @@ def rms_norm(x, gain, eps):
     return x / np.sqrt(np.mean(x * x, axis=-1, keepdims=True) + eps) * f64(gain)
 
 
-def rope_angles(pos, head_dim, theta):
-    """Rotation angle pos * theta^(-2k/dh) of pair k, for every position in `pos`."""
+def rope_inv_freq(head_dim, theta, scaling=None):
+    """Rotation frequencies inv_freq_k = theta^(-2k/dh), k < dh/2.
+
+    scaling = (factor, low_freq_factor, high_freq_factor, original_max_pos)
+    applies Llama-3.1's frequency scaling (a published model property, not
+    part of the paper's method): with wavelength w_k = 2 pi / inv_freq_k,
+    pairs whose w_k is shorter than original_max_pos / high_freq_factor keep
+    their frequency, pairs longer than original_max_pos / low_freq_factor
+    turn factor times slower, and in between the frequency is the blend
+    (1 - a) inv_freq_k / factor + a inv_freq_k with a rising linearly in
+    original_max_pos / w_k from 0 (at the long edge) to 1 (at the short edge).
+    """
     k = np.arange(head_dim // 2, dtype=np.float64)
     inv_freq = float(theta) ** (-2.0 * k / head_dim)
-    return f64(pos)[..., None] * inv_freq
+    if scaling is None:
+        return inv_freq
+    factor, low, high, orig = (float(x) for x in scaling)
+    wavelen = 2.0 * np.pi / inv_freq
+    a = (orig / wavelen - low) / (high - low)
+    blended = (1.0 - a) * inv_freq / factor + a * inv_freq
+    out = np.where(wavelen > orig / low, inv_freq / factor, blended)
+    return np.where(wavelen < orig / high, inv_freq, out)
 
 
-def rope(x, pos, theta):
+def rope_angles(pos, head_dim, theta, scaling=None):
+    """Rotation angle pos * inv_freq_k of pair k, for every position in `pos`."""
+    return f64(pos)[..., None] * rope_inv_freq(head_dim, theta, scaling)
+
+
+def rope(x, pos, theta, scaling=None):
     """Rotate-half RoPE of x [..., H, dh] at positions pos [...] (one per row)."""
     x = f64(x)
     dh = x.shape[-1]
     half = dh // 2
-    ang = rope_angles(pos, dh, theta)[..., None, :]      # broadcast over heads
+    ang = rope_angles(pos, dh, theta, scaling)[..., None, :]      # broadcast over heads
     c, s = np.cos(ang), np.sin(ang)
     x1, x2 = x[..., :half], x[..., half:]
     return np.concatenate([x1 * c - x2 * s, x2 * c + x1 * s], axis=-1)
+
+
+def project(a, lw, name):
+    """a @ W^T for the projection `name` (wq, wk, wv), plus its bias (bq, bk,
+    bv) where the layer has one (Qwen2-style attention projections)."""
+    y = a @ f64(lw[name]).T
+    b = lw.get("b" + name[1:])
+    return y if b is None else y + f64(b)
 
 
 def softmax(s):
@@ -135,8 +168,8 @@ def counter_causal_layer(h, rows, pos_rows, lw, k, v, n, shape):
     fresh queries from the rows' own hidden states at their original
     positions, cached K/V reused (not recomputed).  h: [R, d] -> [R, d]."""
     a = rms_norm(h, lw["attn_norm"], shape.rms_eps)
-    q = (a @ f64(lw["wq"]).T).reshape(len(rows), shape.n_q_heads, shape.head_dim)
-    q = rope(q, pos_rows, shape.rope_theta)
+    q = project(a, lw, "wq").reshape(len(rows), shape.n_q_heads, shape.head_dim)
+    q = rope(q, pos_rows, shape.rope_theta, getattr(shape, "rope_scaling", None))
     o = counter_causal_attention(q, k, v, rows, n)
     h = h + o.reshape(len(rows), -1) @ f64(lw["wo"]).T
     m = rms_norm(h, lw["mlp_norm"], shape.rms_eps)
@@ -295,11 +328,12 @@ def causal_forward(shape, weights, tokens, pos):
         if l == shape.n_layers - 1:
             h_last = h.copy()
         a = rms_norm(h, lw["attn_norm"], shape.rms_eps)
-        q = rope((a @ f64(lw["wq"]).T).reshape(n, shape.n_q_heads, shape.head_dim), pos,
-                 shape.rope_theta)
-        k = rope((a @ f64(lw["wk"]).T).reshape(n, shape.n_kv_heads, shape.head_dim), pos,
-                 shape.rope_theta)
-        v = (a @ f64(lw["wv"]).T).reshape(n, shape.n_kv_heads, shape.head_dim)
+        sc = getattr(shape, "rope_scaling", None)
+        q = rope(project(a, lw, "wq").reshape(n, shape.n_q_heads, shape.head_dim), pos,
+                 shape.rope_theta, sc)
+        k = rope(project(a, lw, "wk").reshape(n, shape.n_kv_heads, shape.head_dim), pos,
+                 shape.rope_theta, sc)
+        v = project(a, lw, "wv").reshape(n, shape.n_kv_heads, shape.head_dim)
         ks.append(k)
         vs.append(v)
         o = causal_attention(q, k, v)

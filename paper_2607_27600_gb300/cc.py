@@ -40,12 +40,14 @@ class cc_model_cfg(ctypes.Structure):
     _fields_ = [("n_layers", ctypes.c_int32), ("d_model", ctypes.c_int32),
                 ("n_q_heads", ctypes.c_int32), ("n_kv_heads", ctypes.c_int32),
                 ("head_dim", ctypes.c_int32), ("d_ff", ctypes.c_int32), ("vocab", ctypes.c_int32),
-                ("rope_theta", ctypes.c_float), ("rms_eps", ctypes.c_float)]
+                ("rope_theta", ctypes.c_float), ("rms_eps", ctypes.c_float),
+                ("rope_scaling_factor", ctypes.c_float), ("rope_low_freq_factor", ctypes.c_float),
+                ("rope_high_freq_factor", ctypes.c_float), ("rope_original_max_pos", ctypes.c_int32)]
 
 
 class cc_layer_weights(ctypes.Structure):
     _fields_ = [(n, ctypes.c_void_p) for n in
-                ("attn_norm", "wq", "wo", "mlp_norm", "w_gate", "w_up", "w_down")]
+                ("attn_norm", "wq", "wo", "mlp_norm", "w_gate", "w_up", "w_down", "bq")]
 
 
 class cc_model_weights(ctypes.Structure):
@@ -152,16 +154,20 @@ def _check(code, where):
 
 
 def model_cfg(shape) -> cc_model_cfg:
-    """cc_model_cfg from any object with the ModelShape fields."""
+    """cc_model_cfg from any object with the ModelShape fields (rope_scaling,
+    if present and not None: (factor, low_freq_factor, high_freq_factor,
+    original_max_position))."""
+    sc = getattr(shape, "rope_scaling", None) or (0.0, 0.0, 0.0, 0)
     return cc_model_cfg(shape.n_layers, shape.d_model, shape.n_q_heads, shape.n_kv_heads,
                         shape.head_dim, shape.d_ff, shape.vocab, float(shape.rope_theta),
-                        float(shape.rms_eps))
+                        float(shape.rms_eps), float(sc[0]), float(sc[1]), float(sc[2]),
+                        int(sc[3]))
 
 
 class Weights:
     """cc_model_weights over a dict of CUDA bf16 tensors (embed, final_norm,
-    lm_head, layers[l] = {attn_norm, wq, wo, mlp_norm, w_gate, w_up, w_down});
-    keeps the tensors alive."""
+    lm_head, layers[l] = {attn_norm, wq, wo, mlp_norm, w_gate, w_up, w_down,
+    optional bq}); keeps the tensors alive."""
 
     def __init__(self, w: dict):
         self.w = w
@@ -172,6 +178,8 @@ class Weights:
                 continue
             for f in ("attn_norm", "wq", "wo", "mlp_norm", "w_gate", "w_up", "w_down"):
                 setattr(self._layers[l], f, _dev_ptr(lw[f], f"layers[{l}].{f}"))
+            if lw.get("bq") is not None:
+                self._layers[l].bq = _dev_ptr(lw["bq"], f"layers[{l}].bq")
         self.c = cc_model_weights(_dev_ptr(w.get("embed"), "embed"),
                                   _dev_ptr(w["final_norm"], "final_norm"),
                                   _dev_ptr(w["lm_head"], "lm_head"), self._layers)

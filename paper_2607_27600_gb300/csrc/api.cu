@@ -159,6 +159,10 @@ cc_status check_cfg(const cc_model_cfg *c) {
   if (c->head_dim != 64 && c->head_dim != 128) return CC_ERR_UNSUPPORTED;
   if (c->d_model % 32 || c->d_ff % 32) return CC_ERR_UNSUPPORTED;
   if (c->n_q_heads / c->n_kv_heads > 256) return CC_ERR_UNSUPPORTED;
+  if (c->rope_scaling_factor != 0.f &&
+      !(c->rope_scaling_factor >= 1.f && c->rope_low_freq_factor > 0.f &&
+        c->rope_high_freq_factor > c->rope_low_freq_factor && c->rope_original_max_pos > 0))
+    return CC_ERR_INVALID_ARG;
   return CC_OK;
 }
 
@@ -194,10 +198,24 @@ ScoreWs score_layout(const cc_model_cfg *c, int batch, int cap, cc_score_mode mo
 }
 
 // RoPE: inv_freq_k / (2 pi) as 0.64 fixed point (angles reduced exactly on the device).
+// With Llama-3.1 scaling, frequencies of long wavelengths are slowed by the
+// factor, short ones kept, and the band between blended linearly in
+// original_max_pos / wavelength.
 void rope_turns(const cc_model_cfg *c, unsigned long long *turns) {
   const int half = c->head_dim / 2;
   for (int k = 0; k < half; ++k) {
-    const double inv_freq = pow((double)c->rope_theta, -2.0 * k / c->head_dim);
+    double inv_freq = pow((double)c->rope_theta, -2.0 * k / c->head_dim);
+    if (c->rope_scaling_factor != 0.f) {
+      const double f = c->rope_scaling_factor, lo = c->rope_low_freq_factor,
+                   hi = c->rope_high_freq_factor, orig = c->rope_original_max_pos;
+      const double wavelen = 2.0 * M_PI / inv_freq;
+      if (wavelen > orig / lo) {
+        inv_freq /= f;
+      } else if (wavelen >= orig / hi) {
+        const double a = (orig / wavelen - lo) / (hi - lo);
+        inv_freq = (1.0 - a) * inv_freq / f + a * inv_freq;
+      }
+    }
     const double t = inv_freq / (2.0 * M_PI);   // < 1
     turns[k] = (unsigned long long)ldexp(t, 64);
   }
@@ -341,6 +359,7 @@ cc_status check_score_args(const cc_model_cfg *c, const cc_model_weights *w, con
                           kv->k[l], kv->v[l]};
     for (const void *p : ptrs)
       if (!p || !aligned16(p)) return CC_ERR_INVALID_ARG;
+    if (lw.bq && !aligned16(lw.bq)) return CC_ERR_INVALID_ARG;
   }
   const void *ptrs[] = {w->final_norm, w->lm_head, ws, kv->h_last, full ? w->embed : nullptr};
   for (const void *p : ptrs)
@@ -391,6 +410,7 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
     gq.p.out = q;
     gq.p.ldo = qd;
     gq.p.pos = kv->pos;
+    gq.p.bias = reinterpret_cast<const __nv_bfloat16 *>(lw.bq);
     gq.p.head_dim = c->head_dim;
     rope_turns(c, gq.p.turns);
     if ((s = run_gemm(gq, EPI_QROPE, CC_KERNEL_GEMM_QROPE, dev->sms, st)) != CC_OK) return s;

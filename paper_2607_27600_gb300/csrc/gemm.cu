@@ -99,14 +99,27 @@ CC_DEV void epilogue_tile(const GemmParams &p, uint32_t tacc, int grow, bool val
         tmem_ld_wait();
         int col = tile_n0 + hb + c0;
         if (!valid || col >= p.N) continue;
+        uint32_t bb1[16], bb2[16];   // bias pairs of columns col.. and col+half.. (0 if none)
+#pragma unroll
+        for (int v = 0; v < 4; ++v) {
+          uint4 u1 = make_uint4(0, 0, 0, 0), u2 = make_uint4(0, 0, 0, 0);
+          if (p.bias) {
+            u1 = reinterpret_cast<const uint4 *>(p.bias + col)[v];
+            u2 = reinterpret_cast<const uint4 *>(p.bias + col + half)[v];
+          }
+          bb1[v * 4] = u1.x; bb1[v * 4 + 1] = u1.y; bb1[v * 4 + 2] = u1.z; bb1[v * 4 + 3] = u1.w;
+          bb2[v * 4] = u2.x; bb2[v * 4 + 1] = u2.y; bb2[v * 4 + 2] = u2.z; bb2[v * 4 + 3] = u2.w;
+        }
         uint32_t o1[16], o2[16];
 #pragma unroll
         for (int k = 0; k < 32; k += 2) {
           float c_a, s_a, c_b, s_b;
           rope_cs(pos, p.turns[c0 + k], c_a, s_a);
           rope_cs(pos, p.turns[c0 + k + 1], c_b, s_b);
-          float a1 = __uint_as_float(x1[k]), a2 = __uint_as_float(x2[k]);
-          float b1 = __uint_as_float(x1[k + 1]), b2 = __uint_as_float(x2[k + 1]);
+          float a1 = __uint_as_float(x1[k]) + bf16_lo(bb1[k / 2]);
+          float a2 = __uint_as_float(x2[k]) + bf16_lo(bb2[k / 2]);
+          float b1 = __uint_as_float(x1[k + 1]) + bf16_hi(bb1[k / 2]);
+          float b2 = __uint_as_float(x2[k + 1]) + bf16_hi(bb2[k / 2]);
           o1[k / 2] = pack_bf16x2(a1 * c_a - a2 * s_a, b1 * c_b - b2 * s_b);
           o2[k / 2] = pack_bf16x2(a2 * c_a + a1 * s_a, b2 * c_b + b1 * s_b);
         }

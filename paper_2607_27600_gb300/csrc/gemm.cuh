@@ -24,6 +24,7 @@ struct GemmParams {
   const void *resid;
   int ld_resid;
   const int32_t *pos;      // EPI_QROPE
+  const __nv_bfloat16 *bias;  // EPI_QROPE: optional per-column bias added before RoPE
   int head_dim;            // EPI_QROPE
   const int32_t *tokens;   // EPI_LSE
   float *z_target;         // EPI_LSE

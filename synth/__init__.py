@@ -15,6 +15,9 @@ Value recipe (all matrices and the embedding as random-init Llama/Qwen
 weights):
   * weight matrices and embedding: N(0, 0.02^2), rounded to bf16;
   * RMSNorm gains: 1;
+  * q/k/v projection biases (shapes with qkv_bias, as Qwen2.5): N(0, 0.5^2),
+    rounded to bf16 -- comparable to the projected values, whose standard
+    deviation is 0.02 sqrt(d) (about 1.2 at d = 3584);
   * token ids: uniform on [0, vocab);
   * positions: 0, 1, ..., n-1 (original positions of a never-evicted cache);
   * synthetic cached K and V (post-RoPE): N(0, (0.02 sqrt(d))^2), the law of a
@@ -30,6 +33,7 @@ import torch
 from .configs import ModelShape, Workload, WORKLOADS, HEADLINE  # noqa: F401
 
 WEIGHT_STD = 0.02
+BIAS_STD = 0.5
 
 
 def stream_seed(seed: int, name: str) -> int:
@@ -84,6 +88,11 @@ def model_weights(shape: ModelShape, seed: int, device="cpu", with_kv_proj: bool
         if with_kv_proj:
             lw["wk"] = normal((kv, d), WEIGHT_STD, seed, f"l{l}.wk", device)
             lw["wv"] = normal((kv, d), WEIGHT_STD, seed, f"l{l}.wv", device)
+        if shape.qkv_bias:
+            lw["bq"] = normal((q,), BIAS_STD, seed, f"l{l}.bq", device)
+            if with_kv_proj:
+                lw["bk"] = normal((kv,), BIAS_STD, seed, f"l{l}.bk", device)
+                lw["bv"] = normal((kv,), BIAS_STD, seed, f"l{l}.bv", device)
         out["layers"][l] = lw
     return out
 

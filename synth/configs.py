@@ -7,7 +7,7 @@ itself follows Sec. 3.1 (counter-causal surprise, fast single-layer
 approximation) and Algorithm DoMemRefresh of arXiv 2607.27600.
 """
 from dataclasses import dataclass, field
-from typing import List
+from typing import List, Optional, Tuple
 
 
 @dataclass(frozen=True)
@@ -21,6 +21,12 @@ class ModelShape:
     vocab: int
     rope_theta: float
     rms_eps: float
+    # Qwen2-style biases on the q/k/v projections (the scorer uses the q bias;
+    # k/v biases live inside the cached K/V)
+    qkv_bias: bool = False
+    # Llama-3.1 RoPE frequency scaling: (factor, low_freq_factor,
+    # high_freq_factor, original_max_position); None = plain RoPE
+    rope_scaling: Optional[Tuple[float, float, float, int]] = None
 
     @property
     def group(self) -> int:
@@ -63,7 +69,7 @@ TINY = ModelShape(n_layers=1, d_model=512, n_q_heads=8, n_kv_heads=2, head_dim=6
 LLAMA3_8B = ModelShape(n_layers=32, d_model=4096, n_q_heads=32, n_kv_heads=8, head_dim=128,
                        d_ff=14336, vocab=128256, rope_theta=5e5, rms_eps=1e-5)
 QWEN25_7B = ModelShape(n_layers=28, d_model=3584, n_q_heads=28, n_kv_heads=4, head_dim=128,
-                       d_ff=18944, vocab=152064, rope_theta=1e6, rms_eps=1e-6)
+                       d_ff=18944, vocab=152064, rope_theta=1e6, rms_eps=1e-6, qkv_bias=True)
 
 WORKLOADS = {
     # tiny single-layer scoring, cache from a causal pass of the same random model

@@ -55,6 +55,13 @@ def test_host_side_validation_without_device(lib):
     assert lib.cc_score_workspace_size(ctypes.byref(bad), 1, 16, 0) == 0
     odd = cc.cc_model_cfg(1, 256, 8, 2, 96, 256, 10, 1e4, 1e-5)    # head_dim 96
     assert lib.cc_score_workspace_size(ctypes.byref(odd), 1, 16, 0) == 0
+    # RoPE scaling: off when zero, else factor >= 1 and 0 < low < high, orig > 0
+    ok = cc.cc_model_cfg(1, 256, 8, 2, 64, 256, 10, 5e5, 1e-5, 8.0, 1.0, 4.0, 8192)
+    assert lib.cc_score_workspace_size(ctypes.byref(ok), 1, 16, 0) > 0
+    for sc in [(0.5, 1.0, 4.0, 8192), (8.0, 4.0, 1.0, 8192), (8.0, 0.0, 4.0, 8192),
+               (8.0, 1.0, 4.0, 0)]:
+        bad_sc = cc.cc_model_cfg(1, 256, 8, 2, 64, 256, 10, 5e5, 1e-5, *sc)
+        assert lib.cc_score_workspace_size(ctypes.byref(bad_sc), 1, 16, 0) == 0, sc
 
 
 def test_workspace_size_formula(lib):

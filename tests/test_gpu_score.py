@@ -194,3 +194,33 @@ def test_compaction_adversarial_lists_bit_exact(pkg, kind):
     np.testing.assert_array_equal(c["tokens"].cpu().numpy(), oracle.compact(before["tokens"], idx, cnt))
     np.testing.assert_array_equal(c["pos"].cpu().numpy(), oracle.compact(before["pos"], idx, cnt))
     assert c["seq_len"].cpu().tolist() == cnt.tolist()
+
+
+@pytest.mark.parametrize("variant", ["qkv_bias", "rope_scaling", "both"])
+def test_model_variants_bias_and_rope_scaling(pkg, variant):
+    """Qwen2-style q/k/v biases (the scorer adds the q bias before RoPE) and
+    Llama-3.1 RoPE frequency scaling, full and fast pass, every row; the
+    variant must move the scores (no silently ignored bias or table)."""
+    from paper_2607_27600_gb300 import cc
+    extra = {"qkv_bias": variant != "rope_scaling",
+             "rope_scaling": None if variant == "qkv_bias" else (8.0, 1.0, 4.0, 64)}
+    shape = ModelShape(**{**SMALL_GPU.__dict__, **extra})
+    seq, cap = [300, 40, 9], 320
+    w_np = to_np(synth.model_weights(shape, 23, with_kv_proj=True))
+    for lw in w_np["layers"]:
+        if "bv" in lw:
+            # a V bias shared by every slot makes each attention output nearly
+            # that bias whatever the queries are; without it the q bias shows
+            lw["bv"] = lw["bv"] * 0
+    c_np = causal_cache(shape, w_np, seq, cap, seed=23)
+    weights, cache = _gpu(pkg, w_np, c_np)
+    # the same cache scored without the variant's effect on the queries
+    plain = ModelShape(**{**shape.__dict__, "rope_scaling": None})
+    w_plain = {**w_np, "layers": [{k: v for k, v in lw.items() if k != "bq"}
+                                  for lw in w_np["layers"]]}
+    for full, fn in ((True, oracle.score_full), (False, oracle.score_layer)):
+        want = fn(shape, w_np, c_np)
+        got = _run_score(pkg, shape, weights, cache, cc.SCORE_LOGIT, full=full)
+        assert rel_err(got, want) < TOL, (variant, full, rel_err(got, want))
+        other = fn(plain, w_plain, c_np)
+        assert rel_err(other, want) > 5 * TOL, (variant, full, rel_err(other, want))

@@ -179,3 +179,98 @@ def test_sensitivity_bf16_rounding_matches_torch():
                         [1.0 + 2.0 ** -8, 1.0 + 3 * 2.0 ** -8, -(1.0 + 2.0 ** -8), 0.0, -0.0]])
     want = torch.from_numpy(x.astype(np.float32)).to(torch.bfloat16).double().numpy()
     np.testing.assert_array_equal(bf16(x), want)
+
+
+# Llama-3.1 scaling parameters (factor, low_freq_factor, high_freq_factor,
+# original_max_position) at Llama-3's theta and head_dim
+LLAMA31_SCALING = (8.0, 1.0, 4.0, 8192)
+
+
+def test_rope_scaling_none_is_plain_rope():
+    inv = oracle.rope_inv_freq(128, 5e5)
+    np.testing.assert_array_equal(inv, 5e5 ** (-np.arange(64) / 64.0))
+    np.testing.assert_array_equal(oracle.rope_angles(np.array([3]), 128, 5e5),
+                                  oracle.rope_angles(np.array([3]), 128, 5e5, None))
+
+
+def test_rope_scaling_bands():
+    """Three bands by wavelength w = 2 pi / inv_freq: below orig/high the
+    frequency is unchanged, above orig/low it is divided by the factor, and in
+    between the ratio scaled/plain is an affine function of inv_freq that
+    reaches 1 at the short edge and 1/factor at the long edge (continuity)."""
+    factor, low, high, orig = LLAMA31_SCALING
+    plain = oracle.rope_inv_freq(128, 5e5)
+    scaled = oracle.rope_inv_freq(128, 5e5, LLAMA31_SCALING)
+    w = 2 * np.pi / plain
+    short, long_ = w < orig / high, w > orig / low
+    mid = ~short & ~long_
+    assert short.sum() > 10 and long_.sum() > 10 and mid.sum() >= 3
+    np.testing.assert_array_equal(scaled[short], plain[short])
+    np.testing.assert_allclose(scaled[long_], plain[long_] / factor, rtol=1e-15)
+    r = scaled[mid] / plain[mid]
+    assert np.all((r > 1 / factor) & (r < 1))
+    slope, icpt = np.polyfit(plain[mid], r, 1)
+    np.testing.assert_allclose(slope * plain[mid] + icpt, r, rtol=1e-12)
+    edge_short = 2 * np.pi / (orig / high)     # inv_freq at w = orig / high
+    edge_long = 2 * np.pi / (orig / low)
+    assert slope * edge_short + icpt == pytest.approx(1.0, rel=1e-12)
+    assert slope * edge_long + icpt == pytest.approx(1 / factor, rel=1e-12)
+    # monotone: frequencies still decrease with k
+    assert np.all(np.diff(scaled) < 0)
+
+
+def test_projection_bias_closed_form():
+    """Wq = 0 with a q bias b: every row's queries are RoPE(b) at its own
+    position, so attention weights are softmax(RoPE(b_t, pos_i) . K_j / sqrt(dh))
+    over j > i; with W_down = 0 the layer output follows in closed form."""
+    from tests._util import SMALL, small_model, causal_cache
+    shape = SMALL.__class__(**{**SMALL.__dict__, "qkv_bias": True, "n_layers": 1})
+    w = small_model(shape, seed=31)
+    c = causal_cache(shape, w, [9], 10, seed=31)
+    lw = w["layers"][0]
+    assert "bq" in lw and np.abs(lw["bq"]).max() > 0.1
+    lw["wq"][:] = 0
+    lw["w_down"][:] = 0
+    s = oracle.score_layer(shape, w, c)
+    g = shape.n_q_heads // shape.n_kv_heads
+    dh, half = shape.head_dim, shape.head_dim // 2
+    k, v = c["k"][0][0].astype(np.float64), c["v"][0][0].astype(np.float64)
+    for i in range(8):
+        o = []
+        for t in range(shape.n_q_heads):
+            b = lw["bq"][t * dh:(t + 1) * dh].astype(np.float64)
+            z = (b[:half] + 1j * b[half:]) * np.exp(1j * i * shape.rope_theta ** (-np.arange(half) / half))
+            q = np.concatenate([z.real, z.imag])
+            logits = np.array([q @ k[j, t // g] for j in range(i + 1, 9)]) / np.sqrt(dh)
+            p = np.exp(logits - logits.max())
+            o.append((p / p.sum()) @ v[i + 1:9, t // g])
+        h = c["h_last"][0, i] + lw["wo"].astype(np.float64) @ np.concatenate(o)
+        u = h / np.sqrt(np.mean(h * h) + shape.rms_eps)
+        assert s[0, i] == pytest.approx(-u @ w["lm_head"][c["tokens"][0, i]], rel=1e-10)
+
+
+def test_biased_scaled_model_is_rope_shift_invariant():
+    """q/k biases added before RoPE, scaled frequencies: the scores still see
+    only relative offsets (a bias added after the rotation would not)."""
+    from tests._util import SMALL, small_model
+    shape = SMALL.__class__(**{**SMALL.__dict__, "qkv_bias": True,
+                               "rope_scaling": (4.0, 1.0, 4.0, 32)})
+    w = small_model(shape, seed=32)
+    n = 10
+    toks = np.random.default_rng(4).integers(0, shape.vocab, size=n)
+
+    def built(offset):
+        pos = np.arange(n) + offset
+        fw = oracle.causal_forward(shape, w, toks, pos)
+        return {"k": [x[None] for x in fw["k"]], "v": [x[None] for x in fw["v"]],
+                "h_last": fw["h_last"][None], "tokens": toks[None], "pos": pos[None],
+                "seq_len": np.array([n])}
+    s0 = oracle.score_full(shape, w, built(0))
+    np.testing.assert_allclose(oracle.score_full(shape, w, built(5003))[0, :n - 1],
+                               s0[0, :n - 1], rtol=1e-9)
+    # the scaling and the biases do change the scores
+    plain = SMALL.__class__(**{**shape.__dict__, "rope_scaling": None})
+    assert not np.allclose(oracle.score_full(plain, w, built(0))[0, :n - 1], s0[0, :n - 1])
+    w0 = {**w, "layers": [{k_: v_ for k_, v_ in lw.items() if not k_.startswith("b")}
+                          for lw in w["layers"]]}
+    assert not np.allclose(oracle.score_full(shape, w0, built(0))[0, :n - 1], s0[0, :n - 1])
