@@ -274,18 +274,25 @@ cc_status gemm_setup(Gemm &g, int epi, const void *A, int K, const void *W, cons
   g.p.status = status;
   g.p.a_split = a_split ? 1 : 0;
   // Tile order for L2 reuse: keep a slab of <= ~40 MB of one operand resident
-  // while the other streams, choosing the order that moves fewer bytes.
+  // (evict-last) while the other streams past (evict-first).  Weight slabs
+  // resident (raster 0) is the default: a group's tiles of one activation row
+  // tile run on consecutive CTAs, so the streamed row tile is read from DRAM
+  // about once per group, and on the Llama-3-8B projections (K = 4096 and
+  // 14336) this order measured 2-4 % faster than the activation-resident one
+  // even where a count of whole-slab re-reads favoured the latter by up to
+  // 16 %.  The activation-resident order is taken only when that count is
+  // below 0.8x (an LM head whose weight is far larger than L2).
   const double budget = 40.0 * (1 << 20);
   const int num_m = (int)((R + 127) / 128), num_n = g.p.n_tiles;
   const double k_a = (a_split ? 2.0 : 1.0) * K;
   const double a_bytes = (double)R * k_a * 2, b_bytes = (double)num_n * 256 * K * 2;
   const double a_slab = 128.0 * k_a * 2, b_slab = 256.0 * K * 2;
-  const int gn = (int)std::max(1.0, std::min((double)num_n, budget / b_slab));
-  const int gm = (int)std::max(1.0, std::min((double)num_m, budget / a_slab));
+  const int gn = (int)std::max(1.0, std::min((double)num_n, floor(budget / b_slab)));
+  const int gm = (int)std::max(1.0, std::min((double)num_m, floor(budget / a_slab)));
   const double t0 = b_bytes + a_bytes * ((num_n + gn - 1) / gn);
   const double t1 = a_bytes + b_bytes * ((num_m + gm - 1) / gm);
-  g.p.raster = t0 <= t1 ? 0 : 1;
-  g.p.group = t0 <= t1 ? gn : gm;
+  g.p.raster = t1 < 0.8 * t0 ? 1 : 0;
+  g.p.group = g.p.raster == 0 ? gn : gm;
   return CC_OK;
 }
 
