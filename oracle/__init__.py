@@ -23,10 +23,16 @@ Parity status per function (what pins it, in tests/test_oracle_*.py):
                            (full == single-layer) invariants
   select_keep              brute-force sort on tiny inputs; forced keeps; identity
   compact                  sequential in-place loop; order preservation
+  memory_causal_attention  torch SDPA with an explicit mask (memory all visible,
+                           chunk causal); n0 = 0 is causal_attention
+  append_chunk             into an empty cache = causal_forward; chunk-by-chunk
+                           appends = one append (no refresh between); the layer's
+                           attention after a compaction by scalar brute force
 The paper prints no worked example with score values, so no pin is a
 printed number; every step of the score is pinned by the checks above.
 """
 from .refresh import (rms_norm, rope, rope_angles, rope_inv_freq, project, softmax,  # noqa: F401
                       counter_causal_attention,
                       causal_attention, silu, swiglu_mlp, counter_causal_layer, score_head,
-                      score_layer, score_full, select_keep, compact, causal_forward)
+                      score_layer, score_full, select_keep, compact, causal_forward,
+                      memory_causal_attention, append_chunk)

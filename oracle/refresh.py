@@ -341,3 +341,73 @@ def causal_forward(shape, weights, tokens, pos):
         m = rms_norm(h, lw["mlp_norm"], shape.rms_eps)
         h = h + swiglu_mlp(m, lw)
     return {"k": ks, "v": vs, "h_last": h_last, "h_final": h}
+
+
+# ----------------------------------------------------------------------------
+# Inference cycle in pre-fill (Algorithm CacheManagedInference / DoInference,
+# chunked mode): a chunk of new tokens runs causally through every layer over
+# the memory the cache holds, and their K, V, tokens, positions and H^(L-1)
+# are appended
+# ----------------------------------------------------------------------------
+
+def memory_causal_attention(q, k, v, n0):
+    """Memory-augmented causal attention (Eq. 3 with the causal mask): chunk
+    row r (cache slot n0 + r) attends every memory slot j < n0 and the chunk
+    slots up to and including its own, i.e. keys j <= n0 + r of the
+    concatenation [K' ; K].  q [h, Hq, dh]; k, v [>= n0 + h, Hkv, dh]."""
+    q = f64(q)
+    h, hq, dh = q.shape
+    hkv = k.shape[1]
+    group = hq // hkv
+    out = np.zeros((h, hq, dh))
+    for r in range(h):
+        last = n0 + r
+        for g in range(hkv):
+            heads = slice(g * group, (g + 1) * group)
+            s = q[r, heads] @ f64(k[:last + 1, g]).T / np.sqrt(dh)
+            out[r, heads] = softmax(s) @ f64(v[:last + 1, g])
+    return out
+
+
+def append_chunk(shape, weights, cache, b, tokens, pos=None):
+    """Append a chunk of tokens to sequence b of `cache` (modified in place):
+    the inference cycle of Algorithm DoInference run over a chunk in batch, as
+    in pre-fill.  Per layer the chunk's queries, keys and values come from its
+    own hidden states (keys and queries rotated at the chunk's positions), the
+    keys and values are written after the sequence's current slots
+    (K <- K (+) k_t, V <- V (+) v_t), and attention sees the memory slots
+    already cached plus the chunk causally (memory_causal_attention).  The
+    tokens (X <- X (+) x_t), positions and H^(L-1) (the input of the last
+    layer, recorded for the fast approximation) are written too, and
+    seq_len[b] grows by the chunk length.  pos defaults to the positions
+    following the last cached one.  Returns the chunk's final hidden states."""
+    n0 = int(cache["seq_len"][b])
+    tokens = np.asarray(tokens)
+    h = len(tokens)
+    if pos is None:
+        start = int(cache["pos"][b][n0 - 1]) + 1 if n0 > 0 else 0
+        pos = np.arange(start, start + h)
+    pos = np.asarray(pos)
+    sl = slice(n0, n0 + h)
+    x = f64(weights["embed"][tokens])
+    sc = getattr(shape, "rope_scaling", None)
+    for l in range(shape.n_layers):
+        lw = weights["layers"][l]
+        if l == shape.n_layers - 1 and cache.get("h_last") is not None:
+            cache["h_last"][b][sl] = x
+        a = rms_norm(x, lw["attn_norm"], shape.rms_eps)
+        q = rope(project(a, lw, "wq").reshape(h, shape.n_q_heads, shape.head_dim), pos,
+                 shape.rope_theta, sc)
+        k = rope(project(a, lw, "wk").reshape(h, shape.n_kv_heads, shape.head_dim), pos,
+                 shape.rope_theta, sc)
+        v = project(a, lw, "wv").reshape(h, shape.n_kv_heads, shape.head_dim)
+        cache["k"][l][b][sl] = k
+        cache["v"][l][b][sl] = v
+        o = memory_causal_attention(q, cache["k"][l][b], cache["v"][l][b], n0)
+        x = x + o.reshape(h, -1) @ f64(lw["wo"]).T
+        m = rms_norm(x, lw["mlp_norm"], shape.rms_eps)
+        x = x + swiglu_mlp(m, lw)
+    cache["tokens"][b][sl] = tokens
+    cache["pos"][b][sl] = pos
+    cache["seq_len"][b] = n0 + h
+    return x
