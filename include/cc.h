@@ -100,8 +100,13 @@ typedef struct {
   const void *w_up;      /* [d_ff][d_model]                  */
   const void *w_down;    /* [d_model][d_ff]                  */
   const void *bq;        /* optional [n_q_heads*head_dim] q-projection bias (Qwen2-style
-                            attention), added before RoPE; NULL = none; 16-byte aligned.
-                            K/V biases belong to the cache builder: cached K/V hold them */
+                            attention), added before RoPE; NULL = none; 16-byte aligned   */
+  /* Key/value projections, read only by cc_append_chunk (the scoring passes
+   * reuse the cached K/V and may leave them NULL). */
+  const void *wk;        /* [n_kv_heads*head_dim][d_model]   */
+  const void *wv;        /* [n_kv_heads*head_dim][d_model]   */
+  const void *bk;        /* optional [n_kv_heads*head_dim] bias (before RoPE); NULL = none */
+  const void *bv;        /* optional [n_kv_heads*head_dim] bias; NULL = none              */
 } cc_layer_weights;
 
 typedef struct {
@@ -177,6 +182,34 @@ size_t cc_compact_workspace_size(const cc_model_cfg *cfg, const cc_kv_cache *cac
 cc_status cc_compact_kv(const cc_model_cfg *cfg, const cc_kv_cache *cache,
                         const int32_t *keep_idx, const int32_t *keep_count, void *ws,
                         size_t ws_bytes, void *stream);
+
+/* ---- inference cycle, pre-fill (Algorithm CacheManagedInference with
+ * DoInference over a chunk of tokens in batch, chunked refresh mode) -------
+ * Appends count[b] tokens to sequence b after its seq_len[b] cached slots:
+ * the chunk runs through every layer l with queries, keys and values from
+ * its own hidden states (keys and queries rotated at the chunk's positions),
+ * writes its keys and values into k[l], v[l] at slots [seq_len[b],
+ * seq_len[b] + count[b]) (K <- K (+) k_t, V <- V (+) v_t), and attends every
+ * cached memory slot plus the chunk causally (memory-augmented attention,
+ * Eq. 3, causal mask: the chunk's slot i sees slots j <= i).  The chunk's
+ * tokens (X <- X (+) x_t) and positions are written to tokens and pos, the
+ * input of the last layer to h_last (if non-NULL, for the fast
+ * approximation), and seq_len[b] grows by count[b].  No next token is
+ * sampled (pre-fill).
+ *   tokens_in: device int32 [batch][max_count], row b holds count[b] ids.
+ *   pos_in:    device int32 [batch][max_count] original positions, or NULL:
+ *              the positions following pos[b][seq_len[b]-1] (0 when empty).
+ *   count:     device int32 [batch]; a count outside [0, max_count] or past
+ *              cap sets CC_ERR_DEVICE_ARG on the device and appends nothing
+ *              to that sequence.
+ * Needs embed and, for every layer, wq, wk, wv, wo, the norms and the MLP
+ * (biases optional); every k[l], v[l] non-NULL.  Asynchronous on `stream`;
+ * the workspace is that of cc_append_workspace_size. */
+size_t cc_append_workspace_size(const cc_model_cfg *cfg, int32_t batch, int32_t cap);
+cc_status cc_append_chunk(const cc_model_cfg *cfg, const cc_model_weights *w,
+                          const cc_kv_cache *cache, const int32_t *tokens_in,
+                          const int32_t *pos_in, const int32_t *count, int32_t max_count,
+                          void *ws, size_t ws_bytes, void *stream);
 
 /* ---- compaction without a workspace -----------------------------------------
  * The paper has no counterpart: this is a library convenience.

@@ -30,7 +30,10 @@ typedef enum {
   CC_KERNEL_SELECT = 10,     /* keep-set radix select                             */
   CC_KERNEL_COMPACT = 11,    /* in-place compaction                               */
   CC_KERNEL_OTHER = 12,      /* kernel-level entry points (cc_kernels.h)          */
-  CC_KERNEL_COUNT = 13
+  CC_KERNEL_GEMM_KV = 13,    /* key (+ RoPE) and value projections (append)       */
+  CC_KERNEL_ATTN_CAUSAL = 14,/* memory-augmented causal attention (append)        */
+  CC_KERNEL_APPEND = 15,     /* append bookkeeping: tokens, positions, H^(L-1)    */
+  CC_KERNEL_COUNT = 16
 } cc_kernel_kind;
 
 /* on != 0: start recording (also clears earlier records); 0: stop. */

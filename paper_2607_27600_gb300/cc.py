@@ -47,7 +47,8 @@ class cc_model_cfg(ctypes.Structure):
 
 class cc_layer_weights(ctypes.Structure):
     _fields_ = [(n, ctypes.c_void_p) for n in
-                ("attn_norm", "wq", "wo", "mlp_norm", "w_gate", "w_up", "w_down", "bq")]
+                ("attn_norm", "wq", "wo", "mlp_norm", "w_gate", "w_up", "w_down", "bq",
+                 "wk", "wv", "bk", "bv")]
 
 
 class cc_model_weights(ctypes.Structure):
@@ -72,6 +73,12 @@ _SIGS = {
     "cc_score_full": (ctypes.c_int, [ctypes.POINTER(cc_model_cfg), ctypes.POINTER(cc_model_weights),
                                      ctypes.POINTER(cc_kv_cache), ctypes.c_int, ctypes.c_void_p,
                                      ctypes.c_void_p, ctypes.c_size_t, ctypes.c_void_p]),
+    "cc_append_workspace_size": (ctypes.c_size_t, [ctypes.POINTER(cc_model_cfg), ctypes.c_int32,
+                                                   ctypes.c_int32]),
+    "cc_append_chunk": (ctypes.c_int, [ctypes.POINTER(cc_model_cfg), ctypes.POINTER(cc_model_weights),
+                                       ctypes.POINTER(cc_kv_cache), ctypes.c_void_p, ctypes.c_void_p,
+                                       ctypes.c_void_p, ctypes.c_int32, ctypes.c_void_p,
+                                       ctypes.c_size_t, ctypes.c_void_p]),
     "cc_select_workspace_size": (ctypes.c_size_t, [ctypes.c_int32, ctypes.c_int32]),
     "cc_select_keep": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int32,
                                       ctypes.c_int32, ctypes.c_void_p, ctypes.c_int32,
@@ -99,7 +106,7 @@ _SIGS = {
     "cc_kernel_name": (ctypes.c_char_p, [ctypes.c_int32]),
     "cc_debug_withhold_compact_unit": (ctypes.c_int, [ctypes.c_int32]),
 }
-KERNEL_COUNT = 13
+KERNEL_COUNT = 16
 
 
 def library_path() -> str:
@@ -167,7 +174,7 @@ def model_cfg(shape) -> cc_model_cfg:
 class Weights:
     """cc_model_weights over a dict of CUDA bf16 tensors (embed, final_norm,
     lm_head, layers[l] = {attn_norm, wq, wo, mlp_norm, w_gate, w_up, w_down,
-    optional bq}); keeps the tensors alive."""
+    optional bq, and wk, wv, bk, bv for the append}); keeps the tensors alive."""
 
     def __init__(self, w: dict):
         self.w = w
@@ -178,8 +185,9 @@ class Weights:
                 continue
             for f in ("attn_norm", "wq", "wo", "mlp_norm", "w_gate", "w_up", "w_down"):
                 setattr(self._layers[l], f, _dev_ptr(lw[f], f"layers[{l}].{f}"))
-            if lw.get("bq") is not None:
-                self._layers[l].bq = _dev_ptr(lw["bq"], f"layers[{l}].bq")
+            for f in ("bq", "wk", "wv", "bk", "bv"):   # optional (wk, wv: append only)
+                if lw.get(f) is not None:
+                    setattr(self._layers[l], f, _dev_ptr(lw[f], f"layers[{l}].{f}"))
         self.c = cc_model_weights(_dev_ptr(w.get("embed"), "embed"),
                                   _dev_ptr(w["final_norm"], "final_norm"),
                                   _dev_ptr(w["lm_head"], "lm_head"), self._layers)
@@ -236,6 +244,22 @@ def cc_score_layer(cfg, weights, cache, mode, scores, ws, stream=None):
 
 def cc_score_full(cfg, weights, cache, mode, scores, ws, stream=None):
     _score("cc_score_full", cfg, weights, cache, mode, scores, ws, stream)
+
+
+def cc_append_workspace_size(cfg, batch: int, cap: int) -> int:
+    return int(load_library().cc_append_workspace_size(ctypes.byref(_cfg(cfg)), batch, cap))
+
+
+def cc_append_chunk(cfg, weights, cache, tokens_in, pos_in, count, max_count: int, ws,
+                    stream=None):
+    """Inference cycle in pre-fill: append count[b] tokens (tokens_in [B, max_count]
+    int32, positions pos_in or None) to every sequence of `cache`, all layers."""
+    c = _cfg(cfg)
+    code = load_library().cc_append_chunk(
+        ctypes.byref(c), ctypes.byref(weights.c), ctypes.byref(cache.c),
+        _dev_ptr(tokens_in, "tokens_in"), _dev_ptr(pos_in, "pos_in"), _dev_ptr(count, "count"),
+        int(max_count), _dev_ptr(ws, "ws"), ws.numel() * ws.element_size(), _stream(stream))
+    _check(code, "cc_append_chunk")
 
 
 def cc_select_workspace_size(batch: int, cap: int) -> int:

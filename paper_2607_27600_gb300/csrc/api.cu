@@ -252,9 +252,11 @@ struct Gemm {
 
 // One GEMM over the cache rows: A [R][K] (bf16 workspace) x W [N][K]^T.
 // a_split: A rows are [hi | lo] (2K values) and the product is hi W^T + lo W^T.
+// rows_hint: rows the GEMM visits at most (the traffic model's A size; 0 =
+// every slot of the batch).
 cc_status gemm_setup(Gemm &g, int epi, const void *A, int K, const void *W, const void *W2, int N,
                      int batch, int cap, const int32_t *seq_len, unsigned *status,
-                     bool a_split = false) {
+                     bool a_split = false, uint64_t rows_hint = 0) {
   const uint64_t R = (uint64_t)batch * cap;
   const int bn = gemm_block_n(epi);
   if (!tmap_rows(&g.a, A, R, a_split ? 2 * K : K, 128)) return tmap_fail();
@@ -283,9 +285,10 @@ cc_status gemm_setup(Gemm &g, int epi, const void *A, int K, const void *W, cons
   // 16 %.  The activation-resident order is taken only when that count is
   // below 0.8x (an LM head whose weight is far larger than L2).
   const double budget = 40.0 * (1 << 20);
-  const int num_m = (int)((R + 127) / 128), num_n = g.p.n_tiles;
+  const uint64_t R_used = rows_hint ? rows_hint : R;
+  const int num_m = (int)((R_used + 127) / 128), num_n = g.p.n_tiles;
   const double k_a = (a_split ? 2.0 : 1.0) * K;
-  const double a_bytes = (double)R * k_a * 2, b_bytes = (double)num_n * 256 * K * 2;
+  const double a_bytes = (double)R_used * k_a * 2, b_bytes = (double)num_n * 256 * K * 2;
   const double a_slab = 128.0 * k_a * 2, b_slab = 256.0 * K * 2;
   const int gn = (int)std::max(1.0, std::min((double)num_n, floor(budget / b_slab)));
   const int gm = (int)std::max(1.0, std::min((double)num_m, floor(budget / a_slab)));
@@ -303,9 +306,13 @@ cc_status run_gemm(Gemm &g, int epi, int kind, int sms, cudaStream_t st) {
 }
 
 // out: [R][Hq*dh] bf16, or with split [R][2*Hq*dh] = [hi | lo] per row.
+// Counter-causal attention over rows [0, seq_len); with row_lo, the causal
+// memory-augmented attention of the inference cycle over rows
+// [row_lo, seq_len) (q_span: rows per sequence at most).
 cc_status run_attention(const cc_model_cfg *c, const void *q, const void *k, const void *v,
                         void *out, const int32_t *seq_len, int batch, int cap, unsigned *status,
-                        cudaStream_t st, bool split = false) {
+                        cudaStream_t st, bool split = false, const int32_t *row_lo = nullptr,
+                        int q_span = 0) {
   const int G = c->n_q_heads / c->n_kv_heads, dh = c->head_dim;
   const int P = attn_positions_per_unit(G);
   const uint64_t R = (uint64_t)batch * cap;
@@ -337,8 +344,159 @@ cc_status run_attention(const cc_model_cfg *c, const void *q, const void *k, con
   p.out_lo = split ? c->n_q_heads * dh : 0;
   p.scale_log2 = (float)(1.4426950408889634 / sqrt((double)dh));
   p.status = status;
-  TimedScope t(CC_KERNEL_ATTENTION, st);
+  p.causal = row_lo ? 1 : 0;
+  p.row_lo = row_lo;
+  p.q_span = row_lo ? q_span : cap;
+  TimedScope t(row_lo ? CC_KERNEL_ATTN_CAUSAL : CC_KERNEL_ATTENTION, st);
   CC_TRY(launch_attention(tq, tk, tv, p, st));
+  return CC_OK;
+}
+
+// ---------------------------------------------------------------------------
+// inference cycle, pre-fill: chunk append over the memory
+// ---------------------------------------------------------------------------
+struct AppendWs {
+  ScoreWs s;          // xn, q, o, h, act rows b*cap + slot (the chunk's rows only are used)
+  size_t lo, hi, total;
+};
+
+AppendWs append_layout(const cc_model_cfg *c, int batch, int cap) {
+  AppendWs w{};
+  w.s = score_layout(c, batch, cap, CC_SCORE_LOGIT, false);
+  size_t off = w.s.total;
+  w.lo = off;
+  off = align256(off + (size_t)batch * 4);
+  w.hi = off;
+  off = align256(off + (size_t)batch * 4);
+  w.total = off;
+  return w;
+}
+
+cc_status check_append_args(const cc_model_cfg *c, const cc_model_weights *w,
+                            const cc_kv_cache *kv, const int32_t *tokens_in,
+                            const int32_t *count, int max_count, void *ws, size_t ws_bytes) {
+  cc_status s = check_cfg(c);
+  if (s != CC_OK) return s;
+  if (!w || !kv || !w->layers || !w->embed || !kv->k || !kv->v || !tokens_in || !count ||
+      max_count < 0)
+    return CC_ERR_INVALID_ARG;
+  if (kv->batch < 1 || kv->cap < 1 || !kv->seq_len || !kv->tokens || !kv->pos)
+    return CC_ERR_INVALID_ARG;
+  if (kv->batch > gemm_max_batch()) return CC_ERR_UNSUPPORTED;
+  if ((uint64_t)kv->batch * kv->cap >= (1ull << 31)) return CC_ERR_UNSUPPORTED;
+  for (int l = 0; l < c->n_layers; ++l) {
+    const cc_layer_weights &lw = w->layers[l];
+    const void *ptrs[] = {lw.attn_norm, lw.wq, lw.wk, lw.wv, lw.wo, lw.mlp_norm, lw.w_gate,
+                          lw.w_up, lw.w_down, kv->k[l], kv->v[l]};
+    for (const void *p : ptrs)
+      if (!p || !aligned16(p)) return CC_ERR_INVALID_ARG;
+    const void *opt[] = {lw.bq, lw.bk, lw.bv};
+    for (const void *p : opt)
+      if (p && !aligned16(p)) return CC_ERR_INVALID_ARG;
+  }
+  if (!aligned16(w->embed) || (kv->h_last && !aligned16(kv->h_last))) return CC_ERR_INVALID_ARG;
+  if (!ws || !aligned16(ws) || ws_bytes < append_layout(c, kv->batch, kv->cap).total)
+    return CC_ERR_WORKSPACE;
+  return CC_OK;
+}
+
+cc_status run_append(const cc_model_cfg *c, const cc_model_weights *w, const cc_kv_cache *kv,
+                     const int32_t *tokens_in, const int32_t *pos_in, const int32_t *count,
+                     int max_count, void *ws, size_t ws_bytes, void *stream) {
+  cc_status s = check_append_args(c, w, kv, tokens_in, count, max_count, ws, ws_bytes);
+  if (s != CC_OK) return s;
+  if (max_count == 0) return CC_OK;
+  DevState *dev;
+  if (!dev_state(&dev)) return device_fail();
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  const int batch = kv->batch, cap = kv->cap, rows = batch * cap;
+  const int d = c->d_model, qd = c->n_q_heads * c->head_dim, kvd = c->n_kv_heads * c->head_dim;
+  const int f = c->d_ff;
+  const AppendWs L = append_layout(c, batch, cap);
+  uint8_t *wsb = reinterpret_cast<uint8_t *>(ws);
+  void *xn = wsb + L.s.xn, *q = wsb + L.s.q, *o = wsb + L.s.o, *act = wsb + L.s.act;
+  float *h = reinterpret_cast<float *>(wsb + L.s.h);
+  int32_t *lo = reinterpret_cast<int32_t *>(wsb + L.lo), *hi = reinterpret_cast<int32_t *>(wsb + L.hi);
+  unsigned *status = dev->status;
+  const uint64_t used = (uint64_t)batch * max_count;   // rows the GEMMs visit at most
+
+  {
+    TimedScope t(CC_KERNEL_APPEND, st);
+    CC_TRY(launch_append_prepare(kv->seq_len, count, tokens_in, pos_in, max_count, kv->tokens,
+                                 kv->pos, lo, hi, batch, cap, status, st));
+  }
+  {
+    TimedScope t(CC_KERNEL_EMBED, st);
+    CC_TRY(launch_embed(w->embed, kv->tokens, h, d, c->vocab, hi, cap, rows, status, st, lo));
+  }
+  for (int l = 0; l < c->n_layers; ++l) {
+    const cc_layer_weights &lw = w->layers[l];
+    if (l == c->n_layers - 1 && kv->h_last) {   // H^(L-1), recorded for the fast approximation
+      TimedScope t(CC_KERNEL_APPEND, st);
+      CC_TRY(launch_store_bf16(h, kv->h_last, d, hi, lo, cap, rows, st));
+    }
+    {
+      TimedScope t(CC_KERNEL_RMSNORM, st);
+      CC_TRY(launch_rmsnorm(h, true, lw.attn_norm, xn, d, c->rms_eps, hi, cap, rows, false, st, lo));
+    }
+    // q = RoPE(xn Wq^T + bq) into the workspace; k = RoPE(xn Wk^T + bk) and
+    // v = xn Wv^T + bv straight into the cache slots of the chunk
+    struct Proj { const void *w, *bias; void *out; int n, epi, kind; };
+    const Proj projs[3] = {{lw.wq, lw.bq, q, qd, EPI_QROPE, CC_KERNEL_GEMM_QROPE},
+                           {lw.wk, lw.bk, kv->k[l], kvd, EPI_QROPE, CC_KERNEL_GEMM_KV},
+                           {lw.wv, lw.bv, kv->v[l], kvd, EPI_BF16, CC_KERNEL_GEMM_KV}};
+    for (const Proj &pj : projs) {
+      Gemm g;
+      if ((s = gemm_setup(g, pj.epi, xn, d, pj.w, nullptr, pj.n, batch, cap, hi, status, false,
+                          used)) != CC_OK)
+        return s;
+      g.p.row_lo = lo;
+      g.p.out = pj.out;
+      g.p.ldo = pj.n;
+      g.p.pos = kv->pos;
+      g.p.bias = reinterpret_cast<const __nv_bfloat16 *>(pj.bias);
+      g.p.head_dim = c->head_dim;
+      if (pj.epi == EPI_QROPE) rope_turns(c, g.p.turns);
+      if ((s = run_gemm(g, pj.epi, pj.kind, dev->sms, st)) != CC_OK) return s;
+    }
+    // o = attention of the chunk rows over the memory and the chunk (causal)
+    if ((s = run_attention(c, q, kv->k[l], kv->v[l], o, hi, batch, cap, status, st, false, lo,
+                           max_count)) != CC_OK)
+      return s;
+    // h += o Wo^T; xn = RMSNorm(h); act = SwiGLU; h += act Wd^T
+    Gemm go;
+    if ((s = gemm_setup(go, EPI_RESID_F32, o, qd, lw.wo, nullptr, d, batch, cap, hi, status,
+                        false, used)) != CC_OK)
+      return s;
+    go.p.row_lo = lo;
+    go.p.out = h;
+    go.p.ldo = d;
+    if ((s = run_gemm(go, EPI_RESID_F32, CC_KERNEL_GEMM_OPROJ, dev->sms, st)) != CC_OK) return s;
+    {
+      TimedScope t(CC_KERNEL_RMSNORM, st);
+      CC_TRY(launch_rmsnorm(h, true, lw.mlp_norm, xn, d, c->rms_eps, hi, cap, rows, false, st, lo));
+    }
+    Gemm gu;
+    if ((s = gemm_setup(gu, EPI_SWIGLU, xn, d, lw.w_gate, lw.w_up, f, batch, cap, hi, status,
+                        false, used)) != CC_OK)
+      return s;
+    gu.p.row_lo = lo;
+    gu.p.out = act;
+    gu.p.ldo = f;
+    if ((s = run_gemm(gu, EPI_SWIGLU, CC_KERNEL_GEMM_GATEUP, dev->sms, st)) != CC_OK) return s;
+    Gemm gd;
+    if ((s = gemm_setup(gd, EPI_RESID_F32, act, f, lw.w_down, nullptr, d, batch, cap, hi, status,
+                        false, used)) != CC_OK)
+      return s;
+    gd.p.row_lo = lo;
+    gd.p.out = h;
+    gd.p.ldo = d;
+    if ((s = run_gemm(gd, EPI_RESID_F32, CC_KERNEL_GEMM_DOWN, dev->sms, st)) != CC_OK) return s;
+  }
+  {
+    TimedScope t(CC_KERNEL_APPEND, st);
+    CC_TRY(launch_append_finish(kv->seq_len, hi, batch, st));
+  }
   return CC_OK;
 }
 
@@ -569,6 +727,18 @@ cc_status compact_bind(CompactPlan &plan, void *ws, cudaStream_t st) {
 // ===========================================================================
 extern "C" {
 
+size_t cc_append_workspace_size(const cc_model_cfg *cfg, int32_t batch, int32_t cap) {
+  if (check_cfg(cfg) != CC_OK || batch < 1 || cap < 1) return 0;
+  return append_layout(cfg, batch, cap).total;
+}
+
+cc_status cc_append_chunk(const cc_model_cfg *cfg, const cc_model_weights *w,
+                          const cc_kv_cache *cache, const int32_t *tokens_in,
+                          const int32_t *pos_in, const int32_t *count, int32_t max_count,
+                          void *ws, size_t ws_bytes, void *stream) {
+  return run_append(cfg, w, cache, tokens_in, pos_in, count, max_count, ws, ws_bytes, stream);
+}
+
 size_t cc_score_workspace_size(const cc_model_cfg *cfg, int32_t batch, int32_t cap,
                                cc_score_mode mode) {
   if (check_cfg(cfg) != CC_OK || batch < 1 || cap < 1) return 0;
@@ -751,7 +921,8 @@ cc_status cc_debug_withhold_compact_unit(int32_t unit) {
 const char *cc_kernel_name(int32_t kind) {
   static const char *names[CC_KERNEL_COUNT] = {
       "rmsnorm", "embed", "gemm_qrope", "attention", "gemm_oproj", "gemm_gateup", "gemm_down",
-      "head_logit", "gemm_lmhead", "lse_combine", "select", "compact", "other"};
+      "head_logit", "gemm_lmhead", "lse_combine", "select", "compact", "other",
+      "gemm_kv", "attention_causal", "append"};
   return (kind >= 0 && kind < CC_KERNEL_COUNT) ? names[kind] : "unknown";
 }
 

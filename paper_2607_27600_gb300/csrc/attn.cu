@@ -1,6 +1,10 @@
 // attn.cu -- counter-causal flash attention on tcgen05 (Sec. 3.1: fresh
 // queries, cached post-RoPE K/V reused, row i attends only slots j with
-// i < j < n).
+// i < j < n).  The same kernel, CAUSAL = true, runs the inference cycle's
+// memory-augmented attention (Eq. 3 with the causal mask): the chunk's rows
+// [row_lo, n) attend slots j <= i, i.e. every memory slot and the chunk
+// causally; key tiles then run from the one holding the block's last row
+// down to slot 0.
 //
 // One CTA = one work unit (sequence b, KV head g, block of P positions).
 // The unit's query rows are the G = Hq/Hkv heads of group g at P
@@ -101,7 +105,7 @@ struct AttnSmem {
   static constexpr int BYTES = OFF_BAR + 256 + 1024;   // barriers + alignment slack
 };
 
-template <int DH>
+template <int DH, bool CAUSAL>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                 const __grid_constant__ CUtensorMap tmV, const __grid_constant__ AttnParams p) {
@@ -130,7 +134,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   // group's streams innermost.  The group size bounds how far apart in time
   // two resident units of one stream read the same K/V tile (chosen so the
   // K/V read in between stays well inside L2).
-  const int blocks_per_stream = (p.cap + P - 1) / P;
+  const int blocks_per_stream = (p.q_span + P - 1) / P;
   const int n_streams = p.batch * p.n_kv_heads;
   const int per_group = p.streams_per_group * blocks_per_stream;
   const int grp = blockIdx.x / per_group;
@@ -141,14 +145,17 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int stream = s0 + (r - pb * gsz);
   const int b = stream / p.n_kv_heads, g = stream - b * p.n_kv_heads;
   int n = p.seq_len[b];
-  if (n < 0 || n > p.cap) {
+  const int q_lo = CAUSAL ? p.row_lo[b] : 0;   // first query slot
+  if (n < 0 || n > p.cap || q_lo < 0 || q_lo > n) {
     if (threadIdx.x == 0) set_status(p.status, CC_ERR_DEVICE_ARG);
     return;
   }
-  const int p0 = pb * P;
+  const int p0 = q_lo + pb * P;
   if (p0 >= n) return;                       // the whole block lies past the sequence end
   const int p_last = min(p0 + P, n) - 1;     // last valid position of the block
-  const int t0 = (p0 + 1) / BKV, t1 = (n - 1) / BKV;
+  // counter-causal: key tiles holding slots p0+1 .. n-1; causal: slots 0 .. p_last
+  const int t0 = CAUSAL ? 0 : (p0 + 1) / BKV;
+  const int t1 = CAUSAL ? p_last / BKV : (n - 1) / BKV;
   const int ntiles = t1 - t0 + 1;
   const size_t row_base = (size_t)b * p.cap;
 
@@ -365,11 +372,11 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
       for (int u = 0; u < 8; ++u) mp[u] = -INFINITY;
       // uniform over the CTA: rows past P*G have zero queries and need no mask
-      const bool need_mask = (j0 <= p0 + P - 1) || (j0 + BKV > n);
+      const bool need_mask = CAUSAL ? (j0 + BKV - 1 > p0) : ((j0 <= p0 + P - 1) || (j0 + BKV > n));
       if (need_mask) {
-        // key j kept iff pos < j < n
-        const int lo = pos - j0;       // keep c > lo
-        const int hi = n - j0;         // keep c < hi
+        // counter-causal: key j kept iff pos < j < n; causal: iff j <= min(pos, n - 1)
+        const int lo = CAUSAL ? -1 : pos - j0;                    // keep c > lo
+        const int hi = CAUSAL ? min(pos, n - 1) - j0 + 1 : n - j0;   // keep c < hi
 #pragma unroll
         for (int c = 0; c < 128; ++c) {
           float x = (c > lo && c < hi) ? __uint_as_float(sr[c]) : -INFINITY;
@@ -493,10 +500,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-template <int DH>
+template <int DH, bool CAUSAL>
 cudaError_t launch_dh(const CUtensorMap &q, const CUtensorMap &k, const CUtensorMap &v,
                       const AttnParams &p, cudaStream_t stream) {
-  auto kern = attn_kernel<DH>;
+  auto kern = attn_kernel<DH, CAUSAL>;
   static bool attr_set[64] = {};
   int dev = 0;
   cudaGetDevice(&dev);
@@ -506,7 +513,7 @@ cudaError_t launch_dh(const CUtensorMap &q, const CUtensorMap &k, const CUtensor
     if (e != cudaSuccess) return e;
     attr_set[dev] = true;
   }
-  const long long units = (long long)p.batch * p.n_kv_heads * ((p.cap + p.P - 1) / p.P);
+  const long long units = (long long)p.batch * p.n_kv_heads * ((p.q_span + p.P - 1) / p.P);
   if (units <= 0) return cudaSuccess;
   // Resident units of one stream start about T / (SMs / streams) apart (T a
   // unit's run time), so between two reads of a K/V tile the resident units
@@ -539,8 +546,13 @@ extern "C" int cc_debug_attn_trace(unsigned long long *out, int n) {
 
 cudaError_t launch_attention(const CUtensorMap &q, const CUtensorMap &k, const CUtensorMap &v,
                              const AttnParams &p, cudaStream_t stream) {
-  if (p.head_dim == 128) return launch_dh<128>(q, k, v, p, stream);
-  if (p.head_dim == 64) return launch_dh<64>(q, k, v, p, stream);
+  if (p.causal) {
+    if (p.head_dim == 128) return launch_dh<128, true>(q, k, v, p, stream);
+    if (p.head_dim == 64) return launch_dh<64, true>(q, k, v, p, stream);
+  } else {
+    if (p.head_dim == 128) return launch_dh<128, false>(q, k, v, p, stream);
+    if (p.head_dim == 64) return launch_dh<64, false>(q, k, v, p, stream);
+  }
   return cudaErrorInvalidValue;
 }
 

@@ -14,6 +14,10 @@ struct AttnParams {
   int out_lo;               // > 0: also write lo = bf16(o - hi) at element offset out_lo
   float scale_log2;         // log2(e) / sqrt(head_dim)
   int streams_per_group;    // unit order (set by launch_attention): see attn.cu
+  int causal;               // 0: counter-causal (rows [0, n) attend (i, n)); 1: causal over
+                            // the memory (rows [row_lo, n) attend [0, i], inference cycle)
+  const int32_t *row_lo;    // causal: device [batch], first query slot of each sequence
+  int q_span;               // query slots per sequence at most (cap, or the chunk size)
   unsigned *status;
 };
 

@@ -269,17 +269,21 @@ CC_DEV float warp_max(float v) {
   return v;
 }
 
-// Row tiles of a ragged batch: sequence b contributes ceil(seq_len[b] / tile)
-// tiles of `tile` rows.  prefix[b] = first tile of sequence b (prefix[batch] =
-// total).  Invalid lengths (outside [0, cap]) count as 0 and are reported.
-// seq_len == nullptr means every sequence is full (cap rows).
-CC_DEV int build_tile_prefix(const int32_t *seq_len, int batch, int cap, int tile, int *prefix,
-                             unsigned *status) {
+// Row tiles of a ragged batch: sequence b contributes the rows (slots)
+// [row_lo[b], seq_len[b]) in ceil((seq_len[b] - row_lo[b]) / tile) tiles of
+// `tile` rows.  prefix[b] = first tile of sequence b (prefix[batch] = total).
+// Invalid ranges (outside [0, cap]) count as 0 and are reported.
+// seq_len == nullptr means every sequence ends at cap; row_lo == nullptr
+// means every range starts at slot 0.
+CC_DEV int build_tile_prefix(const int32_t *seq_len, const int32_t *row_lo, int batch, int cap,
+                             int tile, int *prefix, unsigned *status) {
   int acc = 0;
   for (int b = 0; b < batch; ++b) {
     prefix[b] = acc;
-    int n = seq_len ? seq_len[b] : cap;
-    if (n < 0 || n > cap) {
+    const int hi = seq_len ? seq_len[b] : cap;
+    const int lo = row_lo ? row_lo[b] : 0;
+    int n = hi - lo;
+    if (lo < 0 || hi > cap || n < 0) {
       set_status(status, CC_ERR_DEVICE_ARG);
       n = 0;
     }

@@ -132,6 +132,30 @@ CC_DEV void epilogue_tile(const GemmParams &p, uint32_t tacc, int grow, bool val
         }
       }
     }
+  } else if constexpr (EPI == EPI_BF16) {
+    __nv_bfloat16 *out = reinterpret_cast<__nv_bfloat16 *>(p.out) + (size_t)grow * p.ldo;
+#pragma unroll 1
+    for (int c = 0; c < BN / 32; ++c) {
+      uint32_t r[32];
+      tmem_ld32(tacc + c * 32, r);
+      tmem_ld_wait();
+      const int col = tile_n0 + c * 32;
+      if (!valid || col >= p.N) continue;
+      uint32_t bb[16];
+#pragma unroll
+      for (int v = 0; v < 4; ++v) {
+        const uint4 u = p.bias ? reinterpret_cast<const uint4 *>(p.bias + col)[v] : make_uint4(0, 0, 0, 0);
+        bb[v * 4] = u.x; bb[v * 4 + 1] = u.y; bb[v * 4 + 2] = u.z; bb[v * 4 + 3] = u.w;
+      }
+      uint32_t o[16];
+#pragma unroll
+      for (int k = 0; k < 32; k += 2)
+        o[k / 2] = pack_bf16x2(__uint_as_float(r[k]) + bf16_lo(bb[k / 2]),
+                               __uint_as_float(r[k + 1]) + bf16_hi(bb[k / 2]));
+      uint4 *d = reinterpret_cast<uint4 *>(out + col);
+#pragma unroll
+      for (int v = 0; v < 4; ++v) d[v] = make_uint4(o[v * 4], o[v * 4 + 1], o[v * 4 + 2], o[v * 4 + 3]);
+    }
   } else if constexpr (EPI == EPI_SWIGLU) {
     // columns [0,128) = gate rows nt*128.., [128,256) = up rows nt*128..
     __nv_bfloat16 *out = reinterpret_cast<__nv_bfloat16 *>(p.out) + (size_t)grow * p.ldo;
@@ -251,7 +275,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&tempty[a], 4);
     }
     *abort_flag = 0;
-    build_tile_prefix(p.seq_len, p.batch, p.cap, BM, prefix, p.status);
+    build_tile_prefix(p.seq_len, p.row_lo, p.batch, p.cap, BM, prefix, p.status);
     fence_barrier_init();
   }
   if (warp == 0 && lane == 0) {
@@ -280,7 +304,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         int mt, nt;
         tile_coords(p, tile, num_m, mt, nt);
         const int b = find_seq(prefix, p.batch, mt);
-        const int row0 = b * p.cap + (mt - prefix[b]) * BM;
+        const int row0 = b * p.cap + (p.row_lo ? p.row_lo[b] : 0) + (mt - prefix[b]) * BM;
         for (int kb = 0; kb < nk_total; ++kb) {
           if (!mbar_wait(&empty[stage], phase ^ 1, abort_flag, p.status)) goto producer_done;
           mbar_arrive_expect_tx(&full[stage], A_BYTES + B_BYTES);
@@ -337,7 +361,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       int mt, nt;
       tile_coords(p, tile, num_m, mt, nt);
       const int b = find_seq(prefix, p.batch, mt);
-      const int i = (mt - prefix[b]) * BM + r;
+      const int i = (p.row_lo ? p.row_lo[b] : 0) + (mt - prefix[b]) * BM + r;
       const bool valid = i < (p.seq_len ? p.seq_len[b] : p.cap);
       const int grow = b * p.cap + i;
       if (!mbar_wait(&tfull[acc], acc_phase, abort_flag, p.status)) break;
@@ -391,6 +415,7 @@ cudaError_t launch_gemm(int epi, const CUtensorMap &a, const CUtensorMap &b, con
     case EPI_RESID_F32: return launch<EPI_RESID_F32>(a, b, b2, p, grid, stream);
     case EPI_SWIGLU: return launch<EPI_SWIGLU>(a, b, b2, p, grid, stream);
     case EPI_LSE: return launch<EPI_LSE>(a, b, b2, p, grid, stream);
+    case EPI_BF16: return launch<EPI_BF16>(a, b, b2, p, grid, stream);
     default: return cudaErrorInvalidValue;
   }
 }

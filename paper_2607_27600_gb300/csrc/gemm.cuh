@@ -10,13 +10,15 @@ enum GemmEpi : int {
   EPI_RESID_BF16 = 2, // out fp32 [rows][ldo] = acc + resid bf16 [rows][ld_resid]
   EPI_RESID_F32 = 3,  // out fp32 [rows][ldo] += acc
   EPI_SWIGLU = 4,     // out bf16 [rows][ldo] = silu(A Wg^T) * (A Wu^T)   (B = Wg, B2 = Wu)
-  EPI_LSE = 5         // out float2 [rows][ldo = n_tiles] = (max, sum exp) per vocab tile,
+  EPI_LSE = 5,        // out float2 [rows][ldo = n_tiles] = (max, sum exp) per vocab tile,
                       // z_target[row] = logit of tokens[row]
+  EPI_BF16 = 6        // out bf16 [rows][ldo] = acc (+ bias[col] if bias)
 };
 
 struct GemmParams {
   int batch, cap;
-  const int32_t *seq_len;  // device [batch]
+  const int32_t *seq_len;  // device [batch]: rows of sequence b end at slot seq_len[b]
+  const int32_t *row_lo;   // device [batch] or nullptr: rows start at slot row_lo[b] (else 0)
   int N, K;
   int n_tiles;             // column tiles (of gemm_block_n(epi) columns)
   void *out;
@@ -24,7 +26,7 @@ struct GemmParams {
   const void *resid;
   int ld_resid;
   const int32_t *pos;      // EPI_QROPE
-  const __nv_bfloat16 *bias;  // EPI_QROPE: optional per-column bias added before RoPE
+  const __nv_bfloat16 *bias;  // EPI_QROPE, EPI_BF16: optional per-column bias (before RoPE)
   int head_dim;            // EPI_QROPE
   const int32_t *tokens;   // EPI_LSE
   float *z_target;         // EPI_LSE

@@ -20,6 +20,14 @@ CC_DEV bool row_valid(const int32_t *seq_len, int cap, int row, int &i, int &n) 
   return i < n && n <= cap;
 }
 
+// Row ranges of the inference cycle: slots [row_lo[b], seq_len[b]) (row_lo
+// may be null: from slot 0).
+CC_DEV bool row_in_range(const int32_t *seq_len, const int32_t *row_lo, int cap, int row) {
+  int i, n;
+  if (!row_valid(seq_len, cap, row, i, n)) return false;
+  return !row_lo || i >= row_lo[row / cap];
+}
+
 // 8 bf16 of a uint4 -> float
 CC_DEV void unpack8(const uint4 &v, float *f) {
   f[0] = bf16_lo(v.x); f[1] = bf16_hi(v.x); f[2] = bf16_lo(v.y); f[3] = bf16_hi(v.y);
@@ -56,11 +64,10 @@ CC_DEV float row_inv_rms(const void *row, int d, float eps, int lane) {
 template <bool IN_F32>
 __global__ void __launch_bounds__(kWarps * 32)
     rmsnorm_kernel(const void *x, const __nv_bfloat16 *gain, __nv_bfloat16 *out, int d, float eps,
-                   const int32_t *seq_len, int cap, int rows, int split) {
+                   const int32_t *seq_len, const int32_t *row_lo, int cap, int rows, int split) {
   const int lane = threadIdx.x & 31;
   const int row = blockIdx.x * kWarps + (threadIdx.x >> 5);
-  int i, n;
-  if (row >= rows || !row_valid(seq_len, cap, row, i, n)) return;
+  if (row >= rows || !row_in_range(seq_len, row_lo, cap, row)) return;
   const size_t es = IN_F32 ? 4 : 2;
   const void *xr = reinterpret_cast<const uint8_t *>(x) + (size_t)row * d * es;
   const float inv = row_inv_rms<IN_F32>(xr, d, eps, lane);
@@ -91,11 +98,11 @@ __global__ void __launch_bounds__(kWarps * 32)
 // h (fp32) = embed[tokens[row]]
 __global__ void __launch_bounds__(kWarps * 32)
     embed_kernel(const __nv_bfloat16 *embed, const int32_t *tokens, float *h, int d, int vocab,
-                 const int32_t *seq_len, int cap, int rows, unsigned *status) {
+                 const int32_t *seq_len, const int32_t *row_lo, int cap, int rows,
+                 unsigned *status) {
   const int lane = threadIdx.x & 31;
   const int row = blockIdx.x * kWarps + (threadIdx.x >> 5);
-  int i, n;
-  if (row >= rows || !row_valid(seq_len, cap, row, i, n)) return;
+  if (row >= rows || !row_in_range(seq_len, row_lo, cap, row)) return;
   int tok = tokens[row];
   if (tok < 0 || tok >= vocab) {
     if (lane == 0) set_status(status, CC_ERR_DEVICE_ARG);
@@ -109,6 +116,62 @@ __global__ void __launch_bounds__(kWarps * 32)
     reinterpret_cast<float4 *>(dst + e)[0] = make_float4(f[0], f[1], f[2], f[3]);
     reinterpret_cast<float4 *>(dst + e)[1] = make_float4(f[4], f[5], f[6], f[7]);
   }
+}
+
+// out bf16 [row] = h fp32 [row] for the rows in range (H^(L-1) recorded by
+// the inference cycle).
+__global__ void __launch_bounds__(kWarps * 32)
+    store_bf16_kernel(const float *h, __nv_bfloat16 *out, int d, const int32_t *seq_len,
+                      const int32_t *row_lo, int cap, int rows) {
+  const int lane = threadIdx.x & 31;
+  const int row = blockIdx.x * kWarps + (threadIdx.x >> 5);
+  if (row >= rows || !row_in_range(seq_len, row_lo, cap, row)) return;
+  const float *src = h + (size_t)row * d;
+  __nv_bfloat16 *dst = out + (size_t)row * d;
+  for (int e = lane * 8; e < d; e += 256) {
+    float f[8];
+    load8<true>(src, e, f);
+    uint4 v;
+    v.x = pack_bf16x2(f[0], f[1]);
+    v.y = pack_bf16x2(f[2], f[3]);
+    v.z = pack_bf16x2(f[4], f[5]);
+    v.w = pack_bf16x2(f[6], f[7]);
+    *reinterpret_cast<uint4 *>(dst + e) = v;
+  }
+}
+
+// Inference cycle, start: sequence b (one block) appends count[b] slots after
+// its seq_len[b] current ones: row_lo = seq_len, row_hi = seq_len + count;
+// the chunk's tokens and positions (given, or continuing after the last
+// cached position) are written into the cache.  A count outside
+// [0, max_count] or past cap is reported and appends nothing.
+__global__ void append_prepare_kernel(const int32_t *seq_len, const int32_t *count,
+                                      const int32_t *tok_in, const int32_t *pos_in, int max_count,
+                                      int32_t *tokens, int32_t *pos, int32_t *row_lo,
+                                      int32_t *row_hi, int cap, unsigned *status) {
+  const int b = blockIdx.x;
+  const int lo = seq_len[b];
+  int c = count[b];
+  if (lo < 0 || lo > cap || c < 0 || c > max_count || lo + c > cap) {
+    if (threadIdx.x == 0) set_status(status, CC_ERR_DEVICE_ARG);
+    c = 0;   // nothing appended; seq_len is left as it was
+  }
+  if (threadIdx.x == 0) {
+    row_lo[b] = lo;
+    row_hi[b] = lo + c;
+  }
+  if (c == 0) return;
+  const size_t base = (size_t)b * cap;
+  const int next = lo > 0 ? pos[base + lo - 1] + 1 : 0;
+  for (int i = threadIdx.x; i < c; i += blockDim.x) {
+    tokens[base + lo + i] = tok_in[(size_t)b * max_count + i];
+    pos[base + lo + i] = pos_in ? pos_in[(size_t)b * max_count + i] : next + i;
+  }
+}
+
+__global__ void append_finish_kernel(int32_t *seq_len, const int32_t *row_hi, int batch) {
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b < batch) seq_len[b] = row_hi[b];
 }
 
 // score = -(RMSNorm(h) * g) . W_U[x_i]; last valid slot +inf; past the end -inf.
@@ -180,26 +243,50 @@ unsigned blocks_for(int rows) { return (unsigned)((rows + kWarps - 1) / kWarps);
 }  // namespace
 
 cudaError_t launch_rmsnorm(const void *x, bool x_f32, const void *gain, void *out, int d, float eps,
-                           const int32_t *seq_len, int cap, int rows, bool split, cudaStream_t st) {
+                           const int32_t *seq_len, int cap, int rows, bool split, cudaStream_t st,
+                           const int32_t *row_lo) {
   if (rows <= 0) return cudaSuccess;
   auto *g = reinterpret_cast<const __nv_bfloat16 *>(gain);
   auto *o = reinterpret_cast<__nv_bfloat16 *>(out);
   if (x_f32)
-    rmsnorm_kernel<true><<<blocks_for(rows), kWarps * 32, 0, st>>>(x, g, o, d, eps, seq_len, cap,
-                                                                    rows, split ? 1 : 0);
+    rmsnorm_kernel<true><<<blocks_for(rows), kWarps * 32, 0, st>>>(x, g, o, d, eps, seq_len, row_lo,
+                                                                    cap, rows, split ? 1 : 0);
   else
-    rmsnorm_kernel<false><<<blocks_for(rows), kWarps * 32, 0, st>>>(x, g, o, d, eps, seq_len, cap,
-                                                                     rows, split ? 1 : 0);
+    rmsnorm_kernel<false><<<blocks_for(rows), kWarps * 32, 0, st>>>(x, g, o, d, eps, seq_len, row_lo,
+                                                                     cap, rows, split ? 1 : 0);
   return cudaGetLastError();
 }
 
 cudaError_t launch_embed(const void *embed, const int32_t *tokens, float *h, int d, int vocab,
                          const int32_t *seq_len, int cap, int rows, unsigned *status,
-                         cudaStream_t st) {
+                         cudaStream_t st, const int32_t *row_lo) {
   if (rows <= 0) return cudaSuccess;
   embed_kernel<<<blocks_for(rows), kWarps * 32, 0, st>>>(
-      reinterpret_cast<const __nv_bfloat16 *>(embed), tokens, h, d, vocab, seq_len, cap, rows,
-      status);
+      reinterpret_cast<const __nv_bfloat16 *>(embed), tokens, h, d, vocab, seq_len, row_lo, cap,
+      rows, status);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_store_bf16(const float *h, void *out, int d, const int32_t *seq_len,
+                              const int32_t *row_lo, int cap, int rows, cudaStream_t st) {
+  if (rows <= 0) return cudaSuccess;
+  store_bf16_kernel<<<blocks_for(rows), kWarps * 32, 0, st>>>(
+      h, reinterpret_cast<__nv_bfloat16 *>(out), d, seq_len, row_lo, cap, rows);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_append_prepare(const int32_t *seq_len, const int32_t *count,
+                                  const int32_t *tok_in, const int32_t *pos_in, int max_count,
+                                  int32_t *tokens, int32_t *pos, int32_t *row_lo, int32_t *row_hi,
+                                  int batch, int cap, unsigned *status, cudaStream_t st) {
+  append_prepare_kernel<<<batch, 256, 0, st>>>(seq_len, count, tok_in, pos_in, max_count, tokens,
+                                                pos, row_lo, row_hi, cap, status);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_append_finish(int32_t *seq_len, const int32_t *row_hi, int batch,
+                                 cudaStream_t st) {
+  append_finish_kernel<<<(batch + 255) / 256, 256, 0, st>>>(seq_len, row_hi, batch);
   return cudaGetLastError();
 }
 

@@ -6,12 +6,27 @@ namespace cc {
 
 // out bf16 [rows][d] = x * gain / sqrt(mean(x^2) + eps); x bf16 or fp32 [rows][d].
 // split: out rows are [hi | lo] bf16 [rows][2d] with hi + lo ~= the fp32 value.
+// Row kernels visit rows b*cap + i with row_lo[b] <= i < seq_len[b] (row_lo
+// null: from 0).
 cudaError_t launch_rmsnorm(const void *x, bool x_f32, const void *gain, void *out, int d, float eps,
-                           const int32_t *seq_len, int cap, int rows, bool split, cudaStream_t st);
+                           const int32_t *seq_len, int cap, int rows, bool split, cudaStream_t st,
+                           const int32_t *row_lo = nullptr);
 // h fp32 [rows][d] = embed[tokens[row]]
 cudaError_t launch_embed(const void *embed, const int32_t *tokens, float *h, int d, int vocab,
                          const int32_t *seq_len, int cap, int rows, unsigned *status,
-                         cudaStream_t st);
+                         cudaStream_t st, const int32_t *row_lo = nullptr);
+// out bf16 [rows][d] = h fp32 (H^(L-1) recorded by the inference cycle)
+cudaError_t launch_store_bf16(const float *h, void *out, int d, const int32_t *seq_len,
+                              const int32_t *row_lo, int cap, int rows, cudaStream_t st);
+// Inference cycle: row_lo = seq_len, row_hi = seq_len + count; the chunk's
+// tokens and positions written into the cache slots [row_lo, row_hi).
+cudaError_t launch_append_prepare(const int32_t *seq_len, const int32_t *count,
+                                  const int32_t *tok_in, const int32_t *pos_in, int max_count,
+                                  int32_t *tokens, int32_t *pos, int32_t *row_lo, int32_t *row_hi,
+                                  int batch, int cap, unsigned *status, cudaStream_t st);
+// seq_len = row_hi
+cudaError_t launch_append_finish(int32_t *seq_len, const int32_t *row_hi, int batch,
+                                 cudaStream_t st);
 // scores[row] = -(final-norm(h) . lm_head[tokens[row]]), +inf at the last slot
 cudaError_t launch_head_logit(const float *h, const void *gain, const void *lm_head,
                               const int32_t *tokens, float *scores, int d, int vocab, float eps,

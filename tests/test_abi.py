@@ -51,6 +51,8 @@ def test_host_side_validation_without_device(lib):
     assert lib.cc_select_keep(None, None, 1, 1, None, 0, None, None, None, 0, None) == \
         cc.CC_ERR_INVALID_ARG
     assert lib.cc_score_layer(None, None, None, 0, None, None, 0, None) == cc.CC_ERR_INVALID_ARG
+    assert lib.cc_append_chunk(None, None, None, None, None, None, 1, None, 0, None) == \
+        cc.CC_ERR_INVALID_ARG
     bad = cc.cc_model_cfg(1, 100, 8, 3, 128, 256, 10, 1e4, 1e-5)   # Hq % Hkv != 0
     assert lib.cc_score_workspace_size(ctypes.byref(bad), 1, 16, 0) == 0
     odd = cc.cc_model_cfg(1, 256, 8, 2, 96, 256, 10, 1e4, 1e-5)    # head_dim 96
@@ -71,6 +73,8 @@ def test_workspace_size_formula(lib):
     rows, d, q, f = 8192, 4096, 4096, 14336
     assert n >= rows * (2 * d + 2 * q * 2 + 4 * d + 2 * f)
     assert cc.cc_score_workspace_size(LLAMA3_8B, 1, 8192, cc.SCORE_LOGPROB) > n
+    # the append reuses the scoring rows plus two int32 [batch] range arrays
+    assert cc.cc_append_workspace_size(LLAMA3_8B, 1, 8192) >= n
 
 
 def test_compaction_plan_covers_every_array(lib):

@@ -1,0 +1,171 @@
+"""GPU parity of the inference cycle in pre-fill (cc_append_chunk,
+Algorithm CacheManagedInference / DoInference over a chunk) against the
+oracle's append_chunk, through the C ABI."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+from synth.configs import ModelShape
+from tests._util import causal_cache, rel_err, to_device, to_np
+
+pytestmark = pytest.mark.gpu
+
+TOL = 2e-2
+SMALL_GPU = ModelShape(n_layers=2, d_model=256, n_q_heads=8, n_kv_heads=2, head_dim=64,
+                       d_ff=384, vocab=1000, rope_theta=1e4, rms_eps=1e-5)
+
+
+@pytest.fixture(scope="module")
+def cc():
+    from paper_2607_27600_gb300 import cc as mod
+    mod.load_library()
+    return mod
+
+
+def _rel(got, want):
+    """max |g - o| / max |o| (the attention tests' bar for bf16 outputs)."""
+    got, want = np.asarray(got, np.float64), np.asarray(want, np.float64)
+    return float(np.abs(got - want).max() / max(np.abs(want).max(), 1e-30))
+
+
+def _gpu_append(cc, shape, w_np, c_np, chunks, pos=None):
+    """Runs cc_append_chunk on device copies; returns the device cache (numpy)."""
+    import paper_2607_27600_gb300 as pkg
+    b = len(chunks)
+    mx = max(1, max(len(t) for t in chunks))
+    tok = np.zeros((b, mx), np.int32)
+    ps = np.zeros((b, mx), np.int32)
+    for i, t in enumerate(chunks):
+        tok[i, :len(t)] = t
+        if pos is not None:
+            ps[i, :len(t)] = pos[i]
+    cnt = np.array([len(t) for t in chunks], np.int32)
+    w, c = to_device(w_np), to_device(c_np)
+    weights, cache = pkg.Weights(w), pkg.Cache(c)
+    ws = cc.alloc_workspace(cc.cc_append_workspace_size(shape, b, c["tokens"].shape[1]))
+    cc.cc_append_chunk(shape, weights, cache, torch.from_numpy(tok).cuda(),
+                       None if pos is None else torch.from_numpy(ps).cuda(),
+                       torch.from_numpy(cnt).cuda(), mx, ws)
+    status = cc.cc_get_status()
+    return to_np(c), status, (weights, cache)
+
+
+def _oracle_append(shape, w_np, c_np, chunks, pos=None):
+    c = {k: ([np.asarray(x, np.float64).copy() for x in v] if isinstance(v, list) else
+             np.asarray(v).copy()) for k, v in c_np.items()}
+    for b, t in enumerate(chunks):
+        if len(t):
+            oracle.append_chunk(shape, w_np, c, b, t, None if pos is None else pos[b])
+    return c
+
+
+def _check(shape, got, want, chunks, n0):
+    for b, t in enumerate(chunks):
+        sl = slice(n0[b], n0[b] + len(t))
+        assert got["seq_len"][b] == n0[b] + len(t)
+        np.testing.assert_array_equal(got["tokens"][b, sl], want["tokens"][b, sl])
+        np.testing.assert_array_equal(got["pos"][b, sl], want["pos"][b, sl])
+        if not len(t):
+            continue
+        for l in range(shape.n_layers):
+            assert _rel(got["k"][l][b, sl], want["k"][l][b, sl]) < TOL, ("k", l, b)
+            assert _rel(got["v"][l][b, sl], want["v"][l][b, sl]) < TOL, ("v", l, b)
+        if got.get("h_last") is not None:
+            assert _rel(got["h_last"][b, sl], want["h_last"][b, sl]) < TOL, ("h_last", b)
+        # memory slots untouched
+        for l in range(shape.n_layers):
+            np.testing.assert_array_equal(got["k"][l][b, :n0[b]],
+                                          np.asarray(want["k"][l][b, :n0[b]], np.float32))
+
+
+def _setup(shape, seq, cap, seed):
+    w_np = to_np(synth.model_weights(shape, seed, with_kv_proj=True))
+    c_np = causal_cache(shape, w_np, seq, cap, seed)
+    return w_np, c_np
+
+
+def test_append_into_empty_cache_ragged(cc):
+    """Empty cache, chunks of 300 and 77 tokens: the causal forward."""
+    w_np, c_np = _setup(SMALL_GPU, [0, 0], 320, seed=51)
+    r = np.random.default_rng(51)
+    chunks = [r.integers(0, SMALL_GPU.vocab, size=300), r.integers(0, SMALL_GPU.vocab, size=77)]
+    got, status, _ = _gpu_append(cc, SMALL_GPU, w_np, c_np, chunks)
+    assert status == cc.CC_OK
+    want = _oracle_append(SMALL_GPU, w_np, c_np, chunks)
+    _check(SMALL_GPU, got, want, chunks, [0, 0])
+
+
+@pytest.mark.parametrize("variant", ["plain", "qkv_bias+rope_scaling"])
+def test_append_after_compaction_then_score(cc, variant):
+    """Memory built by the oracle's causal pass, compacted to a seeded keep-set
+    (positions keep their original values), then a chunk appended to each
+    sequence (one of them empty); the appended cache then scores like the
+    oracle's appended cache."""
+    import paper_2607_27600_gb300 as pkg
+    shape = SMALL_GPU if variant == "plain" else ModelShape(
+        **{**SMALL_GPU.__dict__, "qkv_bias": True, "rope_scaling": (8.0, 1.0, 4.0, 64)})
+    w_np, c_np = _setup(shape, [200, 50, 90], 384, seed=52)
+    r = np.random.default_rng(52)
+    keep = np.full((3, 384), -1, np.int32)
+    cnt = np.array([120, 50, 31], np.int32)
+    for b, (n, j) in enumerate(zip([200, 50, 90], cnt)):
+        k = np.sort(np.concatenate([r.choice(n - 1, size=j - 1, replace=False), [n - 1]]))
+        keep[b, :j] = k
+    for key in ("tokens", "pos", "h_last"):
+        c_np[key] = oracle.compact(c_np[key], keep, cnt)
+    c_np["k"] = [oracle.compact(x, keep, cnt) for x in c_np["k"]]
+    c_np["v"] = [oracle.compact(x, keep, cnt) for x in c_np["v"]]
+    c_np["seq_len"] = cnt.copy()
+    chunks = [r.integers(0, shape.vocab, size=130), np.zeros(0, np.int64),
+              r.integers(0, shape.vocab, size=255)]
+    got, status, (weights, cache) = _gpu_append(cc, shape, w_np, c_np, chunks)
+    assert status == cc.CC_OK
+    want = _oracle_append(shape, w_np, c_np, chunks)
+    _check(shape, got, want, chunks, list(cnt))
+    # score the appended caches: GPU on its own, the oracle on its own
+    b, cap = 3, 384
+    scores = torch.full((b, cap), float("nan"), device="cuda")
+    ws = cc.alloc_workspace(cc.cc_score_workspace_size(shape, b, cap, cc.SCORE_LOGIT))
+    cc.cc_score_layer(shape, weights, cache, cc.SCORE_LOGIT, scores, ws)
+    assert cc.cc_get_status() == cc.CC_OK
+    want_s = oracle.score_layer(shape, w_np, want)
+    assert rel_err(scores.cpu().numpy(), want_s) < TOL
+
+
+def test_append_explicit_positions_and_bad_count(cc):
+    """Given positions are stored and used for RoPE; a count past the cap is
+    reported on the device and leaves that sequence as it was."""
+    w_np, c_np = _setup(SMALL_GPU, [40, 60], 128, seed=53)
+    r = np.random.default_rng(53)
+    chunks = [r.integers(0, SMALL_GPU.vocab, size=30), r.integers(0, SMALL_GPU.vocab, size=10)]
+    pos = [np.arange(1000, 1030), np.arange(500, 510) * 3]
+    got, status, _ = _gpu_append(cc, SMALL_GPU, w_np, c_np, chunks, pos=pos)
+    assert status == cc.CC_OK
+    want = _oracle_append(SMALL_GPU, w_np, c_np, chunks, pos=pos)
+    _check(SMALL_GPU, got, want, chunks, [40, 60])
+    np.testing.assert_array_equal(got["pos"][0, 40:70], pos[0])
+    # 100 more slots do not fit in sequence 1 (60 + 100 > 128): nothing appended there
+    chunks2 = [r.integers(0, SMALL_GPU.vocab, size=5), r.integers(0, SMALL_GPU.vocab, size=100)]
+    got2, status2, _ = _gpu_append(cc, SMALL_GPU, w_np, c_np, chunks2)
+    assert status2 == cc.CC_ERR_DEVICE_ARG
+    assert list(got2["seq_len"]) == [45, 60]
+    assert cc.cc_get_status() == cc.CC_OK      # the status word was read and cleared
+
+
+def test_append_llama_shape_chunk_over_long_memory(cc):
+    """Llama-3-8B layer shapes (first two layers), a 1024-token chunk after
+    8192 synthetic memory slots: every appended K/V row of both layers,
+    H^(L-1) and the chunk's positions."""
+    shape = ModelShape(**{**synth.configs.LLAMA3_8B.__dict__, "n_layers": 2})
+    n0, h, cap = 8192, 1024, 9216
+    w = synth.model_weights(shape, 7, device="cuda", with_kv_proj=True)
+    c = synth.synthetic_cache(shape, [n0], cap, 7, device="cuda")
+    w_np, c_np = to_np(w), to_np(c)
+    chunk = synth.tokens((h,), shape.vocab, 7, "chunk").numpy()
+    got, status, _ = _gpu_append(cc, shape, w_np, c_np, [chunk])
+    assert status == cc.CC_OK
+    want = _oracle_append(shape, w_np, c_np, [chunk])
+    _check(shape, got, want, [chunk], [n0])
+    np.testing.assert_array_equal(got["pos"][0, n0:n0 + h], np.arange(n0, n0 + h))
