@@ -568,6 +568,180 @@ def run_reference(args, dist):
                     "d2h_bytes_per_step": 0}}
 
 
+# ---------------------------------------------------------------------------
+# the inference cycle (pre-fill chunk append), --append
+# ---------------------------------------------------------------------------
+
+def append_work(shape, j, h):
+    """Per-launch algorithmic FLOPs / bytes of the append of h tokens after j memory slots."""
+    d, qd, kvd, f, hq, dh = (shape.d_model, shape.q_dim, shape.kv_dim, shape.d_ff,
+                             shape.n_q_heads, shape.head_dim)
+    keys = h * j + h * (h + 1) // 2            # sum over chunk rows of the keys they attend
+    return {"gemm_qrope": ("tensor", 2.0 * h * d * qd),
+            "gemm_kv": ("tensor", 2.0 * h * d * kvd),
+            "attention_causal": ("tensor", 4.0 * dh * hq * keys),
+            "gemm_oproj": ("tensor", 2.0 * h * qd * d),
+            "gemm_gateup": ("tensor", 4.0 * h * d * f),
+            "gemm_down": ("tensor", 2.0 * h * f * d),
+            "rmsnorm": ("hbm", h * (4.0 * d * 2 + 2.0 * d))}
+
+
+def kernel_table(kernels, steps, work_tbl, peaks):
+    table = {}
+    total = max(1e-9, sum(t for _, t in kernels.values()))
+    for name, (cnt, tot) in kernels.items():
+        per = tot / cnt
+        entry = {"launches_per_step": cnt / steps, "ms_per_launch": round(per, 4),
+                 "share": round(tot / total, 4)}
+        if name in work_tbl:
+            bound, amount = work_tbl[name]
+            if bound == "tensor":
+                ach = amount / (per * 1e-3) / 1e12
+                entry.update({"bound": "tensor", "achieved": round(ach, 2), "unit": "TFLOP/s",
+                              "frac": round(ach / peaks["bf16_tflops"], 4)})
+            else:
+                ach = amount / (per * 1e-3) / 1e9
+                entry.update({"bound": "hbm", "achieved": round(ach, 1), "unit": "GB/s",
+                              "frac": round(ach / peaks["hbm_gbs"], 4)})
+        table[name] = entry
+    return table
+
+
+def run_append(args, dist):
+    """Times cc_append_chunk: the workload's `append` tokens after a memory of
+    `budgets[0]` slots (the cache a refresh leaves), through every layer."""
+    import paper_2607_27600_gb300 as pkg
+    from paper_2607_27600_gb300 import cc
+    pkg.load_library()
+    dev = torch.device(f"cuda:{dist.local}")
+    torch.cuda.set_device(dev)
+    wl = synth.WORKLOADS[args.workload]
+    shape = wl.shape
+    j, h = wl.budgets[0], wl.append
+    if h <= 0:
+        raise SystemExit(f"{wl.name} has no append chunk")
+    cap = j + h
+    w = synth.model_weights(shape, wl.seed, device=dev, with_kv_proj=True)
+    cache = synth.synthetic_cache(shape, [j], cap, wl.seed, device=dev)
+    chunk = synth.tokens((1, h), shape.vocab, wl.seed, "bench.chunk", dev)
+    count = torch.tensor([h], dtype=torch.int32, device=dev)
+    weights, kc = pkg.Weights(w), pkg.Cache(cache)
+    ws = cc.alloc_workspace(cc.cc_append_workspace_size(shape, 1, cap), dev)
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def prepare():
+        cache["seq_len"].fill_(j)
+        flush.fill_(1)
+
+    for _ in range(args.warmup):
+        prepare()
+        cc.cc_append_chunk(shape, weights, kc, chunk, None, count, h, ws)
+    torch.cuda.synchronize(dev)
+    if cc.cc_get_status() != cc.CC_OK:
+        raise SystemExit("device status after warm-up")
+    clocks = ClockSampler(dist.local)
+    clocks.start()
+    time.sleep(0.3)
+    dist.barrier()
+    torch.cuda.synchronize(dev)
+    cc.cc_timing_enable(True)
+    ms_steps = []
+    for _ in range(args.steps):
+        prepare()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        cc.cc_append_chunk(shape, weights, kc, chunk, None, count, h, ws)
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+        ms_steps.append(e0.elapsed_time(e1))
+    kernels = cc.cc_timing_collect()
+    cc.cc_timing_enable(False)
+    dist.barrier()
+    ms = dist.max(sum(ms_steps) / len(ms_steps))
+    # end to end: the chunk's token ids and count from pinned host memory, the
+    # new length read back
+    host_tok = chunk.cpu().pin_memory()
+    host_cnt = count.cpu().pin_memory()
+    out_len = torch.empty(1, dtype=torch.int32).pin_memory()
+    e2e = []
+    for _ in range(args.steps):
+        prepare()
+        torch.cuda.synchronize(dev)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        tok_d = host_tok.to(dev, non_blocking=True)
+        cnt_d = host_cnt.to(dev, non_blocking=True)
+        cc.cc_append_chunk(shape, weights, kc, tok_d, None, cnt_d, h, ws)
+        out_len.copy_(cache["seq_len"], non_blocking=True)
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+        e2e.append(e0.elapsed_time(e1))
+    clk = clocks.stop()
+    if cc.cc_get_status() != cc.CC_OK or int(out_len[0]) != j + h:
+        raise SystemExit("append did not complete")
+    e2e_ms = dist.max(sum(e2e) / len(e2e))
+    peaks, peak_src = load_peaks()
+    work = append_work(shape, j, h)
+    table = kernel_table(kernels, args.steps, work, peaks)
+    dom = max(kernels.items(), key=lambda kv: kv[1][1])[0]
+    d = table[dom]
+    flops = sum(work[k][1] * table[k]["launches_per_step"] for k in work
+                if work[k][0] == "tensor" and k in table)
+    line = {
+        "metric": "appended tokens/sec per inference cycle (pre-fill chunk, all layers)",
+        "value": round(h * dist.world / (ms * 1e-3), 1), "unit": "tokens/s",
+        "n_gpus": dist.world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(ms, 4), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded random-init weights N(0,0.02); synthetic memory K/V)",
+        "config": {"workload": wl.name + "/append", "memory_slots": j, "chunk": h,
+                   "layers": shape.n_layers, "d_model": shape.d_model,
+                   "heads": f"{shape.n_q_heads}/{shape.n_kv_heads}x{shape.head_dim}",
+                   "d_ff": shape.d_ff, "step_tflop": round(flops / 1e12, 3),
+                   "l2": "256 MiB written between steps (outside the timed events)",
+                   "parallelism": f"replicas x{dist.world}"},
+        "e2e": {"value": round(h * dist.world / (e2e_ms * 1e-3), 1), "unit": "tokens/s",
+                "h2d_bytes_per_step": int(host_tok.numel() * 4 + 4), "d2h_bytes_per_step": 4,
+                "ms_per_step": round(e2e_ms, 4)},
+        "gpu_launches": int(sum(c for c, _ in kernels.values()) / args.steps),
+        "roofline": {"kernel": dom, "bound": d.get("bound"), "achieved": d.get("achieved"),
+                     "peak": peaks["bf16_tflops"] if d.get("bound") == "tensor" else peaks["hbm_gbs"],
+                     "unit": d.get("unit"), "frac": d.get("frac"), "traffic": None,
+                     "peak_source": f"{peak_src} (bf16 dense burst)"},
+        "kernels": table,
+        "tflops_per_step_achieved": round(flops / (ms * 1e-3) / 1e12, 1),
+        "clocks": clk,
+    }
+    if dist.world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = append_cpu_baseline(shape, w, cache, chunk, j, h)
+    return line
+
+
+def append_cpu_baseline(shape, w, cache, chunk, j, h, sample=8):
+    """The oracle's append timed on the host cores for `sample` chunk tokens
+    through one layer, extrapolated linearly to the chunk and every layer (a
+    row's GEMM work and its attention over ~j memory keys dominate)."""
+    import oracle
+    one = shape.__class__(**{**shape.__dict__, "n_layers": 1})
+    lw = {k: v.float().cpu().numpy() for k, v in w["layers"][0].items()}
+    wn = {"embed": w["embed"].float().cpu().numpy(), "layers": [lw]}
+    cn = {"k": [cache["k"][0].float().cpu().numpy().astype(np.float64)],
+          "v": [cache["v"][0].float().cpu().numpy().astype(np.float64)],
+          "tokens": cache["tokens"].cpu().numpy(), "pos": cache["pos"].cpu().numpy(),
+          "seq_len": np.array([j]), "h_last": None}
+    toks = chunk.cpu().numpy()[0, :sample]
+    t0 = time.perf_counter()
+    oracle.append_chunk(one, wn, cn, 0, toks)
+    dt = time.perf_counter() - t0
+    per_token_layer = dt / sample
+    total = per_token_layer * h * shape.n_layers
+    return {"value": round(h / total, 2), "unit": "tokens/s", "cores": os.cpu_count(),
+            "kind": "oracle",
+            "sample": f"{sample} chunk tokens through 1 layer ({dt:.1f} s), extrapolated linearly "
+                      f"to {h} tokens x {shape.n_layers} layers; numpy fp64"}
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -581,12 +755,20 @@ def main():
     ap.add_argument("--cpu-rows", type=int, default=256)
     ap.add_argument("--ref-rows", type=int, default=32)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--append", action="store_true",
+                    help="time the inference cycle: the workload's append chunk over its "
+                         "budget-sized memory (cc_append_chunk, every layer)")
     args = ap.parse_args()
     if args.warmup < 3:
         raise SystemExit("--warmup must be >= 3")
     dist = Dist()
     try:
-        line = run_reference(args, dist) if args.impl == "reference" else run_ours(args, dist)
+        if args.impl == "reference":
+            line = run_reference(args, dist)
+        elif args.append:
+            line = run_append(args, dist)
+        else:
+            line = run_ours(args, dist)
         if dist.rank == 0 and line is not None:
             print(json.dumps(line), flush=True)
     finally:
