@@ -679,8 +679,8 @@ cc_status compact_plan(const cc_model_cfg *c, const cc_kv_cache *kv, CompactPlan
     A.base = base;
     A.row_bytes = row_bytes;
     A.bulk = bulk ? 1 : 0;
-    A.rows_per_chunk = bulk ? (row_bytes <= kStageBytes ? kStageBytes / row_bytes : 0)
-                            : kStageBytes / 4;
+    A.rows_per_chunk = bulk ? (row_bytes <= p.stage_bytes ? p.stage_bytes / row_bytes : 0)
+                            : p.stage_bytes / 4;
     if (A.rows_per_chunk < 1) return false;
     A.n_chunks = (kv->cap + A.rows_per_chunk - 1) / A.rows_per_chunk;
     A.dep_class = class_of(A.rows_per_chunk);
@@ -689,6 +689,9 @@ cc_status compact_plan(const cc_model_cfg *c, const cc_kv_cache *kv, CompactPlan
     return true;
   };
   const int kv_row = c->n_kv_heads * c->head_dim * 2;
+  // staging shape of the copy kernel for the largest row moved
+  const int max_row = std::max(kv_row, kv->h_last ? c->d_model * 2 : 0);
+  if (!compact_shape(max_row, p.stage_bytes, p.warps)) return CC_ERR_UNSUPPORTED;
   for (int l = 0; l < c->n_layers; ++l) {
     if (!add(kv->k[l], kv_row, true) || !add(kv->v[l], kv_row, true)) return CC_ERR_UNSUPPORTED;
   }

@@ -35,8 +35,7 @@ namespace cc {
 
 namespace {
 
-constexpr int kWarps = CC_COMPACT_WARPS;   // independent two-buffer pipelines per CTA
-constexpr int kThreads = kWarps * 32;
+constexpr int kThreads = kCompactMaxWarps * 32;   // launch bound; p.warps warps run
 
 CC_DEV void st_release(unsigned *p, unsigned v) {
   asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
@@ -83,23 +82,54 @@ __global__ void deps_kernel(const __grid_constant__ CompactParams p) {
 
 // Pre-pass: unit_base[a*batch + b] = first unit of (array a, sequence b),
 // counting ceil(keep_count[b] / rows_per_chunk) units each; the last entry
-// is the number of units.
-__global__ void plan_kernel(const __grid_constant__ CompactParams p) {
-  if (threadIdx.x != 0) return;
-  int acc = 0;
-  for (int a = 0; a < p.n_arrays; ++a) {
-    const int C = p.arr[a].rows_per_chunk;
-    for (int b = 0; b < p.batch; ++b) {
-      p.unit_base[a * p.batch + b] = acc;
+// is the number of units.  One block: an exclusive scan over the
+// (array, sequence) pairs, 1024 pairs per round.
+__global__ void __launch_bounds__(1024) plan_kernel(const __grid_constant__ CompactParams p) {
+  __shared__ int warp_sums[32];
+  __shared__ int carry;
+  const int n_pairs = p.n_arrays * p.batch;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  if (threadIdx.x == 0) carry = 0;
+  __syncthreads();
+  for (int base = 0; base < n_pairs; base += 1024) {
+    const int t = base + threadIdx.x;
+    int units = 0;
+    if (t < n_pairs) {
+      const int a = t / p.batch, b = t - a * p.batch;
+      const int C = p.arr[a].rows_per_chunk;
       int J = p.keep_count[b];
       if (J < 0 || J > p.cap) {
-        set_status(p.status, CC_ERR_DEVICE_ARG);
+        if (a == 0) set_status(p.status, CC_ERR_DEVICE_ARG);
         J = 0;
       }
-      acc += (J + C - 1) / C;
+      units = (J + C - 1) / C;
     }
+    int incl = units;   // inclusive scan within the warp
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int v = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+      if (lane >= o) incl += v;
+    }
+    if (lane == 31) warp_sums[warp] = incl;
+    __syncthreads();
+    if (warp == 0) {
+      const int ws = warp_sums[lane];
+      int wi = ws;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int v = __shfl_up_sync(0xFFFFFFFFu, wi, o);
+        if (lane >= o) wi += v;
+      }
+      warp_sums[lane] = wi - ws;   // exclusive prefix of the warp totals
+    }
+    __syncthreads();
+    const int excl = carry + warp_sums[warp] + incl - units;
+    if (t < n_pairs) p.unit_base[t] = excl;
+    __syncthreads();
+    if (threadIdx.x == 1023) carry = excl + units;
+    __syncthreads();
   }
-  p.unit_base[p.n_arrays * p.batch] = acc;
+  if (threadIdx.x == 0) p.unit_base[n_pairs] = carry;
 }
 
 struct Unit {
@@ -114,10 +144,11 @@ __global__ void __launch_bounds__(kThreads)
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 127) &
                                               ~uintptr_t(127));
-  __shared__ __align__(8) uint64_t bars[kWarps][2];
+  __shared__ __align__(8) uint64_t bars[kCompactMaxWarps][2];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  uint8_t *buf[2] = {smem + (size_t)(warp * 2 + 0) * kStageBytes,
-                     smem + (size_t)(warp * 2 + 1) * kStageBytes};
+  const int n_warps = p.warps;
+  uint8_t *buf[2] = {smem + (size_t)(warp * 2 + 0) * p.stage_bytes,
+                     smem + (size_t)(warp * 2 + 1) * p.stage_bytes};
   if (lane == 0) {
     mbar_init(&bars[warp][0], 1);
     mbar_init(&bars[warp][1], 1);
@@ -135,8 +166,8 @@ __global__ void __launch_bounds__(kThreads)
 
   const int n_pairs = p.n_arrays * p.batch;
   const int total = p.unit_base[n_pairs];
-  const int stride = gridDim.x * kWarps;
-  int next_t = blockIdx.x * kWarps + warp;
+  const int stride = gridDim.x * n_warps;
+  int next_t = blockIdx.x * n_warps + warp;
   auto take = [&]() -> Unit {
     Unit u;
     u.t = next_t;
@@ -272,29 +303,49 @@ __global__ void __launch_bounds__(kThreads)
 
 }  // namespace
 
-size_t compact_stage_bytes() { return (size_t)kWarps * 2 * kStageBytes + 128; }
+bool compact_shape(int max_row_bytes, int &stage_bytes, int &warps) {
+  stage_bytes = kCompactStageBytes;
+  if (max_row_bytes > stage_bytes) stage_bytes = (max_row_bytes + 127) & ~127;
+  warps = (kCompactSmemBytes - 128) / (2 * stage_bytes);
+  if (warps > kCompactMaxWarps) warps = kCompactMaxWarps;
+  return warps >= 1;
+}
+
+size_t compact_smem_bytes(const CompactParams &p) {
+  return (size_t)p.warps * 2 * p.stage_bytes + 128;
+}
 
 cudaError_t launch_compact(const CompactParams &p, int sms, cudaStream_t st) {
-  static int blocks_per_sm[64] = {};
+  // resident CTAs per SM for this shape (the cooperative launch needs all of them)
+  static bool attr_set[64] = {};
+  static int occ_cache[64][kCompactMaxWarps + 1] = {};
+  static int occ_smem[64][kCompactMaxWarps + 1] = {};
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
-  if (!blocks_per_sm[dev]) {
+  if (p.warps < 1 || p.warps > kCompactMaxWarps || p.stage_bytes < 16) return cudaErrorInvalidValue;
+  const size_t smem = compact_smem_bytes(p);
+  if (!attr_set[dev]) {
     cudaError_t e = cudaFuncSetAttribute(compact_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)compact_stage_bytes());
+                                         kCompactSmemBytes);
     if (e != cudaSuccess) return e;
+    attr_set[dev] = true;
+  }
+  if (occ_smem[dev][p.warps] != (int)smem) {
     int n = 0;
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, compact_kernel, kThreads,
-                                                      compact_stage_bytes());
+    cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, compact_kernel, p.warps * 32,
+                                                                  smem);
     if (e != cudaSuccess) return e;
     if (n < 1) return cudaErrorLaunchOutOfResources;
-    blocks_per_sm[dev] = n;
+    occ_cache[dev][p.warps] = n;
+    occ_smem[dev][p.warps] = (int)smem;
   }
+  const int blocks_per_sm = occ_cache[dev][p.warps];
   if (p.total_units <= 0) return cudaSuccess;
   for (int cls = 0; cls < p.n_classes; ++cls) {
     if (p.class_rows[cls] <= 0) return cudaErrorInvalidValue;
   }
-  plan_kernel<<<1, 32, 0, st>>>(p);
+  plan_kernel<<<1, 1024, 0, st>>>(p);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   const dim3 dgrid((p.cap + 255) / 256, p.batch, p.n_classes);
@@ -303,8 +354,8 @@ cudaError_t launch_compact(const CompactParams &p, int sms, cudaStream_t st) {
   if (e != cudaSuccess) return e;
   // cooperative: every warp resident, so the static unit order cannot deadlock
   void *args[] = {const_cast<CompactParams *>(&p)};
-  return cudaLaunchCooperativeKernel((const void *)compact_kernel, dim3(sms * blocks_per_sm[dev]),
-                                     dim3(kThreads), args, compact_stage_bytes(), st);
+  return cudaLaunchCooperativeKernel((const void *)compact_kernel, dim3(sms * blocks_per_sm),
+                                     dim3(p.warps * 32), args, smem, st);
 }
 
 }  // namespace cc

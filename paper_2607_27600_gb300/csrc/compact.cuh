@@ -4,13 +4,14 @@
 
 namespace cc {
 
-#ifndef CC_COMPACT_STAGE_KB
-#define CC_COMPACT_STAGE_KB 12
-#endif
-#ifndef CC_COMPACT_WARPS
-#define CC_COMPACT_WARPS 8
-#endif
-constexpr int kStageBytes = CC_COMPACT_STAGE_KB * 1024;   // shared-memory staging per unit (two per warp)
+// Each warp of the copy kernel runs a two-buffer pipeline of units; a unit
+// stages up to one buffer of rows in shared memory.  Default shape: 12 warps
+// x 2 x 8 KB (measured fastest on Llama-3-8B caches: 2 KB K/V rows, 8 KB
+// H^(L-1) rows).  A cache with a larger row takes that row size as its
+// buffer and fewer warps, so shared memory still fits.
+constexpr int kCompactMaxWarps = 12;
+constexpr int kCompactStageBytes = 8 * 1024;
+constexpr int kCompactSmemBytes = 224 * 1024;   // dynamic shared memory budget of the copy kernel
 constexpr int kMaxCompactArrays = 2 * 128 + 3;
 constexpr int kMaxDepClasses = 3;        // distinct chunk sizes (K/V rows, H rows, 4-byte rows)
 
@@ -41,10 +42,15 @@ struct CompactParams {
   long long class_offset[kMaxDepClasses];
   unsigned *status;
   int withhold_unit;          // test hook: this unit never publishes its flag (-1: none)
+  int stage_bytes;            // shared-memory buffer of a unit (multiple of 128)
+  int warps;                  // warps per CTA (each with two buffers)
   CompactArray arr[kMaxCompactArrays];
 };
 
-size_t compact_stage_bytes();
+// Buffer size and warps per CTA for the largest row a cache moves (bytes);
+// false when one row does not fit the shared-memory budget.
+bool compact_shape(int max_row_bytes, int &stage_bytes, int &warps);
+size_t compact_smem_bytes(const CompactParams &p);
 // Launches the pre-passes and the (cooperative) compaction; `sms` = SM count.
 cudaError_t launch_compact(const CompactParams &p, int sms, cudaStream_t st);
 

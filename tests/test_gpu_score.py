@@ -196,6 +196,32 @@ def test_compaction_adversarial_lists_bit_exact(pkg, kind):
     assert c["seq_len"].cpu().tolist() == cnt.tolist()
 
 
+@pytest.mark.parametrize("d_model", [6144, 16384])
+def test_compaction_wide_rows_bit_exact(pkg, d_model):
+    """H^(L-1) rows wider than the default 8 KB staging buffer (12 KB and
+    32 KB): the copy kernel stages one row per unit with fewer warps."""
+    from paper_2607_27600_gb300 import cc
+    shape = ModelShape(n_layers=1, d_model=d_model, n_q_heads=4, n_kv_heads=2, head_dim=64,
+                       d_ff=256, vocab=100, rope_theta=1e4, rms_eps=1e-5)
+    seq, cap = [700, 300], 768
+    c = synth.synthetic_cache(shape, seq, cap, seed=4, device="cuda")
+    before_h = c["h_last"].float().cpu().numpy()
+    before_k = c["k"][0].float().cpu().numpy()
+    r = np.random.default_rng(8)
+    idx = np.full((2, cap), -1, np.int32)
+    cnt = np.zeros(2, np.int32)
+    for b, n in enumerate(seq):
+        k = np.sort(np.concatenate([r.choice(n - 1, size=n // 3, replace=False), [n - 1]]))
+        idx[b, :len(k)] = k
+        cnt[b] = len(k)
+    cache = pkg.Cache(c)
+    ws = cc.alloc_workspace(cc.cc_compact_workspace_size(shape, cache))
+    cc.cc_compact_kv(shape, cache, torch.from_numpy(idx).cuda(), torch.from_numpy(cnt).cuda(), ws)
+    assert cc.cc_get_status() == cc.CC_OK
+    np.testing.assert_array_equal(c["h_last"].float().cpu().numpy(), oracle.compact(before_h, idx, cnt))
+    np.testing.assert_array_equal(c["k"][0].float().cpu().numpy(), oracle.compact(before_k, idx, cnt))
+
+
 @pytest.mark.parametrize("variant", ["qkv_bias", "rope_scaling", "both"])
 def test_model_variants_bias_and_rope_scaling(pkg, variant):
     """Qwen2-style q/k/v biases (the scorer adds the q bias before RoPE) and
