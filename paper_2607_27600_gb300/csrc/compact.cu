@@ -306,8 +306,9 @@ __global__ void __launch_bounds__(kThreads)
 bool compact_shape(int max_row_bytes, int &stage_bytes, int &warps) {
   stage_bytes = kCompactStageBytes;
   if (max_row_bytes > stage_bytes) stage_bytes = (max_row_bytes + 127) & ~127;
-  warps = (kCompactSmemBytes - 128) / (2 * stage_bytes);
+  warps = kCompactTargetBytes / (2 * stage_bytes);
   if (warps > kCompactMaxWarps) warps = kCompactMaxWarps;
+  if (warps < 1 && 2 * stage_bytes + 128 <= kCompactSmemBytes) warps = 1;
   return warps >= 1;
 }
 

@@ -5,13 +5,15 @@
 namespace cc {
 
 // Each warp of the copy kernel runs a two-buffer pipeline of units; a unit
-// stages up to one buffer of rows in shared memory.  Default shape: 12 warps
-// x 2 x 8 KB (measured fastest on Llama-3-8B caches: 2 KB K/V rows, 8 KB
-// H^(L-1) rows).  A cache with a larger row takes that row size as its
-// buffer and fewer warps, so shared memory still fits.
-constexpr int kCompactMaxWarps = 12;
-constexpr int kCompactStageBytes = 8 * 1024;
-constexpr int kCompactSmemBytes = 224 * 1024;   // dynamic shared memory budget of the copy kernel
+// stages up to one buffer of rows in shared memory.  The buffer is 4 KB, or
+// the largest row the cache moves if that is larger, and a CTA runs as many
+// warps as fill ~192 KB of staging (at most 24): measured fastest on
+// Llama-3-8B caches, 24 x 2 x 4 KB when only 2 KB K/V rows move, 12 x 2 x
+// 8 KB with 8 KB H^(L-1) rows.  Rows up to ~112 KB are supported (one warp).
+constexpr int kCompactMaxWarps = 24;
+constexpr int kCompactStageBytes = 4 * 1024;
+constexpr int kCompactTargetBytes = 192 * 1024;   // staging the shape aims for
+constexpr int kCompactSmemBytes = 224 * 1024;     // dynamic shared memory limit of the copy kernel
 constexpr int kMaxCompactArrays = 2 * 128 + 3;
 constexpr int kMaxDepClasses = 3;        // distinct chunk sizes (K/V rows, H rows, 4-byte rows)
 
