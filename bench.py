@@ -579,6 +579,7 @@ def append_work(shape, j, h):
     keys = h * j + h * (h + 1) // 2            # sum over chunk rows of the keys they attend
     return {"gemm_qrope": ("tensor", 2.0 * h * d * qd),
             "gemm_kv": ("tensor", 2.0 * h * d * kvd),
+            "gemm_qkv": ("tensor", 2.0 * h * d * (qd + 2 * kvd)),
             "attention_causal": ("tensor", 4.0 * dh * hq * keys),
             "gemm_oproj": ("tensor", 2.0 * h * qd * d),
             "gemm_gateup": ("tensor", 4.0 * h * d * f),

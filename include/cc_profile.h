@@ -33,7 +33,8 @@ typedef enum {
   CC_KERNEL_GEMM_KV = 13,    /* key (+ RoPE) and value projections (append)       */
   CC_KERNEL_ATTN_CAUSAL = 14,/* memory-augmented causal attention (append)        */
   CC_KERNEL_APPEND = 15,     /* append bookkeeping: tokens, positions, H^(L-1)    */
-  CC_KERNEL_COUNT = 16
+  CC_KERNEL_GEMM_QKV = 16,   /* fused q/k/v projections (+ RoPE) of the append    */
+  CC_KERNEL_COUNT = 17
 } cc_kernel_kind;
 
 /* on != 0: start recording (also clears earlier records); 0: stop. */

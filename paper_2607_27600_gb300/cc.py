@@ -106,7 +106,7 @@ _SIGS = {
     "cc_kernel_name": (ctypes.c_char_p, [ctypes.c_int32]),
     "cc_debug_withhold_compact_unit": (ctypes.c_int, [ctypes.c_int32]),
 }
-KERNEL_COUNT = 16
+KERNEL_COUNT = 17
 
 
 def library_path() -> str:

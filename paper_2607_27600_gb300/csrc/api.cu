@@ -246,7 +246,7 @@ cc_status device_fail() {
   } while (0)
 
 struct Gemm {
-  CUtensorMap a, b, b2;
+  CUtensorMap a, b, b2, b3;
   GemmParams p;
 };
 
@@ -266,6 +266,7 @@ cc_status gemm_setup(Gemm &g, int epi, const void *A, int K, const void *W, cons
   } else {
     g.b2 = g.b;
   }
+  g.b3 = g.b;
   memset(&g.p, 0, sizeof(g.p));
   g.p.batch = batch;
   g.p.cap = cap;
@@ -299,9 +300,37 @@ cc_status gemm_setup(Gemm &g, int epi, const void *A, int K, const void *W, cons
   return CC_OK;
 }
 
+// Fused q/k/v projections (one GEMM over the stacked weights [Wq; Wk; Wv]):
+// possible when both q_dim and kv_dim are whole 256-column tiles.
+bool qkv_fusable(const cc_model_cfg *c) {
+  return (c->n_q_heads * c->head_dim) % 256 == 0 && (c->n_kv_heads * c->head_dim) % 256 == 0;
+}
+
+cc_status gemm_setup_qkv(Gemm &g, const void *xn, const cc_model_cfg *c,
+                         const cc_layer_weights &lw, int batch, int cap, const int32_t *seq_len,
+                         unsigned *status, uint64_t rows_hint) {
+  const int d = c->d_model, qd = c->n_q_heads * c->head_dim, kvd = c->n_kv_heads * c->head_dim;
+  cc_status s = gemm_setup(g, EPI_QKV, xn, d, lw.wq, nullptr, qd + 2 * kvd, batch, cap, seq_len,
+                           status, false, rows_hint);
+  if (s != CC_OK) return s;
+  if (!tmap_rows(&g.b, lw.wq, qd, d, 256) || !tmap_rows(&g.b2, lw.wk, kvd, d, 256) ||
+      !tmap_rows(&g.b3, lw.wv, kvd, d, 256))
+    return tmap_fail();
+  g.p.n_q_tiles = qd / 256;
+  g.p.n_k_tiles = kvd / 256;
+  g.p.ldo = qd;
+  g.p.ldo_kv = kvd;
+  g.p.bias = reinterpret_cast<const __nv_bfloat16 *>(lw.bq);
+  g.p.bias_k = reinterpret_cast<const __nv_bfloat16 *>(lw.bk);
+  g.p.bias_v = reinterpret_cast<const __nv_bfloat16 *>(lw.bv);
+  g.p.head_dim = c->head_dim;
+  rope_turns(c, g.p.turns);
+  return CC_OK;
+}
+
 cc_status run_gemm(Gemm &g, int epi, int kind, int sms, cudaStream_t st) {
   TimedScope t(kind, st);
-  CC_TRY(launch_gemm(epi, g.a, g.b, g.b2, g.p, sms, st));
+  CC_TRY(launch_gemm(epi, g.a, g.b, g.b2, g.b3, g.p, sms, st));
   return CC_OK;
 }
 
@@ -441,11 +470,22 @@ cc_status run_append(const cc_model_cfg *c, const cc_model_weights *w, const cc_
     }
     // q = RoPE(xn Wq^T + bq) into the workspace; k = RoPE(xn Wk^T + bk) and
     // v = xn Wv^T + bv straight into the cache slots of the chunk
+    if (qkv_fusable(c)) {   // one GEMM over [Wq; Wk; Wv]
+      Gemm g;
+      if ((s = gemm_setup_qkv(g, xn, c, lw, batch, cap, hi, status, used)) != CC_OK) return s;
+      g.p.row_lo = lo;
+      g.p.out = q;
+      g.p.out_k = kv->k[l];
+      g.p.out_v = kv->v[l];
+      g.p.pos = kv->pos;
+      if ((s = run_gemm(g, EPI_QKV, CC_KERNEL_GEMM_QKV, dev->sms, st)) != CC_OK) return s;
+    }
     struct Proj { const void *w, *bias; void *out; int n, epi, kind; };
     const Proj projs[3] = {{lw.wq, lw.bq, q, qd, EPI_QROPE, CC_KERNEL_GEMM_QROPE},
                            {lw.wk, lw.bk, kv->k[l], kvd, EPI_QROPE, CC_KERNEL_GEMM_KV},
                            {lw.wv, lw.bv, kv->v[l], kvd, EPI_BF16, CC_KERNEL_GEMM_KV}};
     for (const Proj &pj : projs) {
+      if (qkv_fusable(c)) break;
       Gemm g;
       if ((s = gemm_setup(g, pj.epi, xn, d, pj.w, nullptr, pj.n, batch, cap, hi, status, false,
                           used)) != CC_OK)
@@ -925,7 +965,7 @@ const char *cc_kernel_name(int32_t kind) {
   static const char *names[CC_KERNEL_COUNT] = {
       "rmsnorm", "embed", "gemm_qrope", "attention", "gemm_oproj", "gemm_gateup", "gemm_down",
       "head_logit", "gemm_lmhead", "lse_combine", "select", "compact", "other",
-      "gemm_kv", "attention_causal", "append"};
+      "gemm_kv", "attention_causal", "append", "gemm_qkv"};
   return (kind >= 0 && kind < CC_KERNEL_COUNT) ? names[kind] : "unknown";
 }
 

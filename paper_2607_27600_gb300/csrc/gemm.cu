@@ -41,6 +41,89 @@ CC_DEV void rope_cs(uint32_t pos, unsigned long long turns, float &c, float &s) 
   __sincosf(ang, &s, &c);
 }
 
+// RoPE'd bf16 store of one accumulator tile row: destination columns
+// [col0, col0 + BN) of out (row stride ldo, n_dest columns in all), each tile
+// holding BN / head_dim whole heads; rotate-half pairs (k, k + dh/2); the
+// bias (optional) is added before the rotation.
+CC_DEV void rope_store(const GemmParams &p, uint32_t tacc, int grow, bool valid,
+                       __nv_bfloat16 *out_base, int ldo, const __nv_bfloat16 *bias, int col0,
+                       int n_dest) {
+  const int half = p.head_dim >> 1;
+  const uint32_t pos = valid ? (uint32_t)p.pos[grow] : 0u;
+  __nv_bfloat16 *out = out_base + (size_t)grow * ldo;
+#pragma unroll 1
+  for (int hb = 0; hb < BN; hb += p.head_dim) {
+#pragma unroll 1
+    for (int c0 = 0; c0 < half; c0 += 32) {
+      uint32_t x1[32], x2[32];
+      tmem_ld32(tacc + hb + c0, x1);
+      tmem_ld32(tacc + hb + half + c0, x2);
+      tmem_ld_wait();
+      int col = col0 + hb + c0;
+      if (!valid || col >= n_dest) continue;
+      uint32_t bb1[16], bb2[16];   // bias pairs of columns col.. and col+half.. (0 if none)
+#pragma unroll
+      for (int v = 0; v < 4; ++v) {
+        uint4 u1 = make_uint4(0, 0, 0, 0), u2 = make_uint4(0, 0, 0, 0);
+        if (bias) {
+          u1 = reinterpret_cast<const uint4 *>(bias + col)[v];
+          u2 = reinterpret_cast<const uint4 *>(bias + col + half)[v];
+        }
+        bb1[v * 4] = u1.x; bb1[v * 4 + 1] = u1.y; bb1[v * 4 + 2] = u1.z; bb1[v * 4 + 3] = u1.w;
+        bb2[v * 4] = u2.x; bb2[v * 4 + 1] = u2.y; bb2[v * 4 + 2] = u2.z; bb2[v * 4 + 3] = u2.w;
+      }
+      uint32_t o1[16], o2[16];
+#pragma unroll
+      for (int k = 0; k < 32; k += 2) {
+        float c_a, s_a, c_b, s_b;
+        rope_cs(pos, p.turns[c0 + k], c_a, s_a);
+        rope_cs(pos, p.turns[c0 + k + 1], c_b, s_b);
+        float a1 = __uint_as_float(x1[k]) + bf16_lo(bb1[k / 2]);
+        float a2 = __uint_as_float(x2[k]) + bf16_lo(bb2[k / 2]);
+        float b1 = __uint_as_float(x1[k + 1]) + bf16_hi(bb1[k / 2]);
+        float b2 = __uint_as_float(x2[k + 1]) + bf16_hi(bb2[k / 2]);
+        o1[k / 2] = pack_bf16x2(a1 * c_a - a2 * s_a, b1 * c_b - b2 * s_b);
+        o2[k / 2] = pack_bf16x2(a2 * c_a + a1 * s_a, b2 * c_b + b1 * s_b);
+      }
+      uint4 *d1 = reinterpret_cast<uint4 *>(out + col);
+      uint4 *d2 = reinterpret_cast<uint4 *>(out + col + half);
+#pragma unroll
+      for (int v = 0; v < 4; ++v) {
+        d1[v] = make_uint4(o1[v * 4], o1[v * 4 + 1], o1[v * 4 + 2], o1[v * 4 + 3]);
+        d2[v] = make_uint4(o2[v * 4], o2[v * 4 + 1], o2[v * 4 + 2], o2[v * 4 + 3]);
+      }
+    }
+  }
+}
+
+// Plain bf16 store (+ optional bias) of one accumulator tile row.
+CC_DEV void plain_store(uint32_t tacc, int grow, bool valid, __nv_bfloat16 *out_base, int ldo,
+                        const __nv_bfloat16 *bias, int col0, int n_dest) {
+  __nv_bfloat16 *out = out_base + (size_t)grow * ldo;
+#pragma unroll 1
+  for (int c = 0; c < BN / 32; ++c) {
+    uint32_t r[32];
+    tmem_ld32(tacc + c * 32, r);
+    tmem_ld_wait();
+    const int col = col0 + c * 32;
+    if (!valid || col >= n_dest) continue;
+    uint32_t bb[16];
+#pragma unroll
+    for (int v = 0; v < 4; ++v) {
+      const uint4 u = bias ? reinterpret_cast<const uint4 *>(bias + col)[v] : make_uint4(0, 0, 0, 0);
+      bb[v * 4] = u.x; bb[v * 4 + 1] = u.y; bb[v * 4 + 2] = u.z; bb[v * 4 + 3] = u.w;
+    }
+    uint32_t o[16];
+#pragma unroll
+    for (int k = 0; k < 32; k += 2)
+      o[k / 2] = pack_bf16x2(__uint_as_float(r[k]) + bf16_lo(bb[k / 2]),
+                             __uint_as_float(r[k + 1]) + bf16_hi(bb[k / 2]));
+    uint4 *d = reinterpret_cast<uint4 *>(out + col);
+#pragma unroll
+    for (int v = 0; v < 4; ++v) d[v] = make_uint4(o[v * 4], o[v * 4 + 1], o[v * 4 + 2], o[v * 4 + 3]);
+  }
+}
+
 template <int EPI>
 CC_DEV void epilogue_tile(const GemmParams &p, uint32_t tacc, int grow, bool valid, int nt,
                           int tile_n0) {
@@ -85,77 +168,23 @@ CC_DEV void epilogue_tile(const GemmParams &p, uint32_t tacc, int grow, bool val
       }
     }
   } else if constexpr (EPI == EPI_QROPE) {
-    // Tile columns = BN / head_dim whole heads; rotate-half pairs (k, k+dh/2).
-    const int half = p.head_dim >> 1;
-    const uint32_t pos = valid ? (uint32_t)p.pos[grow] : 0u;
-    __nv_bfloat16 *out = reinterpret_cast<__nv_bfloat16 *>(p.out) + (size_t)grow * p.ldo;
-#pragma unroll 1
-    for (int hb = 0; hb < BN; hb += p.head_dim) {
-#pragma unroll 1
-      for (int c0 = 0; c0 < half; c0 += 32) {
-        uint32_t x1[32], x2[32];
-        tmem_ld32(tacc + hb + c0, x1);
-        tmem_ld32(tacc + hb + half + c0, x2);
-        tmem_ld_wait();
-        int col = tile_n0 + hb + c0;
-        if (!valid || col >= p.N) continue;
-        uint32_t bb1[16], bb2[16];   // bias pairs of columns col.. and col+half.. (0 if none)
-#pragma unroll
-        for (int v = 0; v < 4; ++v) {
-          uint4 u1 = make_uint4(0, 0, 0, 0), u2 = make_uint4(0, 0, 0, 0);
-          if (p.bias) {
-            u1 = reinterpret_cast<const uint4 *>(p.bias + col)[v];
-            u2 = reinterpret_cast<const uint4 *>(p.bias + col + half)[v];
-          }
-          bb1[v * 4] = u1.x; bb1[v * 4 + 1] = u1.y; bb1[v * 4 + 2] = u1.z; bb1[v * 4 + 3] = u1.w;
-          bb2[v * 4] = u2.x; bb2[v * 4 + 1] = u2.y; bb2[v * 4 + 2] = u2.z; bb2[v * 4 + 3] = u2.w;
-        }
-        uint32_t o1[16], o2[16];
-#pragma unroll
-        for (int k = 0; k < 32; k += 2) {
-          float c_a, s_a, c_b, s_b;
-          rope_cs(pos, p.turns[c0 + k], c_a, s_a);
-          rope_cs(pos, p.turns[c0 + k + 1], c_b, s_b);
-          float a1 = __uint_as_float(x1[k]) + bf16_lo(bb1[k / 2]);
-          float a2 = __uint_as_float(x2[k]) + bf16_lo(bb2[k / 2]);
-          float b1 = __uint_as_float(x1[k + 1]) + bf16_hi(bb1[k / 2]);
-          float b2 = __uint_as_float(x2[k + 1]) + bf16_hi(bb2[k / 2]);
-          o1[k / 2] = pack_bf16x2(a1 * c_a - a2 * s_a, b1 * c_b - b2 * s_b);
-          o2[k / 2] = pack_bf16x2(a2 * c_a + a1 * s_a, b2 * c_b + b1 * s_b);
-        }
-        uint4 *d1 = reinterpret_cast<uint4 *>(out + col);
-        uint4 *d2 = reinterpret_cast<uint4 *>(out + col + half);
-#pragma unroll
-        for (int v = 0; v < 4; ++v) {
-          d1[v] = make_uint4(o1[v * 4], o1[v * 4 + 1], o1[v * 4 + 2], o1[v * 4 + 3]);
-          d2[v] = make_uint4(o2[v * 4], o2[v * 4 + 1], o2[v * 4 + 2], o2[v * 4 + 3]);
-        }
-      }
-    }
+    rope_store(p, tacc, grow, valid, reinterpret_cast<__nv_bfloat16 *>(p.out), p.ldo, p.bias,
+               tile_n0, p.N);
   } else if constexpr (EPI == EPI_BF16) {
-    __nv_bfloat16 *out = reinterpret_cast<__nv_bfloat16 *>(p.out) + (size_t)grow * p.ldo;
-#pragma unroll 1
-    for (int c = 0; c < BN / 32; ++c) {
-      uint32_t r[32];
-      tmem_ld32(tacc + c * 32, r);
-      tmem_ld_wait();
-      const int col = tile_n0 + c * 32;
-      if (!valid || col >= p.N) continue;
-      uint32_t bb[16];
-#pragma unroll
-      for (int v = 0; v < 4; ++v) {
-        const uint4 u = p.bias ? reinterpret_cast<const uint4 *>(p.bias + col)[v] : make_uint4(0, 0, 0, 0);
-        bb[v * 4] = u.x; bb[v * 4 + 1] = u.y; bb[v * 4 + 2] = u.z; bb[v * 4 + 3] = u.w;
-      }
-      uint32_t o[16];
-#pragma unroll
-      for (int k = 0; k < 32; k += 2)
-        o[k / 2] = pack_bf16x2(__uint_as_float(r[k]) + bf16_lo(bb[k / 2]),
-                               __uint_as_float(r[k + 1]) + bf16_hi(bb[k / 2]));
-      uint4 *d = reinterpret_cast<uint4 *>(out + col);
-#pragma unroll
-      for (int v = 0; v < 4; ++v) d[v] = make_uint4(o[v * 4], o[v * 4 + 1], o[v * 4 + 2], o[v * 4 + 3]);
-    }
+    plain_store(tacc, grow, valid, reinterpret_cast<__nv_bfloat16 *>(p.out), p.ldo, p.bias,
+                tile_n0, p.N);
+  } else if constexpr (EPI == EPI_QKV) {
+    // fused projections: column tiles [0, nq) are Q, [nq, nq+nk) K, the rest V
+    const int nq = p.n_q_tiles, nk = p.n_k_tiles;
+    if (nt < nq)
+      rope_store(p, tacc, grow, valid, reinterpret_cast<__nv_bfloat16 *>(p.out), p.ldo, p.bias,
+                 nt * BN, nq * BN);
+    else if (nt < nq + nk)
+      rope_store(p, tacc, grow, valid, reinterpret_cast<__nv_bfloat16 *>(p.out_k), p.ldo_kv,
+                 p.bias_k, (nt - nq) * BN, nk * BN);
+    else
+      plain_store(tacc, grow, valid, reinterpret_cast<__nv_bfloat16 *>(p.out_v), p.ldo_kv,
+                  p.bias_v, (nt - nq - nk) * BN, nk * BN);
   } else if constexpr (EPI == EPI_SWIGLU) {
     // columns [0,128) = gate rows nt*128.., [128,256) = up rows nt*128..
     __nv_bfloat16 *out = reinterpret_cast<__nv_bfloat16 *>(p.out) + (size_t)grow * p.ldo;
@@ -250,7 +279,8 @@ CC_DEV void tile_coords(const GemmParams &p, int t, int num_m, int &m, int &n) {
 template <int EPI>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                const __grid_constant__ CUtensorMap tmB2, const __grid_constant__ GemmParams p) {
+                const __grid_constant__ CUtensorMap tmB2, const __grid_constant__ CUtensorMap tmB3,
+                const __grid_constant__ GemmParams p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                               ~uintptr_t(1023));
@@ -281,7 +311,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 0 && lane == 0) {
     tma_prefetch_desc(&tmA);
     tma_prefetch_desc(&tmB);
-    if (EPI == EPI_SWIGLU) tma_prefetch_desc(&tmB2);
+    if (EPI == EPI_SWIGLU || EPI == EPI_QKV) tma_prefetch_desc(&tmB2);
+    if (EPI == EPI_QKV) tma_prefetch_desc(&tmB3);
   }
   if (warp == 1) tmem_alloc(tmem_slot, 512);
   tc_fence_before();
@@ -316,6 +347,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             tma_load_2d_hint(sB + stage * B_BYTES, &tmB, &full[stage], kw, nt * 128, pol_b);
             tma_load_2d_hint(sB + stage * B_BYTES + B_BYTES / 2, &tmB2, &full[stage], kw, nt * 128,
                              pol_b);
+          } else if constexpr (EPI == EPI_QKV) {
+            const int nq = p.n_q_tiles, nk = p.n_k_tiles;
+            const CUtensorMap *m = nt < nq ? &tmB : (nt < nq + nk ? &tmB2 : &tmB3);
+            const int r0 = (nt < nq ? nt : (nt < nq + nk ? nt - nq : nt - nq - nk)) * BN;
+            tma_load_2d_hint(sB + stage * B_BYTES, m, &full[stage], kw, r0, pol_b);
           } else {
             tma_load_2d_hint(sB + stage * B_BYTES, &tmB, &full[stage], kw, nt * BN, pol_b);
           }
@@ -386,7 +422,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 template <int EPI>
 cudaError_t launch(const CUtensorMap &a, const CUtensorMap &b, const CUtensorMap &b2,
-                   const GemmParams &p, int grid, cudaStream_t stream) {
+                   const CUtensorMap &b3, const GemmParams &p, int grid, cudaStream_t stream) {
   auto kern = gemm_kernel<EPI>;
   static bool attr_set[64] = {};
   int dev = 0;
@@ -397,7 +433,7 @@ cudaError_t launch(const CUtensorMap &a, const CUtensorMap &b, const CUtensorMap
     if (e != cudaSuccess) return e;
     attr_set[dev] = true;
   }
-  kern<<<grid, kThreads, kSmemBytes, stream>>>(a, b, b2, p);
+  kern<<<grid, kThreads, kSmemBytes, stream>>>(a, b, b2, b3, p);
   return cudaGetLastError();
 }
 
@@ -407,15 +443,16 @@ int gemm_block_n(int epi) { return epi == EPI_SWIGLU ? 128 : BN; }
 int gemm_max_batch() { return kMaxBatch; }
 
 cudaError_t launch_gemm(int epi, const CUtensorMap &a, const CUtensorMap &b, const CUtensorMap &b2,
-                        const GemmParams &p, int grid, cudaStream_t stream) {
+                        const CUtensorMap &b3, const GemmParams &p, int grid, cudaStream_t stream) {
   switch (epi) {
-    case EPI_F32: return launch<EPI_F32>(a, b, b2, p, grid, stream);
-    case EPI_QROPE: return launch<EPI_QROPE>(a, b, b2, p, grid, stream);
-    case EPI_RESID_BF16: return launch<EPI_RESID_BF16>(a, b, b2, p, grid, stream);
-    case EPI_RESID_F32: return launch<EPI_RESID_F32>(a, b, b2, p, grid, stream);
-    case EPI_SWIGLU: return launch<EPI_SWIGLU>(a, b, b2, p, grid, stream);
-    case EPI_LSE: return launch<EPI_LSE>(a, b, b2, p, grid, stream);
-    case EPI_BF16: return launch<EPI_BF16>(a, b, b2, p, grid, stream);
+    case EPI_F32: return launch<EPI_F32>(a, b, b2, b3, p, grid, stream);
+    case EPI_QROPE: return launch<EPI_QROPE>(a, b, b2, b3, p, grid, stream);
+    case EPI_RESID_BF16: return launch<EPI_RESID_BF16>(a, b, b2, b3, p, grid, stream);
+    case EPI_RESID_F32: return launch<EPI_RESID_F32>(a, b, b2, b3, p, grid, stream);
+    case EPI_SWIGLU: return launch<EPI_SWIGLU>(a, b, b2, b3, p, grid, stream);
+    case EPI_LSE: return launch<EPI_LSE>(a, b, b2, b3, p, grid, stream);
+    case EPI_BF16: return launch<EPI_BF16>(a, b, b2, b3, p, grid, stream);
+    case EPI_QKV: return launch<EPI_QKV>(a, b, b2, b3, p, grid, stream);
     default: return cudaErrorInvalidValue;
   }
 }

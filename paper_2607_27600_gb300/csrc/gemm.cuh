@@ -12,7 +12,9 @@ enum GemmEpi : int {
   EPI_SWIGLU = 4,     // out bf16 [rows][ldo] = silu(A Wg^T) * (A Wu^T)   (B = Wg, B2 = Wu)
   EPI_LSE = 5,        // out float2 [rows][ldo = n_tiles] = (max, sum exp) per vocab tile,
                       // z_target[row] = logit of tokens[row]
-  EPI_BF16 = 6        // out bf16 [rows][ldo] = acc (+ bias[col] if bias)
+  EPI_BF16 = 6,       // out bf16 [rows][ldo] = acc (+ bias[col] if bias)
+  EPI_QKV = 7         // fused q/k/v projections (B = Wq, B2 = Wk, B3 = Wv, stacked by column
+                      // tiles): Q RoPE'd to out, K RoPE'd to out_k, V to out_v
 };
 
 struct GemmParams {
@@ -37,14 +39,19 @@ struct GemmParams {
                            // row tiles stay resident (A kept, B streamed per group)
   int group;
   int out_split;           // EPI_SWIGLU: out rows are [hi | lo], lo at column offset N
+  int n_q_tiles, n_k_tiles;   // EPI_QKV: column tiles of Q and of K (V has n_k_tiles too)
+  void *out_k, *out_v;        // EPI_QKV: bf16 [rows][ldo_kv] destinations of K and V
+  int ldo_kv;
+  const __nv_bfloat16 *bias_k, *bias_v;   // EPI_QKV: optional biases of K and V
   unsigned long long turns[64];  // EPI_QROPE: inv_freq_k / (2 pi) in 0.64 fixed point
 };
 
 int gemm_block_n(int epi);
 int gemm_max_batch();
-// a: A rows x K (box 64 x 128); b (and b2 for SwiGLU): weights N x K (box 64 x 256,
-// or 64 x 128 for SwiGLU).  grid: persistent CTAs (one per SM).
+// a: A rows x K (box 64 x 128); b (and b2 for SwiGLU, b2 and b3 for the fused
+// projections): weights N x K (box 64 x 256, or 64 x 128 for SwiGLU).
+// grid: persistent CTAs (one per SM).
 cudaError_t launch_gemm(int epi, const CUtensorMap &a, const CUtensorMap &b, const CUtensorMap &b2,
-                        const GemmParams &p, int grid, cudaStream_t stream);
+                        const CUtensorMap &b3, const GemmParams &p, int grid, cudaStream_t stream);
 
 }  // namespace cc
