@@ -14,6 +14,7 @@
 #include <stdio.h>
 
 #include <algorithm>
+#include <atomic>
 #include <mutex>
 
 #include "attn.cuh"
@@ -169,9 +170,12 @@ cc_status check_cfg(const cc_model_cfg *c) {
 size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
 struct ScoreWs {
-  size_t xn, q, o, h, act, part, ztgt, total;
+  size_t xn, q, o, h, act, part, ztgt, flags, total;
   int n_vtiles;
 };
+
+// Per-tile progress flags of split-K GEMMs (at most one wave of tiles split).
+constexpr int kSplitFlags = 1024;
 
 // With CC_SCORE_PRECISE the full pass carries the GEMM activations
 // (normalised inputs, attention output, SwiGLU output) as [hi | lo] bf16
@@ -193,6 +197,7 @@ ScoreWs score_layout(const cc_model_cfg *c, int batch, int cap, cc_score_mode mo
     w.part = take(R * w.n_vtiles * 8);
     w.ztgt = take(R * 4);
   }
+  w.flags = take(kSplitFlags * 4);
   w.total = off;
   return w;
 }
@@ -248,6 +253,7 @@ cc_status device_fail() {
 struct Gemm {
   CUtensorMap a, b, b2, b3;
   GemmParams p;
+  uint64_t rows_est;   // rows visited at most (tile-count estimate on the host)
 };
 
 // One GEMM over the cache rows: A [R][K] (bf16 workspace) x W [N][K]^T.
@@ -287,6 +293,7 @@ cc_status gemm_setup(Gemm &g, int epi, const void *A, int K, const void *W, cons
   // below 0.8x (an LM head whose weight is far larger than L2).
   const double budget = 40.0 * (1 << 20);
   const uint64_t R_used = rows_hint ? rows_hint : R;
+  g.rows_est = R_used;
   const int num_m = (int)((R_used + 127) / 128), num_n = g.p.n_tiles;
   const double k_a = (a_split ? 2.0 : 1.0) * K;
   const double a_bytes = (double)R_used * k_a * 2, b_bytes = (double)num_n * 256 * K * 2;
@@ -325,6 +332,32 @@ cc_status gemm_setup_qkv(Gemm &g, const void *xn, const cc_model_cfg *c,
   g.p.bias_v = reinterpret_cast<const __nv_bfloat16 *>(lw.bv);
   g.p.head_dim = c->head_dim;
   rope_turns(c, g.p.turns);
+  return CC_OK;
+}
+
+// K splits for a residual GEMM with less than one wave of output tiles
+// (short caches): each split is a work item; splits add into the fp32
+// residual in order (flags in the caller's workspace, tagged per launch).
+void plan_k_splits(Gemm &g, int epi, int sms, unsigned *flags) {
+  g.p.k_splits = 1;
+  if (epi != EPI_RESID_F32 || !flags) return;
+  const uint64_t tiles = ((g.rows_est + 127) / 128) * (uint64_t)g.p.n_tiles;
+  const int nk_total = ((g.p.K + 63) / 64) * (g.p.a_split ? 2 : 1);
+  if (tiles == 0 || tiles >= (uint64_t)sms || tiles > (uint64_t)kSplitFlags) return;
+  // >= 64 k-blocks (K >= 4096) per split: shorter splits lose more to the
+  // ordered epilogues than they gain (measured on Qwen2.5 O projections)
+  int splits = std::min<int>((int)(sms / tiles), std::min(8, nk_total / 64));
+  if (splits < 2) return;
+  static std::atomic<unsigned> epoch{0};
+  g.p.k_splits = splits;
+  g.p.split_flags = flags;
+  g.p.epoch = (epoch.fetch_add(1) % (1u << 27)) + 1;   // flags hold epoch * 16 + split
+}
+
+// Zeroes the split-K flags of a workspace once per call (a fresh workspace
+// may hold any bits; later launches tag their values with new epochs).
+cc_status clear_split_flags(unsigned *flags, cudaStream_t st) {
+  CC_TRY(cudaMemsetAsync(flags, 0, kSplitFlags * 4, st));
   return CC_OK;
 }
 
@@ -446,7 +479,9 @@ cc_status run_append(const cc_model_cfg *c, const cc_model_weights *w, const cc_
   void *xn = wsb + L.s.xn, *q = wsb + L.s.q, *o = wsb + L.s.o, *act = wsb + L.s.act;
   float *h = reinterpret_cast<float *>(wsb + L.s.h);
   int32_t *lo = reinterpret_cast<int32_t *>(wsb + L.lo), *hi = reinterpret_cast<int32_t *>(wsb + L.hi);
+  unsigned *flags = reinterpret_cast<unsigned *>(wsb + L.s.flags);
   unsigned *status = dev->status;
+  if ((s = clear_split_flags(flags, st)) != CC_OK) return s;
   const uint64_t used = (uint64_t)batch * max_count;   // rows the GEMMs visit at most
 
   {
@@ -511,6 +546,7 @@ cc_status run_append(const cc_model_cfg *c, const cc_model_weights *w, const cc_
     go.p.row_lo = lo;
     go.p.out = h;
     go.p.ldo = d;
+    plan_k_splits(go, EPI_RESID_F32, dev->sms, flags);
     if ((s = run_gemm(go, EPI_RESID_F32, CC_KERNEL_GEMM_OPROJ, dev->sms, st)) != CC_OK) return s;
     {
       TimedScope t(CC_KERNEL_RMSNORM, st);
@@ -531,6 +567,7 @@ cc_status run_append(const cc_model_cfg *c, const cc_model_weights *w, const cc_
     gd.p.row_lo = lo;
     gd.p.out = h;
     gd.p.ldo = d;
+    plan_k_splits(gd, EPI_RESID_F32, dev->sms, flags);
     if ((s = run_gemm(gd, EPI_RESID_F32, CC_KERNEL_GEMM_DOWN, dev->sms, st)) != CC_OK) return s;
   }
   {
@@ -592,6 +629,8 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
   float *h = reinterpret_cast<float *>(wsb + L.h);
   const int32_t *sl = kv->seq_len;
   unsigned *status = dev->status;
+  unsigned *flags = reinterpret_cast<unsigned *>(wsb + L.flags);
+  if ((s = clear_split_flags(flags, st)) != CC_OK) return s;
 
   if (full) {
     TimedScope t(CC_KERNEL_EMBED, st);
@@ -633,6 +672,7 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
     go.p.ldo = d;
     go.p.resid = kv->h_last;
     go.p.ld_resid = d;
+    plan_k_splits(go, epi_o, dev->sms, flags);
     if ((s = run_gemm(go, epi_o, CC_KERNEL_GEMM_OPROJ, dev->sms, st)) != CC_OK) return s;
     // xn = RMSNorm(h); act = silu(xn Wg^T) * (xn Wu^T)
     {
@@ -654,6 +694,7 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
       return s;
     gd.p.out = h;
     gd.p.ldo = d;
+    plan_k_splits(gd, EPI_RESID_F32, dev->sms, flags);
     if ((s = run_gemm(gd, EPI_RESID_F32, CC_KERNEL_GEMM_DOWN, dev->sms, st)) != CC_OK) return s;
   }
   // head

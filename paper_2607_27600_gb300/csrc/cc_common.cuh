@@ -125,6 +125,31 @@ CC_DEV uint64_t make_policy_evict_first() {
   asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
   return p;
 }
+// Barrier among `threads` threads (a multiple of 32) of the CTA, id 1..15.
+CC_DEV void named_barrier_sync(int id, int threads) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(threads) : "memory");
+}
+CC_DEV void st_release_u32(unsigned *p, unsigned v) {
+  asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+CC_DEV unsigned ld_acquire_u32(const unsigned *p) {
+  unsigned v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+// Waits until *p == want; false (CC_ERR_TIMEOUT recorded) after kWaitLimitNs.
+CC_DEV bool wait_value(const unsigned *p, unsigned want, unsigned *status) {
+  if (ld_acquire_u32(p) == want) return true;
+  const uint64_t t0 = globaltimer();
+  for (uint32_t it = 1;; ++it) {
+    __nanosleep(64);
+    if (ld_acquire_u32(p) == want) return true;
+    if ((it & 255u) == 0 && globaltimer() - t0 > kWaitLimitNs) {
+      set_status(status, CC_ERR_TIMEOUT);
+      return false;
+    }
+  }
+}
 // Contiguous global -> shared copy (16-byte aligned addresses, size % 16 == 0).
 CC_DEV void bulk_load(void *dst, const void *src, uint32_t bytes, uint64_t *bar) {
   asm volatile(

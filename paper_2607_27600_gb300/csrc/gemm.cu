@@ -293,6 +293,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(tempty + 2);
   volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
   int *prefix = reinterpret_cast<int *>(smem + ST * (A_BYTES + B_BYTES) + 256);
+  __shared__ int split_ok;   // K splits: the previous split of the tile has published
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
@@ -323,6 +324,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int total = num_m * p.n_tiles;
   const int nk = (p.K + BK - 1) / BK;           // k-blocks of one operand pass
   const int nk_total = p.a_split ? 2 * nk : nk;  // split A: the hi pass, then the lo pass
+  // Work item = (tile, K split): the splits of a tile are consecutive items.
+  const int S = (EPI == EPI_RESID_F32 && p.k_splits > 1) ? p.k_splits : 1;
+  const int total_items = total * S;
 
   if (warp == 0) {
     if (lane == 0) {  // ---------------- TMA producer
@@ -331,12 +335,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint64_t pol_b = p.raster == 0 ? keep : stream;
       int stage = 0;
       uint32_t phase = 0;
-      for (int tile = blockIdx.x; tile < total; tile += gridDim.x) {
+      for (int item = blockIdx.x; item < total_items; item += gridDim.x) {
+        const int tile = item / S, split = item - tile * S;
         int mt, nt;
         tile_coords(p, tile, num_m, mt, nt);
         const int b = find_seq(prefix, p.batch, mt);
         const int row0 = b * p.cap + (p.row_lo ? p.row_lo[b] : 0) + (mt - prefix[b]) * BM;
-        for (int kb = 0; kb < nk_total; ++kb) {
+        const int kb0 = split * nk_total / S, kb1 = (split + 1) * nk_total / S;
+        for (int kb = kb0; kb < kb1; ++kb) {
           if (!mbar_wait(&empty[stage], phase ^ 1, abort_flag, p.status)) goto producer_done;
           mbar_arrive_expect_tx(&full[stage], A_BYTES + B_BYTES);
           // A column block kb of [hi | lo] (hi and lo halves are K apart), B block kb mod nk
@@ -367,11 +373,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint64_t b_desc0 = make_sdesc_sw128(smem_u32(sB), 16, 1024);
       int stage = 0, acc = 0;
       uint32_t phase = 0, acc_phase = 0;
-      for (int tile = blockIdx.x; tile < total; tile += gridDim.x) {
+      for (int item = blockIdx.x; item < total_items; item += gridDim.x) {
+        const int split = item % S;
+        const int kb0 = split * nk_total / S, kb1 = (split + 1) * nk_total / S;
         if (!mbar_wait(&tempty[acc], acc_phase ^ 1, abort_flag, p.status)) break;
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + acc * BN;
-        for (int kb = 0; kb < nk_total; ++kb) {
+        for (int kb = kb0; kb < kb1; ++kb) {
           if (!mbar_wait(&full[stage], phase, abort_flag, p.status)) goto mma_done;
           tc_fence_after();
           // descriptors of this stage; a K step of 16 columns advances the
@@ -379,7 +387,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint64_t ad = a_desc0 + (uint64_t)(stage * (A_BYTES >> 4));
           const uint64_t bd = b_desc0 + (uint64_t)(stage * (B_BYTES >> 4));
 #pragma unroll
-          for (int k = 0; k < BK / 16; ++k) umma_ss(d_tmem, ad + 2 * k, bd + 2 * k, idesc, (kb | k) != 0);
+          for (int k = 0; k < BK / 16; ++k)
+            umma_ss(d_tmem, ad + 2 * k, bd + 2 * k, idesc, (kb != kb0 || k != 0) ? 1u : 0u);
           umma_commit(&empty[stage]);
           if (++stage == ST) { stage = 0; phase ^= 1; }
         }
@@ -393,7 +402,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int r = q * 32 + lane;   // accumulator row of this thread
     int acc = 0;
     uint32_t acc_phase = 0;
-    for (int tile = blockIdx.x; tile < total; tile += gridDim.x) {
+    for (int item = blockIdx.x; item < total_items; item += gridDim.x) {
+      const int tile = item / S, split = item - tile * S;
       int mt, nt;
       tile_coords(p, tile, num_m, mt, nt);
       const int b = find_seq(prefix, p.batch, mt);
@@ -403,8 +413,26 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!mbar_wait(&tfull[acc], acc_phase, abort_flag, p.status)) break;
       tc_fence_after();
       const uint32_t tacc = tmem_base + acc * BN + (uint32_t(q * 32) << 16);
-      epilogue_tile<EPI>(p, tacc, grow, valid, nt, nt * BN);
+      // K splits add into out in split order (deterministic sums): split s
+      // waits until split s-1 of the tile has published epoch * 16 + s.
+      // Split s-1 is a lower work item, and every CTA takes its items in
+      // increasing order, so the wait always ends (bounded all the same).
+      bool add = true;
+      if (S > 1) {
+        if (warp == 2 && lane == 0)
+          split_ok = split == 0 || wait_value(&p.split_flags[tile], p.epoch * 16u + split, p.status);
+        named_barrier_sync(1, 128);
+        add = split_ok != 0;   // a wait that gave up (status set) skips this split's add
+      }
+      if (add) epilogue_tile<EPI>(p, tacc, grow, valid, nt, nt * BN);
       tc_fence_before();
+      if (S > 1) {
+        named_barrier_sync(1, 128);
+        if (warp == 2 && lane == 0) {
+          __threadfence();
+          st_release_u32(&p.split_flags[tile], p.epoch * 16u + split + 1);
+        }
+      }
       __syncwarp();
       if (lane == 0) mbar_arrive(&tempty[acc]);
       if (++acc == 2) { acc = 0; acc_phase ^= 1; }

@@ -39,6 +39,10 @@ struct GemmParams {
                            // row tiles stay resident (A kept, B streamed per group)
   int group;
   int out_split;           // EPI_SWIGLU: out rows are [hi | lo], lo at column offset N
+  int k_splits;            // EPI_RESID_F32 only: K range split over k_splits work items per
+                           // tile (< one wave of tiles); the splits add into out in order
+  unsigned *split_flags;   // [tiles] (k_splits > 1): per-tile progress, epoch * 16 + split
+  unsigned epoch;          // per-launch tag (>= 1) of split_flags values
   int n_q_tiles, n_k_tiles;   // EPI_QKV: column tiles of Q and of K (V has n_k_tiles too)
   void *out_k, *out_v;        // EPI_QKV: bf16 [rows][ldo_kv] destinations of K and V
   int ldo_kv;

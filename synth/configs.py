@@ -54,6 +54,9 @@ class Workload:
     cycles: int = 1                # refresh cycles (appends of `append` slots between them)
     append: int = 0
     n_sink: int = 0
+    # the paper's own figure for this exact workload, as scored positions/s
+    # (n / refresh latency), if it reports one; another GPU's number: context
+    paper_positions_per_s: float = 0.0
 
     @property
     def batch(self) -> int:
@@ -90,5 +93,16 @@ WORKLOADS = {
                                   131072 + 4096, seed=4, cache_from_causal_pass=False,
                                   cycles=4, append=4096),
 }
+
+# The paper's efficiency benchmark (Table 1): Qwen2.5-7B, a synthetic KV cache
+# of n = 512 or 4096 slots, full L-layer pass and fast single-layer pass
+# (RTX 4090, fp16: 54 / 496 ms full, 7.9 / 52.6 ms fast).  The table does not
+# state the budget; these keep half the slots.
+for _n, _full_ms, _fast_ms in ((512, 54.0, 7.9), (4096, 496.0, 52.6)):
+    for _mode, _ms in (("full", _full_ms), ("layer", _fast_ms)):
+        _name = f"qwen7b-table1-{'full' if _mode == 'full' else 'fast'}-{_n}"
+        WORKLOADS[_name] = Workload(_name, QWEN25_7B, _mode, [_n], [_n // 2], _n, seed=5,
+                                    cache_from_causal_pass=False,
+                                    paper_positions_per_s=_n / (_ms * 1e-3))
 
 HEADLINE = "llama8b-layer-8k"

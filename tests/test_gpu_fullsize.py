@@ -140,6 +140,9 @@ def test_fast_pass_logprob_full_size(pkg):
 # 2e-2 on the first four layers of the same model and shapes.
 FULL32_TOL = 1.5e-1        # bf16 activations, 32 layers
 FULL32_PRECISE_TOL = 1e-1  # hi + lo GEMM activations (CC_SCORE_PRECISE), 32 layers
+# The 28-layer Qwen2.5 pass at 512 slots: held to the 32-layer Llama bar (the
+# same rounding points; fewer layers and keys, so no larger drift expected).
+FULL28_TOL = FULL32_TOL
 
 
 def _full_inputs(n_layers):
@@ -249,3 +252,23 @@ def test_long_context_refresh_cycles(pkg):
         cn["k"][last][:, s0:s1] = f32(c["k"][last][:, s0:s1])
         cn["v"][last][:, s0:s1] = f32(c["v"][last][:, s0:s1])
         cn["seq_len"] = c["seq_len"].cpu().numpy()
+
+
+@pytest.mark.parametrize("name", ["qwen7b-table1-fast-4096", "qwen7b-table1-full-512"])
+def test_paper_table1_workloads(pkg, name):
+    """The paper's efficiency benchmark shapes (Qwen2.5-7B, synthetic cache):
+    the fast pass at 4096 slots on every row, the full 28-layer pass at 512
+    slots on sampled rows, in the launch configuration bench.py times."""
+    from paper_2607_27600_gb300 import cc
+    wl = synth.WORKLOADS[name]
+    fast = wl.mode == "layer"
+    w, c = workload_inputs(wl)
+    got = gpu_scores(pkg, wl.shape, w, c, cc.SCORE_LOGIT, full=not fast)
+    wn, cn = host_view(w, c, lazy=not fast)
+    if fast:
+        want = oracle.score_layer(wl.shape, wn, cn)
+        assert rel_err(got[0, :wl.seq_lens[0]], want[0, :wl.seq_lens[0]]) < TOL
+    else:
+        rows = sample(wl.seq_lens, 10, seed=6)
+        want = oracle.score_full(wl.shape, wn, cn, rows=rows)
+        assert check_rows(got, want, rows) < FULL28_TOL

@@ -250,3 +250,20 @@ def test_model_variants_bias_and_rope_scaling(pkg, variant):
         assert rel_err(got, want) < TOL, (variant, full, rel_err(got, want))
         other = fn(plain, w_plain, c_np)
         assert rel_err(other, want) > 5 * TOL, (variant, full, rel_err(other, want))
+
+
+def test_split_k_residual_gemms_deterministic(pkg):
+    """A short cache with a wide MLP (one output tile per residual GEMM, K =
+    32768): the down projection runs as 8 K splits adding into the residual in
+    order; full and fast pass match the oracle, and two runs are bit-identical."""
+    from paper_2607_27600_gb300 import cc
+    shape = ModelShape(n_layers=2, d_model=256, n_q_heads=8, n_kv_heads=2, head_dim=64,
+                       d_ff=32768, vocab=1000, rope_theta=1e4, rms_eps=1e-5)
+    w_np, c_np = _setup(shape, [100, 37], 128, seed=27)
+    weights, cache = _gpu(pkg, w_np, c_np)
+    for full, fn in ((True, oracle.score_full), (False, oracle.score_layer)):
+        want = fn(shape, w_np, c_np)
+        a = _run_score(pkg, shape, weights, cache, cc.SCORE_LOGIT, full=full)
+        b = _run_score(pkg, shape, weights, cache, cc.SCORE_LOGIT, full=full)
+        assert rel_err(a, want) < TOL, (full, rel_err(a, want))
+        np.testing.assert_array_equal(a, b)
