@@ -25,6 +25,12 @@ Parity status per function (what pins it, in tests/test_oracle_*.py):
   compact                  sequential in-place loop; order preservation
   memory_causal_attention  torch SDPA with an explicit mask (memory all visible,
                            chunk causal); n0 = 0 is causal_attention
+  recency_scores           the position itself (keep-set = most recent slots)
+  key_attention_colsums    column sums = sum of the attention matrix's entries;
+                           each query row sums to 1; torch SDPA weights (library
+                           routine) with keys as queries
+  importance/h2o scores    closed forms (one head, equal keys -> uniform); H2O
+                           over two refreshes = one update with both layer sets
   append_chunk             into an empty cache = causal_forward; chunk-by-chunk
                            appends = one append (no refresh between); the layer's
                            attention after a compaction by scalar brute force
@@ -35,4 +41,5 @@ from .refresh import (rms_norm, rope, rope_angles, rope_inv_freq, project, softm
                       counter_causal_attention,
                       causal_attention, silu, swiglu_mlp, counter_causal_layer, score_head,
                       score_layer, score_full, select_keep, compact, causal_forward,
-                      memory_causal_attention, append_chunk)
+                      memory_causal_attention, append_chunk, recency_scores,
+                      key_attention_colsums, importance_scores, h2o_update, h2o_scores)

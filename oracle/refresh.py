@@ -411,3 +411,80 @@ def append_chunk(shape, weights, cache, b, tokens, pos=None):
     cache["pos"][b][sl] = pos
     cache["seq_len"][b] = n0 + h
     return x
+
+
+# ----------------------------------------------------------------------------
+# The paper's comparison scorers (Sec. 4): sliding window, importance, H2O.
+# They rank the same cached slots for the same keep-set selection and
+# compaction; the attention-based ones use cached keys as proxy queries.
+# ----------------------------------------------------------------------------
+
+def recency_scores(cache):
+    """Sliding window (first in, first out): the score of a slot is its
+    original position, so the keep-set is the most recent slots."""
+    pos = np.asarray(cache["pos"])
+    seq_len = np.asarray(cache["seq_len"])
+    out = np.full(pos.shape, NEG_INF)
+    for b in range(pos.shape[0]):
+        n = int(seq_len[b])
+        out[b, :n] = pos[b, :n]
+    return out
+
+
+def key_attention_colsums(k, n, q_lo):
+    """Attention received by each key under the causal mask when the keys of
+    slots [q_lo, n) act as queries (proxy queries, Sec. 4): for each KV head
+    g, A_g = softmax over j <= i of K_g[i] . K_g[j] / sqrt(dh); returns
+    c[j] = sum_g sum_{i in [q_lo, n), i >= j} A_g[i, j] for j < n.
+    k: [>= n, Hkv, dh]."""
+    k = f64(k)
+    hkv, dh = k.shape[1], k.shape[2]
+    c = np.zeros(n)
+    for g in range(hkv):
+        for i in range(q_lo, n):
+            s = k[:i + 1, g] @ k[i, g] / np.sqrt(dh)
+            c[:i + 1] += softmax(s)
+    return c
+
+
+def importance_scores(shape, cache):
+    """Importance (Sec. 4, after TOVA): the mean attention a token receives in
+    the last layer, with the layer's cached keys as proxy queries and the
+    causal mask: score_j = c[j] / (Hkv * (n - j)), c from
+    key_attention_colsums over every query slot (the n - j queries that see
+    slot j, in each KV head).  Low mean attention is evicted first."""
+    seq_len = np.asarray(cache["seq_len"])
+    kl = cache["k"][shape.n_layers - 1]
+    bsz, cap = kl.shape[0], kl.shape[1]
+    out = np.full((bsz, cap), NEG_INF)
+    for b in range(bsz):
+        n = int(seq_len[b])
+        if n == 0:
+            continue
+        c = key_attention_colsums(kl[b], n, 0)
+        out[b, :n] = c / (shape.n_kv_heads * (n - np.arange(n)))
+    return out
+
+
+def h2o_update(shape, cache, acc, recent):
+    """Heavy-hitter (H2O, Sec. 4): adds to the running total acc [B, cap] the
+    attention each slot receives from the `recent` most recent keys as proxy
+    queries (causal mask), summed over KV heads and every layer."""
+    seq_len = np.asarray(cache["seq_len"])
+    for b in range(acc.shape[0]):
+        n = int(seq_len[b])
+        q_lo = max(0, n - int(recent))
+        for l in range(shape.n_layers):
+            acc[b, :n] += key_attention_colsums(cache["k"][l][b], n, q_lo)
+    return acc
+
+
+def h2o_scores(acc, seq_len, recent):
+    """Refresh scores of H2O: the accumulated attention, with the `recent`
+    most recent slots always kept (+inf); only older slots are evicted."""
+    out = np.full(np.shape(acc), NEG_INF)
+    for b in range(out.shape[0]):
+        n = int(seq_len[b])
+        out[b, :n] = acc[b, :n]
+        out[b, max(0, n - int(recent)):n] = POS_INF
+    return out
