@@ -209,6 +209,17 @@ def algorithmic_work(wl):
     }
 
 
+def keyattn_work(wl, scorer, recent):
+    """FLOPs of one keyattn launch pair (both sweeps: S = K K^T over the
+    causal (query, key) pairs of the proxy queries, 2 dh per pair and head)."""
+    s = wl.shape
+    pairs = 0
+    for n in wl.seq_lens:
+        q_lo = 0 if scorer == "importance" else max(0, n - recent)
+        pairs += sum(i + 1 for i in range(q_lo, n))
+    return ("tensor", 2 * 2.0 * s.head_dim * s.n_kv_heads * pairs)
+
+
 def step_flops(wl):
     s = wl.shape
     w = algorithmic_work(wl)
@@ -248,9 +259,27 @@ def run_ours(args, dist):
     flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
     score_fn = cc.cc_score_layer if fast else cc.cc_score_full
     stream = torch.cuda.current_stream(dev)
+    scorer, recent = args.scorer, args.recent
+    if scorer in ("importance", "h2o"):
+        kws = cc.alloc_workspace(cc.cc_keyattn_workspace_size(shape, b, cap), dev)
+    if scorer == "h2o":   # running totals, compacted with the cache
+        work["h2o_acc"] = torch.zeros(b, cap, dtype=torch.float32, device=dev)
+        cache = pkg.Cache(work)
+        cws = cc.alloc_workspace(cc.cc_compact_workspace_size(shape, cache), dev)
+
+    def score():
+        if scorer == "counter-causal":
+            score_fn(shape, weights, cache, mode, scores, ws)
+        elif scorer == "recency":
+            cc.cc_score_recency(cache, scores)
+        elif scorer == "importance":
+            cc.cc_score_importance(shape, cache, scores, kws)
+        else:
+            cc.cc_h2o_accumulate(shape, cache, recent, kws)
+            cc.cc_score_h2o(cache, recent, scores)
 
     def step():
-        score_fn(shape, weights, cache, mode, scores, ws)
+        score()
         cc.cc_select_keep(scores, cache.d["seq_len"], b, cap, budget, wl.n_sink, keep_idx,
                           keep_count)
         cc.cc_compact_kv(shape, cache, keep_idx, keep_count, cws)
@@ -356,6 +385,8 @@ def run_ours(args, dist):
     # ---- roofline of the dominant kernel (and a per-kernel table)
     peaks, peak_src = load_peaks()
     work_tbl = algorithmic_work(wl)
+    if scorer in ("importance", "h2o"):
+        work_tbl["keyattn"] = keyattn_work(wl, scorer, recent)
     table = {}
     for name, (cnt, tot) in kernels.items():
         per = tot / cnt
@@ -385,14 +416,19 @@ def run_ours(args, dist):
     launches = sum(c for c, _ in kernels.values())
     value = positions * dist.world / (ms * 1e-3)
     # the paper's own figure for this workload (Table 1, another GPU): context only
-    vs_baseline = round(value / wl.paper_positions_per_s, 2) if wl.paper_positions_per_s else None
+    vs_baseline = (round(value / wl.paper_positions_per_s, 2)
+                   if wl.paper_positions_per_s and scorer == "counter-causal" else None)
     line = {
         "metric": "scored KV positions/sec per refresh",
         "value": round(value, 1), "unit": "positions/s", "n_gpus": dist.world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 4),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": vs_baseline, "dtype": "bf16",
         "data": "synthetic (seeded random-init weights N(0,0.02); synthetic KV cache)",
-        "config": {"workload": wl.name, "pass": "fast single-layer" if fast else f"full {shape.n_layers}-layer",
+        "config": {"workload": wl.name, "scorer": scorer,
+                   "pass": ("fast single-layer" if fast else f"full {shape.n_layers}-layer")
+                   if scorer == "counter-causal" else
+                   {"recency": "position", "importance": "last-layer key attention",
+                    "h2o": f"all-layer key attention, {recent} recent proxy queries"}[scorer],
                    "score": args.score, "batch": wl.batch, "seq_lens": wl.seq_lens,
                    "budgets": wl.budgets, "cap": wl.cap, "d_model": shape.d_model,
                    "heads": f"{shape.n_q_heads}/{shape.n_kv_heads}x{shape.head_dim}",
@@ -410,10 +446,10 @@ def run_ours(args, dist):
         "tflops_per_step_achieved": round(step_flops(wl) / (ms * 1e-3) / 1e12, 1),
         "clocks": clk,
     }
-    if wl.paper_positions_per_s:
+    if wl.paper_positions_per_s and scorer == "counter-causal":
         line["paper"] = {"value": round(wl.paper_positions_per_s, 1), "unit": "positions/s",
                          "source": "Table 1: n / refresh latency, Qwen2.5-7B, RTX 4090, fp16"}
-    if dist.world == 1 and not args.no_cpu_baseline:
+    if dist.world == 1 and not args.no_cpu_baseline and scorer == "counter-causal":
         line["cpu_baseline"] = cpu_baseline(wl, w, pristine, scores, args.cpu_rows, args.score)
     return line
 
@@ -774,6 +810,12 @@ def main():
     ap.add_argument("--cpu-rows", type=int, default=256)
     ap.add_argument("--ref-rows", type=int, default=32)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--scorer", choices=["counter-causal", "recency", "importance", "h2o"],
+                    default="counter-causal",
+                    help="refresh scorer: the paper's (default) or one of its comparison "
+                         "scorers (Sec. 4) on the same select/compact path")
+    ap.add_argument("--recent", type=int, default=256,
+                    help="h2o: proxy-query slots (the most recent) per refresh")
     ap.add_argument("--append", action="store_true",
                     help="time the inference cycle: the workload's append chunk over its "
                          "budget-sized memory (cc_append_chunk, every layer)")

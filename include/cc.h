@@ -132,6 +132,9 @@ typedef struct {
   void *h_last;      /* device bf16 [batch][cap][d_model]: H^(L-1), the input of the
                         last layer recorded by the causal pass (fast mode); may be NULL
                         for cc_score_full                                               */
+  float *h2o_acc;    /* optional device fp32 [batch][cap]: running totals of the H2O
+                        comparison scorer (cc_h2o_accumulate), compacted with the cache;
+                        NULL when unused                                                */
 } cc_kv_cache;
 
 /* ---- scoring (Sec. 3.1) ---------------------------------------------------
@@ -210,6 +213,34 @@ cc_status cc_append_chunk(const cc_model_cfg *cfg, const cc_model_weights *w,
                           const cc_kv_cache *cache, const int32_t *tokens_in,
                           const int32_t *pos_in, const int32_t *count, int32_t max_count,
                           void *ws, size_t ws_bytes, void *stream);
+
+/* ---- the paper's comparison scorers (Sec. 4) -------------------------------
+ * They rank the same cached slots for the same cc_select_keep and
+ * cc_compact_kv; the attention-based ones read only the cached keys, which
+ * act as proxy queries (query slot i attends slots j <= i, softmax of
+ * K[i] . K[j] / sqrt(head_dim) per KV head).  scores: device fp32
+ * [batch][cap], -inf past seq_len.
+ *
+ * cc_score_recency -- sliding window (first in, first out): score = the
+ *   slot's original position, so the keep-set is the most recent slots.
+ * cc_score_importance -- importance: mean attention a slot receives in the
+ *   last layer, over the KV heads and the n - j proxy queries that see it.
+ * cc_h2o_accumulate -- heavy hitter (H2O): adds to cache->h2o_acc the
+ *   attention each slot receives from the `recent` most recent keys as proxy
+ *   queries, summed over KV heads and every layer (a running total across
+ *   refreshes; zero it once when the cache starts).
+ * cc_score_h2o -- H2O refresh scores: h2o_acc, with the `recent` most recent
+ *   slots always kept (+inf).
+ * The attention-based scorers need head_dim 64 or 128 and the workspace of
+ * cc_keyattn_workspace_size; results are deterministic (fixed summation
+ * order). */
+cc_status cc_score_recency(const cc_kv_cache *cache, float *scores, void *stream);
+size_t cc_keyattn_workspace_size(const cc_model_cfg *cfg, int32_t batch, int32_t cap);
+cc_status cc_score_importance(const cc_model_cfg *cfg, const cc_kv_cache *cache, float *scores,
+                              void *ws, size_t ws_bytes, void *stream);
+cc_status cc_h2o_accumulate(const cc_model_cfg *cfg, const cc_kv_cache *cache, int32_t recent,
+                            void *ws, size_t ws_bytes, void *stream);
+cc_status cc_score_h2o(const cc_kv_cache *cache, int32_t recent, float *scores, void *stream);
 
 /* ---- compaction without a workspace -----------------------------------------
  * The paper has no counterpart: this is a library convenience.

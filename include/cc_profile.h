@@ -34,7 +34,8 @@ typedef enum {
   CC_KERNEL_ATTN_CAUSAL = 14,/* memory-augmented causal attention (append)        */
   CC_KERNEL_APPEND = 15,     /* append bookkeeping: tokens, positions, H^(L-1)    */
   CC_KERNEL_GEMM_QKV = 16,   /* fused q/k/v projections (+ RoPE) of the append    */
-  CC_KERNEL_COUNT = 17
+  CC_KERNEL_KEYATTN = 17,    /* comparison scorers: attention received per key    */
+  CC_KERNEL_COUNT = 18
 } cc_kernel_kind;
 
 /* on != 0: start recording (also clears earlier records); 0: stop. */

@@ -60,7 +60,8 @@ class cc_kv_cache(ctypes.Structure):
     _fields_ = [("batch", ctypes.c_int32), ("cap", ctypes.c_int32),
                 ("seq_len", ctypes.c_void_p), ("k", ctypes.POINTER(ctypes.c_void_p)),
                 ("v", ctypes.POINTER(ctypes.c_void_p)), ("tokens", ctypes.c_void_p),
-                ("pos", ctypes.c_void_p), ("h_last", ctypes.c_void_p)]
+                ("pos", ctypes.c_void_p), ("h_last", ctypes.c_void_p),
+                ("h2o_acc", ctypes.c_void_p)]
 
 
 _LIB = None
@@ -79,6 +80,18 @@ _SIGS = {
                                        ctypes.POINTER(cc_kv_cache), ctypes.c_void_p, ctypes.c_void_p,
                                        ctypes.c_void_p, ctypes.c_int32, ctypes.c_void_p,
                                        ctypes.c_size_t, ctypes.c_void_p]),
+    "cc_score_recency": (ctypes.c_int, [ctypes.POINTER(cc_kv_cache), ctypes.c_void_p,
+                                        ctypes.c_void_p]),
+    "cc_keyattn_workspace_size": (ctypes.c_size_t, [ctypes.POINTER(cc_model_cfg), ctypes.c_int32,
+                                                    ctypes.c_int32]),
+    "cc_score_importance": (ctypes.c_int, [ctypes.POINTER(cc_model_cfg), ctypes.POINTER(cc_kv_cache),
+                                           ctypes.c_void_p, ctypes.c_void_p, ctypes.c_size_t,
+                                           ctypes.c_void_p]),
+    "cc_h2o_accumulate": (ctypes.c_int, [ctypes.POINTER(cc_model_cfg), ctypes.POINTER(cc_kv_cache),
+                                         ctypes.c_int32, ctypes.c_void_p, ctypes.c_size_t,
+                                         ctypes.c_void_p]),
+    "cc_score_h2o": (ctypes.c_int, [ctypes.POINTER(cc_kv_cache), ctypes.c_int32, ctypes.c_void_p,
+                                    ctypes.c_void_p]),
     "cc_select_workspace_size": (ctypes.c_size_t, [ctypes.c_int32, ctypes.c_int32]),
     "cc_select_keep": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int32,
                                       ctypes.c_int32, ctypes.c_void_p, ctypes.c_int32,
@@ -106,7 +119,7 @@ _SIGS = {
     "cc_kernel_name": (ctypes.c_char_p, [ctypes.c_int32]),
     "cc_debug_withhold_compact_unit": (ctypes.c_int, [ctypes.c_int32]),
 }
-KERNEL_COUNT = 17
+KERNEL_COUNT = 18
 
 
 def library_path() -> str:
@@ -206,7 +219,8 @@ class Cache:
         self._v = (ctypes.c_void_p * len(vs))(*[_dev_ptr(x, "v") for x in vs])
         self.c = cc_kv_cache(b, cap, _dev_ptr(c["seq_len"], "seq_len"), self._k, self._v,
                              _dev_ptr(c["tokens"], "tokens"), _dev_ptr(c["pos"], "pos"),
-                             _dev_ptr(c.get("h_last"), "h_last"))
+                             _dev_ptr(c.get("h_last"), "h_last"),
+                             _dev_ptr(c.get("h2o_acc"), "h2o_acc"))
 
 
 def _cfg(cfg):
@@ -260,6 +274,36 @@ def cc_append_chunk(cfg, weights, cache, tokens_in, pos_in, count, max_count: in
         _dev_ptr(tokens_in, "tokens_in"), _dev_ptr(pos_in, "pos_in"), _dev_ptr(count, "count"),
         int(max_count), _dev_ptr(ws, "ws"), ws.numel() * ws.element_size(), _stream(stream))
     _check(code, "cc_append_chunk")
+
+
+# ---- the paper's comparison scorers (Sec. 4) ---------------------------------
+
+def cc_score_recency(cache, scores, stream=None):
+    _check(load_library().cc_score_recency(ctypes.byref(cache.c), _dev_ptr(scores, "scores"),
+                                           _stream(stream)), "cc_score_recency")
+
+
+def cc_keyattn_workspace_size(cfg, batch: int, cap: int) -> int:
+    return int(load_library().cc_keyattn_workspace_size(ctypes.byref(_cfg(cfg)), batch, cap))
+
+
+def cc_score_importance(cfg, cache, scores, ws, stream=None):
+    _check(load_library().cc_score_importance(
+        ctypes.byref(_cfg(cfg)), ctypes.byref(cache.c), _dev_ptr(scores, "scores"),
+        _dev_ptr(ws, "ws"), ws.numel() * ws.element_size(), _stream(stream)),
+        "cc_score_importance")
+
+
+def cc_h2o_accumulate(cfg, cache, recent: int, ws, stream=None):
+    _check(load_library().cc_h2o_accumulate(
+        ctypes.byref(_cfg(cfg)), ctypes.byref(cache.c), int(recent), _dev_ptr(ws, "ws"),
+        ws.numel() * ws.element_size(), _stream(stream)), "cc_h2o_accumulate")
+
+
+def cc_score_h2o(cache, recent: int, scores, stream=None):
+    _check(load_library().cc_score_h2o(ctypes.byref(cache.c), int(recent),
+                                       _dev_ptr(scores, "scores"), _stream(stream)),
+           "cc_score_h2o")
 
 
 def cc_select_workspace_size(batch: int, cap: int) -> int:

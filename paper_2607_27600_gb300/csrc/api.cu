@@ -20,6 +20,7 @@
 #include "attn.cuh"
 #include "compact.cuh"
 #include "gemm.cuh"
+#include "keyattn.cuh"
 #include "rowops.cuh"
 #include "select.cuh"
 #include "../../include/cc_kernels.h"
@@ -778,6 +779,7 @@ cc_status compact_plan(const cc_model_cfg *c, const cc_kv_cache *kv, CompactPlan
   }
   if (!add(kv->h_last, c->d_model * 2, true)) return CC_ERR_UNSUPPORTED;
   if (!add(kv->tokens, 4, false) || !add(kv->pos, 4, false)) return CC_ERR_INVALID_ARG;
+  if (!add(kv->h2o_acc, 4, false)) return CC_ERR_INVALID_ARG;   // comparison scorer totals
   p.n_arrays = n;
   p.total_units = units;
   if (n < 2 || units < 2) return CC_ERR_INVALID_ARG;   // tokens and pos are always compacted
@@ -810,6 +812,98 @@ cc_status compact_bind(CompactPlan &plan, void *ws, cudaStream_t st) {
 // C ABI
 // ===========================================================================
 extern "C" {
+
+// ---- the paper's comparison scorers (Sec. 4) ---------------------------------
+cc_status cc_score_recency(const cc_kv_cache *kv, float *scores, void *stream) {
+  if (!kv || !scores || !kv->pos || !kv->seq_len || kv->batch < 1 || kv->cap < 1)
+    return CC_ERR_INVALID_ARG;
+  CC_TRY(launch_recency_scores(kv->pos, kv->seq_len, kv->batch, kv->cap, scores,
+                               reinterpret_cast<cudaStream_t>(stream)));
+  return CC_OK;
+}
+
+size_t cc_keyattn_workspace_size(const cc_model_cfg *cfg, int32_t batch, int32_t cap) {
+  if (check_cfg(cfg) != CC_OK || batch < 1 || cap < 1) return 0;
+  const size_t ld = ((size_t)cap + 127) / 128 * 128;
+  return 2 * (size_t)batch * cfg->n_kv_heads * ld * 4;   // lse2 and per-head sums
+}
+
+// One layer's sweeps; out = finish(part) (mean: importance; accumulate: H2O).
+cc_status run_keyattn(const cc_model_cfg *c, const cc_kv_cache *kv, int layer, int recent,
+                      float *out, bool mean, bool accumulate, void *ws, cudaStream_t st,
+                      unsigned *status) {
+  const int batch = kv->batch, cap = kv->cap, dh = c->head_dim;
+  const uint64_t R = (uint64_t)batch * cap;
+  CUtensorMap tk;
+  const uint64_t dims[3] = {(uint64_t)dh, (uint64_t)c->n_kv_heads, R};
+  const uint64_t strides[2] = {(uint64_t)dh * 2, (uint64_t)c->n_kv_heads * dh * 2};
+  const uint32_t box[3] = {64, 1, 128};
+  if (!make_tmap(&tk, kv->k[layer], 3, dims, strides, box)) return tmap_fail();
+  KeyAttnParams p{};
+  p.batch = batch;
+  p.cap = cap;
+  p.n_kv_heads = c->n_kv_heads;
+  p.head_dim = dh;
+  p.seq_len = kv->seq_len;
+  p.q_lo = nullptr;
+  p.recent = recent;
+  p.q_span = recent > 0 ? std::min(recent, cap) : cap;
+  p.ld = (cap + 127) / 128 * 128;
+  p.lse = reinterpret_cast<float *>(ws);
+  p.part = p.lse + (size_t)batch * c->n_kv_heads * p.ld;
+  p.scale_log2 = (float)(1.4426950408889634 / sqrt((double)dh));
+  p.status = status;
+  TimedScope t(CC_KERNEL_KEYATTN, st);
+  CC_TRY(launch_keyattn(tk, p, st));
+  CC_TRY(launch_keyattn_finish(p, out, mean, accumulate, st));
+  return CC_OK;
+}
+
+cc_status check_keyattn_args(const cc_model_cfg *c, const cc_kv_cache *kv, void *ws,
+                             size_t ws_bytes, int l0) {
+  cc_status s = check_cfg(c);
+  if (s != CC_OK) return s;
+  if (!kv || !kv->k || !kv->seq_len || kv->batch < 1 || kv->cap < 1) return CC_ERR_INVALID_ARG;
+  if ((uint64_t)kv->batch * kv->cap >= (1ull << 31)) return CC_ERR_UNSUPPORTED;
+  for (int l = l0; l < c->n_layers; ++l)
+    if (!kv->k[l] || !aligned16(kv->k[l])) return CC_ERR_INVALID_ARG;
+  if (!ws || !aligned16(ws) || ws_bytes < cc_keyattn_workspace_size(c, kv->batch, kv->cap))
+    return CC_ERR_WORKSPACE;
+  return CC_OK;
+}
+
+cc_status cc_score_importance(const cc_model_cfg *cfg, const cc_kv_cache *kv, float *scores,
+                              void *ws, size_t ws_bytes, void *stream) {
+  cc_status s = check_keyattn_args(cfg, kv, ws, ws_bytes, cfg ? cfg->n_layers - 1 : 0);
+  if (s != CC_OK) return s;
+  if (!scores) return CC_ERR_INVALID_ARG;
+  DevState *dev;
+  if (!dev_state(&dev)) return device_fail();
+  return run_keyattn(cfg, kv, cfg->n_layers - 1, 0, scores, true, false, ws,
+                     reinterpret_cast<cudaStream_t>(stream), dev->status);
+}
+
+cc_status cc_h2o_accumulate(const cc_model_cfg *cfg, const cc_kv_cache *kv, int32_t recent,
+                            void *ws, size_t ws_bytes, void *stream) {
+  cc_status s = check_keyattn_args(cfg, kv, ws, ws_bytes, 0);
+  if (s != CC_OK) return s;
+  if (!kv->h2o_acc || recent < 1) return CC_ERR_INVALID_ARG;
+  DevState *dev;
+  if (!dev_state(&dev)) return device_fail();
+  for (int l = 0; l < cfg->n_layers; ++l)
+    if ((s = run_keyattn(cfg, kv, l, recent, kv->h2o_acc, false, true, ws,
+                         reinterpret_cast<cudaStream_t>(stream), dev->status)) != CC_OK)
+      return s;
+  return CC_OK;
+}
+
+cc_status cc_score_h2o(const cc_kv_cache *kv, int32_t recent, float *scores, void *stream) {
+  if (!kv || !scores || !kv->h2o_acc || !kv->seq_len || kv->batch < 1 || kv->cap < 1 || recent < 0)
+    return CC_ERR_INVALID_ARG;
+  CC_TRY(launch_h2o_scores(kv->h2o_acc, kv->seq_len, kv->batch, kv->cap, recent, scores,
+                           reinterpret_cast<cudaStream_t>(stream)));
+  return CC_OK;
+}
 
 size_t cc_append_workspace_size(const cc_model_cfg *cfg, int32_t batch, int32_t cap) {
   if (check_cfg(cfg) != CC_OK || batch < 1 || cap < 1) return 0;
@@ -1006,7 +1100,7 @@ const char *cc_kernel_name(int32_t kind) {
   static const char *names[CC_KERNEL_COUNT] = {
       "rmsnorm", "embed", "gemm_qrope", "attention", "gemm_oproj", "gemm_gateup", "gemm_down",
       "head_logit", "gemm_lmhead", "lse_combine", "select", "compact", "other",
-      "gemm_kv", "attention_causal", "append", "gemm_qkv"};
+      "gemm_kv", "attention_causal", "append", "gemm_qkv", "keyattn"};
   return (kind >= 0 && kind < CC_KERNEL_COUNT) ? names[kind] : "unknown";
 }
 
