@@ -211,13 +211,15 @@ def algorithmic_work(wl):
 
 def keyattn_work(wl, scorer, recent):
     """FLOPs of one keyattn launch pair (both sweeps: S = K K^T over the
-    causal (query, key) pairs of the proxy queries, 2 dh per pair and head)."""
+    causal (query, key) pairs of the proxy queries, 2 dh per pair and head,
+    for the last layer (importance) or every layer (H2O))."""
     s = wl.shape
     pairs = 0
     for n in wl.seq_lens:
         q_lo = 0 if scorer == "importance" else max(0, n - recent)
         pairs += sum(i + 1 for i in range(q_lo, n))
-    return ("tensor", 2 * 2.0 * s.head_dim * s.n_kv_heads * pairs)
+    layers = 1 if scorer == "importance" else s.n_layers   # H2O: every layer in one launch
+    return ("tensor", 2 * 2.0 * s.head_dim * s.n_kv_heads * pairs * layers)
 
 
 def step_flops(wl):

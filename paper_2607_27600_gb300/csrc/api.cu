@@ -824,22 +824,29 @@ cc_status cc_score_recency(const cc_kv_cache *kv, float *scores, void *stream) {
 
 size_t cc_keyattn_workspace_size(const cc_model_cfg *cfg, int32_t batch, int32_t cap) {
   if (check_cfg(cfg) != CC_OK || batch < 1 || cap < 1) return 0;
+  if (cfg->n_layers > kKeyAttnMaxLayers) return 0;
   const size_t ld = ((size_t)cap + 127) / 128 * 128;
-  return 2 * (size_t)batch * cfg->n_kv_heads * ld * 4;   // lse2 and per-head sums
+  // lse2 and per-head sums of every layer (H2O runs all layers in one launch)
+  return 2 * (size_t)cfg->n_layers * batch * cfg->n_kv_heads * ld * 4;
 }
 
-// One layer's sweeps; out = finish(part) (mean: importance; accumulate: H2O).
-cc_status run_keyattn(const cc_model_cfg *c, const cc_kv_cache *kv, int layer, int recent,
+// Sweeps over layers [l0, l1) in one launch each; out = finish(part)
+// (mean: importance; accumulate: H2O).
+cc_status run_keyattn(const cc_model_cfg *c, const cc_kv_cache *kv, int l0, int l1, int recent,
                       float *out, bool mean, bool accumulate, void *ws, cudaStream_t st,
                       unsigned *status) {
   const int batch = kv->batch, cap = kv->cap, dh = c->head_dim;
   const uint64_t R = (uint64_t)batch * cap;
-  CUtensorMap tk;
+  static KeyAttnBatch a;   // ~8 KB: kept off the stack; guarded below
+  static std::mutex mu;
+  std::lock_guard<std::mutex> lk(mu);
+  memset(&a, 0, sizeof(a));
   const uint64_t dims[3] = {(uint64_t)dh, (uint64_t)c->n_kv_heads, R};
   const uint64_t strides[2] = {(uint64_t)dh * 2, (uint64_t)c->n_kv_heads * dh * 2};
   const uint32_t box[3] = {64, 1, 128};
-  if (!make_tmap(&tk, kv->k[layer], 3, dims, strides, box)) return tmap_fail();
-  KeyAttnParams p{};
+  for (int l = l0; l < l1; ++l)
+    if (!make_tmap(&a.k[l - l0], kv->k[l], 3, dims, strides, box)) return tmap_fail();
+  KeyAttnParams &p = a.p;
   p.batch = batch;
   p.cap = cap;
   p.n_kv_heads = c->n_kv_heads;
@@ -848,13 +855,14 @@ cc_status run_keyattn(const cc_model_cfg *c, const cc_kv_cache *kv, int layer, i
   p.q_lo = nullptr;
   p.recent = recent;
   p.q_span = recent > 0 ? std::min(recent, cap) : cap;
+  p.n_layers = l1 - l0;
   p.ld = (cap + 127) / 128 * 128;
   p.lse = reinterpret_cast<float *>(ws);
-  p.part = p.lse + (size_t)batch * c->n_kv_heads * p.ld;
+  p.part = p.lse + (size_t)p.n_layers * batch * c->n_kv_heads * p.ld;
   p.scale_log2 = (float)(1.4426950408889634 / sqrt((double)dh));
   p.status = status;
   TimedScope t(CC_KERNEL_KEYATTN, st);
-  CC_TRY(launch_keyattn(tk, p, st));
+  CC_TRY(launch_keyattn(a, st));
   CC_TRY(launch_keyattn_finish(p, out, mean, accumulate, st));
   return CC_OK;
 }
@@ -865,6 +873,7 @@ cc_status check_keyattn_args(const cc_model_cfg *c, const cc_kv_cache *kv, void 
   if (s != CC_OK) return s;
   if (!kv || !kv->k || !kv->seq_len || kv->batch < 1 || kv->cap < 1) return CC_ERR_INVALID_ARG;
   if ((uint64_t)kv->batch * kv->cap >= (1ull << 31)) return CC_ERR_UNSUPPORTED;
+  if (c->n_layers > kKeyAttnMaxLayers) return CC_ERR_UNSUPPORTED;
   for (int l = l0; l < c->n_layers; ++l)
     if (!kv->k[l] || !aligned16(kv->k[l])) return CC_ERR_INVALID_ARG;
   if (!ws || !aligned16(ws) || ws_bytes < cc_keyattn_workspace_size(c, kv->batch, kv->cap))
@@ -879,7 +888,7 @@ cc_status cc_score_importance(const cc_model_cfg *cfg, const cc_kv_cache *kv, fl
   if (!scores) return CC_ERR_INVALID_ARG;
   DevState *dev;
   if (!dev_state(&dev)) return device_fail();
-  return run_keyattn(cfg, kv, cfg->n_layers - 1, 0, scores, true, false, ws,
+  return run_keyattn(cfg, kv, cfg->n_layers - 1, cfg->n_layers, 0, scores, true, false, ws,
                      reinterpret_cast<cudaStream_t>(stream), dev->status);
 }
 
@@ -890,11 +899,8 @@ cc_status cc_h2o_accumulate(const cc_model_cfg *cfg, const cc_kv_cache *kv, int3
   if (!kv->h2o_acc || recent < 1) return CC_ERR_INVALID_ARG;
   DevState *dev;
   if (!dev_state(&dev)) return device_fail();
-  for (int l = 0; l < cfg->n_layers; ++l)
-    if ((s = run_keyattn(cfg, kv, l, recent, kv->h2o_acc, false, true, ws,
-                         reinterpret_cast<cudaStream_t>(stream), dev->status)) != CC_OK)
-      return s;
-  return CC_OK;
+  return run_keyattn(cfg, kv, 0, cfg->n_layers, recent, kv->h2o_acc, false, true, ws,
+                     reinterpret_cast<cudaStream_t>(stream), dev->status);
 }
 
 cc_status cc_score_h2o(const cc_kv_cache *kv, int32_t recent, float *scores, void *stream) {

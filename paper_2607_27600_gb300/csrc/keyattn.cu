@@ -49,8 +49,9 @@ CC_DEV float ex2(float x) {
 
 template <int DH, int SWEEP>
 __global__ void __launch_bounds__(kThreads)
-    keyattn_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ KeyAttnParams p) {
+    keyattn_kernel(const __grid_constant__ KeyAttnBatch batch_args) {
   using L = KaSmem<DH>;
+  const KeyAttnParams &p = batch_args.p;
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                               ~uintptr_t(1023));
@@ -69,13 +70,15 @@ __global__ void __launch_bounds__(kThreads)
   const int blk = blockIdx.x % per_seq;
   const int bg = blockIdx.x / per_seq;
   const int g = bg % p.n_kv_heads, b = bg / p.n_kv_heads;
+  const int layer = blockIdx.y;
+  const CUtensorMap &tmK = batch_args.k[layer];
   const int n = p.seq_len[b];
   int q_lo = p.q_lo ? p.q_lo[b] : (p.recent > 0 ? max(0, n - p.recent) : 0);
   if (n < 0 || n > p.cap || q_lo < 0 || q_lo > n) {
     if (threadIdx.x == 0) set_status(p.status, CC_ERR_DEVICE_ARG);
     return;
   }
-  const size_t head_off = ((size_t)b * p.n_kv_heads + g) * p.ld;
+  const size_t head_off = (((size_t)layer * p.batch + b) * p.n_kv_heads + g) * p.ld;
   int row0, t_first, t_last;
   if (SWEEP == 0) {   // rows: proxy queries; keys 0 .. the block's last query
     row0 = q_lo + blk * KT;
@@ -233,7 +236,7 @@ __global__ void __launch_bounds__(kThreads)
 }
 
 // out[b][j] = (accumulate ? out : 0) + sum_g part[b][g][j] (/ Hkv (n - j) when mean)
-__global__ void keyattn_finish_kernel(const __grid_constant__ KeyAttnParams p, float *out, int mean,
+__global__ void keyattn_finish_kernel(const KeyAttnParams p, float *out, int mean,
                                       int accumulate) {
   const int b = blockIdx.y;
   const int j = blockIdx.x * blockDim.x + threadIdx.x;
@@ -245,7 +248,9 @@ __global__ void keyattn_finish_kernel(const __grid_constant__ KeyAttnParams p, f
     return;
   }
   float s = 0.f;
-  for (int g = 0; g < p.n_kv_heads; ++g) s += p.part[((size_t)b * p.n_kv_heads + g) * p.ld + j];
+  for (int l = 0; l < p.n_layers; ++l)
+    for (int g = 0; g < p.n_kv_heads; ++g)
+      s += p.part[(((size_t)l * p.batch + b) * p.n_kv_heads + g) * p.ld + j];
   if (mean) s /= (float)p.n_kv_heads * (float)(n - j);
   *o = accumulate ? *o + s : s;
 }
@@ -275,7 +280,8 @@ __global__ void h2o_scores_kernel(const float *acc, const int32_t *seq_len, int 
 }
 
 template <int DH>
-cudaError_t launch_dh(const CUtensorMap &k, const KeyAttnParams &p, cudaStream_t st) {
+cudaError_t launch_dh(const KeyAttnBatch &a, cudaStream_t st) {
+  const KeyAttnParams &p = a.p;
   static bool attr_set[64] = {};
   int dev = 0;
   cudaGetDevice(&dev);
@@ -291,18 +297,21 @@ cudaError_t launch_dh(const CUtensorMap &k, const KeyAttnParams &p, cudaStream_t
   const long long heads = (long long)p.batch * p.n_kv_heads;
   const long long u0 = heads * ((p.q_span + KT - 1) / KT);
   const long long u1 = heads * ((p.cap + KT - 1) / KT);
-  if (u0 > 0) keyattn_kernel<DH, 0><<<(unsigned)u0, kThreads, KaSmem<DH>::BYTES, st>>>(k, p);
+  if (p.n_layers < 1 || p.n_layers > kKeyAttnMaxLayers) return cudaErrorInvalidValue;
+  if (u0 > 0)
+    keyattn_kernel<DH, 0><<<dim3((unsigned)u0, p.n_layers), kThreads, KaSmem<DH>::BYTES, st>>>(a);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  if (u1 > 0) keyattn_kernel<DH, 1><<<(unsigned)u1, kThreads, KaSmem<DH>::BYTES, st>>>(k, p);
+  if (u1 > 0)
+    keyattn_kernel<DH, 1><<<dim3((unsigned)u1, p.n_layers), kThreads, KaSmem<DH>::BYTES, st>>>(a);
   return cudaGetLastError();
 }
 
 }  // namespace
 
-cudaError_t launch_keyattn(const CUtensorMap &k, const KeyAttnParams &p, cudaStream_t st) {
-  if (p.head_dim == 128) return launch_dh<128>(k, p, st);
-  if (p.head_dim == 64) return launch_dh<64>(k, p, st);
+cudaError_t launch_keyattn(const KeyAttnBatch &a, cudaStream_t st) {
+  if (a.p.head_dim == 128) return launch_dh<128>(a, st);
+  if (a.p.head_dim == 64) return launch_dh<64>(a, st);
   return cudaErrorInvalidValue;
 }
 
