@@ -265,9 +265,21 @@ cc_status gemm_setup(Gemm &g, int epi, const void *A, int K, const void *W, cons
                      int batch, int cap, const int32_t *seq_len, unsigned *status,
                      bool a_split = false, uint64_t rows_hint = 0) {
   const uint64_t R = (uint64_t)batch * cap;
-  const int bn = gemm_block_n(epi);
+  const uint64_t R_est = rows_hint ? rows_hint : R;
+  int bn = gemm_block_n(epi);
+  // narrow problems (less than one wave of 256-column tiles): 128-column
+  // tiles double the tiles that share the SMs
+  // (a residual GEMM long enough for two K splits keeps wide tiles and splits
+  // K instead: plan_k_splits, measured faster for the down projection)
+  const int nk_total = ((K + 63) / 64) * (a_split ? 2 : 1);
+  const bool narrowable = epi == EPI_F32 || epi == EPI_QROPE || epi == EPI_RESID_BF16 ||
+                          (epi == EPI_RESID_F32 && nk_total < 128) || epi == EPI_BF16;
+  DevState *dev_info = nullptr;
+  if (narrowable && dev_state(&dev_info) &&
+      ((R_est + 127) / 128) * (uint64_t)((N + 255) / 256) < (uint64_t)dev_info->sms)
+    bn = 128;
   if (!tmap_rows(&g.a, A, R, a_split ? 2 * K : K, 128)) return tmap_fail();
-  if (!tmap_rows(&g.b, W, N, K, epi == EPI_SWIGLU ? 128 : 256)) return tmap_fail();
+  if (!tmap_rows(&g.b, W, N, K, epi == EPI_SWIGLU ? 128 : bn)) return tmap_fail();
   if (epi == EPI_SWIGLU) {
     if (!tmap_rows(&g.b2, W2, N, K, 128)) return tmap_fail();
   } else {
@@ -280,6 +292,7 @@ cc_status gemm_setup(Gemm &g, int epi, const void *A, int K, const void *W, cons
   g.p.seq_len = seq_len;
   g.p.N = N;
   g.p.K = K;
+  g.p.block_n = epi == EPI_SWIGLU ? 256 : bn;
   g.p.n_tiles = (N + bn - 1) / bn;
   g.p.status = status;
   g.p.a_split = a_split ? 1 : 0;
@@ -293,12 +306,13 @@ cc_status gemm_setup(Gemm &g, int epi, const void *A, int K, const void *W, cons
   // 16 %.  The activation-resident order is taken only when that count is
   // below 0.8x (an LM head whose weight is far larger than L2).
   const double budget = 40.0 * (1 << 20);
-  const uint64_t R_used = rows_hint ? rows_hint : R;
+  const uint64_t R_used = R_est;
   g.rows_est = R_used;
   const int num_m = (int)((R_used + 127) / 128), num_n = g.p.n_tiles;
   const double k_a = (a_split ? 2.0 : 1.0) * K;
-  const double a_bytes = (double)R_used * k_a * 2, b_bytes = (double)num_n * 256 * K * 2;
-  const double a_slab = 128.0 * k_a * 2, b_slab = 256.0 * K * 2;
+  const int b_rows = epi == EPI_SWIGLU ? 256 : bn;   // weight rows of one column tile
+  const double a_bytes = (double)R_used * k_a * 2, b_bytes = (double)num_n * b_rows * K * 2;
+  const double a_slab = 128.0 * k_a * 2, b_slab = (double)b_rows * K * 2;
   const int gn = (int)std::max(1.0, std::min((double)num_n, floor(budget / b_slab)));
   const int gm = (int)std::max(1.0, std::min((double)num_m, floor(budget / a_slab)));
   const double t0 = b_bytes + a_bytes * ((num_n + gn - 1) / gn);

@@ -20,9 +20,11 @@ namespace cc {
 
 namespace {
 
+// BN: the widest column tile (256); a launch uses TBN = 256 or, for narrow
+// problems (less than one wave of 256-column tiles), 128.
 constexpr int BM = 128, BN = 256, BK = 64, ST = 4;
 constexpr int A_BYTES = BM * BK * 2;   // 16 KB
-constexpr int B_BYTES = BN * BK * 2;   // 32 KB
+constexpr int B_BYTES = BN * BK * 2;   // 32 KB: shared-memory stage of the widest B tile
 constexpr int kThreads = 192;
 constexpr int kMaxBatch = 1024;
 constexpr size_t kSmemBytes = 1024 /*align slack*/ + ST * (A_BYTES + B_BYTES) + 256 +
@@ -42,9 +44,10 @@ CC_DEV void rope_cs(uint32_t pos, unsigned long long turns, float &c, float &s) 
 }
 
 // RoPE'd bf16 store of one accumulator tile row: destination columns
-// [col0, col0 + BN) of out (row stride ldo, n_dest columns in all), each tile
-// holding BN / head_dim whole heads; rotate-half pairs (k, k + dh/2); the
+// [col0, col0 + TBN) of out (row stride ldo, n_dest columns in all), each tile
+// holding TBN / head_dim whole heads; rotate-half pairs (k, k + dh/2); the
 // bias (optional) is added before the rotation.
+template <int TBN>
 CC_DEV void rope_store(const GemmParams &p, uint32_t tacc, int grow, bool valid,
                        __nv_bfloat16 *out_base, int ldo, const __nv_bfloat16 *bias, int col0,
                        int n_dest) {
@@ -52,7 +55,7 @@ CC_DEV void rope_store(const GemmParams &p, uint32_t tacc, int grow, bool valid,
   const uint32_t pos = valid ? (uint32_t)p.pos[grow] : 0u;
   __nv_bfloat16 *out = out_base + (size_t)grow * ldo;
 #pragma unroll 1
-  for (int hb = 0; hb < BN; hb += p.head_dim) {
+  for (int hb = 0; hb < TBN; hb += p.head_dim) {
 #pragma unroll 1
     for (int c0 = 0; c0 < half; c0 += 32) {
       uint32_t x1[32], x2[32];
@@ -97,11 +100,12 @@ CC_DEV void rope_store(const GemmParams &p, uint32_t tacc, int grow, bool valid,
 }
 
 // Plain bf16 store (+ optional bias) of one accumulator tile row.
+template <int TBN>
 CC_DEV void plain_store(uint32_t tacc, int grow, bool valid, __nv_bfloat16 *out_base, int ldo,
                         const __nv_bfloat16 *bias, int col0, int n_dest) {
   __nv_bfloat16 *out = out_base + (size_t)grow * ldo;
 #pragma unroll 1
-  for (int c = 0; c < BN / 32; ++c) {
+  for (int c = 0; c < TBN / 32; ++c) {
     uint32_t r[32];
     tmem_ld32(tacc + c * 32, r);
     tmem_ld_wait();
@@ -124,13 +128,13 @@ CC_DEV void plain_store(uint32_t tacc, int grow, bool valid, __nv_bfloat16 *out_
   }
 }
 
-template <int EPI>
+template <int EPI, int TBN>
 CC_DEV void epilogue_tile(const GemmParams &p, uint32_t tacc, int grow, bool valid, int nt,
                           int tile_n0) {
   if constexpr (EPI == EPI_F32 || EPI == EPI_RESID_BF16 || EPI == EPI_RESID_F32) {
     float *out = reinterpret_cast<float *>(p.out) + (size_t)grow * p.ldo;
 #pragma unroll 1
-    for (int c = 0; c < BN / 32; ++c) {
+    for (int c = 0; c < TBN / 32; ++c) {
       uint32_t r[32];
       tmem_ld32(tacc + c * 32, r);
       tmem_ld_wait();
@@ -168,23 +172,23 @@ CC_DEV void epilogue_tile(const GemmParams &p, uint32_t tacc, int grow, bool val
       }
     }
   } else if constexpr (EPI == EPI_QROPE) {
-    rope_store(p, tacc, grow, valid, reinterpret_cast<__nv_bfloat16 *>(p.out), p.ldo, p.bias,
-               tile_n0, p.N);
+    rope_store<TBN>(p, tacc, grow, valid, reinterpret_cast<__nv_bfloat16 *>(p.out), p.ldo, p.bias,
+                    tile_n0, p.N);
   } else if constexpr (EPI == EPI_BF16) {
-    plain_store(tacc, grow, valid, reinterpret_cast<__nv_bfloat16 *>(p.out), p.ldo, p.bias,
-                tile_n0, p.N);
+    plain_store<TBN>(tacc, grow, valid, reinterpret_cast<__nv_bfloat16 *>(p.out), p.ldo, p.bias,
+                     tile_n0, p.N);
   } else if constexpr (EPI == EPI_QKV) {
     // fused projections: column tiles [0, nq) are Q, [nq, nq+nk) K, the rest V
     const int nq = p.n_q_tiles, nk = p.n_k_tiles;
     if (nt < nq)
-      rope_store(p, tacc, grow, valid, reinterpret_cast<__nv_bfloat16 *>(p.out), p.ldo, p.bias,
-                 nt * BN, nq * BN);
+      rope_store<TBN>(p, tacc, grow, valid, reinterpret_cast<__nv_bfloat16 *>(p.out), p.ldo,
+                      p.bias, nt * TBN, nq * TBN);
     else if (nt < nq + nk)
-      rope_store(p, tacc, grow, valid, reinterpret_cast<__nv_bfloat16 *>(p.out_k), p.ldo_kv,
-                 p.bias_k, (nt - nq) * BN, nk * BN);
+      rope_store<TBN>(p, tacc, grow, valid, reinterpret_cast<__nv_bfloat16 *>(p.out_k), p.ldo_kv,
+                      p.bias_k, (nt - nq) * TBN, nk * TBN);
     else
-      plain_store(tacc, grow, valid, reinterpret_cast<__nv_bfloat16 *>(p.out_v), p.ldo_kv,
-                  p.bias_v, (nt - nq - nk) * BN, nk * BN);
+      plain_store<TBN>(tacc, grow, valid, reinterpret_cast<__nv_bfloat16 *>(p.out_v), p.ldo_kv,
+                       p.bias_v, (nt - nq - nk) * TBN, nk * TBN);
   } else if constexpr (EPI == EPI_SWIGLU) {
     // columns [0,128) = gate rows nt*128.., [128,256) = up rows nt*128..
     __nv_bfloat16 *out = reinterpret_cast<__nv_bfloat16 *>(p.out) + (size_t)grow * p.ldo;
@@ -225,7 +229,7 @@ CC_DEV void epilogue_tile(const GemmParams &p, uint32_t tacc, int grow, bool val
     float m = -INFINITY, s = 0.f, zt = 0.f;
     bool has_t = false;
 #pragma unroll 1
-    for (int c = 0; c < BN / 32; ++c) {
+    for (int c = 0; c < TBN / 32; ++c) {
       uint32_t r[32];
       tmem_ld32(tacc + c * 32, r);
       tmem_ld_wait();
@@ -276,11 +280,12 @@ CC_DEV void tile_coords(const GemmParams &p, int t, int num_m, int &m, int &n) {
   }
 }
 
-template <int EPI>
+template <int EPI, int TBN>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                 const __grid_constant__ CUtensorMap tmB2, const __grid_constant__ CUtensorMap tmB3,
                 const __grid_constant__ GemmParams p) {
+  constexpr int TB_BYTES = TBN * BK * 2;   // B stage of this launch's tile width
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                               ~uintptr_t(1023));
@@ -344,22 +349,22 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int kb0 = split * nk_total / S, kb1 = (split + 1) * nk_total / S;
         for (int kb = kb0; kb < kb1; ++kb) {
           if (!mbar_wait(&empty[stage], phase ^ 1, abort_flag, p.status)) goto producer_done;
-          mbar_arrive_expect_tx(&full[stage], A_BYTES + B_BYTES);
+          mbar_arrive_expect_tx(&full[stage], A_BYTES + TB_BYTES);
           // A column block kb of [hi | lo] (hi and lo halves are K apart), B block kb mod nk
           const int ka = kb < nk ? kb * BK : p.K + (kb - nk) * BK;
           const int kw = (kb < nk ? kb : kb - nk) * BK;
           tma_load_2d_hint(sA + stage * A_BYTES, &tmA, &full[stage], ka, row0, pol_a);
           if constexpr (EPI == EPI_SWIGLU) {
-            tma_load_2d_hint(sB + stage * B_BYTES, &tmB, &full[stage], kw, nt * 128, pol_b);
-            tma_load_2d_hint(sB + stage * B_BYTES + B_BYTES / 2, &tmB2, &full[stage], kw, nt * 128,
+            tma_load_2d_hint(sB + stage * TB_BYTES, &tmB, &full[stage], kw, nt * 128, pol_b);
+            tma_load_2d_hint(sB + stage * TB_BYTES + TB_BYTES / 2, &tmB2, &full[stage], kw, nt * 128,
                              pol_b);
           } else if constexpr (EPI == EPI_QKV) {
             const int nq = p.n_q_tiles, nk = p.n_k_tiles;
             const CUtensorMap *m = nt < nq ? &tmB : (nt < nq + nk ? &tmB2 : &tmB3);
-            const int r0 = (nt < nq ? nt : (nt < nq + nk ? nt - nq : nt - nq - nk)) * BN;
-            tma_load_2d_hint(sB + stage * B_BYTES, m, &full[stage], kw, r0, pol_b);
+            const int r0 = (nt < nq ? nt : (nt < nq + nk ? nt - nq : nt - nq - nk)) * TBN;
+            tma_load_2d_hint(sB + stage * TB_BYTES, m, &full[stage], kw, r0, pol_b);
           } else {
-            tma_load_2d_hint(sB + stage * B_BYTES, &tmB, &full[stage], kw, nt * BN, pol_b);
+            tma_load_2d_hint(sB + stage * TB_BYTES, &tmB, &full[stage], kw, nt * TBN, pol_b);
           }
           if (++stage == ST) { stage = 0; phase ^= 1; }
         }
@@ -368,7 +373,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp == 1) {
     if (lane == 0) {  // ---------------- MMA issuer
-      constexpr uint32_t idesc = make_idesc_bf16(BM, BN, 0, 0);
+      constexpr uint32_t idesc = make_idesc_bf16(BM, TBN, 0, 0);
       const uint64_t a_desc0 = make_sdesc_sw128(smem_u32(sA), 16, 1024);
       const uint64_t b_desc0 = make_sdesc_sw128(smem_u32(sB), 16, 1024);
       int stage = 0, acc = 0;
@@ -378,14 +383,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int kb0 = split * nk_total / S, kb1 = (split + 1) * nk_total / S;
         if (!mbar_wait(&tempty[acc], acc_phase ^ 1, abort_flag, p.status)) break;
         tc_fence_after();
-        const uint32_t d_tmem = tmem_base + acc * BN;
+        const uint32_t d_tmem = tmem_base + acc * TBN;
         for (int kb = kb0; kb < kb1; ++kb) {
           if (!mbar_wait(&full[stage], phase, abort_flag, p.status)) goto mma_done;
           tc_fence_after();
           // descriptors of this stage; a K step of 16 columns advances the
           // start-address field by 32 bytes (+2 in 16-byte units)
           const uint64_t ad = a_desc0 + (uint64_t)(stage * (A_BYTES >> 4));
-          const uint64_t bd = b_desc0 + (uint64_t)(stage * (B_BYTES >> 4));
+          const uint64_t bd = b_desc0 + (uint64_t)(stage * (TB_BYTES >> 4));
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k)
             umma_ss(d_tmem, ad + 2 * k, bd + 2 * k, idesc, (kb != kb0 || k != 0) ? 1u : 0u);
@@ -412,7 +417,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int grow = b * p.cap + i;
       if (!mbar_wait(&tfull[acc], acc_phase, abort_flag, p.status)) break;
       tc_fence_after();
-      const uint32_t tacc = tmem_base + acc * BN + (uint32_t(q * 32) << 16);
+      const uint32_t tacc = tmem_base + acc * TBN + (uint32_t(q * 32) << 16);
       // K splits add into out in split order (deterministic sums): split s
       // waits until split s-1 of the tile has published epoch * 16 + s.
       // Split s-1 is a lower work item, and every CTA takes its items in
@@ -424,7 +429,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         named_barrier_sync(1, 128);
         add = split_ok != 0;   // a wait that gave up (status set) skips this split's add
       }
-      if (add) epilogue_tile<EPI>(p, tacc, grow, valid, nt, nt * BN);
+      if (add) epilogue_tile<EPI, TBN>(p, tacc, grow, valid, nt, nt * TBN);
       tc_fence_before();
       if (S > 1) {
         named_barrier_sync(1, 128);
@@ -448,10 +453,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-template <int EPI>
-cudaError_t launch(const CUtensorMap &a, const CUtensorMap &b, const CUtensorMap &b2,
-                   const CUtensorMap &b3, const GemmParams &p, int grid, cudaStream_t stream) {
-  auto kern = gemm_kernel<EPI>;
+template <int EPI, int TBN>
+cudaError_t launch_t(const CUtensorMap &a, const CUtensorMap &b, const CUtensorMap &b2,
+                     const CUtensorMap &b3, const GemmParams &p, int grid, cudaStream_t stream) {
+  auto kern = gemm_kernel<EPI, TBN>;
   static bool attr_set[64] = {};
   int dev = 0;
   cudaGetDevice(&dev);
@@ -463,6 +468,19 @@ cudaError_t launch(const CUtensorMap &a, const CUtensorMap &b, const CUtensorMap
   }
   kern<<<grid, kThreads, kSmemBytes, stream>>>(a, b, b2, b3, p);
   return cudaGetLastError();
+}
+
+// SwiGLU (gate and up halves), LSE and the fused q/k/v projections always
+// use 256-wide tiles; the others take p.block_n (128 or 256).
+template <int EPI>
+cudaError_t launch(const CUtensorMap &a, const CUtensorMap &b, const CUtensorMap &b2,
+                   const CUtensorMap &b3, const GemmParams &p, int grid, cudaStream_t stream) {
+  if constexpr (EPI == EPI_SWIGLU || EPI == EPI_LSE || EPI == EPI_QKV) {
+    return launch_t<EPI, BN>(a, b, b2, b3, p, grid, stream);
+  } else {
+    if (p.block_n == 128) return launch_t<EPI, 128>(a, b, b2, b3, p, grid, stream);
+    return launch_t<EPI, BN>(a, b, b2, b3, p, grid, stream);
+  }
 }
 
 }  // namespace

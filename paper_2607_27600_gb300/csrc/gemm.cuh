@@ -22,7 +22,9 @@ struct GemmParams {
   const int32_t *seq_len;  // device [batch]: rows of sequence b end at slot seq_len[b]
   const int32_t *row_lo;   // device [batch] or nullptr: rows start at slot row_lo[b] (else 0)
   int N, K;
-  int n_tiles;             // column tiles (of gemm_block_n(epi) columns)
+  int block_n;             // column tile width: 256, or 128 for narrow problems (not SwiGLU,
+                           // LSE or the fused q/k/v projections)
+  int n_tiles;             // column tiles (of block_n columns; SwiGLU: 128 outputs each)
   void *out;
   int ldo;
   const void *resid;
