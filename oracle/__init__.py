@@ -31,6 +31,8 @@ Parity status per function (what pins it, in tests/test_oracle_*.py):
                            routine) with keys as queries
   importance/h2o scores    closed forms (one head, equal keys -> uniform); H2O
                            over two refreshes = one update with both layer sets
+  decode_step              = the causal forward's next-token argmax at the last
+                           position, step by step over a greedy continuation
   append_chunk             into an empty cache = causal_forward; chunk-by-chunk
                            appends = one append (no refresh between); the layer's
                            attention after a compaction by scalar brute force
@@ -42,4 +44,5 @@ from .refresh import (rms_norm, rope, rope_angles, rope_inv_freq, project, softm
                       causal_attention, silu, swiglu_mlp, counter_causal_layer, score_head,
                       score_layer, score_full, select_keep, compact, causal_forward,
                       memory_causal_attention, append_chunk, recency_scores,
-                      key_attention_colsums, importance_scores, h2o_update, h2o_scores)
+                      key_attention_colsums, importance_scores, h2o_update, h2o_scores,
+                      decode_step)

@@ -488,3 +488,24 @@ def h2o_scores(acc, seq_len, recent):
         out[b, :n] = acc[b, :n]
         out[b, max(0, n - int(recent)):n] = POS_INF
     return out
+
+
+def decode_step(shape, weights, cache, tokens):
+    """One decode step of the inference cycle (Algorithm DoInference for a
+    single token, greedy sampling as in the paper's experiments): each
+    sequence's current token x_t is appended (append_chunk with one token:
+    its K, V and H^(L-1) through every layer, attending the memory and
+    itself), and the final norm and LM head give the logits of the next
+    token.  Returns (next tokens [B], their logits [B], all logits [B, V]);
+    ties go to the lowest token id."""
+    bsz = len(tokens)
+    nxt = np.zeros(bsz, dtype=np.int64)
+    best = np.zeros(bsz)
+    logits = np.zeros((bsz, shape.vocab))
+    for b in range(bsz):
+        x = append_chunk(shape, weights, cache, b, [int(tokens[b])])
+        u = rms_norm(x, weights["final_norm"], shape.rms_eps)
+        logits[b] = (u @ f64(weights["lm_head"]).T)[0]
+        nxt[b] = int(np.argmax(logits[b]))
+        best[b] = logits[b, nxt[b]]
+    return nxt, best, logits

@@ -132,3 +132,27 @@ def test_append_after_compaction_brute_force():
         want = hh + lw["w_down"] @ (gt / (1 + np.exp(-gt)) * up)
         np.testing.assert_allclose(x[ri], want, rtol=1e-10, atol=1e-12)
     assert np.all(np.isfinite(c["k"][0][0, :8])) and c["seq_len"][0] == 8
+
+
+def test_decode_steps_equal_the_causal_forward():
+    """Greedy decoding step by step (append one token, LM head, argmax) gives,
+    at every step, the argmax of the causal forward's final hidden state at
+    the last position of the whole sequence so far; an argmax pin against
+    the logits themselves."""
+    shape = SMALL
+    w = _model(shape, 44)
+    prompt = list(np.random.default_rng(44).integers(0, shape.vocab, size=6))
+    c = _empty_cache(shape, 16)
+    oracle.append_chunk(shape, w, c, 0, prompt[:-1])
+    seq = list(prompt)
+    tok = prompt[-1]
+    for _ in range(4):
+        nxt, best, logits = oracle.decode_step(shape, w, c, [tok])
+        fw = oracle.causal_forward(shape, w, np.array(seq), np.arange(len(seq)))
+        u = fw["h_final"][-1] / np.sqrt(np.mean(fw["h_final"][-1] ** 2) + shape.rms_eps)
+        z = (u * w["final_norm"]) @ w["lm_head"].astype(np.float64).T
+        np.testing.assert_allclose(logits[0], z, rtol=1e-10, atol=1e-12)
+        assert nxt[0] == int(np.argmax(z)) and best[0] == pytest.approx(z.max(), rel=1e-12)
+        assert c["seq_len"][0] == len(seq)
+        tok = int(nxt[0])
+        seq.append(tok)
