@@ -204,11 +204,28 @@ cc_status cc_compact_kv(const cc_model_cfg *cfg, const cc_kv_cache *cache,
  *              the positions following pos[b][seq_len[b]-1] (0 when empty).
  *   count:     device int32 [batch]; a count outside [0, max_count] or past
  *              cap sets CC_ERR_DEVICE_ARG on the device and appends nothing
- *              to that sequence.
+ *              to that sequence.  NULL with max_count == 1: one token each.
  * Needs embed and, for every layer, wq, wk, wv, wo, the norms and the MLP
  * (biases optional); every k[l], v[l] non-NULL.  Asynchronous on `stream`;
  * the workspace is that of cc_append_workspace_size. */
 size_t cc_append_workspace_size(const cc_model_cfg *cfg, int32_t batch, int32_t cap);
+/* ---- inference cycle, decode (Algorithm CacheManagedInference, decode
+ * phase; DoInference for one token with greedy sampling, as in the paper's
+ * experiments) ----------------------------------------------------------------
+ * Appends tokens_in[b] (device int32 [batch], the current token x_t of each
+ * sequence) exactly as cc_append_chunk with one token each, then applies the
+ * final norm and the LM head to that position and writes the next token
+ * next_tokens[b] = argmax of the logits (the lowest id on ties; -1 for a
+ * sequence that could not append: full cache, reported on the device) and,
+ * if next_logit is non-NULL, its logit.  Needs everything cc_append_chunk
+ * needs plus final_norm and lm_head.  Each sequence's row is its own GEMM row
+ * tile: one sequence reads the weights once per step, a batch of B reads
+ * them B times (decode batching across sequences is not fused). */
+size_t cc_decode_workspace_size(const cc_model_cfg *cfg, int32_t batch, int32_t cap);
+cc_status cc_decode_step(const cc_model_cfg *cfg, const cc_model_weights *w,
+                         const cc_kv_cache *cache, const int32_t *tokens_in,
+                         int32_t *next_tokens, float *next_logit, void *ws, size_t ws_bytes,
+                         void *stream);
 cc_status cc_append_chunk(const cc_model_cfg *cfg, const cc_model_weights *w,
                           const cc_kv_cache *cache, const int32_t *tokens_in,
                           const int32_t *pos_in, const int32_t *count, int32_t max_count,

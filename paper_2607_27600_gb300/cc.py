@@ -92,6 +92,12 @@ _SIGS = {
                                          ctypes.c_void_p]),
     "cc_score_h2o": (ctypes.c_int, [ctypes.POINTER(cc_kv_cache), ctypes.c_int32, ctypes.c_void_p,
                                     ctypes.c_void_p]),
+    "cc_decode_workspace_size": (ctypes.c_size_t, [ctypes.POINTER(cc_model_cfg), ctypes.c_int32,
+                                                   ctypes.c_int32]),
+    "cc_decode_step": (ctypes.c_int, [ctypes.POINTER(cc_model_cfg), ctypes.POINTER(cc_model_weights),
+                                      ctypes.POINTER(cc_kv_cache), ctypes.c_void_p, ctypes.c_void_p,
+                                      ctypes.c_void_p, ctypes.c_void_p, ctypes.c_size_t,
+                                      ctypes.c_void_p]),
     "cc_select_workspace_size": (ctypes.c_size_t, [ctypes.c_int32, ctypes.c_int32]),
     "cc_select_keep": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int32,
                                       ctypes.c_int32, ctypes.c_void_p, ctypes.c_int32,
@@ -304,6 +310,19 @@ def cc_score_h2o(cache, recent: int, scores, stream=None):
     _check(load_library().cc_score_h2o(ctypes.byref(cache.c), int(recent),
                                        _dev_ptr(scores, "scores"), _stream(stream)),
            "cc_score_h2o")
+
+
+def cc_decode_workspace_size(cfg, batch: int, cap: int) -> int:
+    return int(load_library().cc_decode_workspace_size(ctypes.byref(_cfg(cfg)), batch, cap))
+
+
+def cc_decode_step(cfg, weights, cache, tokens_in, next_tokens, next_logit, ws, stream=None):
+    """Decode step: append tokens_in [B] (one each), greedy next tokens [B]."""
+    _check(load_library().cc_decode_step(
+        ctypes.byref(_cfg(cfg)), ctypes.byref(weights.c), ctypes.byref(cache.c),
+        _dev_ptr(tokens_in, "tokens_in"), _dev_ptr(next_tokens, "next_tokens"),
+        _dev_ptr(next_logit, "next_logit"), _dev_ptr(ws, "ws"), ws.numel() * ws.element_size(),
+        _stream(stream)), "cc_decode_step")
 
 
 def cc_select_workspace_size(batch: int, cap: int) -> int:

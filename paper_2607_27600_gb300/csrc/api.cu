@@ -454,8 +454,8 @@ cc_status check_append_args(const cc_model_cfg *c, const cc_model_weights *w,
                             const int32_t *count, int max_count, void *ws, size_t ws_bytes) {
   cc_status s = check_cfg(c);
   if (s != CC_OK) return s;
-  if (!w || !kv || !w->layers || !w->embed || !kv->k || !kv->v || !tokens_in || !count ||
-      max_count < 0)
+  if (!w || !kv || !w->layers || !w->embed || !kv->k || !kv->v || !tokens_in || max_count < 0 ||
+      (!count && max_count != 1))   // no count array: one token each
     return CC_ERR_INVALID_ARG;
   if (kv->batch < 1 || kv->cap < 1 || !kv->seq_len || !kv->tokens || !kv->pos)
     return CC_ERR_INVALID_ARG;
@@ -922,6 +922,58 @@ cc_status cc_score_h2o(const cc_kv_cache *kv, int32_t recent, float *scores, voi
     return CC_ERR_INVALID_ARG;
   CC_TRY(launch_h2o_scores(kv->h2o_acc, kv->seq_len, kv->batch, kv->cap, recent, scores,
                            reinterpret_cast<cudaStream_t>(stream)));
+  return CC_OK;
+}
+
+// ---- decode step (greedy): append one token each, LM head, argmax -------------
+size_t decode_part_offset(const cc_model_cfg *c, int batch, int cap) {
+  return align256(append_layout(c, batch, cap).total);
+}
+
+size_t cc_decode_workspace_size(const cc_model_cfg *cfg, int32_t batch, int32_t cap) {
+  if (check_cfg(cfg) != CC_OK || batch < 1 || cap < 1) return 0;
+  const size_t n_tiles = ((size_t)cfg->vocab + 127) / 128;   // column tiles, either width
+  return decode_part_offset(cfg, batch, cap) + align256((size_t)batch * n_tiles * 8);
+}
+
+cc_status cc_decode_step(const cc_model_cfg *cfg, const cc_model_weights *w,
+                         const cc_kv_cache *cache, const int32_t *tokens_in, int32_t *next_tokens,
+                         float *next_logit, void *ws, size_t ws_bytes, void *stream) {
+  if (!cfg || !w || !cache || !tokens_in || !next_tokens || !w->final_norm || !w->lm_head)
+    return CC_ERR_INVALID_ARG;
+  if (check_cfg(cfg) != CC_OK) return check_cfg(cfg);
+  if (!aligned16(w->final_norm) || !aligned16(w->lm_head)) return CC_ERR_INVALID_ARG;
+  if (!ws || ws_bytes < cc_decode_workspace_size(cfg, cache->batch, cache->cap))
+    return CC_ERR_WORKSPACE;
+  cc_status s = run_append(cfg, w, cache, tokens_in, nullptr, nullptr, 1, ws, ws_bytes, stream);
+  if (s != CC_OK) return s;
+  DevState *dev;
+  if (!dev_state(&dev)) return device_fail();
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  const int batch = cache->batch, cap = cache->cap, d = cfg->d_model;
+  const AppendWs L = append_layout(cfg, batch, cap);
+  uint8_t *wsb = reinterpret_cast<uint8_t *>(ws);
+  void *xn = wsb + L.s.xn;
+  float *h = reinterpret_cast<float *>(wsb + L.s.h);
+  int32_t *lo = reinterpret_cast<int32_t *>(wsb + L.lo), *hi = reinterpret_cast<int32_t *>(wsb + L.hi);
+  float2 *part = reinterpret_cast<float2 *>(wsb + decode_part_offset(cfg, batch, cap));
+  {
+    TimedScope t(CC_KERNEL_RMSNORM, st);
+    CC_TRY(launch_rmsnorm(h, true, w->final_norm, xn, d, cfg->rms_eps, hi, cap, batch * cap, false,
+                          st, lo));
+  }
+  Gemm g;
+  if ((s = gemm_setup(g, EPI_ARGMAX, xn, d, w->lm_head, nullptr, cfg->vocab, batch, cap, hi,
+                      dev->status, false, (uint64_t)batch)) != CC_OK)
+    return s;
+  g.p.row_lo = lo;
+  g.p.out = part;
+  g.p.ldo = g.p.n_tiles;
+  if ((s = run_gemm(g, EPI_ARGMAX, CC_KERNEL_GEMM_LMHEAD, dev->sms, st)) != CC_OK) return s;
+  {
+    TimedScope t(CC_KERNEL_APPEND, st);
+    CC_TRY(launch_argmax_combine(part, g.p.n_tiles, lo, hi, batch, next_tokens, next_logit, st));
+  }
   return CC_OK;
 }
 

@@ -257,6 +257,28 @@ CC_DEV void epilogue_tile(const GemmParams &p, uint32_t tacc, int grow, bool val
       reinterpret_cast<float2 *>(p.out)[(size_t)grow * p.ldo + nt] = make_float2(m, s);
       if (has_t) p.z_target[grow] = zt;
     }
+  } else if constexpr (EPI == EPI_ARGMAX) {
+    // the tile's largest logit and its first column (NaN never wins)
+    float m = -INFINITY;
+    int mi = -1;
+#pragma unroll 1
+    for (int c = 0; c < TBN / 32; ++c) {
+      uint32_t r[32];
+      tmem_ld32(tacc + c * 32, r);
+      tmem_ld_wait();
+      const int col = tile_n0 + c * 32;
+#pragma unroll
+      for (int k = 0; k < 32; ++k) {
+        const float v = __uint_as_float(r[k]);
+        if (col + k < p.N && v > m) {
+          m = v;
+          mi = col + k;
+        }
+      }
+    }
+    if (valid)
+      reinterpret_cast<float2 *>(p.out)[(size_t)(grow / p.cap) * p.ldo + nt] =
+          make_float2(m, __int_as_float(mi));
   }
 }
 
@@ -499,6 +521,7 @@ cudaError_t launch_gemm(int epi, const CUtensorMap &a, const CUtensorMap &b, con
     case EPI_LSE: return launch<EPI_LSE>(a, b, b2, b3, p, grid, stream);
     case EPI_BF16: return launch<EPI_BF16>(a, b, b2, b3, p, grid, stream);
     case EPI_QKV: return launch<EPI_QKV>(a, b, b2, b3, p, grid, stream);
+    case EPI_ARGMAX: return launch<EPI_ARGMAX>(a, b, b2, b3, p, grid, stream);
     default: return cudaErrorInvalidValue;
   }
 }

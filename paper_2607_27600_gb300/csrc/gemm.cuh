@@ -13,8 +13,10 @@ enum GemmEpi : int {
   EPI_LSE = 5,        // out float2 [rows][ldo = n_tiles] = (max, sum exp) per vocab tile,
                       // z_target[row] = logit of tokens[row]
   EPI_BF16 = 6,       // out bf16 [rows][ldo] = acc (+ bias[col] if bias)
-  EPI_QKV = 7         // fused q/k/v projections (B = Wq, B2 = Wk, B3 = Wv, stacked by column
+  EPI_QKV = 7,        // fused q/k/v projections (B = Wq, B2 = Wk, B3 = Wv, stacked by column
                       // tiles): Q RoPE'd to out, K RoPE'd to out_k, V to out_v
+  EPI_ARGMAX = 8      // greedy decoding, one valid row per sequence b: out float2
+                      // [b][ldo = n_tiles] = (max, first column of the max) per column tile
 };
 
 struct GemmParams {

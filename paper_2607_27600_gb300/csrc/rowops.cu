@@ -151,7 +151,7 @@ __global__ void append_prepare_kernel(const int32_t *seq_len, const int32_t *cou
                                       int32_t *row_hi, int cap, unsigned *status) {
   const int b = blockIdx.x;
   const int lo = seq_len[b];
-  int c = count[b];
+  int c = count ? count[b] : 1;   // no count array: one token each (a decode step)
   if (lo < 0 || lo > cap || c < 0 || c > max_count || lo + c > cap) {
     if (threadIdx.x == 0) set_status(status, CC_ERR_DEVICE_ARG);
     c = 0;   // nothing appended; seq_len is left as it was
@@ -172,6 +172,41 @@ __global__ void append_prepare_kernel(const int32_t *seq_len, const int32_t *cou
 __global__ void append_finish_kernel(int32_t *seq_len, const int32_t *row_hi, int batch) {
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b < batch) seq_len[b] = row_hi[b];
+}
+
+// Greedy decoding: the next token of sequence b is the first column of the
+// largest logit over the column tiles' (max, column) pairs; -1 when the
+// sequence appended nothing (row_hi == row_lo).
+__global__ void argmax_combine_kernel(const float2 *part, int n_tiles, const int32_t *row_lo,
+                                      const int32_t *row_hi, int batch, int32_t *next,
+                                      float *best) {
+  const int b = blockIdx.x;
+  const int lane = threadIdx.x;
+  float m = -INFINITY;
+  int mi = 0x7FFFFFFF;
+  if (row_hi[b] > row_lo[b]) {
+    for (int t = lane; t < n_tiles; t += 32) {
+      const float2 v = part[(size_t)b * n_tiles + t];
+      const int idx = __float_as_int(v.y);
+      if (idx >= 0 && (v.x > m || (v.x == m && idx < mi))) {
+        m = v.x;
+        mi = idx;
+      }
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float om = __shfl_xor_sync(0xFFFFFFFFu, m, o);
+    const int oi = __shfl_xor_sync(0xFFFFFFFFu, mi, o);
+    if (om > m || (om == m && oi < mi)) {
+      m = om;
+      mi = oi;
+    }
+  }
+  if (lane == 0) {
+    next[b] = mi == 0x7FFFFFFF ? -1 : mi;
+    if (best) best[b] = m;
+  }
 }
 
 // score = -(RMSNorm(h) * g) . W_U[x_i]; last valid slot +inf; past the end -inf.
@@ -281,6 +316,13 @@ cudaError_t launch_append_prepare(const int32_t *seq_len, const int32_t *count,
                                   int batch, int cap, unsigned *status, cudaStream_t st) {
   append_prepare_kernel<<<batch, 256, 0, st>>>(seq_len, count, tok_in, pos_in, max_count, tokens,
                                                 pos, row_lo, row_hi, cap, status);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_argmax_combine(const float2 *part, int n_tiles, const int32_t *row_lo,
+                                  const int32_t *row_hi, int batch, int32_t *next, float *best,
+                                  cudaStream_t st) {
+  argmax_combine_kernel<<<batch, 32, 0, st>>>(part, n_tiles, row_lo, row_hi, batch, next, best);
   return cudaGetLastError();
 }
 

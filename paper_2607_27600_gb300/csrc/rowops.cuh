@@ -27,6 +27,11 @@ cudaError_t launch_append_prepare(const int32_t *seq_len, const int32_t *count,
 // seq_len = row_hi
 cudaError_t launch_append_finish(int32_t *seq_len, const int32_t *row_hi, int batch,
                                  cudaStream_t st);
+// next[b] = first column of the largest logit over the (max, column) tile
+// pairs part[b][n_tiles] (-1 when sequence b appended nothing); best[b] = it
+cudaError_t launch_argmax_combine(const float2 *part, int n_tiles, const int32_t *row_lo,
+                                  const int32_t *row_hi, int batch, int32_t *next, float *best,
+                                  cudaStream_t st);
 // scores[row] = -(final-norm(h) . lm_head[tokens[row]]), +inf at the last slot
 cudaError_t launch_head_logit(const float *h, const void *gain, const void *lm_head,
                               const int32_t *tokens, float *scores, int d, int vocab, float eps,

@@ -228,3 +228,78 @@ def test_cache_managed_loop_qwen_shape(cc):
         # the cache stores bf16: the oracle keeps its own appended rows at that precision
         for x in cn["k"] + cn["v"] + [cn["h_last"]]:
             x[0, j:j + h] = bf16_round(x[0, j:j + h])
+
+
+def _decode_check(next_tok, best, logits, tol=2e-2):
+    """GPU greedy choice vs the oracle's logits: the argmax wherever the
+    top-2 gap exceeds tol (relative to the logits' rms), else a token whose
+    oracle logit is within tol of the max; the GPU's logit matches."""
+    rms = np.sqrt(np.mean(logits * logits))
+    srt = np.sort(logits)[::-1]
+    if (srt[0] - srt[1]) / rms > tol:
+        assert next_tok == int(np.argmax(logits)), (next_tok, int(np.argmax(logits)))
+    else:
+        assert (srt[0] - logits[next_tok]) / rms <= tol
+    assert abs(best - logits[next_tok]) / max(abs(logits[next_tok]), rms) < tol
+
+
+@pytest.mark.parametrize("shape_name", ["small", "llama2"])
+def test_decode_steps_match_oracle(cc, shape_name):
+    """Greedy decode steps (teacher-forced with the oracle's tokens so both
+    sides share the history): next tokens, their logits, appended K/V rows."""
+    import paper_2607_27600_gb300 as pkg
+    if shape_name == "small":
+        shape, seq, cap, seed = SMALL_GPU, [50, 20, 33], 64, 54
+        w_np = to_np(synth.model_weights(shape, seed, with_kv_proj=True))
+        c_np = causal_cache(shape, w_np, seq, cap, seed)
+    else:
+        shape = ModelShape(**{**synth.configs.LLAMA3_8B.__dict__, "n_layers": 2})
+        seq, cap, seed = [700], 712, 55
+        w = synth.model_weights(shape, seed, device="cuda", with_kv_proj=True)
+        c = synth.synthetic_cache(shape, seq, cap, seed, device="cuda")
+        w_np, c_np = to_np(w), to_np(c)
+    b = len(seq)
+    weights, cache = pkg.Weights(to_device(w_np)), None
+    c_dev = to_device(c_np)
+    cache = pkg.Cache(c_dev)
+    cn = {k: ([np.asarray(x, np.float64).copy() for x in v] if isinstance(v, list) else
+              np.asarray(v).copy()) for k, v in c_np.items()}
+    ws = cc.alloc_workspace(cc.cc_decode_workspace_size(shape, b, cap))
+    tok = np.random.default_rng(seed).integers(0, shape.vocab, size=b)
+    nxt = torch.empty(b, dtype=torch.int32, device="cuda")
+    best = torch.empty(b, dtype=torch.float32, device="cuda")
+    for step in range(4):
+        cc.cc_decode_step(shape, weights, cache, torch.from_numpy(tok.astype(np.int32)).cuda(),
+                          nxt, best, ws)
+        assert cc.cc_get_status() == cc.CC_OK
+        o_next, o_best, o_logits = oracle.decode_step(shape, w_np, cn, tok)
+        g_next, g_best = nxt.cpu().numpy(), best.cpu().numpy()
+        for i in range(b):
+            _decode_check(int(g_next[i]), float(g_best[i]), o_logits[i])
+        got = to_np(c_dev)
+        for i in range(b):
+            n1 = int(cn["seq_len"][i])
+            assert int(got["seq_len"][i]) == n1
+            for l in range(shape.n_layers):
+                assert _rel(got["k"][l][i, n1 - 1], cn["k"][l][i, n1 - 1]) < TOL
+                assert _rel(got["v"][l][i, n1 - 1], cn["v"][l][i, n1 - 1]) < TOL
+        # the cache stores bf16: the oracle keeps its appended rows at that precision
+        for x in cn["k"] + cn["v"] + [cn["h_last"]]:
+            for i in range(b):
+                n1 = int(cn["seq_len"][i])
+                x[i, n1 - 1] = bf16_round(x[i, n1 - 1])
+        tok = o_next
+
+
+def test_decode_full_cache_reports_and_skips(cc):
+    import paper_2607_27600_gb300 as pkg
+    w_np, c_np = _setup(SMALL_GPU, [64, 10], 64, seed=56)
+    weights, c_dev = pkg.Weights(to_device(w_np)), to_device(c_np)
+    cache = pkg.Cache(c_dev)
+    ws = cc.alloc_workspace(cc.cc_decode_workspace_size(SMALL_GPU, 2, 64))
+    nxt = torch.empty(2, dtype=torch.int32, device="cuda")
+    cc.cc_decode_step(SMALL_GPU, weights, cache, torch.tensor([3, 4], dtype=torch.int32,
+                                                              device="cuda"), nxt, None, ws)
+    assert cc.cc_get_status() == cc.CC_ERR_DEVICE_ARG
+    assert nxt.cpu().tolist()[0] == -1 and nxt.cpu().tolist()[1] >= 0
+    assert c_dev["seq_len"].cpu().tolist() == [64, 11]
