@@ -775,6 +775,98 @@ def run_append(args, dist):
     return line
 
 
+def run_decode(args, dist):
+    """Times greedy decode steps (cc_decode_step) of one sequence after a
+    memory of `budgets[0]` slots: each step appends the current token through
+    every layer and picks the next one from the LM head."""
+    import paper_2607_27600_gb300 as pkg
+    from paper_2607_27600_gb300 import cc
+    pkg.load_library()
+    dev = torch.device(f"cuda:{dist.local}")
+    torch.cuda.set_device(dev)
+    wl = synth.WORKLOADS[args.workload]
+    shape = wl.shape
+    j = wl.budgets[0]
+    cap = j + args.warmup + 3 * args.steps + 8   # timed, kernel-table and end-to-end steps
+    w = synth.model_weights(shape, wl.seed, device=dev, with_kv_proj=True)
+    cache = synth.synthetic_cache(shape, [j], cap, wl.seed, device=dev)
+    weights, kc = pkg.Weights(w), pkg.Cache(cache)
+    ws = cc.alloc_workspace(cc.cc_decode_workspace_size(shape, 1, cap), dev)
+    tok = torch.tensor([1], dtype=torch.int32, device=dev)
+    nxt = torch.empty(1, dtype=torch.int32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    for _ in range(args.warmup):
+        cc.cc_decode_step(shape, weights, kc, tok, nxt, None, ws)
+        tok.copy_(nxt)
+    torch.cuda.synchronize(dev)
+    if cc.cc_get_status() != cc.CC_OK:
+        raise SystemExit("device status after warm-up")
+    clocks = ClockSampler(dist.local)
+    clocks.start()
+    time.sleep(0.3)
+    dist.barrier()
+    torch.cuda.synchronize(dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        cc.cc_decode_step(shape, weights, kc, tok, nxt, None, ws)
+        tok.copy_(nxt)
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    dist.barrier()
+    ms = dist.max(e0.elapsed_time(e1) / args.steps)
+    cc.cc_timing_enable(True)   # per-kernel table from separate steps
+    for _ in range(args.steps):
+        cc.cc_decode_step(shape, weights, kc, tok, nxt, None, ws)
+        tok.copy_(nxt)
+    torch.cuda.synchronize(dev)
+    kernels = cc.cc_timing_collect()
+    cc.cc_timing_enable(False)
+    # end to end: the current token from pinned host memory, the next one read back
+    host_tok = torch.ones(1, dtype=torch.int32).pin_memory()
+    host_out = torch.empty(1, dtype=torch.int32).pin_memory()
+    e0.record(stream)
+    for _ in range(args.steps // 2):
+        tok.copy_(host_tok, non_blocking=True)
+        cc.cc_decode_step(shape, weights, kc, tok, nxt, None, ws)
+        host_out.copy_(nxt, non_blocking=True)
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    e2e_ms = dist.max(e0.elapsed_time(e1) / max(1, args.steps // 2))
+    clk = clocks.stop()
+    if cc.cc_get_status() != cc.CC_OK or int(host_out[0]) < 0:
+        raise SystemExit("decode did not complete")
+    peaks, peak_src = load_peaks()
+    d, qd, kvd, f = shape.d_model, shape.q_dim, shape.kv_dim, shape.d_ff
+    n_mid = j + args.warmup + args.steps // 2          # cached slots at a typical step
+    work = {"gemm_qkv": ("hbm", 2.0 * d * (qd + 2 * kvd)), "gemm_oproj": ("hbm", 2.0 * qd * d),
+            "gemm_gateup": ("hbm", 4.0 * d * f), "gemm_down": ("hbm", 2.0 * f * d),
+            "gemm_lmhead": ("hbm", 2.0 * shape.vocab * d),
+            "attention_causal": ("hbm", 2.0 * 2 * kvd * n_mid)}
+    table = kernel_table(kernels, args.steps, work, peaks)
+    dom = max(kernels.items(), key=lambda kv: kv[1][1])[0]
+    dd = table[dom]
+    return {
+        "metric": "decoded tokens/sec per sequence (greedy, all layers + LM head)",
+        "value": round(dist.world / (ms * 1e-3), 1), "unit": "tokens/s", "n_gpus": dist.world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 4),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded random-init weights N(0,0.02); synthetic memory K/V)",
+        "config": {"workload": wl.name + "/decode", "memory_slots": j, "batch": 1,
+                   "layers": shape.n_layers, "d_model": shape.d_model, "vocab": shape.vocab,
+                   "l2": "weights (15 GB) far exceed L2: every step streams them from HBM",
+                   "parallelism": f"replicas x{dist.world}"},
+        "e2e": {"value": round(dist.world / (e2e_ms * 1e-3), 1), "unit": "tokens/s",
+                "h2d_bytes_per_step": 4, "d2h_bytes_per_step": 4, "ms_per_step": round(e2e_ms, 4)},
+        "gpu_launches": int(sum(c for c, _ in kernels.values())),
+        "roofline": {"kernel": dom, "bound": dd.get("bound"), "achieved": dd.get("achieved"),
+                     "peak": peaks["hbm_gbs"], "unit": dd.get("unit"), "frac": dd.get("frac"),
+                     "traffic": None, "peak_source": f"{peak_src} (HBM copy)"},
+        "kernels": table,
+        "clocks": clk,
+    }
+
+
 def append_cpu_baseline(shape, w, cache, chunk, j, h, sample=8):
     """The oracle's append timed on the host cores for `sample` chunk tokens
     through one layer, extrapolated linearly to the chunk and every layer (a
@@ -818,6 +910,9 @@ def main():
                          "scorers (Sec. 4) on the same select/compact path")
     ap.add_argument("--recent", type=int, default=256,
                     help="h2o: proxy-query slots (the most recent) per refresh")
+    ap.add_argument("--decode", action="store_true",
+                    help="time greedy decode steps of one sequence over the workload's "
+                         "budget-sized memory (cc_decode_step)")
     ap.add_argument("--append", action="store_true",
                     help="time the inference cycle: the workload's append chunk over its "
                          "budget-sized memory (cc_append_chunk, every layer)")
@@ -830,6 +925,8 @@ def main():
             line = run_reference(args, dist)
         elif args.append:
             line = run_append(args, dist)
+        elif args.decode:
+            line = run_decode(args, dist)
         else:
             line = run_ours(args, dist)
         if dist.rank == 0 and line is not None:
