@@ -778,7 +778,9 @@ def run_append(args, dist):
 def run_decode(args, dist):
     """Times greedy decode steps (cc_decode_step) of one sequence after a
     memory of `budgets[0]` slots: each step appends the current token through
-    every layer and picks the next one from the LM head."""
+    every layer and picks the next one from the LM head.  The steps are
+    replayed from captured graphs (cc_graph_*: one launch per step, the
+    launch-bound path a serving loop uses); eager calls are timed beside."""
     import paper_2607_27600_gb300 as pkg
     from paper_2607_27600_gb300 import cc
     pkg.load_library()
@@ -787,58 +789,77 @@ def run_decode(args, dist):
     wl = synth.WORKLOADS[args.workload]
     shape = wl.shape
     j = wl.budgets[0]
-    cap = j + args.warmup + 3 * args.steps + 8   # timed, kernel-table and end-to-end steps
+    # warm-up, graph-timed, eager-timed, kernel-table and end-to-end steps
+    cap = j + args.warmup + 4 * args.steps + 16
     w = synth.model_weights(shape, wl.seed, device=dev, with_kv_proj=True)
     cache = synth.synthetic_cache(shape, [j], cap, wl.seed, device=dev)
     weights, kc = pkg.Weights(w), pkg.Cache(cache)
     ws = cc.alloc_workspace(cc.cc_decode_workspace_size(shape, 1, cap), dev)
-    tok = torch.tensor([1], dtype=torch.int32, device=dev)
-    nxt = torch.empty(1, dtype=torch.int32, device=dev)
-    stream = torch.cuda.current_stream(dev)
-    for _ in range(args.warmup):
-        cc.cc_decode_step(shape, weights, kc, tok, nxt, None, ws)
-        tok.copy_(nxt)
-    torch.cuda.synchronize(dev)
-    if cc.cc_get_status() != cc.CC_OK:
-        raise SystemExit("device status after warm-up")
-    clocks = ClockSampler(dist.local)
-    clocks.start()
-    time.sleep(0.3)
-    dist.barrier()
-    torch.cuda.synchronize(dev)
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    for _ in range(args.steps):
-        cc.cc_decode_step(shape, weights, kc, tok, nxt, None, ws)
-        tok.copy_(nxt)
-    e1.record(stream)
-    torch.cuda.synchronize(dev)
-    dist.barrier()
-    ms = dist.max(e0.elapsed_time(e1) / args.steps)
-    cc.cc_timing_enable(True)   # per-kernel table from separate steps
-    for _ in range(args.steps):
-        cc.cc_decode_step(shape, weights, kc, tok, nxt, None, ws)
-        tok.copy_(nxt)
-    torch.cuda.synchronize(dev)
-    kernels = cc.cc_timing_collect()
-    cc.cc_timing_enable(False)
-    # end to end: the current token from pinned host memory, the next one read back
-    host_tok = torch.ones(1, dtype=torch.int32).pin_memory()
-    host_out = torch.empty(1, dtype=torch.int32).pin_memory()
-    e0.record(stream)
-    for _ in range(args.steps // 2):
-        tok.copy_(host_tok, non_blocking=True)
-        cc.cc_decode_step(shape, weights, kc, tok, nxt, None, ws)
-        host_out.copy_(nxt, non_blocking=True)
-    e1.record(stream)
-    torch.cuda.synchronize(dev)
-    e2e_ms = dist.max(e0.elapsed_time(e1) / max(1, args.steps // 2))
-    clk = clocks.stop()
-    if cc.cc_get_status() != cc.CC_OK or int(host_out[0]) < 0:
-        raise SystemExit("decode did not complete")
+    tok = [torch.tensor([1], dtype=torch.int32, device=dev),
+           torch.empty(1, dtype=torch.int32, device=dev)]
+    stream = torch.cuda.Stream(dev)   # captured work needs a stream other than the legacy default
+    graphs = []
+    with torch.cuda.stream(stream):
+        for i in range(args.warmup):
+            cc.cc_decode_step(shape, weights, kc, tok[i % 2], tok[1 - i % 2], None, ws)
+        if args.warmup % 2:
+            tok[0].copy_(tok[1])
+        torch.cuda.synchronize(dev)
+        if cc.cc_get_status() != cc.CC_OK:
+            raise SystemExit("device status after warm-up")
+        for a in (0, 1):   # step a: tokens tok[a] -> next tokens tok[1 - a]
+            cc.cc_graph_begin()
+            cc.cc_decode_step(shape, weights, kc, tok[a], tok[1 - a], None, ws)
+            graphs.append(cc.cc_graph_end())
+        clocks = ClockSampler(dist.local)
+        clocks.start()
+        time.sleep(0.3)
+        dist.barrier()
+        torch.cuda.synchronize(dev)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for i in range(args.steps):
+            cc.cc_graph_launch(graphs[i % 2])
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+        dist.barrier()
+        ms = dist.max(e0.elapsed_time(e1) / args.steps)
+        if args.steps % 2:
+            tok[0].copy_(tok[1])
+        e0.record(stream)
+        for i in range(args.steps):
+            cc.cc_decode_step(shape, weights, kc, tok[i % 2], tok[1 - i % 2], None, ws)
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+        eager_ms = dist.max(e0.elapsed_time(e1) / args.steps)
+        if args.steps % 2:
+            tok[0].copy_(tok[1])
+        cc.cc_timing_enable(True)   # per-kernel table from separate (eager) steps
+        for i in range(args.steps):
+            cc.cc_decode_step(shape, weights, kc, tok[i % 2], tok[1 - i % 2], None, ws)
+        torch.cuda.synchronize(dev)
+        kernels = cc.cc_timing_collect()
+        cc.cc_timing_enable(False)
+        # end to end: the current token from pinned host memory, the next one
+        # read back, the step replayed from its graph
+        host_tok = torch.ones(1, dtype=torch.int32).pin_memory()
+        host_out = torch.empty(1, dtype=torch.int32).pin_memory()
+        e0.record(stream)
+        for _ in range(args.steps // 2):
+            tok[0].copy_(host_tok, non_blocking=True)
+            cc.cc_graph_launch(graphs[0])
+            host_out.copy_(tok[1], non_blocking=True)
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+        e2e_ms = dist.max(e0.elapsed_time(e1) / max(1, args.steps // 2))
+        clk = clocks.stop()
+        for g in graphs:
+            cc.cc_graph_destroy(g)
+        if cc.cc_get_status() != cc.CC_OK or int(host_out[0]) < 0:
+            raise SystemExit("decode did not complete")
     peaks, peak_src = load_peaks()
     d, qd, kvd, f = shape.d_model, shape.q_dim, shape.kv_dim, shape.d_ff
-    n_mid = j + args.warmup + args.steps // 2          # cached slots at a typical step
+    n_mid = j + args.warmup + 2 * args.steps + args.steps // 2   # slots at a kernel-table step
     work = {"gemm_qkv": ("hbm", 2.0 * d * (qd + 2 * kvd)), "gemm_oproj": ("hbm", 2.0 * qd * d),
             "gemm_gateup": ("hbm", 4.0 * d * f), "gemm_down": ("hbm", 2.0 * f * d),
             "gemm_lmhead": ("hbm", 2.0 * shape.vocab * d),
@@ -855,6 +876,8 @@ def run_decode(args, dist):
         "config": {"workload": wl.name + "/decode", "memory_slots": j, "batch": 1,
                    "layers": shape.n_layers, "d_model": shape.d_model, "vocab": shape.vocab,
                    "l2": "weights (15 GB) far exceed L2: every step streams them from HBM",
+                   "launch": "one captured graph per step (cc_graph_launch)",
+                   "eager_ms_per_step": round(eager_ms, 4),
                    "parallelism": f"replicas x{dist.world}"},
         "e2e": {"value": round(dist.world / (e2e_ms * 1e-3), 1), "unit": "tokens/s",
                 "h2d_bytes_per_step": 4, "d2h_bytes_per_step": 4, "ms_per_step": round(e2e_ms, 4)},

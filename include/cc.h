@@ -283,6 +283,36 @@ cc_status cc_compact_kv_static(const cc_model_cfg *cfg, const cc_kv_cache *cache
                                const int32_t *keep_idx, const int32_t *keep_count,
                                void *stream);
 
+/* ---- captured call sequences (CUDA graphs) -----------------------------------
+ * The paper has no counterpart: this is a library convenience for
+ * launch-bound loops (a decode step launches several kernels per layer for
+ * one row each, so the host's launch latency, not the GPU, sets its pace).
+ * cc_graph_begin starts capturing `stream` (a stream the caller created: the
+ * legacy default stream cannot be captured; the capture is local to the
+ * calling host thread); the cc_* calls that follow on that stream and thread
+ * enqueue nothing but are recorded; cc_graph_end stops the capture and
+ * returns an executable graph in *out, which cc_graph_launch replays on any
+ * stream as one launch.
+ *   - A replay repeats the recorded calls with the same arguments: the same
+ *     pointers, sizes and host values.  What the kernels read from device
+ *     memory (seq_len, counts, tokens, positions, keep-sets) is read afresh
+ *     at each replay, so a captured decode step or refresh cycle replays over
+ *     a cache that has grown or been compacted since.
+ *   - Make each call once without capture first (first calls on a device
+ *     set kernel attributes and look up device addresses), and keep launch
+ *     timing (cc_timing_enable) off while capturing: cc_graph_begin returns
+ *     CC_ERR_INVALID_ARG otherwise.
+ *   - A captured call that returns an error leaves a partial recording:
+ *     still call cc_graph_end (the stream leaves capture mode), then destroy
+ *     what it returns.
+ *   - cc_graph_end returns CC_ERR_CUDA (and *out = NULL) when the capture
+ *     was invalidated or the graph cannot be instantiated. */
+typedef struct cc_graph cc_graph;
+cc_status cc_graph_begin(void *stream);
+cc_status cc_graph_end(void *stream, cc_graph **out);
+cc_status cc_graph_launch(const cc_graph *g, void *stream);
+cc_status cc_graph_destroy(cc_graph *g);
+
 /* ---- status ---------------------------------------------------------------
  * Synchronises `stream`, returns the first device-side error recorded since
  * the last call (CC_OK if none) on the current device and clears it.

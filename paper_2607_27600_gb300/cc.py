@@ -111,6 +111,10 @@ _SIGS = {
     "cc_compact_kv_static": (ctypes.c_int, [ctypes.POINTER(cc_model_cfg),
                                             ctypes.POINTER(cc_kv_cache), ctypes.c_void_p,
                                             ctypes.c_void_p, ctypes.c_void_p]),
+    "cc_graph_begin": (ctypes.c_int, [ctypes.c_void_p]),
+    "cc_graph_end": (ctypes.c_int, [ctypes.c_void_p, ctypes.POINTER(ctypes.c_void_p)]),
+    "cc_graph_launch": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p]),
+    "cc_graph_destroy": (ctypes.c_int, [ctypes.c_void_p]),
     "cc_get_status": (ctypes.c_int, [ctypes.c_void_p]),
     "cc_status_str": (ctypes.c_char_p, [ctypes.c_int]),
     "cc_last_error": (ctypes.c_char_p, []),
@@ -359,6 +363,28 @@ def cc_compact_kv_static(cfg, cache: Cache, keep_idx, keep_count, stream=None):
                                                _dev_ptr(keep_idx, "keep_idx"),
                                                _dev_ptr(keep_count, "keep_count"), _stream(stream))
     _check(code, "cc_compact_kv_static")
+
+
+def cc_graph_begin(stream=None):
+    """Starts recording the cc_* calls made on `stream` (not the legacy
+    default stream) by this thread.  Replays reuse every pointer recorded:
+    keep the tensors (and the Weights/Cache objects) alive meanwhile."""
+    _check(load_library().cc_graph_begin(_stream(stream)), "cc_graph_begin")
+
+
+def cc_graph_end(stream=None) -> int:
+    """Stops the recording; returns the executable graph's handle."""
+    h = ctypes.c_void_p()
+    _check(load_library().cc_graph_end(_stream(stream), ctypes.byref(h)), "cc_graph_end")
+    return h.value
+
+
+def cc_graph_launch(graph: int, stream=None):
+    _check(load_library().cc_graph_launch(graph, _stream(stream)), "cc_graph_launch")
+
+
+def cc_graph_destroy(graph: int):
+    _check(load_library().cc_graph_destroy(graph), "cc_graph_destroy")
 
 
 def cc_get_status(stream=None) -> int:

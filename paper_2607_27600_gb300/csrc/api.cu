@@ -382,14 +382,37 @@ cc_status run_gemm(Gemm &g, int epi, int kind, int sms, cudaStream_t st) {
   return CC_OK;
 }
 
+// Key splits of the causal attention: at most this many (unit, split) CTAs
+// write partial results, each split covering at least kAttnMinSplitTiles
+// key tiles of 128.
+constexpr int kAttnMaxSplitSlots = 160;
+constexpr int kAttnMinSplitTiles = 4;
+
+struct AttnPartials {
+  float *o = nullptr;      // [kAttnMaxSplitSlots][256][head_dim]
+  float2 *ml = nullptr;    // [kAttnMaxSplitSlots][256]
+};
+
+// Key splits for a launch of `units` CTAs: used when the units fill less
+// than half of the SMs, so that a short chunk over a long memory (a decode
+// step) still spreads its key tiles over the GPU.
+int attn_key_splits(long long units, int cap, int sms) {
+  if (units < 1 || units * 2 > sms) return 1;
+  const long long by_tiles = ((long long)cap + 127) / 128 / kAttnMinSplitTiles;
+  const long long s = std::min({(long long)sms / units, (long long)kAttnMaxSplitSlots / units,
+                                by_tiles});
+  return s >= 2 ? (int)s : 1;
+}
+
 // out: [R][Hq*dh] bf16, or with split [R][2*Hq*dh] = [hi | lo] per row.
 // Counter-causal attention over rows [0, seq_len); with row_lo, the causal
 // memory-augmented attention of the inference cycle over rows
-// [row_lo, seq_len) (q_span: rows per sequence at most).
+// [row_lo, seq_len) (q_span: rows per sequence at most; with partials, key
+// splits when the launch has few units).
 cc_status run_attention(const cc_model_cfg *c, const void *q, const void *k, const void *v,
                         void *out, const int32_t *seq_len, int batch, int cap, unsigned *status,
                         cudaStream_t st, bool split = false, const int32_t *row_lo = nullptr,
-                        int q_span = 0) {
+                        int q_span = 0, const AttnPartials *parts = nullptr, int sms = 0) {
   const int G = c->n_q_heads / c->n_kv_heads, dh = c->head_dim;
   const int P = attn_positions_per_unit(G);
   const uint64_t R = (uint64_t)batch * cap;
@@ -424,6 +447,11 @@ cc_status run_attention(const cc_model_cfg *c, const void *q, const void *k, con
   p.causal = row_lo ? 1 : 0;
   p.row_lo = row_lo;
   p.q_span = row_lo ? q_span : cap;
+  if (parts && parts->o && parts->ml) {
+    p.kv_splits = attn_key_splits(attn_units(p), cap, sms);
+    p.part_o = parts->o;
+    p.part_ml = parts->ml;
+  }
   TimedScope t(row_lo ? CC_KERNEL_ATTN_CAUSAL : CC_KERNEL_ATTENTION, st);
   CC_TRY(launch_attention(tq, tk, tv, p, st));
   return CC_OK;
@@ -434,7 +462,7 @@ cc_status run_attention(const cc_model_cfg *c, const void *q, const void *k, con
 // ---------------------------------------------------------------------------
 struct AppendWs {
   ScoreWs s;          // xn, q, o, h, act rows b*cap + slot (the chunk's rows only are used)
-  size_t lo, hi, total;
+  size_t lo, hi, part_o, part_ml, total;   // part_*: key-split partials of the attention
 };
 
 AppendWs append_layout(const cc_model_cfg *c, int batch, int cap) {
@@ -445,6 +473,10 @@ AppendWs append_layout(const cc_model_cfg *c, int batch, int cap) {
   off = align256(off + (size_t)batch * 4);
   w.hi = off;
   off = align256(off + (size_t)batch * 4);
+  w.part_o = off;
+  off = align256(off + (size_t)kAttnMaxSplitSlots * 256 * c->head_dim * 4);
+  w.part_ml = off;
+  off = align256(off + (size_t)kAttnMaxSplitSlots * 256 * 8);
   w.total = off;
   return w;
 }
@@ -498,6 +530,9 @@ cc_status run_append(const cc_model_cfg *c, const cc_model_weights *w, const cc_
   unsigned *status = dev->status;
   if ((s = clear_split_flags(flags, st)) != CC_OK) return s;
   const uint64_t used = (uint64_t)batch * max_count;   // rows the GEMMs visit at most
+  AttnPartials parts;
+  parts.o = reinterpret_cast<float *>(wsb + L.part_o);
+  parts.ml = reinterpret_cast<float2 *>(wsb + L.part_ml);
 
   {
     TimedScope t(CC_KERNEL_APPEND, st);
@@ -506,17 +541,19 @@ cc_status run_append(const cc_model_cfg *c, const cc_model_weights *w, const cc_
   }
   {
     TimedScope t(CC_KERNEL_EMBED, st);
-    CC_TRY(launch_embed(w->embed, kv->tokens, h, d, c->vocab, hi, cap, rows, status, st, lo));
+    CC_TRY(launch_embed(w->embed, kv->tokens, h, d, c->vocab, hi, cap, rows, status, st, lo,
+                        max_count));
   }
   for (int l = 0; l < c->n_layers; ++l) {
     const cc_layer_weights &lw = w->layers[l];
     if (l == c->n_layers - 1 && kv->h_last) {   // H^(L-1), recorded for the fast approximation
       TimedScope t(CC_KERNEL_APPEND, st);
-      CC_TRY(launch_store_bf16(h, kv->h_last, d, hi, lo, cap, rows, st));
+      CC_TRY(launch_store_bf16(h, kv->h_last, d, hi, lo, cap, rows, st, max_count));
     }
     {
       TimedScope t(CC_KERNEL_RMSNORM, st);
-      CC_TRY(launch_rmsnorm(h, true, lw.attn_norm, xn, d, c->rms_eps, hi, cap, rows, false, st, lo));
+      CC_TRY(launch_rmsnorm(h, true, lw.attn_norm, xn, d, c->rms_eps, hi, cap, rows, false, st, lo,
+                            max_count));
     }
     // q = RoPE(xn Wq^T + bq) into the workspace; k = RoPE(xn Wk^T + bk) and
     // v = xn Wv^T + bv straight into the cache slots of the chunk
@@ -551,7 +588,7 @@ cc_status run_append(const cc_model_cfg *c, const cc_model_weights *w, const cc_
     }
     // o = attention of the chunk rows over the memory and the chunk (causal)
     if ((s = run_attention(c, q, kv->k[l], kv->v[l], o, hi, batch, cap, status, st, false, lo,
-                           max_count)) != CC_OK)
+                           max_count, &parts, dev->sms)) != CC_OK)
       return s;
     // h += o Wo^T; xn = RMSNorm(h); act = SwiGLU; h += act Wd^T
     Gemm go;
@@ -565,7 +602,8 @@ cc_status run_append(const cc_model_cfg *c, const cc_model_weights *w, const cc_
     if ((s = run_gemm(go, EPI_RESID_F32, CC_KERNEL_GEMM_OPROJ, dev->sms, st)) != CC_OK) return s;
     {
       TimedScope t(CC_KERNEL_RMSNORM, st);
-      CC_TRY(launch_rmsnorm(h, true, lw.mlp_norm, xn, d, c->rms_eps, hi, cap, rows, false, st, lo));
+      CC_TRY(launch_rmsnorm(h, true, lw.mlp_norm, xn, d, c->rms_eps, hi, cap, rows, false, st, lo,
+                            max_count));
     }
     Gemm gu;
     if ((s = gemm_setup(gu, EPI_SWIGLU, xn, d, lw.w_gate, lw.w_up, f, batch, cap, hi, status,
@@ -960,7 +998,7 @@ cc_status cc_decode_step(const cc_model_cfg *cfg, const cc_model_weights *w,
   {
     TimedScope t(CC_KERNEL_RMSNORM, st);
     CC_TRY(launch_rmsnorm(h, true, w->final_norm, xn, d, cfg->rms_eps, hi, cap, batch * cap, false,
-                          st, lo));
+                          st, lo, 1));
   }
   Gemm g;
   if ((s = gemm_setup(g, EPI_ARGMAX, xn, d, w->lm_head, nullptr, cfg->vocab, batch, cap, hi,
@@ -1125,6 +1163,58 @@ cc_status cc_counter_causal_attention(const void *q, const void *k, const void *
   c.head_dim = head_dim;
   return run_attention(&c, q, k, v, out, seq_len, batch, cap, dev->status,
                        reinterpret_cast<cudaStream_t>(stream));
+}
+
+// ---- captured call sequences ------------------------------------------------
+
+struct cc_graph {
+  cudaGraphExec_t exec;
+};
+
+cc_status cc_graph_begin(void *stream) {
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  if (!st) return CC_ERR_INVALID_ARG;   // the legacy default stream cannot be captured
+  {
+    std::lock_guard<std::mutex> lk(g_mu);
+    if (g_timing.on) return CC_ERR_INVALID_ARG;
+  }
+  DevState *dev;
+  if (!dev_state(&dev)) return device_fail();
+  CC_TRY(cudaStreamBeginCapture(st, cudaStreamCaptureModeThreadLocal));
+  return CC_OK;
+}
+
+cc_status cc_graph_end(void *stream, cc_graph **out) {
+  if (out) *out = nullptr;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  if (!st) return CC_ERR_INVALID_ARG;
+  cudaGraph_t graph = nullptr;
+  cudaError_t e = cudaStreamEndCapture(st, &graph);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaStreamEndCapture");
+  if (!out) {
+    cudaGraphDestroy(graph);
+    return CC_ERR_INVALID_ARG;
+  }
+  cudaGraphExec_t exec = nullptr;
+  e = cudaGraphInstantiate(&exec, graph, 0);
+  cudaGraphDestroy(graph);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGraphInstantiate");
+  *out = new cc_graph{exec};
+  return CC_OK;
+}
+
+cc_status cc_graph_launch(const cc_graph *g, void *stream) {
+  if (!g) return CC_ERR_INVALID_ARG;
+  CC_TRY(cudaGraphLaunch(g->exec, reinterpret_cast<cudaStream_t>(stream)));
+  return CC_OK;
+}
+
+cc_status cc_graph_destroy(cc_graph *g) {
+  if (!g) return CC_OK;
+  cudaError_t e = cudaGraphExecDestroy(g->exec);
+  delete g;
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGraphExecDestroy");
+  return CC_OK;
 }
 
 // ---- launch timing (include/cc_profile.h) ----------------------------------

@@ -105,6 +105,40 @@ struct AttnSmem {
   static constexpr int BYTES = OFF_BAR + 256 + 1024;   // barriers + alignment slack
 };
 
+// Work unit `unit_id` -> (sequence b, KV head g, positions p0..p_last).
+// Unit order: streams (sequence, KV head) in groups of streams_per_group;
+// within a group, position blocks outermost (longest units first), the
+// group's streams innermost.  The group size bounds how far apart in time
+// two resident units of one stream read the same K/V tile (chosen so the
+// K/V read in between stays well inside L2).  q_lo: first query slot
+// (causal mode).  valid is false for a bad length (reported) or a block past
+// the sequence end.
+struct UnitInfo {
+  int b, g, n, q_lo, p0, p_last;
+  bool bad, valid;
+};
+CC_DEV UnitInfo decode_unit(const AttnParams &p, int unit_id, bool causal) {
+  UnitInfo u{};
+  const int blocks_per_stream = (p.q_span + p.P - 1) / p.P;
+  const int n_streams = p.batch * p.n_kv_heads;
+  const int per_group = p.streams_per_group * blocks_per_stream;
+  const int grp = unit_id / per_group;
+  const int s0 = grp * p.streams_per_group;
+  const int gsz = min(p.streams_per_group, n_streams - s0);
+  const int r = unit_id - grp * per_group;
+  const int pb = r / gsz;
+  const int stream = s0 + (r - pb * gsz);
+  u.b = stream / p.n_kv_heads;
+  u.g = stream - u.b * p.n_kv_heads;
+  u.n = p.seq_len[u.b];
+  u.q_lo = causal ? p.row_lo[u.b] : 0;
+  u.bad = u.n < 0 || u.n > p.cap || u.q_lo < 0 || u.q_lo > u.n;
+  u.p0 = u.q_lo + pb * p.P;
+  u.valid = !u.bad && u.p0 < u.n;
+  u.p_last = min(u.p0 + p.P, u.n) - 1;
+  return u;
+}
+
 template <int DH, bool CAUSAL>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
@@ -129,36 +163,34 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int G = p.group, P = p.P;
-  // Unit order: streams (sequence, KV head) in groups of streams_per_group;
-  // within a group, position blocks outermost (longest units first), the
-  // group's streams innermost.  The group size bounds how far apart in time
-  // two resident units of one stream read the same K/V tile (chosen so the
-  // K/V read in between stays well inside L2).
-  const int blocks_per_stream = (p.q_span + P - 1) / P;
-  const int n_streams = p.batch * p.n_kv_heads;
-  const int per_group = p.streams_per_group * blocks_per_stream;
-  const int grp = blockIdx.x / per_group;
-  const int s0 = grp * p.streams_per_group;
-  const int gsz = min(p.streams_per_group, n_streams - s0);
-  const int r = blockIdx.x - grp * per_group;
-  const int pb = r / gsz;
-  const int stream = s0 + (r - pb * gsz);
-  const int b = stream / p.n_kv_heads, g = stream - b * p.n_kv_heads;
-  int n = p.seq_len[b];
-  const int q_lo = CAUSAL ? p.row_lo[b] : 0;   // first query slot
-  if (n < 0 || n > p.cap || q_lo < 0 || q_lo > n) {
+  // Key splits (few units): the splits of a unit are consecutive CTAs.
+  const int S = p.kv_splits > 1 ? p.kv_splits : 1;
+  const int unit_id = blockIdx.x / S, split = blockIdx.x - unit_id * S;
+  const UnitInfo u = decode_unit(p, unit_id, CAUSAL);
+  if (u.bad) {
     if (threadIdx.x == 0) set_status(p.status, CC_ERR_DEVICE_ARG);
     return;
   }
-  const int p0 = q_lo + pb * P;
-  if (p0 >= n) return;                       // the whole block lies past the sequence end
-  const int p_last = min(p0 + P, n) - 1;     // last valid position of the block
+  if (!u.valid) return;                      // the whole block lies past the sequence end
+  const int b = u.b, g = u.g, n = u.n, p0 = u.p0, p_last = u.p_last;
   // counter-causal: key tiles holding slots p0+1 .. n-1; causal: slots 0 .. p_last
   const int t0 = CAUSAL ? 0 : (p0 + 1) / BKV;
   const int t1 = CAUSAL ? p_last / BKV : (n - 1) / BKV;
-  const int ntiles = t1 - t0 + 1;
+  const int ntiles_unit = t1 - t0 + 1;
   const size_t row_base = (size_t)b * p.cap;
+  // this CTA's share of the unit's key tiles (all of them without splits):
+  // local iteration `it` handles tile t_hi - it; the tail tile is t_top
+  const int t_top = t1;
+  const int it_off = S > 1 ? split * max(ntiles_unit, 0) / S : 0;
+  const int ntiles = S > 1 ? (split + 1) * max(ntiles_unit, 0) / S - it_off : ntiles_unit;
+  const int t_hi = t1 - it_off;
+  const size_t part_slot = ((size_t)unit_id * S + split) * 256;
 
+  if (S > 1 && ntiles <= 0) {   // nothing for this split: an empty partial
+    for (int R = threadIdx.x; R < 256; R += blockDim.x)
+      p.part_ml[part_slot + R] = make_float2(-INFINITY, 0.f);
+    return;
+  }
   if (ntiles <= 0) {   // no slot after the block: every row attends nothing -> 0
     for (int idx = threadIdx.x; idx < (p_last - p0 + 1) * G; idx += blockDim.x) {
       int pos = p0 + idx / G, hl = idx % G;
@@ -218,7 +250,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     (int)row_base + p0);
     }
     for (int it = 0; it < ntiles; ++it) {
-      const int t = t1 - it, s = it % KST;   // key tiles from the sequence end downwards
+      const int t = t_hi - it, s = it % KST;   // key tiles from the sequence end downwards
       const uint32_t ph = (it / KST) & 1;
       const int krow = (int)row_base + t * BKV;
       int ok = 1;
@@ -240,7 +272,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       ok = __shfl_sync(0xFFFFFFFFu, ok, 0);
       if (!ok) break;
-      if (t == t1 && n - t * BKV < BKV) {
+      if (t == t_top && n - t * BKV < BKV) {
         // rows past the sequence end may hold any bits; P is 0 there, but
         // 0 * NaN would still poison O, so zero them before the PV product
         if (!mbar_wait(&v_full[s], ph, abort_flag, p.status)) break;
@@ -297,12 +329,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         umma_commit(&k_empty[0]);
       }
       for (int it = 0; ok && it < ntiles; ++it) {
-        const int t = t1 - it, s = it % KST;
+        const int t = t_hi - it, s = it % KST;
         const uint32_t ph = (it / KST) & 1;
         TRACE(true, it, 14);
         if (!(ok = mbar_wait(&v_full[s], ph, abort_flag, p.status))) break;
         TRACE(true, it, 15);
-        if (t == t1 && n - t * BKV < BKV)
+        if (t == t_top && n - t * BKV < BKV)
           if (!(ok = mbar_wait(v_fixed, 0, abort_flag, p.status))) break;
         for (int h = 0; h < 2; ++h) {
           TRACE(true, it, 12 + h);
@@ -356,7 +388,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     float m_used = -INFINITY, l = 0.f;   // m_used: reference max of the raw scores
     bool ok = true;
     for (int it = 0; it < ntiles; ++it) {
-      const int j0 = (t1 - it) * BKV;
+      const int j0 = (t_hi - it) * BKV;
       if (!(ok = mbar_wait(&s_ready[h], it & 1, abort_flag, p.status))) break;
       TRACE(q == 0 && lane == 0, it, 0 + h);
       tc_fence_after();
@@ -456,7 +488,22 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     // ---- epilogue: O / l -> bf16 -> out[row_base + pos][g*G + hl][:]
     if (ok) ok = mbar_wait(&o_done[h], 0, abort_flag, p.status);
-    if (ok) {
+    if (ok && S > 1) {   // key split: this CTA's unnormalised O and (max, sum) per row
+      tc_fence_after();
+      float *po = p.part_o + (part_slot + R) * DH;
+#pragma unroll 1
+      for (int c = 0; c < DH; c += 32) {
+        uint32_t o[32];
+        tmem_ld32(o_t + c, o);
+        tmem_ld_wait();
+#pragma unroll
+        for (int v = 0; v < 8; ++v)
+          reinterpret_cast<float4 *>(po + c)[v] =
+              make_float4(__uint_as_float(o[v * 4]), __uint_as_float(o[v * 4 + 1]),
+                          __uint_as_float(o[v * 4 + 2]), __uint_as_float(o[v * 4 + 3]));
+      }
+      p.part_ml[part_slot + R] = make_float2(m_used, l);
+    } else if (ok) {
       tc_fence_after();
       const bool store = row_used && pos <= p_last;
       const float inv = l > 0.f ? 1.f / l : 0.f;
@@ -500,6 +547,42 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
+// Key splits: out = sum_s 2^((m_s - m*) c) O_s / sum_s 2^((m_s - m*) c) l_s
+// per row (m* the largest reference max, c = log2(e)/sqrt(dh)), splits in
+// order; bf16 (and lo) stores as the kernel's own epilogue.  Block = one row
+// of one unit, a thread per head_dim element.
+template <bool CAUSAL>
+__global__ void attn_combine_kernel(const __grid_constant__ AttnParams p) {
+  const int R = blockIdx.x, unit_id = blockIdx.y, d = threadIdx.x;
+  const UnitInfo u = decode_unit(p, unit_id, CAUSAL);
+  const int G = p.group;
+  if (!u.valid || R >= p.P * G) return;
+  const int pos = u.p0 + R / G, hl = R % G;
+  if (pos > u.p_last) return;
+  const int S = p.kv_splits;
+  const float c = p.scale_log2;
+  float m = -INFINITY;
+  for (int s = 0; s < S; ++s) {
+    const float2 ml = p.part_ml[((size_t)unit_id * S + s) * 256 + R];
+    if (ml.y > 0.f) m = fmaxf(m, ml.x);
+  }
+  float o = 0.f, l = 0.f;
+  for (int s = 0; s < S; ++s) {
+    const size_t slot = ((size_t)unit_id * S + s) * 256 + R;
+    const float2 ml = p.part_ml[slot];
+    if (!(ml.y > 0.f)) continue;
+    const float wgt = exp2f((ml.x - m) * c);
+    l += wgt * ml.y;
+    o += wgt * p.part_o[slot * p.head_dim + d];
+  }
+  const float v = l > 0.f ? o / l : 0.f;
+  __nv_bfloat16 *dst = p.out + ((size_t)u.b * p.cap + pos) * p.out_ld +
+                       (size_t)(u.g * G + hl) * p.head_dim + d;
+  const __nv_bfloat16 hi = __float2bfloat16_rn(v);
+  *dst = hi;
+  if (p.out_lo > 0) dst[p.out_lo] = __float2bfloat16_rn(v - __bfloat162float(hi));
+}
+
 template <int DH, bool CAUSAL>
 cudaError_t launch_dh(const CUtensorMap &q, const CUtensorMap &k, const CUtensorMap &v,
                       const AttnParams &p, cudaStream_t stream) {
@@ -513,7 +596,7 @@ cudaError_t launch_dh(const CUtensorMap &q, const CUtensorMap &k, const CUtensor
     if (e != cudaSuccess) return e;
     attr_set[dev] = true;
   }
-  const long long units = (long long)p.batch * p.n_kv_heads * ((p.q_span + p.P - 1) / p.P);
+  const long long units = attn_units(p);
   if (units <= 0) return cudaSuccess;
   // Resident units of one stream start about T / (SMs / streams) apart (T a
   // unit's run time), so between two reads of a K/V tile the resident units
@@ -530,13 +613,24 @@ cudaError_t launch_dh(const CUtensorMap &q, const CUtensorMap &k, const CUtensor
   const int n_streams = p.batch * p.n_kv_heads;
   AttnParams pp = p;
   pp.streams_per_group = (int)fmax(1.0, fmin((double)n_streams, floor(sqrt(kReuseBytes / per_stream2))));
-  kern<<<(unsigned)units, kThreads, AttnSmem<DH>::BYTES, stream>>>(q, k, v, pp);
+  const int S = pp.kv_splits > 1 ? pp.kv_splits : 1;
+  if (S > 1 && (!pp.part_o || !pp.part_ml)) return cudaErrorInvalidValue;
+  kern<<<(unsigned)(units * S), kThreads, AttnSmem<DH>::BYTES, stream>>>(q, k, v, pp);
+  if (S > 1) {
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    attn_combine_kernel<CAUSAL><<<dim3(256, (unsigned)units), DH, 0, stream>>>(pp);
+  }
   return cudaGetLastError();
 }
 
 }  // namespace
 
 int attn_positions_per_unit(int group) { return 256 / group; }
+
+long long attn_units(const AttnParams &p) {
+  return (long long)p.batch * p.n_kv_heads * ((p.q_span + p.P - 1) / p.P);
+}
 
 #ifdef CC_ATTN_TRACE
 extern "C" int cc_debug_attn_trace(unsigned long long *out, int n) {

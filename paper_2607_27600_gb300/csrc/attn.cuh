@@ -18,10 +18,17 @@ struct AttnParams {
                             // the memory (rows [row_lo, n) attend [0, i], inference cycle)
   const int32_t *row_lo;    // causal: device [batch], first query slot of each sequence
   int q_span;               // query slots per sequence at most (cap, or the chunk size)
+  int kv_splits;            // > 1: each unit's key tiles split over kv_splits CTAs (few units)
+  float *part_o;            // kv_splits > 1: [unit][split][256 rows][head_dim] unnormalised O
+  float2 *part_ml;          // kv_splits > 1: [unit][split][256 rows] (reference max, row sum)
   unsigned *status;
 };
 
 int attn_positions_per_unit(int group);
+// Work units of a launch (before key splits) and the partial-result floats
+// per unit and split (kv_splits > 1).
+long long attn_units(const AttnParams &p);
+constexpr int kAttnPartRowFloats = 256;   // rows of a unit (times head_dim + 2 floats each)
 // q: 3-D map over Q [rows][Hq][dh], box {64, group, P}; k, v: 3-D maps over
 // the cache [batch*cap][Hkv][dh], box {64, 1, 128}; all 128-byte swizzled.
 cudaError_t launch_attention(const CUtensorMap &q, const CUtensorMap &k, const CUtensorMap &v,

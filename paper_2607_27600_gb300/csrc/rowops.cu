@@ -28,6 +28,22 @@ CC_DEV bool row_in_range(const int32_t *seq_len, const int32_t *row_lo, int cap,
   return !row_lo || i >= row_lo[row / cap];
 }
 
+// Warp w -> its cache row.  With a span (and row_lo), warps cover only the
+// chunk rows: warp w takes slot row_lo[b] + k of sequence b = w / span,
+// k = w % span; otherwise warp w takes row w of the whole cache.
+CC_DEV bool warp_row(const int32_t *seq_len, const int32_t *row_lo, int cap, int rows, int span,
+                     int w, int &row) {
+  if (span > 0 && row_lo) {
+    const int b = w / span;
+    if (b >= rows / cap) return false;
+    const int i = row_lo[b] + (w - b * span), n = seq_len[b];
+    row = b * cap + i;
+    return i >= 0 && i < n && n <= cap;
+  }
+  row = w;
+  return row < rows && row_in_range(seq_len, row_lo, cap, row);
+}
+
 // 8 bf16 of a uint4 -> float
 CC_DEV void unpack8(const uint4 &v, float *f) {
   f[0] = bf16_lo(v.x); f[1] = bf16_hi(v.x); f[2] = bf16_lo(v.y); f[3] = bf16_hi(v.y);
@@ -64,10 +80,12 @@ CC_DEV float row_inv_rms(const void *row, int d, float eps, int lane) {
 template <bool IN_F32>
 __global__ void __launch_bounds__(kWarps * 32)
     rmsnorm_kernel(const void *x, const __nv_bfloat16 *gain, __nv_bfloat16 *out, int d, float eps,
-                   const int32_t *seq_len, const int32_t *row_lo, int cap, int rows, int split) {
+                   const int32_t *seq_len, const int32_t *row_lo, int cap, int rows, int span,
+                   int split) {
   const int lane = threadIdx.x & 31;
-  const int row = blockIdx.x * kWarps + (threadIdx.x >> 5);
-  if (row >= rows || !row_in_range(seq_len, row_lo, cap, row)) return;
+  int row;
+  if (!warp_row(seq_len, row_lo, cap, rows, span, blockIdx.x * kWarps + (threadIdx.x >> 5), row))
+    return;
   const size_t es = IN_F32 ? 4 : 2;
   const void *xr = reinterpret_cast<const uint8_t *>(x) + (size_t)row * d * es;
   const float inv = row_inv_rms<IN_F32>(xr, d, eps, lane);
@@ -98,11 +116,12 @@ __global__ void __launch_bounds__(kWarps * 32)
 // h (fp32) = embed[tokens[row]]
 __global__ void __launch_bounds__(kWarps * 32)
     embed_kernel(const __nv_bfloat16 *embed, const int32_t *tokens, float *h, int d, int vocab,
-                 const int32_t *seq_len, const int32_t *row_lo, int cap, int rows,
+                 const int32_t *seq_len, const int32_t *row_lo, int cap, int rows, int span,
                  unsigned *status) {
   const int lane = threadIdx.x & 31;
-  const int row = blockIdx.x * kWarps + (threadIdx.x >> 5);
-  if (row >= rows || !row_in_range(seq_len, row_lo, cap, row)) return;
+  int row;
+  if (!warp_row(seq_len, row_lo, cap, rows, span, blockIdx.x * kWarps + (threadIdx.x >> 5), row))
+    return;
   int tok = tokens[row];
   if (tok < 0 || tok >= vocab) {
     if (lane == 0) set_status(status, CC_ERR_DEVICE_ARG);
@@ -122,10 +141,11 @@ __global__ void __launch_bounds__(kWarps * 32)
 // the inference cycle).
 __global__ void __launch_bounds__(kWarps * 32)
     store_bf16_kernel(const float *h, __nv_bfloat16 *out, int d, const int32_t *seq_len,
-                      const int32_t *row_lo, int cap, int rows) {
+                      const int32_t *row_lo, int cap, int rows, int span) {
   const int lane = threadIdx.x & 31;
-  const int row = blockIdx.x * kWarps + (threadIdx.x >> 5);
-  if (row >= rows || !row_in_range(seq_len, row_lo, cap, row)) return;
+  int row;
+  if (!warp_row(seq_len, row_lo, cap, rows, span, blockIdx.x * kWarps + (threadIdx.x >> 5), row))
+    return;
   const float *src = h + (size_t)row * d;
   __nv_bfloat16 *dst = out + (size_t)row * d;
   for (int e = lane * 8; e < d; e += 256) {
@@ -275,38 +295,44 @@ __global__ void __launch_bounds__(kWarps * 32)
 
 unsigned blocks_for(int rows) { return (unsigned)((rows + kWarps - 1) / kWarps); }
 
+// warps of a row launch: one per cache row, or batch * span with a span
+int warps_for(int rows, int cap, int span, const int32_t *row_lo) {
+  return span > 0 && row_lo ? rows / cap * span : rows;
+}
+
 }  // namespace
 
 cudaError_t launch_rmsnorm(const void *x, bool x_f32, const void *gain, void *out, int d, float eps,
                            const int32_t *seq_len, int cap, int rows, bool split, cudaStream_t st,
-                           const int32_t *row_lo) {
+                           const int32_t *row_lo, int span) {
   if (rows <= 0) return cudaSuccess;
   auto *g = reinterpret_cast<const __nv_bfloat16 *>(gain);
   auto *o = reinterpret_cast<__nv_bfloat16 *>(out);
+  const unsigned blocks = blocks_for(warps_for(rows, cap, span, row_lo));
   if (x_f32)
-    rmsnorm_kernel<true><<<blocks_for(rows), kWarps * 32, 0, st>>>(x, g, o, d, eps, seq_len, row_lo,
-                                                                    cap, rows, split ? 1 : 0);
+    rmsnorm_kernel<true><<<blocks, kWarps * 32, 0, st>>>(x, g, o, d, eps, seq_len, row_lo, cap, rows,
+                                                          span, split ? 1 : 0);
   else
-    rmsnorm_kernel<false><<<blocks_for(rows), kWarps * 32, 0, st>>>(x, g, o, d, eps, seq_len, row_lo,
-                                                                     cap, rows, split ? 1 : 0);
+    rmsnorm_kernel<false><<<blocks, kWarps * 32, 0, st>>>(x, g, o, d, eps, seq_len, row_lo, cap,
+                                                           rows, span, split ? 1 : 0);
   return cudaGetLastError();
 }
 
 cudaError_t launch_embed(const void *embed, const int32_t *tokens, float *h, int d, int vocab,
                          const int32_t *seq_len, int cap, int rows, unsigned *status,
-                         cudaStream_t st, const int32_t *row_lo) {
+                         cudaStream_t st, const int32_t *row_lo, int span) {
   if (rows <= 0) return cudaSuccess;
-  embed_kernel<<<blocks_for(rows), kWarps * 32, 0, st>>>(
+  embed_kernel<<<blocks_for(warps_for(rows, cap, span, row_lo)), kWarps * 32, 0, st>>>(
       reinterpret_cast<const __nv_bfloat16 *>(embed), tokens, h, d, vocab, seq_len, row_lo, cap,
-      rows, status);
+      rows, span, status);
   return cudaGetLastError();
 }
 
 cudaError_t launch_store_bf16(const float *h, void *out, int d, const int32_t *seq_len,
-                              const int32_t *row_lo, int cap, int rows, cudaStream_t st) {
+                              const int32_t *row_lo, int cap, int rows, cudaStream_t st, int span) {
   if (rows <= 0) return cudaSuccess;
-  store_bf16_kernel<<<blocks_for(rows), kWarps * 32, 0, st>>>(
-      h, reinterpret_cast<__nv_bfloat16 *>(out), d, seq_len, row_lo, cap, rows);
+  store_bf16_kernel<<<blocks_for(warps_for(rows, cap, span, row_lo)), kWarps * 32, 0, st>>>(
+      h, reinterpret_cast<__nv_bfloat16 *>(out), d, seq_len, row_lo, cap, rows, span);
   return cudaGetLastError();
 }
 

@@ -7,17 +7,19 @@ namespace cc {
 // out bf16 [rows][d] = x * gain / sqrt(mean(x^2) + eps); x bf16 or fp32 [rows][d].
 // split: out rows are [hi | lo] bf16 [rows][2d] with hi + lo ~= the fp32 value.
 // Row kernels visit rows b*cap + i with row_lo[b] <= i < seq_len[b] (row_lo
-// null: from 0).
+// null: from 0).  span > 0 (with row_lo): seq_len[b] - row_lo[b] <= span, and
+// the launch has batch * span warps instead of one per cache row.
 cudaError_t launch_rmsnorm(const void *x, bool x_f32, const void *gain, void *out, int d, float eps,
                            const int32_t *seq_len, int cap, int rows, bool split, cudaStream_t st,
-                           const int32_t *row_lo = nullptr);
+                           const int32_t *row_lo = nullptr, int span = 0);
 // h fp32 [rows][d] = embed[tokens[row]]
 cudaError_t launch_embed(const void *embed, const int32_t *tokens, float *h, int d, int vocab,
                          const int32_t *seq_len, int cap, int rows, unsigned *status,
-                         cudaStream_t st, const int32_t *row_lo = nullptr);
+                         cudaStream_t st, const int32_t *row_lo = nullptr, int span = 0);
 // out bf16 [rows][d] = h fp32 (H^(L-1) recorded by the inference cycle)
 cudaError_t launch_store_bf16(const float *h, void *out, int d, const int32_t *seq_len,
-                              const int32_t *row_lo, int cap, int rows, cudaStream_t st);
+                              const int32_t *row_lo, int cap, int rows, cudaStream_t st,
+                              int span = 0);
 // Inference cycle: row_lo = seq_len, row_hi = seq_len + count; the chunk's
 // tokens and positions written into the cache slots [row_lo, row_hi).
 cudaError_t launch_append_prepare(const int32_t *seq_len, const int32_t *count,

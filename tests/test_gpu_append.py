@@ -158,6 +158,21 @@ def test_append_explicit_positions_and_bad_count(cc):
     assert cc.cc_get_status() == cc.CC_OK      # the status word was read and cleared
 
 
+def test_append_short_chunks_over_long_memory_key_splits(cc):
+    """Short ragged chunks (5, 20, 1 tokens) after 1500, 300 and 1999 memory
+    slots: six attention units, so each unit's key tiles are split over
+    several CTAs (4 on a 152-SM GPU) and merged by the combine kernel; the
+    300-slot sequence has fewer tiles than splits (an empty split)."""
+    seq, cap = [1500, 300, 1999], 2048
+    w_np, c_np = _setup(SMALL_GPU, seq, cap, seed=57)
+    r = np.random.default_rng(57)
+    chunks = [r.integers(0, SMALL_GPU.vocab, size=m) for m in (5, 20, 1)]
+    got, status, _ = _gpu_append(cc, SMALL_GPU, w_np, c_np, chunks)
+    assert status == cc.CC_OK
+    want = _oracle_append(SMALL_GPU, w_np, c_np, chunks)
+    _check(SMALL_GPU, got, want, chunks, seq)
+
+
 def test_append_llama_shape_chunk_over_long_memory(cc):
     """Llama-3-8B layer shapes (first two layers), a 1024-token chunk after
     8192 synthetic memory slots: every appended K/V row of both layers,
@@ -243,18 +258,21 @@ def _decode_check(next_tok, best, logits, tol=2e-2):
     assert abs(best - logits[next_tok]) / max(abs(logits[next_tok]), rms) < tol
 
 
-@pytest.mark.parametrize("shape_name", ["small", "llama2"])
+@pytest.mark.parametrize("shape_name", ["small", "small-long", "llama2", "llama2-long"])
 def test_decode_steps_match_oracle(cc, shape_name):
     """Greedy decode steps (teacher-forced with the oracle's tokens so both
-    sides share the history): next tokens, their logits, appended K/V rows."""
+    sides share the history): next tokens, their logits, appended K/V rows.
+    The -long cases attend over enough slots that the attention splits each
+    unit's key tiles across CTAs (4 and 8 splits on a 152-SM GPU)."""
     import paper_2607_27600_gb300 as pkg
-    if shape_name == "small":
-        shape, seq, cap, seed = SMALL_GPU, [50, 20, 33], 64, 54
+    if shape_name.startswith("small"):
+        shape, seed = SMALL_GPU, 54
+        seq, cap = ([50, 20, 33], 64) if shape_name == "small" else ([1500, 300, 1999], 2048)
         w_np = to_np(synth.model_weights(shape, seed, with_kv_proj=True))
         c_np = causal_cache(shape, w_np, seq, cap, seed)
     else:
         shape = ModelShape(**{**synth.configs.LLAMA3_8B.__dict__, "n_layers": 2})
-        seq, cap, seed = [700], 712, 55
+        seq, cap, seed = ([700], 712, 55) if shape_name == "llama2" else ([4000], 4100, 58)
         w = synth.model_weights(shape, seed, device="cuda", with_kv_proj=True)
         c = synth.synthetic_cache(shape, seq, cap, seed, device="cuda")
         w_np, c_np = to_np(w), to_np(c)
