@@ -20,6 +20,7 @@
 #include "attn.cuh"
 #include "compact.cuh"
 #include "gemm.cuh"
+#include "gemv.cuh"
 #include "keyattn.cuh"
 #include "rowops.cuh"
 #include "select.cuh"
@@ -123,7 +124,8 @@ EncodeTiledFn encode_fn() {
 
 // bf16 tensor of `rank` dims (dims[0] contiguous), strides in bytes for dims 1.., 128B swizzle.
 bool make_tmap(CUtensorMap *m, const void *base, int rank, const uint64_t *dims,
-               const uint64_t *strides, const uint32_t *box) {
+               const uint64_t *strides, const uint32_t *box,
+               CUtensorMapSwizzle swizzle = CU_TENSOR_MAP_SWIZZLE_128B) {
   EncodeTiledFn fn = encode_fn();
   if (!fn) return false;
   cuuint64_t d[5], s[4];
@@ -135,7 +137,7 @@ bool make_tmap(CUtensorMap *m, const void *base, int rank, const uint64_t *dims,
     if (i > 0) s[i - 1] = strides[i - 1];
   }
   return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, rank, const_cast<void *>(base), d, s, bx, es,
-            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle,
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
@@ -509,6 +511,82 @@ cc_status check_append_args(const cc_model_cfg *c, const cc_model_weights *w,
   return CC_OK;
 }
 
+// Decode-sized appends (one row per sequence, at most kGemvMaxRows
+// sequences) run the layer products as weight-streaming GEMVs with the
+// RMSNorms fused in: the tile GEMM would cover the weights with a few dozen
+// CTAs for a single row.  Shared memory bounds the staged rows (K of every
+// product, with the largest warp-partial buffer a plan can need).
+bool gemv_decode_ok(const cc_model_cfg *c, int batch, int max_count) {
+  if (max_count != 1 || batch < 1 || batch > kGemvMaxRows) return false;
+  if (c->n_kv_heads * c->head_dim < 16 || c->vocab < 16) return false;   // 16 output rows at least
+  const int ks[3] = {c->d_model, c->n_q_heads * c->head_dim, c->d_ff};
+  for (int K : ks) {
+    if (K < kGemvBoxK) return false;   // boxes no wider than the weights
+    GemvParams p{};
+    p.batch = batch;
+    p.K = K;
+    p.n_seg = 0;
+    if (K % 8 || !gemv_plan(p, 1)) return false;
+  }
+  return true;
+}
+
+// One GEMV launch: up to three weight matrices (segments) over the same rows.
+struct GemvCall {
+  GemvLaunch l{};
+  const void *w[kGemvMaxSegs][2] = {};
+  void add(const void *w0, const void *w1, const void *bias, void *out, int ldo, int n, int epi) {
+    GemvSeg &sg = l.p.seg[l.p.n_seg];
+    sg = GemvSeg{};
+    sg.bias = reinterpret_cast<const __nv_bfloat16 *>(bias);
+    sg.out = out;
+    sg.ldo = ldo;
+    sg.N = n;
+    sg.epi = epi;
+    w[l.p.n_seg][0] = w0;
+    w[l.p.n_seg][1] = w1;
+    ++l.p.n_seg;
+  }
+};
+
+GemvCall gemv_call(const cc_model_cfg *c, const cc_kv_cache *kv, const int32_t *lo,
+                   const int32_t *hi, unsigned *status, const void *x, int ldx, int K,
+                   const void *norm_gain) {
+  GemvCall g;
+  GemvParams &p = g.l.p;
+  p.batch = kv->batch;
+  p.cap = kv->cap;
+  p.row_lo = lo;
+  p.row_hi = hi;
+  p.pos = kv->pos;
+  p.head_dim = c->head_dim;
+  p.eps = c->rms_eps;
+  p.status = status;
+  p.x = x;
+  p.ldx = ldx;
+  p.K = K;
+  p.norm_gain = reinterpret_cast<const __nv_bfloat16 *>(norm_gain);
+  rope_turns(c, p.turns);
+  return g;
+}
+
+cc_status run_gemv(GemvCall &g, int kind, int sms, cudaStream_t st) {
+  GemvParams &p = g.l.p;
+  if (!gemv_plan(p, sms)) return CC_ERR_UNSUPPORTED;
+  for (int s = 0; s < p.n_seg; ++s) {
+    const uint64_t dims[2] = {(uint64_t)p.K, (uint64_t)p.seg[s].N};
+    const uint64_t strides[1] = {(uint64_t)p.K * 2};
+    const uint32_t box[2] = {(uint32_t)kGemvBoxK, 8};
+    for (int j = 0; j < 2; ++j)
+      if (g.w[s][j] && !make_tmap(&g.l.w[s][j], g.w[s][j], 2, dims, strides, box,
+                                  CU_TENSOR_MAP_SWIZZLE_NONE))
+        return tmap_fail();
+  }
+  TimedScope t(kind, st);
+  CC_TRY(launch_gemv(g.l, st));
+  return CC_OK;
+}
+
 cc_status run_append(const cc_model_cfg *c, const cc_model_weights *w, const cc_kv_cache *kv,
                      const int32_t *tokens_in, const int32_t *pos_in, const int32_t *count,
                      int max_count, void *ws, size_t ws_bytes, void *stream) {
@@ -533,6 +611,7 @@ cc_status run_append(const cc_model_cfg *c, const cc_model_weights *w, const cc_
   AttnPartials parts;
   parts.o = reinterpret_cast<float *>(wsb + L.part_o);
   parts.ml = reinterpret_cast<float2 *>(wsb + L.part_ml);
+  const bool use_gemv = gemv_decode_ok(c, batch, max_count);
 
   {
     TimedScope t(CC_KERNEL_APPEND, st);
@@ -550,14 +629,20 @@ cc_status run_append(const cc_model_cfg *c, const cc_model_weights *w, const cc_
       TimedScope t(CC_KERNEL_APPEND, st);
       CC_TRY(launch_store_bf16(h, kv->h_last, d, hi, lo, cap, rows, st, max_count));
     }
-    {
+    if (use_gemv) {   // RMSNorm fused; q, k and v in one launch
+      GemvCall g = gemv_call(c, kv, lo, hi, status, h, d, d, lw.attn_norm);
+      g.add(lw.wq, nullptr, lw.bq, q, qd, qd, GEMV_ROPE);
+      g.add(lw.wk, nullptr, lw.bk, kv->k[l], kvd, kvd, GEMV_ROPE);
+      g.add(lw.wv, nullptr, lw.bv, kv->v[l], kvd, kvd, GEMV_BF16);
+      if ((s = run_gemv(g, CC_KERNEL_GEMM_QKV, dev->sms, st)) != CC_OK) return s;
+    } else {
       TimedScope t(CC_KERNEL_RMSNORM, st);
       CC_TRY(launch_rmsnorm(h, true, lw.attn_norm, xn, d, c->rms_eps, hi, cap, rows, false, st, lo,
                             max_count));
     }
     // q = RoPE(xn Wq^T + bq) into the workspace; k = RoPE(xn Wk^T + bk) and
     // v = xn Wv^T + bv straight into the cache slots of the chunk
-    if (qkv_fusable(c)) {   // one GEMM over [Wq; Wk; Wv]
+    if (!use_gemv && qkv_fusable(c)) {   // one GEMM over [Wq; Wk; Wv]
       Gemm g;
       if ((s = gemm_setup_qkv(g, xn, c, lw, batch, cap, hi, status, used)) != CC_OK) return s;
       g.p.row_lo = lo;
@@ -572,7 +657,7 @@ cc_status run_append(const cc_model_cfg *c, const cc_model_weights *w, const cc_
                            {lw.wk, lw.bk, kv->k[l], kvd, EPI_QROPE, CC_KERNEL_GEMM_KV},
                            {lw.wv, lw.bv, kv->v[l], kvd, EPI_BF16, CC_KERNEL_GEMM_KV}};
     for (const Proj &pj : projs) {
-      if (qkv_fusable(c)) break;
+      if (use_gemv || qkv_fusable(c)) break;
       Gemm g;
       if ((s = gemm_setup(g, pj.epi, xn, d, pj.w, nullptr, pj.n, batch, cap, hi, status, false,
                           used)) != CC_OK)
@@ -591,6 +676,18 @@ cc_status run_append(const cc_model_cfg *c, const cc_model_weights *w, const cc_
                            max_count, &parts, dev->sms)) != CC_OK)
       return s;
     // h += o Wo^T; xn = RMSNorm(h); act = SwiGLU; h += act Wd^T
+    if (use_gemv) {
+      GemvCall go = gemv_call(c, kv, lo, hi, status, o, qd, qd, nullptr);
+      go.add(lw.wo, nullptr, nullptr, h, d, d, GEMV_RESID_F32);
+      if ((s = run_gemv(go, CC_KERNEL_GEMM_OPROJ, dev->sms, st)) != CC_OK) return s;
+      GemvCall gu = gemv_call(c, kv, lo, hi, status, h, d, d, lw.mlp_norm);
+      gu.add(lw.w_gate, lw.w_up, nullptr, act, f, f, GEMV_SWIGLU);
+      if ((s = run_gemv(gu, CC_KERNEL_GEMM_GATEUP, dev->sms, st)) != CC_OK) return s;
+      GemvCall gd = gemv_call(c, kv, lo, hi, status, act, f, f, nullptr);
+      gd.add(lw.w_down, nullptr, nullptr, h, d, d, GEMV_RESID_F32);
+      if ((s = run_gemv(gd, CC_KERNEL_GEMM_DOWN, dev->sms, st)) != CC_OK) return s;
+      continue;
+    }
     Gemm go;
     if ((s = gemm_setup(go, EPI_RESID_F32, o, qd, lw.wo, nullptr, d, batch, cap, hi, status,
                         false, used)) != CC_OK)
@@ -964,13 +1061,17 @@ cc_status cc_score_h2o(const cc_kv_cache *kv, int32_t recent, float *scores, voi
 }
 
 // ---- decode step (greedy): append one token each, LM head, argmax -------------
+constexpr int kDecodeMinParts = 1024;   // argmax pairs per sequence the workspace holds at least
+
 size_t decode_part_offset(const cc_model_cfg *c, int batch, int cap) {
   return align256(append_layout(c, batch, cap).total);
 }
 
 size_t cc_decode_workspace_size(const cc_model_cfg *cfg, int32_t batch, int32_t cap) {
   if (check_cfg(cfg) != CC_OK || batch < 1 || cap < 1) return 0;
-  const size_t n_tiles = ((size_t)cfg->vocab + 127) / 128;   // column tiles, either width
+  // (max, column) pairs per sequence: one per LM-head column tile of either
+  // width, or one per CTA of the weight-streaming LM head
+  const size_t n_tiles = std::max<size_t>(((size_t)cfg->vocab + 127) / 128, kDecodeMinParts);
   return decode_part_offset(cfg, batch, cap) + align256((size_t)batch * n_tiles * 8);
 }
 
@@ -995,6 +1096,16 @@ cc_status cc_decode_step(const cc_model_cfg *cfg, const cc_model_weights *w,
   float *h = reinterpret_cast<float *>(wsb + L.s.h);
   int32_t *lo = reinterpret_cast<int32_t *>(wsb + L.lo), *hi = reinterpret_cast<int32_t *>(wsb + L.hi);
   float2 *part = reinterpret_cast<float2 *>(wsb + decode_part_offset(cfg, batch, cap));
+  if (gemv_decode_ok(cfg, batch, 1) && dev->sms <= kDecodeMinParts) {
+    // final norm fused; one (max, first column) pair per CTA
+    GemvCall g = gemv_call(cfg, cache, lo, hi, dev->status, h, d, d, w->final_norm);
+    g.add(w->lm_head, nullptr, nullptr, nullptr, 0, cfg->vocab, GEMV_ARGMAX);
+    g.l.p.part = part;
+    if ((s = run_gemv(g, CC_KERNEL_GEMM_LMHEAD, dev->sms, st)) != CC_OK) return s;
+    TimedScope t(CC_KERNEL_APPEND, st);
+    CC_TRY(launch_argmax_combine(part, g.l.p.part_ld, lo, hi, batch, next_tokens, next_logit, st));
+    return CC_OK;
+  }
   {
     TimedScope t(CC_KERNEL_RMSNORM, st);
     CC_TRY(launch_rmsnorm(h, true, w->final_norm, xn, d, cfg->rms_eps, hi, cap, batch * cap, false,

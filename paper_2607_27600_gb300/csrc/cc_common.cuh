@@ -283,6 +283,19 @@ CC_DEV uint32_t pack_bf16x2(float lo, float hi) {
 CC_DEV float bf16_lo(uint32_t v) { return __uint_as_float(v << 16); }
 CC_DEV float bf16_hi(uint32_t v) { return __uint_as_float(v & 0xFFFF0000u); }
 
+CC_DEV float silu(float x) { return x / (1.0f + __expf(-x)); }
+
+// cos/sin of pos * inv_freq, with the angle reduced exactly: turns is
+// inv_freq / (2 pi) in 0.64 fixed point, so pos * turns mod 2^64 is the
+// fractional number of turns; its top 32 bits, read as a signed fraction of
+// a turn, give the angle in [-pi, pi).
+CC_DEV void rope_cs(uint32_t pos, unsigned long long turns, float &c, float &s) {
+  unsigned long long frac = (unsigned long long)pos * turns;
+  int32_t t32 = (int32_t)(frac >> 32);
+  float ang = (float)t32 * 1.4629180792671596e-09f;   // 2 pi / 2^32
+  __sincosf(ang, &s, &c);
+}
+
 CC_DEV float warp_sum(float v) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, o);

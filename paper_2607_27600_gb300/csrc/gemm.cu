@@ -30,19 +30,6 @@ constexpr int kMaxBatch = 1024;
 constexpr size_t kSmemBytes = 1024 /*align slack*/ + ST * (A_BYTES + B_BYTES) + 256 +
                               (kMaxBatch + 1) * sizeof(int);
 
-CC_DEV float silu(float x) { return x / (1.0f + __expf(-x)); }
-
-// cos/sin of pos * inv_freq, with the angle reduced exactly: turns is
-// inv_freq / (2 pi) in 0.64 fixed point, so pos * turns mod 2^64 is the
-// fractional number of turns; its top 32 bits, read as a signed fraction of
-// a turn, give the angle in [-pi, pi).
-CC_DEV void rope_cs(uint32_t pos, unsigned long long turns, float &c, float &s) {
-  unsigned long long frac = (unsigned long long)pos * turns;
-  int32_t t32 = (int32_t)(frac >> 32);
-  float ang = (float)t32 * 1.4629180792671596e-09f;   // 2 pi / 2^32
-  __sincosf(ang, &s, &c);
-}
-
 // RoPE'd bf16 store of one accumulator tile row: destination columns
 // [col0, col0 + TBN) of out (row stride ldo, n_dest columns in all), each tile
 // holding TBN / head_dim whole heads; rotate-half pairs (k, k + dh/2); the
