@@ -406,6 +406,15 @@ int attn_key_splits(long long units, int cap, int sms) {
   return s >= 2 ? (int)s : 1;
 }
 
+// Key splits of the decode attention (one query row per unit): up to one
+// CTA per SM in all, each split at least two chunks of 128 keys.
+int attn_decode_splits(long long units, int cap, int sms) {
+  const long long by_keys = std::max(1LL, ((long long)cap + 255) / 256);
+  const long long s = std::min({std::max(1LL, (long long)sms / units),
+                                std::max(1LL, (long long)kAttnMaxSplitSlots / units), by_keys});
+  return (int)s;
+}
+
 // out: [R][Hq*dh] bf16, or with split [R][2*Hq*dh] = [hi | lo] per row.
 // Counter-causal attention over rows [0, seq_len); with row_lo, the causal
 // memory-augmented attention of the inference cycle over rows
@@ -449,6 +458,19 @@ cc_status run_attention(const cc_model_cfg *c, const void *q, const void *k, con
   p.causal = row_lo ? 1 : 0;
   p.row_lo = row_lo;
   p.q_span = row_lo ? q_span : cap;
+  const long long units = attn_units(p);
+  if (row_lo && q_span == 1 && G <= kDecMaxG && parts && parts->o && parts->ml &&
+      units <= kAttnMaxSplitSlots) {   // one query row per sequence: the decode kernel
+    p.kv_splits = attn_decode_splits(units, cap, sms);
+    p.part_o = parts->o;
+    p.part_ml = parts->ml;
+    p.q = reinterpret_cast<const __nv_bfloat16 *>(q);
+    p.k = reinterpret_cast<const __nv_bfloat16 *>(k);
+    p.v = reinterpret_cast<const __nv_bfloat16 *>(v);
+    TimedScope t(CC_KERNEL_ATTN_CAUSAL, st);
+    CC_TRY(launch_attention_decode(p, st));
+    return CC_OK;
+  }
   if (parts && parts->o && parts->ml) {
     p.kv_splits = attn_key_splits(attn_units(p), cap, sms);
     p.part_o = parts->o;

@@ -550,9 +550,16 @@ __global__ void __launch_bounds__(kThreads, 1)
 // Key splits: out = sum_s 2^((m_s - m*) c) O_s / sum_s 2^((m_s - m*) c) l_s
 // per row (m* the largest reference max, c = log2(e)/sqrt(dh)), splits in
 // order; bf16 (and lo) stores as the kernel's own epilogue.  Block = one row
-// of one unit, a thread per head_dim element.
+// of one unit, a thread per head_dim element: the splits' (max, sum) pairs
+// are loaded in parallel and weighted once in shared memory, then every
+// thread sums its element over the splits with eight loads in flight.
+constexpr int kCombineMaxSplits = 256;
+
 template <bool CAUSAL>
 __global__ void attn_combine_kernel(const __grid_constant__ AttnParams p) {
+  __shared__ float wgt[kCombineMaxSplits];
+  __shared__ float lsum[kCombineMaxSplits];
+  __shared__ float red[4];
   const int R = blockIdx.x, unit_id = blockIdx.y, d = threadIdx.x;
   const UnitInfo u = decode_unit(p, unit_id, CAUSAL);
   const int G = p.group;
@@ -561,20 +568,35 @@ __global__ void attn_combine_kernel(const __grid_constant__ AttnParams p) {
   if (pos > u.p_last) return;
   const int S = p.kv_splits;
   const float c = p.scale_log2;
+  const size_t base = (size_t)unit_id * S * 256 + R;   // split s's row: base + s * 256
+  // reference max over the splits that saw keys
   float m = -INFINITY;
-  for (int s = 0; s < S; ++s) {
-    const float2 ml = p.part_ml[((size_t)unit_id * S + s) * 256 + R];
+  for (int s = d; s < S; s += blockDim.x) {
+    const float2 ml = p.part_ml[base + (size_t)s * 256];
+    wgt[s] = ml.x;
+    lsum[s] = ml.y;
     if (ml.y > 0.f) m = fmaxf(m, ml.x);
   }
-  float o = 0.f, l = 0.f;
-  for (int s = 0; s < S; ++s) {
-    const size_t slot = ((size_t)unit_id * S + s) * 256 + R;
-    const float2 ml = p.part_ml[slot];
-    if (!(ml.y > 0.f)) continue;
-    const float wgt = exp2f((ml.x - m) * c);
-    l += wgt * ml.y;
-    o += wgt * p.part_o[slot * p.head_dim + d];
+  m = warp_max(m);
+  if ((d & 31) == 0) red[d >> 5] = m;
+  __syncthreads();
+  m = red[0];
+  for (int w = 1; w < (int)(blockDim.x >> 5); ++w) m = fmaxf(m, red[w]);
+  for (int s = d; s < S; s += blockDim.x)
+    wgt[s] = lsum[s] > 0.f ? exp2f((wgt[s] - m) * c) : 0.f;
+  __syncthreads();
+  float l = 0.f;
+  for (int s = 0; s < S; ++s) l += wgt[s] * lsum[s];
+  float o = 0.f;
+  int s = 0;
+  for (; s + 8 <= S; s += 8) {
+    float v[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) v[k] = p.part_o[(base + (size_t)(s + k) * 256) * p.head_dim + d];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) o += wgt[s + k] * v[k];
   }
+  for (; s < S; ++s) o += wgt[s] * p.part_o[(base + (size_t)s * 256) * p.head_dim + d];
   const float v = l > 0.f ? o / l : 0.f;
   __nv_bfloat16 *dst = p.out + ((size_t)u.b * p.cap + pos) * p.out_ld +
                        (size_t)(u.g * G + hl) * p.head_dim + d;
@@ -624,6 +646,231 @@ cudaError_t launch_dh(const CUtensorMap &q, const CUtensorMap &k, const CUtensor
   return cudaGetLastError();
 }
 
+// ---------------------------------------------------------------------------
+// Decode attention: one query row per sequence (q_span == 1), at most
+// kDecMaxG query heads per KV head.  For a single query row the products are
+// a few hundred FMAs per key, so CUDA cores in fp32 suffice and the K/V bytes
+// bound the time: CTA = (unit, key split); chunks of 128 keys are copied to
+// shared memory with cp.async (double-buffered; K rows padded by 16 bytes so
+// the score pass's column reads are conflict-free); per chunk the scores, an
+// online softmax (log2 domain, reference max in raw units as the tile kernel
+// keeps it) and P V; each CTA writes the partial (O, max, sum) rows that
+// attn_combine_kernel merges.
+// ---------------------------------------------------------------------------
+constexpr int kDecChunk = 128;
+constexpr int kDecThreads = 256;   // = 2 * kDecChunk: the score pass takes a key and half its dims
+
+template <int DH>
+struct DecSmem {
+  static constexpr int K_ROW = DH * 2 + 16;
+  static constexpr int V_ROW = DH * 2;
+  static constexpr int K_BYTES = kDecChunk * K_ROW;
+  static constexpr int V_BYTES = kDecChunk * V_ROW;
+  static constexpr int BUF = K_BYTES + V_BYTES;
+  static constexpr int OFF_Q = 2 * BUF;                                 // fp32 [G][DH]
+  static constexpr int OFF_S = OFF_Q + kDecMaxG * DH * 4;               // fp32 [2][G][chunk]
+  static constexpr int OFF_P = OFF_S + 2 * kDecMaxG * kDecChunk * 4;    // fp32 [G][chunk]
+  static constexpr int OFF_F = OFF_P + kDecMaxG * kDecChunk * 4;        // fp32 [G]
+  static constexpr int BYTES = OFF_F + kDecMaxG * 4;
+};
+
+CC_DEV void cp_async16(void *dst, const void *src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)), "l"(src)
+               : "memory");
+}
+CC_DEV void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+CC_DEV void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
+template <int DH>
+__global__ void __launch_bounds__(kDecThreads) attn_decode_kernel(const __grid_constant__ AttnParams p) {
+  using L = DecSmem<DH>;
+  extern __shared__ __align__(128) uint8_t smem[];
+  const int S = p.kv_splits;
+  const int unit_id = blockIdx.x / S, split = blockIdx.x - unit_id * S;
+  const UnitInfo u = decode_unit(p, unit_id, true);
+  if (u.bad) {
+    if (threadIdx.x == 0) set_status(p.status, CC_ERR_DEVICE_ARG);
+    return;
+  }
+  if (!u.valid) return;
+  const int G = p.group, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int pos = u.p0;            // the unit's one query slot
+  const int n_keys = pos + 1;      // causal: keys 0 .. pos
+  const int nch = (n_keys + kDecChunk - 1) / kDecChunk;
+  const int c_lo = split * nch / S, c_hi = (split + 1) * nch / S;
+  const size_t slot = ((size_t)unit_id * S + split) * 256;
+  if (c_lo >= c_hi) {   // nothing for this split: an empty partial
+    if (tid < G) p.part_ml[slot + tid] = make_float2(-INFINITY, 0.f);
+    return;
+  }
+  float *qs = reinterpret_cast<float *>(smem + L::OFF_Q);
+  float *sbuf = reinterpret_cast<float *>(smem + L::OFF_S);
+  float *pbuf = reinterpret_cast<float *>(smem + L::OFF_P);
+  float *fbuf = reinterpret_cast<float *>(smem + L::OFF_F);
+  const size_t row_base = (size_t)u.b * p.cap;
+  const int Hkv = p.n_kv_heads;
+
+  auto issue = [&](int c, int buf) {
+    uint8_t *kb = smem + buf * L::BUF, *vb = kb + L::K_BYTES;
+    constexpr int PIECES = DH * 2 / 16;   // 16-byte pieces of a row
+    for (int i = tid; i < kDecChunk * PIECES; i += kDecThreads) {
+      const int r = i / PIECES, e = i - r * PIECES;
+      const int j = c * kDecChunk + r;
+      uint8_t *kd = kb + r * L::K_ROW + e * 16, *vd = vb + r * L::V_ROW + e * 16;
+      if (j < n_keys) {
+        const size_t off = ((row_base + j) * Hkv + u.g) * (size_t)DH + e * 8;
+        cp_async16(kd, p.k + off);
+        cp_async16(vd, p.v + off);
+      } else {   // past the last key: zeros (P is 0 there, V must be finite)
+        *reinterpret_cast<uint4 *>(kd) = make_uint4(0, 0, 0, 0);
+        *reinterpret_cast<uint4 *>(vd) = make_uint4(0, 0, 0, 0);
+      }
+    }
+    cp_async_commit();
+  };
+  issue(c_lo, 0);
+  for (int i = tid; i < G * DH; i += kDecThreads) {
+    const int h = i / DH, d = i - h * DH;
+    qs[i] = __bfloat162float(
+        p.q[(row_base + pos) * (size_t)p.n_q_heads * DH + (size_t)(u.g * G + h) * DH + d]);
+  }
+
+  constexpr int DPT = DH / 32;   // P V: warp h < G owns head h, lane the dims lane*DPT..
+  float m_h = -INFINITY, l_h = 0.f;
+  float o[DPT];
+#pragma unroll
+  for (int i = 0; i < DPT; ++i) o[i] = 0.f;
+  const float c2 = p.scale_log2;
+  for (int c = c_lo; c < c_hi; ++c) {
+    const int buf = (c - c_lo) & 1;
+    if (c + 1 < c_hi) {
+      issue(c + 1, buf ^ 1);
+      cp_async_wait<1>();
+    } else {
+      cp_async_wait<0>();
+    }
+    __syncthreads();
+    const uint8_t *kb = smem + buf * L::BUF, *vb = kb + L::K_BYTES;
+    {   // scores: thread = (key j, half of the dims)
+      const int j = tid & (kDecChunk - 1), half = tid / kDecChunk;
+      const uint8_t *kr = kb + j * L::K_ROW + half * DH;
+      float sc[kDecMaxG];
+#pragma unroll
+      for (int h = 0; h < kDecMaxG; ++h) sc[h] = 0.f;
+#pragma unroll
+      for (int d8 = 0; d8 < DH / 16; ++d8) {
+        const uint4 kv = *reinterpret_cast<const uint4 *>(kr + d8 * 16);
+        const float kf[8] = {bf16_lo(kv.x), bf16_hi(kv.x), bf16_lo(kv.y), bf16_hi(kv.y),
+                             bf16_lo(kv.z), bf16_hi(kv.z), bf16_lo(kv.w), bf16_hi(kv.w)};
+        const int d0 = half * (DH / 2) + d8 * 8;
+#pragma unroll
+        for (int h = 0; h < kDecMaxG; ++h) {
+          if (h < G) {
+            const float4 qa = *reinterpret_cast<const float4 *>(qs + h * DH + d0);
+            const float4 qb = *reinterpret_cast<const float4 *>(qs + h * DH + d0 + 4);
+            float a = sc[h];
+            a = fmaf(kf[0], qa.x, a); a = fmaf(kf[1], qa.y, a);
+            a = fmaf(kf[2], qa.z, a); a = fmaf(kf[3], qa.w, a);
+            a = fmaf(kf[4], qb.x, a); a = fmaf(kf[5], qb.y, a);
+            a = fmaf(kf[6], qb.z, a); a = fmaf(kf[7], qb.w, a);
+            sc[h] = a;
+          }
+        }
+      }
+#pragma unroll
+      for (int h = 0; h < kDecMaxG; ++h)
+        if (h < G) sbuf[(half * kDecMaxG + h) * kDecChunk + j] = sc[h];
+    }
+    __syncthreads();
+    if (warp < G) {   // online softmax of head h = warp over the chunk
+      const int h = warp;
+      float sv[kDecChunk / 32];
+      float cm = -INFINITY;
+#pragma unroll
+      for (int q = 0; q < kDecChunk / 32; ++q) {
+        const int j = lane + 32 * q;
+        float v = sbuf[h * kDecChunk + j] + sbuf[(kDecMaxG + h) * kDecChunk + j];
+        if (c * kDecChunk + j >= n_keys) v = -INFINITY;
+        sv[q] = v;
+        cm = fmaxf(cm, v);
+      }
+      cm = warp_max(cm);
+      const float m_new = fmaxf(m_h, cm);
+      const bool any = m_new != -INFINITY;
+      const float factor = any ? fast_exp2((m_h - m_new) * c2) : 1.f;   // 0 when m_h = -inf
+      float ls = 0.f;
+#pragma unroll
+      for (int q = 0; q < kDecChunk / 32; ++q) {
+        const float pv = any ? fast_exp2((sv[q] - m_new) * c2) : 0.f;
+        pbuf[h * kDecChunk + lane + 32 * q] = pv;
+        ls += pv;
+      }
+      ls = warp_sum(ls);
+      l_h = l_h * factor + ls;
+      m_h = m_new;
+      if (lane == 0) fbuf[h] = factor;
+    }
+    __syncthreads();
+    if (warp < G) {   // O = O * factor + P V
+      const int h = warp;
+      const float f = fbuf[h];
+#pragma unroll
+      for (int i = 0; i < DPT; ++i) o[i] *= f;
+      const float *ph = pbuf + h * kDecChunk;
+#pragma unroll 4
+      for (int j = 0; j < kDecChunk; ++j) {
+        const float pj = ph[j];
+        const uint8_t *vr = vb + j * L::V_ROW + lane * DPT * 2;
+        if constexpr (DPT == 4) {
+          const uint2 v = *reinterpret_cast<const uint2 *>(vr);
+          o[0] = fmaf(pj, bf16_lo(v.x), o[0]);
+          o[1] = fmaf(pj, bf16_hi(v.x), o[1]);
+          o[2] = fmaf(pj, bf16_lo(v.y), o[2]);
+          o[3] = fmaf(pj, bf16_hi(v.y), o[3]);
+        } else {
+          const uint32_t v = *reinterpret_cast<const uint32_t *>(vr);
+          o[0] = fmaf(pj, bf16_lo(v), o[0]);
+          o[1] = fmaf(pj, bf16_hi(v), o[1]);
+        }
+      }
+    }
+    __syncthreads();
+  }
+  if (warp < G) {   // partial row R = head warp of the unit's one position
+    float *po = p.part_o + (slot + warp) * DH + lane * DPT;
+#pragma unroll
+    for (int i = 0; i < DPT; ++i) po[i] = o[i];
+    if (lane == 0) p.part_ml[slot + warp] = make_float2(m_h, l_h);
+  }
+}
+
+template <int DH>
+cudaError_t launch_decode_dh(const AttnParams &p, cudaStream_t stream) {
+  static bool attr_set[64] = {};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev < 64 && !attr_set[dev]) {
+    cudaError_t e = cudaFuncSetAttribute(attn_decode_kernel<DH>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         DecSmem<DH>::BYTES);
+    if (e != cudaSuccess) return e;
+    attr_set[dev] = true;
+  }
+  const long long units = attn_units(p);
+  if (units <= 0) return cudaSuccess;
+  AttnParams pp = p;
+  pp.streams_per_group = p.batch * p.n_kv_heads;
+  attn_decode_kernel<DH><<<(unsigned)(units * pp.kv_splits), kDecThreads, DecSmem<DH>::BYTES,
+                           stream>>>(pp);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  attn_combine_kernel<true><<<dim3((unsigned)p.group, (unsigned)units), DH, 0, stream>>>(pp);
+  return cudaGetLastError();
+}
+
 }  // namespace
 
 int attn_positions_per_unit(int group) { return 256 / group; }
@@ -637,6 +884,15 @@ extern "C" int cc_debug_attn_trace(unsigned long long *out, int n) {
   return (int)cudaMemcpyFromSymbol(out, g_attn_trace, sizeof(unsigned long long) * (n < 1024 ? n : 1024));
 }
 #endif
+
+cudaError_t launch_attention_decode(const AttnParams &p, cudaStream_t stream) {
+  if (!p.causal || p.q_span != 1 || p.group > kDecMaxG || p.kv_splits < 1 || !p.q || !p.k ||
+      !p.v || !p.part_o || !p.part_ml)
+    return cudaErrorInvalidValue;
+  if (p.head_dim == 128) return launch_decode_dh<128>(p, stream);
+  if (p.head_dim == 64) return launch_decode_dh<64>(p, stream);
+  return cudaErrorInvalidValue;
+}
 
 cudaError_t launch_attention(const CUtensorMap &q, const CUtensorMap &k, const CUtensorMap &v,
                              const AttnParams &p, cudaStream_t stream) {

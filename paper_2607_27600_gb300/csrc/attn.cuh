@@ -21,8 +21,11 @@ struct AttnParams {
   int kv_splits;            // > 1: each unit's key tiles split over kv_splits CTAs (few units)
   float *part_o;            // kv_splits > 1: [unit][split][256 rows][head_dim] unnormalised O
   float2 *part_ml;          // kv_splits > 1: [unit][split][256 rows] (reference max, row sum)
+  const __nv_bfloat16 *q, *k, *v;   // decode kernel: Q [rows][Hq][dh], cache [rows][Hkv][dh]
   unsigned *status;
 };
+
+constexpr int kDecMaxG = 8;   // query heads per KV head the decode kernel takes at most
 
 int attn_positions_per_unit(int group);
 // Work units of a launch (before key splits) and the partial-result floats
@@ -33,5 +36,9 @@ constexpr int kAttnPartRowFloats = 256;   // rows of a unit (times head_dim + 2 
 // the cache [batch*cap][Hkv][dh], box {64, 1, 128}; all 128-byte swizzled.
 cudaError_t launch_attention(const CUtensorMap &q, const CUtensorMap &k, const CUtensorMap &v,
                              const AttnParams &p, cudaStream_t stream);
+// Causal attention of one query row per sequence (q_span == 1, group <=
+// kDecMaxG): CUDA-core kernel over kv_splits (>= 1) key ranges per unit, then
+// the combine; needs q, k, v, part_o and part_ml.
+cudaError_t launch_attention_decode(const AttnParams &p, cudaStream_t stream);
 
 }  // namespace cc
