@@ -560,6 +560,8 @@ __global__ void attn_combine_kernel(const __grid_constant__ AttnParams p) {
   __shared__ float wgt[kCombineMaxSplits];
   __shared__ float lsum[kCombineMaxSplits];
   __shared__ float red[4];
+  pdl_trigger();
+  pdl_wait();
   const int R = blockIdx.x, unit_id = blockIdx.y, d = threadIdx.x;
   const UnitInfo u = decode_unit(p, unit_id, CAUSAL);
   const int G = p.group;
@@ -688,6 +690,8 @@ template <int DH>
 __global__ void __launch_bounds__(kDecThreads) attn_decode_kernel(const __grid_constant__ AttnParams p) {
   using L = DecSmem<DH>;
   extern __shared__ __align__(128) uint8_t smem[];
+  pdl_trigger();   // the combine may launch (it waits for this grid before reading)
+  pdl_wait();      // q and the new token's K/V come from the projection just before
   const int S = p.kv_splits;
   const int unit_id = blockIdx.x / S, split = blockIdx.x - unit_id * S;
   const UnitInfo u = decode_unit(p, unit_id, true);
@@ -863,12 +867,11 @@ cudaError_t launch_decode_dh(const AttnParams &p, cudaStream_t stream) {
   if (units <= 0) return cudaSuccess;
   AttnParams pp = p;
   pp.streams_per_group = p.batch * p.n_kv_heads;
-  attn_decode_kernel<DH><<<(unsigned)(units * pp.kv_splits), kDecThreads, DecSmem<DH>::BYTES,
-                           stream>>>(pp);
-  cudaError_t e = cudaGetLastError();
+  cudaError_t e = launch_pdl(attn_decode_kernel<DH>, dim3((unsigned)(units * pp.kv_splits)),
+                             dim3(kDecThreads), DecSmem<DH>::BYTES, stream, pp);
   if (e != cudaSuccess) return e;
-  attn_combine_kernel<true><<<dim3((unsigned)p.group, (unsigned)units), DH, 0, stream>>>(pp);
-  return cudaGetLastError();
+  return launch_pdl(attn_combine_kernel<true>, dim3((unsigned)p.group, (unsigned)units), dim3(DH),
+                    0, stream, pp);
 }
 
 }  // namespace

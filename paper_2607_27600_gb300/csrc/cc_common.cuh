@@ -8,6 +8,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <utility>
+
 #include "../../include/cc.h"
 
 #define CC_DEV __device__ __forceinline__
@@ -126,6 +128,16 @@ CC_DEV uint64_t make_policy_evict_first() {
   return p;
 }
 // Barrier among `threads` threads (a multiple of 32) of the CTA, id 1..15.
+// Programmatic dependent launch: a kernel launched with the programmatic
+// stream-serialization attribute may start before its predecessor in the
+// stream has finished.  pdl_trigger: this CTA lets the next such kernel
+// launch (it launches once every CTA of this grid has triggered or exited);
+// pdl_wait: blocks until the predecessor grid has completed and its writes
+// are visible (a no-op for a kernel launched without the attribute).  A
+// kernel touches nothing its predecessors write before pdl_wait.
+CC_DEV void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+CC_DEV void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 CC_DEV void named_barrier_sync(int id, int threads) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(threads) : "memory");
 }
@@ -272,6 +284,24 @@ CC_DEV void tmem_st32(uint32_t taddr, const uint32_t (&r)[32]) {
       : "memory");
 }
 CC_DEV void tmem_st_wait() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
+
+// Launches kern<<<grid, block, smem, st>>>(args...) with programmatic stream
+// serialization allowed (see pdl_wait).
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                              cudaStream_t st, Args &&...args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, std::forward<Args>(args)...);
+}
 
 // ---------------------------------------------------------------------------
 // small numeric helpers

@@ -92,6 +92,10 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
   const int g_begin = (int)((long long)blockIdx.x * p.n_groups / gridDim.x);
   const int g_end = (int)((long long)(blockIdx.x + 1) * p.n_groups / gridDim.x);
 
+  // The next product may launch now: its producer streams its own weights
+  // while this grid finishes (every CTA here holds one SM's shared memory,
+  // so a waiting dependent never takes an SM this grid still needs).
+  pdl_trigger();
   if (threadIdx.x == 0) {
     for (int s = 0; s < NS; ++s) {
       mbar_init(&full[s], 1);
@@ -104,15 +108,11 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
     abort_s = 0;
     fence_barrier_init();
   }
-  if (threadIdx.x < B) {
-    const int b = threadIdx.x;
-    const int lo = p.row_lo[b], hi = p.row_hi[b];
-    rows[b] = (hi > lo && lo >= 0 && hi <= p.cap) ? b * p.cap + lo : -1;
-  }
   __syncthreads();
 
   if (warp == kGemvConsumers) {
     // ------------------------------------------------------------ producer
+    // (weights only: nothing an earlier kernel writes, so no pdl_wait)
     if (lane == 0) {
       for (int s = 0; s < p.n_seg; ++s) {
         tma_prefetch_desc(&l.w[s][0]);
@@ -149,6 +149,13 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
     }
   } else {
     // ------------------------------------------------------------ consumers
+    pdl_wait();   // the rows, the outputs and the row ranges come from earlier kernels
+    if (threadIdx.x < B) {
+      const int b = threadIdx.x;
+      const int lo = p.row_lo[b], hi = p.row_hi[b];
+      rows[b] = (hi > lo && lo >= 0 && hi <= p.cap) ? b * p.cap + lo : -1;
+    }
+    named_barrier_sync(1, kGemvConsumers * 32);
     // 1. stage the batch rows (zeros past K and for rows without a token)
     for (int b = 0; b < B; ++b) {
       const int row = rows[b];
@@ -367,8 +374,8 @@ cudaError_t launch_gemv(const GemvLaunch &l, cudaStream_t st) {
     attr_set[dev] = true;
   }
   auto kern = p.ks == 4 ? gemv_kernel<4> : p.ks == 2 ? gemv_kernel<2> : gemv_kernel<1>;
-  kern<<<p.ctas, kThreads, L.total, st>>>(l, (unsigned)L.xs, (unsigned)L.res, (unsigned)L.bars);
-  return cudaGetLastError();
+  return launch_pdl(kern, dim3(p.ctas), dim3(kThreads), L.total, st, l, (unsigned)L.xs,
+                    (unsigned)L.res, (unsigned)L.bars);
 }
 
 }  // namespace cc
