@@ -33,6 +33,10 @@ Parity status per function (what pins it, in tests/test_oracle_*.py):
                            over two refreshes = one update with both layer sets
   decode_step              = the causal forward's next-token argmax at the last
                            position, step by step over a greedy continuation
+  e4m3_decode/e4m3_encode  values the format's definition names (1, 2, -1, 448,
+                           2^-6, 2^-9, NaN); encode(decode(c)) = c for every finite
+                           code; ties to the even code; saturation; torch's
+                           float8_e4m3fn cast (library routine) in range
   append_chunk             into an empty cache = causal_forward; chunk-by-chunk
                            appends = one append (no refresh between); the layer's
                            attention after a compaction by scalar brute force
@@ -46,3 +50,4 @@ from .refresh import (rms_norm, rope, rope_angles, rope_inv_freq, project, softm
                       memory_causal_attention, append_chunk, recency_scores,
                       key_attention_colsums, importance_scores, h2o_update, h2o_scores,
                       decode_step)
+from .fp8 import e4m3_decode, e4m3_encode, kv_quantize  # noqa: F401

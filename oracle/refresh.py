@@ -37,6 +37,8 @@ Any float dtype is accepted and widened to fp64.
 """
 import numpy as np
 
+from .fp8 import kv_quantize
+
 NEG_INF = -np.inf
 POS_INF = np.inf
 
@@ -375,7 +377,9 @@ def append_chunk(shape, weights, cache, b, tokens, pos=None):
     in pre-fill.  Per layer the chunk's queries, keys and values come from its
     own hidden states (keys and queries rotated at the chunk's positions), the
     keys and values are written after the sequence's current slots
-    (K <- K (+) k_t, V <- V (+) v_t), and attention sees the memory slots
+    (K <- K (+) k_t, V <- V (+) v_t; in an e4m3 cache, one with
+    cache["kv_scale"][l] = (K scale, V scale), as the cache stores them:
+    fp8.kv_quantize), and attention sees the memory slots
     already cached plus the chunk causally (memory_causal_attention).  The
     tokens (X <- X (+) x_t), positions and H^(L-1) (the input of the last
     layer, recorded for the fast approximation) are written too, and
@@ -401,6 +405,9 @@ def append_chunk(shape, weights, cache, b, tokens, pos=None):
         k = rope(project(a, lw, "wk").reshape(h, shape.n_kv_heads, shape.head_dim), pos,
                  shape.rope_theta, sc)
         v = project(a, lw, "wv").reshape(h, shape.n_kv_heads, shape.head_dim)
+        if cache.get("kv_scale") is not None:   # e4m3 cache: rows stored as code * scale
+            k = kv_quantize(k, cache["kv_scale"][l][0])
+            v = kv_quantize(v, cache["kv_scale"][l][1])
         cache["k"][l][b][sl] = k
         cache["v"][l][b][sl] = v
         o = memory_causal_attention(q, cache["k"][l][b], cache["v"][l][b], n0)
