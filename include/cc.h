@@ -63,6 +63,19 @@ typedef enum {
   CC_SCORE_PRECISE = 0x100
 } cc_score_mode;
 
+/* Element format of the cached keys and values.  The paper keeps the model's
+ * own precision; the e4m3 format is a variant that halves the cache: an
+ * element is code * scale, with one scale per layer for K and one for V (the
+ * OCP FP8 E4M3 code: bias 7, no infinities, largest finite 448).  The
+ * scoring passes, the compaction, cc_append_chunk and cc_decode_step take
+ * either format (appends write codes rounded to nearest, saturating at
+ * +-448); the attention-based comparison scorers and
+ * cc_counter_causal_attention take bf16 only (CC_ERR_UNSUPPORTED). */
+typedef enum {
+  CC_KV_BF16 = 0,
+  CC_KV_E4M3 = 1
+} cc_kv_format;
+
 /* Decoder shape (Llama/Qwen pre-norm block: RMSNorm, GQA attention with
  * rotate-half RoPE, RMSNorm, SwiGLU MLP; final RMSNorm; untied LM head). */
 typedef struct {
@@ -124,8 +137,9 @@ typedef struct {
   int32_t batch;
   int32_t cap;
   int32_t *seq_len;  /* device int32 [batch]; cc_compact_kv sets it to keep_count     */
-  void *const *k;    /* HOST array [n_layers] of device bf16 [batch][cap][Hkv][head_dim];
-                        an entry may be NULL where a call does not need that layer     */
+  void *const *k;    /* HOST array [n_layers] of device [batch][cap][Hkv][head_dim]
+                        elements (bf16, or e4m3 bytes: kv_format); an entry may be
+                        NULL where a call does not need that layer                     */
   void *const *v;    /* same layout as k                                               */
   int32_t *tokens;   /* device int32 [batch][cap]: the token buffer X                  */
   int32_t *pos;      /* device int32 [batch][cap]: original position ids (>= 0)        */
@@ -135,6 +149,10 @@ typedef struct {
   float *h2o_acc;    /* optional device fp32 [batch][cap]: running totals of the H2O
                         comparison scorer (cc_h2o_accumulate), compacted with the cache;
                         NULL when unused                                                */
+  int32_t kv_format; /* cc_kv_format of k and v (0 = bf16)                               */
+  const float *kv_scale; /* CC_KV_E4M3: HOST array [n_layers][2] = (K scale, V scale) of
+                        each layer, finite and > 0; the value of an element is its code
+                        times the scale.  Ignored for bf16.                             */
 } cc_kv_cache;
 
 /* ---- scoring (Sec. 3.1) ---------------------------------------------------

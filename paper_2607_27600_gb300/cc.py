@@ -61,7 +61,10 @@ class cc_kv_cache(ctypes.Structure):
                 ("seq_len", ctypes.c_void_p), ("k", ctypes.POINTER(ctypes.c_void_p)),
                 ("v", ctypes.POINTER(ctypes.c_void_p)), ("tokens", ctypes.c_void_p),
                 ("pos", ctypes.c_void_p), ("h_last", ctypes.c_void_p),
-                ("h2o_acc", ctypes.c_void_p)]
+                ("h2o_acc", ctypes.c_void_p), ("kv_format", ctypes.c_int32),
+                ("kv_scale", ctypes.POINTER(ctypes.c_float))]
+
+KV_BF16, KV_E4M3 = 0, 1
 
 
 _LIB = None
@@ -217,9 +220,10 @@ class Weights:
 
 
 class Cache:
-    """cc_kv_cache over a dict of CUDA tensors (k[l], v[l] bf16 [B, cap, Hkv, dh];
-    tokens, pos int32 [B, cap]; seq_len int32 [B]; h_last bf16 [B, cap, d] or
-    None); keeps the tensors alive."""
+    """cc_kv_cache over a dict of CUDA tensors (k[l], v[l] bf16 [B, cap, Hkv, dh],
+    or e4m3 codes (uint8) when the dict holds "kv_scale": per layer the (K, V)
+    scales; tokens, pos int32 [B, cap]; seq_len int32 [B]; h_last bf16
+    [B, cap, d] or None); keeps the tensors alive."""
 
     def __init__(self, c: dict):
         self.d = c
@@ -227,10 +231,18 @@ class Cache:
         ks, vs = c["k"], c["v"]
         self._k = (ctypes.c_void_p * len(ks))(*[_dev_ptr(x, "k") for x in ks])
         self._v = (ctypes.c_void_p * len(vs))(*[_dev_ptr(x, "v") for x in vs])
+        sc = c.get("kv_scale")
+        fmt, self._scale = KV_BF16, None
+        if sc is not None:
+            flat = [float(x) for pair in sc for x in pair]
+            if len(flat) != 2 * len(ks):
+                raise ValueError("kv_scale needs one (K, V) pair per layer")
+            self._scale = (ctypes.c_float * len(flat))(*flat)
+            fmt = KV_E4M3
         self.c = cc_kv_cache(b, cap, _dev_ptr(c["seq_len"], "seq_len"), self._k, self._v,
                              _dev_ptr(c["tokens"], "tokens"), _dev_ptr(c["pos"], "pos"),
                              _dev_ptr(c.get("h_last"), "h_last"),
-                             _dev_ptr(c.get("h2o_acc"), "h2o_acc"))
+                             _dev_ptr(c.get("h2o_acc"), "h2o_acc"), fmt, self._scale)
 
 
 def _cfg(cfg):

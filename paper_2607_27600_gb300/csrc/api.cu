@@ -15,6 +15,7 @@
 
 #include <algorithm>
 #include <atomic>
+#include <cmath>
 #include <mutex>
 
 #include "attn.cuh"
@@ -125,7 +126,8 @@ EncodeTiledFn encode_fn() {
 // bf16 tensor of `rank` dims (dims[0] contiguous), strides in bytes for dims 1.., 128B swizzle.
 bool make_tmap(CUtensorMap *m, const void *base, int rank, const uint64_t *dims,
                const uint64_t *strides, const uint32_t *box,
-               CUtensorMapSwizzle swizzle = CU_TENSOR_MAP_SWIZZLE_128B) {
+               CUtensorMapSwizzle swizzle = CU_TENSOR_MAP_SWIZZLE_128B,
+               CUtensorMapDataType dtype = CU_TENSOR_MAP_DATA_TYPE_BFLOAT16) {
   EncodeTiledFn fn = encode_fn();
   if (!fn) return false;
   cuuint64_t d[5], s[4];
@@ -136,7 +138,7 @@ bool make_tmap(CUtensorMap *m, const void *base, int rank, const uint64_t *dims,
     es[i] = 1;
     if (i > 0) s[i - 1] = strides[i - 1];
   }
-  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, rank, const_cast<void *>(base), d, s, bx, es,
+  return fn(m, dtype, rank, const_cast<void *>(base), d, s, bx, es,
             CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle,
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
@@ -171,6 +173,32 @@ cc_status check_cfg(const cc_model_cfg *c) {
 }
 
 size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+// Element format of layer l's cached K/V.
+struct KvFmt {
+  bool fp8 = false;
+  float k_scale = 1.f, v_scale = 1.f;
+};
+KvFmt kv_fmt(const cc_kv_cache *kv, int l) {
+  KvFmt f;
+  if (kv->kv_format == CC_KV_E4M3) {
+    f.fp8 = true;
+    f.k_scale = kv->kv_scale[2 * l];
+    f.v_scale = kv->kv_scale[2 * l + 1];
+  }
+  return f;
+}
+int kv_elem_bytes(const cc_kv_cache *kv) { return kv->kv_format == CC_KV_E4M3 ? 1 : 2; }
+
+// The cache's format fields: a known format; e4m3 needs finite positive
+// scales for every layer.
+bool kv_format_ok(const cc_model_cfg *c, const cc_kv_cache *kv) {
+  if (kv->kv_format == CC_KV_BF16) return true;
+  if (kv->kv_format != CC_KV_E4M3 || !kv->kv_scale) return false;
+  for (int i = 0; i < 2 * c->n_layers; ++i)
+    if (!(kv->kv_scale[i] > 0.f) || !std::isfinite(kv->kv_scale[i])) return false;
+  return true;
+}
 
 struct ScoreWs {
   size_t xn, q, o, h, act, part, ztgt, flags, total;
@@ -423,7 +451,8 @@ int attn_decode_splits(long long units, int cap, int sms) {
 cc_status run_attention(const cc_model_cfg *c, const void *q, const void *k, const void *v,
                         void *out, const int32_t *seq_len, int batch, int cap, unsigned *status,
                         cudaStream_t st, bool split = false, const int32_t *row_lo = nullptr,
-                        int q_span = 0, const AttnPartials *parts = nullptr, int sms = 0) {
+                        int q_span = 0, const AttnPartials *parts = nullptr, int sms = 0,
+                        KvFmt kvf = KvFmt()) {
   const int G = c->n_q_heads / c->n_kv_heads, dh = c->head_dim;
   const int P = attn_positions_per_unit(G);
   const uint64_t R = (uint64_t)batch * cap;
@@ -434,7 +463,16 @@ cc_status run_attention(const cc_model_cfg *c, const void *q, const void *k, con
     const uint32_t box[3] = {64, (uint32_t)G, (uint32_t)P};
     if (!make_tmap(&tq, q, 3, dims, strides, box)) return tmap_fail();
   }
-  {
+  if (kvf.fp8) {   // e4m3 bytes, one unswizzled box per 128-key tile (converted in the kernel)
+    const uint64_t dims[3] = {(uint64_t)dh, (uint64_t)c->n_kv_heads, R};
+    const uint64_t strides[2] = {(uint64_t)dh, (uint64_t)c->n_kv_heads * dh};
+    const uint32_t box[3] = {(uint32_t)dh, 1, 128};
+    if (!make_tmap(&tk, k, 3, dims, strides, box, CU_TENSOR_MAP_SWIZZLE_NONE,
+                   CU_TENSOR_MAP_DATA_TYPE_UINT8) ||
+        !make_tmap(&tv, v, 3, dims, strides, box, CU_TENSOR_MAP_SWIZZLE_NONE,
+                   CU_TENSOR_MAP_DATA_TYPE_UINT8))
+      return tmap_fail();
+  } else {
     const uint64_t dims[3] = {(uint64_t)dh, (uint64_t)c->n_kv_heads, R};
     const uint64_t strides[2] = {(uint64_t)dh * 2, (uint64_t)c->n_kv_heads * dh * 2};
     const uint32_t box[3] = {64, 1, 128};
@@ -453,7 +491,11 @@ cc_status run_attention(const cc_model_cfg *c, const void *q, const void *k, con
   p.out = reinterpret_cast<__nv_bfloat16 *>(out);
   p.out_ld = c->n_q_heads * dh * (split ? 2 : 1);
   p.out_lo = split ? c->n_q_heads * dh : 0;
-  p.scale_log2 = (float)(1.4426950408889634 / sqrt((double)dh));
+  // e4m3 cache: S = Q . (codes * k_scale), so the K scale joins the softmax
+  // scale; O = v_scale * P . codes, applied with the normalisation
+  p.scale_log2 = (float)(1.4426950408889634 / sqrt((double)dh) * kvf.k_scale);
+  p.kv_fp8 = kvf.fp8 ? 1 : 0;
+  p.v_scale = kvf.v_scale;
   p.status = status;
   p.causal = row_lo ? 1 : 0;
   p.row_lo = row_lo;
@@ -465,8 +507,8 @@ cc_status run_attention(const cc_model_cfg *c, const void *q, const void *k, con
     p.part_o = parts->o;
     p.part_ml = parts->ml;
     p.q = reinterpret_cast<const __nv_bfloat16 *>(q);
-    p.k = reinterpret_cast<const __nv_bfloat16 *>(k);
-    p.v = reinterpret_cast<const __nv_bfloat16 *>(v);
+    p.k = k;
+    p.v = v;
     TimedScope t(CC_KERNEL_ATTN_CAUSAL, st);
     CC_TRY(launch_attention_decode(p, st));
     return CC_OK;
@@ -513,7 +555,8 @@ cc_status check_append_args(const cc_model_cfg *c, const cc_model_weights *w,
   if (!w || !kv || !w->layers || !w->embed || !kv->k || !kv->v || !tokens_in || max_count < 0 ||
       (!count && max_count != 1))   // no count array: one token each
     return CC_ERR_INVALID_ARG;
-  if (kv->batch < 1 || kv->cap < 1 || !kv->seq_len || !kv->tokens || !kv->pos)
+  if (kv->batch < 1 || kv->cap < 1 || !kv->seq_len || !kv->tokens || !kv->pos ||
+      !kv_format_ok(c, kv))
     return CC_ERR_INVALID_ARG;
   if (kv->batch > gemm_max_batch()) return CC_ERR_UNSUPPORTED;
   if ((uint64_t)kv->batch * kv->cap >= (1ull << 31)) return CC_ERR_UNSUPPORTED;
@@ -647,6 +690,7 @@ cc_status run_append(const cc_model_cfg *c, const cc_model_weights *w, const cc_
   }
   for (int l = 0; l < c->n_layers; ++l) {
     const cc_layer_weights &lw = w->layers[l];
+    const KvFmt kvf = kv_fmt(kv, l);   // e4m3 cache: K/V rows written as codes of value / scale
     if (l == c->n_layers - 1 && kv->h_last) {   // H^(L-1), recorded for the fast approximation
       TimedScope t(CC_KERNEL_APPEND, st);
       CC_TRY(launch_store_bf16(h, kv->h_last, d, hi, lo, cap, rows, st, max_count));
@@ -656,6 +700,10 @@ cc_status run_append(const cc_model_cfg *c, const cc_model_weights *w, const cc_
       g.add(lw.wq, nullptr, lw.bq, q, qd, qd, GEMV_ROPE);
       g.add(lw.wk, nullptr, lw.bk, kv->k[l], kvd, kvd, GEMV_ROPE);
       g.add(lw.wv, nullptr, lw.bv, kv->v[l], kvd, kvd, GEMV_BF16);
+      for (int j = 1; j < 3; ++j) {
+        g.l.p.seg[j].fp8 = kvf.fp8 ? 1 : 0;
+        g.l.p.seg[j].qscale = 1.f / (j == 1 ? kvf.k_scale : kvf.v_scale);
+      }
       if ((s = run_gemv(g, CC_KERNEL_GEMM_QKV, dev->sms, st)) != CC_OK) return s;
     } else {
       TimedScope t(CC_KERNEL_RMSNORM, st);
@@ -672,6 +720,9 @@ cc_status run_append(const cc_model_cfg *c, const cc_model_weights *w, const cc_
       g.p.out_k = kv->k[l];
       g.p.out_v = kv->v[l];
       g.p.pos = kv->pos;
+      g.p.kv_fp8 = kvf.fp8 ? 1 : 0;
+      g.p.k_qscale = 1.f / kvf.k_scale;
+      g.p.v_qscale = 1.f / kvf.v_scale;
       if ((s = run_gemm(g, EPI_QKV, CC_KERNEL_GEMM_QKV, dev->sms, st)) != CC_OK) return s;
     }
     struct Proj { const void *w, *bias; void *out; int n, epi, kind; };
@@ -690,12 +741,17 @@ cc_status run_append(const cc_model_cfg *c, const cc_model_weights *w, const cc_
       g.p.pos = kv->pos;
       g.p.bias = reinterpret_cast<const __nv_bfloat16 *>(pj.bias);
       g.p.head_dim = c->head_dim;
+      if (pj.kind == CC_KERNEL_GEMM_KV) {   // K or V rows into the cache
+        g.p.kv_fp8 = kvf.fp8 ? 1 : 0;
+        g.p.k_qscale = 1.f / kvf.k_scale;
+        g.p.v_qscale = 1.f / kvf.v_scale;
+      }
       if (pj.epi == EPI_QROPE) rope_turns(c, g.p.turns);
       if ((s = run_gemm(g, pj.epi, pj.kind, dev->sms, st)) != CC_OK) return s;
     }
     // o = attention of the chunk rows over the memory and the chunk (causal)
     if ((s = run_attention(c, q, kv->k[l], kv->v[l], o, hi, batch, cap, status, st, false, lo,
-                           max_count, &parts, dev->sms)) != CC_OK)
+                           max_count, &parts, dev->sms, kvf)) != CC_OK)
       return s;
     // h += o Wo^T; xn = RMSNorm(h); act = SwiGLU; h += act Wd^T
     if (use_gemv) {
@@ -760,7 +816,8 @@ cc_status check_score_args(const cc_model_cfg *c, const cc_model_weights *w, con
   if ((base_mode != CC_SCORE_LOGIT && base_mode != CC_SCORE_LOGPROB) ||
       (mode & ~(0xFF | CC_SCORE_PRECISE)))
     return CC_ERR_INVALID_ARG;
-  if (kv->batch < 1 || kv->cap < 1 || !kv->seq_len || !kv->tokens || !kv->pos)
+  if (kv->batch < 1 || kv->cap < 1 || !kv->seq_len || !kv->tokens || !kv->pos ||
+      !kv_format_ok(c, kv))
     return CC_ERR_INVALID_ARG;
   if (kv->batch > gemm_max_batch()) return CC_ERR_UNSUPPORTED;
   if ((uint64_t)kv->batch * kv->cap >= (1ull << 31)) return CC_ERR_UNSUPPORTED;
@@ -831,7 +888,8 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
     rope_turns(c, gq.p.turns);
     if ((s = run_gemm(gq, EPI_QROPE, CC_KERNEL_GEMM_QROPE, dev->sms, st)) != CC_OK) return s;
     // O = counter-causal attention
-    if ((s = run_attention(c, q, kv->k[l], kv->v[l], o, sl, batch, cap, status, st, split)) !=
+    if ((s = run_attention(c, q, kv->k[l], kv->v[l], o, sl, batch, cap, status, st, split,
+                           nullptr, 0, nullptr, 0, kv_fmt(kv, l))) !=
         CC_OK)
       return s;
     // h = h + O Wo^T  (fast mode: h = H^(L-1) + O Wo^T)
@@ -909,7 +967,7 @@ cc_status compact_plan(const cc_model_cfg *c, const cc_kv_cache *kv, CompactPlan
   cc_status s = check_cfg(c);
   if (s != CC_OK) return s;
   if (!kv || kv->batch < 1 || kv->cap < 1 || !kv->k || !kv->v || !kv->tokens || !kv->pos ||
-      !kv->seq_len)
+      !kv->seq_len || !kv_format_ok(c, kv))
     return CC_ERR_INVALID_ARG;
   CompactParams &p = plan.p;
   memset(&p, 0, sizeof(p));
@@ -941,7 +999,7 @@ cc_status compact_plan(const cc_model_cfg *c, const cc_kv_cache *kv, CompactPlan
     units += kv->batch * A.n_chunks;
     return true;
   };
-  const int kv_row = c->n_kv_heads * c->head_dim * 2;
+  const int kv_row = c->n_kv_heads * c->head_dim * kv_elem_bytes(kv);
   // staging shape of the copy kernel for the largest row moved
   const int max_row = std::max(kv_row, kv->h_last ? c->d_model * 2 : 0);
   if (!compact_shape(max_row, p.stage_bytes, p.warps)) return CC_ERR_UNSUPPORTED;
@@ -1045,6 +1103,7 @@ cc_status check_keyattn_args(const cc_model_cfg *c, const cc_kv_cache *kv, void 
   if (!kv || !kv->k || !kv->seq_len || kv->batch < 1 || kv->cap < 1) return CC_ERR_INVALID_ARG;
   if ((uint64_t)kv->batch * kv->cap >= (1ull << 31)) return CC_ERR_UNSUPPORTED;
   if (c->n_layers > kKeyAttnMaxLayers) return CC_ERR_UNSUPPORTED;
+  if (kv->kv_format != CC_KV_BF16) return CC_ERR_UNSUPPORTED;   // bf16 keys only
   for (int l = l0; l < c->n_layers; ++l)
     if (!kv->k[l] || !aligned16(kv->k[l])) return CC_ERR_INVALID_ARG;
   if (!ws || !aligned16(ws) || ws_bytes < cc_keyattn_workspace_size(c, kv->batch, kv->cap))

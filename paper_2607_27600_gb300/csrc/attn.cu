@@ -22,7 +22,14 @@
 //                     zeroes V rows past the sequence end in the last tile
 //   warp 9            TMEM owner + tcgen05.mma issuer:
 //                     S_h = Q_h K^T (SS),  O_h += P_h V (TS, P from TMEM)
-//   warps 10, 11      idle (complete the third warpgroup)
+//   warps 10, 11      idle (complete the third warpgroup); with an e4m3 cache
+//                     (FP8) they convert: Q bf16 -> f16 once, then every K and
+//                     V tile from the fp8 staging buffer (TMA, unswizzled) into
+//                     the 128-byte-swizzled f16 stage the MMA reads, zeroing V
+//                     rows past the sequence end; the MMAs then run on f16
+//                     operands (Q, K, V and P all f16: e4m3 -> f16 is exact),
+//                     the K scale folded into the softmax scale and the V
+//                     scale into the output normalisation
 //
 // TMEM columns: S0 [0,128)  S1 [128,256)  O0 [256,256+DH)  O1 [256+DH, 256+2DH)
 #include "attn.cuh"
@@ -93,17 +100,32 @@ CC_DEV float2 exp2_poly2(float2 x) {
                      __uint_as_float(__float_as_uint(p.y) + (__float_as_uint(t.y) << 23)));
 }
 
-template <int DH>
+template <int DH, bool FP8 = false>
 struct AttnSmem {
   static constexpr int NH = DH / 64;                 // 64-element (128-byte) column halves
   static constexpr int Q_BYTES = NH * 256 * 128;     // 256 rows
-  static constexpr int KV_BYTES = NH * BKV * 128;    // one K (or V) tile
+  static constexpr int KV_BYTES = NH * BKV * 128;    // one K (or V) tile (2-byte elements)
+  static constexpr int STG_BYTES = FP8 ? BKV * DH : 0;   // one fp8 K (or V) tile, unswizzled
   static constexpr int OFF_Q = 0;
   static constexpr int OFF_K = OFF_Q + Q_BYTES;
   static constexpr int OFF_V = OFF_K + KST * KV_BYTES;
-  static constexpr int OFF_BAR = OFF_V + KST * KV_BYTES;
+  static constexpr int OFF_STG = OFF_V + KST * KV_BYTES;   // [K, V] staging (FP8)
+  static constexpr int OFF_BAR = OFF_STG + 2 * STG_BYTES;
   static constexpr int BYTES = OFF_BAR + 256 + 1024;   // barriers + alignment slack
 };
+
+// e4m3 pair (low 16 bits) -> f16 pair, exact; bf16 pair -> f16 pair; f16 pack.
+CC_DEV uint32_t e4m3x2_to_f16x2(uint32_t two) {
+  uint32_t r;
+  asm("cvt.rn.f16x2.e4m3x2 %0, %1;" : "=r"(r) : "h"((unsigned short)(two & 0xFFFFu)));
+  return r;
+}
+CC_DEV uint32_t pack_f16x2(float lo, float hi) {
+  uint32_t r;
+  asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+  return r;
+}
+CC_DEV uint32_t bf16x2_to_f16x2(uint32_t w) { return pack_f16x2(bf16_lo(w), bf16_hi(w)); }
 
 // Work unit `unit_id` -> (sequence b, KV head g, positions p0..p_last).
 // Unit order: streams (sequence, KV head) in groups of streams_per_group;
@@ -139,11 +161,11 @@ CC_DEV UnitInfo decode_unit(const AttnParams &p, int unit_id, bool causal) {
   return u;
 }
 
-template <int DH, bool CAUSAL>
+template <int DH, bool CAUSAL, bool FP8>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                 const __grid_constant__ CUtensorMap tmV, const __grid_constant__ AttnParams p) {
-  using L = AttnSmem<DH>;
+  using L = AttnSmem<DH, FP8>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                               ~uintptr_t(1023));
@@ -158,7 +180,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t *p_ready = s_ready + 2;         // [2] (keys 0..63 of P when split)
   uint64_t *p_ready_hi = p_ready + 2;      // [2] keys 64..127 of P (split hand-over)
   uint64_t *o_done = p_ready_hi + 2;       // [2]
-  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(o_done + 2);
+  uint64_t *stg_full = o_done + 2;         // [2] FP8: fp8 K / V tile in the staging buffer
+  uint64_t *stg_empty = stg_full + 2;      // [2] FP8: staging converted (free)
+  uint64_t *q_conv = stg_empty + 2;        // FP8: Q converted to f16
+  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(q_conv + 1);
   volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -205,13 +230,20 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (threadIdx.x == 0) {
     mbar_init(q_full, 1);
-    for (int s = 0; s < KST; ++s) {
-      mbar_init(&k_full[s], 1);
+    for (int s = 0; s < KST; ++s) {   // FP8: K/V stages are filled by the 64 converter threads
+      mbar_init(&k_full[s], FP8 ? 64 : 1);
       mbar_init(&k_empty[s], 1);
-      mbar_init(&v_full[s], 1);
+      mbar_init(&v_full[s], FP8 ? 64 : 1);
       mbar_init(&v_empty[s], 1);
     }
     mbar_init(v_fixed, 1);
+    if (FP8) {
+      for (int i = 0; i < 2; ++i) {
+        mbar_init(&stg_full[i], 1);
+        mbar_init(&stg_empty[i], 64);
+      }
+      mbar_init(q_conv, 64);
+    }
     for (int h = 0; h < 2; ++h) {
       mbar_init(&s_ready[h], 1);
       mbar_init(&p_ready[h], 128);
@@ -249,48 +281,75 @@ __global__ void __launch_bounds__(kThreads, 1)
         tma_load_3d(smem + L::OFF_Q + hh * 256 * 128, &tmQ, q_full, hh * 64, g * G,
                     (int)row_base + p0);
     }
-    for (int it = 0; it < ntiles; ++it) {
-      const int t = t_hi - it, s = it % KST;   // key tiles from the sequence end downwards
-      const uint32_t ph = (it / KST) & 1;
-      const int krow = (int)row_base + t * BKV;
-      int ok = 1;
-      if (lane == 0) {
-        ok = mbar_wait(&k_empty[s], ph ^ 1, abort_flag, p.status);
-        if (ok) {
-          mbar_arrive_expect_tx(&k_full[s], L::KV_BYTES);
-          for (int hh = 0; hh < L::NH; ++hh)
-            tma_load_3d(smem + L::OFF_K + s * L::KV_BYTES + hh * BKV * 128, &tmK, &k_full[s],
-                        hh * 64, g, krow);
-          ok = mbar_wait(&v_empty[s], ph ^ 1, abort_flag, p.status);
+    if constexpr (FP8) {
+      // fp8 tiles into the one staging buffer; the converters fill the stages
+      for (int it = 0; it < ntiles; ++it) {
+        const int t = t_hi - it;
+        const uint32_t sp = it & 1;
+        const int krow = (int)row_base + t * BKV;
+        int ok = 1;
+        if (lane == 0) {
+          ok = mbar_wait(&stg_empty[0], sp ^ 1, abort_flag, p.status);
+          if (ok) {
+            mbar_arrive_expect_tx(&stg_full[0], L::STG_BYTES);
+            tma_load_3d(smem + L::OFF_STG, &tmK, &stg_full[0], 0, g, krow);
+            ok = mbar_wait(&stg_empty[1], sp ^ 1, abort_flag, p.status);
+          }
+          if (ok) {
+            mbar_arrive_expect_tx(&stg_full[1], L::STG_BYTES);
+            tma_load_3d(smem + L::OFF_STG + L::STG_BYTES, &tmV, &stg_full[1], 0, g, krow);
+          }
         }
-        if (ok) {
-          mbar_arrive_expect_tx(&v_full[s], L::KV_BYTES);
-          for (int hh = 0; hh < L::NH; ++hh)
-            tma_load_3d(smem + L::OFF_V + s * L::KV_BYTES + hh * BKV * 128, &tmV, &v_full[s],
-                        hh * 64, g, krow);
-        }
+        ok = __shfl_sync(0xFFFFFFFFu, ok, 0);
+        if (!ok) break;
       }
-      ok = __shfl_sync(0xFFFFFFFFu, ok, 0);
-      if (!ok) break;
-      if (t == t_top && n - t * BKV < BKV) {
-        // rows past the sequence end may hold any bits; P is 0 there, but
-        // 0 * NaN would still poison O, so zero them before the PV product
-        if (!mbar_wait(&v_full[s], ph, abort_flag, p.status)) break;
-        const int first = n - t * BKV;
-        uint8_t *vs = smem + L::OFF_V + s * L::KV_BYTES;
-        for (int hh = 0; hh < L::NH; ++hh)
-          for (int idx = first * 8 + lane; idx < BKV * 8; idx += 32)
-            reinterpret_cast<uint4 *>(vs + hh * BKV * 128)[idx] = make_uint4(0, 0, 0, 0);
-        fence_proxy_async_smem();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(v_fixed);
+    } else {
+      for (int it = 0; it < ntiles; ++it) {
+        const int t = t_hi - it, s = it % KST;   // key tiles from the sequence end downwards
+        const uint32_t ph = (it / KST) & 1;
+        const int krow = (int)row_base + t * BKV;
+        int ok = 1;
+        if (lane == 0) {
+          ok = mbar_wait(&k_empty[s], ph ^ 1, abort_flag, p.status);
+          if (ok) {
+            mbar_arrive_expect_tx(&k_full[s], L::KV_BYTES);
+            for (int hh = 0; hh < L::NH; ++hh)
+              tma_load_3d(smem + L::OFF_K + s * L::KV_BYTES + hh * BKV * 128, &tmK, &k_full[s],
+                          hh * 64, g, krow);
+            ok = mbar_wait(&v_empty[s], ph ^ 1, abort_flag, p.status);
+          }
+          if (ok) {
+            mbar_arrive_expect_tx(&v_full[s], L::KV_BYTES);
+            for (int hh = 0; hh < L::NH; ++hh)
+              tma_load_3d(smem + L::OFF_V + s * L::KV_BYTES + hh * BKV * 128, &tmV, &v_full[s],
+                          hh * 64, g, krow);
+          }
+        }
+        ok = __shfl_sync(0xFFFFFFFFu, ok, 0);
+        if (!ok) break;
+        if (t == t_top && n - t * BKV < BKV) {
+          // rows past the sequence end may hold any bits; P is 0 there, but
+          // 0 * NaN would still poison O, so zero them before the PV product
+          if (!mbar_wait(&v_full[s], ph, abort_flag, p.status)) break;
+          const int first = n - t * BKV;
+          uint8_t *vs = smem + L::OFF_V + s * L::KV_BYTES;
+          for (int hh = 0; hh < L::NH; ++hh)
+            for (int idx = first * 8 + lane; idx < BKV * 8; idx += 32)
+              reinterpret_cast<uint4 *>(vs + hh * BKV * 128)[idx] = make_uint4(0, 0, 0, 0);
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(v_fixed);
+        }
       }
     }
     } else if (warp == 9) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
-      constexpr uint32_t idesc_qk = make_idesc_bf16(128, BKV, 0, 0);
-      constexpr uint32_t idesc_pv = make_idesc_bf16(128, DH, 0, 1);
+      // FP8: every operand (Q, K, V, P) is f16; otherwise every operand is bf16
+      constexpr uint32_t idesc_qk =
+          FP8 ? make_idesc_f16(128, BKV, 0, 0) : make_idesc_bf16(128, BKV, 0, 0);
+      constexpr uint32_t idesc_pv =
+          FP8 ? make_idesc_f16(128, DH, 0, 1) : make_idesc_bf16(128, DH, 0, 1);
       // Shared-memory descriptors built once; a K step only advances the
       // start-address field (16-byte units): +2 per 16 columns of a 128-byte
       // row (Q, K), +128 per 16 keys of V.  The issuing thread shares its SM
@@ -318,7 +377,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           umma_ss(tmem + h * 128, qd[h][hh] + ko, kd[st][hh] + ko, idesc_qk, kk > 0);
         }
       };
-      bool ok = mbar_wait(q_full, 0, abort_flag, p.status);
+      bool ok = mbar_wait(FP8 ? q_conv : q_full, 0, abort_flag, p.status);
       if (ok) ok = mbar_wait(&k_full[0], 0, abort_flag, p.status);
       if (ok) {
         tc_fence_after();
@@ -334,7 +393,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         TRACE(true, it, 14);
         if (!(ok = mbar_wait(&v_full[s], ph, abort_flag, p.status))) break;
         TRACE(true, it, 15);
-        if (t == t_top && n - t * BKV < BKV)
+        if (!FP8 && t == t_top && n - t * BKV < BKV)
           if (!(ok = mbar_wait(v_fixed, 0, abort_flag, p.status))) break;
         for (int h = 0; h < 2; ++h) {
           TRACE(true, it, 12 + h);
@@ -369,6 +428,57 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
       }
+    }
+    } else if (FP8 && warp >= 10) {
+    // ------------------------------------------------------------ converters (FP8)
+    const int ct = threadIdx.x - 10 * 32;   // 0 .. 63
+    bool ok = mbar_wait(q_full, 0, abort_flag, p.status);
+    if (ok) {   // Q bf16 -> f16 in place (same layout, element by element)
+      uint4 *qv = reinterpret_cast<uint4 *>(smem + L::OFF_Q);
+      for (int i = ct; i < L::Q_BYTES / 16; i += 64) {
+        uint4 x = qv[i];
+        x.x = bf16x2_to_f16x2(x.x);
+        x.y = bf16x2_to_f16x2(x.y);
+        x.z = bf16x2_to_f16x2(x.z);
+        x.w = bf16x2_to_f16x2(x.w);
+        qv[i] = x;
+      }
+      fence_proxy_async_smem();
+      mbar_arrive(q_conv);
+    }
+    // fp8 [BKV][DH] (row r, 8 elements at column 8j) -> f16 stage: 128-byte
+    // rows per 64-column half, 16-byte chunk c of row r at chunk c ^ (r & 7)
+    // (the TMA's 128-byte swizzle); rows >= zero_from are written as zeros
+    auto convert = [&](const uint8_t *src, uint8_t *dst, int zero_from) {
+      for (int i = ct; i < BKV * L::NH * 8; i += 64) {
+        const int r = i / (L::NH * 8), rem = i - r * (L::NH * 8), hh = rem >> 3, c = rem & 7;
+        uint4 o = make_uint4(0, 0, 0, 0);
+        if (r < zero_from) {
+          const uint2 x = *reinterpret_cast<const uint2 *>(src + r * DH + hh * 64 + c * 8);
+          o.x = e4m3x2_to_f16x2(x.x);
+          o.y = e4m3x2_to_f16x2(x.x >> 16);
+          o.z = e4m3x2_to_f16x2(x.y);
+          o.w = e4m3x2_to_f16x2(x.y >> 16);
+        }
+        *reinterpret_cast<uint4 *>(dst + hh * BKV * 128 + r * 128 + ((c ^ (r & 7)) << 4)) = o;
+      }
+      fence_proxy_async_smem();
+    };
+    for (int it = 0; ok && it < ntiles; ++it) {
+      const int t = t_hi - it, s = it % KST;
+      const uint32_t ph = (it / KST) & 1, sp = it & 1;
+      if (!(ok = mbar_wait(&stg_full[0], sp, abort_flag, p.status))) break;
+      if (!(ok = mbar_wait(&k_empty[s], ph ^ 1, abort_flag, p.status))) break;
+      convert(smem + L::OFF_STG, smem + L::OFF_K + s * L::KV_BYTES, BKV);
+      mbar_arrive(&stg_empty[0]);
+      mbar_arrive(&k_full[s]);
+      if (!(ok = mbar_wait(&stg_full[1], sp, abort_flag, p.status))) break;
+      if (!(ok = mbar_wait(&v_empty[s], ph ^ 1, abort_flag, p.status))) break;
+      // V rows past the sequence end may hold any bits (0 * NaN would poison O)
+      const int keep = (t == t_top && n - t * BKV < BKV) ? n - t * BKV : BKV;
+      convert(smem + L::OFF_STG + L::STG_BYTES, smem + L::OFF_V + s * L::KV_BYTES, keep);
+      mbar_arrive(&stg_empty[1]);
+      mbar_arrive(&v_full[s]);
     }
     }
   } else {
@@ -468,7 +578,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             e = exp2_poly2(y);
           else
             e = make_float2(fast_exp2(y.x), fast_exp2(y.y));
-          pk[k / 2] = pack_bf16x2(e.x, e.y);
+          pk[k / 2] = FP8 ? pack_f16x2(e.x, e.y) : pack_bf16x2(e.x, e.y);
           lsum = __fadd2_rn(lsum, e);
         }
         tmem_st16(s_t + c0 / 2, pk);
@@ -506,7 +616,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     } else if (ok) {
       tc_fence_after();
       const bool store = row_used && pos <= p_last;
-      const float inv = l > 0.f ? 1.f / l : 0.f;
+      const float inv = l > 0.f ? p.v_scale / l : 0.f;   // V scale: e4m3 cache (else 1)
       __nv_bfloat16 *dst =
           p.out + (row_base + (store ? pos : 0)) * p.out_ld + (size_t)(g * G + hl) * DH;
 #pragma unroll 1
@@ -599,7 +709,7 @@ __global__ void attn_combine_kernel(const __grid_constant__ AttnParams p) {
     for (int k = 0; k < 8; ++k) o += wgt[s + k] * v[k];
   }
   for (; s < S; ++s) o += wgt[s] * p.part_o[(base + (size_t)s * 256) * p.head_dim + d];
-  const float v = l > 0.f ? o / l : 0.f;
+  const float v = l > 0.f ? o * p.v_scale / l : 0.f;
   __nv_bfloat16 *dst = p.out + ((size_t)u.b * p.cap + pos) * p.out_ld +
                        (size_t)(u.g * G + hl) * p.head_dim + d;
   const __nv_bfloat16 hi = __float2bfloat16_rn(v);
@@ -607,16 +717,16 @@ __global__ void attn_combine_kernel(const __grid_constant__ AttnParams p) {
   if (p.out_lo > 0) dst[p.out_lo] = __float2bfloat16_rn(v - __bfloat162float(hi));
 }
 
-template <int DH, bool CAUSAL>
+template <int DH, bool CAUSAL, bool FP8>
 cudaError_t launch_dh(const CUtensorMap &q, const CUtensorMap &k, const CUtensorMap &v,
                       const AttnParams &p, cudaStream_t stream) {
-  auto kern = attn_kernel<DH, CAUSAL>;
+  auto kern = attn_kernel<DH, CAUSAL, FP8>;
   static bool attr_set[64] = {};
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev < 64 && !attr_set[dev]) {
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         AttnSmem<DH>::BYTES);
+                                         AttnSmem<DH, FP8>::BYTES);
     if (e != cudaSuccess) return e;
     attr_set[dev] = true;
   }
@@ -639,7 +749,7 @@ cudaError_t launch_dh(const CUtensorMap &q, const CUtensorMap &k, const CUtensor
   pp.streams_per_group = (int)fmax(1.0, fmin((double)n_streams, floor(sqrt(kReuseBytes / per_stream2))));
   const int S = pp.kv_splits > 1 ? pp.kv_splits : 1;
   if (S > 1 && (!pp.part_o || !pp.part_ml)) return cudaErrorInvalidValue;
-  kern<<<(unsigned)(units * S), kThreads, AttnSmem<DH>::BYTES, stream>>>(q, k, v, pp);
+  kern<<<(unsigned)(units * S), kThreads, AttnSmem<DH, FP8>::BYTES, stream>>>(q, k, v, pp);
   if (S > 1) {
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
@@ -662,10 +772,13 @@ cudaError_t launch_dh(const CUtensorMap &q, const CUtensorMap &k, const CUtensor
 constexpr int kDecChunk = 128;
 constexpr int kDecThreads = 256;   // = 2 * kDecChunk: the score pass takes a key and half its dims
 
-template <int DH>
+// K rows padded so the score pass's column reads are conflict-free: bf16
+// rows +16 bytes (16-byte reads), e4m3 rows +8 bytes (8-byte reads).
+template <int DH, bool FP8>
 struct DecSmem {
-  static constexpr int K_ROW = DH * 2 + 16;
-  static constexpr int V_ROW = DH * 2;
+  static constexpr int EB = FP8 ? 1 : 2;   // bytes per cached element
+  static constexpr int K_ROW = DH * EB + (FP8 ? 8 : 16);
+  static constexpr int V_ROW = DH * EB;
   static constexpr int K_BYTES = kDecChunk * K_ROW;
   static constexpr int V_BYTES = kDecChunk * V_ROW;
   static constexpr int BUF = K_BYTES + V_BYTES;
@@ -680,15 +793,39 @@ CC_DEV void cp_async16(void *dst, const void *src) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)), "l"(src)
                : "memory");
 }
+CC_DEV void cp_async8(void *dst, const void *src) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 8;" ::"r"(smem_u32(dst)), "l"(src)
+               : "memory");
+}
 CC_DEV void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+
+// 8 cached elements -> float: bf16 (16 bytes) or e4m3 codes (8 bytes, via f16)
+template <bool FP8>
+CC_DEV void load8_kv(const uint8_t *src, float *f) {
+  if constexpr (FP8) {
+    const uint2 x = *reinterpret_cast<const uint2 *>(src);
+    const uint32_t h[4] = {e4m3x2_to_f16x2(x.x), e4m3x2_to_f16x2(x.x >> 16),
+                           e4m3x2_to_f16x2(x.y), e4m3x2_to_f16x2(x.y >> 16)};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float2 v = __half22float2(*reinterpret_cast<const __half2 *>(&h[i]));
+      f[2 * i] = v.x;
+      f[2 * i + 1] = v.y;
+    }
+  } else {
+    const uint4 x = *reinterpret_cast<const uint4 *>(src);
+    f[0] = bf16_lo(x.x); f[1] = bf16_hi(x.x); f[2] = bf16_lo(x.y); f[3] = bf16_hi(x.y);
+    f[4] = bf16_lo(x.z); f[5] = bf16_hi(x.z); f[6] = bf16_lo(x.w); f[7] = bf16_hi(x.w);
+  }
+}
 template <int N>
 CC_DEV void cp_async_wait() {
   asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
 }
 
-template <int DH>
+template <int DH, bool FP8>
 __global__ void __launch_bounds__(kDecThreads) attn_decode_kernel(const __grid_constant__ AttnParams p) {
-  using L = DecSmem<DH>;
+  using L = DecSmem<DH, FP8>;
   extern __shared__ __align__(128) uint8_t smem[];
   pdl_trigger();   // the combine may launch (it waits for this grid before reading)
   pdl_wait();      // q and the new token's K/V come from the projection just before
@@ -717,21 +854,34 @@ __global__ void __launch_bounds__(kDecThreads) attn_decode_kernel(const __grid_c
   const size_t row_base = (size_t)u.b * p.cap;
   const int Hkv = p.n_kv_heads;
 
+  const uint8_t *kg = reinterpret_cast<const uint8_t *>(p.k);
+  const uint8_t *vg = reinterpret_cast<const uint8_t *>(p.v);
   auto issue = [&](int c, int buf) {
     uint8_t *kb = smem + buf * L::BUF, *vb = kb + L::K_BYTES;
-    constexpr int PIECES = DH * 2 / 16;   // 16-byte pieces of a row
-    for (int i = tid; i < kDecChunk * PIECES; i += kDecThreads) {
-      const int r = i / PIECES, e = i - r * PIECES;
+    // K in DH/8 pieces per row (16 bytes bf16, 8 bytes e4m3), V in 16-byte pieces
+    constexpr int KP = DH / 8, KPB = 8 * L::EB, VP = DH * L::EB / 16;
+    for (int i = tid; i < kDecChunk * KP; i += kDecThreads) {
+      const int r = i / KP, e = i - r * KP;
       const int j = c * kDecChunk + r;
-      uint8_t *kd = kb + r * L::K_ROW + e * 16, *vd = vb + r * L::V_ROW + e * 16;
+      uint8_t *kd = kb + r * L::K_ROW + e * KPB;
       if (j < n_keys) {
-        const size_t off = ((row_base + j) * Hkv + u.g) * (size_t)DH + e * 8;
-        cp_async16(kd, p.k + off);
-        cp_async16(vd, p.v + off);
-      } else {   // past the last key: zeros (P is 0 there, V must be finite)
+        const uint8_t *src = kg + (((row_base + j) * Hkv + u.g) * (size_t)DH) * L::EB + e * KPB;
+        if constexpr (FP8) cp_async8(kd, src);
+        else cp_async16(kd, src);
+      } else if constexpr (FP8) {
+        *reinterpret_cast<uint2 *>(kd) = make_uint2(0, 0);
+      } else {
         *reinterpret_cast<uint4 *>(kd) = make_uint4(0, 0, 0, 0);
-        *reinterpret_cast<uint4 *>(vd) = make_uint4(0, 0, 0, 0);
       }
+    }
+    for (int i = tid; i < kDecChunk * VP; i += kDecThreads) {
+      const int r = i / VP, e = i - r * VP;
+      const int j = c * kDecChunk + r;
+      uint8_t *vd = vb + r * L::V_ROW + e * 16;
+      if (j < n_keys)   // past the last key: zeros (P is 0 there, V must be finite)
+        cp_async16(vd, vg + (((row_base + j) * Hkv + u.g) * (size_t)DH) * L::EB + e * 16);
+      else
+        *reinterpret_cast<uint4 *>(vd) = make_uint4(0, 0, 0, 0);
     }
     cp_async_commit();
   };
@@ -760,15 +910,14 @@ __global__ void __launch_bounds__(kDecThreads) attn_decode_kernel(const __grid_c
     const uint8_t *kb = smem + buf * L::BUF, *vb = kb + L::K_BYTES;
     {   // scores: thread = (key j, half of the dims)
       const int j = tid & (kDecChunk - 1), half = tid / kDecChunk;
-      const uint8_t *kr = kb + j * L::K_ROW + half * DH;
+      const uint8_t *kr = kb + j * L::K_ROW + half * (DH / 2) * L::EB;
       float sc[kDecMaxG];
 #pragma unroll
       for (int h = 0; h < kDecMaxG; ++h) sc[h] = 0.f;
 #pragma unroll
       for (int d8 = 0; d8 < DH / 16; ++d8) {
-        const uint4 kv = *reinterpret_cast<const uint4 *>(kr + d8 * 16);
-        const float kf[8] = {bf16_lo(kv.x), bf16_hi(kv.x), bf16_lo(kv.y), bf16_hi(kv.y),
-                             bf16_lo(kv.z), bf16_hi(kv.z), bf16_lo(kv.w), bf16_hi(kv.w)};
+        float kf[8];
+        load8_kv<FP8>(kr + d8 * 8 * L::EB, kf);
         const int d0 = half * (DH / 2) + d8 * 8;
 #pragma unroll
         for (int h = 0; h < kDecMaxG; ++h) {
@@ -827,8 +976,16 @@ __global__ void __launch_bounds__(kDecThreads) attn_decode_kernel(const __grid_c
 #pragma unroll 4
       for (int j = 0; j < kDecChunk; ++j) {
         const float pj = ph[j];
-        const uint8_t *vr = vb + j * L::V_ROW + lane * DPT * 2;
-        if constexpr (DPT == 4) {
+        const uint8_t *vr = vb + j * L::V_ROW + lane * DPT * L::EB;
+        if constexpr (FP8) {
+#pragma unroll
+          for (int i = 0; i < DPT; i += 2) {
+            const uint32_t hv = e4m3x2_to_f16x2(*reinterpret_cast<const uint16_t *>(vr + i));
+            const float2 v = __half22float2(*reinterpret_cast<const __half2 *>(&hv));
+            o[i] = fmaf(pj, v.x, o[i]);
+            o[i + 1] = fmaf(pj, v.y, o[i + 1]);
+          }
+        } else if constexpr (DPT == 4) {
           const uint2 v = *reinterpret_cast<const uint2 *>(vr);
           o[0] = fmaf(pj, bf16_lo(v.x), o[0]);
           o[1] = fmaf(pj, bf16_hi(v.x), o[1]);
@@ -851,15 +1008,15 @@ __global__ void __launch_bounds__(kDecThreads) attn_decode_kernel(const __grid_c
   }
 }
 
-template <int DH>
+template <int DH, bool FP8>
 cudaError_t launch_decode_dh(const AttnParams &p, cudaStream_t stream) {
   static bool attr_set[64] = {};
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev < 64 && !attr_set[dev]) {
-    cudaError_t e = cudaFuncSetAttribute(attn_decode_kernel<DH>,
+    cudaError_t e = cudaFuncSetAttribute(attn_decode_kernel<DH, FP8>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         DecSmem<DH>::BYTES);
+                                         DecSmem<DH, FP8>::BYTES);
     if (e != cudaSuccess) return e;
     attr_set[dev] = true;
   }
@@ -867,8 +1024,8 @@ cudaError_t launch_decode_dh(const AttnParams &p, cudaStream_t stream) {
   if (units <= 0) return cudaSuccess;
   AttnParams pp = p;
   pp.streams_per_group = p.batch * p.n_kv_heads;
-  cudaError_t e = launch_pdl(attn_decode_kernel<DH>, dim3((unsigned)(units * pp.kv_splits)),
-                             dim3(kDecThreads), DecSmem<DH>::BYTES, stream, pp);
+  cudaError_t e = launch_pdl(attn_decode_kernel<DH, FP8>, dim3((unsigned)(units * pp.kv_splits)),
+                             dim3(kDecThreads), DecSmem<DH, FP8>::BYTES, stream, pp);
   if (e != cudaSuccess) return e;
   return launch_pdl(attn_combine_kernel<true>, dim3((unsigned)p.group, (unsigned)units), dim3(DH),
                     0, stream, pp);
@@ -892,19 +1049,31 @@ cudaError_t launch_attention_decode(const AttnParams &p, cudaStream_t stream) {
   if (!p.causal || p.q_span != 1 || p.group > kDecMaxG || p.kv_splits < 1 || !p.q || !p.k ||
       !p.v || !p.part_o || !p.part_ml)
     return cudaErrorInvalidValue;
-  if (p.head_dim == 128) return launch_decode_dh<128>(p, stream);
-  if (p.head_dim == 64) return launch_decode_dh<64>(p, stream);
+  const bool f8 = p.kv_fp8 != 0;
+  if (p.head_dim == 128)
+    return f8 ? launch_decode_dh<128, true>(p, stream) : launch_decode_dh<128, false>(p, stream);
+  if (p.head_dim == 64)
+    return f8 ? launch_decode_dh<64, true>(p, stream) : launch_decode_dh<64, false>(p, stream);
   return cudaErrorInvalidValue;
 }
 
 cudaError_t launch_attention(const CUtensorMap &q, const CUtensorMap &k, const CUtensorMap &v,
                              const AttnParams &p, cudaStream_t stream) {
+  const bool f8 = p.kv_fp8 != 0;
   if (p.causal) {
-    if (p.head_dim == 128) return launch_dh<128, true>(q, k, v, p, stream);
-    if (p.head_dim == 64) return launch_dh<64, true>(q, k, v, p, stream);
+    if (p.head_dim == 128)
+      return f8 ? launch_dh<128, true, true>(q, k, v, p, stream)
+                : launch_dh<128, true, false>(q, k, v, p, stream);
+    if (p.head_dim == 64)
+      return f8 ? launch_dh<64, true, true>(q, k, v, p, stream)
+                : launch_dh<64, true, false>(q, k, v, p, stream);
   } else {
-    if (p.head_dim == 128) return launch_dh<128, false>(q, k, v, p, stream);
-    if (p.head_dim == 64) return launch_dh<64, false>(q, k, v, p, stream);
+    if (p.head_dim == 128)
+      return f8 ? launch_dh<128, false, true>(q, k, v, p, stream)
+                : launch_dh<128, false, false>(q, k, v, p, stream);
+    if (p.head_dim == 64)
+      return f8 ? launch_dh<64, false, true>(q, k, v, p, stream)
+                : launch_dh<64, false, false>(q, k, v, p, stream);
   }
   return cudaErrorInvalidValue;
 }

@@ -5,6 +5,7 @@
 
 #include <cuda.h>
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -241,6 +242,17 @@ __host__ __device__ constexpr uint32_t make_idesc_bf16(int M, int N, int a_mn, i
          | (uint32_t(M >> 4) << 24);        // M / 16
 }
 
+// Instruction descriptor for kind::f16 with f16 A and B (A and B always share
+// one type), fp32 D.
+__host__ __device__ constexpr uint32_t make_idesc_f16(int M, int N, int a_mn, int b_mn) {
+  return (1u << 4)                          // D format: f32
+         | (0u << 7)                        // A format: f16
+         | (0u << 10)                       // B format: f16
+         | (uint32_t(a_mn) << 15) | (uint32_t(b_mn) << 16)
+         | (uint32_t(N >> 3) << 17)         // N / 8
+         | (uint32_t(M >> 4) << 24);        // M / 16
+}
+
 // Shared-memory matrix descriptor, 128-byte swizzle (rows of 128 bytes,
 // 8-row / 1024-byte swizzle atoms).  lbo/sbo in bytes.
 CC_DEV uint64_t make_sdesc_sw128(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
@@ -312,6 +324,14 @@ CC_DEV uint32_t pack_bf16x2(float lo, float hi) {
 }
 CC_DEV float bf16_lo(uint32_t v) { return __uint_as_float(v << 16); }
 CC_DEV float bf16_hi(uint32_t v) { return __uint_as_float(v & 0xFFFF0000u); }
+
+// Two e4m3 codes (lo in the low byte): round to nearest even, saturating to
+// +-448 (the e4m3 K/V cache's element encoding).
+CC_DEV uint32_t pack_e4m3x2(float lo, float hi) {
+  unsigned short r;
+  asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;" : "=h"(r) : "f"(hi), "f"(lo));
+  return r;
+}
 
 CC_DEV float silu(float x) { return x / (1.0f + __expf(-x)); }
 

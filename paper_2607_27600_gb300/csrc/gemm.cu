@@ -34,13 +34,15 @@ constexpr size_t kSmemBytes = 1024 /*align slack*/ + ST * (A_BYTES + B_BYTES) + 
 // [col0, col0 + TBN) of out (row stride ldo, n_dest columns in all), each tile
 // holding TBN / head_dim whole heads; rotate-half pairs (k, k + dh/2); the
 // bias (optional) is added before the rotation.
-template <int TBN>
-CC_DEV void rope_store(const GemmParams &p, uint32_t tacc, int grow, bool valid,
-                       __nv_bfloat16 *out_base, int ldo, const __nv_bfloat16 *bias, int col0,
-                       int n_dest) {
+// F8: the destination is an e4m3 cache (one byte per element, the value
+// times qscale = 1 / the layer's scale; pack_e4m3x2).
+template <int TBN, bool F8 = false>
+CC_DEV void rope_store(const GemmParams &p, uint32_t tacc, int grow, bool valid, void *out_base,
+                       int ldo, const __nv_bfloat16 *bias, int col0, int n_dest,
+                       float qscale = 1.f) {
   const int half = p.head_dim >> 1;
   const uint32_t pos = valid ? (uint32_t)p.pos[grow] : 0u;
-  __nv_bfloat16 *out = out_base + (size_t)grow * ldo;
+  uint8_t *out = reinterpret_cast<uint8_t *>(out_base) + (size_t)grow * ldo * (F8 ? 1 : 2);
 #pragma unroll 1
   for (int hb = 0; hb < TBN; hb += p.head_dim) {
 #pragma unroll 1
@@ -72,13 +74,28 @@ CC_DEV void rope_store(const GemmParams &p, uint32_t tacc, int grow, bool valid,
         float a2 = __uint_as_float(x2[k]) + bf16_lo(bb2[k / 2]);
         float b1 = __uint_as_float(x1[k + 1]) + bf16_hi(bb1[k / 2]);
         float b2 = __uint_as_float(x2[k + 1]) + bf16_hi(bb2[k / 2]);
-        o1[k / 2] = pack_bf16x2(a1 * c_a - a2 * s_a, b1 * c_b - b2 * s_b);
-        o2[k / 2] = pack_bf16x2(a2 * c_a + a1 * s_a, b2 * c_b + b1 * s_b);
+        if constexpr (F8) {   // two codes per pair, four per word
+          const uint32_t e1 = pack_e4m3x2((a1 * c_a - a2 * s_a) * qscale,
+                                          (b1 * c_b - b2 * s_b) * qscale);
+          const uint32_t e2 = pack_e4m3x2((a2 * c_a + a1 * s_a) * qscale,
+                                          (b2 * c_b + b1 * s_b) * qscale);
+          if ((k & 2) == 0) {
+            o1[k / 4] = e1;
+            o2[k / 4] = e2;
+          } else {
+            o1[k / 4] |= e1 << 16;
+            o2[k / 4] |= e2 << 16;
+          }
+        } else {
+          o1[k / 2] = pack_bf16x2(a1 * c_a - a2 * s_a, b1 * c_b - b2 * s_b);
+          o2[k / 2] = pack_bf16x2(a2 * c_a + a1 * s_a, b2 * c_b + b1 * s_b);
+        }
       }
-      uint4 *d1 = reinterpret_cast<uint4 *>(out + col);
-      uint4 *d2 = reinterpret_cast<uint4 *>(out + col + half);
+      constexpr int EB = F8 ? 1 : 2;
+      uint4 *d1 = reinterpret_cast<uint4 *>(out + (size_t)col * EB);
+      uint4 *d2 = reinterpret_cast<uint4 *>(out + (size_t)(col + half) * EB);
 #pragma unroll
-      for (int v = 0; v < 4; ++v) {
+      for (int v = 0; v < 2 * EB; ++v) {   // 32 elements: 64 bytes bf16, 32 e4m3
         d1[v] = make_uint4(o1[v * 4], o1[v * 4 + 1], o1[v * 4 + 2], o1[v * 4 + 3]);
         d2[v] = make_uint4(o2[v * 4], o2[v * 4 + 1], o2[v * 4 + 2], o2[v * 4 + 3]);
       }
@@ -86,11 +103,13 @@ CC_DEV void rope_store(const GemmParams &p, uint32_t tacc, int grow, bool valid,
   }
 }
 
-// Plain bf16 store (+ optional bias) of one accumulator tile row.
-template <int TBN>
-CC_DEV void plain_store(uint32_t tacc, int grow, bool valid, __nv_bfloat16 *out_base, int ldo,
-                        const __nv_bfloat16 *bias, int col0, int n_dest) {
-  __nv_bfloat16 *out = out_base + (size_t)grow * ldo;
+// Plain bf16 store (+ optional bias) of one accumulator tile row; F8: e4m3
+// codes of (value + bias) * qscale instead.
+template <int TBN, bool F8 = false>
+CC_DEV void plain_store(uint32_t tacc, int grow, bool valid, void *out_base, int ldo,
+                        const __nv_bfloat16 *bias, int col0, int n_dest, float qscale = 1.f) {
+  constexpr int EB = F8 ? 1 : 2;
+  uint8_t *out = reinterpret_cast<uint8_t *>(out_base) + (size_t)grow * ldo * EB;
 #pragma unroll 1
   for (int c = 0; c < TBN / 32; ++c) {
     uint32_t r[32];
@@ -106,12 +125,21 @@ CC_DEV void plain_store(uint32_t tacc, int grow, bool valid, __nv_bfloat16 *out_
     }
     uint32_t o[16];
 #pragma unroll
-    for (int k = 0; k < 32; k += 2)
-      o[k / 2] = pack_bf16x2(__uint_as_float(r[k]) + bf16_lo(bb[k / 2]),
-                             __uint_as_float(r[k + 1]) + bf16_hi(bb[k / 2]));
-    uint4 *d = reinterpret_cast<uint4 *>(out + col);
+    for (int k = 0; k < 32; k += 2) {
+      const float y0 = __uint_as_float(r[k]) + bf16_lo(bb[k / 2]);
+      const float y1 = __uint_as_float(r[k + 1]) + bf16_hi(bb[k / 2]);
+      if constexpr (F8) {
+        const uint32_t e = pack_e4m3x2(y0 * qscale, y1 * qscale);
+        if ((k & 2) == 0) o[k / 4] = e;
+        else o[k / 4] |= e << 16;
+      } else {
+        o[k / 2] = pack_bf16x2(y0, y1);
+      }
+    }
+    uint4 *d = reinterpret_cast<uint4 *>(out + (size_t)col * EB);
 #pragma unroll
-    for (int v = 0; v < 4; ++v) d[v] = make_uint4(o[v * 4], o[v * 4 + 1], o[v * 4 + 2], o[v * 4 + 3]);
+    for (int v = 0; v < 2 * EB; ++v)   // 32 elements: 64 bytes bf16, 32 e4m3
+      d[v] = make_uint4(o[v * 4], o[v * 4 + 1], o[v * 4 + 2], o[v * 4 + 3]);
   }
 }
 
@@ -158,24 +186,33 @@ CC_DEV void epilogue_tile(const GemmParams &p, uint32_t tacc, int grow, bool val
         }
       }
     }
-  } else if constexpr (EPI == EPI_QROPE) {
-    rope_store<TBN>(p, tacc, grow, valid, reinterpret_cast<__nv_bfloat16 *>(p.out), p.ldo, p.bias,
-                    tile_n0, p.N);
-  } else if constexpr (EPI == EPI_BF16) {
-    plain_store<TBN>(tacc, grow, valid, reinterpret_cast<__nv_bfloat16 *>(p.out), p.ldo, p.bias,
-                     tile_n0, p.N);
+  } else if constexpr (EPI == EPI_QROPE) {   // kv_fp8: the K rows of an e4m3 cache
+    if (p.kv_fp8)
+      rope_store<TBN, true>(p, tacc, grow, valid, p.out, p.ldo, p.bias, tile_n0, p.N, p.k_qscale);
+    else
+      rope_store<TBN>(p, tacc, grow, valid, p.out, p.ldo, p.bias, tile_n0, p.N);
+  } else if constexpr (EPI == EPI_BF16) {    // kv_fp8: the V rows of an e4m3 cache
+    if (p.kv_fp8)
+      plain_store<TBN, true>(tacc, grow, valid, p.out, p.ldo, p.bias, tile_n0, p.N, p.v_qscale);
+    else
+      plain_store<TBN>(tacc, grow, valid, p.out, p.ldo, p.bias, tile_n0, p.N);
   } else if constexpr (EPI == EPI_QKV) {
     // fused projections: column tiles [0, nq) are Q, [nq, nq+nk) K, the rest V
     const int nq = p.n_q_tiles, nk = p.n_k_tiles;
     if (nt < nq)
-      rope_store<TBN>(p, tacc, grow, valid, reinterpret_cast<__nv_bfloat16 *>(p.out), p.ldo,
-                      p.bias, nt * TBN, nq * TBN);
+      rope_store<TBN>(p, tacc, grow, valid, p.out, p.ldo, p.bias, nt * TBN, nq * TBN);
+    else if (nt < nq + nk && p.kv_fp8)
+      rope_store<TBN, true>(p, tacc, grow, valid, p.out_k, p.ldo_kv, p.bias_k, (nt - nq) * TBN,
+                            nk * TBN, p.k_qscale);
     else if (nt < nq + nk)
-      rope_store<TBN>(p, tacc, grow, valid, reinterpret_cast<__nv_bfloat16 *>(p.out_k), p.ldo_kv,
-                      p.bias_k, (nt - nq) * TBN, nk * TBN);
+      rope_store<TBN>(p, tacc, grow, valid, p.out_k, p.ldo_kv, p.bias_k, (nt - nq) * TBN,
+                      nk * TBN);
+    else if (p.kv_fp8)
+      plain_store<TBN, true>(tacc, grow, valid, p.out_v, p.ldo_kv, p.bias_v, (nt - nq - nk) * TBN,
+                             nk * TBN, p.v_qscale);
     else
-      plain_store<TBN>(tacc, grow, valid, reinterpret_cast<__nv_bfloat16 *>(p.out_v), p.ldo_kv,
-                       p.bias_v, (nt - nq - nk) * TBN, nk * TBN);
+      plain_store<TBN>(tacc, grow, valid, p.out_v, p.ldo_kv, p.bias_v, (nt - nq - nk) * TBN,
+                       nk * TBN);
   } else if constexpr (EPI == EPI_SWIGLU) {
     // columns [0,128) = gate rows nt*128.., [128,256) = up rows nt*128..
     __nv_bfloat16 *out = reinterpret_cast<__nv_bfloat16 *>(p.out) + (size_t)grow * p.ldo;

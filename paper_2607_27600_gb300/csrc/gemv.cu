@@ -294,9 +294,16 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
             }
             float c, sn;
             rope_cs((uint32_t)p.pos[row], p.turns[n1 % p.head_dim], c, sn);
-            __nv_bfloat16 *o = reinterpret_cast<__nv_bfloat16 *>(sg.out) + (size_t)row * sg.ldo;
-            o[n1] = __float2bfloat16_rn(a1 * c - a2 * sn);
-            o[n2] = __float2bfloat16_rn(a2 * c + a1 * sn);
+            const float y1 = a1 * c - a2 * sn, y2 = a2 * c + a1 * sn;
+            if (sg.fp8) {
+              uint8_t *o = reinterpret_cast<uint8_t *>(sg.out) + (size_t)row * sg.ldo;
+              o[n1] = (uint8_t)pack_e4m3x2(y1 * sg.qscale, 0.f);
+              o[n2] = (uint8_t)pack_e4m3x2(y2 * sg.qscale, 0.f);
+            } else {
+              __nv_bfloat16 *o = reinterpret_cast<__nv_bfloat16 *>(sg.out) + (size_t)row * sg.ldo;
+              o[n1] = __float2bfloat16_rn(y1);
+              o[n2] = __float2bfloat16_rn(y2);
+            }
           } else if (sg.epi == GEMV_SWIGLU) {
             const int u = gl * 8 + j;
             if (u < sg.N)
@@ -310,8 +317,12 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
               reinterpret_cast<float *>(sg.out)[(size_t)row * sg.ldo + u] += v;
             } else {
               const float bb = sg.bias ? __bfloat162float(sg.bias[u]) : 0.f;
-              reinterpret_cast<__nv_bfloat16 *>(sg.out)[(size_t)row * sg.ldo + u] =
-                  __float2bfloat16_rn(v + bb);
+              if (sg.fp8)
+                reinterpret_cast<uint8_t *>(sg.out)[(size_t)row * sg.ldo + u] =
+                    (uint8_t)pack_e4m3x2((v + bb) * sg.qscale, 0.f);
+              else
+                reinterpret_cast<__nv_bfloat16 *>(sg.out)[(size_t)row * sg.ldo + u] =
+                    __float2bfloat16_rn(v + bb);
             }
           }
         }

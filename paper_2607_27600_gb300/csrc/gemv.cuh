@@ -40,6 +40,8 @@ struct GemvSeg {
   int ldo;
   int N, epi;
   int groups, group0;         // this segment's row groups: [group0, group0 + groups)
+  int fp8;                    // ROPE, BF16: out is an e4m3 cache (bytes, value * qscale)
+  float qscale;
 };
 
 struct GemvParams {
