@@ -155,7 +155,7 @@ class ClockSampler:
 # workload setup
 # ---------------------------------------------------------------------------
 
-def make_inputs(wl, device):
+def make_inputs(wl, device, kv_fp8=False):
     """Weights and cache of the workload on `device` (seeded synthetic)."""
     shape = wl.shape
     fast = wl.mode == "layer"
@@ -164,31 +164,53 @@ def make_inputs(wl, device):
     # the refresh compacts every layer's cache; the fast pass reads only the last layer's
     cache = synth.synthetic_cache(shape, wl.seq_lens, wl.cap, wl.seed, device=device,
                                   with_h_last=fast)
+    if kv_fp8:
+        to_e4m3_cache(cache)
     return w, cache
 
 
+def to_e4m3_cache(cache, headroom=2.0):
+    """The synthetic cache stored as e4m3 codes: per layer and tensor scale =
+    max |x| * headroom / 448, codes cast by torch (float8_e4m3fn); the scales
+    go to cache["kv_scale"]."""
+    scales = []
+    for l in range(len(cache["k"])):
+        pair = []
+        for key in ("k", "v"):
+            x = cache[key][l].float()
+            sc = max(float(x.abs().max()), 1e-3) * headroom / 448.0
+            cache[key][l] = (x / sc).to(torch.float8_e4m3fn).view(torch.uint8)
+            pair.append(sc)
+            del x
+        scales.append(tuple(pair))
+    cache["kv_scale"] = scales
+    return cache
+
+
 def clone_cache(c):
-    return {k: ([x.clone() if x is not None else None for x in v] if isinstance(v, list)
-                else (v.clone() if v is not None else None)) for k, v in c.items()}
+    def cl(x):
+        return x.clone() if isinstance(x, torch.Tensor) else x
+    return {k: ([cl(x) for x in v] if isinstance(v, list) else cl(v)) for k, v in c.items()}
 
 
 def restore_cache(dst, src):
     for k, v in src.items():
         if isinstance(v, list):
             for a, b in zip(dst[k], v):
-                if a is not None:
+                if isinstance(a, torch.Tensor):
                     a.copy_(b, non_blocking=True)
-        elif v is not None:
+        elif isinstance(v, torch.Tensor):
             dst[k].copy_(v, non_blocking=True)
 
 
-def algorithmic_work(wl):
-    """Per-launch algorithmic FLOPs / bytes of each kernel kind for one step."""
+def algorithmic_work(wl, kv_bytes=2):
+    """Per-launch algorithmic FLOPs / bytes of each kernel kind for one step
+    (kv_bytes: bytes per cached K/V element, 1 for the e4m3 cache)."""
     s = wl.shape
     n_rows = sum(wl.seq_lens)
     d, qd, f, hq, dh = s.d_model, s.q_dim, s.d_ff, s.n_q_heads, s.head_dim
     pairs = sum(n * (n - 1) for n in wl.seq_lens)          # 2 x (pairs j > i)
-    kv_row = s.kv_dim * 2
+    kv_row = s.kv_dim * kv_bytes
     moved = sum(max(0, min(b, n)) for b, n in zip(wl.budgets, wl.seq_lens))
     n_arrays_kv = 2 * s.n_layers
     h_row = d * 2 if wl.mode == "layer" else 0
@@ -248,7 +270,7 @@ def run_ours(args, dist):
     if wl.cycles > 1 and not args.single_cycle:
         raise SystemExit("multi-cycle workloads: use --single-cycle (the first refresh is timed)")
 
-    w, pristine = make_inputs(wl, dev)
+    w, pristine = make_inputs(wl, dev, args.kv_fp8)
     work = clone_cache(pristine)
     weights, cache = pkg.Weights(w), pkg.Cache(work)
     b, cap = wl.batch, wl.cap
@@ -386,7 +408,7 @@ def run_ours(args, dist):
 
     # ---- roofline of the dominant kernel (and a per-kernel table)
     peaks, peak_src = load_peaks()
-    work_tbl = algorithmic_work(wl)
+    work_tbl = algorithmic_work(wl, 1 if args.kv_fp8 else 2)
     if scorer in ("importance", "h2o"):
         work_tbl["keyattn"] = keyattn_work(wl, scorer, recent)
     table = {}
@@ -427,6 +449,7 @@ def run_ours(args, dist):
         "higher_is_better": True, "scaling": "weak", "vs_baseline": vs_baseline, "dtype": "bf16",
         "data": "synthetic (seeded random-init weights N(0,0.02); synthetic KV cache)",
         "config": {"workload": wl.name, "scorer": scorer,
+                   "kv_cache": "e4m3 (per-layer scales)" if args.kv_fp8 else "bf16",
                    "pass": ("fast single-layer" if fast else f"full {shape.n_layers}-layer")
                    if scorer == "counter-causal" else
                    {"recency": "position", "importance": "last-layer key attention",
@@ -499,12 +522,22 @@ def host_inputs(wl, w, cache):
             lw[l] = {k: f32(v) for k, v in x.items()}
     wn = {"embed": f32(w["embed"]), "final_norm": f32(w["final_norm"]),
           "lm_head": f32(w["lm_head"]), "layers": lw}
-    kf = [f32(cache["k"][l]) if (not fast or l == last) else None for l in range(wl.shape.n_layers)]
-    vf = [f32(cache["v"][l]) if (not fast or l == last) else None for l in range(wl.shape.n_layers)]
+    sc = cache.get("kv_scale")
+    if sc is not None:   # e4m3 cache: the oracle gets the codes' values
+        import oracle
+
+        def kvf(key, l):
+            return oracle.e4m3_decode(cache[key][l].cpu().numpy()) * sc[l][0 if key == "k" else 1]
+    else:
+        def kvf(key, l):
+            return f32(cache[key][l])
+    kf = [kvf("k", l) if (not fast or l == last) else None for l in range(wl.shape.n_layers)]
+    vf = [kvf("v", l) if (not fast or l == last) else None for l in range(wl.shape.n_layers)]
     cn = {"k": kf, "v": vf, "tokens": cache["tokens"].cpu().numpy(), "pos": cache["pos"].cpu().numpy(),
           "seq_len": cache["seq_len"].cpu().numpy(), "h_last": f32(cache["h_last"])}
-    raw = {"k": [x.view(torch.int16).cpu().numpy() for x in cache["k"]],
-           "v": [x.view(torch.int16).cpu().numpy() for x in cache["v"]],
+    kv_raw = torch.uint8 if sc is not None else torch.int16
+    raw = {"k": [x.view(kv_raw).cpu().numpy() for x in cache["k"]],
+           "v": [x.view(kv_raw).cpu().numpy() for x in cache["v"]],
            "h": None if cache["h_last"] is None else cache["h_last"].view(torch.int16).cpu().numpy()}
     return wn, cn, raw
 
@@ -676,6 +709,8 @@ def run_append(args, dist):
     cap = j + h
     w = synth.model_weights(shape, wl.seed, device=dev, with_kv_proj=True)
     cache = synth.synthetic_cache(shape, [j], cap, wl.seed, device=dev)
+    if args.kv_fp8:
+        to_e4m3_cache(cache)
     chunk = synth.tokens((1, h), shape.vocab, wl.seed, "bench.chunk", dev)
     count = torch.tensor([h], dtype=torch.int32, device=dev)
     weights, kc = pkg.Weights(w), pkg.Cache(cache)
@@ -753,6 +788,7 @@ def run_append(args, dist):
         "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (seeded random-init weights N(0,0.02); synthetic memory K/V)",
         "config": {"workload": wl.name + "/append", "memory_slots": j, "chunk": h,
+                   "kv_cache": "e4m3 (per-layer scales)" if args.kv_fp8 else "bf16",
                    "layers": shape.n_layers, "d_model": shape.d_model,
                    "heads": f"{shape.n_q_heads}/{shape.n_kv_heads}x{shape.head_dim}",
                    "d_ff": shape.d_ff, "step_tflop": round(flops / 1e12, 3),
@@ -793,6 +829,8 @@ def run_decode(args, dist):
     cap = j + args.warmup + 4 * args.steps + 16
     w = synth.model_weights(shape, wl.seed, device=dev, with_kv_proj=True)
     cache = synth.synthetic_cache(shape, [j], cap, wl.seed, device=dev)
+    if args.kv_fp8:
+        to_e4m3_cache(cache)
     weights, kc = pkg.Weights(w), pkg.Cache(cache)
     ws = cc.alloc_workspace(cc.cc_decode_workspace_size(shape, 1, cap), dev)
     tok = [torch.tensor([1], dtype=torch.int32, device=dev),
@@ -863,7 +901,7 @@ def run_decode(args, dist):
     work = {"gemm_qkv": ("hbm", 2.0 * d * (qd + 2 * kvd)), "gemm_oproj": ("hbm", 2.0 * qd * d),
             "gemm_gateup": ("hbm", 4.0 * d * f), "gemm_down": ("hbm", 2.0 * f * d),
             "gemm_lmhead": ("hbm", 2.0 * shape.vocab * d),
-            "attention_causal": ("hbm", 2.0 * 2 * kvd * n_mid)}
+            "attention_causal": ("hbm", 2.0 * (1 if args.kv_fp8 else 2) * kvd * n_mid)}
     table = kernel_table(kernels, args.steps, work, peaks)
     dom = max(kernels.items(), key=lambda kv: kv[1][1])[0]
     dd = table[dom]
@@ -874,6 +912,7 @@ def run_decode(args, dist):
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (seeded random-init weights N(0,0.02); synthetic memory K/V)",
         "config": {"workload": wl.name + "/decode", "memory_slots": j, "batch": 1,
+                   "kv_cache": "e4m3 (per-layer scales)" if args.kv_fp8 else "bf16",
                    "layers": shape.n_layers, "d_model": shape.d_model, "vocab": shape.vocab,
                    "l2": "weights (15 GB) far exceed L2: every step streams them from HBM",
                    "launch": "one captured graph per step (cc_graph_launch)",
@@ -927,6 +966,8 @@ def main():
     ap.add_argument("--cpu-rows", type=int, default=256)
     ap.add_argument("--ref-rows", type=int, default=32)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--kv-fp8", action="store_true",
+                    help="store the cache's K/V as e4m3 codes with per-layer scales")
     ap.add_argument("--scorer", choices=["counter-causal", "recency", "importance", "h2o"],
                     default="counter-causal",
                     help="refresh scorer: the paper's (default) or one of its comparison "

@@ -105,7 +105,12 @@ struct AttnSmem {
   static constexpr int NH = DH / 64;                 // 64-element (128-byte) column halves
   static constexpr int Q_BYTES = NH * 256 * 128;     // 256 rows
   static constexpr int KV_BYTES = NH * BKV * 128;    // one K (or V) tile (2-byte elements)
-  static constexpr int STG_BYTES = FP8 ? BKV * DH : 0;   // one fp8 K (or V) tile, unswizzled
+  // FP8, head_dim 128: the fp8 tile lands in the upper half of its own f16
+  // stage and is expanded in place (no staging); head_dim 64: one staging
+  // buffer per K and V
+  static constexpr bool IN_PLACE = FP8 && DH == 128;
+  static constexpr int FP8_TILE = BKV * DH;            // bytes of one fp8 K (or V) tile
+  static constexpr int STG_BYTES = (FP8 && !IN_PLACE) ? FP8_TILE : 0;
   static constexpr int OFF_Q = 0;
   static constexpr int OFF_K = OFF_Q + Q_BYTES;
   static constexpr int OFF_V = OFF_K + KST * KV_BYTES;
@@ -183,7 +188,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t *stg_full = o_done + 2;         // [2] FP8: fp8 K / V tile in the staging buffer
   uint64_t *stg_empty = stg_full + 2;      // [2] FP8: staging converted (free)
   uint64_t *q_conv = stg_empty + 2;        // FP8: Q converted to f16
-  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(q_conv + 1);
+  uint64_t *k_load = q_conv + 1;           // [KST] FP8 in place: fp8 K tile in stage s
+  uint64_t *v_load = k_load + KST;         // [KST] FP8 in place: fp8 V tile in stage s
+  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(v_load + KST);
   volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -243,6 +250,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_init(&stg_empty[i], 64);
       }
       mbar_init(q_conv, 64);
+      for (int s = 0; s < KST; ++s) {
+        mbar_init(&k_load[s], 1);
+        mbar_init(&v_load[s], 1);
+      }
     }
     for (int h = 0; h < 2; ++h) {
       mbar_init(&s_ready[h], 1);
@@ -281,7 +292,31 @@ __global__ void __launch_bounds__(kThreads, 1)
         tma_load_3d(smem + L::OFF_Q + hh * 256 * 128, &tmQ, q_full, hh * 64, g * G,
                     (int)row_base + p0);
     }
-    if constexpr (FP8) {
+    if constexpr (L::IN_PLACE) {
+      // fp8 tiles into the upper half of their own stage (converted in place)
+      for (int it = 0; it < ntiles; ++it) {
+        const int t = t_hi - it, s = it % KST;
+        const uint32_t ph = (it / KST) & 1;
+        const int krow = (int)row_base + t * BKV;
+        int ok = 1;
+        if (lane == 0) {
+          ok = mbar_wait(&k_empty[s], ph ^ 1, abort_flag, p.status);
+          if (ok) {
+            mbar_arrive_expect_tx(&k_load[s], L::FP8_TILE);
+            tma_load_3d(smem + L::OFF_K + s * L::KV_BYTES + L::KV_BYTES / 2, &tmK, &k_load[s], 0, g,
+                        krow);
+            ok = mbar_wait(&v_empty[s], ph ^ 1, abort_flag, p.status);
+          }
+          if (ok) {
+            mbar_arrive_expect_tx(&v_load[s], L::FP8_TILE);
+            tma_load_3d(smem + L::OFF_V + s * L::KV_BYTES + L::KV_BYTES / 2, &tmV, &v_load[s], 0, g,
+                        krow);
+          }
+        }
+        ok = __shfl_sync(0xFFFFFFFFu, ok, 0);
+        if (!ok) break;
+      }
+    } else if constexpr (FP8) {
       // fp8 tiles into the one staging buffer; the converters fill the stages
       for (int it = 0; it < ntiles; ++it) {
         const int t = t_hi - it;
@@ -464,7 +499,45 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       fence_proxy_async_smem();
     };
-    for (int it = 0; ok && it < ntiles; ++it) {
+    // head_dim 128 in place: the fp8 tile sits in the stage's upper 16 KB
+    // (row r = 128 bytes at 16K + 128 r); 8 lanes own a row, lane j its bytes
+    // 16j..16j+15 (dims 16j..16j+15).  The f16 row r of the upper column
+    // half occupies exactly the bytes of fp8 row r, so the 8 lanes read the
+    // whole row before any of them writes (syncwarp); rows are split between
+    // the two warps, so no other warp touches them.
+    auto convert_in_place = [&](uint8_t *base, int zero_from) {
+      const int j = ct & 7;
+      const int hh = j >> 2, c = (j & 3) * 2;
+      for (int r = ct >> 3; r < BKV; r += 8) {
+        const uint4 x = *reinterpret_cast<const uint4 *>(base + L::KV_BYTES / 2 + r * 128 + j * 16);
+        __syncwarp();
+        uint4 a = make_uint4(0, 0, 0, 0), b = make_uint4(0, 0, 0, 0);
+        if (r < zero_from) {
+          a = make_uint4(e4m3x2_to_f16x2(x.x), e4m3x2_to_f16x2(x.x >> 16), e4m3x2_to_f16x2(x.y),
+                         e4m3x2_to_f16x2(x.y >> 16));
+          b = make_uint4(e4m3x2_to_f16x2(x.z), e4m3x2_to_f16x2(x.z >> 16), e4m3x2_to_f16x2(x.w),
+                         e4m3x2_to_f16x2(x.w >> 16));
+        }
+        uint8_t *row = base + hh * BKV * 128 + r * 128;
+        *reinterpret_cast<uint4 *>(row + ((c ^ (r & 7)) << 4)) = a;
+        *reinterpret_cast<uint4 *>(row + (((c + 1) ^ (r & 7)) << 4)) = b;
+      }
+      fence_proxy_async_smem();
+    };
+    if constexpr (L::IN_PLACE) {
+      for (int it = 0; ok && it < ntiles; ++it) {
+        const int t = t_hi - it, s = it % KST;
+        const uint32_t ph = (it / KST) & 1;
+        if (!(ok = mbar_wait(&k_load[s], ph, abort_flag, p.status))) break;
+        convert_in_place(smem + L::OFF_K + s * L::KV_BYTES, BKV);
+        mbar_arrive(&k_full[s]);
+        if (!(ok = mbar_wait(&v_load[s], ph, abort_flag, p.status))) break;
+        const int keep = (t == t_top && n - t * BKV < BKV) ? n - t * BKV : BKV;
+        convert_in_place(smem + L::OFF_V + s * L::KV_BYTES, keep);
+        mbar_arrive(&v_full[s]);
+      }
+    }
+    for (int it = 0; !L::IN_PLACE && ok && it < ntiles; ++it) {
       const int t = t_hi - it, s = it % KST;
       const uint32_t ph = (it / KST) & 1, sp = it & 1;
       if (!(ok = mbar_wait(&stg_full[0], sp, abort_flag, p.status))) break;
