@@ -92,6 +92,12 @@ WORKLOADS = {
     "qwen7b-layer-128k": Workload("qwen7b-layer-128k", QWEN25_7B, "layer", [131072], [8192],
                                   131072 + 4096, seed=4, cache_from_causal_pass=False,
                                   cycles=4, append=4096),
+    # profiling case of the decode kernels: Qwen2.5-7B layer shapes, two layers
+    # (about 1.6 GB of weights with the LM head), 8192 memory slots
+    "qwen7b-2layer-8k": Workload("qwen7b-2layer-8k",
+                                 ModelShape(**{**QWEN25_7B.__dict__, "n_layers": 2}), "layer",
+                                 [8192], [8192], 8192 + 4096, seed=6,
+                                 cache_from_causal_pass=False, append=4096),
 }
 
 # The paper's efficiency benchmark (Table 1): Qwen2.5-7B, a synthetic KV cache
