@@ -153,6 +153,19 @@ typedef struct {
   const float *kv_scale; /* CC_KV_E4M3: HOST array [n_layers][2] = (K scale, V scale) of
                         each layer, finite and > 0; the value of an element is its code
                         times the scale.  Ignored for bf16.                             */
+  /* Paged K/V (NULL block_table: k[l], v[l] are slot-major [batch][cap] buffers).
+   * With a block table, k[l] and v[l] are page pools [n_pages][page_size][Hkv][head_dim]
+   * and logical slot i of sequence b lives at pool row
+   *   block_table[b * (cap / page_size) + i / page_size] * page_size + i % page_size.
+   * page_size is a multiple of 128 and divides cap; every entry a sequence uses
+   * (slots below cap) names a distinct page in [0, n_pages) (an entry outside that range
+   * is reported as CC_ERR_DEVICE_ARG on the device and its rows are skipped).  Only K
+   * and V are paged: tokens, pos, h_last and h2o_acc stay [batch][cap].  The compaction
+   * moves rows between the pages of a sequence and leaves the table as it is: pages past
+   * the new length are the caller's to reuse. */
+  const int32_t *block_table; /* device int32 [batch][cap / page_size], or NULL          */
+  int32_t page_size;
+  int32_t n_pages;
 } cc_kv_cache;
 
 /* ---- scoring (Sec. 3.1) ---------------------------------------------------

@@ -62,7 +62,9 @@ class cc_kv_cache(ctypes.Structure):
                 ("v", ctypes.POINTER(ctypes.c_void_p)), ("tokens", ctypes.c_void_p),
                 ("pos", ctypes.c_void_p), ("h_last", ctypes.c_void_p),
                 ("h2o_acc", ctypes.c_void_p), ("kv_format", ctypes.c_int32),
-                ("kv_scale", ctypes.POINTER(ctypes.c_float))]
+                ("kv_scale", ctypes.POINTER(ctypes.c_float)),
+                ("block_table", ctypes.c_void_p), ("page_size", ctypes.c_int32),
+                ("n_pages", ctypes.c_int32)]
 
 KV_BF16, KV_E4M3 = 0, 1
 
@@ -223,7 +225,9 @@ class Cache:
     """cc_kv_cache over a dict of CUDA tensors (k[l], v[l] bf16 [B, cap, Hkv, dh],
     or e4m3 codes (uint8) when the dict holds "kv_scale": per layer the (K, V)
     scales; tokens, pos int32 [B, cap]; seq_len int32 [B]; h_last bf16
-    [B, cap, d] or None); keeps the tensors alive."""
+    [B, cap, d] or None); with "block_table" (int32 [B, cap // page_size]),
+    "page_size" and k[l], v[l] page pools [n_pages, page_size, Hkv, dh] the
+    K/V are paged.  Keeps the tensors alive."""
 
     def __init__(self, c: dict):
         self.d = c
@@ -239,10 +243,15 @@ class Cache:
                 raise ValueError("kv_scale needs one (K, V) pair per layer")
             self._scale = (ctypes.c_float * len(flat))(*flat)
             fmt = KV_E4M3
+        table, page, n_pages = c.get("block_table"), 0, 0
+        if table is not None:
+            page = int(c["page_size"])
+            n_pages = int(next(x for x in ks if x is not None).shape[0])
         self.c = cc_kv_cache(b, cap, _dev_ptr(c["seq_len"], "seq_len"), self._k, self._v,
                              _dev_ptr(c["tokens"], "tokens"), _dev_ptr(c["pos"], "pos"),
                              _dev_ptr(c.get("h_last"), "h_last"),
-                             _dev_ptr(c.get("h2o_acc"), "h2o_acc"), fmt, self._scale)
+                             _dev_ptr(c.get("h2o_acc"), "h2o_acc"), fmt, self._scale,
+                             _dev_ptr(table, "block_table"), page, n_pages)
 
 
 def _cfg(cfg):

@@ -174,10 +174,28 @@ cc_status check_cfg(const cc_model_cfg *c) {
 
 size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
-// Element format of layer l's cached K/V.
+// Paging of the cache's K/V (table nullptr: slot-major [batch][cap]) and the
+// rows of the K/V buffers (the pool, or batch * cap).
+KvPaging kv_paging(const cc_kv_cache *kv) {
+  KvPaging pg{};
+  if (kv->block_table) {
+    pg.table = kv->block_table;
+    pg.page = kv->page_size;
+    pg.pages_per_seq = kv->cap / kv->page_size;
+    pg.n_pages = kv->n_pages;
+  }
+  return pg;
+}
+uint64_t kv_buffer_rows(const cc_kv_cache *kv) {
+  return kv->block_table ? (uint64_t)kv->n_pages * kv->page_size : (uint64_t)kv->batch * kv->cap;
+}
+
+// Element format and layout of layer l's cached K/V.
 struct KvFmt {
   bool fp8 = false;
   float k_scale = 1.f, v_scale = 1.f;
+  KvPaging pg{};        // paged K/V (table nullptr: slot-major)
+  uint64_t rows = 0;    // rows of the K/V buffers (0: batch * cap)
 };
 KvFmt kv_fmt(const cc_kv_cache *kv, int l) {
   KvFmt f;
@@ -186,6 +204,8 @@ KvFmt kv_fmt(const cc_kv_cache *kv, int l) {
     f.k_scale = kv->kv_scale[2 * l];
     f.v_scale = kv->kv_scale[2 * l + 1];
   }
+  f.pg = kv_paging(kv);
+  f.rows = kv_buffer_rows(kv);
   return f;
 }
 int kv_elem_bytes(const cc_kv_cache *kv) { return kv->kv_format == CC_KV_E4M3 ? 1 : 2; }
@@ -193,6 +213,11 @@ int kv_elem_bytes(const cc_kv_cache *kv) { return kv->kv_format == CC_KV_E4M3 ? 
 // The cache's format fields: a known format; e4m3 needs finite positive
 // scales for every layer.
 bool kv_format_ok(const cc_model_cfg *c, const cc_kv_cache *kv) {
+  if (kv->block_table) {   // pages of whole 128-slot key tiles that divide cap
+    if (kv->page_size < 128 || kv->page_size % 128 || kv->cap % kv->page_size ||
+        kv->n_pages < 1 || (uint64_t)kv->n_pages * kv->page_size >= (1ull << 31))
+      return false;
+  }
   if (kv->kv_format == CC_KV_BF16) return true;
   if (kv->kv_format != CC_KV_E4M3 || !kv->kv_scale) return false;
   for (int i = 0; i < 2 * c->n_layers; ++i)
@@ -463,8 +488,9 @@ cc_status run_attention(const cc_model_cfg *c, const void *q, const void *k, con
     const uint32_t box[3] = {64, (uint32_t)G, (uint32_t)P};
     if (!make_tmap(&tq, q, 3, dims, strides, box)) return tmap_fail();
   }
+  const uint64_t RK = kvf.rows ? kvf.rows : R;   // K/V buffer rows (paged: the pool)
   if (kvf.fp8) {   // e4m3 bytes, one unswizzled box per 128-key tile (converted in the kernel)
-    const uint64_t dims[3] = {(uint64_t)dh, (uint64_t)c->n_kv_heads, R};
+    const uint64_t dims[3] = {(uint64_t)dh, (uint64_t)c->n_kv_heads, RK};
     const uint64_t strides[2] = {(uint64_t)dh, (uint64_t)c->n_kv_heads * dh};
     const uint32_t box[3] = {(uint32_t)dh, 1, 128};
     if (!make_tmap(&tk, k, 3, dims, strides, box, CU_TENSOR_MAP_SWIZZLE_NONE,
@@ -473,7 +499,7 @@ cc_status run_attention(const cc_model_cfg *c, const void *q, const void *k, con
                    CU_TENSOR_MAP_DATA_TYPE_UINT8))
       return tmap_fail();
   } else {
-    const uint64_t dims[3] = {(uint64_t)dh, (uint64_t)c->n_kv_heads, R};
+    const uint64_t dims[3] = {(uint64_t)dh, (uint64_t)c->n_kv_heads, RK};
     const uint64_t strides[2] = {(uint64_t)dh * 2, (uint64_t)c->n_kv_heads * dh * 2};
     const uint32_t box[3] = {64, 1, 128};
     if (!make_tmap(&tk, k, 3, dims, strides, box)) return tmap_fail();
@@ -496,6 +522,8 @@ cc_status run_attention(const cc_model_cfg *c, const void *q, const void *k, con
   p.scale_log2 = (float)(1.4426950408889634 / sqrt((double)dh) * kvf.k_scale);
   p.kv_fp8 = kvf.fp8 ? 1 : 0;
   p.v_scale = kvf.v_scale;
+  p.pg = kvf.pg;
+  p.kv_rows = (int)RK;
   p.status = status;
   p.causal = row_lo ? 1 : 0;
   p.row_lo = row_lo;
@@ -700,10 +728,12 @@ cc_status run_append(const cc_model_cfg *c, const cc_model_weights *w, const cc_
       g.add(lw.wq, nullptr, lw.bq, q, qd, qd, GEMV_ROPE);
       g.add(lw.wk, nullptr, lw.bk, kv->k[l], kvd, kvd, GEMV_ROPE);
       g.add(lw.wv, nullptr, lw.bv, kv->v[l], kvd, kvd, GEMV_BF16);
-      for (int j = 1; j < 3; ++j) {
+      for (int j = 1; j < 3; ++j) {   // K and V into the cache (e4m3 codes; paged rows)
         g.l.p.seg[j].fp8 = kvf.fp8 ? 1 : 0;
         g.l.p.seg[j].qscale = 1.f / (j == 1 ? kvf.k_scale : kvf.v_scale);
+        g.l.p.seg[j].kv_dest = 1;
       }
+      g.l.p.pg = kvf.pg;
       if ((s = run_gemv(g, CC_KERNEL_GEMM_QKV, dev->sms, st)) != CC_OK) return s;
     } else {
       TimedScope t(CC_KERNEL_RMSNORM, st);
@@ -723,6 +753,7 @@ cc_status run_append(const cc_model_cfg *c, const cc_model_weights *w, const cc_
       g.p.kv_fp8 = kvf.fp8 ? 1 : 0;
       g.p.k_qscale = 1.f / kvf.k_scale;
       g.p.v_qscale = 1.f / kvf.v_scale;
+      g.p.pg = kvf.pg;
       if ((s = run_gemm(g, EPI_QKV, CC_KERNEL_GEMM_QKV, dev->sms, st)) != CC_OK) return s;
     }
     struct Proj { const void *w, *bias; void *out; int n, epi, kind; };
@@ -742,6 +773,8 @@ cc_status run_append(const cc_model_cfg *c, const cc_model_weights *w, const cc_
       g.p.bias = reinterpret_cast<const __nv_bfloat16 *>(pj.bias);
       g.p.head_dim = c->head_dim;
       if (pj.kind == CC_KERNEL_GEMM_KV) {   // K or V rows into the cache
+        g.p.kv_dest = 1;
+        g.p.pg = kvf.pg;
         g.p.kv_fp8 = kvf.fp8 ? 1 : 0;
         g.p.k_qscale = 1.f / kvf.k_scale;
         g.p.v_qscale = 1.f / kvf.v_scale;
@@ -983,13 +1016,14 @@ cc_status compact_plan(const cc_model_cfg *c, const cc_kv_cache *kv, CompactPlan
     p.class_chunks[p.n_classes] = (kv->cap + rows - 1) / rows;
     return p.n_classes++;
   };
-  auto add = [&](void *base, int row_bytes, bool bulk) -> bool {
+  auto add = [&](void *base, int row_bytes, bool bulk, bool paged = false) -> bool {
     if (!base) return true;
     if (n >= kMaxCompactArrays || !aligned16(base)) return false;
     CompactArray &A = p.arr[n++];
     A.base = base;
     A.row_bytes = row_bytes;
     A.bulk = bulk ? 1 : 0;
+    A.paged = paged ? 1 : 0;
     A.rows_per_chunk = bulk ? (row_bytes <= p.stage_bytes ? p.stage_bytes / row_bytes : 0)
                             : p.stage_bytes / 4;
     if (A.rows_per_chunk < 1) return false;
@@ -1003,8 +1037,11 @@ cc_status compact_plan(const cc_model_cfg *c, const cc_kv_cache *kv, CompactPlan
   // staging shape of the copy kernel for the largest row moved
   const int max_row = std::max(kv_row, kv->h_last ? c->d_model * 2 : 0);
   if (!compact_shape(max_row, p.stage_bytes, p.warps)) return CC_ERR_UNSUPPORTED;
+  p.pg = kv_paging(kv);   // K/V rows through the block table when paged
+  const bool paged = kv->block_table != nullptr;
   for (int l = 0; l < c->n_layers; ++l) {
-    if (!add(kv->k[l], kv_row, true) || !add(kv->v[l], kv_row, true)) return CC_ERR_UNSUPPORTED;
+    if (!add(kv->k[l], kv_row, true, paged) || !add(kv->v[l], kv_row, true, paged))
+      return CC_ERR_UNSUPPORTED;
   }
   if (!add(kv->h_last, c->d_model * 2, true)) return CC_ERR_UNSUPPORTED;
   if (!add(kv->tokens, 4, false) || !add(kv->pos, 4, false)) return CC_ERR_INVALID_ARG;
@@ -1070,12 +1107,16 @@ cc_status run_keyattn(const cc_model_cfg *c, const cc_kv_cache *kv, int l0, int 
   static std::mutex mu;
   std::lock_guard<std::mutex> lk(mu);
   memset(&a, 0, sizeof(a));
-  const uint64_t dims[3] = {(uint64_t)dh, (uint64_t)c->n_kv_heads, R};
+  const uint64_t RK = kv_buffer_rows(kv);   // K buffer rows (paged: the pool)
+  (void)R;
+  const uint64_t dims[3] = {(uint64_t)dh, (uint64_t)c->n_kv_heads, RK};
   const uint64_t strides[2] = {(uint64_t)dh * 2, (uint64_t)c->n_kv_heads * dh * 2};
   const uint32_t box[3] = {64, 1, 128};
   for (int l = l0; l < l1; ++l)
     if (!make_tmap(&a.k[l - l0], kv->k[l], 3, dims, strides, box)) return tmap_fail();
   KeyAttnParams &p = a.p;
+  p.pg = kv_paging(kv);
+  p.kv_rows = (int)RK;
   p.batch = batch;
   p.cap = cap;
   p.n_kv_heads = c->n_kv_heads;
@@ -1104,6 +1145,7 @@ cc_status check_keyattn_args(const cc_model_cfg *c, const cc_kv_cache *kv, void 
   if ((uint64_t)kv->batch * kv->cap >= (1ull << 31)) return CC_ERR_UNSUPPORTED;
   if (c->n_layers > kKeyAttnMaxLayers) return CC_ERR_UNSUPPORTED;
   if (kv->kv_format != CC_KV_BF16) return CC_ERR_UNSUPPORTED;   // bf16 keys only
+  if (!kv_format_ok(c, kv)) return CC_ERR_INVALID_ARG;
   for (int l = l0; l < c->n_layers; ++l)
     if (!kv->k[l] || !aligned16(kv->k[l])) return CC_ERR_INVALID_ARG;
   if (!ws || !aligned16(ws) || ws_bytes < cc_keyattn_workspace_size(c, kv->batch, kv->cap))

@@ -217,6 +217,16 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int ntiles = S > 1 ? (split + 1) * max(ntiles_unit, 0) / S - it_off : ntiles_unit;
   const int t_hi = t1 - it_off;
   const size_t part_slot = ((size_t)unit_id * S + split) * 256;
+  // pool row of key tile t (paged) or b*cap + 128 t; a bad page reads zeros
+  // (a coordinate past the maps) and is reported
+  auto tile_row = [&](int t) -> int {
+    const long long r = kv_row(p.pg, p.cap, b, t * BKV);
+    if (r < 0) {
+      set_status(p.status, CC_ERR_DEVICE_ARG);
+      return p.kv_rows;
+    }
+    return (int)r;
+  };
 
   if (S > 1 && ntiles <= 0) {   // nothing for this split: an empty partial
     for (int R = threadIdx.x; R < 256; R += blockDim.x)
@@ -297,7 +307,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int it = 0; it < ntiles; ++it) {
         const int t = t_hi - it, s = it % KST;
         const uint32_t ph = (it / KST) & 1;
-        const int krow = (int)row_base + t * BKV;
+        const int krow = tile_row(t);
         int ok = 1;
         if (lane == 0) {
           ok = mbar_wait(&k_empty[s], ph ^ 1, abort_flag, p.status);
@@ -321,7 +331,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int it = 0; it < ntiles; ++it) {
         const int t = t_hi - it;
         const uint32_t sp = it & 1;
-        const int krow = (int)row_base + t * BKV;
+        const int krow = tile_row(t);
         int ok = 1;
         if (lane == 0) {
           ok = mbar_wait(&stg_empty[0], sp ^ 1, abort_flag, p.status);
@@ -342,7 +352,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int it = 0; it < ntiles; ++it) {
         const int t = t_hi - it, s = it % KST;   // key tiles from the sequence end downwards
         const uint32_t ph = (it / KST) & 1;
-        const int krow = (int)row_base + t * BKV;
+        const int krow = tile_row(t);
         int ok = 1;
         if (lane == 0) {
           ok = mbar_wait(&k_empty[s], ph ^ 1, abort_flag, p.status);
@@ -933,12 +943,15 @@ __global__ void __launch_bounds__(kDecThreads) attn_decode_kernel(const __grid_c
     uint8_t *kb = smem + buf * L::BUF, *vb = kb + L::K_BYTES;
     // K in DH/8 pieces per row (16 bytes bf16, 8 bytes e4m3), V in 16-byte pieces
     constexpr int KP = DH / 8, KPB = 8 * L::EB, VP = DH * L::EB / 16;
+    // pool row of the chunk's first key (a chunk lies in one page); -1: bad page
+    const long long cbase = kv_row(p.pg, p.cap, u.b, c * kDecChunk);
+    if (cbase < 0 && tid == 0) set_status(p.status, CC_ERR_DEVICE_ARG);
     for (int i = tid; i < kDecChunk * KP; i += kDecThreads) {
       const int r = i / KP, e = i - r * KP;
       const int j = c * kDecChunk + r;
       uint8_t *kd = kb + r * L::K_ROW + e * KPB;
-      if (j < n_keys) {
-        const uint8_t *src = kg + (((row_base + j) * Hkv + u.g) * (size_t)DH) * L::EB + e * KPB;
+      if (j < n_keys && cbase >= 0) {
+        const uint8_t *src = kg + (((size_t)(cbase + r) * Hkv + u.g) * (size_t)DH) * L::EB + e * KPB;
         if constexpr (FP8) cp_async8(kd, src);
         else cp_async16(kd, src);
       } else if constexpr (FP8) {
@@ -951,8 +964,8 @@ __global__ void __launch_bounds__(kDecThreads) attn_decode_kernel(const __grid_c
       const int r = i / VP, e = i - r * VP;
       const int j = c * kDecChunk + r;
       uint8_t *vd = vb + r * L::V_ROW + e * 16;
-      if (j < n_keys)   // past the last key: zeros (P is 0 there, V must be finite)
-        cp_async16(vd, vg + (((row_base + j) * Hkv + u.g) * (size_t)DH) * L::EB + e * 16);
+      if (j < n_keys && cbase >= 0)   // past the last key: zeros (P is 0 there, V must be finite)
+        cp_async16(vd, vg + (((size_t)(cbase + r) * Hkv + u.g) * (size_t)DH) * L::EB + e * 16);
       else
         *reinterpret_cast<uint4 *>(vd) = make_uint4(0, 0, 0, 0);
     }

@@ -202,6 +202,19 @@ __global__ void __launch_bounds__(kThreads)
     return s;
   };
 
+  // Row of slot k of sequence b in array A (paged K/V: the pool row, -1 for
+  // a bad block-table entry, which is reported and its row left alone).
+  auto arow = [&](const CompactArray &A, int b, int k) -> long long {
+    if (!A.paged) return (long long)b * p.cap + k;
+    const long long r = kv_row(p.pg, p.cap, b, k);
+    if (r < 0) set_status(p.status, CC_ERR_DEVICE_ARG);
+    return r;
+  };
+  // A bulk row moves when its source differs and both rows exist.
+  auto moves = [&](const CompactArray &A, int b, int k, int src) {
+    return src != k && (!A.paged || (arow(A, b, k) >= 0 && arow(A, b, src) >= 0));
+  };
+
   // Issues the reads of unit u into buffer slot s.
   auto load = [&](Unit &u, int s) {
     if (u.t >= total || u.k0 >= u.k1) return;
@@ -211,16 +224,16 @@ __global__ void __launch_bounds__(kThreads)
     const size_t seq_off = (size_t)u.b * p.cap;
     if (A.bulk) {
       int moving = 0;
-      for (int k = u.k0 + lane; k < u.k1; k += 32) moving += (source(kidx, k, false) != k);
+      for (int k = u.k0 + lane; k < u.k1; k += 32) moving += moves(A, u.b, k, source(kidx, k, false));
       moving = __reduce_add_sync(0xFFFFFFFFu, moving);
       if (moving == 0) return;
       if (lane == 0) mbar_arrive_expect_tx(&bars[warp][s], (uint32_t)(moving * A.row_bytes));
       __syncwarp();
       for (int k = u.k0 + lane; k < u.k1; k += 32) {
         const int src = source(kidx, k, true);
-        if (src != k)
+        if (moves(A, u.b, k, src))
           bulk_load(buf[s] + (size_t)(k - u.k0) * A.row_bytes,
-                    base + (seq_off + src) * A.row_bytes, A.row_bytes, &bars[warp][s]);
+                    base + (size_t)arow(A, u.b, src) * A.row_bytes, A.row_bytes, &bars[warp][s]);
       }
       u.loaded = true;
     } else {   // 4-byte rows: plain loads staged in shared memory
@@ -280,8 +293,8 @@ __global__ void __launch_bounds__(kThreads)
       if (A.bulk) {
         if (cur.loaded) {
           for (int k = cur.k0 + lane; k < cur.k1; k += 32)
-            if (source(kidx, k, false) != k)
-              bulk_store(base + (seq_off + k) * A.row_bytes,
+            if (moves(A, cur.b, k, source(kidx, k, false)))
+              bulk_store(base + (size_t)arow(A, cur.b, k) * A.row_bytes,
                          buf[s] + (size_t)(k - cur.k0) * A.row_bytes, A.row_bytes);
           bulk_commit();
         }

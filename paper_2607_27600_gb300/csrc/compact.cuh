@@ -24,6 +24,7 @@ struct CompactArray {
   int rows_per_chunk;  // destination slots per unit
   int n_chunks;        // chunks per sequence = ceil(cap / rows_per_chunk) (upper bound of units)
   int dep_class;       // chunk-size class (index into the readers table)
+  int paged;           // bulk K/V arrays of a paged cache: rows through CompactParams::pg
 };
 
 struct CompactParams {
@@ -46,6 +47,7 @@ struct CompactParams {
   int withhold_unit;          // test hook: this unit never publishes its flag (-1: none)
   int stage_bytes;            // shared-memory buffer of a unit (multiple of 128)
   int warps;                  // warps per CTA (each with two buffers)
+  KvPaging pg;                // paged K/V arrays: pool row of logical slot (b, i)
   CompactArray arr[kMaxCompactArrays];
 };
 

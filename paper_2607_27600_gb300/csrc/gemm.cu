@@ -36,13 +36,15 @@ constexpr size_t kSmemBytes = 1024 /*align slack*/ + ST * (A_BYTES + B_BYTES) + 
 // bias (optional) is added before the rotation.
 // F8: the destination is an e4m3 cache (one byte per element, the value
 // times qscale = 1 / the layer's scale; pack_e4m3x2).
+// orow: the output row (grow, or the cache row of a paged K destination; < 0: skip)
 template <int TBN, bool F8 = false>
-CC_DEV void rope_store(const GemmParams &p, uint32_t tacc, int grow, bool valid, void *out_base,
-                       int ldo, const __nv_bfloat16 *bias, int col0, int n_dest,
+CC_DEV void rope_store(const GemmParams &p, uint32_t tacc, int grow, long long orow, bool valid,
+                       void *out_base, int ldo, const __nv_bfloat16 *bias, int col0, int n_dest,
                        float qscale = 1.f) {
   const int half = p.head_dim >> 1;
+  valid = valid && orow >= 0;
   const uint32_t pos = valid ? (uint32_t)p.pos[grow] : 0u;
-  uint8_t *out = reinterpret_cast<uint8_t *>(out_base) + (size_t)grow * ldo * (F8 ? 1 : 2);
+  uint8_t *out = reinterpret_cast<uint8_t *>(out_base) + (size_t)(valid ? orow : 0) * ldo * (F8 ? 1 : 2);
 #pragma unroll 1
   for (int hb = 0; hb < TBN; hb += p.head_dim) {
 #pragma unroll 1
@@ -106,10 +108,11 @@ CC_DEV void rope_store(const GemmParams &p, uint32_t tacc, int grow, bool valid,
 // Plain bf16 store (+ optional bias) of one accumulator tile row; F8: e4m3
 // codes of (value + bias) * qscale instead.
 template <int TBN, bool F8 = false>
-CC_DEV void plain_store(uint32_t tacc, int grow, bool valid, void *out_base, int ldo,
+CC_DEV void plain_store(uint32_t tacc, long long orow, bool valid, void *out_base, int ldo,
                         const __nv_bfloat16 *bias, int col0, int n_dest, float qscale = 1.f) {
   constexpr int EB = F8 ? 1 : 2;
-  uint8_t *out = reinterpret_cast<uint8_t *>(out_base) + (size_t)grow * ldo * EB;
+  valid = valid && orow >= 0;
+  uint8_t *out = reinterpret_cast<uint8_t *>(out_base) + (size_t)(valid ? orow : 0) * ldo * EB;
 #pragma unroll 1
   for (int c = 0; c < TBN / 32; ++c) {
     uint32_t r[32];
@@ -141,6 +144,15 @@ CC_DEV void plain_store(uint32_t tacc, int grow, bool valid, void *out_base, int
     for (int v = 0; v < 2 * EB; ++v)   // 32 elements: 64 bytes bf16, 32 e4m3
       d[v] = make_uint4(o[v * 4], o[v * 4 + 1], o[v * 4 + 2], o[v * 4 + 3]);
   }
+}
+
+// Cache row of workspace row grow = b * cap + i (paged: through the block
+// table); a bad page is reported and the row skipped (-1).
+CC_DEV long long cache_row(const GemmParams &p, int grow, bool valid) {
+  const int b = grow / p.cap;
+  const long long r = kv_row(p.pg, p.cap, b, grow - b * p.cap);
+  if (r < 0 && valid) set_status(p.status, CC_ERR_DEVICE_ARG);
+  return r;
 }
 
 template <int EPI, int TBN>
@@ -187,31 +199,35 @@ CC_DEV void epilogue_tile(const GemmParams &p, uint32_t tacc, int grow, bool val
       }
     }
   } else if constexpr (EPI == EPI_QROPE) {   // kv_fp8: the K rows of an e4m3 cache
+    const long long orow = p.kv_dest ? cache_row(p, grow, valid) : grow;
     if (p.kv_fp8)
-      rope_store<TBN, true>(p, tacc, grow, valid, p.out, p.ldo, p.bias, tile_n0, p.N, p.k_qscale);
+      rope_store<TBN, true>(p, tacc, grow, orow, valid, p.out, p.ldo, p.bias, tile_n0, p.N,
+                            p.k_qscale);
     else
-      rope_store<TBN>(p, tacc, grow, valid, p.out, p.ldo, p.bias, tile_n0, p.N);
+      rope_store<TBN>(p, tacc, grow, orow, valid, p.out, p.ldo, p.bias, tile_n0, p.N);
   } else if constexpr (EPI == EPI_BF16) {    // kv_fp8: the V rows of an e4m3 cache
+    const long long orow = p.kv_dest ? cache_row(p, grow, valid) : grow;
     if (p.kv_fp8)
-      plain_store<TBN, true>(tacc, grow, valid, p.out, p.ldo, p.bias, tile_n0, p.N, p.v_qscale);
+      plain_store<TBN, true>(tacc, orow, valid, p.out, p.ldo, p.bias, tile_n0, p.N, p.v_qscale);
     else
-      plain_store<TBN>(tacc, grow, valid, p.out, p.ldo, p.bias, tile_n0, p.N);
+      plain_store<TBN>(tacc, orow, valid, p.out, p.ldo, p.bias, tile_n0, p.N);
   } else if constexpr (EPI == EPI_QKV) {
-    // fused projections: column tiles [0, nq) are Q, [nq, nq+nk) K, the rest V
+    // fused projections: column tiles [0, nq) are Q, [nq, nq+nk) K, the rest V (cache rows)
     const int nq = p.n_q_tiles, nk = p.n_k_tiles;
+    const long long crow = nt < nq ? grow : cache_row(p, grow, valid);
     if (nt < nq)
-      rope_store<TBN>(p, tacc, grow, valid, p.out, p.ldo, p.bias, nt * TBN, nq * TBN);
+      rope_store<TBN>(p, tacc, grow, grow, valid, p.out, p.ldo, p.bias, nt * TBN, nq * TBN);
     else if (nt < nq + nk && p.kv_fp8)
-      rope_store<TBN, true>(p, tacc, grow, valid, p.out_k, p.ldo_kv, p.bias_k, (nt - nq) * TBN,
-                            nk * TBN, p.k_qscale);
+      rope_store<TBN, true>(p, tacc, grow, crow, valid, p.out_k, p.ldo_kv, p.bias_k,
+                            (nt - nq) * TBN, nk * TBN, p.k_qscale);
     else if (nt < nq + nk)
-      rope_store<TBN>(p, tacc, grow, valid, p.out_k, p.ldo_kv, p.bias_k, (nt - nq) * TBN,
+      rope_store<TBN>(p, tacc, grow, crow, valid, p.out_k, p.ldo_kv, p.bias_k, (nt - nq) * TBN,
                       nk * TBN);
     else if (p.kv_fp8)
-      plain_store<TBN, true>(tacc, grow, valid, p.out_v, p.ldo_kv, p.bias_v, (nt - nq - nk) * TBN,
+      plain_store<TBN, true>(tacc, crow, valid, p.out_v, p.ldo_kv, p.bias_v, (nt - nq - nk) * TBN,
                              nk * TBN, p.v_qscale);
     else
-      plain_store<TBN>(tacc, grow, valid, p.out_v, p.ldo_kv, p.bias_v, (nt - nq - nk) * TBN,
+      plain_store<TBN>(tacc, crow, valid, p.out_v, p.ldo_kv, p.bias_v, (nt - nq - nk) * TBN,
                        nk * TBN);
   } else if constexpr (EPI == EPI_SWIGLU) {
     // columns [0,128) = gate rows nt*128.., [128,256) = up rows nt*128..

@@ -284,6 +284,14 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
           const int j = idx / B, b = idx - j * B;
           const int row = rows[b];
           if (row < 0) continue;
+          long long orow = row;   // K / V cache row (paged: through the block table)
+          if (sg.kv_dest) {
+            orow = kv_row(p.pg, p.cap, b, row - b * p.cap);
+            if (orow < 0) {
+              set_status(p.status, CC_ERR_DEVICE_ARG);
+              continue;
+            }
+          }
           if (sg.epi == GEMV_ROPE) {
             const int half = p.head_dim >> 1;
             const int n1 = box_row(p, sg, gl, 0) + j, n2 = n1 + half;
@@ -296,11 +304,11 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
             rope_cs((uint32_t)p.pos[row], p.turns[n1 % p.head_dim], c, sn);
             const float y1 = a1 * c - a2 * sn, y2 = a2 * c + a1 * sn;
             if (sg.fp8) {
-              uint8_t *o = reinterpret_cast<uint8_t *>(sg.out) + (size_t)row * sg.ldo;
+              uint8_t *o = reinterpret_cast<uint8_t *>(sg.out) + (size_t)orow * sg.ldo;
               o[n1] = (uint8_t)pack_e4m3x2(y1 * sg.qscale, 0.f);
               o[n2] = (uint8_t)pack_e4m3x2(y2 * sg.qscale, 0.f);
             } else {
-              __nv_bfloat16 *o = reinterpret_cast<__nv_bfloat16 *>(sg.out) + (size_t)row * sg.ldo;
+              __nv_bfloat16 *o = reinterpret_cast<__nv_bfloat16 *>(sg.out) + (size_t)orow * sg.ldo;
               o[n1] = __float2bfloat16_rn(y1);
               o[n2] = __float2bfloat16_rn(y2);
             }
@@ -318,10 +326,10 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
             } else {
               const float bb = sg.bias ? __bfloat162float(sg.bias[u]) : 0.f;
               if (sg.fp8)
-                reinterpret_cast<uint8_t *>(sg.out)[(size_t)row * sg.ldo + u] =
+                reinterpret_cast<uint8_t *>(sg.out)[(size_t)orow * sg.ldo + u] =
                     (uint8_t)pack_e4m3x2((v + bb) * sg.qscale, 0.f);
               else
-                reinterpret_cast<__nv_bfloat16 *>(sg.out)[(size_t)row * sg.ldo + u] =
+                reinterpret_cast<__nv_bfloat16 *>(sg.out)[(size_t)orow * sg.ldo + u] =
                     __float2bfloat16_rn(v + bb);
             }
           }

@@ -42,6 +42,7 @@ struct GemvSeg {
   int groups, group0;         // this segment's row groups: [group0, group0 + groups)
   int fp8;                    // ROPE, BF16: out is an e4m3 cache (bytes, value * qscale)
   float qscale;
+  int kv_dest;                // ROPE, BF16: out holds K / V cache rows (through pg when paged)
 };
 
 struct GemvParams {
@@ -57,6 +58,7 @@ struct GemvParams {
   const int32_t *pos;               // ROPE: original positions [batch * cap]
   int head_dim;
   unsigned long long turns[64];     // ROPE: inv_freq_k / (2 pi) in 0.64 fixed point
+  KvPaging pg;                      // paged cache rows of kv_dest segments
   float2 *part;                     // ARGMAX: [batch][part_ld], part_ld = ctas
   int part_ld;
   unsigned *status;

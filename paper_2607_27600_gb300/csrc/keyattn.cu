@@ -97,7 +97,16 @@ __global__ void __launch_bounds__(kThreads)
     t_last = (n - 1) / KT;
   }
   const int ntiles = t_last - t_first + 1;
-  const size_t seq_row = (size_t)b * p.cap;
+  // pool row of the key tile starting at slot i (paged: one page holds it);
+  // a bad page reads zeros (a coordinate past the map) and is reported
+  auto tile_row = [&](int i) -> int {
+    const long long r = kv_row(p.pg, p.cap, b, i);
+    if (r < 0) {
+      set_status(p.status, CC_ERR_DEVICE_ARG);
+      return p.kv_rows;
+    }
+    return (int)r;
+  };
 
   if (threadIdx.x == 0) {
     mbar_init(row_full, 1);
@@ -124,8 +133,7 @@ __global__ void __launch_bounds__(kThreads)
       tma_prefetch_desc(&tmK);
       mbar_arrive_expect_tx(row_full, L::TILE);
       for (int hh = 0; hh < L::NH; ++hh)
-        tma_load_3d(smem + L::OFF_ROW + hh * KT * 128, &tmK, row_full, hh * 64, g,
-                    (int)(seq_row + row0));
+        tma_load_3d(smem + L::OFF_ROW + hh * KT * 128, &tmK, row_full, hh * 64, g, tile_row(row0));
       for (int it = 0; it < ntiles; ++it) {
         const int t = t_first + it, s = it % KST;
         const uint32_t ph = (it / KST) & 1;
@@ -133,7 +141,7 @@ __global__ void __launch_bounds__(kThreads)
         mbar_arrive_expect_tx(&str_full[s], L::TILE + (SWEEP == 1 ? KT * 4 : 0));
         for (int hh = 0; hh < L::NH; ++hh)
           tma_load_3d(smem + L::OFF_STR + s * L::TILE + hh * KT * 128, &tmK, &str_full[s], hh * 64,
-                      g, (int)(seq_row + (size_t)t * KT));
+                      g, tile_row(t * KT));
         if (SWEEP == 1)
           bulk_load(smem + L::OFF_LSE + s * KT * 4, p.lse + head_off + (size_t)t * KT, KT * 4,
                     &str_full[s]);
