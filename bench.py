@@ -155,7 +155,7 @@ class ClockSampler:
 # workload setup
 # ---------------------------------------------------------------------------
 
-def make_inputs(wl, device, kv_fp8=False):
+def make_inputs(wl, device, kv_fp8=False, paged=0):
     """Weights and cache of the workload on `device` (seeded synthetic)."""
     shape = wl.shape
     fast = wl.mode == "layer"
@@ -166,7 +166,39 @@ def make_inputs(wl, device, kv_fp8=False):
                                   with_h_last=fast)
     if kv_fp8:
         to_e4m3_cache(cache)
+    if paged:
+        to_paged_cache(cache, paged, wl.seed)
     return w, cache
+
+
+def to_paged_cache(cache, page, seed):
+    """The cache's K/V moved into page pools (pages of `page` slots in a
+    seeded random order) with a block table; the slot-major buffers freed."""
+    b, cap = cache["tokens"].shape
+    per = cap // page
+    perm = np.random.default_rng(seed).permutation(b * per).reshape(b, per)
+    dev = cache["tokens"].device
+    idx = torch.from_numpy(perm.reshape(-1)).to(dev).long()
+    for key in ("k", "v"):
+        for l, x in enumerate(cache[key]):
+            pool = torch.empty((b * per, page) + tuple(x.shape[2:]), dtype=x.dtype, device=dev)
+            pool[idx] = x.reshape((b * per, page) + tuple(x.shape[2:]))
+            cache[key][l] = pool
+            del x
+    cache["block_table"] = torch.from_numpy(perm.astype(np.int32)).to(dev)
+    cache["page_size"] = page
+    return cache
+
+
+def logical_kv(cache, key, l):
+    """Slot-major [B, cap, Hkv, dh] view of K or V layer l (gathered from the
+    pages of a paged cache)."""
+    x = cache[key][l]
+    if cache.get("block_table") is None:
+        return x
+    t = cache["block_table"].long()
+    b, per = t.shape
+    return x[t.reshape(-1)].reshape((b, per * cache["page_size"]) + tuple(x.shape[2:]))
 
 
 def to_e4m3_cache(cache, headroom=2.0):
@@ -270,7 +302,7 @@ def run_ours(args, dist):
     if wl.cycles > 1 and not args.single_cycle:
         raise SystemExit("multi-cycle workloads: use --single-cycle (the first refresh is timed)")
 
-    w, pristine = make_inputs(wl, dev, args.kv_fp8)
+    w, pristine = make_inputs(wl, dev, args.kv_fp8, args.paged)
     work = clone_cache(pristine)
     weights, cache = pkg.Weights(w), pkg.Cache(work)
     b, cap = wl.batch, wl.cap
@@ -449,7 +481,8 @@ def run_ours(args, dist):
         "higher_is_better": True, "scaling": "weak", "vs_baseline": vs_baseline, "dtype": "bf16",
         "data": "synthetic (seeded random-init weights N(0,0.02); synthetic KV cache)",
         "config": {"workload": wl.name, "scorer": scorer,
-                   "kv_cache": "e4m3 (per-layer scales)" if args.kv_fp8 else "bf16",
+                   "kv_cache": ("e4m3 (per-layer scales)" if args.kv_fp8 else "bf16") +
+                               (f", paged ({args.paged}-slot pages)" if args.paged else ""),
                    "pass": ("fast single-layer" if fast else f"full {shape.n_layers}-layer")
                    if scorer == "counter-causal" else
                    {"recency": "position", "importance": "last-layer key attention",
@@ -527,17 +560,20 @@ def host_inputs(wl, w, cache):
         import oracle
 
         def kvf(key, l):
-            return oracle.e4m3_decode(cache[key][l].cpu().numpy()) * sc[l][0 if key == "k" else 1]
+            return (oracle.e4m3_decode(logical_kv(cache, key, l).cpu().numpy()) *
+                    sc[l][0 if key == "k" else 1])
     else:
         def kvf(key, l):
-            return f32(cache[key][l])
+            return f32(logical_kv(cache, key, l))
     kf = [kvf("k", l) if (not fast or l == last) else None for l in range(wl.shape.n_layers)]
     vf = [kvf("v", l) if (not fast or l == last) else None for l in range(wl.shape.n_layers)]
     cn = {"k": kf, "v": vf, "tokens": cache["tokens"].cpu().numpy(), "pos": cache["pos"].cpu().numpy(),
           "seq_len": cache["seq_len"].cpu().numpy(), "h_last": f32(cache["h_last"])}
     kv_raw = torch.uint8 if sc is not None else torch.int16
-    raw = {"k": [x.view(kv_raw).cpu().numpy() for x in cache["k"]],
-           "v": [x.view(kv_raw).cpu().numpy() for x in cache["v"]],
+    raw = {"k": [logical_kv(cache, "k", l).view(kv_raw).cpu().numpy()
+                 for l in range(len(cache["k"]))],
+           "v": [logical_kv(cache, "v", l).view(kv_raw).cpu().numpy()
+                 for l in range(len(cache["v"]))],
            "h": None if cache["h_last"] is None else cache["h_last"].view(torch.int16).cpu().numpy()}
     return wn, cn, raw
 
@@ -968,6 +1004,9 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--kv-fp8", action="store_true",
                     help="store the cache's K/V as e4m3 codes with per-layer scales")
+    ap.add_argument("--paged", type=int, default=0, metavar="SLOTS",
+                    help="keep the refresh bench's K/V in page pools of SLOTS-slot pages "
+                         "(a multiple of 128) in a shuffled order, with a block table")
     ap.add_argument("--scorer", choices=["counter-causal", "recency", "importance", "h2o"],
                     default="counter-causal",
                     help="refresh scorer: the paper's (default) or one of its comparison "
