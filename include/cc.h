@@ -76,6 +76,15 @@ typedef enum {
   CC_KV_E4M3 = 1
 } cc_kv_format;
 
+/* Order of the cached K/V buffers of a (not paged) cache: slot-major
+ * [batch][cap][Hkv][head_dim] (one slot's heads together), or head-major
+ * [batch][Hkv][cap][head_dim] (each KV head's slots together, as many model
+ * runtimes keep their caches).  Every entry point takes either. */
+typedef enum {
+  CC_KV_SLOT_MAJOR = 0,
+  CC_KV_HEAD_MAJOR = 1
+} cc_kv_layout;
+
 /* Decoder shape (Llama/Qwen pre-norm block: RMSNorm, GQA attention with
  * rotate-half RoPE, RMSNorm, SwiGLU MLP; final RMSNorm; untied LM head). */
 typedef struct {
@@ -166,6 +175,8 @@ typedef struct {
   const int32_t *block_table; /* device int32 [batch][cap / page_size], or NULL          */
   int32_t page_size;
   int32_t n_pages;
+  int32_t kv_layout;  /* cc_kv_layout of k and v (0 = slot-major); a head-major cache is
+                         not paged                                                      */
 } cc_kv_cache;
 
 /* ---- scoring (Sec. 3.1) ---------------------------------------------------

@@ -64,9 +64,10 @@ class cc_kv_cache(ctypes.Structure):
                 ("h2o_acc", ctypes.c_void_p), ("kv_format", ctypes.c_int32),
                 ("kv_scale", ctypes.POINTER(ctypes.c_float)),
                 ("block_table", ctypes.c_void_p), ("page_size", ctypes.c_int32),
-                ("n_pages", ctypes.c_int32)]
+                ("n_pages", ctypes.c_int32), ("kv_layout", ctypes.c_int32)]
 
 KV_BF16, KV_E4M3 = 0, 1
+KV_SLOT_MAJOR, KV_HEAD_MAJOR = 0, 1
 
 
 _LIB = None
@@ -227,7 +228,8 @@ class Cache:
     scales; tokens, pos int32 [B, cap]; seq_len int32 [B]; h_last bf16
     [B, cap, d] or None); with "block_table" (int32 [B, cap // page_size]),
     "page_size" and k[l], v[l] page pools [n_pages, page_size, Hkv, dh] the
-    K/V are paged.  Keeps the tensors alive."""
+    K/V are paged; with "kv_layout": KV_HEAD_MAJOR, k[l], v[l] are
+    [B, Hkv, cap, dh].  Keeps the tensors alive."""
 
     def __init__(self, c: dict):
         self.d = c
@@ -251,7 +253,8 @@ class Cache:
                              _dev_ptr(c["tokens"], "tokens"), _dev_ptr(c["pos"], "pos"),
                              _dev_ptr(c.get("h_last"), "h_last"),
                              _dev_ptr(c.get("h2o_acc"), "h2o_acc"), fmt, self._scale,
-                             _dev_ptr(table, "block_table"), page, n_pages)
+                             _dev_ptr(table, "block_table"), page, n_pages,
+                             int(c.get("kv_layout", KV_SLOT_MAJOR)))
 
 
 def _cfg(cfg):

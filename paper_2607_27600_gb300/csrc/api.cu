@@ -176,8 +176,10 @@ size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
 // Paging of the cache's K/V (table nullptr: slot-major [batch][cap]) and the
 // rows of the K/V buffers (the pool, or batch * cap).
-KvPaging kv_paging(const cc_kv_cache *kv) {
-  KvPaging pg{};
+KvLayout kv_layout(const cc_model_cfg *c, const cc_kv_cache *kv) {
+  KvLayout pg{};
+  pg.hkv = c->n_kv_heads;
+  pg.head_major = kv->kv_layout == CC_KV_HEAD_MAJOR ? 1 : 0;
   if (kv->block_table) {
     pg.table = kv->block_table;
     pg.page = kv->page_size;
@@ -194,17 +196,17 @@ uint64_t kv_buffer_rows(const cc_kv_cache *kv) {
 struct KvFmt {
   bool fp8 = false;
   float k_scale = 1.f, v_scale = 1.f;
-  KvPaging pg{};        // paged K/V (table nullptr: slot-major)
+  KvLayout pg{};        // paged K/V (table nullptr: slot-major)
   uint64_t rows = 0;    // rows of the K/V buffers (0: batch * cap)
 };
-KvFmt kv_fmt(const cc_kv_cache *kv, int l) {
+KvFmt kv_fmt(const cc_model_cfg *c, const cc_kv_cache *kv, int l) {
   KvFmt f;
   if (kv->kv_format == CC_KV_E4M3) {
     f.fp8 = true;
     f.k_scale = kv->kv_scale[2 * l];
     f.v_scale = kv->kv_scale[2 * l + 1];
   }
-  f.pg = kv_paging(kv);
+  f.pg = kv_layout(c, kv);
   f.rows = kv_buffer_rows(kv);
   return f;
 }
@@ -213,6 +215,8 @@ int kv_elem_bytes(const cc_kv_cache *kv) { return kv->kv_format == CC_KV_E4M3 ? 
 // The cache's format fields: a known format; e4m3 needs finite positive
 // scales for every layer.
 bool kv_format_ok(const cc_model_cfg *c, const cc_kv_cache *kv) {
+  if (kv->kv_layout != CC_KV_SLOT_MAJOR && kv->kv_layout != CC_KV_HEAD_MAJOR) return false;
+  if (kv->kv_layout == CC_KV_HEAD_MAJOR && kv->block_table) return false;   // not paged
   if (kv->block_table) {   // pages of whole 128-slot key tiles that divide cap
     if (kv->page_size < 128 || kv->page_size % 128 || kv->cap % kv->page_size ||
         kv->n_pages < 1 || (uint64_t)kv->n_pages * kv->page_size >= (1ull << 31))
@@ -489,21 +493,27 @@ cc_status run_attention(const cc_model_cfg *c, const void *q, const void *k, con
     if (!make_tmap(&tq, q, 3, dims, strides, box)) return tmap_fail();
   }
   const uint64_t RK = kvf.rows ? kvf.rows : R;   // K/V buffer rows (paged: the pool)
+  const bool hm = kvf.pg.head_major != 0;
+  // slot-major maps (dh, Hkv, rows), box (.., 1, 128 slots); head-major maps
+  // (dh, cap, batch*Hkv), box (.., 128 slots, 1): the same shared-memory image
+  const int eb = kvf.fp8 ? 1 : 2;
+  const uint64_t kv_dims[3] = {(uint64_t)dh, hm ? (uint64_t)cap : (uint64_t)c->n_kv_heads,
+                               hm ? (uint64_t)batch * c->n_kv_heads : RK};
+  const uint64_t kv_strides[2] = {(uint64_t)dh * eb,
+                                  hm ? (uint64_t)cap * dh * eb : (uint64_t)c->n_kv_heads * dh * eb};
   if (kvf.fp8) {   // e4m3 bytes, one unswizzled box per 128-key tile (converted in the kernel)
-    const uint64_t dims[3] = {(uint64_t)dh, (uint64_t)c->n_kv_heads, RK};
-    const uint64_t strides[2] = {(uint64_t)dh, (uint64_t)c->n_kv_heads * dh};
-    const uint32_t box[3] = {(uint32_t)dh, 1, 128};
+    const uint64_t *dims = kv_dims;
+    const uint64_t *strides = kv_strides;
+    const uint32_t box[3] = {(uint32_t)dh, hm ? 128u : 1u, hm ? 1u : 128u};
     if (!make_tmap(&tk, k, 3, dims, strides, box, CU_TENSOR_MAP_SWIZZLE_NONE,
                    CU_TENSOR_MAP_DATA_TYPE_UINT8) ||
         !make_tmap(&tv, v, 3, dims, strides, box, CU_TENSOR_MAP_SWIZZLE_NONE,
                    CU_TENSOR_MAP_DATA_TYPE_UINT8))
       return tmap_fail();
   } else {
-    const uint64_t dims[3] = {(uint64_t)dh, (uint64_t)c->n_kv_heads, RK};
-    const uint64_t strides[2] = {(uint64_t)dh * 2, (uint64_t)c->n_kv_heads * dh * 2};
-    const uint32_t box[3] = {64, 1, 128};
-    if (!make_tmap(&tk, k, 3, dims, strides, box)) return tmap_fail();
-    if (!make_tmap(&tv, v, 3, dims, strides, box)) return tmap_fail();
+    const uint32_t box[3] = {64, hm ? 128u : 1u, hm ? 1u : 128u};
+    if (!make_tmap(&tk, k, 3, kv_dims, kv_strides, box)) return tmap_fail();
+    if (!make_tmap(&tv, v, 3, kv_dims, kv_strides, box)) return tmap_fail();
   }
   AttnParams p{};
   p.batch = batch;
@@ -718,7 +728,7 @@ cc_status run_append(const cc_model_cfg *c, const cc_model_weights *w, const cc_
   }
   for (int l = 0; l < c->n_layers; ++l) {
     const cc_layer_weights &lw = w->layers[l];
-    const KvFmt kvf = kv_fmt(kv, l);   // e4m3 cache: K/V rows written as codes of value / scale
+    const KvFmt kvf = kv_fmt(c, kv, l);   // e4m3 cache: K/V rows written as codes of value / scale
     if (l == c->n_layers - 1 && kv->h_last) {   // H^(L-1), recorded for the fast approximation
       TimedScope t(CC_KERNEL_APPEND, st);
       CC_TRY(launch_store_bf16(h, kv->h_last, d, hi, lo, cap, rows, st, max_count));
@@ -922,7 +932,7 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
     if ((s = run_gemm(gq, EPI_QROPE, CC_KERNEL_GEMM_QROPE, dev->sms, st)) != CC_OK) return s;
     // O = counter-causal attention
     if ((s = run_attention(c, q, kv->k[l], kv->v[l], o, sl, batch, cap, status, st, split,
-                           nullptr, 0, nullptr, 0, kv_fmt(kv, l))) !=
+                           nullptr, 0, nullptr, 0, kv_fmt(c, kv, l))) !=
         CC_OK)
       return s;
     // h = h + O Wo^T  (fast mode: h = H^(L-1) + O Wo^T)
@@ -1016,7 +1026,8 @@ cc_status compact_plan(const cc_model_cfg *c, const cc_kv_cache *kv, CompactPlan
     p.class_chunks[p.n_classes] = (kv->cap + rows - 1) / rows;
     return p.n_classes++;
   };
-  auto add = [&](void *base, int row_bytes, bool bulk, bool paged = false) -> bool {
+  auto add = [&](void *base, int row_bytes, bool bulk, bool paged = false,
+                 bool head_major = false) -> bool {
     if (!base) return true;
     if (n >= kMaxCompactArrays || !aligned16(base)) return false;
     CompactArray &A = p.arr[n++];
@@ -1024,6 +1035,7 @@ cc_status compact_plan(const cc_model_cfg *c, const cc_kv_cache *kv, CompactPlan
     A.row_bytes = row_bytes;
     A.bulk = bulk ? 1 : 0;
     A.paged = paged ? 1 : 0;
+    A.head_major = head_major ? 1 : 0;
     A.rows_per_chunk = bulk ? (row_bytes <= p.stage_bytes ? p.stage_bytes / row_bytes : 0)
                             : p.stage_bytes / 4;
     if (A.rows_per_chunk < 1) return false;
@@ -1037,10 +1049,11 @@ cc_status compact_plan(const cc_model_cfg *c, const cc_kv_cache *kv, CompactPlan
   // staging shape of the copy kernel for the largest row moved
   const int max_row = std::max(kv_row, kv->h_last ? c->d_model * 2 : 0);
   if (!compact_shape(max_row, p.stage_bytes, p.warps)) return CC_ERR_UNSUPPORTED;
-  p.pg = kv_paging(kv);   // K/V rows through the block table when paged
+  p.pg = kv_layout(c, kv);   // K/V rows through the block table when paged
   const bool paged = kv->block_table != nullptr;
+  const bool hm = kv->kv_layout == CC_KV_HEAD_MAJOR;   // rows of Hkv segments
   for (int l = 0; l < c->n_layers; ++l) {
-    if (!add(kv->k[l], kv_row, true, paged) || !add(kv->v[l], kv_row, true, paged))
+    if (!add(kv->k[l], kv_row, true, paged, hm) || !add(kv->v[l], kv_row, true, paged, hm))
       return CC_ERR_UNSUPPORTED;
   }
   if (!add(kv->h_last, c->d_model * 2, true)) return CC_ERR_UNSUPPORTED;
@@ -1109,13 +1122,16 @@ cc_status run_keyattn(const cc_model_cfg *c, const cc_kv_cache *kv, int l0, int 
   memset(&a, 0, sizeof(a));
   const uint64_t RK = kv_buffer_rows(kv);   // K buffer rows (paged: the pool)
   (void)R;
-  const uint64_t dims[3] = {(uint64_t)dh, (uint64_t)c->n_kv_heads, RK};
-  const uint64_t strides[2] = {(uint64_t)dh * 2, (uint64_t)c->n_kv_heads * dh * 2};
-  const uint32_t box[3] = {64, 1, 128};
+  const bool hm = kv->kv_layout == CC_KV_HEAD_MAJOR;   // see run_attention
+  const uint64_t dims[3] = {(uint64_t)dh, hm ? (uint64_t)cap : (uint64_t)c->n_kv_heads,
+                            hm ? (uint64_t)batch * c->n_kv_heads : RK};
+  const uint64_t strides[2] = {(uint64_t)dh * 2,
+                               hm ? (uint64_t)cap * dh * 2 : (uint64_t)c->n_kv_heads * dh * 2};
+  const uint32_t box[3] = {64, hm ? 128u : 1u, hm ? 1u : 128u};
   for (int l = l0; l < l1; ++l)
     if (!make_tmap(&a.k[l - l0], kv->k[l], 3, dims, strides, box)) return tmap_fail();
   KeyAttnParams &p = a.p;
-  p.pg = kv_paging(kv);
+  p.pg = kv_layout(c, kv);
   p.kv_rows = (int)RK;
   p.batch = batch;
   p.cap = cap;

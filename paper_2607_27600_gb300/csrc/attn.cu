@@ -220,6 +220,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   // pool row of key tile t (paged) or b*cap + 128 t; a bad page reads zeros
   // (a coordinate past the maps) and is reported
   auto tile_row = [&](int t) -> int {
+    if (p.pg.head_major) return 0;   // coordinates (slot, b*Hkv + g) instead
     const long long r = kv_row(p.pg, p.cap, b, t * BKV);
     if (r < 0) {
       set_status(p.status, CC_ERR_DEVICE_ARG);
@@ -308,19 +309,22 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int t = t_hi - it, s = it % KST;
         const uint32_t ph = (it / KST) & 1;
         const int krow = tile_row(t);
+        // TMA coordinates after the head_dim one: (KV head, row), or head-major (slot, b*Hkv + g)
+        const int kc1 = p.pg.head_major ? t * BKV : g;
+        const int kc2 = p.pg.head_major ? b * p.n_kv_heads + g : krow;
         int ok = 1;
         if (lane == 0) {
           ok = mbar_wait(&k_empty[s], ph ^ 1, abort_flag, p.status);
           if (ok) {
             mbar_arrive_expect_tx(&k_load[s], L::FP8_TILE);
-            tma_load_3d(smem + L::OFF_K + s * L::KV_BYTES + L::KV_BYTES / 2, &tmK, &k_load[s], 0, g,
-                        krow);
+            tma_load_3d(smem + L::OFF_K + s * L::KV_BYTES + L::KV_BYTES / 2, &tmK, &k_load[s], 0,
+                        kc1, kc2);
             ok = mbar_wait(&v_empty[s], ph ^ 1, abort_flag, p.status);
           }
           if (ok) {
             mbar_arrive_expect_tx(&v_load[s], L::FP8_TILE);
-            tma_load_3d(smem + L::OFF_V + s * L::KV_BYTES + L::KV_BYTES / 2, &tmV, &v_load[s], 0, g,
-                        krow);
+            tma_load_3d(smem + L::OFF_V + s * L::KV_BYTES + L::KV_BYTES / 2, &tmV, &v_load[s], 0,
+                        kc1, kc2);
           }
         }
         ok = __shfl_sync(0xFFFFFFFFu, ok, 0);
@@ -332,17 +336,20 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int t = t_hi - it;
         const uint32_t sp = it & 1;
         const int krow = tile_row(t);
+        // TMA coordinates after the head_dim one: (KV head, row), or head-major (slot, b*Hkv + g)
+        const int kc1 = p.pg.head_major ? t * BKV : g;
+        const int kc2 = p.pg.head_major ? b * p.n_kv_heads + g : krow;
         int ok = 1;
         if (lane == 0) {
           ok = mbar_wait(&stg_empty[0], sp ^ 1, abort_flag, p.status);
           if (ok) {
             mbar_arrive_expect_tx(&stg_full[0], L::STG_BYTES);
-            tma_load_3d(smem + L::OFF_STG, &tmK, &stg_full[0], 0, g, krow);
+            tma_load_3d(smem + L::OFF_STG, &tmK, &stg_full[0], 0, kc1, kc2);
             ok = mbar_wait(&stg_empty[1], sp ^ 1, abort_flag, p.status);
           }
           if (ok) {
             mbar_arrive_expect_tx(&stg_full[1], L::STG_BYTES);
-            tma_load_3d(smem + L::OFF_STG + L::STG_BYTES, &tmV, &stg_full[1], 0, g, krow);
+            tma_load_3d(smem + L::OFF_STG + L::STG_BYTES, &tmV, &stg_full[1], 0, kc1, kc2);
           }
         }
         ok = __shfl_sync(0xFFFFFFFFu, ok, 0);
@@ -353,6 +360,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int t = t_hi - it, s = it % KST;   // key tiles from the sequence end downwards
         const uint32_t ph = (it / KST) & 1;
         const int krow = tile_row(t);
+        // TMA coordinates after the head_dim one: (KV head, row), or head-major (slot, b*Hkv + g)
+        const int kc1 = p.pg.head_major ? t * BKV : g;
+        const int kc2 = p.pg.head_major ? b * p.n_kv_heads + g : krow;
         int ok = 1;
         if (lane == 0) {
           ok = mbar_wait(&k_empty[s], ph ^ 1, abort_flag, p.status);
@@ -360,14 +370,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_arrive_expect_tx(&k_full[s], L::KV_BYTES);
             for (int hh = 0; hh < L::NH; ++hh)
               tma_load_3d(smem + L::OFF_K + s * L::KV_BYTES + hh * BKV * 128, &tmK, &k_full[s],
-                          hh * 64, g, krow);
+                          hh * 64, kc1, kc2);
             ok = mbar_wait(&v_empty[s], ph ^ 1, abort_flag, p.status);
           }
           if (ok) {
             mbar_arrive_expect_tx(&v_full[s], L::KV_BYTES);
             for (int hh = 0; hh < L::NH; ++hh)
               tma_load_3d(smem + L::OFF_V + s * L::KV_BYTES + hh * BKV * 128, &tmV, &v_full[s],
-                          hh * 64, g, krow);
+                          hh * 64, kc1, kc2);
           }
         }
         ok = __shfl_sync(0xFFFFFFFFu, ok, 0);
@@ -943,15 +953,17 @@ __global__ void __launch_bounds__(kDecThreads) attn_decode_kernel(const __grid_c
     uint8_t *kb = smem + buf * L::BUF, *vb = kb + L::K_BYTES;
     // K in DH/8 pieces per row (16 bytes bf16, 8 bytes e4m3), V in 16-byte pieces
     constexpr int KP = DH / 8, KPB = 8 * L::EB, VP = DH * L::EB / 16;
-    // pool row of the chunk's first key (a chunk lies in one page); -1: bad page
-    const long long cbase = kv_row(p.pg, p.cap, u.b, c * kDecChunk);
+    // vector index of the chunk's first key (a chunk lies in one page; head-major:
+    // consecutive slots are consecutive vectors, else Hkv apart); -1: bad page
+    const long long cbase = kv_vec(p.pg, p.cap, u.b, u.g, c * kDecChunk);
+    const int vstep = p.pg.head_major ? 1 : Hkv;
     if (cbase < 0 && tid == 0) set_status(p.status, CC_ERR_DEVICE_ARG);
     for (int i = tid; i < kDecChunk * KP; i += kDecThreads) {
       const int r = i / KP, e = i - r * KP;
       const int j = c * kDecChunk + r;
       uint8_t *kd = kb + r * L::K_ROW + e * KPB;
       if (j < n_keys && cbase >= 0) {
-        const uint8_t *src = kg + (((size_t)(cbase + r) * Hkv + u.g) * (size_t)DH) * L::EB + e * KPB;
+        const uint8_t *src = kg + ((size_t)(cbase + (long long)r * vstep) * DH) * L::EB + e * KPB;
         if constexpr (FP8) cp_async8(kd, src);
         else cp_async16(kd, src);
       } else if constexpr (FP8) {
@@ -965,7 +977,7 @@ __global__ void __launch_bounds__(kDecThreads) attn_decode_kernel(const __grid_c
       const int j = c * kDecChunk + r;
       uint8_t *vd = vb + r * L::V_ROW + e * 16;
       if (j < n_keys && cbase >= 0)   // past the last key: zeros (P is 0 there, V must be finite)
-        cp_async16(vd, vg + (((size_t)(cbase + r) * Hkv + u.g) * (size_t)DH) * L::EB + e * 16);
+        cp_async16(vd, vg + ((size_t)(cbase + (long long)r * vstep) * DH) * L::EB + e * 16);
       else
         *reinterpret_cast<uint4 *>(vd) = make_uint4(0, 0, 0, 0);
     }

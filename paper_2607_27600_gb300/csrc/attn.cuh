@@ -26,7 +26,7 @@ struct AttnParams {
   int kv_fp8;               // K/V are e4m3 codes: the tile kernel converts them to f16 in
                             // shared memory; the K scale is folded into scale_log2
   float v_scale;            // output = v_scale * (P V) / l (1 for a bf16 cache)
-  KvPaging pg;              // paged K/V (pg.table nullptr: slot-major)
+  KvLayout pg;              // paged K/V (pg.table nullptr: slot-major)
   int kv_rows;              // rows of the K/V tensor maps (a coordinate there reads zeros)
   unsigned *status;
 };

@@ -325,20 +325,31 @@ CC_DEV uint32_t pack_bf16x2(float lo, float hi) {
 CC_DEV float bf16_lo(uint32_t v) { return __uint_as_float(v << 16); }
 CC_DEV float bf16_hi(uint32_t v) { return __uint_as_float(v & 0xFFFF0000u); }
 
-// Paged K/V: the pool row of logical slot i of sequence b.  Pages hold `page`
+// K/V layout.  Paged K/V: the pool row of logical slot i of sequence b.  Pages hold `page`
 // slots (a multiple of 128, so a key tile never straddles two pages); the
 // block table has pages_per_seq entries per sequence.  Without a table the
 // buffers are slot-major: row b * cap + i.  An entry outside [0, n_pages)
 // gives -1 (callers skip the row and report it).
-struct KvPaging {
+// Head-major buffers ([batch][Hkv][cap][head_dim], not paged) keep each KV
+// head's vectors of a sequence contiguous instead.
+struct KvLayout {
   const int32_t *table;   // device [batch][pages_per_seq], or nullptr
   int page, pages_per_seq, n_pages;
+  int head_major;         // [batch][Hkv][cap][head_dim]
+  int hkv;                // KV heads
 };
-CC_DEV long long kv_row(const KvPaging &pg, int cap, int b, int i) {
+CC_DEV long long kv_row(const KvLayout &pg, int cap, int b, int i) {
   if (!pg.table) return (long long)b * cap + i;
   const int e = pg.table[(size_t)b * pg.pages_per_seq + i / pg.page];
   if (e < 0 || e >= pg.n_pages) return -1;
   return (long long)e * pg.page + i % pg.page;
+}
+// Index (in head_dim-element vectors) of KV head g's vector of slot i of
+// sequence b in the K or V buffer; -1 for a bad page.
+CC_DEV long long kv_vec(const KvLayout &L, int cap, int b, int g, int i) {
+  if (L.head_major) return ((long long)b * L.hkv + g) * cap + i;
+  const long long r = kv_row(L, cap, b, i);
+  return r < 0 ? -1 : r * L.hkv + g;
 }
 
 // Two e4m3 codes (lo in the low byte): round to nearest even, saturating to

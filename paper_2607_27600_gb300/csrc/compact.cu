@@ -210,6 +210,28 @@ __global__ void __launch_bounds__(kThreads)
     if (r < 0) set_status(p.status, CC_ERR_DEVICE_ARG);
     return r;
   };
+  // Copies one bulk row (slot k of sequence b) between global memory and a
+  // shared-memory row; head-major arrays move it as Hkv segments.
+  auto row_load = [&](const CompactArray &A, int b, int src, uint8_t *dst, uint64_t *bar) {
+    uint8_t *base = reinterpret_cast<uint8_t *>(A.base);
+    if (A.head_major) {
+      const int seg = A.row_bytes / p.pg.hkv;
+      for (int g = 0; g < p.pg.hkv; ++g)
+        bulk_load(dst + g * seg, base + (((size_t)b * p.pg.hkv + g) * p.cap + src) * seg, seg, bar);
+    } else {
+      bulk_load(dst, base + (size_t)arow(A, b, src) * A.row_bytes, A.row_bytes, bar);
+    }
+  };
+  auto row_store = [&](const CompactArray &A, int b, int k, const uint8_t *src) {
+    uint8_t *base = reinterpret_cast<uint8_t *>(A.base);
+    if (A.head_major) {
+      const int seg = A.row_bytes / p.pg.hkv;
+      for (int g = 0; g < p.pg.hkv; ++g)
+        bulk_store(base + (((size_t)b * p.pg.hkv + g) * p.cap + k) * seg, src + g * seg, seg);
+    } else {
+      bulk_store(base + (size_t)arow(A, b, k) * A.row_bytes, src, A.row_bytes);
+    }
+  };
   // A bulk row moves when its source differs and both rows exist.
   auto moves = [&](const CompactArray &A, int b, int k, int src) {
     return src != k && (!A.paged || (arow(A, b, k) >= 0 && arow(A, b, src) >= 0));
@@ -232,8 +254,7 @@ __global__ void __launch_bounds__(kThreads)
       for (int k = u.k0 + lane; k < u.k1; k += 32) {
         const int src = source(kidx, k, true);
         if (moves(A, u.b, k, src))
-          bulk_load(buf[s] + (size_t)(k - u.k0) * A.row_bytes,
-                    base + (size_t)arow(A, u.b, src) * A.row_bytes, A.row_bytes, &bars[warp][s]);
+          row_load(A, u.b, src, buf[s] + (size_t)(k - u.k0) * A.row_bytes, &bars[warp][s]);
       }
       u.loaded = true;
     } else {   // 4-byte rows: plain loads staged in shared memory
@@ -294,8 +315,7 @@ __global__ void __launch_bounds__(kThreads)
         if (cur.loaded) {
           for (int k = cur.k0 + lane; k < cur.k1; k += 32)
             if (moves(A, cur.b, k, source(kidx, k, false)))
-              bulk_store(base + (size_t)arow(A, cur.b, k) * A.row_bytes,
-                         buf[s] + (size_t)(k - cur.k0) * A.row_bytes, A.row_bytes);
+              row_store(A, cur.b, k, buf[s] + (size_t)(k - cur.k0) * A.row_bytes);
           bulk_commit();
         }
       } else {

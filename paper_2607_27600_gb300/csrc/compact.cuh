@@ -25,6 +25,8 @@ struct CompactArray {
   int n_chunks;        // chunks per sequence = ceil(cap / rows_per_chunk) (upper bound of units)
   int dep_class;       // chunk-size class (index into the readers table)
   int paged;           // bulk K/V arrays of a paged cache: rows through CompactParams::pg
+  int head_major;      // bulk K/V arrays [batch][Hkv][cap][row_bytes / Hkv]: a row is Hkv
+                       // segments, one in each KV head's buffer
 };
 
 struct CompactParams {
@@ -47,7 +49,7 @@ struct CompactParams {
   int withhold_unit;          // test hook: this unit never publishes its flag (-1: none)
   int stage_bytes;            // shared-memory buffer of a unit (multiple of 128)
   int warps;                  // warps per CTA (each with two buffers)
-  KvPaging pg;                // paged K/V arrays: pool row of logical slot (b, i)
+  KvLayout pg;                // paged K/V arrays: pool row of logical slot (b, i)
   CompactArray arr[kMaxCompactArrays];
 };
 

@@ -37,14 +37,28 @@ constexpr size_t kSmemBytes = 1024 /*align slack*/ + ST * (A_BYTES + B_BYTES) + 
 // F8: the destination is an e4m3 cache (one byte per element, the value
 // times qscale = 1 / the layer's scale; pack_e4m3x2).
 // orow: the output row (grow, or the cache row of a paged K destination; < 0: skip)
+// Address of output column c of row `orow` (element size EB), or with a
+// head-major cache destination (hm) of head c / head_dim's vector of slot
+// grow % cap (32-column chunks never straddle two heads).
+template <int EB>
+CC_DEV uint8_t *out_at(const GemmParams &p, uint8_t *base, long long orow, int ldo, bool hm,
+                       int grow, int c) {
+  if (hm) {
+    const int b = grow / p.cap, i = grow - b * p.cap;
+    return base + ((((size_t)b * p.pg.hkv + c / p.head_dim) * p.cap + i) * p.head_dim +
+                   c % p.head_dim) * EB;
+  }
+  return base + ((size_t)orow * ldo + c) * EB;
+}
+
 template <int TBN, bool F8 = false>
 CC_DEV void rope_store(const GemmParams &p, uint32_t tacc, int grow, long long orow, bool valid,
                        void *out_base, int ldo, const __nv_bfloat16 *bias, int col0, int n_dest,
-                       float qscale = 1.f) {
+                       float qscale = 1.f, bool hm = false) {
   const int half = p.head_dim >> 1;
   valid = valid && orow >= 0;
   const uint32_t pos = valid ? (uint32_t)p.pos[grow] : 0u;
-  uint8_t *out = reinterpret_cast<uint8_t *>(out_base) + (size_t)(valid ? orow : 0) * ldo * (F8 ? 1 : 2);
+  uint8_t *base = reinterpret_cast<uint8_t *>(out_base);
 #pragma unroll 1
   for (int hb = 0; hb < TBN; hb += p.head_dim) {
 #pragma unroll 1
@@ -94,8 +108,8 @@ CC_DEV void rope_store(const GemmParams &p, uint32_t tacc, int grow, long long o
         }
       }
       constexpr int EB = F8 ? 1 : 2;
-      uint4 *d1 = reinterpret_cast<uint4 *>(out + (size_t)col * EB);
-      uint4 *d2 = reinterpret_cast<uint4 *>(out + (size_t)(col + half) * EB);
+      uint4 *d1 = reinterpret_cast<uint4 *>(out_at<EB>(p, base, orow, ldo, hm, grow, col));
+      uint4 *d2 = reinterpret_cast<uint4 *>(out_at<EB>(p, base, orow, ldo, hm, grow, col + half));
 #pragma unroll
       for (int v = 0; v < 2 * EB; ++v) {   // 32 elements: 64 bytes bf16, 32 e4m3
         d1[v] = make_uint4(o1[v * 4], o1[v * 4 + 1], o1[v * 4 + 2], o1[v * 4 + 3]);
@@ -108,11 +122,12 @@ CC_DEV void rope_store(const GemmParams &p, uint32_t tacc, int grow, long long o
 // Plain bf16 store (+ optional bias) of one accumulator tile row; F8: e4m3
 // codes of (value + bias) * qscale instead.
 template <int TBN, bool F8 = false>
-CC_DEV void plain_store(uint32_t tacc, long long orow, bool valid, void *out_base, int ldo,
-                        const __nv_bfloat16 *bias, int col0, int n_dest, float qscale = 1.f) {
+CC_DEV void plain_store(const GemmParams &p, uint32_t tacc, int grow, long long orow, bool valid,
+                        void *out_base, int ldo, const __nv_bfloat16 *bias, int col0, int n_dest,
+                        float qscale = 1.f, bool hm = false) {
   constexpr int EB = F8 ? 1 : 2;
   valid = valid && orow >= 0;
-  uint8_t *out = reinterpret_cast<uint8_t *>(out_base) + (size_t)(valid ? orow : 0) * ldo * EB;
+  uint8_t *base = reinterpret_cast<uint8_t *>(out_base);
 #pragma unroll 1
   for (int c = 0; c < TBN / 32; ++c) {
     uint32_t r[32];
@@ -139,7 +154,7 @@ CC_DEV void plain_store(uint32_t tacc, long long orow, bool valid, void *out_bas
         o[k / 2] = pack_bf16x2(y0, y1);
       }
     }
-    uint4 *d = reinterpret_cast<uint4 *>(out + (size_t)col * EB);
+    uint4 *d = reinterpret_cast<uint4 *>(out_at<EB>(p, base, orow, ldo, hm, grow, col));
 #pragma unroll
     for (int v = 0; v < 2 * EB; ++v)   // 32 elements: 64 bytes bf16, 32 e4m3
       d[v] = make_uint4(o[v * 4], o[v * 4 + 1], o[v * 4 + 2], o[v * 4 + 3]);
@@ -200,35 +215,39 @@ CC_DEV void epilogue_tile(const GemmParams &p, uint32_t tacc, int grow, bool val
     }
   } else if constexpr (EPI == EPI_QROPE) {   // kv_fp8: the K rows of an e4m3 cache
     const long long orow = p.kv_dest ? cache_row(p, grow, valid) : grow;
+    const bool hm = p.kv_dest && p.pg.head_major;
     if (p.kv_fp8)
       rope_store<TBN, true>(p, tacc, grow, orow, valid, p.out, p.ldo, p.bias, tile_n0, p.N,
-                            p.k_qscale);
+                            p.k_qscale, hm);
     else
-      rope_store<TBN>(p, tacc, grow, orow, valid, p.out, p.ldo, p.bias, tile_n0, p.N);
+      rope_store<TBN>(p, tacc, grow, orow, valid, p.out, p.ldo, p.bias, tile_n0, p.N, 1.f, hm);
   } else if constexpr (EPI == EPI_BF16) {    // kv_fp8: the V rows of an e4m3 cache
     const long long orow = p.kv_dest ? cache_row(p, grow, valid) : grow;
+    const bool hm = p.kv_dest && p.pg.head_major;
     if (p.kv_fp8)
-      plain_store<TBN, true>(tacc, orow, valid, p.out, p.ldo, p.bias, tile_n0, p.N, p.v_qscale);
+      plain_store<TBN, true>(p, tacc, grow, orow, valid, p.out, p.ldo, p.bias, tile_n0, p.N,
+                             p.v_qscale, hm);
     else
-      plain_store<TBN>(tacc, orow, valid, p.out, p.ldo, p.bias, tile_n0, p.N);
+      plain_store<TBN>(p, tacc, grow, orow, valid, p.out, p.ldo, p.bias, tile_n0, p.N, 1.f, hm);
   } else if constexpr (EPI == EPI_QKV) {
     // fused projections: column tiles [0, nq) are Q, [nq, nq+nk) K, the rest V (cache rows)
     const int nq = p.n_q_tiles, nk = p.n_k_tiles;
     const long long crow = nt < nq ? grow : cache_row(p, grow, valid);
+    const bool hm = p.pg.head_major != 0;   // the K and V parts
     if (nt < nq)
       rope_store<TBN>(p, tacc, grow, grow, valid, p.out, p.ldo, p.bias, nt * TBN, nq * TBN);
     else if (nt < nq + nk && p.kv_fp8)
       rope_store<TBN, true>(p, tacc, grow, crow, valid, p.out_k, p.ldo_kv, p.bias_k,
-                            (nt - nq) * TBN, nk * TBN, p.k_qscale);
+                            (nt - nq) * TBN, nk * TBN, p.k_qscale, hm);
     else if (nt < nq + nk)
       rope_store<TBN>(p, tacc, grow, crow, valid, p.out_k, p.ldo_kv, p.bias_k, (nt - nq) * TBN,
-                      nk * TBN);
+                      nk * TBN, 1.f, hm);
     else if (p.kv_fp8)
-      plain_store<TBN, true>(tacc, crow, valid, p.out_v, p.ldo_kv, p.bias_v, (nt - nq - nk) * TBN,
-                             nk * TBN, p.v_qscale);
+      plain_store<TBN, true>(p, tacc, grow, crow, valid, p.out_v, p.ldo_kv, p.bias_v,
+                             (nt - nq - nk) * TBN, nk * TBN, p.v_qscale, hm);
     else
-      plain_store<TBN>(tacc, crow, valid, p.out_v, p.ldo_kv, p.bias_v, (nt - nq - nk) * TBN,
-                       nk * TBN);
+      plain_store<TBN>(p, tacc, grow, crow, valid, p.out_v, p.ldo_kv, p.bias_v,
+                       (nt - nq - nk) * TBN, nk * TBN, 1.f, hm);
   } else if constexpr (EPI == EPI_SWIGLU) {
     // columns [0,128) = gate rows nt*128.., [128,256) = up rows nt*128..
     __nv_bfloat16 *out = reinterpret_cast<__nv_bfloat16 *>(p.out) + (size_t)grow * p.ldo;

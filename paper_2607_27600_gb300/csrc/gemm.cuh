@@ -53,7 +53,7 @@ struct GemmParams {
   const __nv_bfloat16 *bias_k, *bias_v;   // EPI_QKV: optional biases of K and V
   int kv_dest;                // EPI_QROPE / EPI_BF16: the output is K / V cache rows (paged
                               // through pg; EPI_QKV: always for its K and V parts)
-  KvPaging pg;                // paged K/V (pg.table nullptr: row b * cap + i)
+  KvLayout pg;                // paged K/V (pg.table nullptr: row b * cap + i)
   int kv_fp8;                 // EPI_QKV: K and V destinations are e4m3 (one byte each);
                               // EPI_QROPE / EPI_BF16: the destination is e4m3 K / V
   float k_qscale, v_qscale;   // kv_fp8: 1 / the K and V scales (code = rne(value * qscale))

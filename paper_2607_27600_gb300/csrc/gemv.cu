@@ -292,6 +292,14 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
               continue;
             }
           }
+          // element index of output column n (head-major cache: head n / head_dim's vector)
+          const bool hm = sg.kv_dest && p.pg.head_major;
+          auto el = [&](int n) -> size_t {
+            if (hm)
+              return (((size_t)b * p.pg.hkv + n / p.head_dim) * p.cap + (row - b * p.cap)) *
+                         p.head_dim + n % p.head_dim;
+            return (size_t)orow * sg.ldo + n;
+          };
           if (sg.epi == GEMV_ROPE) {
             const int half = p.head_dim >> 1;
             const int n1 = box_row(p, sg, gl, 0) + j, n2 = n1 + half;
@@ -304,13 +312,13 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
             rope_cs((uint32_t)p.pos[row], p.turns[n1 % p.head_dim], c, sn);
             const float y1 = a1 * c - a2 * sn, y2 = a2 * c + a1 * sn;
             if (sg.fp8) {
-              uint8_t *o = reinterpret_cast<uint8_t *>(sg.out) + (size_t)orow * sg.ldo;
-              o[n1] = (uint8_t)pack_e4m3x2(y1 * sg.qscale, 0.f);
-              o[n2] = (uint8_t)pack_e4m3x2(y2 * sg.qscale, 0.f);
+              uint8_t *o = reinterpret_cast<uint8_t *>(sg.out);
+              o[el(n1)] = (uint8_t)pack_e4m3x2(y1 * sg.qscale, 0.f);
+              o[el(n2)] = (uint8_t)pack_e4m3x2(y2 * sg.qscale, 0.f);
             } else {
-              __nv_bfloat16 *o = reinterpret_cast<__nv_bfloat16 *>(sg.out) + (size_t)orow * sg.ldo;
-              o[n1] = __float2bfloat16_rn(y1);
-              o[n2] = __float2bfloat16_rn(y2);
+              __nv_bfloat16 *o = reinterpret_cast<__nv_bfloat16 *>(sg.out);
+              o[el(n1)] = __float2bfloat16_rn(y1);
+              o[el(n2)] = __float2bfloat16_rn(y2);
             }
           } else if (sg.epi == GEMV_SWIGLU) {
             const int u = gl * 8 + j;
@@ -326,11 +334,10 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
             } else {
               const float bb = sg.bias ? __bfloat162float(sg.bias[u]) : 0.f;
               if (sg.fp8)
-                reinterpret_cast<uint8_t *>(sg.out)[(size_t)orow * sg.ldo + u] =
+                reinterpret_cast<uint8_t *>(sg.out)[el(u)] =
                     (uint8_t)pack_e4m3x2((v + bb) * sg.qscale, 0.f);
               else
-                reinterpret_cast<__nv_bfloat16 *>(sg.out)[(size_t)orow * sg.ldo + u] =
-                    __float2bfloat16_rn(v + bb);
+                reinterpret_cast<__nv_bfloat16 *>(sg.out)[el(u)] = __float2bfloat16_rn(v + bb);
             }
           }
         }

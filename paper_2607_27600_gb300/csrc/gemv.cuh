@@ -58,7 +58,7 @@ struct GemvParams {
   const int32_t *pos;               // ROPE: original positions [batch * cap]
   int head_dim;
   unsigned long long turns[64];     // ROPE: inv_freq_k / (2 pi) in 0.64 fixed point
-  KvPaging pg;                      // paged cache rows of kv_dest segments
+  KvLayout pg;                      // paged cache rows of kv_dest segments
   float2 *part;                     // ARGMAX: [batch][part_ld], part_ld = ctas
   int part_ld;
   unsigned *status;

@@ -100,6 +100,7 @@ __global__ void __launch_bounds__(kThreads)
   // pool row of the key tile starting at slot i (paged: one page holds it);
   // a bad page reads zeros (a coordinate past the map) and is reported
   auto tile_row = [&](int i) -> int {
+    if (p.pg.head_major) return b * p.n_kv_heads + g;   // coordinates (slot, b*Hkv + g)
     const long long r = kv_row(p.pg, p.cap, b, i);
     if (r < 0) {
       set_status(p.status, CC_ERR_DEVICE_ARG);
@@ -133,7 +134,8 @@ __global__ void __launch_bounds__(kThreads)
       tma_prefetch_desc(&tmK);
       mbar_arrive_expect_tx(row_full, L::TILE);
       for (int hh = 0; hh < L::NH; ++hh)
-        tma_load_3d(smem + L::OFF_ROW + hh * KT * 128, &tmK, row_full, hh * 64, g, tile_row(row0));
+        tma_load_3d(smem + L::OFF_ROW + hh * KT * 128, &tmK, row_full, hh * 64,
+                    p.pg.head_major ? row0 : g, tile_row(row0));
       for (int it = 0; it < ntiles; ++it) {
         const int t = t_first + it, s = it % KST;
         const uint32_t ph = (it / KST) & 1;
@@ -141,7 +143,7 @@ __global__ void __launch_bounds__(kThreads)
         mbar_arrive_expect_tx(&str_full[s], L::TILE + (SWEEP == 1 ? KT * 4 : 0));
         for (int hh = 0; hh < L::NH; ++hh)
           tma_load_3d(smem + L::OFF_STR + s * L::TILE + hh * KT * 128, &tmK, &str_full[s], hh * 64,
-                      g, tile_row(t * KT));
+                      p.pg.head_major ? t * KT : g, tile_row(t * KT));
         if (SWEEP == 1)
           bulk_load(smem + L::OFF_LSE + s * KT * 4, p.lse + head_off + (size_t)t * KT, KT * 4,
                     &str_full[s]);

@@ -16,7 +16,7 @@ struct KeyAttnParams {
   float *part;             // [n_layers][batch][Hkv][ld]: per-head attention received by each key
   int ld;                  // cap rounded up to 128
   float scale_log2;        // log2(e) / sqrt(head_dim)
-  KvPaging pg;             // paged K (pg.table nullptr: slot-major)
+  KvLayout pg;             // paged K (pg.table nullptr: slot-major)
   int kv_rows;             // rows of the K tensor maps (a coordinate there reads zeros)
   unsigned *status;
 };
