@@ -155,7 +155,7 @@ class ClockSampler:
 # workload setup
 # ---------------------------------------------------------------------------
 
-def make_inputs(wl, device, kv_fp8=False, paged=0):
+def make_inputs(wl, device, kv_fp8=False, paged=0, head_major=False):
     """Weights and cache of the workload on `device` (seeded synthetic)."""
     shape = wl.shape
     fast = wl.mode == "layer"
@@ -168,6 +168,10 @@ def make_inputs(wl, device, kv_fp8=False, paged=0):
         to_e4m3_cache(cache)
     if paged:
         to_paged_cache(cache, paged, wl.seed)
+    if head_major:   # [B, Hkv, cap, dh] buffers
+        for key in ("k", "v"):
+            cache[key] = [x.permute(0, 2, 1, 3).contiguous() for x in cache[key]]
+        cache["kv_layout"] = 1
     return w, cache
 
 
@@ -194,6 +198,8 @@ def logical_kv(cache, key, l):
     """Slot-major [B, cap, Hkv, dh] view of K or V layer l (gathered from the
     pages of a paged cache)."""
     x = cache[key][l]
+    if cache.get("kv_layout", 0) == 1:
+        return x.permute(0, 2, 1, 3)
     if cache.get("block_table") is None:
         return x
     t = cache["block_table"].long()
@@ -302,7 +308,7 @@ def run_ours(args, dist):
     if wl.cycles > 1 and not args.single_cycle:
         raise SystemExit("multi-cycle workloads: use --single-cycle (the first refresh is timed)")
 
-    w, pristine = make_inputs(wl, dev, args.kv_fp8, args.paged)
+    w, pristine = make_inputs(wl, dev, args.kv_fp8, args.paged, args.head_major)
     work = clone_cache(pristine)
     weights, cache = pkg.Weights(w), pkg.Cache(work)
     b, cap = wl.batch, wl.cap
@@ -482,7 +488,8 @@ def run_ours(args, dist):
         "data": "synthetic (seeded random-init weights N(0,0.02); synthetic KV cache)",
         "config": {"workload": wl.name, "scorer": scorer,
                    "kv_cache": ("e4m3 (per-layer scales)" if args.kv_fp8 else "bf16") +
-                               (f", paged ({args.paged}-slot pages)" if args.paged else ""),
+                               (f", paged ({args.paged}-slot pages)" if args.paged else "") +
+                               (", head-major" if args.head_major else ""),
                    "pass": ("fast single-layer" if fast else f"full {shape.n_layers}-layer")
                    if scorer == "counter-causal" else
                    {"recency": "position", "importance": "last-layer key attention",
@@ -1004,6 +1011,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--kv-fp8", action="store_true",
                     help="store the cache's K/V as e4m3 codes with per-layer scales")
+    ap.add_argument("--head-major", action="store_true",
+                    help="keep the refresh bench's K/V head-major ([B, Hkv, cap, dh])")
     ap.add_argument("--paged", type=int, default=0, metavar="SLOTS",
                     help="keep the refresh bench's K/V in page pools of SLOTS-slot pages "
                          "(a multiple of 128) in a shuffled order, with a block table")
