@@ -871,13 +871,14 @@ def run_decode(args, dist):
     # warm-up, graph-timed, eager-timed, kernel-table and end-to-end steps
     cap = j + args.warmup + 4 * args.steps + 16
     w = synth.model_weights(shape, wl.seed, device=dev, with_kv_proj=True)
-    cache = synth.synthetic_cache(shape, [j], cap, wl.seed, device=dev)
+    B = args.batch   # sequences decoded together (each with its own memory of j slots)
+    cache = synth.synthetic_cache(shape, [j] * B, cap, wl.seed, device=dev)
     if args.kv_fp8:
         to_e4m3_cache(cache)
     weights, kc = pkg.Weights(w), pkg.Cache(cache)
-    ws = cc.alloc_workspace(cc.cc_decode_workspace_size(shape, 1, cap), dev)
-    tok = [torch.tensor([1], dtype=torch.int32, device=dev),
-           torch.empty(1, dtype=torch.int32, device=dev)]
+    ws = cc.alloc_workspace(cc.cc_decode_workspace_size(shape, B, cap), dev)
+    tok = [torch.ones(B, dtype=torch.int32, device=dev),
+           torch.empty(B, dtype=torch.int32, device=dev)]
     stream = torch.cuda.Stream(dev)   # captured work needs a stream other than the legacy default
     graphs = []
     with torch.cuda.stream(stream):
@@ -923,8 +924,8 @@ def run_decode(args, dist):
         cc.cc_timing_enable(False)
         # end to end: the current token from pinned host memory, the next one
         # read back, the step replayed from its graph
-        host_tok = torch.ones(1, dtype=torch.int32).pin_memory()
-        host_out = torch.empty(1, dtype=torch.int32).pin_memory()
+        host_tok = torch.ones(B, dtype=torch.int32).pin_memory()
+        host_out = torch.empty(B, dtype=torch.int32).pin_memory()
         e0.record(stream)
         for _ in range(args.steps // 2):
             tok[0].copy_(host_tok, non_blocking=True)
@@ -936,7 +937,7 @@ def run_decode(args, dist):
         clk = clocks.stop()
         for g in graphs:
             cc.cc_graph_destroy(g)
-        if cc.cc_get_status() != cc.CC_OK or int(host_out[0]) < 0:
+        if cc.cc_get_status() != cc.CC_OK or int(host_out.min()) < 0:
             raise SystemExit("decode did not complete")
     peaks, peak_src = load_peaks()
     d, qd, kvd, f = shape.d_model, shape.q_dim, shape.kv_dim, shape.d_ff
@@ -944,25 +945,27 @@ def run_decode(args, dist):
     work = {"gemm_qkv": ("hbm", 2.0 * d * (qd + 2 * kvd)), "gemm_oproj": ("hbm", 2.0 * qd * d),
             "gemm_gateup": ("hbm", 4.0 * d * f), "gemm_down": ("hbm", 2.0 * f * d),
             "gemm_lmhead": ("hbm", 2.0 * shape.vocab * d),
-            "attention_causal": ("hbm", 2.0 * (1 if args.kv_fp8 else 2) * kvd * n_mid)}
+            "attention_causal": ("hbm", 2.0 * (1 if args.kv_fp8 else 2) * kvd * n_mid * B)}
     table = kernel_table(kernels, args.steps, work, peaks)
     dom = max(kernels.items(), key=lambda kv: kv[1][1])[0]
     dd = table[dom]
     return {
-        "metric": "decoded tokens/sec per sequence (greedy, all layers + LM head)",
-        "value": round(dist.world / (ms * 1e-3), 1), "unit": "tokens/s", "n_gpus": dist.world,
+        "metric": ("decoded tokens/sec per sequence (greedy, all layers + LM head)" if B == 1 else
+                   f"decoded tokens/sec, {B} sequences per step (greedy, all layers + LM head)"),
+        "value": round(dist.world * B / (ms * 1e-3), 1), "unit": "tokens/s", "n_gpus": dist.world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 4),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (seeded random-init weights N(0,0.02); synthetic memory K/V)",
-        "config": {"workload": wl.name + "/decode", "memory_slots": j, "batch": 1,
+        "config": {"workload": wl.name + "/decode", "memory_slots": j, "batch": B,
                    "kv_cache": "e4m3 (per-layer scales)" if args.kv_fp8 else "bf16",
                    "layers": shape.n_layers, "d_model": shape.d_model, "vocab": shape.vocab,
                    "l2": "weights (15 GB) far exceed L2: every step streams them from HBM",
                    "launch": "one captured graph per step (cc_graph_launch)",
                    "eager_ms_per_step": round(eager_ms, 4),
                    "parallelism": f"replicas x{dist.world}"},
-        "e2e": {"value": round(dist.world / (e2e_ms * 1e-3), 1), "unit": "tokens/s",
-                "h2d_bytes_per_step": 4, "d2h_bytes_per_step": 4, "ms_per_step": round(e2e_ms, 4)},
+        "e2e": {"value": round(dist.world * B / (e2e_ms * 1e-3), 1), "unit": "tokens/s",
+                "h2d_bytes_per_step": 4 * B, "d2h_bytes_per_step": 4 * B,
+                "ms_per_step": round(e2e_ms, 4)},
         "gpu_launches": int(sum(c for c, _ in kernels.values())),
         "roofline": {"kernel": dom, "bound": dd.get("bound"), "achieved": dd.get("achieved"),
                      "peak": peaks["hbm_gbs"], "unit": dd.get("unit"), "frac": dd.get("frac"),
@@ -1011,6 +1014,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--kv-fp8", action="store_true",
                     help="store the cache's K/V as e4m3 codes with per-layer scales")
+    ap.add_argument("--batch", type=int, default=1,
+                    help="--decode: sequences decoded together (1-4 take the GEMV path)")
     ap.add_argument("--head-major", action="store_true",
                     help="keep the refresh bench's K/V head-major ([B, Hkv, cap, dh])")
     ap.add_argument("--paged", type=int, default=0, metavar="SLOTS",
