@@ -48,30 +48,7 @@ constexpr int kRegsLaunch = 168, kRegsSoftmax = 216, kRegsProducer = 64;
 static_assert(2 * 128 * kRegsSoftmax + 128 * kRegsProducer <= kThreads * kRegsLaunch,
               "register split exceeds the launch allocation");
 
-#ifndef CC_ATTN_EMU_EVERY
-#define CC_ATTN_EMU_EVERY 0   // every n-th pair of exponentials on the FMA pipe (0: none)
-#endif
-#ifndef CC_ATTN_SPLIT_P
-#define CC_ATTN_SPLIT_P 0     // hand P to the MMA in two 64-key halves
-#endif
 
-#ifdef CC_ATTN_TRACE
-// Diagnostic build only: cycle stamps of one CTA's first tiles.
-// slot = (tile * 16 + event); events: 0/1 S ready seen (half 0/1), 2/3 S loaded,
-// 4/5 P stored (warp 0 of the half), 6/7 MMA PV issued, 8..11 P stored by warps
-// 0..3 of half 0, 12/13 MMA thread enters its P wait (half 0/1).
-__device__ unsigned long long g_attn_trace[64 * 16];
-#define TRACE(cond, it, ev)                                                          \
-  do {                                                                              \
-    if ((cond) && blockIdx.x == CC_ATTN_TRACE && (it) < 64) {                       \
-      unsigned long long c_;                                                        \
-      asm volatile("mov.u64 %0, %%clock64;" : "=l"(c_));                            \
-      g_attn_trace[(it) * 16 + (ev)] = c_;                                           \
-    }                                                                               \
-  } while (0)
-#else
-#define TRACE(cond, it, ev) do { } while (0)
-#endif
 
 // 2^x by the PTX ex2.approx instruction (2 ulp; 2^-inf = 0).
 CC_DEV float fast_exp2(float x) {
@@ -80,25 +57,6 @@ CC_DEV float fast_exp2(float x) {
   return y;
 }
 
-// 2^x for a pair on the FMA pipe, x finite (clamped to >= -125): x = j + f
-// with j = round(x) (adding 1.5*2^23 leaves j in the low mantissa bits) and
-// f in [-1/2, 1/2]; 2^f by a cubic fitted to minimise the relative error on
-// [-1/2, 1/2] (max 7.5e-5, below bf16's half ulp); 2^j added to the exponent
-// field as an integer.  Coefficients re-derived by tests/test_exp2_poly.py.
-CC_DEV float2 exp2_poly2(float2 x) {
-  constexpr float kMagic = 12582912.0f;   // 1.5 * 2^23
-  x.x = fmaxf(x.x, -125.f);
-  x.y = fmaxf(x.y, -125.f);
-  const float2 t = __fadd2_rn(x, make_float2(kMagic, kMagic));
-  const float2 j = __fadd2_rn(t, make_float2(-kMagic, -kMagic));
-  const float2 f = __fadd2_rn(x, make_float2(-j.x, -j.y));
-  float2 p = __ffma2_rn(f, make_float2(0.05517164245247841f, 0.05517164245247841f),
-                        make_float2(0.2426111251115799f, 0.2426111251115799f));
-  p = __ffma2_rn(p, f, make_float2(0.6932609677314758f, 0.6932609677314758f));
-  p = __ffma2_rn(p, f, make_float2(0.9999280571937561f, 0.9999280571937561f));
-  return make_float2(__uint_as_float(__float_as_uint(p.x) + (__float_as_uint(t.x) << 23)),
-                     __uint_as_float(__float_as_uint(p.y) + (__float_as_uint(t.y) << 23)));
-}
 
 template <int DH, bool FP8 = false>
 struct AttnSmem {
@@ -183,8 +141,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t *v_fixed = v_empty + KST;       // tail tile: V rows past n zeroed
   uint64_t *s_ready = v_fixed + 1;         // [2]
   uint64_t *p_ready = s_ready + 2;         // [2] (keys 0..63 of P when split)
-  uint64_t *p_ready_hi = p_ready + 2;      // [2] keys 64..127 of P (split hand-over)
-  uint64_t *o_done = p_ready_hi + 2;       // [2]
+  uint64_t *o_done = p_ready + 2;          // [2]
   uint64_t *stg_full = o_done + 2;         // [2] FP8: fp8 K / V tile in the staging buffer
   uint64_t *stg_empty = stg_full + 2;      // [2] FP8: staging converted (free)
   uint64_t *q_conv = stg_empty + 2;        // FP8: Q converted to f16
@@ -269,7 +226,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int h = 0; h < 2; ++h) {
       mbar_init(&s_ready[h], 1);
       mbar_init(&p_ready[h], 128);
-      mbar_init(&p_ready_hi[h], 128);
       mbar_init(&o_done[h], 1);
     }
     *abort_flag = 0;
@@ -445,22 +401,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int it = 0; ok && it < ntiles; ++it) {
         const int t = t_hi - it, s = it % KST;
         const uint32_t ph = (it / KST) & 1;
-        TRACE(true, it, 14);
         if (!(ok = mbar_wait(&v_full[s], ph, abort_flag, p.status))) break;
-        TRACE(true, it, 15);
         if (!FP8 && t == t_top && n - t * BKV < BKV)
           if (!(ok = mbar_wait(v_fixed, 0, abort_flag, p.status))) break;
         for (int h = 0; h < 2; ++h) {
-          TRACE(true, it, 12 + h);
           if (!(ok = mbar_wait(&p_ready[h], it & 1, abort_flag, p.status))) break;
-          TRACE(true, it, 6 + h);
           tc_fence_after();
 #pragma unroll
           for (int kk = 0; kk < BKV / 16; ++kk) {
-            if (CC_ATTN_SPLIT_P && kk == BKV / 32) {   // second half of P
-              if (!(ok = mbar_wait(&p_ready_hi[h], it & 1, abort_flag, p.status))) break;
-              tc_fence_after();
-            }
             // B = V tile, MN-major: 64-column halves 16 KB apart (LBO),
             // 8-key groups 1024 B apart (SBO); A = P_h, bf16 pairs in TMEM.
             umma_ts(tmem + 256 + h * DH, tmem + h * 128 + kk * 8, vd[s] + kk * 128, idesc_pv,
@@ -473,9 +421,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (h == 0)
               if (!(ok = mbar_wait(&k_full[s2], ((it + 1) / KST) & 1, abort_flag, p.status))) break;
             tc_fence_after();
-            TRACE(h == 0, it, 10);
             issue_qk(it + 1, h);
-            TRACE(h == 0, it, 11);
             umma_commit(&s_ready[h]);
             if (h == 1) umma_commit(&k_empty[s2]);
           } else {
@@ -593,7 +539,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int it = 0; it < ntiles; ++it) {
       const int j0 = (t_hi - it) * BKV;
       if (!(ok = mbar_wait(&s_ready[h], it & 1, abort_flag, p.status))) break;
-      TRACE(q == 0 && lane == 0, it, 0 + h);
       tc_fence_after();
       uint32_t sr[128];
       tmem_ld32(s_t + 0, *reinterpret_cast<uint32_t(*)[32]>(&sr[0]));
@@ -601,7 +546,6 @@ __global__ void __launch_bounds__(kThreads, 1)
       tmem_ld32(s_t + 64, *reinterpret_cast<uint32_t(*)[32]>(&sr[64]));
       tmem_ld32(s_t + 96, *reinterpret_cast<uint32_t(*)[32]>(&sr[96]));
       tmem_ld_wait();
-      TRACE(q == 0 && lane == 0, it, 2 + h);
       // row max with 8 independent partial maxima (a short dependency chain)
       float mp[8];
 #pragma unroll
@@ -651,7 +595,6 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
       };
-      if (CC_ATTN_SPLIT_P) rescale();
       // p = 2^(s*sl2 - m*sl2): one packed FMA per pair, bf16 P into TMEM over S,
       // the row sum l in fp32
       const float nm = (m_used == -INFINITY) ? 0.f : -m_used * sl2;
@@ -664,30 +607,17 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int k = 0; k < 32; k += 2) {
           const float2 y = __ffma2_rn(make_float2(__uint_as_float(sr[c0 + k]),
                                                   __uint_as_float(sr[c0 + k + 1])), sl2v, nmv);
-          float2 e;
-          if (CC_ATTN_EMU_EVERY > 0 && ((c0 + k) / 2) % (CC_ATTN_EMU_EVERY > 0 ? CC_ATTN_EMU_EVERY : 1) ==
-                                           (CC_ATTN_EMU_EVERY > 0 ? CC_ATTN_EMU_EVERY : 1) - 1 &&
-              !need_mask)
-            e = exp2_poly2(y);
-          else
-            e = make_float2(fast_exp2(y.x), fast_exp2(y.y));
+          const float2 e = make_float2(fast_exp2(y.x), fast_exp2(y.y));
           pk[k / 2] = FP8 ? pack_f16x2(e.x, e.y) : pack_bf16x2(e.x, e.y);
           lsum = __fadd2_rn(lsum, e);
         }
         tmem_st16(s_t + c0 / 2, pk);
-        if (CC_ATTN_SPLIT_P && c0 == 32) {   // keys 0..63 ready: the MMA may start P V
-          tmem_st_wait();
-          tc_fence_before();
-          mbar_arrive(&p_ready[h]);
-        }
       }
       l += lsum.x + lsum.y;
-      if (!CC_ATTN_SPLIT_P) rescale();   // after P is written: S registers free for the O rows
+      rescale();   // after P is written: S registers free for the O rows
       tmem_st_wait();
       tc_fence_before();
-      TRACE(q == 0 && lane == 0, it, 4 + h);
-      TRACE(h == 0 && lane == 0 && q < 2, it, 8 + q);
-      mbar_arrive(CC_ATTN_SPLIT_P ? &p_ready_hi[h] : &p_ready[h]);
+      mbar_arrive(&p_ready[h]);
     }
     // ---- epilogue: O / l -> bf16 -> out[row_base + pos][g*G + hl][:]
     if (ok) ok = mbar_wait(&o_done[h], 0, abort_flag, p.status);
@@ -1137,11 +1067,6 @@ long long attn_units(const AttnParams &p) {
   return (long long)p.batch * p.n_kv_heads * ((p.q_span + p.P - 1) / p.P);
 }
 
-#ifdef CC_ATTN_TRACE
-extern "C" int cc_debug_attn_trace(unsigned long long *out, int n) {
-  return (int)cudaMemcpyFromSymbol(out, g_attn_trace, sizeof(unsigned long long) * (n < 1024 ? n : 1024));
-}
-#endif
 
 cudaError_t launch_attention_decode(const AttnParams &p, cudaStream_t stream) {
   if (!p.causal || p.q_span != 1 || p.group > kDecMaxG || p.kv_splits < 1 || !p.q || !p.k ||
