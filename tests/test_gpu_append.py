@@ -258,16 +258,20 @@ def _decode_check(next_tok, best, logits, tol=2e-2):
     assert abs(best - logits[next_tok]) / max(abs(logits[next_tok]), rms) < tol
 
 
-@pytest.mark.parametrize("shape_name", ["small", "small-long", "llama2", "llama2-long"])
+@pytest.mark.parametrize("shape_name", ["small", "small-long", "small-batch6", "llama2",
+                                        "llama2-long"])
 def test_decode_steps_match_oracle(cc, shape_name):
     """Greedy decode steps (teacher-forced with the oracle's tokens so both
     sides share the history): next tokens, their logits, appended K/V rows.
     The -long cases attend over enough slots that the attention splits each
-    unit's key tiles across CTAs (4 and 8 splits on a 152-SM GPU)."""
+    unit's key tiles across CTAs (4 and 8 splits on a 152-SM GPU); six
+    sequences take the tile GEMMs instead of the weight-streaming GEMVs."""
     import paper_2607_27600_gb300 as pkg
     if shape_name.startswith("small"):
         shape, seed = SMALL_GPU, 54
-        seq, cap = ([50, 20, 33], 64) if shape_name == "small" else ([1500, 300, 1999], 2048)
+        seq, cap = {"small": ([50, 20, 33], 64), "small-long": ([1500, 300, 1999], 2048),
+                    # more than four sequences: the tile GEMMs with the argmax epilogue
+                    "small-batch6": ([50, 20, 33, 1, 60, 41], 64)}[shape_name]
         w_np = to_np(synth.model_weights(shape, seed, with_kv_proj=True))
         c_np = causal_cache(shape, w_np, seq, cap, seed)
     else:
