@@ -258,8 +258,10 @@ def algorithmic_work(wl, kv_bytes=2):
         "gemm_oproj": ("tensor", 2.0 * n_rows * qd * d),
         "gemm_gateup": ("tensor", 4.0 * n_rows * d * f),
         "gemm_down": ("tensor", 2.0 * n_rows * f * d),
-        # final norm + gather-dot: h (fp32) read twice, W_U row read once, score written
-        "head_logit": ("hbm", n_rows * (8.0 * d + 2.0 * d + 4.0)),
+        # combine of the down projection's per-tile (sum h^2, sum h g W_U[x_i]) partials
+        # (the gather-dot itself runs in that GEMM's epilogue): partials and token
+        # read, score written
+        "head_logit": ("hbm", n_rows * (8.0 * -(-d // 256) + 8.0)),
         "gemm_lmhead": ("tensor", 2.0 * n_rows * d * s.vocab),
         "rmsnorm": ("hbm", n_rows * (4.0 * d * 2 + 2.0 * d)),
         # each kept slot: read + write of every layer's K and V row, H row, token, position

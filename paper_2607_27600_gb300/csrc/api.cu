@@ -230,8 +230,9 @@ bool kv_format_ok(const cc_model_cfg *c, const cc_kv_cache *kv) {
 }
 
 struct ScoreWs {
-  size_t xn, q, o, h, act, part, ztgt, flags, total;
+  size_t xn, q, o, h, act, part, ztgt, hpart, flags, total;
   int n_vtiles;
+  int n_htiles;   // logit mode: column tiles of the down projection (at most d / 128)
 };
 
 // Per-tile progress flags of split-K GEMMs (at most one wave of tiles split).
@@ -253,9 +254,12 @@ ScoreWs score_layout(const cc_model_cfg *c, int batch, int cap, cc_score_mode mo
   w.h = take(R * d * 4);
   w.act = take(R * f * 2 * split);
   w.n_vtiles = (c->vocab + 255) / 256;
+  w.n_htiles = (int)((d + 127) / 128);
   if ((mode & 0xFF) == CC_SCORE_LOGPROB) {
     w.part = take(R * w.n_vtiles * 8);
     w.ztgt = take(R * 4);
+  } else {
+    w.hpart = take(R * w.n_htiles * 8);
   }
   w.flags = take(kSplitFlags * 4);
   w.total = off;
@@ -332,7 +336,8 @@ cc_status gemm_setup(Gemm &g, int epi, const void *A, int K, const void *W, cons
   // K instead: plan_k_splits, measured faster for the down projection)
   const int nk_total = ((K + 63) / 64) * (a_split ? 2 : 1);
   const bool narrowable = epi == EPI_F32 || epi == EPI_QROPE || epi == EPI_RESID_BF16 ||
-                          (epi == EPI_RESID_F32 && nk_total < 128) || epi == EPI_BF16;
+                          ((epi == EPI_RESID_F32 || epi == EPI_RESID_LOGIT) && nk_total < 128) ||
+                          epi == EPI_BF16;
   DevState *dev_info = nullptr;
   if (narrowable && dev_state(&dev_info) &&
       ((R_est + 127) / 128) * (uint64_t)((N + 255) / 256) < (uint64_t)dev_info->sms)
@@ -414,7 +419,7 @@ cc_status gemm_setup_qkv(Gemm &g, const void *xn, const cc_model_cfg *c,
 // residual in order (flags in the caller's workspace, tagged per launch).
 void plan_k_splits(Gemm &g, int epi, int sms, unsigned *flags) {
   g.p.k_splits = 1;
-  if (epi != EPI_RESID_F32 || !flags) return;
+  if ((epi != EPI_RESID_F32 && epi != EPI_RESID_LOGIT) || !flags) return;
   const uint64_t tiles = ((g.rows_est + 127) / 128) * (uint64_t)g.p.n_tiles;
   const int nk_total = ((g.p.K + 63) / 64) * (g.p.a_split ? 2 : 1);
   if (tiles == 0 || tiles >= (uint64_t)sms || tiles > (uint64_t)kSplitFlags) return;
@@ -903,6 +908,7 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
   unsigned *status = dev->status;
   unsigned *flags = reinterpret_cast<unsigned *>(wsb + L.flags);
   if ((s = clear_split_flags(flags, st)) != CC_OK) return s;
+  int n_htiles = 0;   // column tiles of the fused head's partials
 
   if (full) {
     TimedScope t(CC_KERNEL_EMBED, st);
@@ -960,21 +966,32 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
     gu.p.ldo = split ? 2 * f : f;
     gu.p.out_split = split ? 1 : 0;
     if ((s = run_gemm(gu, EPI_SWIGLU, CC_KERNEL_GEMM_GATEUP, dev->sms, st)) != CC_OK) return s;
-    // h = h + act Wd^T
+    // h = h + act Wd^T; in logit mode the last layer's add is fused with the
+    // head: per column tile, partial sums of h^2 and of h * g . W_U[x_i]
+    const int epi_d = logit && l == c->n_layers - 1 ? EPI_RESID_LOGIT : EPI_RESID_F32;
     Gemm gd;
-    if ((s = gemm_setup(gd, EPI_RESID_F32, act, f, lw.w_down, nullptr, d, batch, cap, sl,
-                        status, split)) != CC_OK)
+    if ((s = gemm_setup(gd, epi_d, act, f, lw.w_down, nullptr, d, batch, cap, sl, status,
+                        split)) != CC_OK)
       return s;
     gd.p.out = h;
     gd.p.ldo = d;
-    plan_k_splits(gd, EPI_RESID_F32, dev->sms, flags);
-    if ((s = run_gemm(gd, EPI_RESID_F32, CC_KERNEL_GEMM_DOWN, dev->sms, st)) != CC_OK) return s;
+    if (epi_d == EPI_RESID_LOGIT) {
+      gd.p.tokens = kv->tokens;
+      gd.p.head_gain = reinterpret_cast<const __nv_bfloat16 *>(w->final_norm);
+      gd.p.head_w = reinterpret_cast<const __nv_bfloat16 *>(w->lm_head);
+      gd.p.vocab = c->vocab;
+      gd.p.head_part = reinterpret_cast<float2 *>(wsb + L.hpart);
+      n_htiles = gd.p.n_tiles;
+    }
+    plan_k_splits(gd, epi_d, dev->sms, flags);
+    if ((s = run_gemm(gd, epi_d, CC_KERNEL_GEMM_DOWN, dev->sms, st)) != CC_OK) return s;
   }
   // head
   if (logit) {
     TimedScope t(CC_KERNEL_HEAD_LOGIT, st);
-    CC_TRY(launch_head_logit(h, w->final_norm, w->lm_head, kv->tokens, scores, d, c->vocab,
-                             c->rms_eps, sl, cap, rows, status, st));
+    CC_TRY(launch_head_logit(reinterpret_cast<const float2 *>(wsb + L.hpart), n_htiles,
+                             kv->tokens, scores, d, c->vocab, c->rms_eps, sl, cap, rows, status,
+                             st));
   } else {
     {
       TimedScope t(CC_KERNEL_RMSNORM, st);

@@ -2,7 +2,7 @@
 // (bf16 operands, fp32 accumulation in TMEM) with the epilogues the
 // counter-causal layer needs (Sec. 3.1, the "standard" layer re-run over the
 // cache): RoPE'd query projection, residual adds, SwiGLU, LM-head
-// log-sum-exp partials.
+// log-sum-exp partials, and the last residual add fused with the logit head.
 //
 // Rows are the cache slots of a ragged batch: sequence b owns rows
 // b*cap + [0, seq_len[b]).  Only row tiles that hold valid slots are visited
@@ -170,10 +170,57 @@ CC_DEV long long cache_row(const GemmParams &p, int grow, bool valid) {
   return r;
 }
 
+// The final residual row x = out + acc of one tile (never stored): partial
+// sum of x^2 and partial dot of x * gain with the lm_head row of the slot's
+// own token, the two sums the logit score (Sec. 3.1) needs from this tile.
+template <int TBN>
+CC_DEV void logit_partials(const GemmParams &p, uint32_t tacc, int grow, bool valid, int nt,
+                           int tile_n0) {
+  const float *src = reinterpret_cast<const float *>(p.out) + (size_t)grow * p.ldo;
+  int tok = valid ? p.tokens[grow] : 0;
+  if (tok < 0 || tok >= p.vocab) tok = 0;   // reported by the combine
+  const __nv_bfloat16 *wrow = p.head_w + (size_t)tok * p.N;
+  float ss = 0.f, z = 0.f;
+#pragma unroll 1
+  for (int c = 0; c < TBN / 32; ++c) {
+    uint32_t r[32];
+    tmem_ld32(tacc + c * 32, r);
+    tmem_ld_wait();
+    const int col = tile_n0 + c * 32;
+    if (!valid || col >= p.N) continue;
+    const float4 *hs = reinterpret_cast<const float4 *>(src + col);
+    const uint4 *gs = reinterpret_cast<const uint4 *>(p.head_gain + col);
+    const uint4 *ws = reinterpret_cast<const uint4 *>(wrow + col);
+#pragma unroll
+    for (int v = 0; v < 4; ++v) {   // 8 columns
+      const uint4 g = gs[v], w = ws[v];
+      const float4 h0 = hs[2 * v], h1 = hs[2 * v + 1];
+      const float hv[8] = {h0.x, h0.y, h0.z, h0.w, h1.x, h1.y, h1.z, h1.w};
+      const uint32_t gw[4] = {g.x, g.y, g.z, g.w}, ww[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        const float x = __uint_as_float(r[v * 8 + k]) + hv[k];
+        const float gk = (k & 1) ? bf16_hi(gw[k / 2]) : bf16_lo(gw[k / 2]);
+        const float wk = (k & 1) ? bf16_hi(ww[k / 2]) : bf16_lo(ww[k / 2]);
+        ss = fmaf(x, x, ss);
+        z = fmaf(x * gk, wk, z);
+      }
+    }
+  }
+  if (valid) p.head_part[(size_t)grow * p.n_tiles + nt] = make_float2(ss, z);
+}
+
 template <int EPI, int TBN>
 CC_DEV void epilogue_tile(const GemmParams &p, uint32_t tacc, int grow, bool valid, int nt,
-                          int tile_n0) {
-  if constexpr (EPI == EPI_F32 || EPI == EPI_RESID_BF16 || EPI == EPI_RESID_F32) {
+                          int tile_n0, bool last) {
+  if constexpr (EPI == EPI_RESID_LOGIT) {
+    if (last) {
+      logit_partials<TBN>(p, tacc, grow, valid, nt, tile_n0);
+      return;
+    }
+  }
+  if constexpr (EPI == EPI_F32 || EPI == EPI_RESID_BF16 || EPI == EPI_RESID_F32 ||
+                EPI == EPI_RESID_LOGIT) {
     float *out = reinterpret_cast<float *>(p.out) + (size_t)grow * p.ldo;
 #pragma unroll 1
     for (int c = 0; c < TBN / 32; ++c) {
@@ -205,7 +252,7 @@ CC_DEV void epilogue_tile(const GemmParams &p, uint32_t tacc, int grow, bool val
         for (int v = 0; v < 8; ++v) {
           float4 o = make_float4(__uint_as_float(r[v * 4 + 0]), __uint_as_float(r[v * 4 + 1]),
                                  __uint_as_float(r[v * 4 + 2]), __uint_as_float(r[v * 4 + 3]));
-          if constexpr (EPI == EPI_RESID_F32) {
+          if constexpr (EPI == EPI_RESID_F32 || EPI == EPI_RESID_LOGIT) {
             float4 h = dst[v];
             o.x += h.x; o.y += h.y; o.z += h.z; o.w += h.w;
           }
@@ -411,7 +458,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int nk = (p.K + BK - 1) / BK;           // k-blocks of one operand pass
   const int nk_total = p.a_split ? 2 * nk : nk;  // split A: the hi pass, then the lo pass
   // Work item = (tile, K split): the splits of a tile are consecutive items.
-  const int S = (EPI == EPI_RESID_F32 && p.k_splits > 1) ? p.k_splits : 1;
+  const int S = ((EPI == EPI_RESID_F32 || EPI == EPI_RESID_LOGIT) && p.k_splits > 1) ? p.k_splits
+                                                                                     : 1;
   const int total_items = total * S;
 
   if (warp == 0) {
@@ -510,7 +558,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         named_barrier_sync(1, 128);
         add = split_ok != 0;   // a wait that gave up (status set) skips this split's add
       }
-      if (add) epilogue_tile<EPI, TBN>(p, tacc, grow, valid, nt, nt * TBN);
+      if (add) epilogue_tile<EPI, TBN>(p, tacc, grow, valid, nt, nt * TBN, split == S - 1);
       tc_fence_before();
       if (S > 1) {
         named_barrier_sync(1, 128);
@@ -581,6 +629,7 @@ cudaError_t launch_gemm(int epi, const CUtensorMap &a, const CUtensorMap &b, con
     case EPI_BF16: return launch<EPI_BF16>(a, b, b2, b3, p, grid, stream);
     case EPI_QKV: return launch<EPI_QKV>(a, b, b2, b3, p, grid, stream);
     case EPI_ARGMAX: return launch<EPI_ARGMAX>(a, b, b2, b3, p, grid, stream);
+    case EPI_RESID_LOGIT: return launch<EPI_RESID_LOGIT>(a, b, b2, b3, p, grid, stream);
     default: return cudaErrorInvalidValue;
   }
 }

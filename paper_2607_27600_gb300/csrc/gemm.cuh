@@ -15,8 +15,11 @@ enum GemmEpi : int {
   EPI_BF16 = 6,       // out bf16 [rows][ldo] = acc (+ bias[col] if bias)
   EPI_QKV = 7,        // fused q/k/v projections (B = Wq, B2 = Wk, B3 = Wv, stacked by column
                       // tiles): Q RoPE'd to out, K RoPE'd to out_k, V to out_v
-  EPI_ARGMAX = 8      // greedy decoding, one valid row per sequence b: out float2
+  EPI_ARGMAX = 8,     // greedy decoding, one valid row per sequence b: out float2
                       // [b][ldo = n_tiles] = (max, first column of the max) per column tile
+  EPI_RESID_LOGIT = 9 // the last residual add fused with the logit head: x = out + acc
+                      // (fp32 [rows][ldo], not stored back); head_part float2 [rows][n_tiles]
+                      // = per column tile (sum x^2, sum x * head_gain * head_w[tokens[row]])
 };
 
 struct GemmParams {
@@ -34,7 +37,11 @@ struct GemmParams {
   const int32_t *pos;      // EPI_QROPE
   const __nv_bfloat16 *bias;  // EPI_QROPE, EPI_BF16: optional per-column bias (before RoPE)
   int head_dim;            // EPI_QROPE
-  const int32_t *tokens;   // EPI_LSE
+  const int32_t *tokens;   // EPI_LSE, EPI_RESID_LOGIT
+  const __nv_bfloat16 *head_gain;   // EPI_RESID_LOGIT: final-norm gain [N]
+  const __nv_bfloat16 *head_w;      // EPI_RESID_LOGIT: lm_head [vocab][N]
+  int vocab;                        // EPI_RESID_LOGIT (tokens outside [0, vocab) read row 0)
+  float2 *head_part;                // EPI_RESID_LOGIT: [rows][n_tiles]
   float *z_target;         // EPI_LSE
   unsigned *status;
   int a_split;             // A rows are [hi | lo] (2K values): D = hi W^T + lo W^T
@@ -43,8 +50,10 @@ struct GemmParams {
                            // row tiles stay resident (A kept, B streamed per group)
   int group;
   int out_split;           // EPI_SWIGLU: out rows are [hi | lo], lo at column offset N
-  int k_splits;            // EPI_RESID_F32 only: K range split over k_splits work items per
-                           // tile (< one wave of tiles); the splits add into out in order
+  int k_splits;            // EPI_RESID_F32 / EPI_RESID_LOGIT only: K range split over
+                           // k_splits work items per tile (< one wave of tiles); the splits
+                           // add into out in order (EPI_RESID_LOGIT: the last one takes the
+                           // partials instead)
   unsigned *split_flags;   // [tiles] (k_splits > 1): per-tile progress, epoch * 16 + split
   unsigned epoch;          // per-launch tag (>= 1) of split_flags values
   int n_q_tiles, n_k_tiles;   // EPI_QKV: column tiles of Q and of K (V has n_k_tiles too)

@@ -229,11 +229,13 @@ __global__ void argmax_combine_kernel(const float2 *part, int n_tiles, const int
   }
 }
 
-// score = -(RMSNorm(h) * g) . W_U[x_i]; last valid slot +inf; past the end -inf.
+// score = -(RMSNorm(h) * g) . W_U[x_i] = -(sum h g W_U[x_i]) / rms(h), from
+// the down projection's per-column-tile partials (sum h^2, sum h g W_U[x_i]);
+// last valid slot +inf; past the end -inf.
 __global__ void __launch_bounds__(kWarps * 32)
-    head_logit_kernel(const float *h, const __nv_bfloat16 *gain, const __nv_bfloat16 *lm_head,
-                      const int32_t *tokens, float *scores, int d, int vocab, float eps,
-                      const int32_t *seq_len, int cap, int rows, unsigned *status) {
+    head_logit_kernel(const float2 *part, int n_tiles, const int32_t *tokens, float *scores,
+                      int d, int vocab, float eps, const int32_t *seq_len, int cap, int rows,
+                      unsigned *status) {
   const int lane = threadIdx.x & 31;
   const int row = blockIdx.x * kWarps + (threadIdx.x >> 5);
   if (row >= rows) return;
@@ -246,25 +248,18 @@ __global__ void __launch_bounds__(kWarps * 32)
     if (lane == 0) scores[row] = INFINITY;
     return;
   }
-  int tok = tokens[row];
-  if (tok < 0 || tok >= vocab) {
-    if (lane == 0) set_status(status, CC_ERR_DEVICE_ARG);
-    tok = 0;
+  const int tok = tokens[row];
+  if ((tok < 0 || tok >= vocab) && lane == 0) set_status(status, CC_ERR_DEVICE_ARG);
+  const float2 *pr = part + (size_t)row * n_tiles;
+  float ss = 0.f, z = 0.f;
+  for (int t = lane; t < n_tiles; t += 32) {
+    const float2 v = pr[t];
+    ss += v.x;
+    z += v.y;
   }
-  const float *hr = h + (size_t)row * d;
-  const float inv = row_inv_rms<true>(hr, d, eps, lane);
-  const __nv_bfloat16 *w = lm_head + (size_t)tok * d;
-  float z = 0.f;
-  for (int e = lane * 8; e < d; e += 256) {
-    float f[8], gf[8], wf[8];
-    load8<true>(hr, e, f);
-    unpack8(*reinterpret_cast<const uint4 *>(gain + e), gf);
-    unpack8(*reinterpret_cast<const uint4 *>(w + e), wf);
-#pragma unroll
-    for (int k = 0; k < 8; ++k) z = fmaf(f[k] * gf[k], wf[k], z);
-  }
-  z = warp_sum(z) * inv;
-  if (lane == 0) scores[row] = -z;
+  ss = warp_sum(ss);
+  z = warp_sum(z);
+  if (lane == 0) scores[row] = -(z * rsqrtf(ss / (float)d + eps));
 }
 
 // score = -(z_target - logsumexp) from per-tile (max, sum exp) partials.
@@ -358,15 +353,13 @@ cudaError_t launch_append_finish(int32_t *seq_len, const int32_t *row_hi, int ba
   return cudaGetLastError();
 }
 
-cudaError_t launch_head_logit(const float *h, const void *gain, const void *lm_head,
-                              const int32_t *tokens, float *scores, int d, int vocab, float eps,
-                              const int32_t *seq_len, int cap, int rows, unsigned *status,
-                              cudaStream_t st) {
+cudaError_t launch_head_logit(const float2 *part, int n_tiles, const int32_t *tokens,
+                              float *scores, int d, int vocab, float eps, const int32_t *seq_len,
+                              int cap, int rows, unsigned *status, cudaStream_t st) {
   if (rows <= 0) return cudaSuccess;
-  head_logit_kernel<<<blocks_for(rows), kWarps * 32, 0, st>>>(
-      h, reinterpret_cast<const __nv_bfloat16 *>(gain),
-      reinterpret_cast<const __nv_bfloat16 *>(lm_head), tokens, scores, d, vocab, eps, seq_len,
-      cap, rows, status);
+  head_logit_kernel<<<blocks_for(rows), kWarps * 32, 0, st>>>(part, n_tiles, tokens, scores, d,
+                                                             vocab, eps, seq_len, cap, rows,
+                                                             status);
   return cudaGetLastError();
 }
 

@@ -34,11 +34,12 @@ cudaError_t launch_append_finish(int32_t *seq_len, const int32_t *row_hi, int ba
 cudaError_t launch_argmax_combine(const float2 *part, int n_tiles, const int32_t *row_lo,
                                   const int32_t *row_hi, int batch, int32_t *next, float *best,
                                   cudaStream_t st);
-// scores[row] = -(final-norm(h) . lm_head[tokens[row]]), +inf at the last slot
-cudaError_t launch_head_logit(const float *h, const void *gain, const void *lm_head,
-                              const int32_t *tokens, float *scores, int d, int vocab, float eps,
-                              const int32_t *seq_len, int cap, int rows, unsigned *status,
-                              cudaStream_t st);
+// scores[row] = -(final-norm(h) . lm_head[tokens[row]]) from the per-tile
+// partials part[row][n_tiles] = (sum h^2, sum h * gain * lm_head[tokens[row]])
+// of the fused down projection; +inf at the last slot
+cudaError_t launch_head_logit(const float2 *part, int n_tiles, const int32_t *tokens,
+                              float *scores, int d, int vocab, float eps, const int32_t *seq_len,
+                              int cap, int rows, unsigned *status, cudaStream_t st);
 // scores[row] = logsumexp - z_target, +inf at the last slot
 cudaError_t launch_lse_combine(const float2 *part, int n_tiles, const float *z_target,
                                float *scores, const int32_t *seq_len, int cap, int rows,
