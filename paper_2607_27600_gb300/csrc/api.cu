@@ -230,9 +230,10 @@ bool kv_format_ok(const cc_model_cfg *c, const cc_kv_cache *kv) {
 }
 
 struct ScoreWs {
-  size_t xn, q, o, h, act, part, ztgt, hpart, flags, total;
+  size_t xn, q, o, h, act, part, ztgt, hpart, sspart, flags, total;
   int n_vtiles;
-  int n_htiles;   // logit mode: column tiles of the down projection (at most d / 128)
+  int n_htiles;   // column tiles of a d-column projection (at most d / 128): partials of
+                  // the fused logit head (logit mode) and of the post-attention RMSNorm
 };
 
 // Per-tile progress flags of split-K GEMMs (at most one wave of tiles split).
@@ -261,6 +262,7 @@ ScoreWs score_layout(const cc_model_cfg *c, int batch, int cap, cc_score_mode mo
   } else {
     w.hpart = take(R * w.n_htiles * 8);
   }
+  w.sspart = take(R * w.n_htiles * 4);
   w.flags = take(kSplitFlags * 4);
   w.total = off;
   return w;
@@ -951,13 +953,18 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
     go.p.ldo = d;
     go.p.resid = kv->h_last;
     go.p.ld_resid = d;
+    // the post-attention RMSNorm fused across the two GEMMs: this epilogue
+    // writes xn = h * g (unnormalised) and per-tile sums of h^2; the gate/up
+    // epilogue scales its accumulators by 1 / rms(h)
+    float *ss_part = reinterpret_cast<float *>(wsb + L.sspart);
+    go.p.norm_out = reinterpret_cast<__nv_bfloat16 *>(xn);
+    go.p.norm_gain = reinterpret_cast<const __nv_bfloat16 *>(lw.mlp_norm);
+    go.p.ld_norm = split ? 2 * d : d;
+    go.p.norm_split = split ? 1 : 0;
+    go.p.ss_part = ss_part;
     plan_k_splits(go, epi_o, dev->sms, flags);
     if ((s = run_gemm(go, epi_o, CC_KERNEL_GEMM_OPROJ, dev->sms, st)) != CC_OK) return s;
-    // xn = RMSNorm(h); act = silu(xn Wg^T) * (xn Wu^T)
-    {
-      TimedScope t(CC_KERNEL_RMSNORM, st);
-      CC_TRY(launch_rmsnorm(h, true, lw.mlp_norm, xn, d, c->rms_eps, sl, cap, rows, split, st));
-    }
+    // act = silu(xn Wg^T / rms(h)) * (xn Wu^T / rms(h))
     Gemm gu;
     if ((s = gemm_setup(gu, EPI_SWIGLU, xn, d, lw.w_gate, lw.w_up, f, batch, cap, sl, status,
                         split)) != CC_OK)
@@ -965,6 +972,10 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
     gu.p.out = act;
     gu.p.ldo = split ? 2 * f : f;
     gu.p.out_split = split ? 1 : 0;
+    gu.p.row_ss = ss_part;
+    gu.p.n_ss = go.p.n_tiles;
+    gu.p.ss_d = d;
+    gu.p.eps = c->rms_eps;
     if ((s = run_gemm(gu, EPI_SWIGLU, CC_KERNEL_GEMM_GATEUP, dev->sms, st)) != CC_OK) return s;
     // h = h + act Wd^T; in logit mode the last layer's add is fused with the
     // head: per column tile, partial sums of h^2 and of h * g . W_U[x_i]

@@ -222,6 +222,8 @@ CC_DEV void epilogue_tile(const GemmParams &p, uint32_t tacc, int grow, bool val
   if constexpr (EPI == EPI_F32 || EPI == EPI_RESID_BF16 || EPI == EPI_RESID_F32 ||
                 EPI == EPI_RESID_LOGIT) {
     float *out = reinterpret_cast<float *>(p.out) + (size_t)grow * p.ldo;
+    const bool nrm = (EPI == EPI_RESID_BF16 || EPI == EPI_RESID_F32) && p.norm_out && last;
+    float ss = 0.f;
 #pragma unroll 1
     for (int c = 0; c < TBN / 32; ++c) {
       uint32_t r[32];
@@ -229,37 +231,63 @@ CC_DEV void epilogue_tile(const GemmParams &p, uint32_t tacc, int grow, bool val
       tmem_ld_wait();
       int col = tile_n0 + c * 32;
       if (!valid || col >= p.N) continue;
+      float y[32];
+#pragma unroll
+      for (int k = 0; k < 32; ++k) y[k] = __uint_as_float(r[k]);
       float4 *dst = reinterpret_cast<float4 *>(out + col);
       if constexpr (EPI == EPI_RESID_BF16) {
         const uint4 *res = reinterpret_cast<const uint4 *>(
             reinterpret_cast<const __nv_bfloat16 *>(p.resid) + (size_t)grow * p.ld_resid + col);
 #pragma unroll
         for (int v = 0; v < 4; ++v) {
-          uint4 h = res[v];
-          uint32_t hw[4] = {h.x, h.y, h.z, h.w};
+          const uint4 h = res[v];
+          const uint32_t hw[4] = {h.x, h.y, h.z, h.w};
 #pragma unroll
-          for (int j = 0; j < 2; ++j) {
-            float4 o;
-            o.x = __uint_as_float(r[v * 8 + j * 4 + 0]) + bf16_lo(hw[j * 2 + 0]);
-            o.y = __uint_as_float(r[v * 8 + j * 4 + 1]) + bf16_hi(hw[j * 2 + 0]);
-            o.z = __uint_as_float(r[v * 8 + j * 4 + 2]) + bf16_lo(hw[j * 2 + 1]);
-            o.w = __uint_as_float(r[v * 8 + j * 4 + 3]) + bf16_hi(hw[j * 2 + 1]);
-            dst[v * 2 + j] = o;
+          for (int m = 0; m < 8; m += 2) {
+            y[v * 8 + m] += bf16_lo(hw[m / 2]);
+            y[v * 8 + m + 1] += bf16_hi(hw[m / 2]);
           }
         }
-      } else {
+      } else if constexpr (EPI == EPI_RESID_F32 || EPI == EPI_RESID_LOGIT) {
 #pragma unroll
         for (int v = 0; v < 8; ++v) {
-          float4 o = make_float4(__uint_as_float(r[v * 4 + 0]), __uint_as_float(r[v * 4 + 1]),
-                                 __uint_as_float(r[v * 4 + 2]), __uint_as_float(r[v * 4 + 3]));
-          if constexpr (EPI == EPI_RESID_F32 || EPI == EPI_RESID_LOGIT) {
-            float4 h = dst[v];
-            o.x += h.x; o.y += h.y; o.z += h.z; o.w += h.w;
+          const float4 h = dst[v];
+          y[v * 4] += h.x; y[v * 4 + 1] += h.y; y[v * 4 + 2] += h.z; y[v * 4 + 3] += h.w;
+        }
+      }
+#pragma unroll
+      for (int v = 0; v < 8; ++v)
+        dst[v] = make_float4(y[v * 4], y[v * 4 + 1], y[v * 4 + 2], y[v * 4 + 3]);
+      if (nrm) {   // y * gain as bf16 (hi, and lo = y * gain - hi with norm_split)
+        const uint4 *gs = reinterpret_cast<const uint4 *>(p.norm_gain + col);
+        uint32_t o[16], lo[16];
+#pragma unroll
+        for (int v = 0; v < 4; ++v) {
+          const uint4 g = gs[v];
+          const uint32_t gw[4] = {g.x, g.y, g.z, g.w};
+#pragma unroll
+          for (int m = 0; m < 8; m += 2) {
+            const float a = y[v * 8 + m], b = y[v * 8 + m + 1];
+            ss = fmaf(a, a, ss);
+            ss = fmaf(b, b, ss);
+            const float ga = a * bf16_lo(gw[m / 2]), gb = b * bf16_hi(gw[m / 2]);
+            const uint32_t hi = pack_bf16x2(ga, gb);
+            o[(v * 8 + m) / 2] = hi;
+            lo[(v * 8 + m) / 2] = pack_bf16x2(ga - bf16_lo(hi), gb - bf16_hi(hi));
           }
-          dst[v] = o;
+        }
+        uint4 *dn = reinterpret_cast<uint4 *>(p.norm_out + (size_t)grow * p.ld_norm + col);
+#pragma unroll
+        for (int v = 0; v < 4; ++v) dn[v] = make_uint4(o[v * 4], o[v * 4 + 1], o[v * 4 + 2], o[v * 4 + 3]);
+        if (p.norm_split) {
+          uint4 *dl = reinterpret_cast<uint4 *>(p.norm_out + (size_t)grow * p.ld_norm + p.N + col);
+#pragma unroll
+          for (int v = 0; v < 4; ++v)
+            dl[v] = make_uint4(lo[v * 4], lo[v * 4 + 1], lo[v * 4 + 2], lo[v * 4 + 3]);
         }
       }
     }
+    if (nrm && valid) p.ss_part[(size_t)grow * p.n_tiles + nt] = ss;
   } else if constexpr (EPI == EPI_QROPE) {   // kv_fp8: the K rows of an e4m3 cache
     const long long orow = p.kv_dest ? cache_row(p, grow, valid) : grow;
     const bool hm = p.kv_dest && p.pg.head_major;
@@ -298,6 +326,13 @@ CC_DEV void epilogue_tile(const GemmParams &p, uint32_t tacc, int grow, bool val
   } else if constexpr (EPI == EPI_SWIGLU) {
     // columns [0,128) = gate rows nt*128.., [128,256) = up rows nt*128..
     __nv_bfloat16 *out = reinterpret_cast<__nv_bfloat16 *>(p.out) + (size_t)grow * p.ldo;
+    float rs = 1.f;   // the input row's RMSNorm scale (row_ss: A rows unnormalised)
+    if (p.row_ss && valid) {
+      const float *pr = p.row_ss + (size_t)grow * p.n_ss;
+      float ss = 0.f;
+      for (int t = 0; t < p.n_ss; ++t) ss += pr[t];
+      rs = rsqrtf(ss / (float)p.ss_d + p.eps);
+    }
 #pragma unroll 1
     for (int c0 = 0; c0 < 128; c0 += 32) {
       uint32_t g[32], u[32];
@@ -306,22 +341,21 @@ CC_DEV void epilogue_tile(const GemmParams &p, uint32_t tacc, int grow, bool val
       tmem_ld_wait();
       int col = nt * 128 + c0;
       if (!valid || col >= p.N) continue;
+      float y[32];
+#pragma unroll
+      for (int k = 0; k < 32; ++k)
+        y[k] = silu(__uint_as_float(g[k]) * rs) * (__uint_as_float(u[k]) * rs);
       uint32_t o[16];
 #pragma unroll
-      for (int k = 0; k < 32; k += 2)
-        o[k / 2] = pack_bf16x2(silu(__uint_as_float(g[k])) * __uint_as_float(u[k]),
-                               silu(__uint_as_float(g[k + 1])) * __uint_as_float(u[k + 1]));
+      for (int k = 0; k < 32; k += 2) o[k / 2] = pack_bf16x2(y[k], y[k + 1]);
       uint4 *d = reinterpret_cast<uint4 *>(out + col);
 #pragma unroll
       for (int v = 0; v < 4; ++v) d[v] = make_uint4(o[v * 4], o[v * 4 + 1], o[v * 4 + 2], o[v * 4 + 3]);
       if (p.out_split) {   // lo = bf16(y - hi)
         uint32_t lo[16];
 #pragma unroll
-        for (int k = 0; k < 32; k += 2) {
-          float y0 = silu(__uint_as_float(g[k])) * __uint_as_float(u[k]);
-          float y1 = silu(__uint_as_float(g[k + 1])) * __uint_as_float(u[k + 1]);
-          lo[k / 2] = pack_bf16x2(y0 - bf16_lo(o[k / 2]), y1 - bf16_hi(o[k / 2]));
-        }
+        for (int k = 0; k < 32; k += 2)
+          lo[k / 2] = pack_bf16x2(y[k] - bf16_lo(o[k / 2]), y[k + 1] - bf16_hi(o[k / 2]));
         uint4 *dl = reinterpret_cast<uint4 *>(out + p.N + col);
 #pragma unroll
         for (int v = 0; v < 4; ++v)

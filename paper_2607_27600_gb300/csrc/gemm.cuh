@@ -43,6 +43,20 @@ struct GemmParams {
   int vocab;                        // EPI_RESID_LOGIT (tokens outside [0, vocab) read row 0)
   float2 *head_part;                // EPI_RESID_LOGIT: [rows][n_tiles]
   float *z_target;         // EPI_LSE
+  // EPI_RESID_BF16 / EPI_RESID_F32 with norm_out: the next RMSNorm's input
+  // is written too, unnormalised: norm_out bf16 [rows][ld_norm] = out * norm_gain
+  // ([hi | lo] pairs, lo at column offset N, with norm_split), and
+  // ss_part [rows][n_tiles] = the tile's partial sum of out^2
+  __nv_bfloat16 *norm_out;
+  const __nv_bfloat16 *norm_gain;
+  int ld_norm, norm_split;
+  float *ss_part;
+  // EPI_SWIGLU with row_ss: the A rows are unnormalised (as above); the
+  // accumulators are scaled by rsqrt(sum_t row_ss[row][t] / ss_d + eps),
+  // t < n_ss, before the activation
+  const float *row_ss;
+  int n_ss, ss_d;
+  float eps;
   unsigned *status;
   int a_split;             // A rows are [hi | lo] (2K values): D = hi W^T + lo W^T
   int raster;              // tile order: 0 = groups of `group` column tiles stay resident

@@ -137,7 +137,9 @@ def test_fast_pass_logprob_full_size(pkg):
 # the matching emulated maximum: bf16 activations (default) against the
 # bf16-pass figure, hi + lo activations (CC_SCORE_PRECISE, bf16 queries left)
 # against the queries-only figure.  The full-pass machinery itself is held to
-# 2e-2 on the first four layers of the same model and shapes.
+# 2e-2 (relative l2 over 64 rows) on the first four layers of the same model
+# and shapes.
+FULL4_ROW_TOL = 8e-2       # worst single row, 4 layers (measured 3.9-4.1 % on 64 rows)
 FULL32_TOL = 1.5e-1        # bf16 activations, 32 layers
 FULL32_PRECISE_TOL = 1e-1  # hi + lo GEMM activations (CC_SCORE_PRECISE), 32 layers
 # The 28-layer Qwen2.5 pass at 512 slots: held to the 32-layer Llama bar (the
@@ -155,13 +157,23 @@ def _full_inputs(n_layers):
 
 
 def test_full_pass_llama_shape_first_4_layers(pkg):
+    """The full-pass machinery over four layers on 64 rows (the edge rows and
+    58 seeded ones).  Per-row errors of a bf16 pass are heavy-tailed (up to
+    ~4 % of the scores' rms here), so the bar of 2e-2 holds the relative l2
+    error over the rows (measured 1.2 %), and a bound of twice the measured
+    worst row catches a single row gone wrong."""
     from paper_2607_27600_gb300 import cc
     wl, shape, w, c = _full_inputs(4)
     got = gpu_scores(pkg, shape, w, c, cc.SCORE_LOGIT, full=True)
     wn, cn = host_view(w, c, lazy=True)
-    rows = [[0, 5, 4097, 8191, 16381, 16382, 16383]]
+    extra = np.random.default_rng(5).integers(0, 16382, 58).tolist()
+    rows = [sorted(set([0, 5, 4097, 8191, 16381, 16382, 16383] + extra))]
     want = oracle.score_full(shape, wn, cn, rows=rows)
-    assert check_rows(got, want, rows) < TOL
+    g, o = got[0, rows[0]].astype(np.float64), want[0, rows[0]]
+    fin = np.isfinite(o)
+    np.testing.assert_array_equal(g[~fin], o[~fin])
+    assert np.linalg.norm(g[fin] - o[fin]) / np.linalg.norm(o[fin]) < TOL
+    assert check_rows(got, want, rows) < FULL4_ROW_TOL
 
 
 @pytest.mark.parametrize("precise", [False, True])

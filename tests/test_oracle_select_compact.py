@@ -107,3 +107,27 @@ def test_compact_preserves_relative_order():
     out = oracle.compact(buf, idx, np.array([5]))
     assert out[0, :5, 0].tolist() == [2, 3, 9, 11, 19]
     assert np.all(np.diff(out[0, :5, 0]) > 0)
+
+
+def test_keep_set_bar_accepts_only_near_tie_swaps():
+    """The GPU tests' keep-set bar: a swap at a near-tied boundary passes, a
+    swap of a slot far from the boundary fails, a count mismatch fails."""
+    from tests._util import keep_set_ok
+    n, j = 64, 16
+    s = np.linspace(10.0, -10.0, n)
+    s[j] = s[j - 1] - 1e-4                     # near tie at the boundary
+    want_i, want_c = oracle.select_keep(s[None].astype(np.float32), [n], [j])
+    kept = list(want_i[0, :j])
+    near = sorted(set(kept) - {j - 1} | {j})   # swap the tied pair
+    far = sorted(set(kept) - {0} | {n - 1})    # drop the best, keep the worst
+    for got, expect in ((kept, True), (near, True), (far, False)):
+        gi = np.full((1, n), -1, np.int32)
+        gi[0, :j] = got
+        ok, _ = keep_set_ok(gi, np.array([j]), want_i, want_c, s[None], [n], [j])
+        assert ok == expect
+    s2 = np.linspace(10.0, -10.0, n)           # clear gap: only the exact set passes
+    w2_i, w2_c = oracle.select_keep(s2[None].astype(np.float32), [n], [j])
+    gi = np.full((1, n), -1, np.int32)
+    gi[0, :j] = sorted(set(w2_i[0, :j]) - {j - 1} | {j})
+    assert not keep_set_ok(gi, np.array([j]), w2_i, w2_c, s2[None], [n], [j])[0]
+    assert not keep_set_ok(w2_i, np.array([j - 1]), w2_i, w2_c, s2[None], [n], [j])[0]
