@@ -412,22 +412,35 @@ def run_ours(args, dist):
         h2d -= host["k"].numel() * host["k"].element_size() * 2
     d2h = out_idx.numel() * 4 + out_cnt.numel() * 4
 
+    # K/V uploads run on a copy stream and the library waits for each layer's
+    # event right before the layer's first K/V reader (cc_kv_cache.kv_ready),
+    # so they overlap the kernels ahead of it; the host link is one queue, so
+    # they start once the inputs of the first kernels have landed
+    up = torch.cuda.Stream(dev)
+    n_l = len(work["k"])
+    kv_layers = [n_l - 1] if fast else list(range(n_l))
+    ready = [torch.cuda.Event() if l in kv_layers else None for l in range(n_l)]
+    for e in ready:
+        if e is not None:
+            e.record(up)
+
     def e2e_step():
-        if fast:
-            work["h_last"].copy_(host["h_last"], non_blocking=True)
-            work["k"][-1].copy_(host["k"], non_blocking=True)
-            work["v"][-1].copy_(host["v"], non_blocking=True)
-        else:
-            for dst, src in zip(work["k"], host["k_all"]):
-                dst.copy_(src, non_blocking=True)
-            for dst, src in zip(work["v"], host["v_all"]):
-                dst.copy_(src, non_blocking=True)
+        work["seq_len"].copy_(host["seq_len"], non_blocking=True)
         work["tokens"].copy_(host["tokens"], non_blocking=True)
         work["pos"].copy_(host["pos"], non_blocking=True)
-        work["seq_len"].copy_(host["seq_len"], non_blocking=True)
+        if fast:
+            work["h_last"].copy_(host["h_last"], non_blocking=True)
+        up.wait_stream(stream)
+        with torch.cuda.stream(up):
+            for l in kv_layers:
+                work["k"][l].copy_(host["k"] if fast else host["k_all"][l], non_blocking=True)
+                work["v"][l].copy_(host["v"] if fast else host["v_all"][l], non_blocking=True)
+                ready[l].record(up)
         step()
         out_idx.copy_(keep_idx, non_blocking=True)
         out_cnt.copy_(keep_count, non_blocking=True)
+
+    cache.set_kv_ready(ready)
 
     e2e_ms = []
     for i in range(args.steps):
@@ -441,6 +454,7 @@ def run_ours(args, dist):
         t1.record(stream)
         torch.cuda.synchronize(dev)
         e2e_ms.append(t0.elapsed_time(t1))
+    cache.set_kv_ready(None)
     clk = clocks.stop()
     e2e_ms_max = dist.max(sum(e2e_ms) / len(e2e_ms))
     status = cc.cc_get_status()
@@ -461,8 +475,6 @@ def run_ours(args, dist):
                  "share": round(tot / max(1e-9, sum(t for _, t in kernels.values())), 4)}
         if name in work_tbl:
             bound, amount = work_tbl[name]
-            if name == "rmsnorm":
-                amount = amount   # per launch, same row count every launch
             if bound == "tensor":
                 ach = amount / (per * 1e-3) / 1e12
                 entry.update({"bound": "tensor", "achieved": round(ach, 2), "unit": "TFLOP/s",

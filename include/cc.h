@@ -177,6 +177,15 @@ typedef struct {
   int32_t n_pages;
   int32_t kv_layout;  /* cc_kv_layout of k and v (0 = slot-major); a head-major cache is
                          not paged                                                      */
+  /* Optional HOST array [n_layers] of cudaEvent_t (as void *; the array or any entry may
+   * be NULL): the caller's writes of layer l's K/V may still be in flight on another
+   * stream when a call is enqueued; the call's stream waits for kv_ready[l] right before
+   * its first kernel that reads or writes layer l's K/V (the scoring pass before layer
+   * l's attention, the append and decode at the start of layer l, the comparison scorers
+   * and the compaction before their launch), so an upload of the cache overlaps the
+   * kernels that do not need it.  Events recorded outside a graph capture cannot be
+   * waited on inside one (CC_ERR_CUDA). */
+  void *const *kv_ready;
 } cc_kv_cache;
 
 /* ---- scoring (Sec. 3.1) ---------------------------------------------------

@@ -64,7 +64,8 @@ class cc_kv_cache(ctypes.Structure):
                 ("h2o_acc", ctypes.c_void_p), ("kv_format", ctypes.c_int32),
                 ("kv_scale", ctypes.POINTER(ctypes.c_float)),
                 ("block_table", ctypes.c_void_p), ("page_size", ctypes.c_int32),
-                ("n_pages", ctypes.c_int32), ("kv_layout", ctypes.c_int32)]
+                ("n_pages", ctypes.c_int32), ("kv_layout", ctypes.c_int32),
+                ("kv_ready", ctypes.POINTER(ctypes.c_void_p))]
 
 KV_BF16, KV_E4M3 = 0, 1
 KV_SLOT_MAJOR, KV_HEAD_MAJOR = 0, 1
@@ -229,7 +230,8 @@ class Cache:
     [B, cap, d] or None); with "block_table" (int32 [B, cap // page_size]),
     "page_size" and k[l], v[l] page pools [n_pages, page_size, Hkv, dh] the
     K/V are paged; with "kv_layout": KV_HEAD_MAJOR, k[l], v[l] are
-    [B, Hkv, cap, dh].  Keeps the tensors alive."""
+    [B, Hkv, cap, dh].  Keeps the tensors alive.  set_kv_ready() attaches the
+    per-layer events of K/V uploads still in flight on another stream."""
 
     def __init__(self, c: dict):
         self.d = c
@@ -254,7 +256,26 @@ class Cache:
                              _dev_ptr(c.get("h_last"), "h_last"),
                              _dev_ptr(c.get("h2o_acc"), "h2o_acc"), fmt, self._scale,
                              _dev_ptr(table, "block_table"), page, n_pages,
-                             int(c.get("kv_layout", KV_SLOT_MAJOR)))
+                             int(c.get("kv_layout", KV_SLOT_MAJOR)), None)
+        self._ready = None
+
+    def set_kv_ready(self, events):
+        """events: one torch.cuda.Event (already recorded once) or None per
+        layer, or None for no waits (cc_kv_cache.kv_ready)."""
+        if events is None:
+            self._ready = None
+            self.c.kv_ready = None
+            return
+        if len(events) != len(self._k):
+            raise ValueError("kv_ready needs one entry per layer")
+        handles = []
+        for e in events:
+            h = 0 if e is None else int(e.cuda_event)
+            if e is not None and h == 0:
+                raise ValueError("record a kv_ready event once before attaching it")
+            handles.append(h or None)
+        self._ready = (ctypes.c_void_p * len(handles))(*handles)
+        self.c.kv_ready = self._ready
 
 
 def _cfg(cfg):

@@ -30,6 +30,8 @@
 #include <vector>
 
 namespace cc {
+
+cudaError_t wait_kv_ready(const cc_kv_cache *kv, int l0, int l1, cudaStream_t st);
 __device__ unsigned g_status_word;   // first device-side error since the last cc_get_status
 }
 
@@ -736,6 +738,7 @@ cc_status run_append(const cc_model_cfg *c, const cc_model_weights *w, const cc_
   for (int l = 0; l < c->n_layers; ++l) {
     const cc_layer_weights &lw = w->layers[l];
     const KvFmt kvf = kv_fmt(c, kv, l);   // e4m3 cache: K/V rows written as codes of value / scale
+    CC_TRY(wait_kv_ready(kv, l, l + 1, st));
     if (l == c->n_layers - 1 && kv->h_last) {   // H^(L-1), recorded for the fast approximation
       TimedScope t(CC_KERNEL_APPEND, st);
       CC_TRY(launch_store_bf16(h, kv->h_last, d, hi, lo, cap, rows, st, max_count));
@@ -939,6 +942,7 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
     rope_turns(c, gq.p.turns);
     if ((s = run_gemm(gq, EPI_QROPE, CC_KERNEL_GEMM_QROPE, dev->sms, st)) != CC_OK) return s;
     // O = counter-causal attention
+    CC_TRY(wait_kv_ready(kv, l, l + 1, st));
     if ((s = run_attention(c, q, kv->k[l], kv->v[l], o, sl, batch, cap, status, st, split,
                            nullptr, 0, nullptr, 0, kv_fmt(c, kv, l))) !=
         CC_OK)
@@ -1175,6 +1179,7 @@ cc_status run_keyattn(const cc_model_cfg *c, const cc_kv_cache *kv, int l0, int 
   p.part = p.lse + (size_t)p.n_layers * batch * c->n_kv_heads * p.ld;
   p.scale_log2 = (float)(1.4426950408889634 / sqrt((double)dh));
   p.status = status;
+  CC_TRY(wait_kv_ready(kv, l0, l1, st));
   TimedScope t(CC_KERNEL_KEYATTN, st);
   CC_TRY(launch_keyattn(a, st));
   CC_TRY(launch_keyattn_finish(p, out, mean, accumulate, st));
@@ -1371,6 +1376,7 @@ cc_status cc_compact_kv(const cc_model_cfg *cfg, const cc_kv_cache *cache,
   plan.p.status = dev->status;
   plan.p.withhold_unit = g_withhold_unit;
   g_withhold_unit = -1;
+  CC_TRY(wait_kv_ready(cache, 0, cfg->n_layers, st));
   TimedScope t(CC_KERNEL_COMPACT, st);
   CC_TRY(launch_compact(plan.p, dev->sms, st));
   return CC_OK;
@@ -1550,6 +1556,18 @@ const char *cc_kernel_name(int32_t kind) {
 #include "internal.h"
 
 namespace cc {
+
+// cc_kv_cache.kv_ready: the caller's uploads of layers [l0, l1) land before what follows on st
+cudaError_t wait_kv_ready(const cc_kv_cache *kv, int l0, int l1, cudaStream_t st) {
+  if (!kv->kv_ready) return cudaSuccess;
+  for (int l = l0; l < l1; ++l) {
+    if (!kv->kv_ready[l]) continue;
+    const cudaError_t e = cudaStreamWaitEvent(st, reinterpret_cast<cudaEvent_t>(kv->kv_ready[l]), 0);
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
 
 cc_status compact_plan_build(const cc_model_cfg *cfg, const cc_kv_cache *cache, CompactParams &p,
                              size_t &scratch_bytes) {

@@ -65,6 +65,7 @@ extern "C" cc_status cc_compact_kv_static(const cc_model_cfg *cfg, const cc_kv_c
   p.keep_count = keep_count;
   p.seq_len = cache->seq_len;
   p.status = status;
+  if (cc::wait_kv_ready(cache, 0, cfg->n_layers, st) != cudaSuccess) return CC_ERR_CUDA;
   if (cc::launch_compact(p, sms, st) != cudaSuccess) return CC_ERR_CUDA;
   return CC_OK;
 }

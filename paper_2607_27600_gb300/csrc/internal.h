@@ -15,5 +15,8 @@ cc_status compact_plan_bind(const cc_model_cfg *cfg, const cc_kv_cache *cache, C
                             void *scratch, cudaStream_t st);
 // Status-word address and SM count of the current device.
 bool current_device_info(unsigned **status, int *sms);
+// Makes `st` wait for the caller's K/V-ready events (cc_kv_cache.kv_ready) of
+// layers [l0, l1).
+cudaError_t wait_kv_ready(const cc_kv_cache *kv, int l0, int l1, cudaStream_t st);
 
 }  // namespace cc

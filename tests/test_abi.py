@@ -92,3 +92,26 @@ def test_compaction_plan_covers_every_array(lib):
     n_full = lib.cc_compact_workspace_size(ctypes.byref(cfg), ctypes.byref(full))
     n_x = lib.cc_compact_workspace_size(ctypes.byref(cfg), ctypes.byref(only_x))
     assert n_x > 256 and n_full > n_x
+
+
+def _header_struct_fields(name):
+    src = open(os.path.join(ROOT, "include", "cc.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    m = re.search(r"typedef struct\s*\{([^}]*)\}\s*" + name + r"\s*;", src)
+    assert m, name
+    fields = []
+    for decl in m.group(1).split(";"):
+        decl = decl.strip()
+        if decl:
+            fields += [re.findall(r"(\w+)\s*$", part.strip())[0] for part in decl.split(",")]
+    return fields
+
+
+@pytest.mark.parametrize("name", ["cc_model_cfg", "cc_layer_weights", "cc_model_weights",
+                                  "cc_kv_cache"])
+def test_binding_structs_match_the_header(name):
+    """The ctypes mirrors of the public structs list the header's fields in
+    the header's order (a missing or reordered field would shift every later
+    member the library reads)."""
+    from paper_2607_27600_gb300 import cc
+    assert [f[0] for f in getattr(cc, name)._fields_] == _header_struct_fields(name)
