@@ -826,13 +826,15 @@ cc_status run_append(const cc_model_cfg *c, const cc_model_weights *w, const cc_
     go.p.row_lo = lo;
     go.p.out = h;
     go.p.ldo = d;
+    // the post-attention RMSNorm fused across the O and gate/up epilogues
+    // (as in the scoring pass)
+    float *ss_part = reinterpret_cast<float *>(wsb + L.s.sspart);
+    go.p.norm_out = reinterpret_cast<__nv_bfloat16 *>(xn);
+    go.p.norm_gain = reinterpret_cast<const __nv_bfloat16 *>(lw.mlp_norm);
+    go.p.ld_norm = d;
+    go.p.ss_part = ss_part;
     plan_k_splits(go, EPI_RESID_F32, dev->sms, flags);
     if ((s = run_gemm(go, EPI_RESID_F32, CC_KERNEL_GEMM_OPROJ, dev->sms, st)) != CC_OK) return s;
-    {
-      TimedScope t(CC_KERNEL_RMSNORM, st);
-      CC_TRY(launch_rmsnorm(h, true, lw.mlp_norm, xn, d, c->rms_eps, hi, cap, rows, false, st, lo,
-                            max_count));
-    }
     Gemm gu;
     if ((s = gemm_setup(gu, EPI_SWIGLU, xn, d, lw.w_gate, lw.w_up, f, batch, cap, hi, status,
                         false, used)) != CC_OK)
@@ -840,6 +842,10 @@ cc_status run_append(const cc_model_cfg *c, const cc_model_weights *w, const cc_
     gu.p.row_lo = lo;
     gu.p.out = act;
     gu.p.ldo = f;
+    gu.p.row_ss = ss_part;
+    gu.p.n_ss = go.p.n_tiles;
+    gu.p.ss_d = d;
+    gu.p.eps = c->rms_eps;
     if ((s = run_gemm(gu, EPI_SWIGLU, CC_KERNEL_GEMM_GATEUP, dev->sms, st)) != CC_OK) return s;
     Gemm gd;
     if ((s = gemm_setup(gd, EPI_RESID_F32, act, f, lw.w_down, nullptr, d, batch, cap, hi, status,
