@@ -1075,7 +1075,7 @@ cc_status compact_plan(const cc_model_cfg *c, const cc_kv_cache *kv, CompactPlan
     A.paged = paged ? 1 : 0;
     A.head_major = head_major ? 1 : 0;
     A.rows_per_chunk = bulk ? (row_bytes <= p.stage_bytes ? p.stage_bytes / row_bytes : 0)
-                            : p.stage_bytes / 4;
+                            : std::min(kCompactSmallRows, p.stage_bytes / 4);
     if (A.rows_per_chunk < 1) return false;
     A.n_chunks = (kv->cap + A.rows_per_chunk - 1) / A.rows_per_chunk;
     A.dep_class = class_of(A.rows_per_chunk);
@@ -1090,16 +1090,19 @@ cc_status compact_plan(const cc_model_cfg *c, const cc_kv_cache *kv, CompactPlan
   p.pg = kv_layout(c, kv);   // K/V rows through the block table when paged
   const bool paged = kv->block_table != nullptr;
   const bool hm = kv->kv_layout == CC_KV_HEAD_MAJOR;   // rows of Hkv segments
+  // the 4-byte arrays first: their gathers then overlap the bulk copies
+  // instead of trailing them (units run in ascending order)
+  if (!add(kv->tokens, 4, false) || !add(kv->pos, 4, false)) return CC_ERR_INVALID_ARG;
+  if (!add(kv->h2o_acc, 4, false)) return CC_ERR_INVALID_ARG;   // comparison scorer totals
   for (int l = 0; l < c->n_layers; ++l) {
     if (!add(kv->k[l], kv_row, true, paged, hm) || !add(kv->v[l], kv_row, true, paged, hm))
       return CC_ERR_UNSUPPORTED;
   }
   if (!add(kv->h_last, c->d_model * 2, true)) return CC_ERR_UNSUPPORTED;
-  if (!add(kv->tokens, 4, false) || !add(kv->pos, 4, false)) return CC_ERR_INVALID_ARG;
-  if (!add(kv->h2o_acc, 4, false)) return CC_ERR_INVALID_ARG;   // comparison scorer totals
   p.n_arrays = n;
   p.total_units = units;
   if (n < 2 || units < 2) return CC_ERR_INVALID_ARG;   // tokens and pos are always compacted
+  compact_cache_units(p);
   size_t deps_entries = 0;
   for (int c = 0; c < p.n_classes; ++c) {
     p.class_offset[c] = (long long)deps_entries;

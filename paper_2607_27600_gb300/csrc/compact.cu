@@ -160,12 +160,16 @@ __global__ void __launch_bounds__(kThreads)
       p.seq_len[b] = (j >= 0 && j <= p.cap) ? j : 0;
     }
   }
-  __syncwarp();
+  const int n_pairs = p.n_arrays * p.batch;
+  int *ub_smem = reinterpret_cast<int *>(smem + (size_t)n_warps * 2 * p.stage_bytes);
+  if (p.ub_cached)
+    for (int i = threadIdx.x; i <= n_pairs; i += blockDim.x) ub_smem[i] = p.unit_base[i];
+  __syncthreads();
+  const int *unit_base = p.ub_cached ? ub_smem : p.unit_base;
   uint32_t phase[2] = {0, 0};
   volatile int no_abort = 0;
 
-  const int n_pairs = p.n_arrays * p.batch;
-  const int total = p.unit_base[n_pairs];
+  const int total = unit_base[n_pairs];
   const int stride = gridDim.x * n_warps;
   int next_t = blockIdx.x * n_warps + warp;
   auto take = [&]() -> Unit {
@@ -178,11 +182,11 @@ __global__ void __launch_bounds__(kThreads)
     int lo = 0, hi = n_pairs - 1;   // last pair whose first unit <= t
     while (lo < hi) {
       const int mid = (lo + hi + 1) >> 1;
-      if (p.unit_base[mid] <= u.t) lo = mid; else hi = mid - 1;
+      if (unit_base[mid] <= u.t) lo = mid; else hi = mid - 1;
     }
     u.a = lo / p.batch;
     u.b = lo - u.a * p.batch;
-    u.c = u.t - p.unit_base[lo];
+    u.c = u.t - unit_base[lo];
     const CompactArray &A = p.arr[u.a];
     int J = p.keep_count[u.b];
     if (J < 0 || J > p.cap) J = 0;
@@ -259,6 +263,7 @@ __global__ void __launch_bounds__(kThreads)
       u.loaded = true;
     } else {   // 4-byte rows: plain loads staged in shared memory
       uint32_t *st = reinterpret_cast<uint32_t *>(buf[s]);
+#pragma unroll 8
       for (int k = u.k0 + lane; k < u.k1; k += 32)
         st[k - u.k0] = reinterpret_cast<const uint32_t *>(base)[seq_off + source(kidx, k, true)];
     }
@@ -299,7 +304,7 @@ __global__ void __launch_bounds__(kThreads)
                               (size_t)cur.b * p.class_chunks[A.dep_class] + cur.c];
         const int hi = min(d.y, cur.c - 1);
         for (int c2 = max(d.x, 0); c2 <= hi && go; ++c2) {
-          go = wait_flag(&p.flags[p.unit_base[cur.a * p.batch + cur.b] + c2], p.status);
+          go = wait_flag(&p.flags[unit_base[cur.a * p.batch + cur.b] + c2], p.status);
           waited = true;
         }
       }
@@ -345,8 +350,14 @@ bool compact_shape(int max_row_bytes, int &stage_bytes, int &warps) {
   return warps >= 1;
 }
 
+void compact_cache_units(CompactParams &p) {
+  const size_t table = (((size_t)p.n_arrays * p.batch + 1) * sizeof(int) + 15) & ~size_t(15);
+  p.ub_cached = (size_t)p.warps * 2 * p.stage_bytes + 128 + table <= (size_t)kCompactSmemBytes;
+}
+
 size_t compact_smem_bytes(const CompactParams &p) {
-  return (size_t)p.warps * 2 * p.stage_bytes + 128;
+  const size_t table = p.ub_cached ? ((size_t)p.n_arrays * p.batch + 1) * sizeof(int) : 0;
+  return (size_t)p.warps * 2 * p.stage_bytes + 128 + ((table + 15) & ~size_t(15));
 }
 
 cudaError_t launch_compact(const CompactParams &p, int sms, cudaStream_t st) {

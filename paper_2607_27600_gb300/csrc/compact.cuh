@@ -15,6 +15,10 @@ constexpr int kCompactStageBytes = 4 * 1024;
 constexpr int kCompactTargetBytes = 192 * 1024;   // staging the shape aims for
 constexpr int kCompactSmemBytes = 224 * 1024;     // dynamic shared memory limit of the copy kernel
 constexpr int kMaxCompactArrays = 2 * 128 + 3;
+// Slots per unit of a 4-byte array (tokens, positions, H2O totals): eight
+// gathers per lane, so a sequence's few units spread over many warps
+// instead of one warp walking all of them.
+constexpr int kCompactSmallRows = 256;
 constexpr int kMaxDepClasses = 3;        // distinct chunk sizes (K/V rows, H rows, 4-byte rows)
 
 struct CompactArray {
@@ -49,6 +53,9 @@ struct CompactParams {
   int withhold_unit;          // test hook: this unit never publishes its flag (-1: none)
   int stage_bytes;            // shared-memory buffer of a unit (multiple of 128)
   int warps;                  // warps per CTA (each with two buffers)
+  int ub_cached;              // unit_base is copied into shared memory after the buffers
+                              // (n_arrays * batch + 1 entries fit): a unit's lookup of its
+                              // (array, sequence) then costs no global round trips
   KvLayout pg;                // paged K/V arrays: pool row of logical slot (b, i)
   CompactArray arr[kMaxCompactArrays];
 };
@@ -56,6 +63,8 @@ struct CompactParams {
 // Buffer size and warps per CTA for the largest row a cache moves (bytes);
 // false when one row does not fit the shared-memory budget.
 bool compact_shape(int max_row_bytes, int &stage_bytes, int &warps);
+// Sets p.ub_cached when the unit table fits beside the staging buffers.
+void compact_cache_units(CompactParams &p);
 size_t compact_smem_bytes(const CompactParams &p);
 // Launches the pre-passes and the (cooperative) compaction; `sms` = SM count.
 cudaError_t launch_compact(const CompactParams &p, int sms, cudaStream_t st);
