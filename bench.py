@@ -264,12 +264,12 @@ def algorithmic_work(wl, kv_bytes=2):
         "head_logit": ("hbm", n_rows * (8.0 * -(-d // 256) + 8.0)),
         "gemm_lmhead": ("tensor", 2.0 * n_rows * d * s.vocab),
         # the pre-attention norm (the post-attention one is fused into the O / gate-up
-        # GEMMs): input row read twice (bf16 H^(L-1) in layer mode, fp32 h in the
-        # full pass), bf16 row written
-        "rmsnorm": ("hbm", n_rows * ((2.0 if wl.mode == "layer" else 4.0) * d * 2 + 2.0 * d)),
+        # GEMMs): input row read (bf16 H^(L-1) in layer mode, fp32 h in the full
+        # pass), bf16 row written
+        "rmsnorm": ("hbm", n_rows * ((2.0 if wl.mode == "layer" else 4.0) * d + 2.0 * d)),
         # each kept slot: read + write of every layer's K and V row, H row, token, position
         "compact": ("hbm", 2.0 * moved * (n_arrays_kv * kv_row + h_row + 8)),
-        # 9 passes over the scores (8 radix passes + the emit pass)
+        # at most 9 passes over the scores (up to 8 radix passes + the emit pass)
         "select": ("hbm", 9.0 * 4.0 * n_rows),
     }
 

@@ -4,10 +4,13 @@
 // One CTA (1024 threads) per sequence.  Each slot j gets the unique 64-bit
 // key (monotone(score_j) << 32) | j, so "descending score, ties toward the
 // later slot" is plain descending key order and exactly J keys are >= the
-// J-th largest key T.  T is found by an 8-pass MSB radix select (8 bits per
-// pass, warp-level digit search over a shared histogram); a final pass flags
-// key >= T and writes the kept slots in ascending slot order through a
-// block-wide prefix scan.
+// J-th largest key T.  T is found by an MSB radix select (8 bits per pass,
+// warp-level digit search over a shared histogram, at most 8 passes); it
+// stops early once the bucket holding the boundary has exactly as many keys
+// as are still needed: then every key of the bucket is kept, and the prefix
+// with all lower bits zero is a threshold with exactly J keys at or above it.
+// A final pass flags key >= T and writes the kept slots in ascending slot
+// order through a block-wide prefix scan.
 #include "select.cuh"
 
 namespace cc {
@@ -64,7 +67,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                   int n_sink, int32_t *keep_idx, int32_t *keep_count, unsigned *status) {
   __shared__ unsigned hist[256];
   __shared__ int wsum[33];
-  __shared__ int s_digit, s_above;
+  __shared__ int s_digit, s_above, s_count;
   const int b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int n = seq_len[b];
   if (n < 0 || n > cap) {
@@ -119,7 +122,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         unsigned run = excl;
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
-          if (run + c[e] >= (unsigned)k) { s_digit = base - e; s_above = (int)run; break; }
+          if (run + c[e] >= (unsigned)k) {
+            s_digit = base - e;
+            s_above = (int)run;
+            s_count = (int)c[e];
+            break;
+          }
           run += c[e];
         }
       }
@@ -127,7 +135,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncthreads();
     prefix |= uint64_t(s_digit) << shift;
     k -= s_above;
+    const bool settled = s_count == k;   // the whole bucket is kept
     __syncthreads();
+    if (settled) break;
   }
   const uint64_t T = prefix;
 

@@ -117,13 +117,20 @@ def test_tiny_refresh_keep_set_and_compaction(pkg, tiny):
     assert cache.d["seq_len"].cpu().tolist() == gc.tolist()
 
 
-@pytest.mark.parametrize("seq,budget,n_sink", [([512], [128], 0), ([512, 300, 1, 7], [64, 300, 1, 3], 2),
-                                               ([4096, 5000], [1000, 17], 0)])
-def test_select_exact_vs_oracle_on_same_scores(pkg, seq, budget, n_sink):
+@pytest.mark.parametrize("seq,budget,n_sink,dist", [
+    ([512], [128], 0, "ties"), ([512, 300, 1, 7], [64, 300, 1, 3], 2, "ties"),
+    ([4096, 5000], [1000, 17], 0, "ties"),
+    # continuous scores: the radix select settles after a few passes
+    ([32768, 8192, 131072, 9], [8192, 8191, 1000, 2], 1, "normal"),
+    ([8192], [2048], 0, "normal")])
+def test_select_exact_vs_oracle_on_same_scores(pkg, seq, budget, n_sink, dist):
     from paper_2607_27600_gb300 import cc
     cap = max(seq)
     r = np.random.default_rng(len(seq))
-    s = r.integers(-20, 20, size=(len(seq), cap)).astype(np.float32) * 0.25   # many ties
+    if dist == "ties":
+        s = r.integers(-20, 20, size=(len(seq), cap)).astype(np.float32) * 0.25   # many ties
+    else:
+        s = r.standard_normal((len(seq), cap)).astype(np.float32)
     s[0, 3] = np.nan
     s[0, 10] = np.inf
     s[-1, 0] = -np.inf
