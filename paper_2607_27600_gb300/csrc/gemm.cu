@@ -27,8 +27,14 @@ constexpr int A_BYTES = BM * BK * 2;   // 16 KB
 constexpr int B_BYTES = BN * BK * 2;   // 32 KB: shared-memory stage of the widest B tile
 constexpr int kThreads = 192;
 constexpr int kMaxBatch = 1024;
+// fp32 epilogues stage each 32 x 32 accumulator chunk of a warp in shared
+// memory (rows padded to 36 floats: 16-byte aligned, conflict-free float4
+// accesses in both directions)
+constexpr int kStageLd = 36;
+constexpr int kStageBytes = 4 * 32 * kStageLd * 4;   // the four epilogue warps
+constexpr size_t kPrefixBytes = ((kMaxBatch + 1) * sizeof(int) + 15) & ~size_t(15);
 constexpr size_t kSmemBytes = 1024 /*align slack*/ + ST * (A_BYTES + B_BYTES) + 256 +
-                              (kMaxBatch + 1) * sizeof(int);
+                              kPrefixBytes + kStageBytes;
 
 // RoPE'd bf16 store of one accumulator tile row: destination columns
 // [col0, col0 + TBN) of out (row stride ldo, n_dest columns in all), each tile
@@ -170,124 +176,181 @@ CC_DEV long long cache_row(const GemmParams &p, int grow, bool valid) {
   return r;
 }
 
+// Chunk c of a warp's accumulator (32 rows x 32 columns, one row per lane as
+// tcgen05.ld delivers it) into the warp's staging tile; afterwards lane l
+// reads row 4 * i + l / 8 (i = 0..7), columns 4 * (l % 8) .. +4, so global
+// reads and writes run along rows (whole 128-byte lines per 8 lanes).
+CC_DEV void stage_chunk(float *stage, const uint32_t (&r)[32], int lane) {
+  float4 *srow = reinterpret_cast<float4 *>(stage + lane * kStageLd);
+#pragma unroll
+  for (int v = 0; v < 8; ++v)
+    srow[v] = make_float4(__uint_as_float(r[v * 4]), __uint_as_float(r[v * 4 + 1]),
+                          __uint_as_float(r[v * 4 + 2]), __uint_as_float(r[v * 4 + 3]));
+  __syncwarp();
+}
+
+// Sum over the 8 lanes that share a row in the staged layout.
+CC_DEV float row8_sum(float v) {
+  v += __shfl_xor_sync(0xFFFFFFFFu, v, 1);
+  v += __shfl_xor_sync(0xFFFFFFFFu, v, 2);
+  v += __shfl_xor_sync(0xFFFFFFFFu, v, 4);
+  return v;
+}
+
 // The final residual row x = out + acc of one tile (never stored): partial
 // sum of x^2 and partial dot of x * gain with the lm_head row of the slot's
 // own token, the two sums the logit score (Sec. 3.1) needs from this tile.
+// The warp's rows are consecutive and its valid rows a prefix of them.
 template <int TBN>
 CC_DEV void logit_partials(const GemmParams &p, uint32_t tacc, int grow, bool valid, int nt,
-                           int tile_n0) {
-  const float *src = reinterpret_cast<const float *>(p.out) + (size_t)grow * p.ldo;
+                           int tile_n0, float *stage) {
+  const int lane = threadIdx.x & 31, cq = (lane & 7) * 4;
+  const int nv = __popc(__ballot_sync(0xFFFFFFFFu, valid));
+  const int grow0 = __shfl_sync(0xFFFFFFFFu, grow, 0);
   int tok = valid ? p.tokens[grow] : 0;
   if (tok < 0 || tok >= p.vocab) tok = 0;   // reported by the combine
-  const __nv_bfloat16 *wrow = p.head_w + (size_t)tok * p.N;
-  float ss = 0.f, z = 0.f;
+  int tok_i[8];
+#pragma unroll
+  for (int i = 0; i < 8; ++i) tok_i[i] = __shfl_sync(0xFFFFFFFFu, tok, 4 * i + (lane >> 3));
+  float ss[8], z[8];
+#pragma unroll
+  for (int i = 0; i < 8; ++i) ss[i] = z[i] = 0.f;
 #pragma unroll 1
   for (int c = 0; c < TBN / 32; ++c) {
     uint32_t r[32];
     tmem_ld32(tacc + c * 32, r);
     tmem_ld_wait();
     const int col = tile_n0 + c * 32;
-    if (!valid || col >= p.N) continue;
-    const float4 *hs = reinterpret_cast<const float4 *>(src + col);
-    const uint4 *gs = reinterpret_cast<const uint4 *>(p.head_gain + col);
-    const uint4 *ws = reinterpret_cast<const uint4 *>(wrow + col);
+    if (col >= p.N) continue;   // warp-uniform
+    stage_chunk(stage, r, lane);
+    const uint2 g = *reinterpret_cast<const uint2 *>(p.head_gain + col + cq);
+    const float g4[4] = {bf16_lo(g.x), bf16_hi(g.x), bf16_lo(g.y), bf16_hi(g.y)};
+    float4 hv[8];
+    uint2 wv[8];
 #pragma unroll
-    for (int v = 0; v < 4; ++v) {   // 8 columns
-      const uint4 g = gs[v], w = ws[v];
-      const float4 h0 = hs[2 * v], h1 = hs[2 * v + 1];
-      const float hv[8] = {h0.x, h0.y, h0.z, h0.w, h1.x, h1.y, h1.z, h1.w};
-      const uint32_t gw[4] = {g.x, g.y, g.z, g.w}, ww[4] = {w.x, w.y, w.z, w.w};
+    for (int i = 0; i < 8; ++i) {   // every load first
+      const int rr = 4 * i + (lane >> 3);
+      hv[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+      wv[i] = make_uint2(0u, 0u);
+      if (rr >= nv) continue;
+      hv[i] = *reinterpret_cast<const float4 *>(
+          reinterpret_cast<const float *>(p.out) + (size_t)(grow0 + rr) * p.ldo + col + cq);
+      wv[i] = *reinterpret_cast<const uint2 *>(p.head_w + (size_t)tok_i[i] * p.N + col + cq);
+    }
 #pragma unroll
-      for (int k = 0; k < 8; ++k) {
-        const float x = __uint_as_float(r[v * 8 + k]) + hv[k];
-        const float gk = (k & 1) ? bf16_hi(gw[k / 2]) : bf16_lo(gw[k / 2]);
-        const float wk = (k & 1) ? bf16_hi(ww[k / 2]) : bf16_lo(ww[k / 2]);
-        ss = fmaf(x, x, ss);
-        z = fmaf(x * gk, wk, z);
+    for (int i = 0; i < 8; ++i) {
+      const int rr = 4 * i + (lane >> 3);
+      const float4 a = *reinterpret_cast<const float4 *>(stage + rr * kStageLd + cq);
+      const float x[4] = {a.x + hv[i].x, a.y + hv[i].y, a.z + hv[i].z, a.w + hv[i].w};
+      const float w4[4] = {bf16_lo(wv[i].x), bf16_hi(wv[i].x), bf16_lo(wv[i].y), bf16_hi(wv[i].y)};
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {   // rows past nv add zeros and are never written
+        ss[i] = fmaf(x[k], x[k], ss[i]);
+        z[i] = fmaf(x[k] * g4[k], w4[k], z[i]);
       }
     }
+    __syncwarp();   // the staging tile is rewritten by the next chunk
   }
-  if (valid) p.head_part[(size_t)grow * p.n_tiles + nt] = make_float2(ss, z);
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const float a = row8_sum(ss[i]), b = row8_sum(z[i]);
+    const int rr = 4 * i + (lane >> 3);
+    if ((lane & 7) == 0 && rr < nv)
+      p.head_part[(size_t)(grow0 + rr) * p.n_tiles + nt] = make_float2(a, b);
+  }
+}
+
+// fp32 outputs (EPI_F32, EPI_RESID_*), through the staging tile: out = acc
+// (+ bf16 resid, or += for RESID_F32); with norm_out (last K split) also
+// bf16(out * norm_gain) (and the lo part) and the tile's partial sum of out^2.
+template <int EPI, int TBN>
+CC_DEV void f32_epilogue(const GemmParams &p, uint32_t tacc, int grow, bool valid, int nt,
+                         int tile_n0, bool last, float *stage) {
+  const int lane = threadIdx.x & 31, cq = (lane & 7) * 4;
+  const int nv = __popc(__ballot_sync(0xFFFFFFFFu, valid));
+  const int grow0 = __shfl_sync(0xFFFFFFFFu, grow, 0);
+  const bool nrm = (EPI == EPI_RESID_BF16 || EPI == EPI_RESID_F32) && p.norm_out && last;
+  float ss[8];
+#pragma unroll
+  for (int i = 0; i < 8; ++i) ss[i] = 0.f;
+#pragma unroll 1
+  for (int c = 0; c < TBN / 32; ++c) {
+    uint32_t r[32];
+    tmem_ld32(tacc + c * 32, r);
+    tmem_ld_wait();
+    const int col = tile_n0 + c * 32;
+    if (col >= p.N) continue;   // warp-uniform
+    stage_chunk(stage, r, lane);
+    float g4[4] = {0.f, 0.f, 0.f, 0.f};
+    if (nrm) {
+      const uint2 g = *reinterpret_cast<const uint2 *>(p.norm_gain + col + cq);
+      g4[0] = bf16_lo(g.x); g4[1] = bf16_hi(g.x); g4[2] = bf16_lo(g.y); g4[3] = bf16_hi(g.y);
+    }
+    // all eight rows' loads first (the stores below could alias them, so the
+    // compiler would not hoist them), then the arithmetic and the stores
+    float4 a[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int rr = 4 * i + (lane >> 3);
+      a[i] = *reinterpret_cast<const float4 *>(stage + rr * kStageLd + cq);
+      if (rr >= nv) continue;
+      const size_t row = (size_t)(grow0 + rr);
+      if constexpr (EPI == EPI_RESID_BF16) {
+        const uint2 h = *reinterpret_cast<const uint2 *>(
+            reinterpret_cast<const __nv_bfloat16 *>(p.resid) + row * p.ld_resid + col + cq);
+        a[i].x += bf16_lo(h.x); a[i].y += bf16_hi(h.x); a[i].z += bf16_lo(h.y); a[i].w += bf16_hi(h.y);
+      } else if constexpr (EPI == EPI_RESID_F32 || EPI == EPI_RESID_LOGIT) {
+        const float4 h = *reinterpret_cast<const float4 *>(
+            reinterpret_cast<const float *>(p.out) + row * p.ldo + col + cq);
+        a[i].x += h.x; a[i].y += h.y; a[i].z += h.z; a[i].w += h.w;
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int rr = 4 * i + (lane >> 3);
+      if (rr >= nv) continue;
+      const size_t row = (size_t)(grow0 + rr);
+      *reinterpret_cast<float4 *>(reinterpret_cast<float *>(p.out) + row * p.ldo + col + cq) = a[i];
+      if (nrm) {
+        ss[i] = fmaf(a[i].x, a[i].x, ss[i]);
+        ss[i] = fmaf(a[i].y, a[i].y, ss[i]);
+        ss[i] = fmaf(a[i].z, a[i].z, ss[i]);
+        ss[i] = fmaf(a[i].w, a[i].w, ss[i]);
+        const float y0 = a[i].x * g4[0], y1 = a[i].y * g4[1], y2 = a[i].z * g4[2],
+                    y3 = a[i].w * g4[3];
+        const uint32_t h0 = pack_bf16x2(y0, y1), h1 = pack_bf16x2(y2, y3);
+        __nv_bfloat16 *dn = p.norm_out + row * p.ld_norm + col + cq;
+        *reinterpret_cast<uint2 *>(dn) = make_uint2(h0, h1);
+        if (p.norm_split)   // lo = y * gain - hi, at column offset N
+          *reinterpret_cast<uint2 *>(dn + p.N) =
+              make_uint2(pack_bf16x2(y0 - bf16_lo(h0), y1 - bf16_hi(h0)),
+                         pack_bf16x2(y2 - bf16_lo(h1), y3 - bf16_hi(h1)));
+      }
+    }
+    __syncwarp();   // the staging tile is rewritten by the next chunk
+  }
+  if (nrm) {
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const float v = row8_sum(ss[i]);
+      const int rr = 4 * i + (lane >> 3);
+      if ((lane & 7) == 0 && rr < nv) p.ss_part[(size_t)(grow0 + rr) * p.n_tiles + nt] = v;
+    }
+  }
 }
 
 template <int EPI, int TBN>
 CC_DEV void epilogue_tile(const GemmParams &p, uint32_t tacc, int grow, bool valid, int nt,
-                          int tile_n0, bool last) {
+                          int tile_n0, bool last, float *stage) {
   if constexpr (EPI == EPI_RESID_LOGIT) {
     if (last) {
-      logit_partials<TBN>(p, tacc, grow, valid, nt, tile_n0);
+      logit_partials<TBN>(p, tacc, grow, valid, nt, tile_n0, stage);
       return;
     }
   }
   if constexpr (EPI == EPI_F32 || EPI == EPI_RESID_BF16 || EPI == EPI_RESID_F32 ||
                 EPI == EPI_RESID_LOGIT) {
-    float *out = reinterpret_cast<float *>(p.out) + (size_t)grow * p.ldo;
-    const bool nrm = (EPI == EPI_RESID_BF16 || EPI == EPI_RESID_F32) && p.norm_out && last;
-    float ss = 0.f;
-#pragma unroll 1
-    for (int c = 0; c < TBN / 32; ++c) {
-      uint32_t r[32];
-      tmem_ld32(tacc + c * 32, r);
-      tmem_ld_wait();
-      int col = tile_n0 + c * 32;
-      if (!valid || col >= p.N) continue;
-      float y[32];
-#pragma unroll
-      for (int k = 0; k < 32; ++k) y[k] = __uint_as_float(r[k]);
-      float4 *dst = reinterpret_cast<float4 *>(out + col);
-      if constexpr (EPI == EPI_RESID_BF16) {
-        const uint4 *res = reinterpret_cast<const uint4 *>(
-            reinterpret_cast<const __nv_bfloat16 *>(p.resid) + (size_t)grow * p.ld_resid + col);
-#pragma unroll
-        for (int v = 0; v < 4; ++v) {
-          const uint4 h = res[v];
-          const uint32_t hw[4] = {h.x, h.y, h.z, h.w};
-#pragma unroll
-          for (int m = 0; m < 8; m += 2) {
-            y[v * 8 + m] += bf16_lo(hw[m / 2]);
-            y[v * 8 + m + 1] += bf16_hi(hw[m / 2]);
-          }
-        }
-      } else if constexpr (EPI == EPI_RESID_F32 || EPI == EPI_RESID_LOGIT) {
-#pragma unroll
-        for (int v = 0; v < 8; ++v) {
-          const float4 h = dst[v];
-          y[v * 4] += h.x; y[v * 4 + 1] += h.y; y[v * 4 + 2] += h.z; y[v * 4 + 3] += h.w;
-        }
-      }
-#pragma unroll
-      for (int v = 0; v < 8; ++v)
-        dst[v] = make_float4(y[v * 4], y[v * 4 + 1], y[v * 4 + 2], y[v * 4 + 3]);
-      if (nrm) {   // y * gain as bf16 (hi, and lo = y * gain - hi with norm_split)
-        const uint4 *gs = reinterpret_cast<const uint4 *>(p.norm_gain + col);
-        uint32_t o[16], lo[16];
-#pragma unroll
-        for (int v = 0; v < 4; ++v) {
-          const uint4 g = gs[v];
-          const uint32_t gw[4] = {g.x, g.y, g.z, g.w};
-#pragma unroll
-          for (int m = 0; m < 8; m += 2) {
-            const float a = y[v * 8 + m], b = y[v * 8 + m + 1];
-            ss = fmaf(a, a, ss);
-            ss = fmaf(b, b, ss);
-            const float ga = a * bf16_lo(gw[m / 2]), gb = b * bf16_hi(gw[m / 2]);
-            const uint32_t hi = pack_bf16x2(ga, gb);
-            o[(v * 8 + m) / 2] = hi;
-            lo[(v * 8 + m) / 2] = pack_bf16x2(ga - bf16_lo(hi), gb - bf16_hi(hi));
-          }
-        }
-        uint4 *dn = reinterpret_cast<uint4 *>(p.norm_out + (size_t)grow * p.ld_norm + col);
-#pragma unroll
-        for (int v = 0; v < 4; ++v) dn[v] = make_uint4(o[v * 4], o[v * 4 + 1], o[v * 4 + 2], o[v * 4 + 3]);
-        if (p.norm_split) {
-          uint4 *dl = reinterpret_cast<uint4 *>(p.norm_out + (size_t)grow * p.ld_norm + p.N + col);
-#pragma unroll
-          for (int v = 0; v < 4; ++v)
-            dl[v] = make_uint4(lo[v * 4], lo[v * 4 + 1], lo[v * 4 + 2], lo[v * 4 + 3]);
-        }
-      }
-    }
-    if (nrm && valid) p.ss_part[(size_t)grow * p.n_tiles + nt] = ss;
+    f32_epilogue<EPI, TBN>(p, tacc, grow, valid, nt, tile_n0, last, stage);
   } else if constexpr (EPI == EPI_QROPE) {   // kv_fp8: the K rows of an e4m3 cache
     const long long orow = p.kv_dest ? cache_row(p, grow, valid) : grow;
     const bool hm = p.kv_dest && p.pg.head_major;
@@ -460,6 +523,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(tempty + 2);
   volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
   int *prefix = reinterpret_cast<int *>(smem + ST * (A_BYTES + B_BYTES) + 256);
+  float *stage_all = reinterpret_cast<float *>(smem + ST * (A_BYTES + B_BYTES) + 256 + kPrefixBytes);
   __shared__ int split_ok;   // K splits: the previous split of the tile has published
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -592,7 +656,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         named_barrier_sync(1, 128);
         add = split_ok != 0;   // a wait that gave up (status set) skips this split's add
       }
-      if (add) epilogue_tile<EPI, TBN>(p, tacc, grow, valid, nt, nt * TBN, split == S - 1);
+      if (add)
+        epilogue_tile<EPI, TBN>(p, tacc, grow, valid, nt, nt * TBN, split == S - 1,
+                                stage_all + q * 32 * kStageLd);
       tc_fence_before();
       if (S > 1) {
         named_barrier_sync(1, 128);
