@@ -181,3 +181,54 @@ def test_rope_shift_invariance(model):
     s2 = oracle.score_layer(SMALL, model, built(7))
     np.testing.assert_allclose(s2[0, :n - 1], oracle.score_layer(SMALL, model, built(0))[0, :n - 1],
                                rtol=1e-9)
+
+
+def test_worked_example_by_hand():
+    """A three-slot cache small enough to score with a pencil (Sec. 3.1, the
+    surprise of each cached token given only its future; Algorithm
+    DoMemRefresh, keep the J highest and compact).  One layer, d = 2, one
+    head, eps = 0.  W_q = 0 makes every attention score 0, so slot i averages
+    the values of slots i+1 .. n-1; W_o = I adds that average to h_i; W_down = 0
+    silences the MLP; gains are 1; W_U rows are e_0, e_1 and e_0 + e_1.
+
+      slot  token  h_i       v_i        o_i            h_i + o_i   RMSNorm
+      0     0      (1, 1)    (5, 5)     (v1+v2)/2=(0,2)   (1, 3)     (1, 3)/sqrt(5)
+      1     1      (1, -1)   (1, 1)     v2 = (-1, 3)      (0, 2)     (0, sqrt(2))
+      2     2      (2, 0)    (-1, 3)    no future: +inf
+      3     (stale slot past n = 3: -inf, never read)
+
+    logit scores: -W_U[x_i] . RMSNorm = -1/sqrt(5), -sqrt(2), +inf.
+    log-prob scores: logsumexp(z_i) - z_i[x_i] with z_0 = (1, 3, 4)/sqrt(5),
+    z_1 = (0, sqrt(2), sqrt(2)).  Budget J = 2 keeps slots 0 and 2 in both
+    modes; compaction moves slot 2 to slot 1."""
+    import math
+    from synth.configs import ModelShape
+    shape = ModelShape(n_layers=1, d_model=2, n_q_heads=1, n_kv_heads=1, head_dim=2, d_ff=2,
+                       vocab=3, rope_theta=1e4, rms_eps=0.0)
+    eye, zero, ones = np.eye(2), np.zeros((2, 2)), np.ones(2)
+    h = np.array([[1.0, 1.0], [1.0, -1.0], [2.0, 0.0], [7.0, 7.0]])
+    lw = {"attn_norm": ones, "wq": zero, "wk": eye, "wv": eye, "wo": eye, "mlp_norm": ones,
+          "w_gate": eye, "w_up": eye, "w_down": zero}
+    w = {"layers": [lw], "final_norm": ones, "lm_head": np.array([[1.0, 0], [0, 1.0], [1.0, 1.0]]),
+         "embed": np.array([[1.0, 1.0], [1.0, -1.0], [2.0, 0.0]])}
+    v = np.array([[5.0, 5.0], [1.0, 1.0], [-1.0, 3.0], [100.0, -100.0]])[None, :, None, :]
+    k = np.arange(8.0).reshape(1, 4, 1, 2)
+    cache = {"k": [k], "v": [v], "tokens": np.array([[0, 1, 2, 0]]),
+             "pos": np.array([[0, 1, 2, 3]]), "seq_len": np.array([3]), "h_last": h[None]}
+
+    def lse(*z):
+        return math.log(sum(math.exp(t) for t in z))
+
+    s5, s2 = math.sqrt(5.0), math.sqrt(2.0)
+    want = {"logit": [-1 / s5, -s2],
+            "logprob": [lse(1 / s5, 3 / s5, 4 / s5) - 1 / s5, lse(0.0, s2, s2) - s2]}
+    for mode, (w0, w1) in want.items():
+        for got in (oracle.score_layer(shape, w, cache, mode),
+                    oracle.score_full(shape, w, cache, mode)):   # embed rows = h: same pass
+            np.testing.assert_allclose(got[0, :2], [w0, w1], rtol=1e-14, atol=1e-14)
+            assert got[0, 2] == np.inf and got[0, 3] == -np.inf
+            idx, cnt = oracle.select_keep(got.astype(np.float32), [3], [2])
+            assert cnt.tolist() == [2] and idx[0, :2].tolist() == [0, 2]
+    np.testing.assert_array_equal(oracle.compact(cache["tokens"], idx, cnt)[0, :2], [0, 2])
+    np.testing.assert_array_equal(oracle.compact(v, idx, cnt)[0, :2, 0], v[0, [0, 2], 0])
+    np.testing.assert_array_equal(oracle.compact(h[None], idx, cnt)[0, :2], h[[0, 2]])
