@@ -232,3 +232,23 @@ def test_worked_example_by_hand():
     np.testing.assert_array_equal(oracle.compact(cache["tokens"], idx, cnt)[0, :2], [0, 2])
     np.testing.assert_array_equal(oracle.compact(v, idx, cnt)[0, :2, 0], v[0, [0, 2], 0])
     np.testing.assert_array_equal(oracle.compact(h[None], idx, cnt)[0, :2], h[[0, 2]])
+
+
+def test_logprob_scores_are_a_distribution_over_the_target_token(model, cache):
+    """In the fast pass a slot's hidden state comes from H^(L-1) and its own
+    K/V are never attended (only later slots are), so its token id enters the
+    score only as the target: re-scoring one slot with every vocabulary entry
+    as its token must give probabilities exp(-score) that sum to 1 (the
+    surprise is -log P(x_i | its future), Sec. 3.1), and logit-mode scores
+    differ from them by one constant per slot."""
+    b, n = 0, SEQ[0]
+    for i in (0, 4, n - 2):
+        lp, lg = [], []
+        for v in range(SMALL.vocab):
+            c = copy.deepcopy(cache)
+            c["tokens"][b, i] = v
+            lp.append(oracle.score_layer(SMALL, model, c, "logprob", rows=[[i], None, None])[b, i])
+            lg.append(oracle.score_layer(SMALL, model, c, "logit", rows=[[i], None, None])[b, i])
+        lp, lg = np.array(lp), np.array(lg)
+        assert abs(np.exp(-lp).sum() - 1.0) < 1e-12
+        np.testing.assert_allclose(lp - lg, np.full(SMALL.vocab, (lp - lg)[0]), rtol=0, atol=1e-12)
