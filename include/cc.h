@@ -183,8 +183,8 @@ typedef struct {
    * its first kernel that reads or writes layer l's K/V (the scoring pass before layer
    * l's attention, the append and decode at the start of layer l, the comparison scorers
    * and the compaction before their launch), so an upload of the cache overlaps the
-   * kernels that do not need it.  Events recorded outside a graph capture cannot be
-   * waited on inside one (CC_ERR_CUDA). */
+   * kernels that do not need it.  Leave kv_ready NULL for calls recorded into a graph
+   * (cc_graph_begin): the waits are for eager calls whose inputs are still arriving. */
   void *const *kv_ready;
 } cc_kv_cache;
 
