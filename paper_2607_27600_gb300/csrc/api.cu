@@ -1578,28 +1578,22 @@ cudaError_t wait_kv_ready(const cc_kv_cache *kv, int l0, int l1, cudaStream_t st
 }
 
 
-cc_status compact_plan_build(const cc_model_cfg *cfg, const cc_kv_cache *cache, CompactParams &p,
-                             size_t &scratch_bytes) {
-  static CompactPlan plan;
-  static std::mutex mu;
-  std::lock_guard<std::mutex> lk(mu);
-  cc_status s = compact_plan(cfg, cache, plan);
-  if (s != CC_OK) return s;
-  p = plan.p;
-  scratch_bytes = plan.ws_bytes;
-  return CC_OK;
-}
-
 cc_status compact_plan_bind(const cc_model_cfg *cfg, const cc_kv_cache *cache, CompactParams &p,
-                            void *scratch, cudaStream_t st) {
+                            void *scratch, size_t scratch_cap, cudaStream_t st) {
   static CompactPlan plan;
   static std::mutex mu;
   std::lock_guard<std::mutex> lk(mu);
   cc_status s = compact_plan(cfg, cache, plan);
   if (s != CC_OK) return s;
+  if (plan.ws_bytes > scratch_cap) return CC_ERR_WORKSPACE;
   if ((s = compact_bind(plan, scratch, st)) != CC_OK) return s;
   p = plan.p;
   return CC_OK;
+}
+
+cudaError_t launch_compact_timed(const CompactParams &p, int sms, cudaStream_t st) {
+  TimedScope t(CC_KERNEL_COMPACT, st);
+  return launch_compact(p, sms, st);
 }
 
 bool current_device_info(unsigned **status, int *sms) {

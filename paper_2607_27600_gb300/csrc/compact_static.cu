@@ -47,25 +47,25 @@ extern "C" cc_status cc_compact_kv_static(const cc_model_cfg *cfg, const cc_kv_c
   static cc::CompactParams p;   // large kernel-parameter block; guarded by mu
   static std::mutex mu;
   std::lock_guard<std::mutex> lk(mu);
-  size_t need = 0;
-  cc_status s = cc::compact_plan_build(cfg, cache, p, need);
-  if (s != CC_OK) return s;
+  if (!cfg || !cache) return CC_ERR_INVALID_ARG;
   if (!keep_idx || !keep_count) return CC_ERR_INVALID_ARG;
-  if (need > kStaticScratchBytes) return CC_ERR_WORKSPACE;   // cache too large for the array
   unsigned char *scratch = nullptr;
-  if ((s = scratch_address(&scratch)) != CC_OK) return s;
+  cc_status s = scratch_address(&scratch);
+  if (s != CC_OK) return s;
   unsigned *status = nullptr;
   int sms = 0;
   if (!cc::current_device_info(&status, &sms)) return CC_ERR_CUDA;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-  // the flags start at zero and the readers table at -1 (cleared on `st`);
-  // the array keeps the last call's contents
-  if ((s = cc::compact_plan_bind(cfg, cache, p, scratch, st)) != CC_OK) return s;
+  // one plan build: rejected (CC_ERR_WORKSPACE, nothing enqueued) when its
+  // scratch exceeds the array; else the flags start at zero and the readers
+  // table at -1 (cleared on `st`), since the array keeps the last call's contents
+  if ((s = cc::compact_plan_bind(cfg, cache, p, scratch, kStaticScratchBytes, st)) != CC_OK)
+    return s;
   p.keep_idx = keep_idx;
   p.keep_count = keep_count;
   p.seq_len = cache->seq_len;
   p.status = status;
   if (cc::wait_kv_ready(cache, 0, cfg->n_layers, st) != cudaSuccess) return CC_ERR_CUDA;
-  if (cc::launch_compact(p, sms, st) != cudaSuccess) return CC_ERR_CUDA;
+  if (cc::launch_compact_timed(p, sms, st) != cudaSuccess) return CC_ERR_CUDA;
   return CC_OK;
 }

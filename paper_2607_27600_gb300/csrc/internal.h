@@ -5,14 +5,15 @@
 
 namespace cc {
 
-// Builds the compaction plan of `cache` (arrays, work units) and the scratch
-// bytes it needs; same checks as cc_compact_kv.
-cc_status compact_plan_build(const cc_model_cfg *cfg, const cc_kv_cache *cache, CompactParams &p,
-                             size_t &scratch_bytes);
-// Builds the plan with its scratch at `scratch` and enqueues on `st` the
-// clearing of what must start cleared.
+// Builds the compaction plan of `cache` (arrays, work units; the same checks
+// as cc_compact_kv) once, rejects it with CC_ERR_WORKSPACE when its scratch
+// exceeds `scratch_cap` bytes, else places the scratch at `scratch` and
+// enqueues on `st` the clearing of what must start cleared.
 cc_status compact_plan_bind(const cc_model_cfg *cfg, const cc_kv_cache *cache, CompactParams &p,
-                            void *scratch, cudaStream_t st);
+                            void *scratch, size_t scratch_cap, cudaStream_t st);
+// launch_compact inside the same launch-timing scope as cc_compact_kv's
+// (cc_profile.h, kind CC_KERNEL_COMPACT).
+cudaError_t launch_compact_timed(const CompactParams &p, int sms, cudaStream_t st);
 // Status-word address and SM count of the current device.
 bool current_device_info(unsigned **status, int *sms);
 // Makes `st` wait for the caller's K/V-ready events (cc_kv_cache.kv_ready) of

@@ -22,9 +22,13 @@ constexpr uint32_t kKeyPosInf = 0xFF800000u;   // monotone key of +inf
 constexpr uint32_t kKeyNegInf = 0x007FFFFFu;   // monotone key of -inf
 
 // float -> uint32 whose unsigned order is the float order; NaN ranks as -inf.
+// -0.0 and +0.0 compare equal as floats, so both take the key of +0.0 (a
+// score -logit is -0.0 for a logit of exactly zero); their tie then goes to
+// the later slot like any other.
 CC_DEV uint32_t monotone_key(float f) {
   uint32_t u = __float_as_uint(f);
   if ((u & 0x7F800000u) == 0x7F800000u && (u & 0x007FFFFFu)) return kKeyNegInf;
+  if ((u & 0x7FFFFFFFu) == 0u) u = 0u;
   return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
 }
 

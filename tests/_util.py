@@ -88,13 +88,16 @@ def to_device(x, device="cuda"):
     return t.to(device)
 
 
-def keep_set_ok(got_idx, got_cnt, want_idx, want_cnt, oracle_scores, seq_lens, budgets, tol=2e-2):
-    """Keep-set criterion (the keep-set is the top-J slots by score): identical
-    where the oracle's score gap at the budget boundary exceeds `tol` (relative
-    to the scores' rms); otherwise every slot kept by one side only is a near
-    tie: its oracle score lies within `tol` x rms of the oracle's J-th score,
-    where rounding of scores within the bar may order them either way.
-    Returns (ok, details)."""
+def keep_set_ok(got_idx, got_cnt, want_idx, want_cnt, oracle_scores, seq_lens, budgets, tol=2e-2,
+                min_overlap=0.995):
+    """Keep-set bar (the keep-set is the top-J slots by score): identical
+    where the oracle's score gap at the budget boundary exceeds `tol`
+    (relative to the scores' rms); otherwise at least `min_overlap` of the
+    oracle's kept slots kept (99.5 %: at J < 200 that allows no swap at all),
+    and every slot kept by one side only a near tie -- its oracle score within
+    `tol` x rms of the oracle's J-th score, where rounding of scores within the
+    bar may order them either way.  Returns (ok, details): per sequence
+    (b, gap, overlap, slots kept by one side only)."""
     details = []
     ok = True
     for b, (n, j) in enumerate(zip(seq_lens, budgets)):
@@ -114,6 +117,7 @@ def keep_set_ok(got_idx, got_cnt, want_idx, want_cnt, oracle_scores, seq_lens, b
             ok &= g == w
         else:
             thr = srt[jj - 1]
+            ok &= overlap >= min_overlap
             ok &= all(np.isfinite(s[i]) and abs(s[i] - thr) <= tol * rms for i in diff)
         details.append((b, gap, overlap, len(diff)))
     return bool(ok), details

@@ -1,32 +1,38 @@
 """How far does bf16 arithmetic move the exact counter-causal score of a deep
-random model?  -- TEST INFRASTRUCTURE (a study script over the oracle).
+random model?  A study over the oracle (test infrastructure, not collected by
+pytest: the file name does not start with test_).
 
 The oracle computes the full counter-causal pass (Sec. 3.1) in fp64.  A GPU
-pass must round some intermediates to bf16 to use the tensor cores.  This
-script re-runs the oracle's layer with bf16 rounding inserted at chosen
-points and reports, per layer, the score's max relative error against the
-exact fp64 pass (the parity metric: |g - o| / max(|o|, rms(o))):
+pass rounds some intermediates to use the bf16 tensor cores.  This script
+re-runs the oracle's layer with rounding inserted at chosen points and
+reports, per layer, the score's max relative error against the exact fp64
+pass (the parity metric: |g - o| / max(|o|, rms(o))).  A "split" operand is
+carried as the bf16 pair hi = bf16(x), lo = bf16(x - hi) (hi + lo is x to
+about 2^-17 relative; a tensor-core product then runs once per half):
 
-  queries      only the queries entering QK^T are rounded (every other step exact)
-  activations  every GEMM input (normalised inputs, attention output,
-               SwiGLU output) and the queries are rounded
+  queries      only the queries entering Q K^T rounded (every other step exact)
+  activations  every GEMM input (normalised inputs, attention output, SwiGLU
+               output) and the queries rounded
   bf16-pass    as `activations`, plus the attention probabilities P rounded
-               before P V and the residual stream kept in fp32: every rounding
-               point of a bf16 tensor-core pass
+               before P V and the residual stream kept in fp32: every
+               rounding point of a bf16 tensor-core pass
+  split-act    GEMM inputs split; queries and P single bf16; fp32 residual
+  split-q      GEMM inputs and queries split; P single bf16; fp32 residual
+  split-all    GEMM inputs, queries and P split; fp32 residual
 
 The drift measured here is a property of the arithmetic and of the random
-model, not of any kernel; the 32-layer full-pass tolerances of the parity
-tests are derived from it.  It imports only the oracle and the seeded input
+model, not of any kernel; the full-pass tolerances of the parity tests are
+derived from it.  It imports only the oracle and the seeded input
 generators, never the CUDA path.
 
-    python -m oracle.sensitivity --layers 32 --n 16384 --rows 4
+    python -m tests.study_fullpass_precision --layers 32 --n 16384 --rows 96
 """
 import argparse
 import sys
 
 import numpy as np
 
-from . import refresh as R
+from oracle import refresh as R
 
 
 def bf16(x):
@@ -37,9 +43,21 @@ def bf16(x):
     return u.astype(np.uint32).view(np.float32).astype(np.float64)
 
 
-def attention_rounded_p(q, k, v, rows, n):
-    """Counter-causal attention with the probabilities rounded to bf16 before
-    P V (the row sum taken from the unrounded values)."""
+def split(x):
+    """x carried as the bf16 pair (hi, lo): the value hi + lo, computed from
+    the fp32 rounding of x as a GPU epilogue would."""
+    x32 = np.asarray(x, np.float64).astype(np.float32).astype(np.float64)
+    hi = bf16(x32)
+    return hi + bf16(x32 - hi)
+
+
+def exact(x):
+    return x
+
+
+def attention_rounded_p(q, k, v, rows, n, rp):
+    """Counter-causal attention with the probabilities passed through `rp`
+    before P V (the row sum taken from the unrounded values)."""
     out = np.zeros(q.shape)
     group = q.shape[1] // k.shape[1]
     for r, i in enumerate(rows):
@@ -49,21 +67,35 @@ def attention_rounded_p(q, k, v, rows, n):
             hs = slice(g * group, (g + 1) * group)
             s = q[r, hs] @ R.f64(k[i + 1:n, g]).T / np.sqrt(q.shape[-1])
             p = np.exp(s - s.max(axis=1, keepdims=True))
-            out[r, hs] = (bf16(p) @ R.f64(v[i + 1:n, g])) / p.sum(axis=1, keepdims=True)
+            out[r, hs] = (rp(p) @ R.f64(v[i + 1:n, g])) / p.sum(axis=1, keepdims=True)
     return out
 
 
-def layer(h, rows, pos, lw, k, v, n, shape, round_q, round_act, round_p=False):
-    rq = bf16 if round_q else (lambda x: x)
-    ra = bf16 if round_act else (lambda x: x)
-    rh = (lambda x: x.astype(np.float32).astype(np.float64)) if round_p else (lambda x: x)
+def fp32(x):
+    return x.astype(np.float32).astype(np.float64)
+
+
+# name -> (query rounding, GEMM-input rounding, P rounding, residual rounding)
+VARIANTS = {
+    "exact": (exact, exact, exact, exact),
+    "queries": (bf16, exact, exact, exact),
+    "activations": (bf16, bf16, exact, exact),
+    "bf16-pass": (bf16, bf16, bf16, fp32),
+    "split-act": (bf16, split, bf16, fp32),
+    "split-q": (split, split, bf16, fp32),
+    "split-all": (split, split, split, fp32),
+}
+
+
+def layer(h, rows, pos, lw, k, v, n, shape, rounding):
+    rq, ra, rp, rh = rounding
     a = ra(R.rms_norm(h, lw["attn_norm"], shape.rms_eps))
     q = (a @ R.f64(lw["wq"]).T).reshape(len(rows), shape.n_q_heads, shape.head_dim)
     q = rq(R.rope(q, pos, shape.rope_theta))
-    if round_p:
-        o = ra(attention_rounded_p(q, k, v, rows, n))
-    else:
+    if rp is exact:
         o = ra(R.counter_causal_attention(q, k, v, rows, n))
+    else:
+        o = ra(attention_rounded_p(q, k, v, rows, n, rp))
     h = rh(h + o.reshape(len(rows), -1) @ R.f64(lw["wo"]).T)
     m = ra(R.rms_norm(h, lw["mlp_norm"], shape.rms_eps))
     act = ra(R.silu(m @ R.f64(lw["w_gate"]).T) * (m @ R.f64(lw["w_up"]).T))
@@ -76,6 +108,7 @@ def main(argv=None):
     ap.add_argument("--n", type=int, default=16384)
     ap.add_argument("--rows", type=int, default=4)
     ap.add_argument("--seed", type=int, default=3)
+    ap.add_argument("--variants", type=str, default=",".join(v for v in VARIANTS if v != "exact"))
     ap.add_argument("--row-list", type=str, default="",
                     help="comma-separated slots to follow (default: --rows evenly spaced)")
     args = ap.parse_args(argv)
@@ -83,17 +116,16 @@ def main(argv=None):
     from synth.configs import LLAMA3_8B
     shape = LLAMA3_8B
     n, seed = args.n, args.seed
+    names = [v for v in args.variants.split(",") if v]
     rows = (np.array([int(x) for x in args.row_list.split(",")]) if args.row_list
             else np.unique(np.linspace(0, n - 3, args.rows).astype(np.int64)))
     toks = synth.tokens((n,), shape.vocab, seed, "study.tokens").numpy()
     emb = synth.normal((shape.vocab, shape.d_model), 0.02, seed, "embed").float().numpy()
     lm = synth.normal((shape.vocab, shape.d_model), 0.02, seed, "lm_head").float().numpy()
     pos = np.arange(n)[rows]
-    variants = {"exact": (False, False, False), "queries": (True, False, False),
-                "activations": (True, True, False), "bf16-pass": (True, True, True)}
-    hs = {v: R.f64(emb[toks[rows]]) for v in variants}
+    hs = {v: R.f64(emb[toks[rows]]) for v in ["exact"] + names}
     ones = np.ones(shape.d_model)
-    print("layer  queries  activations  bf16-pass", flush=True)
+    print("layer  " + "  ".join(f"{v:>11s}" for v in names), flush=True)
     for l in range(args.layers):
         lw = {name: synth.normal(shp, 0.02, seed, f"l{l}.{name}").float().numpy() for name, shp in
               (("wq", (shape.q_dim, shape.d_model)), ("wo", (shape.d_model, shape.q_dim)),
@@ -103,22 +135,21 @@ def main(argv=None):
         std = synth.kv_std(shape)
         k = synth.normal((n, shape.n_kv_heads, shape.head_dim), std, seed, f"study.k{l}").float().numpy()
         v = synth.normal((n, shape.n_kv_heads, shape.head_dim), std, seed, f"study.v{l}").float().numpy()
-        for name, (rq, ra, rp) in variants.items():
-            hs[name] = layer(hs[name], rows, pos, lw, k, v, n, shape, rq, ra, rp)
+        for name in hs:
+            hs[name] = layer(hs[name], rows, pos, lw, k, v, n, shape, VARIANTS[name])
         sc = {name: R.score_head(hs[name], toks[rows], ones, lm, "logit", shape.rms_eps)
-              for name in variants}
+              for name in hs}
         ref = sc["exact"]
         rms = np.sqrt(np.mean(ref * ref))
         err = {name: float(np.max(np.abs(sc[name] - ref) / np.maximum(np.abs(ref), rms)))
-               for name in ("queries", "activations", "bf16-pass")}
-        print(f"{l:5d}  {err['queries']:.4f}   {err['activations']:.4f}       {err['bf16-pass']:.4f}",
-              flush=True)
+               for name in names}
+        print(f"{l:5d}  " + "  ".join(f"{err[v]:11.5f}" for v in names), flush=True)
     # per-row errors after the last layer: the tail of the drift's distribution
     print("after the last layer, per-row error quantiles (50 / 90 / 99 / max):")
-    for name in ("queries", "activations", "bf16-pass"):
+    for name in names:
         e = np.abs(sc[name] - ref) / np.maximum(np.abs(ref), rms)
         q = np.quantile(e, [0.5, 0.9, 0.99, 1.0])
-        print(f"  {name:12s} " + "  ".join(f"{x:.4f}" for x in q), flush=True)
+        print(f"  {name:12s} " + "  ".join(f"{x:.5f}" for x in q), flush=True)
     return 0
 
 

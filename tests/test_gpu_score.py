@@ -122,13 +122,22 @@ def test_tiny_refresh_keep_set_and_compaction(pkg, tiny):
     ([4096, 5000], [1000, 17], 0, "ties"),
     # continuous scores: the radix select settles after a few passes
     ([32768, 8192, 131072, 9], [8192, 8191, 1000, 2], 1, "normal"),
-    ([8192], [2048], 0, "normal")])
+    ([8192], [2048], 0, "normal"),
+    # +0.0 and -0.0 interleaved at the boundary (equal as floats: the later slot wins)
+    ([512, 300, 64], [128, 150, 1], 0, "signed_zeros"), ([4096], [2048], 3, "signed_zeros")])
 def test_select_exact_vs_oracle_on_same_scores(pkg, seq, budget, n_sink, dist):
     from paper_2607_27600_gb300 import cc
     cap = max(seq)
     r = np.random.default_rng(len(seq))
     if dist == "ties":
         s = r.integers(-20, 20, size=(len(seq), cap)).astype(np.float32) * 0.25   # many ties
+    elif dist == "signed_zeros":
+        # half the slots zero of either sign, the rest +-1: the budget boundary
+        # falls among the zeros
+        s = np.where(r.random((len(seq), cap)) < 0.5, 0.0,
+                     np.sign(r.standard_normal((len(seq), cap)))).astype(np.float32)
+        s = np.where((s == 0) & (r.random((len(seq), cap)) < 0.5), np.float32(-0.0), s)
+        s[:, 1] = -0.0   # a NaN next to a -0.0 too
     else:
         s = r.standard_normal((len(seq), cap)).astype(np.float32)
     s[0, 3] = np.nan

@@ -173,7 +173,7 @@ def test_score_head_logprob_matches_scipy():
 
 
 def test_sensitivity_bf16_rounding_matches_torch():
-    from oracle.sensitivity import bf16
+    from tests.study_fullpass_precision import bf16
     r = rng(21)
     x = np.concatenate([r.normal(size=1000) * 10.0 ** r.integers(-6, 6, size=1000),
                         [1.0 + 2.0 ** -8, 1.0 + 3 * 2.0 ** -8, -(1.0 + 2.0 ** -8), 0.0, -0.0]])

@@ -54,6 +54,24 @@ def test_select_ties_prefer_later_slot_and_keep_sinks():
     assert idx[0, :3].tolist() == [0, 1, 7]
 
 
+def test_select_signed_zeros_tie_to_the_later_slot():
+    # -0.0 == +0.0 as floats: a score -logit of an exactly-zero logit is -0.0
+    # and ties with +0.0; the later slot wins whatever the signs
+    s = np.array([[0.0, -0.0, -1.0]], np.float32)
+    idx, cnt = oracle.select_keep(s, [3], [1])
+    assert idx[0, :1].tolist() == [1]
+    s = np.array([[-0.0, 0.0, -1.0]], np.float32)
+    idx, cnt = oracle.select_keep(s, [3], [1])
+    assert idx[0, :1].tolist() == [1]
+    r = np.random.default_rng(5)
+    for _ in range(20):
+        s = np.where(r.random(50) < 0.5, np.float32(-0.0), np.float32(0.0)).astype(np.float32)
+        s[r.integers(0, 50, 5)] = r.choice([np.nan, 1.0, -1.0], 5)
+        budget = int(r.integers(1, 50))
+        idx, cnt = oracle.select_keep(s[None], [50], [budget])
+        assert idx[0, :cnt[0]].tolist() == brute_keep(s, 50, budget, 0)
+
+
 def test_select_keeps_highest_exactly():
     s = np.array([[0.5, 3.0, -1.0, 2.0, 2.5, -7.0]], np.float32)
     idx, cnt = oracle.select_keep(s, [6], [3])
@@ -110,24 +128,36 @@ def test_compact_preserves_relative_order():
 
 
 def test_keep_set_bar_accepts_only_near_tie_swaps():
-    """The GPU tests' keep-set bar: a swap at a near-tied boundary passes, a
-    swap of a slot far from the boundary fails, a count mismatch fails."""
+    """The GPU tests' keep-set bar: swaps at a near-tied boundary pass while
+    the overlap stays >= 99.5 %, a third swap (overlap 99.25 % at J = 400)
+    fails, a swap of a slot far from the boundary fails, a count mismatch
+    fails, and at J < 200 a single near-tie swap already fails."""
     from tests._util import keep_set_ok
-    n, j = 64, 16
+    n, j = 1000, 400
     s = np.linspace(10.0, -10.0, n)
-    s[j] = s[j - 1] - 1e-4                     # near tie at the boundary
+    s[j - 3:j + 3] = s[j - 1] - 1e-4 * np.arange(6)   # six near-tied slots at the boundary
     want_i, want_c = oracle.select_keep(s[None].astype(np.float32), [n], [j])
     kept = list(want_i[0, :j])
-    near = sorted(set(kept) - {j - 1} | {j})   # swap the tied pair
+
+    def swap(k):   # drop the k lowest kept, take the k highest dropped
+        return sorted(set(kept) - set(range(j - k, j)) | set(range(j, j + k)))
     far = sorted(set(kept) - {0} | {n - 1})    # drop the best, keep the worst
-    for got, expect in ((kept, True), (near, True), (far, False)):
+    for got, expect in ((kept, True), (swap(1), True), (swap(2), True), (swap(3), False),
+                        (far, False)):
         gi = np.full((1, n), -1, np.int32)
         gi[0, :j] = got
-        ok, _ = keep_set_ok(gi, np.array([j]), want_i, want_c, s[None], [n], [j])
-        assert ok == expect
-    s2 = np.linspace(10.0, -10.0, n)           # clear gap: only the exact set passes
-    w2_i, w2_c = oracle.select_keep(s2[None].astype(np.float32), [n], [j])
-    gi = np.full((1, n), -1, np.int32)
-    gi[0, :j] = sorted(set(w2_i[0, :j]) - {j - 1} | {j})
-    assert not keep_set_ok(gi, np.array([j]), w2_i, w2_c, s2[None], [n], [j])[0]
-    assert not keep_set_ok(w2_i, np.array([j - 1]), w2_i, w2_c, s2[None], [n], [j])[0]
+        ok, det = keep_set_ok(gi, np.array([j]), want_i, want_c, s[None], [n], [j])
+        assert ok == expect, det
+    small = 16                                 # J < 200: 99.5 % means identical
+    s1 = np.linspace(10.0, -10.0, 64)
+    s1[small] = s1[small - 1] - 1e-4
+    w1_i, w1_c = oracle.select_keep(s1[None].astype(np.float32), [64], [small])
+    gi = np.full((1, 64), -1, np.int32)
+    gi[0, :small] = sorted(set(w1_i[0, :small]) - {small - 1} | {small})
+    assert not keep_set_ok(gi, np.array([small]), w1_i, w1_c, s1[None], [64], [small])[0]
+    s2 = np.linspace(10.0, -10.0, 64)          # clear gap: only the exact set passes
+    w2_i, w2_c = oracle.select_keep(s2[None].astype(np.float32), [64], [small])
+    gi = np.full((1, 64), -1, np.int32)
+    gi[0, :small] = sorted(set(w2_i[0, :small]) - {small - 1} | {small})
+    assert not keep_set_ok(gi, np.array([small]), w2_i, w2_c, s2[None], [64], [small])[0]
+    assert not keep_set_ok(w2_i, np.array([small - 1]), w2_i, w2_c, s2[None], [64], [small])[0]

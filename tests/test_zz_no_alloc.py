@@ -60,7 +60,9 @@ def test_static_scratch_rejects_caches_beyond_its_size():
     from paper_2607_27600_gb300 import cc
     big = ModelShape(n_layers=64, d_model=256, n_q_heads=8, n_kv_heads=2, head_dim=64, d_ff=384,
                      vocab=1000, rope_theta=1e4, rms_eps=1e-5)
-    cap = 1 << 19          # 128 K/V arrays x 2048 units + tokens/pos: > 262080 unit flags
+    # 128 K/V arrays of 256-byte rows move in 4 KB units of 16 slots: 2^19 / 16 = 32768
+    # units per array, so about 4.2 M four-byte unit flags (16 MiB) > the 1 MiB array
+    cap = 1 << 19
     tiny = torch.zeros(16, dtype=torch.bfloat16, device="cuda")   # pointers are not dereferenced
     c = {"k": [tiny] * 64, "v": [tiny] * 64, "h_last": None,
          "tokens": torch.zeros(1, 1, dtype=torch.int32, device="cuda"),
