@@ -300,20 +300,75 @@ def step_flops(wl):
 # our arm
 # ---------------------------------------------------------------------------
 
-def run_ours(args, dist):
+def causal_pass_cache(wl, w, dev, chunk=4096):
+    """The workload's cache as the inference cycle leaves it (Algorithm
+    CacheManagedInference in pre-fill): a causal pass of the random model over
+    seeded uniform token ids, appended chunk by chunk with cc_append_chunk
+    (every layer's post-RoPE K/V, tokens, positions 0..n-1 and, for the fast
+    pass, H^(L-1)).  Slots past a sequence's end stay zero.  Untimed set-up."""
     import paper_2607_27600_gb300 as pkg
     from paper_2607_27600_gb300 import cc
-    pkg.load_library()
-    dev = torch.device(f"cuda:{dist.local}")
-    torch.cuda.set_device(dev)
-    wl = synth.WORKLOADS[args.workload]
-    shape = wl.shape
-    mode = cc.SCORE_LOGPROB if args.score == "logprob" else cc.SCORE_LOGIT
-    fast = wl.mode == "layer"
-    if wl.cycles > 1 and not args.single_cycle:
-        raise SystemExit("multi-cycle workloads: use --single-cycle (the first refresh is timed)")
+    shape, b, cap = wl.shape, wl.batch, wl.cap
+    kv = (b, cap, shape.n_kv_heads, shape.head_dim)
+    cache = {"k": [torch.zeros(kv, dtype=torch.bfloat16, device=dev) for _ in range(shape.n_layers)],
+             "v": [torch.zeros(kv, dtype=torch.bfloat16, device=dev) for _ in range(shape.n_layers)],
+             "tokens": torch.zeros(b, cap, dtype=torch.int32, device=dev),
+             "pos": torch.zeros(b, cap, dtype=torch.int32, device=dev),
+             "seq_len": torch.zeros(b, dtype=torch.int32, device=dev),
+             "h_last": (torch.zeros(b, cap, shape.d_model, dtype=torch.bfloat16, device=dev)
+                        if wl.mode == "layer" else None)}
+    toks = synth.tokens((b, cap), shape.vocab, wl.seed, "bench.cache.tokens", dev)
+    weights, kc = pkg.Weights(w), pkg.Cache(cache)
+    ws = cc.alloc_workspace(cc.cc_append_workspace_size(shape, b, cap), dev)
+    for s0 in range(0, max(wl.seq_lens), chunk):
+        cnt = torch.tensor([max(0, min(chunk, n - s0)) for n in wl.seq_lens], dtype=torch.int32,
+                           device=dev)
+        tin = torch.zeros(b, chunk, dtype=torch.int32, device=dev)
+        width = min(chunk, cap - s0)
+        tin[:, :width] = toks[:, s0:s0 + width]
+        cc.cc_append_chunk(shape, weights, kc, tin, None, cnt, chunk, ws)
+    torch.cuda.synchronize(dev)
+    status = cc.cc_get_status()
+    if status != cc.CC_OK or cache["seq_len"].cpu().tolist() != list(wl.seq_lens):
+        raise SystemExit(f"causal pass did not fill the cache: {cc.cc_status_str(status)}")
+    del ws
+    return cache
 
-    w, pristine = make_inputs(wl, dev, args.kv_fp8, args.paged, args.head_major)
+
+def bench_inputs(args, wl, dev):
+    """Weights and pristine cache of a workload: the cache from the causal pass
+    (default) or drawn directly (--synthetic-cache), then the requested layout
+    variants."""
+    fast = wl.mode == "layer"
+    if args.synthetic_cache or args.kv_fp8 or args.paged or args.head_major:
+        return make_inputs(wl, dev, args.kv_fp8, args.paged, args.head_major), "synthetic draws"
+    w = synth.model_weights(wl.shape, wl.seed, device=dev, with_kv_proj=True, with_embed=True)
+    cache = causal_pass_cache(wl, w, dev)
+    if wl.cycles > 1:   # the refresh cycles append through every layer
+        return (w, cache), "causal pass of the random model over seeded uniform token ids (cc_append_chunk)"
+    if fast:   # the fast pass reads only the last layer's weights
+        w["layers"] = [None] * (wl.shape.n_layers - 1) + [w["layers"][-1]]
+        w["embed"] = None
+    for lw in w["layers"]:
+        if lw is not None:
+            for key in ("wk", "wv", "bk", "bv"):
+                lw.pop(key, None)
+    torch.cuda.empty_cache()
+    return (w, cache), "causal pass of the random model over seeded uniform token ids (cc_append_chunk)"
+
+
+def refresh_record(args, dist, wl, w, pristine, mode, steps, with_e2e=True, with_cpu=True):
+    """Times one refresh of `wl` (score + select + compaction of every layer)
+    over `steps` steps: device-resident inputs with CUDA events on the
+    launching stream; the same steps again with events around every library
+    launch (per-kernel table, roofline); with_e2e, the same step through the
+    public API with its inputs from pinned host memory; with_cpu, the oracle
+    on the host cores."""
+    import paper_2607_27600_gb300 as pkg
+    from paper_2607_27600_gb300 import cc
+    dev = torch.device(f"cuda:{dist.local}")
+    shape = wl.shape
+    fast = wl.mode == "layer"
     work = clone_cache(pristine)
     weights, cache = pkg.Weights(w), pkg.Cache(work)
     b, cap = wl.batch, wl.cap
@@ -361,16 +416,16 @@ def run_ours(args, dist):
     torch.cuda.synchronize(dev)
     status = cc.cc_get_status()
     if status != cc.CC_OK:
-        raise SystemExit(f"device status after warm-up: {cc.cc_status_str(status)}")
+        raise SystemExit(f"{wl.name}: device status after warm-up: {cc.cc_status_str(status)}")
 
     clocks = ClockSampler(dist.local)
     clocks.start()
     time.sleep(0.3)
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-          for _ in range(args.steps)]
+          for _ in range(steps)]
     dist.barrier()
     torch.cuda.synchronize(dev)
-    for i in range(args.steps):
+    for i in range(steps):
         prepare()
         ev[i][0].record(stream)
         step()
@@ -378,47 +433,102 @@ def run_ours(args, dist):
     torch.cuda.synchronize(dev)
     dist.barrier()
     step_ms = [a.elapsed_time(bb) for a, bb in ev]
+    ref_idx, ref_cnt = keep_idx.cpu(), keep_count.cpu()   # the last timed step's keep-set
     # per-kernel table: the same steps again with CUDA events around every
     # library launch (kept out of the timed steps above, whose launches they
     # would slow down)
     cc.cc_timing_enable(True)
-    for i in range(args.steps):
+    for i in range(steps):
         prepare()
         step()
     torch.cuda.synchronize(dev)
     kernels = cc.cc_timing_collect()
     cc.cc_timing_enable(False)
-    ms_local = sum(step_ms) / args.steps
-    ms = dist.max(ms_local)
+    ms = dist.max(sum(step_ms) / steps)
     status = cc.cc_get_status()
     if status != cc.CC_OK:
-        raise SystemExit(f"device status after timing: {cc.cc_status_str(status)}")
+        raise SystemExit(f"{wl.name}: device status after timing: {cc.cc_status_str(status)}")
+    positions = sum(wl.seq_lens)
 
-    # ---- end to end through the public API with host inputs
-    host = {"h_last": pristine["h_last"].cpu().pin_memory() if fast else None,
-            "k": pristine["k"][-1].cpu().pin_memory(), "v": pristine["v"][-1].cpu().pin_memory(),
-            "tokens": pristine["tokens"].cpu().pin_memory(),
-            "pos": pristine["pos"].cpu().pin_memory(),
-            "seq_len": pristine["seq_len"].cpu().pin_memory()}
-    if not fast:   # the full pass reads every layer's K/V
-        host["k_all"] = [x.cpu().pin_memory() for x in pristine["k"]]
-        host["v_all"] = [x.cpu().pin_memory() for x in pristine["v"]]
-    out_idx = torch.empty(b, cap, dtype=torch.int32).pin_memory()
-    out_cnt = torch.empty(b, dtype=torch.int32).pin_memory()
-    h2d = sum(t.numel() * t.element_size() for k, t in host.items()
-              if isinstance(t, torch.Tensor))
-    if not fast:
-        h2d += sum(t.numel() * t.element_size() for t in host["k_all"] + host["v_all"])
-        h2d -= host["k"].numel() * host["k"].element_size() * 2
-    d2h = out_idx.numel() * 4 + out_cnt.numel() * 4
+    e2e = None
+    if with_e2e:
+        e2e = e2e_leg(args, dist, wl, work, pristine, cache, step, keep_idx, keep_count, flush,
+                      stream, steps)
+        if not (torch.equal(e2e.pop("keep_idx"), ref_idx) and
+                torch.equal(e2e.pop("keep_count"), ref_cnt)):
+            raise SystemExit(f"{wl.name}: the end-to-end keep-set differs from the "
+                             "device-resident step's")
+    clk = clocks.stop()
 
-    # K/V uploads run on a copy stream and the library waits for each layer's
-    # event right before the layer's first K/V reader (cc_kv_cache.kv_ready),
-    # so they overlap the kernels ahead of it; the host link is one queue, so
-    # they start once the inputs of the first kernels have landed
-    up = torch.cuda.Stream(dev)
+    peaks, peak_src = load_peaks()
+    work_tbl = algorithmic_work(wl, 1 if args.kv_fp8 else 2)
+    if scorer in ("importance", "h2o"):
+        work_tbl["keyattn"] = keyattn_work(wl, scorer, recent)
+    table = kernel_table(kernels, steps, work_tbl, peaks)
+    dom = max(kernels.items(), key=lambda kv: kv[1][1])[0]
+    precise = bool(mode & cc.SCORE_PRECISE)
+    traffic = None if precise else read_traffic(dom, wl.name)
+    d = table[dom]
+    roof = {"kernel": dom, "bound": d.get("bound"), "achieved": d.get("achieved"),
+            "peak": peaks["bf16_tflops"] if d.get("bound") == "tensor" else peaks["hbm_gbs"],
+            "unit": d.get("unit"), "frac": d.get("frac"), "traffic": traffic,
+            "peak_source": f"{peak_src} ({'bf16 dense burst' if d.get('bound') == 'tensor' else 'HBM copy'})"}
+    value = positions * dist.world / (ms * 1e-3)
+    rec = {
+        "workload": wl.name, "value": round(value, 1), "unit": "positions/s",
+        "ms_per_step": round(ms, 4), "steps": steps,
+        "mode": ("precise: [hi | lo] bf16 pairs for activations, queries and P"
+                 if precise else "bf16 operands, fp32 accumulation"),
+        "pass": ("fast single-layer" if fast else f"full {shape.n_layers}-layer")
+        if scorer == "counter-causal" else
+        {"recency": "position", "importance": "last-layer key attention",
+         "h2o": f"all-layer key attention, {recent} recent proxy queries"}[scorer],
+        "tflops_per_step_achieved": (round(step_flops(wl) / (ms * 1e-3) / 1e12, 1)
+                                     if scorer == "counter-causal" else None),
+        "step_tflop": round(step_flops(wl) / 1e12, 3) if scorer == "counter-causal" else None,
+        "gpu_launches": int(sum(c for c, _ in kernels.values())),
+        "roofline": roof, "kernels": table, "clocks": clk,
+    }
+    if precise:
+        rec["roofline"]["note"] = ("algorithmic FLOPs of the pass; the precise mode issues each "
+                                   "product once per operand half (about twice these FLOPs)")
+    if e2e is not None:
+        rec["e2e"] = {"value": round(positions * dist.world / (e2e["ms"] * 1e-3), 1),
+                      "unit": "positions/s", "h2d_bytes_per_step": e2e["h2d"],
+                      "d2h_bytes_per_step": e2e["d2h"], "ms_per_step": round(e2e["ms"], 4)}
+    if (with_cpu and dist.world == 1 and not args.no_cpu_baseline and
+            scorer == "counter-causal"):
+        rec["cpu_baseline"] = OracleLeg(wl, w, pristine, args.score).cpu_baseline(
+            scores.cpu().numpy())
+    return rec
+
+
+def e2e_leg(args, dist, wl, work, pristine, cache, step, keep_idx, keep_count, flush, stream,
+            steps):
+    """The refresh through the public API with the step's inputs in pinned
+    host memory: H^(L-1) (fast pass), token ids, positions and lengths on the
+    compute stream; each scored layer's K/V on a copy stream that the library
+    waits on per layer (cc_kv_cache.kv_ready), so the uploads overlap the
+    kernels ahead of that layer's first K/V reader; the keep-set read back.
+    Copies and reads are inside the timed region."""
+    dev = torch.device(f"cuda:{dist.local}")
+    fast = wl.mode == "layer"
+    b, cap = wl.batch, wl.cap
     n_l = len(work["k"])
     kv_layers = [n_l - 1] if fast else list(range(n_l))
+    host = {"h_last": pristine["h_last"].cpu().pin_memory() if fast else None,
+            "tokens": pristine["tokens"].cpu().pin_memory(),
+            "pos": pristine["pos"].cpu().pin_memory(),
+            "seq_len": pristine["seq_len"].cpu().pin_memory(),
+            "k": {l: pristine["k"][l].cpu().pin_memory() for l in kv_layers},
+            "v": {l: pristine["v"][l].cpu().pin_memory() for l in kv_layers}}
+    out_idx = torch.empty(b, cap, dtype=torch.int32).pin_memory()
+    out_cnt = torch.empty(b, dtype=torch.int32).pin_memory()
+    h2d = sum(t.numel() * t.element_size() for key in ("h_last", "tokens", "pos", "seq_len")
+              for t in [host[key]] if t is not None)
+    h2d += sum(t.numel() * t.element_size() for key in ("k", "v") for t in host[key].values())
+    d2h = out_idx.numel() * 4 + out_cnt.numel() * 4
+    up = torch.cuda.Stream(dev)
     ready = [torch.cuda.Event() if l in kv_layers else None for l in range(n_l)]
     for e in ready:
         if e is not None:
@@ -433,110 +543,216 @@ def run_ours(args, dist):
         up.wait_stream(stream)
         with torch.cuda.stream(up):
             for l in kv_layers:
-                work["k"][l].copy_(host["k"] if fast else host["k_all"][l], non_blocking=True)
-                work["v"][l].copy_(host["v"] if fast else host["v_all"][l], non_blocking=True)
+                work["k"][l].copy_(host["k"][l], non_blocking=True)
+                work["v"][l].copy_(host["v"][l], non_blocking=True)
                 ready[l].record(up)
         step()
         out_idx.copy_(keep_idx, non_blocking=True)
         out_cnt.copy_(keep_count, non_blocking=True)
 
     cache.set_kv_ready(ready)
-
     e2e_ms = []
-    for i in range(args.steps):
-        restore_cache(work, pristine)   # the rest of the device-resident cache
-        flush.fill_(1)
-        torch.cuda.synchronize(dev)
-        t0 = torch.cuda.Event(enable_timing=True)
-        t1 = torch.cuda.Event(enable_timing=True)
-        t0.record(stream)
-        e2e_step()
-        t1.record(stream)
-        torch.cuda.synchronize(dev)
-        e2e_ms.append(t0.elapsed_time(t1))
-    cache.set_kv_ready(None)
-    clk = clocks.stop()
-    e2e_ms_max = dist.max(sum(e2e_ms) / len(e2e_ms))
+    try:
+        for _ in range(steps):
+            restore_cache(work, pristine)   # the rest of the device-resident cache
+            flush.fill_(1)
+            torch.cuda.synchronize(dev)
+            t0 = torch.cuda.Event(enable_timing=True)
+            t1 = torch.cuda.Event(enable_timing=True)
+            t0.record(stream)
+            e2e_step()
+            t1.record(stream)
+            torch.cuda.synchronize(dev)
+            e2e_ms.append(t0.elapsed_time(t1))
+    finally:
+        cache.set_kv_ready(None)
+    from paper_2607_27600_gb300 import cc
     status = cc.cc_get_status()
     if status != cc.CC_OK:
-        raise SystemExit(f"device status after e2e: {cc.cc_status_str(status)}")
-    # sanity: the e2e keep-set equals the device-resident one of the last timed step
-    positions = sum(wl.seq_lens)
+        raise SystemExit(f"{wl.name}: device status after e2e: {cc.cc_status_str(status)}")
+    return {"ms": dist.max(sum(e2e_ms) / len(e2e_ms)), "h2d": int(h2d), "d2h": int(d2h),
+            "keep_idx": out_idx.clone(), "keep_count": out_cnt.clone()}
 
-    # ---- roofline of the dominant kernel (and a per-kernel table)
-    peaks, peak_src = load_peaks()
-    work_tbl = algorithmic_work(wl, 1 if args.kv_fp8 else 2)
-    if scorer in ("importance", "h2o"):
-        work_tbl["keyattn"] = keyattn_work(wl, scorer, recent)
-    table = {}
-    for name, (cnt, tot) in kernels.items():
-        per = tot / cnt
-        entry = {"launches_per_step": cnt / args.steps, "ms_per_launch": round(per, 4),
-                 "share": round(tot / max(1e-9, sum(t for _, t in kernels.values())), 4)}
-        if name in work_tbl:
-            bound, amount = work_tbl[name]
-            if bound == "tensor":
-                ach = amount / (per * 1e-3) / 1e12
-                entry.update({"bound": "tensor", "achieved": round(ach, 2), "unit": "TFLOP/s",
-                              "frac": round(ach / peaks["bf16_tflops"], 4)})
-            else:
-                ach = amount / (per * 1e-3) / 1e9
-                entry.update({"bound": "hbm", "achieved": round(ach, 1), "unit": "GB/s",
-                              "frac": round(ach / peaks["hbm_gbs"], 4)})
-        table[name] = entry
-    dom = max(kernels.items(), key=lambda kv: kv[1][1])[0]
-    traffic = read_traffic(dom, wl.name)
-    d = table[dom]
-    roof = {"kernel": dom, "bound": d.get("bound"), "achieved": d.get("achieved"),
-            "peak": peaks["bf16_tflops"] if d.get("bound") == "tensor" else peaks["hbm_gbs"],
-            "unit": d.get("unit"), "frac": d.get("frac"), "traffic": traffic,
-            "peak_source": f"{peak_src} ({'bf16 dense burst' if d.get('bound') == 'tensor' else 'HBM copy'})"}
 
-    launches = sum(c for c, _ in kernels.values())
-    value = positions * dist.world / (ms * 1e-3)
+def cycles_record(args, dist, wl, w, pristine, steps):
+    """The workload's refresh cycles as configured (Algorithm
+    CacheManagedInference, chunked): one step = the refresh of the whole
+    cache, then for each later cycle the inference cycle's append of
+    `wl.append` new tokens through every layer (cc_append_chunk, seeded token
+    ids, positions continuing) and the next refresh.  Appends and refreshes
+    are timed separately with CUDA events; positions/s per refresh cycle."""
+    import paper_2607_27600_gb300 as pkg
+    from paper_2607_27600_gb300 import cc
+    dev = torch.device(f"cuda:{dist.local}")
+    shape = wl.shape
+    full_w = w
+    work = clone_cache(pristine)
+    weights, cache = pkg.Weights(full_w), pkg.Cache(work)
+    b, cap = wl.batch, wl.cap
+    mode = cc.SCORE_LOGIT
+    scores = torch.empty(b, cap, dtype=torch.float32, device=dev)
+    keep_idx = torch.empty(b, cap, dtype=torch.int32, device=dev)
+    keep_count = torch.empty(b, dtype=torch.int32, device=dev)
+    budget = torch.tensor(wl.budgets, dtype=torch.int32, device=dev)
+    ws = cc.alloc_workspace(cc.cc_score_workspace_size(shape, b, cap, mode), dev)
+    cws = cc.alloc_workspace(cc.cc_compact_workspace_size(shape, cache), dev)
+    aws = cc.alloc_workspace(cc.cc_append_workspace_size(shape, b, cap), dev)
+    chunks = [synth.tokens((b, wl.append), shape.vocab, wl.seed, f"bench.cycle{c}", dev)
+              for c in range(1, wl.cycles)]
+    count = torch.full((b,), wl.append, dtype=torch.int32, device=dev)
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def refresh():
+        cc.cc_score_layer(shape, weights, cache, mode, scores, ws)
+        cc.cc_select_keep(scores, cache.d["seq_len"], b, cap, budget, wl.n_sink, keep_idx,
+                          keep_count)
+        cc.cc_compact_kv(shape, cache, keep_idx, keep_count, cws)
+
+    def one_step(evs=None):
+        for c in range(wl.cycles):
+            if c > 0:
+                if evs is not None:
+                    evs[c]["append"][0].record(stream)
+                cc.cc_append_chunk(shape, weights, cache, chunks[c - 1], None, count, wl.append,
+                                   aws)
+                if evs is not None:
+                    evs[c]["append"][1].record(stream)
+            if evs is not None:
+                evs[c]["refresh"][0].record(stream)
+            refresh()
+            if evs is not None:
+                evs[c]["refresh"][1].record(stream)
+
+    def prepare():
+        restore_cache(work, pristine)
+        flush.fill_(1)
+
+    for _ in range(args.warmup):
+        prepare()
+        one_step()
+    torch.cuda.synchronize(dev)
+    status = cc.cc_get_status()
+    if status != cc.CC_OK:
+        raise SystemExit(f"{wl.name}: device status after warm-up: {cc.cc_status_str(status)}")
+    clocks = ClockSampler(dist.local)
+    clocks.start()
+    time.sleep(0.3)
+
+    def pair():
+        return (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+    per_step = []
+    dist.barrier()
+    for _ in range(steps):
+        prepare()
+        torch.cuda.synchronize(dev)
+        evs = [{"append": pair(), "refresh": pair()} for _ in range(wl.cycles)]
+        one_step(evs)
+        torch.cuda.synchronize(dev)
+        per_step.append([{k: v[0].elapsed_time(v[1]) for k, v in e.items()
+                          if k == "refresh" or c > 0} for c, e in enumerate(evs)])
+    dist.barrier()
+    clk = clocks.stop()
+    status = cc.cc_get_status()
+    if status != cc.CC_OK:
+        raise SystemExit(f"{wl.name}: device status after timing: {cc.cc_status_str(status)}")
+    cycles = []
+    n = wl.seq_lens[0]
+    for c in range(wl.cycles):
+        if c > 0:
+            n = wl.budgets[0] + wl.append
+        r_ms = dist.max(sum(s[c]["refresh"] for s in per_step) / steps)
+        e = {"cycle": c + 1, "scored_positions": n * b, "refresh_ms": round(r_ms, 4),
+             "positions_per_s": round(n * b * dist.world / (r_ms * 1e-3), 1)}
+        if c > 0:
+            a_ms = dist.max(sum(s[c]["append"] for s in per_step) / steps)
+            e.update({"append_tokens": wl.append * b, "append_ms": round(a_ms, 4),
+                      "append_tokens_per_s": round(wl.append * b * dist.world / (a_ms * 1e-3), 1)})
+        cycles.append(e)
+    total_pos = sum(e["scored_positions"] for e in cycles)
+    total_ms = sum(e["refresh_ms"] for e in cycles)
+    return {"workload": wl.name, "value": round(total_pos * dist.world / (total_ms * 1e-3), 1),
+            "unit": "positions/s",
+            "value_basis": "all cycles' scored positions / the cycles' refresh time "
+                           "(appends timed separately)",
+            "steps": steps, "pass": "fast single-layer", "cycles": cycles, "clocks": clk}
+
+
+def run_suite(args, dist):
+    """The default bench line: the headline workload (the full-model pass over
+    all 32 layers of the Llama-3-8B shape, the largest single-GPU workload
+    with a full pass) plus, in the same line, its precise mode, the ragged
+    32k single-layer batch and the long-context refresh cycles."""
+    import paper_2607_27600_gb300 as pkg
+    from paper_2607_27600_gb300 import cc
+    pkg.load_library()
+    dev = torch.device(f"cuda:{dist.local}")
+    torch.cuda.set_device(dev)
+    wl = synth.WORKLOADS[args.workload]
+    mode = cc.SCORE_LOGPROB if args.score == "logprob" else cc.SCORE_LOGIT
+    if args.precise:
+        mode |= cc.SCORE_PRECISE
+    if wl.cycles > 1 and args.scorer == "counter-causal" and not args.single_cycle:
+        (w, pristine), cache_src = bench_inputs(args, wl, dev)
+        rec = cycles_record(args, dist, wl, w, pristine, args.steps)
+        return suite_line(args, dist, wl, rec, cache_src, records={})
+    (w, pristine), cache_src = bench_inputs(args, wl, dev)
+    head = refresh_record(args, dist, wl, w, pristine, mode, args.steps)
+    records = {}
+    if not args.no_records and args.scorer == "counter-causal" and dist.world >= 1:
+        sub = min(args.steps, 10)
+        if not args.precise:
+            records[wl.name + "/precise"] = refresh_record(
+                args, dist, wl, w, pristine, mode | cc.SCORE_PRECISE, sub, with_e2e=False,
+                with_cpu=False)
+        if args.workload == synth.HEADLINE:
+            del w, pristine
+            torch.cuda.empty_cache()
+            for name in synth.RECORDS:
+                rwl = synth.WORKLOADS[name]
+                (rw, rp), _ = bench_inputs(args, rwl, dev)
+                if rwl.cycles > 1:
+                    records[name] = cycles_record(args, dist, rwl, rw, rp, sub)
+                else:
+                    records[name] = refresh_record(args, dist, rwl, rw, rp, mode, args.steps)
+                del rw, rp
+                torch.cuda.empty_cache()
+    return suite_line(args, dist, wl, head, cache_src, records)
+
+
+def suite_line(args, dist, wl, head, cache_src, records):
+    shape = wl.shape
     # the paper's own figure for this workload (Table 1, another GPU): context only
-    vs_baseline = (round(value / wl.paper_positions_per_s, 2)
-                   if wl.paper_positions_per_s and scorer == "counter-causal" else None)
+    vs_baseline = (round(head["value"] / wl.paper_positions_per_s, 2)
+                   if wl.paper_positions_per_s and args.scorer == "counter-causal" else None)
     line = {
         "metric": "scored KV positions/sec per refresh",
-        "value": round(value, 1), "unit": "positions/s", "n_gpus": dist.world,
-        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 4),
+        "value": head["value"], "unit": "positions/s", "n_gpus": dist.world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": head.get("ms_per_step"),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": vs_baseline, "dtype": "bf16",
-        "data": "synthetic (seeded random-init weights N(0,0.02); synthetic KV cache)",
-        "config": {"workload": wl.name, "scorer": scorer,
+        "data": f"synthetic (seeded random-init weights N(0,0.02); cache: {cache_src})",
+        "config": {"workload": wl.name, "scorer": args.scorer,
                    "kv_cache": ("e4m3 (per-layer scales)" if args.kv_fp8 else "bf16") +
                                (f", paged ({args.paged}-slot pages)" if args.paged else "") +
                                (", head-major" if args.head_major else ""),
-                   "pass": ("fast single-layer" if fast else f"full {shape.n_layers}-layer")
-                   if scorer == "counter-causal" else
-                   {"recency": "position", "importance": "last-layer key attention",
-                    "h2o": f"all-layer key attention, {recent} recent proxy queries"}[scorer],
+                   "pass": head.get("pass"), "mode": head.get("mode"),
                    "score": args.score, "batch": wl.batch, "seq_lens": wl.seq_lens,
                    "budgets": wl.budgets, "cap": wl.cap, "d_model": shape.d_model,
                    "heads": f"{shape.n_q_heads}/{shape.n_kv_heads}x{shape.head_dim}",
                    "d_ff": shape.d_ff, "vocab": shape.vocab,
-                   "layers_compacted": shape.n_layers,
-                   "step_tflop": (round(step_flops(wl) / 1e12, 3) if scorer == "counter-causal"
-                                  else None),
+                   "layers_compacted": shape.n_layers, "step_tflop": head.get("step_tflop"),
                    "l2": "cache restored + 256 MiB written between steps (outside the timed events)",
                    "parallelism": f"replicas x{dist.world}"},
-        "e2e": {"value": round(positions * dist.world / (e2e_ms_max * 1e-3), 1),
-                "unit": "positions/s", "h2d_bytes_per_step": int(h2d),
-                "d2h_bytes_per_step": int(d2h), "ms_per_step": round(e2e_ms_max, 4)},
-        "gpu_launches": int(launches),
-        "roofline": roof,
-        "kernels": table,
-        # the counter-causal pass's algorithmic FLOPs (the comparison scorers' are
-        # in their keyattn entry)
-        "tflops_per_step_achieved": (round(step_flops(wl) / (ms * 1e-3) / 1e12, 1)
-                                     if scorer == "counter-causal" else None),
-        "clocks": clk,
     }
-    if wl.paper_positions_per_s and scorer == "counter-causal":
+    for key in ("e2e", "gpu_launches", "roofline", "kernels", "tflops_per_step_achieved",
+                "clocks", "cpu_baseline", "cycles", "value_basis"):
+        if key in head:
+            line[key] = head[key]
+    if wl.paper_positions_per_s and args.scorer == "counter-causal":
         line["paper"] = {"value": round(wl.paper_positions_per_s, 1), "unit": "positions/s",
                          "source": "Table 1: n / refresh latency, Qwen2.5-7B, RTX 4090, fp16"}
-    if dist.world == 1 and not args.no_cpu_baseline and scorer == "counter-causal":
-        line["cpu_baseline"] = cpu_baseline(wl, w, pristine, scores, args.cpu_rows, args.score)
+    if records:
+        line["records"] = records
     return line
 
 
@@ -571,16 +787,17 @@ def csrc_digest():
 # the oracle on the host cores (CPU baseline / reference arm)
 # ---------------------------------------------------------------------------
 
-def host_inputs(wl, w, cache):
-    """numpy copies (bf16 widened to fp32; K/V of the compacted layers kept as raw 16-bit)."""
+def host_inputs(wl, w, cache, layers):
+    """numpy copies for the oracle (bf16 widened to fp32) of the weights and
+    K/V of `layers` (a list of layer indices), and raw 16-bit (or e4m3 byte)
+    K/V rows of those layers for the compaction."""
     def f32(t):
         return None if t is None else t.float().cpu().numpy()
-    last = wl.shape.n_layers - 1
-    fast = wl.mode == "layer"
-    lw = [None] * wl.shape.n_layers
-    for l, x in enumerate(w["layers"]):
-        if x is not None:
-            lw[l] = {k: f32(v) for k, v in x.items()}
+    nl = wl.shape.n_layers
+    lw = [None] * nl
+    for l in layers:
+        x = w["layers"][l]
+        lw[l] = {k: f32(v) for k, v in x.items() if k not in ("wk", "wv", "bk", "bv")}
     wn = {"embed": f32(w["embed"]), "final_norm": f32(w["final_norm"]),
           "lm_head": f32(w["lm_head"]), "layers": lw}
     sc = cache.get("kv_scale")
@@ -593,69 +810,15 @@ def host_inputs(wl, w, cache):
     else:
         def kvf(key, l):
             return f32(logical_kv(cache, key, l))
-    kf = [kvf("k", l) if (not fast or l == last) else None for l in range(wl.shape.n_layers)]
-    vf = [kvf("v", l) if (not fast or l == last) else None for l in range(wl.shape.n_layers)]
+    kf = [kvf("k", l) if l in layers else None for l in range(nl)]
+    vf = [kvf("v", l) if l in layers else None for l in range(nl)]
     cn = {"k": kf, "v": vf, "tokens": cache["tokens"].cpu().numpy(), "pos": cache["pos"].cpu().numpy(),
           "seq_len": cache["seq_len"].cpu().numpy(), "h_last": f32(cache["h_last"])}
     kv_raw = torch.uint8 if sc is not None else torch.int16
-    raw = {"k": [logical_kv(cache, "k", l).view(kv_raw).cpu().numpy()
-                 for l in range(len(cache["k"]))],
-           "v": [logical_kv(cache, "v", l).view(kv_raw).cpu().numpy()
-                 for l in range(len(cache["v"]))],
+    raw = {"k": [logical_kv(cache, "k", l).view(kv_raw).cpu().numpy() for l in layers],
+           "v": [logical_kv(cache, "v", l).view(kv_raw).cpu().numpy() for l in layers],
            "h": None if cache["h_last"] is None else cache["h_last"].view(torch.int16).cpu().numpy()}
     return wn, cn, raw
-
-
-def sample_rows(wl, count, seed=0):
-    r = np.random.default_rng(seed)
-    rows = []
-    per = max(2, count // wl.batch)
-    for n in wl.seq_lens:
-        pick = {0, n - 2, n - 1} | set(r.choice(n, size=min(n, per), replace=False).tolist())
-        rows.append(sorted(x for x in pick if 0 <= x < n)[:max(per, 3)])
-    return rows
-
-
-def _oracle_score_time(wl, wn, cn, rows, score_mode):
-    import oracle
-    fn = oracle.score_layer if wl.mode == "layer" else oracle.score_full
-    t0 = time.perf_counter()
-    fn(wl.shape, wn, cn, mode=score_mode, rows=rows)
-    return time.perf_counter() - t0, sum(len(r) for r in rows)
-
-
-def oracle_fixed_cost(wl, wn, cn, score_mode, small, large):
-    """Per-call cost of the oracle's scoring that does not grow with the rows
-    (widening the weights to fp64), from two sample sizes."""
-    t1, n1 = _oracle_score_time(wl, wn, cn, sample_rows(wl, small, seed=11), score_mode)
-    t2, n2 = _oracle_score_time(wl, wn, cn, sample_rows(wl, large, seed=12), score_mode)
-    per_row = max(0.0, (t2 - t1) / max(1, n2 - n1))
-    return max(0.0, t1 - n1 * per_row)
-
-
-def oracle_refresh_time(wl, wn, cn, raw, scores_np, rows, score_mode, fixed):
-    """Seconds the oracle takes for one refresh of the whole workload: its
-    scoring timed on the sampled rows and extrapolated linearly in the row
-    count (rows are independent given the cache; the per-call fixed cost is
-    counted once), plus its select and compaction run in full."""
-    import oracle
-    t_rows, n_sampled = _oracle_score_time(wl, wn, cn, rows, score_mode)
-    per_row = max(0.0, t_rows - fixed) / n_sampled
-    t1 = time.perf_counter()
-    idx, cnt = oracle.select_keep(scores_np, cn["seq_len"], wl.budgets, wl.n_sink)
-    t_sel = time.perf_counter() - t1
-    t2 = time.perf_counter()
-    for arrs in (raw["k"], raw["v"]):
-        for a in arrs:
-            oracle.compact(a, idx, cnt)
-    if raw["h"] is not None:
-        oracle.compact(raw["h"], idx, cnt)
-    oracle.compact(cn["tokens"], idx, cnt)
-    oracle.compact(cn["pos"], idx, cnt)
-    t_cmp = time.perf_counter() - t2
-    positions = sum(wl.seq_lens)
-    total = fixed + per_row * positions + t_sel + t_cmp
-    return total, n_sampled, t_rows, t_sel, t_cmp
 
 
 def cores_used():
@@ -665,54 +828,162 @@ def cores_used():
         return os.cpu_count()
 
 
-def cpu_baseline(wl, w, cache, scores_dev, n_rows, score_mode):
-    wn, cn, raw = host_inputs(wl, w, cache)
-    scores_np = scores_dev.cpu().numpy()
-    fixed = oracle_fixed_cost(wl, wn, cn, score_mode, n_rows // 4, n_rows // 2)
-    rows = sample_rows(wl, n_rows)
-    total, ns, t_rows, t_sel, t_cmp = oracle_refresh_time(wl, wn, cn, raw, scores_np, rows,
-                                                          score_mode, fixed)
-    return {"value": round(sum(wl.seq_lens) / total, 3), "unit": "positions/s",
-            "cores": cores_used(), "kind": "oracle",
-            "sample": (f"{ns} sampled rows scored ({t_rows:.1f} s incl. {fixed:.1f} s per-call "
-                       f"fixed cost), extrapolated linearly to {sum(wl.seq_lens)} rows, + full "
-                       f"select ({t_sel:.2f} s) + full compaction ({t_cmp:.2f} s); numpy fp64, "
-                       f"BLAS threads = cores")}
+class OracleLeg:
+    """The oracle, as it stands, timed on the host cores on a bounded sample of
+    one refresh of a workload; both the cpu_baseline of our arm and the
+    reference arm use it with the same sample sizes.
+
+    A refresh is scoring, select and compaction.  Scoring rows are independent
+    given the cache and every layer of a pass repeats the same work, so the
+    sample scores `rows` rows drawn uniformly over all positions through
+    `layers` layers (all of the fast pass's one layer; the first two of a full
+    pass, a truncated model), and the time extrapolates linearly: per-call
+    fixed cost (widening each sampled layer's weights) from two sample sizes,
+    times L / layers, plus the per-row cost times N.  Select runs in full; the
+    compaction moves tokens, positions and H^(L-1) in full and the K/V of the
+    sampled layers, extrapolated to all L layers.  Every extrapolated figure is
+    labelled as such."""
+
+    def __init__(self, wl, w, cache, score_mode):
+        import dataclasses
+        self.wl, self.mode = wl, score_mode
+        nl = wl.shape.n_layers
+        self.fast = wl.mode == "layer"
+        self.layers = [nl - 1] if self.fast else list(range(min(2, nl)))
+        self.shape = wl.shape if self.fast else dataclasses.replace(wl.shape,
+                                                                     n_layers=len(self.layers))
+        self.kv_layers = [nl - 1] if self.fast else self.layers
+        self.wn, self.cn, self.raw = host_inputs(wl, w, cache, sorted(set(self.layers)))
+        # sample sizes large enough that the per-row cost stands out of the
+        # per-call fixed cost in the fit
+        self.rows_small, self.rows_large = (64, 128) if self.fast else (16, 32)
+        self.positions = sum(wl.seq_lens)
+        self.fixed = None
+
+    def sample(self, count, seed):
+        """`count` rows drawn uniformly over all of the workload's positions."""
+        r = np.random.default_rng(seed)
+        flat = np.sort(r.choice(self.positions, size=min(count, self.positions), replace=False))
+        starts = np.cumsum([0] + list(self.wl.seq_lens))
+        return [(flat[(flat >= starts[b]) & (flat < starts[b + 1])] - starts[b]).tolist()
+                for b in range(self.wl.batch)]
+
+    def _score(self, rows):
+        import oracle
+        fn = oracle.score_layer if self.fast else oracle.score_full
+        t0 = time.perf_counter()
+        fn(self.shape, self.wn, self.cn, mode=self.mode, rows=rows)
+        return time.perf_counter() - t0, sum(len(r) for r in rows)
+
+    def fit(self):
+        """Per-call fixed cost of the sampled scoring, from two sample sizes
+        (after one untimed call that pays the one-time set-up)."""
+        self._score(self.sample(self.rows_small, seed=10))
+        t1, n1 = self._score(self.sample(self.rows_small, seed=11))
+        t2, n2 = self._score(self.sample(self.rows_large, seed=12))
+        per_row = max(0.0, (t2 - t1) / max(1, n2 - n1))
+        self.fixed = max(0.0, t1 - n1 * per_row)
+        return self.fixed
+
+    def step(self, scores_np, seed):
+        """One sampled refresh; returns (measured seconds, extrapolated seconds
+        of the whole refresh, details)."""
+        import oracle
+        if self.fixed is None:
+            self.fit()
+        w0 = time.perf_counter()
+        t_rows, n_rows = self._score(self.sample(self.rows_large, seed))
+        t1 = time.perf_counter()
+        idx, cnt = oracle.select_keep(scores_np, self.cn["seq_len"], self.wl.budgets,
+                                      self.wl.n_sink)
+        t_sel = time.perf_counter() - t1
+        t2 = time.perf_counter()
+        for arrs in (self.raw["k"], self.raw["v"]):
+            for a in arrs:
+                oracle.compact(a, idx, cnt)
+        t_kv = time.perf_counter() - t2
+        t3 = time.perf_counter()
+        if self.raw["h"] is not None:
+            oracle.compact(self.raw["h"], idx, cnt)
+        oracle.compact(self.cn["tokens"], idx, cnt)
+        oracle.compact(self.cn["pos"], idx, cnt)
+        t_small = time.perf_counter() - t3
+        measured = time.perf_counter() - w0
+        nl = self.wl.shape.n_layers
+        lf = nl / len(self.layers) if not self.fast else 1.0
+        per_row = max(0.0, t_rows - self.fixed) / n_rows
+        t_score = lf * (self.fixed + per_row * self.positions)
+        t_compact = t_small + t_kv * nl / len(self.kv_layers)
+        total = t_score + t_sel + t_compact
+        return measured, total, {"rows": n_rows, "t_rows": t_rows, "t_sel": t_sel,
+                                 "t_compact": t_compact}
+
+    def describe(self, d):
+        lay = ("its one layer" if self.fast else
+               f"{len(self.layers)} of {self.wl.shape.n_layers} layers (a truncated model), "
+               f"x{self.wl.shape.n_layers // len(self.layers)}")
+        return (f"{d['rows']} rows drawn uniformly over {self.positions} positions scored through "
+                f"{lay} ({d['t_rows']:.2f} s, per-call fixed cost {self.fixed:.2f} s fitted from "
+                f"{self.rows_small} and {self.rows_large} rows), extrapolated linearly to every "
+                f"row; full select ({d['t_sel']:.3f} s); compaction of tokens, positions and "
+                f"H^(L-1) in full and of {len(self.kv_layers)} layers' K/V, extrapolated to "
+                f"{self.wl.shape.n_layers} layers ({d['t_compact']:.2f} s); numpy fp64, BLAS "
+                f"threads = cores")
+
+    def cpu_baseline(self, scores_np):
+        measured, total, d = self.step(scores_np, seed=0)
+        return {"value": round(self.positions / total, 3), "unit": "positions/s",
+                "cores": cores_used(), "kind": "oracle", "extrapolated": True,
+                "sample_s": round(measured, 2), "sample": self.describe(d)}
 
 
 def run_reference(args, dist):
+    """The reference arm: the oracle (CPU) timed on a bounded sample of the
+    same workload per step (OracleLeg), rank 0 only."""
     if dist.rank != 0:
         return None
     wl = synth.WORKLOADS[args.workload]
     dev = torch.device("cuda:0") if torch.cuda.is_available() else torch.device("cpu")
-    w, cache = make_inputs(wl, dev)
-    wn, cn, raw = host_inputs(wl, w, cache)
+    if dev.type == "cuda":
+        torch.cuda.set_device(dev)
+    # the oracle's inputs come from the seeded generators alone (the cache drawn
+    # directly: the oracle's time does not depend on the values); only the
+    # layers the sample runs are drawn
+    nl = wl.shape.n_layers
+    sampled = [nl - 1] if wl.mode == "layer" else list(range(min(2, nl)))
+    w = synth.model_weights(wl.shape, wl.seed, device=dev, layers=sampled,
+                            with_embed=wl.mode == "full")
+    cache = synth.synthetic_cache(wl.shape, wl.seq_lens, wl.cap, wl.seed, device=dev,
+                                  layers=sampled, with_h_last=wl.mode == "layer")
+    leg = OracleLeg(wl, w, cache, args.score)
+    del w, cache
     r = np.random.default_rng(1)
-    scores_np = r.standard_normal(size=cn["tokens"].shape).astype(np.float32)
+    scores_np = r.standard_normal(size=leg.cn["tokens"].shape).astype(np.float32)
     for b, n in enumerate(wl.seq_lens):
         scores_np[b, n - 1] = np.inf
-    times = []
-    ns = 0
-    fixed = oracle_fixed_cost(wl, wn, cn, args.score, max(2, args.ref_rows // 2),
-                              args.ref_rows * 3 // 2)
+    leg.fit()
+    measured, extrap = [], []
+    d = None
     for i in range(args.warmup + args.steps):
-        rows = sample_rows(wl, args.ref_rows, seed=i)
-        total, ns, *_ = oracle_refresh_time(wl, wn, cn, raw, scores_np, rows, args.score, fixed)
+        m, total, d = leg.step(scores_np, seed=100 + i)
         if i >= args.warmup:
-            times.append(total)
-    ms = 1e3 * sum(times) / len(times)
-    positions = sum(wl.seq_lens)
-    value = positions / (ms * 1e-3)
-    sample = (f"per step {ns} sampled rows scored by the oracle, extrapolated linearly to "
-              f"{positions} rows (per-call fixed cost {fixed:.1f} s counted once), + full "
-              f"select and compaction")
+            measured.append(m)
+            extrap.append(total)
+    ms = 1e3 * sum(measured) / len(measured)
+    ex_ms = 1e3 * sum(extrap) / len(extrap)
+    positions = leg.positions
+    value = positions / (ex_ms * 1e-3)
     return {"impl": "reference", "metric": "scored KV positions/sec per refresh",
             "value": round(value, 3), "unit": "positions/s", "n_gpus": dist.world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 2),
+            "ms_per_step_is": "measured wall time of one sampled step",
+            "extrapolated_ms_per_refresh": round(ex_ms, 1),
+            "value_basis": "positions / the extrapolated time of one whole refresh",
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic", "config": {"workload": wl.name, "score": args.score},
             "cpu_baseline": {"value": round(value, 3), "unit": "positions/s", "cores": cores_used(),
-                             "kind": "oracle", "sample": sample},
+                             "kind": "oracle", "extrapolated": True,
+                             "sample_s": round(ms / 1e3, 2), "sample": leg.describe(d)},
             "e2e": {"value": round(value, 3), "unit": "positions/s", "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
 
@@ -1030,9 +1301,13 @@ def main():
     ap.add_argument("--score", choices=["logit", "logprob"], default="logit")
     ap.add_argument("--single-cycle", action="store_true",
                     help="time only the first refresh of a multi-cycle workload")
-    ap.add_argument("--cpu-rows", type=int, default=256)
-    ap.add_argument("--ref-rows", type=int, default=32)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--precise", action="store_true",
+                    help="time the precise mode (CC_SCORE_PRECISE) as the headline")
+    ap.add_argument("--no-records", action="store_true",
+                    help="only the named workload (no precise-mode and other-workload records)")
+    ap.add_argument("--synthetic-cache", action="store_true",
+                    help="draw the cache directly instead of building it by a causal pass")
     ap.add_argument("--kv-fp8", action="store_true",
                     help="store the cache's K/V as e4m3 codes with per-layer scales")
     ap.add_argument("--batch", type=int, default=1,
@@ -1066,7 +1341,7 @@ def main():
         elif args.decode:
             line = run_decode(args, dist)
         else:
-            line = run_ours(args, dist)
+            line = run_suite(args, dist)
         if dist.rank == 0 and line is not None:
             print(json.dumps(line), flush=True)
     finally:

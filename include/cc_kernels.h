@@ -33,6 +33,20 @@ cc_status cc_counter_causal_attention(const void *q, const void *k, const void *
                                       int32_t cap, int32_t n_q_heads, int32_t n_kv_heads,
                                       int32_t head_dim, void *stream);
 
+/* The same counter-causal attention (Sec. 3.1, Eq. 2) with the queries and
+ * the output carried as bf16 pairs hi + lo (hi = bf16(x), lo = bf16(x - hi),
+ * x to about 2^-17 relative): q and out rows are
+ * [hi: n_q_heads*head_dim | lo: n_q_heads*head_dim] bf16, so q and out are
+ * [batch*cap][2*n_q_heads][head_dim].  On the tensor cores
+ * S = q_hi k^T + q_lo k^T, and the probabilities enter P V as P_hi + P_lo.
+ * This is the attention of the precise scoring pass (CC_SCORE_PRECISE).
+ * k, v, seq_len and the shape rules are those of cc_counter_causal_attention;
+ * rows i >= seq_len[b] of out are not written. */
+cc_status cc_counter_causal_attention_split(const void *q, const void *k, const void *v,
+                                            const int32_t *seq_len, void *out, int32_t batch,
+                                            int32_t cap, int32_t n_q_heads, int32_t n_kv_heads,
+                                            int32_t head_dim, void *stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -130,6 +130,8 @@ _SIGS = {
                                      ctypes.c_void_p]),
     "cc_counter_causal_attention": (ctypes.c_int, [ctypes.c_void_p] * 5 + [ctypes.c_int32] * 5
                                     + [ctypes.c_void_p]),
+    "cc_counter_causal_attention_split": (ctypes.c_int, [ctypes.c_void_p] * 5
+                                          + [ctypes.c_int32] * 5 + [ctypes.c_void_p]),
     "cc_timing_enable": (ctypes.c_int, [ctypes.c_int32]),
     "cc_timing_collect": (ctypes.c_int, [ctypes.POINTER(ctypes.c_int32),
                                          ctypes.POINTER(ctypes.c_double)]),
@@ -448,6 +450,14 @@ def cc_counter_causal_attention(q, k, v, seq_len, out, batch, cap, n_q_heads, n_
         _dev_ptr(q, "q"), _dev_ptr(k, "k"), _dev_ptr(v, "v"), _dev_ptr(seq_len, "seq_len"),
         _dev_ptr(out, "out"), batch, cap, n_q_heads, n_kv_heads, head_dim, _stream(stream))
     _check(code, "cc_counter_causal_attention")
+
+
+def cc_counter_causal_attention_split(q, k, v, seq_len, out, batch, cap, n_q_heads, n_kv_heads,
+                                      head_dim, stream=None):
+    code = load_library().cc_counter_causal_attention_split(
+        _dev_ptr(q, "q"), _dev_ptr(k, "k"), _dev_ptr(v, "v"), _dev_ptr(seq_len, "seq_len"),
+        _dev_ptr(out, "out"), batch, cap, n_q_heads, n_kv_heads, head_dim, _stream(stream))
+    _check(code, "cc_counter_causal_attention_split")
 
 
 def cc_timing_enable(on: bool):

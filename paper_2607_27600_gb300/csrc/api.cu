@@ -241,18 +241,18 @@ struct ScoreWs {
 // Per-tile progress flags of split-K GEMMs (at most one wave of tiles split).
 constexpr int kSplitFlags = 1024;
 
-// With CC_SCORE_PRECISE the full pass carries the GEMM activations
-// (normalised inputs, attention output, SwiGLU output) as [hi | lo] bf16
-// pairs: split = 2 copies per row.
-ScoreWs score_layout(const cc_model_cfg *c, int batch, int cap, cc_score_mode mode, bool full) {
+// With CC_SCORE_PRECISE either pass carries the GEMM activations
+// (normalised inputs, attention output, SwiGLU output) and the queries as
+// [hi | lo] bf16 pairs: split = 2 copies per row.
+ScoreWs score_layout(const cc_model_cfg *c, int batch, int cap, cc_score_mode mode, bool split_rows) {
   ScoreWs w{};
   const size_t R = (size_t)batch * cap;
   const size_t d = c->d_model, qd = (size_t)c->n_q_heads * c->head_dim, f = c->d_ff;
-  const size_t split = full ? 2 : 1;
+  const size_t split = split_rows ? 2 : 1;
   size_t off = 0;
   auto take = [&](size_t bytes) { size_t o = off; off = align256(off + bytes); return o; };
   w.xn = take(R * d * 2 * split);
-  w.q = take(R * qd * 2);
+  w.q = take(R * qd * 2 * split);
   w.o = take(R * qd * 2 * split);
   w.h = take(R * d * 4);
   w.act = take(R * f * 2 * split);
@@ -490,14 +490,17 @@ cc_status run_attention(const cc_model_cfg *c, const void *q, const void *k, con
                         void *out, const int32_t *seq_len, int batch, int cap, unsigned *status,
                         cudaStream_t st, bool split = false, const int32_t *row_lo = nullptr,
                         int q_span = 0, const AttnPartials *parts = nullptr, int sms = 0,
-                        KvFmt kvf = KvFmt()) {
+                        KvFmt kvf = KvFmt(), bool q_split = false) {
   const int G = c->n_q_heads / c->n_kv_heads, dh = c->head_dim;
   const int P = attn_positions_per_unit(G);
   const uint64_t R = (uint64_t)batch * cap;
+  if (q_split && (row_lo || kvf.fp8)) return CC_ERR_UNSUPPORTED;
   CUtensorMap tq, tk, tv;
   {
-    const uint64_t dims[3] = {(uint64_t)dh, (uint64_t)c->n_q_heads, R};
-    const uint64_t strides[2] = {(uint64_t)dh * 2, (uint64_t)c->n_q_heads * dh * 2};
+    // q_split: rows [hi heads | lo heads], the map spans both (lo at head Hq + t)
+    const uint64_t qh = (uint64_t)c->n_q_heads * (q_split ? 2 : 1);
+    const uint64_t dims[3] = {(uint64_t)dh, qh, R};
+    const uint64_t strides[2] = {(uint64_t)dh * 2, qh * dh * 2};
     const uint32_t box[3] = {64, (uint32_t)G, (uint32_t)P};
     if (!make_tmap(&tq, q, 3, dims, strides, box)) return tmap_fail();
   }
@@ -536,6 +539,7 @@ cc_status run_attention(const cc_model_cfg *c, const void *q, const void *k, con
   p.out = reinterpret_cast<__nv_bfloat16 *>(out);
   p.out_ld = c->n_q_heads * dh * (split ? 2 : 1);
   p.out_lo = split ? c->n_q_heads * dh : 0;
+  p.q_split = q_split ? 1 : 0;
   // e4m3 cache: S = Q . (codes * k_scale), so the K scale joins the softmax
   // scale; O = v_scale * P . codes, applied with the normalisation
   p.scale_log2 = (float)(1.4426950408889634 / sqrt((double)dh) * kvf.k_scale);
@@ -894,7 +898,7 @@ cc_status check_score_args(const cc_model_cfg *c, const cc_model_weights *w, con
   const void *ptrs[] = {w->final_norm, w->lm_head, ws, kv->h_last, full ? w->embed : nullptr};
   for (const void *p : ptrs)
     if (p && !aligned16(p)) return CC_ERR_INVALID_ARG;
-  if (!ws || ws_bytes < score_layout(c, kv->batch, kv->cap, mode, full && (mode & CC_SCORE_PRECISE)).total)
+  if (!ws || ws_bytes < score_layout(c, kv->batch, kv->cap, mode, (mode & CC_SCORE_PRECISE) != 0).total)
     return CC_ERR_WORKSPACE;
   return CC_OK;
 }
@@ -909,7 +913,10 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   const int batch = kv->batch, cap = kv->cap, rows = batch * cap;
   const int d = c->d_model, qd = c->n_q_heads * c->head_dim, f = c->d_ff;
-  const bool split = full && (mode & CC_SCORE_PRECISE);   // [hi | lo] GEMM activations
+  const bool split = (mode & CC_SCORE_PRECISE) != 0;   // [hi | lo] GEMM activations
+  // [hi | lo] queries and attention probabilities too (a bf16 cache; with an
+  // e4m3 cache the attention's operands are f16 and the queries stay single)
+  const bool split_q = split && kv->kv_format != CC_KV_E4M3;
   const ScoreWs L = score_layout(c, batch, cap, mode, split);
   const bool logit = (mode & 0xFF) == CC_SCORE_LOGIT;
   uint8_t *wsb = reinterpret_cast<uint8_t *>(ws);
@@ -941,7 +948,8 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
                         split)) != CC_OK)
       return s;
     gq.p.out = q;
-    gq.p.ldo = qd;
+    gq.p.ldo = split_q ? 2 * qd : qd;
+    gq.p.out_split = split_q ? 1 : 0;
     gq.p.pos = kv->pos;
     gq.p.bias = reinterpret_cast<const __nv_bfloat16 *>(lw.bq);
     gq.p.head_dim = c->head_dim;
@@ -950,8 +958,7 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
     // O = counter-causal attention
     CC_TRY(wait_kv_ready(kv, l, l + 1, st));
     if ((s = run_attention(c, q, kv->k[l], kv->v[l], o, sl, batch, cap, status, st, split,
-                           nullptr, 0, nullptr, 0, kv_fmt(c, kv, l))) !=
-        CC_OK)
+                           nullptr, 0, nullptr, 0, kv_fmt(c, kv, l), split_q)) != CC_OK)
       return s;
     // h = h + O Wo^T  (fast mode: h = H^(L-1) + O Wo^T)
     Gemm go;
@@ -1437,10 +1444,10 @@ cc_status cc_linear_f32(const void *x, const void *w, float *y, int32_t rows, in
   return run_gemm(g, EPI_F32, CC_KERNEL_OTHER, dev->sms, reinterpret_cast<cudaStream_t>(stream));
 }
 
-cc_status cc_counter_causal_attention(const void *q, const void *k, const void *v,
-                                      const int32_t *seq_len, void *out, int32_t batch,
-                                      int32_t cap, int32_t n_q_heads, int32_t n_kv_heads,
-                                      int32_t head_dim, void *stream) {
+static cc_status attention_entry(const void *q, const void *k, const void *v,
+                                 const int32_t *seq_len, void *out, int32_t batch, int32_t cap,
+                                 int32_t n_q_heads, int32_t n_kv_heads, int32_t head_dim,
+                                 void *stream, bool split) {
   if (!q || !k || !v || !seq_len || !out || batch < 1 || cap < 1 || n_q_heads < 1 ||
       n_kv_heads < 1 || n_q_heads % n_kv_heads)
     return CC_ERR_INVALID_ARG;
@@ -1455,7 +1462,24 @@ cc_status cc_counter_causal_attention(const void *q, const void *k, const void *
   c.n_kv_heads = n_kv_heads;
   c.head_dim = head_dim;
   return run_attention(&c, q, k, v, out, seq_len, batch, cap, dev->status,
-                       reinterpret_cast<cudaStream_t>(stream));
+                       reinterpret_cast<cudaStream_t>(stream), split, nullptr, 0, nullptr, 0,
+                       KvFmt(), split);
+}
+
+cc_status cc_counter_causal_attention(const void *q, const void *k, const void *v,
+                                      const int32_t *seq_len, void *out, int32_t batch,
+                                      int32_t cap, int32_t n_q_heads, int32_t n_kv_heads,
+                                      int32_t head_dim, void *stream) {
+  return attention_entry(q, k, v, seq_len, out, batch, cap, n_q_heads, n_kv_heads, head_dim,
+                         stream, false);
+}
+
+cc_status cc_counter_causal_attention_split(const void *q, const void *k, const void *v,
+                                            const int32_t *seq_len, void *out, int32_t batch,
+                                            int32_t cap, int32_t n_q_heads, int32_t n_kv_heads,
+                                            int32_t head_dim, void *stream) {
+  return attention_entry(q, k, v, seq_len, out, batch, cap, n_q_heads, n_kv_heads, head_dim,
+                         stream, true);
 }
 
 // ---- captured call sequences ------------------------------------------------

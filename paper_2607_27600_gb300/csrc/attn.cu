@@ -20,6 +20,15 @@
 //                     P (bf16) written back over S in TMEM, final O / l
 //   warp 8            TMA producer (Q once; K and V tiles, 2 stages each);
 //                     zeroes V rows past the sequence end in the last tile
+//
+// SPLIT (the precise scoring pass over a bf16 cache): the queries arrive as
+// bf16 pairs hi + lo (hi = bf16(q), lo = bf16(q - hi)), so S = Q_hi K^T +
+// Q_lo K^T accumulates both products in TMEM, and P is handed to P V as the
+// pair P_hi (TMEM columns [0, 64) of the S block) + P_lo (columns [64, 128)),
+// two TS products into O.  K and V are exact bf16 inputs, so every operand of
+// both contractions then carries about 16 significant bits.  The second Q
+// tile costs 64 KB of shared memory at head_dim 128; the V ring then has one
+// stage.
 //   warp 9            TMEM owner + tcgen05.mma issuer:
 //                     S_h = Q_h K^T (SS),  O_h += P_h V (TS, P from TMEM)
 //   warps 10, 11      idle (complete the third warpgroup); with an e4m3 cache
@@ -58,11 +67,13 @@ CC_DEV float fast_exp2(float x) {
 }
 
 
-template <int DH, bool FP8 = false>
+template <int DH, bool FP8 = false, bool SPLIT = false>
 struct AttnSmem {
   static constexpr int NH = DH / 64;                 // 64-element (128-byte) column halves
   static constexpr int Q_BYTES = NH * 256 * 128;     // 256 rows
   static constexpr int KV_BYTES = NH * BKV * 128;    // one K (or V) tile (2-byte elements)
+  // V stages: one when the second (lo) Q tile of SPLIT leaves no room for two
+  static constexpr int KSTV = (SPLIT && DH == 128) ? 1 : KST;
   // FP8, head_dim 128: the fp8 tile lands in the upper half of its own f16
   // stage and is expanded in place (no staging); head_dim 64: one staging
   // buffer per K and V
@@ -70,11 +81,14 @@ struct AttnSmem {
   static constexpr int FP8_TILE = BKV * DH;            // bytes of one fp8 K (or V) tile
   static constexpr int STG_BYTES = (FP8 && !IN_PLACE) ? FP8_TILE : 0;
   static constexpr int OFF_Q = 0;
-  static constexpr int OFF_K = OFF_Q + Q_BYTES;
+  static constexpr int OFF_QLO = OFF_Q + Q_BYTES;          // SPLIT: the lo tile of Q
+  static constexpr int OFF_K = OFF_QLO + (SPLIT ? Q_BYTES : 0);
   static constexpr int OFF_V = OFF_K + KST * KV_BYTES;
-  static constexpr int OFF_STG = OFF_V + KST * KV_BYTES;   // [K, V] staging (FP8)
+  static constexpr int OFF_STG = OFF_V + KSTV * KV_BYTES;  // [K, V] staging (FP8)
   static constexpr int OFF_BAR = OFF_STG + 2 * STG_BYTES;
   static constexpr int BYTES = OFF_BAR + 256 + 1024;   // barriers + alignment slack
+  static_assert(BYTES <= 232448, "shared memory of a CTA exceeds 227 KB");
+  static_assert(!(SPLIT && FP8), "split queries take bf16 K/V operands");
 };
 
 // e4m3 pair (low 16 bits) -> f16 pair, exact; bf16 pair -> f16 pair; f16 pack.
@@ -124,11 +138,11 @@ CC_DEV UnitInfo decode_unit(const AttnParams &p, int unit_id, bool causal) {
   return u;
 }
 
-template <int DH, bool CAUSAL, bool FP8>
+template <int DH, bool CAUSAL, bool FP8, bool SPLIT>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                 const __grid_constant__ CUtensorMap tmV, const __grid_constant__ AttnParams p) {
-  using L = AttnSmem<DH, FP8>;
+  using L = AttnSmem<DH, FP8, SPLIT>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                               ~uintptr_t(1023));
@@ -244,9 +258,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     // them once so their S rows are exact zeros (finite, never NaN) and the
     // softmax can treat every row of a tile alike (no per-row mask path).
     if (G * P < 256) {
-      for (int hh = 0; hh < L::NH; ++hh)
-        for (int idx = G * P * 8 + lane; idx < 256 * 8; idx += 32)
-          reinterpret_cast<uint4 *>(smem + L::OFF_Q + hh * 256 * 128)[idx] = make_uint4(0, 0, 0, 0);
+      for (int qt = 0; qt < (SPLIT ? 2 : 1); ++qt)
+        for (int hh = 0; hh < L::NH; ++hh)
+          for (int idx = G * P * 8 + lane; idx < 256 * 8; idx += 32)
+            reinterpret_cast<uint4 *>(smem + L::OFF_Q + qt * L::Q_BYTES + hh * 256 * 128)[idx] =
+                make_uint4(0, 0, 0, 0);
       fence_proxy_async_smem();
       __syncwarp();
     }
@@ -254,10 +270,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       tma_prefetch_desc(&tmQ);
       tma_prefetch_desc(&tmK);
       tma_prefetch_desc(&tmV);
-      mbar_arrive_expect_tx(q_full, L::NH * 128 * G * P);
+      mbar_arrive_expect_tx(q_full, (SPLIT ? 2 : 1) * L::NH * 128 * G * P);
       for (int hh = 0; hh < L::NH; ++hh)
         tma_load_3d(smem + L::OFF_Q + hh * 256 * 128, &tmQ, q_full, hh * 64, g * G,
                     (int)row_base + p0);
+      if constexpr (SPLIT)   // lo heads follow the hi heads in each row
+        for (int hh = 0; hh < L::NH; ++hh)
+          tma_load_3d(smem + L::OFF_QLO + hh * 256 * 128, &tmQ, q_full, hh * 64,
+                      p.n_q_heads + g * G, (int)row_base + p0);
     }
     if constexpr (L::IN_PLACE) {
       // fp8 tiles into the upper half of their own stage (converted in place)
@@ -315,6 +335,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int it = 0; it < ntiles; ++it) {
         const int t = t_hi - it, s = it % KST;   // key tiles from the sequence end downwards
         const uint32_t ph = (it / KST) & 1;
+        const int sv = it % L::KSTV;             // V stage (one stage with SPLIT, head_dim 128)
+        const uint32_t phv = (it / L::KSTV) & 1;
         const int krow = tile_row(t);
         // TMA coordinates after the head_dim one: (KV head, row), or head-major (slot, b*Hkv + g)
         const int kc1 = p.pg.head_major ? t * BKV : g;
@@ -327,12 +349,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int hh = 0; hh < L::NH; ++hh)
               tma_load_3d(smem + L::OFF_K + s * L::KV_BYTES + hh * BKV * 128, &tmK, &k_full[s],
                           hh * 64, kc1, kc2);
-            ok = mbar_wait(&v_empty[s], ph ^ 1, abort_flag, p.status);
+            ok = mbar_wait(&v_empty[sv], phv ^ 1, abort_flag, p.status);
           }
           if (ok) {
-            mbar_arrive_expect_tx(&v_full[s], L::KV_BYTES);
+            mbar_arrive_expect_tx(&v_full[sv], L::KV_BYTES);
             for (int hh = 0; hh < L::NH; ++hh)
-              tma_load_3d(smem + L::OFF_V + s * L::KV_BYTES + hh * BKV * 128, &tmV, &v_full[s],
+              tma_load_3d(smem + L::OFF_V + sv * L::KV_BYTES + hh * BKV * 128, &tmV, &v_full[sv],
                           hh * 64, kc1, kc2);
           }
         }
@@ -341,9 +363,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (t == t_top && n - t * BKV < BKV) {
           // rows past the sequence end may hold any bits; P is 0 there, but
           // 0 * NaN would still poison O, so zero them before the PV product
-          if (!mbar_wait(&v_full[s], ph, abort_flag, p.status)) break;
+          if (!mbar_wait(&v_full[sv], phv, abort_flag, p.status)) break;
           const int first = n - t * BKV;
-          uint8_t *vs = smem + L::OFF_V + s * L::KV_BYTES;
+          uint8_t *vs = smem + L::OFF_V + sv * L::KV_BYTES;
           for (int hh = 0; hh < L::NH; ++hh)
             for (int idx = first * 8 + lane; idx < BKV * 8; idx += 32)
               reinterpret_cast<uint4 *>(vs + hh * BKV * 128)[idx] = make_uint4(0, 0, 0, 0);
@@ -365,28 +387,36 @@ __global__ void __launch_bounds__(kThreads, 1)
       // start-address field (16-byte units): +2 per 16 columns of a 128-byte
       // row (Q, K), +128 per 16 keys of V.  The issuing thread shares its SM
       // sub-partition with softmax warps, so each MMA costs a few instructions.
-      uint64_t qd[2][L::NH], kd[KST][L::NH], vd[KST];
-      const uint32_t q_s = smem_u32(smem + L::OFF_Q);
+      constexpr int NQ = SPLIT ? 2 : 1;   // Q tiles: hi (and lo)
+      uint64_t qd[NQ][2][L::NH], kd[KST][L::NH], vd[L::KSTV];
 #pragma unroll
-      for (int h = 0; h < 2; ++h)
+      for (int qt = 0; qt < NQ; ++qt)
 #pragma unroll
-        for (int hh = 0; hh < L::NH; ++hh)
-          qd[h][hh] = make_sdesc_sw128(q_s + hh * 256 * 128 + h * 128 * 128, 16, 1024);
+        for (int h = 0; h < 2; ++h)
 #pragma unroll
-      for (int st = 0; st < KST; ++st) {
+          for (int hh = 0; hh < L::NH; ++hh)
+            qd[qt][h][hh] = make_sdesc_sw128(smem_u32(smem + L::OFF_Q + qt * L::Q_BYTES) +
+                                                 hh * 256 * 128 + h * 128 * 128,
+                                             16, 1024);
+#pragma unroll
+      for (int st = 0; st < KST; ++st)
 #pragma unroll
         for (int hh = 0; hh < L::NH; ++hh)
           kd[st][hh] = make_sdesc_sw128(smem_u32(smem + L::OFF_K + st * L::KV_BYTES) + hh * BKV * 128,
                                         16, 1024);
+#pragma unroll
+      for (int st = 0; st < L::KSTV; ++st)
         vd[st] = make_sdesc_sw128(smem_u32(smem + L::OFF_V + st * L::KV_BYTES), BKV * 128, 1024);
-      }
       auto issue_qk = [&](int it, int h) {
         const int st = it % KST;
 #pragma unroll
-        for (int kk = 0; kk < DH / 16; ++kk) {
-          const int hh = kk >> 2, ko = (kk & 3) * 2;
-          umma_ss(tmem + h * 128, qd[h][hh] + ko, kd[st][hh] + ko, idesc_qk, kk > 0);
-        }
+        for (int qt = 0; qt < NQ; ++qt)   // SPLIT: S = Q_hi K^T + Q_lo K^T
+#pragma unroll
+          for (int kk = 0; kk < DH / 16; ++kk) {
+            const int hh = kk >> 2, ko = (kk & 3) * 2;
+            umma_ss(tmem + h * 128, qd[qt][h][hh] + ko, kd[st][hh] + ko, idesc_qk,
+                    (qt > 0 || kk > 0) ? 1u : 0u);
+          }
       };
       bool ok = mbar_wait(FP8 ? q_conv : q_full, 0, abort_flag, p.status);
       if (ok) ok = mbar_wait(&k_full[0], 0, abort_flag, p.status);
@@ -399,8 +429,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         umma_commit(&k_empty[0]);
       }
       for (int it = 0; ok && it < ntiles; ++it) {
-        const int t = t_hi - it, s = it % KST;
-        const uint32_t ph = (it / KST) & 1;
+        const int t = t_hi - it, s = it % L::KSTV;   // V stage
+        const uint32_t ph = (it / L::KSTV) & 1;
         if (!(ok = mbar_wait(&v_full[s], ph, abort_flag, p.status))) break;
         if (!FP8 && t == t_top && n - t * BKV < BKV)
           if (!(ok = mbar_wait(v_fixed, 0, abort_flag, p.status))) break;
@@ -408,12 +438,15 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (!(ok = mbar_wait(&p_ready[h], it & 1, abort_flag, p.status))) break;
           tc_fence_after();
 #pragma unroll
-          for (int kk = 0; kk < BKV / 16; ++kk) {
-            // B = V tile, MN-major: 64-column halves 16 KB apart (LBO),
-            // 8-key groups 1024 B apart (SBO); A = P_h, bf16 pairs in TMEM.
-            umma_ts(tmem + 256 + h * DH, tmem + h * 128 + kk * 8, vd[s] + kk * 128, idesc_pv,
-                    (it > 0 || kk > 0) ? 1u : 0u);
-          }
+          for (int pt = 0; pt < NQ; ++pt)   // SPLIT: O += P_hi V + P_lo V
+#pragma unroll
+            for (int kk = 0; kk < BKV / 16; ++kk) {
+              // B = V tile, MN-major: 64-column halves 16 KB apart (LBO),
+              // 8-key groups 1024 B apart (SBO); A = P_h, bf16 pairs in TMEM
+              // (P_lo 64 columns after P_hi).
+              umma_ts(tmem + 256 + h * DH, tmem + h * 128 + pt * 64 + kk * 8, vd[s] + kk * 128,
+                      idesc_pv, (it > 0 || kk > 0 || pt > 0) ? 1u : 0u);
+            }
           if (!ok) break;
           if (h == 1) umma_commit(&v_empty[s]);
           if (it + 1 < ntiles) {
@@ -603,15 +636,19 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
       for (int c0 = 0; c0 < 128; c0 += 32) {
         uint32_t pk[16];
+        [[maybe_unused]] uint32_t pl[16];
 #pragma unroll
         for (int k = 0; k < 32; k += 2) {
           const float2 y = __ffma2_rn(make_float2(__uint_as_float(sr[c0 + k]),
                                                   __uint_as_float(sr[c0 + k + 1])), sl2v, nmv);
           const float2 e = make_float2(fast_exp2(y.x), fast_exp2(y.y));
           pk[k / 2] = FP8 ? pack_f16x2(e.x, e.y) : pack_bf16x2(e.x, e.y);
+          if constexpr (SPLIT)   // P_lo = bf16(p - P_hi)
+            pl[k / 2] = pack_bf16x2(e.x - bf16_lo(pk[k / 2]), e.y - bf16_hi(pk[k / 2]));
           lsum = __fadd2_rn(lsum, e);
         }
         tmem_st16(s_t + c0 / 2, pk);
+        if constexpr (SPLIT) tmem_st16(s_t + 64 + c0 / 2, pl);
       }
       l += lsum.x + lsum.y;
       rescale();   // after P is written: S registers free for the O rows
@@ -740,16 +777,17 @@ __global__ void attn_combine_kernel(const __grid_constant__ AttnParams p) {
   if (p.out_lo > 0) dst[p.out_lo] = __float2bfloat16_rn(v - __bfloat162float(hi));
 }
 
-template <int DH, bool CAUSAL, bool FP8>
+template <int DH, bool CAUSAL, bool FP8, bool SPLIT = false>
 cudaError_t launch_dh(const CUtensorMap &q, const CUtensorMap &k, const CUtensorMap &v,
                       const AttnParams &p, cudaStream_t stream) {
-  auto kern = attn_kernel<DH, CAUSAL, FP8>;
+  using L = AttnSmem<DH, FP8, SPLIT>;
+  auto kern = attn_kernel<DH, CAUSAL, FP8, SPLIT>;
   static bool attr_set[64] = {};
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev < 64 && !attr_set[dev]) {
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         AttnSmem<DH, FP8>::BYTES);
+                                         L::BYTES);
     if (e != cudaSuccess) return e;
     attr_set[dev] = true;
   }
@@ -772,7 +810,7 @@ cudaError_t launch_dh(const CUtensorMap &q, const CUtensorMap &k, const CUtensor
   pp.streams_per_group = (int)fmax(1.0, fmin((double)n_streams, floor(sqrt(kReuseBytes / per_stream2))));
   const int S = pp.kv_splits > 1 ? pp.kv_splits : 1;
   if (S > 1 && (!pp.part_o || !pp.part_ml)) return cudaErrorInvalidValue;
-  kern<<<(unsigned)(units * S), kThreads, AttnSmem<DH, FP8>::BYTES, stream>>>(q, k, v, pp);
+  kern<<<(unsigned)(units * S), kThreads, L::BYTES, stream>>>(q, k, v, pp);
   if (S > 1) {
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
@@ -1090,6 +1128,10 @@ cudaError_t launch_attention(const CUtensorMap &q, const CUtensorMap &k, const C
     if (p.head_dim == 64)
       return f8 ? launch_dh<64, true, true>(q, k, v, p, stream)
                 : launch_dh<64, true, false>(q, k, v, p, stream);
+  } else if (p.q_split) {   // the precise scoring pass: bf16 cache only
+    if (f8) return cudaErrorInvalidValue;
+    if (p.head_dim == 128) return launch_dh<128, false, false, true>(q, k, v, p, stream);
+    if (p.head_dim == 64) return launch_dh<64, false, false, true>(q, k, v, p, stream);
   } else {
     if (p.head_dim == 128)
       return f8 ? launch_dh<128, false, true>(q, k, v, p, stream)

@@ -12,6 +12,9 @@ struct AttnParams {
   __nv_bfloat16 *out;       // row r, head t at out + r*out_ld + t*head_dim
   int out_ld;               // elements per output row (n_q_heads*head_dim, or twice that)
   int out_lo;               // > 0: also write lo = bf16(o - hi) at element offset out_lo
+  int q_split;              // counter-causal, bf16 cache: Q rows are [hi | lo] bf16 pairs
+                            // (the Q map spans 2 * n_q_heads heads, lo at head n_q_heads + t):
+                            // S = Q_hi K^T + Q_lo K^T, and P enters P V as hi + lo too
   float scale_log2;         // log2(e) / sqrt(head_dim)
   int streams_per_group;    // unit order (set by launch_attention): see attn.cu
   int causal;               // 0: counter-causal (rows [0, n) attend (i, n)); 1: causal over
@@ -38,7 +41,7 @@ int attn_positions_per_unit(int group);
 // per unit and split (kv_splits > 1).
 long long attn_units(const AttnParams &p);
 constexpr int kAttnPartRowFloats = 256;   // rows of a unit (times head_dim + 2 floats each)
-// q: 3-D map over Q [rows][Hq][dh], box {64, group, P}; k, v: 3-D maps over
+// q: 3-D map over Q [rows][Hq][dh] (q_split: [rows][2 Hq][dh]), box {64, group, P}; k, v: 3-D maps over
 // the cache [batch*cap][Hkv][dh], box {64, 1, 128}; all 128-byte swizzled.
 // With kv_fp8: k, v are byte maps over the e4m3 cache, box {dh, 1, 128},
 // unswizzled.

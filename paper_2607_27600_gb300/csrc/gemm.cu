@@ -57,10 +57,12 @@ CC_DEV uint8_t *out_at(const GemmParams &p, uint8_t *base, long long orow, int l
   return base + ((size_t)orow * ldo + c) * EB;
 }
 
+// lo_off > 0 (bf16 only): also the lo half of each value, bf16(y - hi), at
+// element offset lo_off of the row (the precise pass's [hi | lo] queries).
 template <int TBN, bool F8 = false>
 CC_DEV void rope_store(const GemmParams &p, uint32_t tacc, int grow, long long orow, bool valid,
                        void *out_base, int ldo, const __nv_bfloat16 *bias, int col0, int n_dest,
-                       float qscale = 1.f, bool hm = false) {
+                       float qscale = 1.f, bool hm = false, int lo_off = 0) {
   const int half = p.head_dim >> 1;
   valid = valid && orow >= 0;
   const uint32_t pos = valid ? (uint32_t)p.pos[grow] : 0u;
@@ -87,6 +89,7 @@ CC_DEV void rope_store(const GemmParams &p, uint32_t tacc, int grow, long long o
         bb2[v * 4] = u2.x; bb2[v * 4 + 1] = u2.y; bb2[v * 4 + 2] = u2.z; bb2[v * 4 + 3] = u2.w;
       }
       uint32_t o1[16], o2[16];
+      [[maybe_unused]] uint32_t l1[16], l2[16];
 #pragma unroll
       for (int k = 0; k < 32; k += 2) {
         float c_a, s_a, c_b, s_b;
@@ -109,8 +112,12 @@ CC_DEV void rope_store(const GemmParams &p, uint32_t tacc, int grow, long long o
             o2[k / 4] |= e2 << 16;
           }
         } else {
-          o1[k / 2] = pack_bf16x2(a1 * c_a - a2 * s_a, b1 * c_b - b2 * s_b);
-          o2[k / 2] = pack_bf16x2(a2 * c_a + a1 * s_a, b2 * c_b + b1 * s_b);
+          const float y1a = a1 * c_a - a2 * s_a, y1b = b1 * c_b - b2 * s_b;
+          const float y2a = a2 * c_a + a1 * s_a, y2b = b2 * c_b + b1 * s_b;
+          o1[k / 2] = pack_bf16x2(y1a, y1b);
+          o2[k / 2] = pack_bf16x2(y2a, y2b);
+          l1[k / 2] = pack_bf16x2(y1a - bf16_lo(o1[k / 2]), y1b - bf16_hi(o1[k / 2]));
+          l2[k / 2] = pack_bf16x2(y2a - bf16_lo(o2[k / 2]), y2b - bf16_hi(o2[k / 2]));
         }
       }
       constexpr int EB = F8 ? 1 : 2;
@@ -120,6 +127,18 @@ CC_DEV void rope_store(const GemmParams &p, uint32_t tacc, int grow, long long o
       for (int v = 0; v < 2 * EB; ++v) {   // 32 elements: 64 bytes bf16, 32 e4m3
         d1[v] = make_uint4(o1[v * 4], o1[v * 4 + 1], o1[v * 4 + 2], o1[v * 4 + 3]);
         d2[v] = make_uint4(o2[v * 4], o2[v * 4 + 1], o2[v * 4 + 2], o2[v * 4 + 3]);
+      }
+      if constexpr (!F8) {
+        if (lo_off > 0) {
+          uint4 *e1 = reinterpret_cast<uint4 *>(out_at<EB>(p, base, orow, ldo, hm, grow, col + lo_off));
+          uint4 *e2 = reinterpret_cast<uint4 *>(
+              out_at<EB>(p, base, orow, ldo, hm, grow, col + half + lo_off));
+#pragma unroll
+          for (int v = 0; v < 4; ++v) {
+            e1[v] = make_uint4(l1[v * 4], l1[v * 4 + 1], l1[v * 4 + 2], l1[v * 4 + 3]);
+            e2[v] = make_uint4(l2[v * 4], l2[v * 4 + 1], l2[v * 4 + 2], l2[v * 4 + 3]);
+          }
+        }
       }
     }
   }
@@ -358,7 +377,8 @@ CC_DEV void epilogue_tile(const GemmParams &p, uint32_t tacc, int grow, bool val
       rope_store<TBN, true>(p, tacc, grow, orow, valid, p.out, p.ldo, p.bias, tile_n0, p.N,
                             p.k_qscale, hm);
     else
-      rope_store<TBN>(p, tacc, grow, orow, valid, p.out, p.ldo, p.bias, tile_n0, p.N, 1.f, hm);
+      rope_store<TBN>(p, tacc, grow, orow, valid, p.out, p.ldo, p.bias, tile_n0, p.N, 1.f, hm,
+                      p.out_split ? p.N : 0);
   } else if constexpr (EPI == EPI_BF16) {    // kv_fp8: the V rows of an e4m3 cache
     const long long orow = p.kv_dest ? cache_row(p, grow, valid) : grow;
     const bool hm = p.kv_dest && p.pg.head_major;

@@ -63,7 +63,8 @@ struct GemmParams {
                            // (B kept in L2, A streamed per group); 1 = groups of `group`
                            // row tiles stay resident (A kept, B streamed per group)
   int group;
-  int out_split;           // EPI_SWIGLU: out rows are [hi | lo], lo at column offset N
+  int out_split;           // EPI_SWIGLU, EPI_QROPE (not into the cache): out rows are
+                           // [hi | lo], lo at column offset N
   int k_splits;            // EPI_RESID_F32 / EPI_RESID_LOGIT only: K range split over
                            // k_splits work items per tile (< one wave of tiles); the splits
                            // add into out in order (EPI_RESID_LOGIT: the last one takes the

@@ -30,7 +30,7 @@ import hashlib
 
 import torch
 
-from .configs import ModelShape, Workload, WORKLOADS, HEADLINE  # noqa: F401
+from .configs import ModelShape, Workload, WORKLOADS, HEADLINE, RECORDS  # noqa: F401
 
 WEIGHT_STD = 0.02
 BIAS_STD = 0.5

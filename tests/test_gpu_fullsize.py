@@ -125,26 +125,28 @@ def test_fast_pass_logprob_full_size(pkg):
     assert check_rows(got, want, rows) < TOL
 
 
-# Tolerances of the 32-layer full pass, derived from the arithmetic (not the
-# stated 2e-2).  oracle/sensitivity.py re-runs the exact fp64 pass of a random
-# Llama-3-8B-shaped model (n = 16384, 96 rows) with bf16 rounding at chosen
-# points: rounding only the queries entering QK^T moves the score by up to
-# 5.5 % (max over rows and layers); every rounding point of a bf16
-# tensor-core pass (GEMM inputs, queries, P, fp32 residual) by up to 8.9 %
-# (per-row quantiles after layer 31: 50 % 1.7 %, 90 % 5.0 %, 99 % 6.9 %).  The
-# GPU pass is another rounding sequence on another model instance, i.e.
-# another draw from that heavy-tailed spread, so each tolerance is about 1.7x
-# the matching emulated maximum: bf16 activations (default) against the
-# bf16-pass figure, hi + lo activations (CC_SCORE_PRECISE, bf16 queries left)
-# against the queries-only figure.  The full-pass machinery itself is held to
-# 2e-2 (relative l2 over 64 rows) on the first four layers of the same model
-# and shapes.
-FULL4_ROW_TOL = 8e-2       # worst single row, 4 layers (measured 3.9-4.1 % on 64 rows)
-FULL32_TOL = 1.5e-1        # bf16 activations, 32 layers
-FULL32_PRECISE_TOL = 1e-1  # hi + lo GEMM activations (CC_SCORE_PRECISE), 32 layers
-# The 28-layer Qwen2.5 pass at 512 slots: held to the 32-layer Llama bar (the
-# same rounding points; fewer layers and keys, so no larger drift expected).
-FULL28_TOL = FULL32_TOL
+# Two modes of the full pass (Sec. 3.1, all L layers with fresh queries).
+#
+# CC_SCORE_PRECISE carries every tensor-core operand that is not an exact bf16
+# input as a bf16 pair hi + lo: the GEMM activations, the queries entering
+# Q K^T and the probabilities entering P V (K, V and the weights are exact
+# bf16 inputs).  It is held to the stated bar: max relative error 2e-2 on
+# every sampled row.  tests/study_fullpass_precision.py emulates it in fp64
+# ("split-all": 3e-5 after the first layer, 6e-5 after eight of 32).
+#
+# The default mode keeps single bf16 activations, queries and P (what a bf16
+# model computes at inference, about half the precise mode's cost).  On this
+# deep random model its drift is a property of the arithmetic: the study's
+# "bf16-pass" rounding moves the score by up to 8.9 % (max over 96 rows and 32
+# layers; per-row quantiles after layer 31: 50 % 1.7 %, 90 % 5.0 %, 99 %
+# 6.9 %), so this mode's bars are derived from that spread and labelled as
+# such: about 1.7x the emulated maximum at 32 layers, and at 4 layers the
+# relative l2 error over the rows within 2e-2 with a worst-row cap.
+DEFAULT_FULL4_ROW_TOL = 8e-2   # default mode, worst single row at 4 layers (measured 3.9-4.1 %)
+DEFAULT_FULL32_TOL = 1.5e-1    # default mode, 32 layers
+# The 28-layer Qwen2.5 pass at 512 slots: the default mode held to the 32-layer
+# Llama bar (the same rounding points; fewer layers and keys).
+DEFAULT_FULL28_TOL = DEFAULT_FULL32_TOL
 
 
 def _full_inputs(n_layers):
@@ -156,36 +158,47 @@ def _full_inputs(n_layers):
     return wl, shape, w, c
 
 
+def _full_rows(n, count, seed):
+    """The edge rows (first, sequence end, the last slot's +inf) and seeded
+    others: `count` distinct rows in all."""
+    edge = {0, 5, n // 4 + 1, n // 2 - 1, n - 3, n - 2, n - 1}
+    r = np.random.default_rng(seed)
+    extra = r.choice(np.setdiff1d(np.arange(n), list(edge)), size=count - len(edge), replace=False)
+    return [sorted(edge | set(extra.tolist()))]
+
+
 def test_full_pass_llama_shape_first_4_layers(pkg):
-    """The full-pass machinery over four layers on 64 rows (the edge rows and
-    58 seeded ones).  Per-row errors of a bf16 pass are heavy-tailed (up to
-    ~4 % of the scores' rms here), so the bar of 2e-2 holds the relative l2
-    error over the rows (measured 1.2 %), and a bound of twice the measured
-    worst row catches a single row gone wrong."""
+    """The full-pass machinery over four layers of the Llama-3-8B shape on 64
+    rows: the precise mode within the stated 2e-2 on every row; the default
+    mode within 2e-2 relative l2 over the rows and its worst row within the
+    derived cap."""
     from paper_2607_27600_gb300 import cc
     wl, shape, w, c = _full_inputs(4)
-    got = gpu_scores(pkg, shape, w, c, cc.SCORE_LOGIT, full=True)
+    precise = gpu_scores(pkg, shape, w, c, cc.SCORE_LOGIT | cc.SCORE_PRECISE, full=True)
+    default = gpu_scores(pkg, shape, w, c, cc.SCORE_LOGIT, full=True)
     wn, cn = host_view(w, c, lazy=True)
-    extra = np.random.default_rng(5).integers(0, 16382, 58).tolist()
-    rows = [sorted(set([0, 5, 4097, 8191, 16381, 16382, 16383] + extra))]
+    rows = _full_rows(wl.seq_lens[0], 64, seed=5)
     want = oracle.score_full(shape, wn, cn, rows=rows)
-    g, o = got[0, rows[0]].astype(np.float64), want[0, rows[0]]
+    assert check_rows(precise, want, rows) < TOL
+    g, o = default[0, rows[0]].astype(np.float64), want[0, rows[0]]
     fin = np.isfinite(o)
     np.testing.assert_array_equal(g[~fin], o[~fin])
     assert np.linalg.norm(g[fin] - o[fin]) / np.linalg.norm(o[fin]) < TOL
-    assert check_rows(got, want, rows) < FULL4_ROW_TOL
+    assert check_rows(default, want, rows) < DEFAULT_FULL4_ROW_TOL
 
 
-@pytest.mark.parametrize("precise", [False, True])
-def test_full_pass_32_layers_sampled_rows(pkg, precise):
+def test_full_pass_32_layers_sampled_rows(pkg):
+    """llama8b-full-16k, all 32 layers, 64 rows: the precise mode within the
+    stated 2e-2 max relative error; the default mode within its derived bar."""
     from paper_2607_27600_gb300 import cc
     wl, shape, w, c = _full_inputs(32)
-    mode = cc.SCORE_LOGIT | (cc.SCORE_PRECISE if precise else 0)
-    got = gpu_scores(pkg, shape, w, c, mode, full=True)
+    precise = gpu_scores(pkg, shape, w, c, cc.SCORE_LOGIT | cc.SCORE_PRECISE, full=True)
+    default = gpu_scores(pkg, shape, w, c, cc.SCORE_LOGIT, full=True)
     wn, cn = host_view(w, c, lazy=True)
-    rows = [[0, 5, 8191, 16381, 16382, 16383]]
+    rows = _full_rows(wl.seq_lens[0], 64, seed=7)
     want = oracle.score_full(shape, wn, cn, rows=rows)
-    assert check_rows(got, want, rows) < (FULL32_PRECISE_TOL if precise else FULL32_TOL)
+    assert check_rows(precise, want, rows) < TOL
+    assert check_rows(default, want, rows) < DEFAULT_FULL32_TOL
 
 
 def test_headline_keep_set_full_oracle(pkg):
@@ -210,6 +223,41 @@ def test_headline_keep_set_full_oracle(pkg):
     assert np.array_equal(gc, oc) and np.array_equal(gi[0, :oc[0]], oi[0, :oc[0]])
     wi, wc = oracle.select_keep(want.astype(np.float32), wl.seq_lens, wl.budgets)
     ok, det = keep_set_ok(gi, gc, wi, wc, want, wl.seq_lens, wl.budgets)
+    assert ok, det
+
+
+def test_ragged_batch_keep_set_per_sequence_budget(pkg):
+    """llama8b-layer-32k-ragged (Algorithm DoMemRefresh per sequence, budgets
+    25 % of each length): the whole batch scored and selected on the GPU in
+    one call each, as bench.py times it; the 8192-slot sequence's keep-set
+    (budget 2048) checked against the oracle's scores of every one of its
+    rows: identical where the boundary gap exceeds the tolerance, else >= 99.5 %
+    overlap with near-tie swaps only; the other sequences' keep-sets equal the
+    oracle's select on the GPU's own scores."""
+    from paper_2607_27600_gb300 import cc
+    wl = synth.WORKLOADS["llama8b-layer-32k-ragged"]
+    w, c = workload_inputs(wl)
+    got = gpu_scores(pkg, wl.shape, w, c, cc.SCORE_LOGIT, full=False)
+    b, cap = c["tokens"].shape
+    idx = torch.empty(b, cap, dtype=torch.int32, device="cuda")
+    cnt = torch.empty(b, dtype=torch.int32, device="cuda")
+    cc.cc_select_keep(torch.from_numpy(got).cuda(), c["seq_len"], b, cap,
+                      torch.tensor(wl.budgets, dtype=torch.int32, device="cuda"), 0, idx, cnt)
+    assert cc.cc_get_status() == cc.CC_OK
+    gi, gc = idx.cpu().numpy(), cnt.cpu().numpy()
+    oi, oc = oracle.select_keep(got, wl.seq_lens, wl.budgets)
+    assert np.array_equal(gc, oc)
+    for s_ in range(b):
+        assert np.array_equal(gi[s_, :oc[s_]], oi[s_, :oc[s_]]), s_
+    seq = int(np.argmin(wl.seq_lens))               # the 8192-slot sequence
+    n = wl.seq_lens[seq]
+    wn, cn = host_view(w, c)
+    rows = [np.arange(n) if s_ == seq else np.array([], np.int64) for s_ in range(b)]
+    want = oracle.score_layer(wl.shape, wn, cn, rows=rows)
+    assert rel_err(got[seq, :n], want[seq, :n]) < TOL
+    wi, wc = oracle.select_keep(want[seq:seq + 1].astype(np.float32), [n], [wl.budgets[seq]])
+    ok, det = keep_set_ok(gi[seq:seq + 1], gc[seq:seq + 1], wi, wc, want[seq:seq + 1], [n],
+                          [wl.budgets[seq]])
     assert ok, det
 
 
@@ -269,8 +317,9 @@ def test_long_context_refresh_cycles(pkg):
 @pytest.mark.parametrize("name", ["qwen7b-table1-fast-4096", "qwen7b-table1-full-512"])
 def test_paper_table1_workloads(pkg, name):
     """The paper's efficiency benchmark shapes (Qwen2.5-7B, synthetic cache):
-    the fast pass at 4096 slots on every row, the full 28-layer pass at 512
-    slots on sampled rows, in the launch configuration bench.py times."""
+    the fast pass at 4096 slots on every row; the full 28-layer pass at 512
+    slots on 96 rows, the precise mode within the stated 2e-2 and the default
+    mode within its derived bar; in the launch configuration bench.py times."""
     from paper_2607_27600_gb300 import cc
     wl = synth.WORKLOADS[name]
     fast = wl.mode == "layer"
@@ -281,6 +330,8 @@ def test_paper_table1_workloads(pkg, name):
         want = oracle.score_layer(wl.shape, wn, cn)
         assert rel_err(got[0, :wl.seq_lens[0]], want[0, :wl.seq_lens[0]]) < TOL
     else:
-        rows = sample(wl.seq_lens, 10, seed=6)
+        precise = gpu_scores(pkg, wl.shape, w, c, cc.SCORE_LOGIT | cc.SCORE_PRECISE, full=True)
+        rows = _full_rows(wl.seq_lens[0], 96, seed=6)
         want = oracle.score_full(wl.shape, wn, cn, rows=rows)
-        assert check_rows(got, want, rows) < FULL28_TOL
+        assert check_rows(precise, want, rows) < TOL
+        assert check_rows(got, want, rows) < DEFAULT_FULL28_TOL

@@ -86,10 +86,11 @@ def test_decode_graph_replays_match_oracle(cc):
 
 
 def test_refresh_cycle_graph_over_two_cache_states(cc):
-    """Fast scoring, keep-set selection and compaction captured once, then
-    replayed over two different cache contents (lengths and budgets too)
-    copied into the same buffers: scores within tolerance, the keep-set
-    exact against the oracle's select on the replay's own scores, compaction
+    """Fast scoring (the precise mode), keep-set selection and compaction
+    captured once, then replayed over two different cache contents (lengths
+    and budgets too) copied into the same buffers: scores within tolerance,
+    the keep-set within the stated bar against the oracle's scores and exact
+    against the oracle's select on the replay's own scores, compaction
     bit-exact."""
     import paper_2607_27600_gb300 as pkg
     shape, cap = SMALL_GPU, 320
@@ -104,13 +105,14 @@ def test_refresh_cycle_graph_over_two_cache_states(cc):
     scores = torch.empty((b, cap), dtype=torch.float32, device="cuda")
     keep_idx = torch.empty((b, cap), dtype=torch.int32, device="cuda")
     keep_count = torch.empty(b, dtype=torch.int32, device="cuda")
-    sws = cc.alloc_workspace(cc.cc_score_workspace_size(shape, b, cap, cc.SCORE_LOGIT))
+    mode = cc.SCORE_LOGIT | cc.SCORE_PRECISE
+    sws = cc.alloc_workspace(cc.cc_score_workspace_size(shape, b, cap, mode))
     kws = cc.alloc_workspace(cc.cc_select_workspace_size(b, cap))
     cws = cc.alloc_workspace(cc.cc_compact_workspace_size(shape, cache))
     s = torch.cuda.Stream()
 
     def cycle():
-        cc.cc_score_layer(shape, weights, cache, cc.SCORE_LOGIT, scores, sws)
+        cc.cc_score_layer(shape, weights, cache, mode, scores, sws)
         cc.cc_select_keep(scores, c_dev["seq_len"], b, cap, budget, 0, keep_idx, keep_count, kws)
         cc.cc_compact_kv(shape, cache, keep_idx, keep_count, cws)
 

@@ -118,3 +118,63 @@ def test_attention_past_slots_do_not_leak(cc):
     torch.cuda.synchronize()
     assert torch.equal(o1[300:], o2[300:])
     assert not torch.equal(o1[:299], o2[:299])
+
+
+def _split_pair(x):
+    """fp64 -> bf16 pair (hi, lo) with hi = bf16(x), lo = bf16(x - hi)."""
+    hi = torch.from_numpy(np.asarray(x, np.float32)).to(torch.bfloat16)
+    lo = (torch.from_numpy(np.asarray(x, np.float64)) - hi.double()).float().to(torch.bfloat16)
+    return hi, lo
+
+
+@pytest.mark.parametrize("hq,hkv,dh,seq", [(32, 8, 128, [384, 301]), (8, 2, 64, [384, 1]),
+                                           (28, 4, 128, [129, 255]), (12, 2, 128, [2, 384]),
+                                           (10, 2, 64, [3, 200])])
+def test_attention_split_operands_match_oracle_tightly(cc, hq, hkv, dh, seq):
+    """The precise pass's attention: queries in as hi + lo, probabilities into
+    P V as hi + lo, output out as hi + lo.  With K and V exact bf16 inputs the
+    only roundings left are about 2^-17 relative (the pairs) and fp32
+    arithmetic, so the output matches the oracle's fp64 attention of the same
+    queries within 1e-4 of its scale (a single bf16 operand would miss by
+    about 2^-9)."""
+    batch, cap = len(seq), 384
+    q = synth.normal((batch * cap, hq, dh), 1.0, 50 + dh, "q").double().numpy()
+    q = q * (1 + 1e-3 * synth.normal(q.shape, 1.0, 51, "qj").double().numpy())   # not bf16 values
+    k = synth.normal((batch, cap, hkv, dh), 1.5, 50 + dh, "k")
+    v = synth.normal((batch, cap, hkv, dh), 1.0, 50 + dh, "v")
+    qh, ql = _split_pair(q)
+    qpair = torch.cat([qh, ql], dim=1).cuda()                 # [rows][2 hq][dh]
+    out = torch.full((batch * cap, 2 * hq, dh), float("nan"), dtype=torch.bfloat16, device="cuda")
+    sl = torch.tensor(seq, dtype=torch.int32, device="cuda")
+    cc.cc_counter_causal_attention_split(qpair, k.cuda(), v.cuda(), sl, out, batch, cap, hq, hkv,
+                                         dh)
+    assert cc.cc_get_status() == cc.CC_OK
+    o = out.double().cpu()
+    got = (o[:, :hq] + o[:, hq:]).numpy().reshape(batch, cap, hq, dh)
+    qx = (qh.double() + ql.double()).numpy().reshape(batch, cap, hq, dh)   # the value the pair holds
+    kn, vn = k.float().numpy(), v.float().numpy()
+    for b, n in enumerate(seq):
+        r = np.arange(n)
+        want = oracle.counter_causal_attention(qx[b, r], kn[b], vn[b], r, n)
+        err = np.abs(got[b, r] - want).max()
+        assert err <= 1e-4 * max(1.0, np.abs(want).max()), (b, n, err)
+        np.testing.assert_array_equal(got[b, n - 1], 0.0)
+
+
+def test_attention_split_needs_the_lo_halves(cc):
+    """Dropping the lo halves of the queries moves the output by the bf16
+    rounding of q (far beyond the split bar), so the kernel really reads them."""
+    batch, cap, hq, hkv, dh = 1, 256, 8, 2, 128
+    q = synth.normal((cap, hq, dh), 1.0, 60, "q").double().numpy() * (1 + 1e-3)
+    k = synth.normal((batch, cap, hkv, dh), 2.0, 60, "k").cuda()
+    v = synth.normal((batch, cap, hkv, dh), 1.0, 60, "v").cuda()
+    qh, ql = _split_pair(q)
+    sl = torch.tensor([cap], dtype=torch.int32, device="cuda")
+    outs = []
+    for lo in (ql, torch.zeros_like(ql)):
+        out = torch.zeros(cap, 2 * hq, dh, dtype=torch.bfloat16, device="cuda")
+        cc.cc_counter_causal_attention_split(torch.cat([qh, lo], dim=1).cuda(), k, v, sl, out,
+                                             batch, cap, hq, hkv, dh)
+        torch.cuda.synchronize()
+        outs.append((out[:, :hq].double() + out[:, hq:].double()).cpu())
+    assert (outs[0] - outs[1]).abs().max().item() > 1e-3
