@@ -20,6 +20,17 @@
 //                     P (bf16) written back over S in TMEM, final O / l
 //   warp 8            TMA producer (Q once; K and V tiles, 2 stages each);
 //                     zeroes V rows past the sequence end in the last tile
+//   warp 9            TMEM owner + tcgen05.mma issuer of M-half 0:
+//                     S_h = Q_h K^T (SS),  O_h += P_h V (TS, P from TMEM)
+//   warp 10           tcgen05.mma issuer of M-half 1
+//   warp 11           idle (completes the third warpgroup)
+//
+// With an e4m3 cache (FP8) warp 9 issues both halves' products and warps 10
+// and 11 convert: Q bf16 -> f16 once, then every K and V tile from the fp8
+// staging buffer (TMA, unswizzled) into the 128-byte-swizzled f16 stage the
+// MMA reads, zeroing V rows past the sequence end; the MMAs then run on f16
+// operands (Q, K, V and P all f16: e4m3 -> f16 is exact), the K scale folded
+// into the softmax scale and the V scale into the output normalisation.
 //
 // SPLIT (the precise scoring pass over a bf16 cache): the queries arrive as
 // bf16 pairs hi + lo (hi = bf16(q), lo = bf16(q - hi)), so S = Q_hi K^T +
@@ -29,16 +40,6 @@
 // both contractions then carries about 16 significant bits.  The second Q
 // tile costs 64 KB of shared memory at head_dim 128; the V ring then has one
 // stage.
-//   warp 9            TMEM owner + tcgen05.mma issuer:
-//                     S_h = Q_h K^T (SS),  O_h += P_h V (TS, P from TMEM)
-//   warps 10, 11      idle (complete the third warpgroup); with an e4m3 cache
-//                     (FP8) they convert: Q bf16 -> f16 once, then every K and
-//                     V tile from the fp8 staging buffer (TMA, unswizzled) into
-//                     the 128-byte-swizzled f16 stage the MMA reads, zeroing V
-//                     rows past the sequence end; the MMAs then run on f16
-//                     operands (Q, K, V and P all f16: e4m3 -> f16 is exact),
-//                     the K scale folded into the softmax scale and the V
-//                     scale into the output normalisation
 //
 // TMEM columns: S0 [0,128)  S1 [128,256)  O0 [256,256+DH)  O1 [256+DH, 256+2DH)
 #include "attn.cuh"
@@ -143,6 +144,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                 const __grid_constant__ CUtensorMap tmV, const __grid_constant__ AttnParams p) {
   using L = AttnSmem<DH, FP8, SPLIT>;
+  constexpr bool kTwoIssuers = !FP8;   // warp 10 issues half 1's products (FP8: it converts)
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                               ~uintptr_t(1023));
@@ -161,7 +163,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t *q_conv = stg_empty + 2;        // FP8: Q converted to f16
   uint64_t *k_load = q_conv + 1;           // [KST] FP8 in place: fp8 K tile in stage s
   uint64_t *v_load = k_load + KST;         // [KST] FP8 in place: fp8 V tile in stage s
-  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(v_load + KST);
+  uint64_t *turn = v_load + KST;           // [2] two issuers: issuer h may issue its next burst
+  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(turn + 2);
   volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -221,9 +224,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(q_full, 1);
     for (int s = 0; s < KST; ++s) {   // FP8: K/V stages are filled by the 64 converter threads
       mbar_init(&k_full[s], FP8 ? 64 : 1);
-      mbar_init(&k_empty[s], 1);
+      mbar_init(&k_empty[s], kTwoIssuers ? 2 : 1);   // one commit per MMA issuer
       mbar_init(&v_full[s], FP8 ? 64 : 1);
-      mbar_init(&v_empty[s], 1);
+      mbar_init(&v_empty[s], kTwoIssuers ? 2 : 1);
     }
     mbar_init(v_fixed, 1);
     if (FP8) {
@@ -238,6 +241,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
     for (int h = 0; h < 2; ++h) {
+      mbar_init(&turn[h], 1);
       mbar_init(&s_ready[h], 1);
       mbar_init(&p_ready[h], 128);
       mbar_init(&o_done[h], 1);
@@ -375,9 +379,23 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
     }
-    } else if (warp == 9) {
-    // ------------------------------------------------------------ MMA issuer
+    } else if (warp == 9 || (kTwoIssuers && warp == 10)) {
+    // ------------------------------------------------------------ MMA issuers
+    // One issuing thread per M-half (warp 9: half 0, warp 10: half 1), or
+    // warp 9 for both halves with an e4m3 cache (warps 10-11 convert).  An
+    // issuing thread blocks while the tensor pipe's short queue is full, so a
+    // lone issuer leaves the pipe idle during its own barrier waits between
+    // bursts.  Two issuers take turns: a burst is one half's products for
+    // one key tile (PV(t, h) then QK(t+1, h)), bursts alternate half 0,
+    // half 1, half 0, ... (so the halves' softmaxes stay out of phase and
+    // each overlaps the other half's products), and each issuer does its own
+    // waits (P ready, K/V tiles) while the other one's burst runs; only the
+    // hand-over of the turn lies between bursts, covered by the products
+    // still queued.  Each half's products stay in one thread's program order
+    // (PV(t) before QK(t+1): P lives in S's columns), so every result is
+    // deterministic.
     if (lane == 0) {
+      const int h_lo = kTwoIssuers ? warp - 9 : 0, h_hi = kTwoIssuers ? warp - 9 : 1;
       // FP8: every operand (Q, K, V, P) is f16; otherwise every operand is bf16
       constexpr uint32_t idesc_qk =
           FP8 ? make_idesc_f16(128, BKV, 0, 0) : make_idesc_bf16(128, BKV, 0, 0);
@@ -385,8 +403,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           FP8 ? make_idesc_f16(128, DH, 0, 1) : make_idesc_bf16(128, DH, 0, 1);
       // Shared-memory descriptors built once; a K step only advances the
       // start-address field (16-byte units): +2 per 16 columns of a 128-byte
-      // row (Q, K), +128 per 16 keys of V.  The issuing thread shares its SM
-      // sub-partition with softmax warps, so each MMA costs a few instructions.
+      // row (Q, K), +128 per 16 keys of V.
       constexpr int NQ = SPLIT ? 2 : 1;   // Q tiles: hi (and lo)
       uint64_t qd[NQ][2][L::NH], kd[KST][L::NH], vd[L::KSTV];
 #pragma unroll
@@ -407,26 +424,45 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
       for (int st = 0; st < L::KSTV; ++st)
         vd[st] = make_sdesc_sw128(smem_u32(smem + L::OFF_V + st * L::KV_BYTES), BKV * 128, 1024);
-      auto issue_qk = [&](int it, int h) {
+      // pass_at >= 0: hand the turn over once that many products of the
+      // burst remain to be issued (the other issuer's wake-up then overlaps
+      // the products still queued)
+      auto issue_qk = [&](int it, int h, auto &&pass, int pass_at) {
         const int st = it % KST;
+        constexpr int kN = NQ * (DH / 16);
 #pragma unroll
         for (int qt = 0; qt < NQ; ++qt)   // SPLIT: S = Q_hi K^T + Q_lo K^T
 #pragma unroll
           for (int kk = 0; kk < DH / 16; ++kk) {
             const int hh = kk >> 2, ko = (kk & 3) * 2;
+            if (kN - (qt * (DH / 16) + kk) == pass_at) pass();
             umma_ss(tmem + h * 128, qd[qt][h][hh] + ko, kd[st][hh] + ko, idesc_qk,
                     (qt > 0 || kk > 0) ? 1u : 0u);
           }
       };
+      constexpr int kPassAt = 4;   // products left in a burst when the turn is handed over
+      // turns: this issuer's burst kb follows the other issuer's previous
+      // burst (half 0 opens; half 1's burst kb follows half 0's burst kb)
+      int kb = 0;
+      auto take_turn = [&]() -> bool {
+        if (!kTwoIssuers) return true;
+        if (h_lo == 0) return kb == 0 || mbar_wait(&turn[0], (kb - 1) & 1, abort_flag, p.status);
+        return mbar_wait(&turn[1], kb & 1, abort_flag, p.status);
+      };
+      auto pass_turn = [&]() {
+        if (kTwoIssuers) mbar_arrive(&turn[1 - h_lo]);
+        ++kb;
+      };
       bool ok = mbar_wait(FP8 ? q_conv : q_full, 0, abort_flag, p.status);
       if (ok) ok = mbar_wait(&k_full[0], 0, abort_flag, p.status);
+      if (ok) ok = take_turn();
       if (ok) {
         tc_fence_after();
-        issue_qk(0, 0);
-        umma_commit(&s_ready[0]);
-        issue_qk(0, 1);
-        umma_commit(&s_ready[1]);
-        umma_commit(&k_empty[0]);
+        for (int h = h_lo; h <= h_hi; ++h) {
+          issue_qk(0, h, pass_turn, h == h_hi ? kPassAt : -1);
+          umma_commit(&s_ready[h]);
+        }
+        umma_commit(&k_empty[0]);   // one arrival per issuer
       }
       for (int it = 0; ok && it < ntiles; ++it) {
         const int t = t_hi - it, s = it % L::KSTV;   // V stage
@@ -434,8 +470,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!(ok = mbar_wait(&v_full[s], ph, abort_flag, p.status))) break;
         if (!FP8 && t == t_top && n - t * BKV < BKV)
           if (!(ok = mbar_wait(v_fixed, 0, abort_flag, p.status))) break;
-        for (int h = 0; h < 2; ++h) {
+        for (int h = h_lo; h <= h_hi; ++h) {
           if (!(ok = mbar_wait(&p_ready[h], it & 1, abort_flag, p.status))) break;
+          const int s2 = (it + 1) % KST;   // the next key tile's stage
+          if (it + 1 < ntiles && h == h_lo)   // waited before the burst, not inside it
+            if (!(ok = mbar_wait(&k_full[s2], ((it + 1) / KST) & 1, abort_flag, p.status))) break;
+          if (!(ok = take_turn())) break;
           tc_fence_after();
 #pragma unroll
           for (int pt = 0; pt < NQ; ++pt)   // SPLIT: O += P_hi V + P_lo V
@@ -447,18 +487,14 @@ __global__ void __launch_bounds__(kThreads, 1)
               umma_ts(tmem + 256 + h * DH, tmem + h * 128 + pt * 64 + kk * 8, vd[s] + kk * 128,
                       idesc_pv, (it > 0 || kk > 0 || pt > 0) ? 1u : 0u);
             }
-          if (!ok) break;
-          if (h == 1) umma_commit(&v_empty[s]);
+          if (h == h_hi) umma_commit(&v_empty[s]);   // one arrival per issuer
           if (it + 1 < ntiles) {
-            const int s2 = (it + 1) % KST;
-            if (h == 0)
-              if (!(ok = mbar_wait(&k_full[s2], ((it + 1) / KST) & 1, abort_flag, p.status))) break;
-            tc_fence_after();
-            issue_qk(it + 1, h);
+            issue_qk(it + 1, h, pass_turn, kPassAt);
             umma_commit(&s_ready[h]);
-            if (h == 1) umma_commit(&k_empty[s2]);
+            if (h == h_hi) umma_commit(&k_empty[s2]);
           } else {
             umma_commit(&o_done[h]);
+            pass_turn();
           }
         }
       }
