@@ -440,7 +440,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     (qt > 0 || kk > 0) ? 1u : 0u);
           }
       };
-      constexpr int kPassAt = 4;   // products left in a burst when the turn is handed over
+      constexpr int kPassAt = 2;   // products left in a burst when the turn is handed over (1-3 measured alike; 6 and 8 slower)
       // turns: this issuer's burst kb follows the other issuer's previous
       // burst (half 0 opens; half 1's burst kb follows half 0's burst kb)
       int kb = 0;
