@@ -689,6 +689,11 @@ def run_suite(args, dist):
     dev = torch.device(f"cuda:{dist.local}")
     torch.cuda.set_device(dev)
     wl = synth.WORKLOADS[args.workload]
+    if args.layers:   # profiling: the same per-layer launches on a shallower model
+        import dataclasses
+        wl = dataclasses.replace(wl, name=f"{wl.name}[{args.layers} layers]",
+                                 shape=dataclasses.replace(wl.shape, n_layers=args.layers))
+        args.no_records = True
     mode = cc.SCORE_LOGPROB if args.score == "logprob" else cc.SCORE_LOGIT
     if args.precise:
         mode |= cc.SCORE_PRECISE
@@ -1308,6 +1313,9 @@ def main():
                     help="only the named workload (no precise-mode and other-workload records)")
     ap.add_argument("--synthetic-cache", action="store_true",
                     help="draw the cache directly instead of building it by a causal pass")
+    ap.add_argument("--layers", type=int, default=0,
+                    help="profiling only: truncate the model to this many layers (every "
+                         "launch keeps its full-size shape; the line is not a headline)")
     ap.add_argument("--kv-fp8", action="store_true",
                     help="store the cache's K/V as e4m3 codes with per-layer scales")
     ap.add_argument("--batch", type=int, default=1,
