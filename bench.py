@@ -382,6 +382,12 @@ def refresh_record(args, dist, wl, w, pristine, mode, steps, with_e2e=True, with
     score_fn = cc.cc_score_layer if fast else cc.cc_score_full
     stream = torch.cuda.current_stream(dev)
     scorer, recent = args.scorer, args.recent
+    row_shard = None
+    if args.shard == "rows" and scorer == "counter-causal":
+        # this rank's rows of one refresh, then the MAX all-reduce of the scores
+        from paper_2607_27600_gb300 import shard as shard_mod
+        row_shard = shard_mod.RowShard(shape, not fast, wl.seq_lens, dist.rank, dist.world,
+                                       device=dev)
     if scorer in ("importance", "h2o"):
         kws = cc.alloc_workspace(cc.cc_keyattn_workspace_size(shape, b, cap), dev)
     if scorer == "h2o":   # running totals, compacted with the cache
@@ -390,7 +396,10 @@ def refresh_record(args, dist, wl, w, pristine, mode, steps, with_e2e=True, with
         cws = cc.alloc_workspace(cc.cc_compact_workspace_size(shape, cache), dev)
 
     def score():
-        if scorer == "counter-causal":
+        if row_shard is not None:
+            row_shard.score(shape, weights, cache, mode, scores, ws)
+            shard_mod.merge_scores(scores)
+        elif scorer == "counter-causal":
             score_fn(shape, weights, cache, mode, scores, ws)
         elif scorer == "recency":
             cc.cc_score_recency(cache, scores)
@@ -473,7 +482,9 @@ def refresh_record(args, dist, wl, w, pristine, mode, steps, with_e2e=True, with
             "peak": peaks["bf16_tflops"] if d.get("bound") == "tensor" else peaks["hbm_gbs"],
             "unit": d.get("unit"), "frac": d.get("frac"), "traffic": traffic,
             "peak_source": f"{peak_src} ({'bf16 dense burst' if d.get('bound') == 'tensor' else 'HBM copy'})"}
-    value = positions * dist.world / (ms * 1e-3)
+    # replicas: every rank refreshes its own copy (weak scaling); row shards:
+    # the ranks share one refresh (strong scaling)
+    value = positions * (1 if row_shard is not None else dist.world) / (ms * 1e-3)
     rec = {
         "workload": wl.name, "value": round(value, 1), "unit": "positions/s",
         "ms_per_step": round(ms, 4), "steps": steps,
@@ -489,11 +500,15 @@ def refresh_record(args, dist, wl, w, pristine, mode, steps, with_e2e=True, with
         "gpu_launches": int(sum(c for c, _ in kernels.values())),
         "roofline": roof, "kernels": table, "clocks": clk,
     }
+    if row_shard is not None:
+        rec["shard"] = {"rows_this_rank": row_shard.rows(), "ranks": dist.world,
+                        "plan": "cc_partition_rows: contiguous blocks of equal estimated cost"}
     if precise:
         rec["roofline"]["note"] = ("algorithmic FLOPs of the pass; the precise mode issues each "
                                    "product once per operand half (about twice these FLOPs)")
     if e2e is not None:
-        rec["e2e"] = {"value": round(positions * dist.world / (e2e["ms"] * 1e-3), 1),
+        rec["e2e"] = {"value": round(positions * (1 if row_shard is not None else dist.world) /
+                                     (e2e["ms"] * 1e-3), 1),
                       "unit": "positions/s", "h2d_bytes_per_step": e2e["h2d"],
                       "d2h_bytes_per_step": e2e["d2h"], "ms_per_step": round(e2e["ms"], 4)}
     if (with_cpu and dist.world == 1 and not args.no_cpu_baseline and
@@ -734,7 +749,8 @@ def suite_line(args, dist, wl, head, cache_src, records):
         "metric": "scored KV positions/sec per refresh",
         "value": head["value"], "unit": "positions/s", "n_gpus": dist.world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": head.get("ms_per_step"),
-        "higher_is_better": True, "scaling": "weak", "vs_baseline": vs_baseline, "dtype": "bf16",
+        "higher_is_better": True, "scaling": "strong" if args.shard == "rows" else "weak",
+        "vs_baseline": vs_baseline, "dtype": "bf16",
         "data": f"synthetic (seeded random-init weights N(0,0.02); cache: {cache_src})",
         "config": {"workload": wl.name, "scorer": args.scorer,
                    "kv_cache": ("e4m3 (per-layer scales)" if args.kv_fp8 else "bf16") +
@@ -747,9 +763,11 @@ def suite_line(args, dist, wl, head, cache_src, records):
                    "d_ff": shape.d_ff, "vocab": shape.vocab,
                    "layers_compacted": shape.n_layers, "step_tflop": head.get("step_tflop"),
                    "l2": "cache restored + 256 MiB written between steps (outside the timed events)",
-                   "parallelism": f"replicas x{dist.world}"},
+                   "parallelism": (f"row shards x{dist.world} (one refresh split by query "
+                                   f"rows, MAX all-reduce of the scores)" if args.shard == "rows"
+                                   else f"replicas x{dist.world}")},
     }
-    for key in ("e2e", "gpu_launches", "roofline", "kernels", "tflops_per_step_achieved",
+    for key in ("shard", "e2e", "gpu_launches", "roofline", "kernels", "tflops_per_step_achieved",
                 "clocks", "cpu_baseline", "cycles", "value_basis"):
         if key in head:
             line[key] = head[key]
@@ -1313,6 +1331,9 @@ def main():
                     help="only the named workload (no precise-mode and other-workload records)")
     ap.add_argument("--synthetic-cache", action="store_true",
                     help="draw the cache directly instead of building it by a causal pass")
+    ap.add_argument("--shard", choices=["replicas", "rows"], default="replicas",
+                    help="N > 1: every rank refreshes its own replica (default), or the ranks "
+                         "split one refresh by query rows (cc_score_rows + a MAX all-reduce)")
     ap.add_argument("--layers", type=int, default=0,
                     help="profiling only: truncate the model to this many layers (every "
                          "launch keeps its full-size shape; the line is not a headline)")

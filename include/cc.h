@@ -216,6 +216,45 @@ cc_status cc_score_full(const cc_model_cfg *cfg, const cc_model_weights *w,
                         const cc_kv_cache *cache, cc_score_mode mode, float *scores,
                         void *ws, size_t ws_bytes, void *stream);
 
+/* ---- one refresh sharded over several GPUs by query rows ----------------------
+ * Given the cache, a row's score depends only on its own input (token or
+ * H^(L-1) row) and on the cached K/V of the later slots, which the pass
+ * reuses without recomputing them (Sec. 3.1); so the rows of one refresh
+ * can be split between processes that each hold the cache.
+ *
+ * cc_score_rows -- cc_score_layer (full = 0) or cc_score_full (full = 1)
+ * restricted to the rows row_lo[b] <= i < row_hi[b] of each sequence
+ * (row_lo, row_hi: device int32 [batch], 0 <= row_lo[b] <= row_hi[b] <=
+ * seq_len[b], else CC_ERR_DEVICE_ARG on the device and those rows skipped).
+ * Each row still attends every later slot up to seq_len[b].  Those rows get
+ * their scores (slot seq_len[b]-1 gets +inf when in range) and every other
+ * entry of scores [batch][cap] gets -inf, so the element-wise maximum of the
+ * ranks' buffers (one MAX all-reduce of batch * cap floats) is the whole
+ * refresh's scores.  A row's score is bit-identical to the one
+ * cc_score_layer / cc_score_full writes for it with the same cache and mode.
+ * Same workspace as those calls.  row_lo and row_hi must both be null (every
+ * row) or both be given. */
+cc_status cc_score_rows(const cc_model_cfg *cfg, const cc_model_weights *w,
+                        const cc_kv_cache *cache, cc_score_mode mode, int32_t full,
+                        const int32_t *row_lo, const int32_t *row_hi, float *scores, void *ws,
+                        size_t ws_bytes, void *stream);
+
+/* cc_partition_rows -- host-side plan: splits every sequence's rows [0,
+ * seq_len[b]) into `world` contiguous blocks, block r for rank r, of equal
+ * estimated cost.  A row's cost per layer is its projections' FLOPs (the
+ * same for every row) plus its attention's, which grows with the number of
+ * later slots, so the early rows cost more and get the shorter blocks.
+ * Interior boundaries are multiples of `align` (>= 1; 128 matches the row
+ * tiles of the projections).  seq_len: HOST int32 [batch]; row_lo, row_hi:
+ * HOST int32 [world][batch] written with rank r's block of sequence b at
+ * [r * batch + b].  The blocks of a sequence are disjoint, ascending and
+ * cover it exactly (a short sequence leaves some blocks empty).  Needs no
+ * GPU.  CC_ERR_INVALID_ARG on null pointers, world < 1, align < 1 or a
+ * negative length. */
+cc_status cc_partition_rows(const cc_model_cfg *cfg, int32_t full, const int32_t *seq_len,
+                            int32_t batch, int32_t world, int32_t align, int32_t *row_lo,
+                            int32_t *row_hi);
+
 /* ---- keep-set (Algorithm DoMemRefresh: sigma = argsort, keep sigma[1:J]) ---
  * For each sequence b keeps J_b = min(budget[b], seq_len[b]) slots: the
  * highest scores, ties broken toward the later slot, NaN ranked as -inf,

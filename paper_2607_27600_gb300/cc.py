@@ -26,7 +26,7 @@ STATUS_NAMES = {0: "CC_OK", 1: "CC_ERR_INVALID_ARG", 2: "CC_ERR_CUDA", 3: "CC_ER
                 7: "CC_ERR_DEVICE_ARG"}
 SCORE_LOGIT = 0
 SCORE_LOGPROB = 1
-SCORE_PRECISE = 0x100   # flag: hi + lo bf16 GEMM activations in the full pass
+SCORE_PRECISE = 0x100   # flag: hi + lo bf16 GEMM activations, queries and P (either pass)
 
 
 class CCError(RuntimeError):
@@ -81,6 +81,15 @@ _SIGS = {
     "cc_score_full": (ctypes.c_int, [ctypes.POINTER(cc_model_cfg), ctypes.POINTER(cc_model_weights),
                                      ctypes.POINTER(cc_kv_cache), ctypes.c_int, ctypes.c_void_p,
                                      ctypes.c_void_p, ctypes.c_size_t, ctypes.c_void_p]),
+    "cc_score_rows": (ctypes.c_int, [ctypes.POINTER(cc_model_cfg), ctypes.POINTER(cc_model_weights),
+                                     ctypes.POINTER(cc_kv_cache), ctypes.c_int, ctypes.c_int32,
+                                     ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,
+                                     ctypes.c_void_p, ctypes.c_size_t, ctypes.c_void_p]),
+    "cc_partition_rows": (ctypes.c_int, [ctypes.POINTER(cc_model_cfg), ctypes.c_int32,
+                                         ctypes.POINTER(ctypes.c_int32), ctypes.c_int32,
+                                         ctypes.c_int32, ctypes.c_int32,
+                                         ctypes.POINTER(ctypes.c_int32),
+                                         ctypes.POINTER(ctypes.c_int32)]),
     "cc_append_workspace_size": (ctypes.c_size_t, [ctypes.POINTER(cc_model_cfg), ctypes.c_int32,
                                                    ctypes.c_int32]),
     "cc_append_chunk": (ctypes.c_int, [ctypes.POINTER(cc_model_cfg), ctypes.POINTER(cc_model_weights),
@@ -315,6 +324,34 @@ def cc_score_layer(cfg, weights, cache, mode, scores, ws, stream=None):
 
 def cc_score_full(cfg, weights, cache, mode, scores, ws, stream=None):
     _score("cc_score_full", cfg, weights, cache, mode, scores, ws, stream)
+
+
+def cc_score_rows(cfg, weights, cache, mode, full: bool, row_lo, row_hi, scores, ws, stream=None):
+    """Scores only rows [row_lo[b], row_hi[b]) of each sequence (device int32
+    [batch] each, or both None for every row); every other entry of `scores`
+    gets -inf."""
+    code = load_library().cc_score_rows(
+        ctypes.byref(_cfg(cfg)), ctypes.byref(weights.c), ctypes.byref(cache.c), int(mode),
+        1 if full else 0, _dev_ptr(row_lo, "row_lo"), _dev_ptr(row_hi, "row_hi"),
+        _dev_ptr(scores, "scores"), _dev_ptr(ws, "ws"), ws.numel() * ws.element_size(),
+        _stream(stream))
+    _check(code, "cc_score_rows")
+
+
+def cc_partition_rows(cfg, full: bool, seq_lens, world: int, align: int = 128):
+    """Host-side plan of a refresh split over `world` ranks: returns
+    (row_lo, row_hi), int32 numpy [world][batch]; rank r scores rows
+    [row_lo[r][b], row_hi[r][b]) of sequence b.  Needs no GPU."""
+    import numpy as np
+    sl = np.ascontiguousarray(np.asarray(seq_lens, dtype=np.int32))
+    lo = np.zeros((world, sl.size), np.int32)
+    hi = np.zeros((world, sl.size), np.int32)
+    p32 = ctypes.POINTER(ctypes.c_int32)
+    code = load_library().cc_partition_rows(
+        ctypes.byref(_cfg(cfg)), 1 if full else 0, sl.ctypes.data_as(p32), int(sl.size),
+        int(world), int(align), lo.ctypes.data_as(p32), hi.ctypes.data_as(p32))
+    _check(code, "cc_partition_rows")
+    return lo, hi
 
 
 def cc_append_workspace_size(cfg, batch: int, cap: int) -> int:

@@ -490,7 +490,8 @@ cc_status run_attention(const cc_model_cfg *c, const void *q, const void *k, con
                         void *out, const int32_t *seq_len, int batch, int cap, unsigned *status,
                         cudaStream_t st, bool split = false, const int32_t *row_lo = nullptr,
                         int q_span = 0, const AttnPartials *parts = nullptr, int sms = 0,
-                        KvFmt kvf = KvFmt(), bool q_split = false) {
+                        KvFmt kvf = KvFmt(), bool q_split = false,
+                        const int32_t *range_lo = nullptr, const int32_t *range_hi = nullptr) {
   const int G = c->n_q_heads / c->n_kv_heads, dh = c->head_dim;
   const int P = attn_positions_per_unit(G);
   const uint64_t R = (uint64_t)batch * cap;
@@ -549,7 +550,9 @@ cc_status run_attention(const cc_model_cfg *c, const void *q, const void *k, con
   p.kv_rows = (int)RK;
   p.status = status;
   p.causal = row_lo ? 1 : 0;
-  p.row_lo = row_lo;
+  // counter-causal row range [range_lo, range_hi) (cc_score_rows); causal: row_lo
+  p.row_lo = row_lo ? row_lo : range_lo;
+  p.row_hi = row_lo ? nullptr : range_hi;
   p.q_span = row_lo ? q_span : cap;
   const long long units = attn_units(p);
   if (row_lo && q_span == 1 && G <= kDecMaxG && parts && parts->o && parts->ml &&
@@ -903,11 +906,16 @@ cc_status check_score_args(const cc_model_cfg *c, const cc_model_weights *w, con
   return CC_OK;
 }
 
+// rng_lo / rng_hi (device [batch], or both null): score only the rows
+// [rng_lo[b], rng_hi[b]) of each sequence, each attending every later slot;
+// every row kernel then visits those rows alone and the head writes only
+// their scores (cc_score_rows).
 cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_kv_cache *kv,
                     cc_score_mode mode, float *scores, void *ws, size_t ws_bytes, void *stream,
-                    bool full) {
+                    bool full, const int32_t *rng_lo = nullptr, const int32_t *rng_hi = nullptr) {
   cc_status s = check_score_args(c, w, kv, mode, scores, ws, ws_bytes, full);
   if (s != CC_OK) return s;
+  if ((rng_lo == nullptr) != (rng_hi == nullptr)) return CC_ERR_INVALID_ARG;
   DevState *dev;
   if (!dev_state(&dev)) return device_fail();
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
@@ -922,7 +930,9 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
   uint8_t *wsb = reinterpret_cast<uint8_t *>(ws);
   void *xn = wsb + L.xn, *q = wsb + L.q, *o = wsb + L.o, *act = wsb + L.act;
   float *h = reinterpret_cast<float *>(wsb + L.h);
-  const int32_t *sl = kv->seq_len;
+  // the row kernels' row ends (the range's, or the sequence ends); attention
+  // keys always run to the sequence end
+  const int32_t *sl = rng_hi ? rng_hi : kv->seq_len;
   unsigned *status = dev->status;
   unsigned *flags = reinterpret_cast<unsigned *>(wsb + L.flags);
   if ((s = clear_split_flags(flags, st)) != CC_OK) return s;
@@ -930,7 +940,7 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
 
   if (full) {
     TimedScope t(CC_KERNEL_EMBED, st);
-    CC_TRY(launch_embed(w->embed, kv->tokens, h, d, c->vocab, sl, cap, rows, status, st));
+    CC_TRY(launch_embed(w->embed, kv->tokens, h, d, c->vocab, sl, cap, rows, status, st, rng_lo));
   }
   const int l0 = full ? 0 : c->n_layers - 1;
   for (int l = l0; l < c->n_layers; ++l) {
@@ -940,13 +950,14 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
     {
       TimedScope t(CC_KERNEL_RMSNORM, st);
       CC_TRY(launch_rmsnorm(first_from_bf16 ? kv->h_last : (const void *)h, !first_from_bf16,
-                            lw.attn_norm, xn, d, c->rms_eps, sl, cap, rows, split, st));
+                            lw.attn_norm, xn, d, c->rms_eps, sl, cap, rows, split, st, rng_lo));
     }
     // Q = RoPE(xn Wq^T)
     Gemm gq;
     if ((s = gemm_setup(gq, EPI_QROPE, xn, d, lw.wq, nullptr, qd, batch, cap, sl, status,
                         split)) != CC_OK)
       return s;
+    gq.p.row_lo = rng_lo;
     gq.p.out = q;
     gq.p.ldo = split_q ? 2 * qd : qd;
     gq.p.out_split = split_q ? 1 : 0;
@@ -957,8 +968,9 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
     if ((s = run_gemm(gq, EPI_QROPE, CC_KERNEL_GEMM_QROPE, dev->sms, st)) != CC_OK) return s;
     // O = counter-causal attention
     CC_TRY(wait_kv_ready(kv, l, l + 1, st));
-    if ((s = run_attention(c, q, kv->k[l], kv->v[l], o, sl, batch, cap, status, st, split,
-                           nullptr, 0, nullptr, 0, kv_fmt(c, kv, l), split_q)) != CC_OK)
+    if ((s = run_attention(c, q, kv->k[l], kv->v[l], o, kv->seq_len, batch, cap, status, st,
+                           split, nullptr, 0, nullptr, 0, kv_fmt(c, kv, l), split_q, rng_lo,
+                           rng_hi)) != CC_OK)
       return s;
     // h = h + O Wo^T  (fast mode: h = H^(L-1) + O Wo^T)
     Gemm go;
@@ -966,6 +978,7 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
     if ((s = gemm_setup(go, epi_o, o, qd, lw.wo, nullptr, d, batch, cap, sl, status, split)) !=
         CC_OK)
       return s;
+    go.p.row_lo = rng_lo;
     go.p.out = h;
     go.p.ldo = d;
     go.p.resid = kv->h_last;
@@ -986,6 +999,7 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
     if ((s = gemm_setup(gu, EPI_SWIGLU, xn, d, lw.w_gate, lw.w_up, f, batch, cap, sl, status,
                         split)) != CC_OK)
       return s;
+    gu.p.row_lo = rng_lo;
     gu.p.out = act;
     gu.p.ldo = split ? 2 * f : f;
     gu.p.out_split = split ? 1 : 0;
@@ -1001,6 +1015,7 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
     if ((s = gemm_setup(gd, epi_d, act, f, lw.w_down, nullptr, d, batch, cap, sl, status,
                         split)) != CC_OK)
       return s;
+    gd.p.row_lo = rng_lo;
     gd.p.out = h;
     gd.p.ldo = d;
     if (epi_d == EPI_RESID_LOGIT) {
@@ -1018,12 +1033,13 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
   if (logit) {
     TimedScope t(CC_KERNEL_HEAD_LOGIT, st);
     CC_TRY(launch_head_logit(reinterpret_cast<const float2 *>(wsb + L.hpart), n_htiles,
-                             kv->tokens, scores, d, c->vocab, c->rms_eps, sl, cap, rows, status,
-                             st));
+                             kv->tokens, scores, d, c->vocab, c->rms_eps, kv->seq_len, cap, rows,
+                             status, st, rng_lo, rng_hi));
   } else {
     {
       TimedScope t(CC_KERNEL_RMSNORM, st);
-      CC_TRY(launch_rmsnorm(h, true, w->final_norm, xn, d, c->rms_eps, sl, cap, rows, split, st));
+      CC_TRY(launch_rmsnorm(h, true, w->final_norm, xn, d, c->rms_eps, sl, cap, rows, split, st,
+                            rng_lo));
     }
     Gemm gl;
     if ((s = gemm_setup(gl, EPI_LSE, xn, d, w->lm_head, nullptr, c->vocab, batch, cap, sl,
@@ -1031,13 +1047,15 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
       return s;
     float2 *part = reinterpret_cast<float2 *>(wsb + L.part);
     float *zt = reinterpret_cast<float *>(wsb + L.ztgt);
+    gl.p.row_lo = rng_lo;
     gl.p.out = part;
     gl.p.ldo = L.n_vtiles;
     gl.p.tokens = kv->tokens;
     gl.p.z_target = zt;
     if ((s = run_gemm(gl, EPI_LSE, CC_KERNEL_GEMM_LMHEAD, dev->sms, st)) != CC_OK) return s;
     TimedScope t(CC_KERNEL_LSE_COMBINE, st);
-    CC_TRY(launch_lse_combine(part, L.n_vtiles, zt, scores, sl, cap, rows, st));
+    CC_TRY(launch_lse_combine(part, L.n_vtiles, zt, scores, kv->seq_len, cap, rows, st, rng_lo,
+                              rng_hi));
   }
   return CC_OK;
 }
@@ -1342,6 +1360,55 @@ cc_status cc_score_full(const cc_model_cfg *cfg, const cc_model_weights *w,
                         const cc_kv_cache *cache, cc_score_mode mode, float *scores, void *ws,
                         size_t ws_bytes, void *stream) {
   return run_score(cfg, w, cache, mode, scores, ws, ws_bytes, stream, true);
+}
+
+cc_status cc_score_rows(const cc_model_cfg *cfg, const cc_model_weights *w,
+                        const cc_kv_cache *cache, cc_score_mode mode, int32_t full,
+                        const int32_t *row_lo, const int32_t *row_hi, float *scores, void *ws,
+                        size_t ws_bytes, void *stream) {
+  return run_score(cfg, w, cache, mode, scores, ws, ws_bytes, stream, full != 0, row_lo, row_hi);
+}
+
+cc_status cc_partition_rows(const cc_model_cfg *cfg, int32_t full, const int32_t *seq_len,
+                            int32_t batch, int32_t world, int32_t align, int32_t *row_lo,
+                            int32_t *row_hi) {
+  if (!cfg || !seq_len || !row_lo || !row_hi || batch < 1 || world < 1 || align < 1)
+    return CC_ERR_INVALID_ARG;
+  // the cost model needs positive sizes only (no kernel runs here)
+  if (cfg->d_model < 1 || cfg->n_q_heads < 1 || cfg->head_dim < 1 || cfg->d_ff < 1)
+    return CC_ERR_INVALID_ARG;
+  (void)full;   // every layer repeats the same per-row work: the split is the same
+  // per row and layer: projections 2 d (2 Hq dh) + 6 d F FLOPs, attention
+  // 4 dh Hq per later slot
+  const double g = 4.0 * cfg->d_model * (double)cfg->n_q_heads * cfg->head_dim +
+                   6.0 * cfg->d_model * (double)cfg->d_ff;
+  const double a = 4.0 * cfg->head_dim * (double)cfg->n_q_heads;
+  for (int b = 0; b < batch; ++b) {
+    const int64_t n = seq_len[b];
+    if (n < 0) return CC_ERR_INVALID_ARG;
+    // cost of rows [0, k): g k + a (k (n - 1) - k (k - 1) / 2), increasing in k
+    auto cost = [&](int64_t k) {
+      return g * k + a * ((double)k * (n - 1) - (double)k * (k - 1) / 2.0);
+    };
+    const double total = cost(n);
+    int64_t prev = 0;
+    for (int r = 0; r < world; ++r) {
+      int64_t hi = n;
+      if (r + 1 < world) {
+        const double target = total * (r + 1) / world;
+        int64_t lo_k = prev, hi_k = n;   // smallest k with cost(k) >= target
+        while (lo_k < hi_k) {
+          const int64_t mid = (lo_k + hi_k) / 2;
+          if (cost(mid) >= target) hi_k = mid; else lo_k = mid + 1;
+        }
+        hi = std::min<int64_t>(n, std::max<int64_t>(prev, (lo_k + align / 2) / align * align));
+      }
+      row_lo[(size_t)r * batch + b] = (int32_t)prev;
+      row_hi[(size_t)r * batch + b] = (int32_t)hi;
+      prev = hi;
+    }
+  }
+  return CC_OK;
 }
 
 size_t cc_select_workspace_size(int32_t batch, int32_t cap) {

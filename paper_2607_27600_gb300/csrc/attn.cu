@@ -106,6 +106,10 @@ CC_DEV uint32_t pack_f16x2(float lo, float hi) {
 CC_DEV uint32_t bf16x2_to_f16x2(uint32_t w) { return pack_f16x2(bf16_lo(w), bf16_hi(w)); }
 
 // Work unit `unit_id` -> (sequence b, KV head g, positions p0..p_last).
+// Counter-causal rows run over [row_lo, row_hi) when a range is given (keys
+// still up to the sequence end); a row's result does not depend on the range
+// (the extra key tiles of a unit that starts lower are fully masked for it
+// and add exact zeros).
 // Unit order: streams (sequence, KV head) in groups of streams_per_group;
 // within a group, position blocks outermost (longest units first), the
 // group's streams innermost.  The group size bounds how far apart in time
@@ -131,11 +135,13 @@ CC_DEV UnitInfo decode_unit(const AttnParams &p, int unit_id, bool causal) {
   u.b = stream / p.n_kv_heads;
   u.g = stream - u.b * p.n_kv_heads;
   u.n = p.seq_len[u.b];
-  u.q_lo = causal ? p.row_lo[u.b] : 0;
-  u.bad = u.n < 0 || u.n > p.cap || u.q_lo < 0 || u.q_lo > u.n;
+  u.q_lo = (causal || p.row_lo) ? p.row_lo[u.b] : 0;
+  // query rows end: the sequence end, or a counter-causal row range's end
+  const int q_hi = (!causal && p.row_hi) ? p.row_hi[u.b] : u.n;
+  u.bad = u.n < 0 || u.n > p.cap || u.q_lo < 0 || u.q_lo > q_hi || q_hi > u.n;
   u.p0 = u.q_lo + pb * p.P;
-  u.valid = !u.bad && u.p0 < u.n;
-  u.p_last = min(u.p0 + p.P, u.n) - 1;
+  u.valid = !u.bad && u.p0 < q_hi;
+  u.p_last = min(u.p0 + p.P, q_hi) - 1;
   return u;
 }
 

@@ -19,7 +19,12 @@ struct AttnParams {
   int streams_per_group;    // unit order (set by launch_attention): see attn.cu
   int causal;               // 0: counter-causal (rows [0, n) attend (i, n)); 1: causal over
                             // the memory (rows [row_lo, n) attend [0, i], inference cycle)
-  const int32_t *row_lo;    // causal: device [batch], first query slot of each sequence
+  const int32_t *row_lo;    // causal: device [batch], first query slot of each sequence;
+                            // counter-causal: null (rows from slot 0) or, with row_hi, the
+                            // first row of a range
+  const int32_t *row_hi;    // counter-causal: null (rows up to seq_len) or device [batch]:
+                            // only rows [row_lo, row_hi) are computed, each still attending
+                            // every later slot up to seq_len (cc_score_rows)
   int q_span;               // query slots per sequence at most (cap, or the chunk size)
   int kv_splits;            // > 1: each unit's key tiles split over kv_splits CTAs (few units)
   float *part_o;            // kv_splits > 1: [unit][split][256 rows][head_dim] unnormalised O

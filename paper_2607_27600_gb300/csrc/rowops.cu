@@ -20,6 +20,16 @@ CC_DEV bool row_valid(const int32_t *seq_len, int cap, int row, int &i, int &n) 
   return i < n && n <= cap;
 }
 
+// Scoring a row range (cc_score_rows): only slots [rng_lo[b], rng_hi[b])
+// are scored, every other slot gets -inf (so that the element-wise maximum of
+// the ranks' buffers assembles the whole refresh); without a range (rng_hi
+// null) every slot is scored.
+CC_DEV bool in_score_range(const int32_t *rng_lo, const int32_t *rng_hi, int cap, int row) {
+  if (!rng_hi) return true;
+  const int b = row / cap, i = row - b * cap;
+  return i >= rng_lo[b] && i < rng_hi[b];
+}
+
 // Row ranges of the inference cycle: slots [row_lo[b], seq_len[b]) (row_lo
 // may be null: from slot 0).
 CC_DEV bool row_in_range(const int32_t *seq_len, const int32_t *row_lo, int cap, int row) {
@@ -269,12 +279,13 @@ __global__ void argmax_combine_kernel(const float2 *part, int n_tiles, const int
 __global__ void __launch_bounds__(kWarps * 32)
     head_logit_kernel(const float2 *part, int n_tiles, const int32_t *tokens, float *scores,
                       int d, int vocab, float eps, const int32_t *seq_len, int cap, int rows,
-                      unsigned *status) {
+                      unsigned *status, const int32_t *rng_lo, const int32_t *rng_hi) {
   const int lane = threadIdx.x & 31;
   const int row = blockIdx.x * kWarps + (threadIdx.x >> 5);
   if (row >= rows) return;
   int i, n;
-  if (!row_valid(seq_len, cap, row, i, n)) {
+  // rows outside the range (another rank's) and past the sequence end: -inf
+  if (!in_score_range(rng_lo, rng_hi, cap, row) || !row_valid(seq_len, cap, row, i, n)) {
     if (lane == 0) scores[row] = -INFINITY;
     return;
   }
@@ -299,12 +310,14 @@ __global__ void __launch_bounds__(kWarps * 32)
 // score = -(z_target - logsumexp) from per-tile (max, sum exp) partials.
 __global__ void __launch_bounds__(kWarps * 32)
     lse_combine_kernel(const float2 *part, int n_tiles, const float *z_target, float *scores,
-                       const int32_t *seq_len, int cap, int rows) {
+                       const int32_t *seq_len, int cap, int rows, const int32_t *rng_lo,
+                       const int32_t *rng_hi) {
   const int lane = threadIdx.x & 31;
   const int row = blockIdx.x * kWarps + (threadIdx.x >> 5);
   if (row >= rows) return;
   int i, n;
-  if (!row_valid(seq_len, cap, row, i, n)) {
+  // rows outside the range (another rank's) and past the sequence end: -inf
+  if (!in_score_range(rng_lo, rng_hi, cap, row) || !row_valid(seq_len, cap, row, i, n)) {
     if (lane == 0) scores[row] = -INFINITY;
     return;
   }
@@ -389,20 +402,21 @@ cudaError_t launch_append_finish(int32_t *seq_len, const int32_t *row_hi, int ba
 
 cudaError_t launch_head_logit(const float2 *part, int n_tiles, const int32_t *tokens,
                               float *scores, int d, int vocab, float eps, const int32_t *seq_len,
-                              int cap, int rows, unsigned *status, cudaStream_t st) {
+                              int cap, int rows, unsigned *status, cudaStream_t st,
+                              const int32_t *rng_lo, const int32_t *rng_hi) {
   if (rows <= 0) return cudaSuccess;
   head_logit_kernel<<<blocks_for(rows), kWarps * 32, 0, st>>>(part, n_tiles, tokens, scores, d,
                                                              vocab, eps, seq_len, cap, rows,
-                                                             status);
+                                                             status, rng_lo, rng_hi);
   return cudaGetLastError();
 }
 
 cudaError_t launch_lse_combine(const float2 *part, int n_tiles, const float *z_target,
                                float *scores, const int32_t *seq_len, int cap, int rows,
-                               cudaStream_t st) {
+                               cudaStream_t st, const int32_t *rng_lo, const int32_t *rng_hi) {
   if (rows <= 0) return cudaSuccess;
   lse_combine_kernel<<<blocks_for(rows), kWarps * 32, 0, st>>>(part, n_tiles, z_target, scores,
-                                                              seq_len, cap, rows);
+                                                              seq_len, cap, rows, rng_lo, rng_hi);
   return cudaGetLastError();
 }
 
