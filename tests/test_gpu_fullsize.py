@@ -179,6 +179,8 @@ def test_full_pass_llama_shape_first_4_layers(pkg):
     wn, cn = host_view(w, c, lazy=True)
     rows = _full_rows(wl.seq_lens[0], 64, seed=5)
     want = oracle.score_full(shape, wn, cn, rows=rows)
+    print(f"4 layers, 64 rows: precise max {check_rows(precise, want, rows):.2e}, "
+          f"default max {check_rows(default, want, rows):.2e}")
     assert check_rows(precise, want, rows) < TOL
     g, o = default[0, rows[0]].astype(np.float64), want[0, rows[0]]
     fin = np.isfinite(o)
@@ -197,6 +199,8 @@ def test_full_pass_32_layers_sampled_rows(pkg):
     wn, cn = host_view(w, c, lazy=True)
     rows = _full_rows(wl.seq_lens[0], 64, seed=7)
     want = oracle.score_full(shape, wn, cn, rows=rows)
+    print(f"32 layers, 64 rows: precise max {check_rows(precise, want, rows):.2e}, "
+          f"default max {check_rows(default, want, rows):.2e}")
     assert check_rows(precise, want, rows) < TOL
     assert check_rows(default, want, rows) < DEFAULT_FULL32_TOL
 
@@ -333,5 +337,7 @@ def test_paper_table1_workloads(pkg, name):
         precise = gpu_scores(pkg, wl.shape, w, c, cc.SCORE_LOGIT | cc.SCORE_PRECISE, full=True)
         rows = _full_rows(wl.seq_lens[0], 96, seed=6)
         want = oracle.score_full(wl.shape, wn, cn, rows=rows)
+        print(f"28 layers, 96 rows: precise max {check_rows(precise, want, rows):.2e}, "
+              f"default max {check_rows(got, want, rows):.2e}")
         assert check_rows(precise, want, rows) < TOL
         assert check_rows(got, want, rows) < DEFAULT_FULL28_TOL
