@@ -807,7 +807,7 @@ def suite_line(args, dist, wl, head, cache_src, records):
 
 def read_traffic(kernel, workload):
     """DRAM bytes per launch from a committed ncu summary, when it matches the
-    current kernel sources; else None."""
+    current sources of that kernel; else None."""
     p = os.path.join(ROOT, "profiles", "dram_traffic.json")
     if not os.path.exists(p):
         return None
@@ -815,18 +815,32 @@ def read_traffic(kernel, workload):
         with open(p) as f:
             tbl = json.load(f)
         e = tbl.get(workload, {}).get(kernel)
-        if not e or e.get("csrc_sha") != csrc_digest():
+        if not e or e.get("sources_sha") != kernel_digest(kernel):
             return None
         return e.get("bytes_per_launch")
     except Exception:
         return None
 
 
-def csrc_digest():
+# the CUDA sources each kernel kind is built from (its own file, its header,
+# the shared PTX wrappers)
+KERNEL_SOURCES = {
+    "gemm": ["gemm.cu", "gemm.cuh", "cc_common.cuh"],
+    "attention": ["attn.cu", "attn.cuh", "cc_common.cuh"],
+    "compact": ["compact.cu", "compact.cuh", "cc_common.cuh"],
+    "select": ["select.cu", "select.cuh", "cc_common.cuh"],
+    "rowops": ["rowops.cu", "rowops.cuh", "cc_common.cuh"],
+}
+
+
+def kernel_digest(kernel):
+    """Hash of the sources of one kernel kind (e.g. gemm_gateup -> gemm.cu, ...)."""
     import hashlib
+    fam = ("gemm" if kernel.startswith("gemm") else "attention" if kernel.startswith("attention")
+           else kernel if kernel in KERNEL_SOURCES else "rowops")
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2607_27600_gb300", "csrc")
-    for f in sorted(os.listdir(csrc)):
+    for f in KERNEL_SOURCES[fam]:
         with open(os.path.join(csrc, f), "rb") as fh:
             h.update(f.encode() + fh.read())
     return h.hexdigest()[:16]
