@@ -49,14 +49,21 @@ namespace cc {
 namespace {
 
 constexpr int BKV = 128;        // keys per tile
+constexpr bool kFp8TwoIssuers = false;  // e4m3 cache: one issuer, two converter warps (measured: turn-taking issuers with one converter warp are slower, 1.13 vs 0.65 ms at 8k)
 constexpr int KST = 2;          // K and V pipeline stages
 constexpr int kThreads = 384;   // 3 warpgroups: softmax 0, softmax 1, producer/MMA
 // Register split after launch (setmaxnreg): the block is launched with 168
-// registers per thread (64512 in all); the producer/MMA warpgroup drops to
-// 64 and the two softmax warpgroups rise to 216: 2*128*216 + 128*64 = 63488.
-constexpr int kRegsLaunch = 168, kRegsSoftmax = 216, kRegsProducer = 64;
-static_assert(2 * 128 * kRegsSoftmax + 128 * kRegsProducer <= kThreads * kRegsLaunch,
-              "register split exceeds the launch allocation");
+// registers per thread (64512 in all); the producer/MMA warpgroup gives some
+// up and the two softmax warpgroups take them: bf16 operands 224 / 56, an
+// e4m3 cache (whose converters run in the third warpgroup) 208 / 88 -- the
+// splits at which each variant compiles without (or, split operands, with the
+// fewest) spills; 2 * 128 * softmax + 128 * producer <= 384 * 168.
+constexpr int kRegsLaunch = 168;
+template <bool FP8> struct RegSplit {
+  static constexpr int softmax = FP8 ? 208 : 224, producer = FP8 ? 88 : 56;
+  static_assert(2 * 128 * softmax + 128 * producer <= kThreads * kRegsLaunch,
+                "register split exceeds the launch allocation");
+};
 
 
 
@@ -150,7 +157,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                 const __grid_constant__ CUtensorMap tmV, const __grid_constant__ AttnParams p) {
   using L = AttnSmem<DH, FP8, SPLIT>;
-  constexpr bool kTwoIssuers = !FP8;   // warp 10 issues half 1's products (FP8: it converts)
+  // two turn-taking issuers (warps 9, 10); with an e4m3 cache warp 11 alone
+  // converts (kFp8TwoIssuers), else warp 9 issues both halves and warps 10-11 convert
+  constexpr bool kTwoIssuers = !FP8 || kFp8TwoIssuers;
+  constexpr int kConvWarp0 = kTwoIssuers ? 11 : 10;            // FP8: first converter warp
+  constexpr int kConvThreads = (12 - kConvWarp0) * 32;
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                               ~uintptr_t(1023));
@@ -229,18 +240,18 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (threadIdx.x == 0) {
     mbar_init(q_full, 1);
     for (int s = 0; s < KST; ++s) {   // FP8: K/V stages are filled by the 64 converter threads
-      mbar_init(&k_full[s], FP8 ? 64 : 1);
+      mbar_init(&k_full[s], FP8 ? kConvThreads : 1);
       mbar_init(&k_empty[s], kTwoIssuers ? 2 : 1);   // one commit per MMA issuer
-      mbar_init(&v_full[s], FP8 ? 64 : 1);
+      mbar_init(&v_full[s], FP8 ? kConvThreads : 1);
       mbar_init(&v_empty[s], kTwoIssuers ? 2 : 1);
     }
     mbar_init(v_fixed, 1);
     if (FP8) {
       for (int i = 0; i < 2; ++i) {
         mbar_init(&stg_full[i], 1);
-        mbar_init(&stg_empty[i], 64);
+        mbar_init(&stg_empty[i], kConvThreads);
       }
-      mbar_init(q_conv, 64);
+      mbar_init(q_conv, kConvThreads);
       for (int s = 0; s < KST; ++s) {
         mbar_init(&k_load[s], 1);
         mbar_init(&v_load[s], 1);
@@ -261,7 +272,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   if (warp >= 8) {
-    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegsProducer));
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(RegSplit<FP8>::producer));
     if (warp == 8) {
     // ------------------------------------------------------------ producer
     // Rows P*G..255 of the Q tile exist when G does not divide 256: zero
@@ -505,13 +516,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
     }
-    } else if (FP8 && warp >= 10) {
+    } else if (FP8 && warp >= kConvWarp0) {
     // ------------------------------------------------------------ converters (FP8)
-    const int ct = threadIdx.x - 10 * 32;   // 0 .. 63
+    const int ct = threadIdx.x - kConvWarp0 * 32;   // 0 .. kConvThreads - 1
     bool ok = mbar_wait(q_full, 0, abort_flag, p.status);
     if (ok) {   // Q bf16 -> f16 in place (same layout, element by element)
       uint4 *qv = reinterpret_cast<uint4 *>(smem + L::OFF_Q);
-      for (int i = ct; i < L::Q_BYTES / 16; i += 64) {
+      for (int i = ct; i < L::Q_BYTES / 16; i += kConvThreads) {
         uint4 x = qv[i];
         x.x = bf16x2_to_f16x2(x.x);
         x.y = bf16x2_to_f16x2(x.y);
@@ -526,7 +537,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // rows per 64-column half, 16-byte chunk c of row r at chunk c ^ (r & 7)
     // (the TMA's 128-byte swizzle); rows >= zero_from are written as zeros
     auto convert = [&](const uint8_t *src, uint8_t *dst, int zero_from) {
-      for (int i = ct; i < BKV * L::NH * 8; i += 64) {
+      for (int i = ct; i < BKV * L::NH * 8; i += kConvThreads) {
         const int r = i / (L::NH * 8), rem = i - r * (L::NH * 8), hh = rem >> 3, c = rem & 7;
         uint4 o = make_uint4(0, 0, 0, 0);
         if (r < zero_from) {
@@ -549,7 +560,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     auto convert_in_place = [&](uint8_t *base, int zero_from) {
       const int j = ct & 7;
       const int hh = j >> 2, c = (j & 3) * 2;
-      for (int r = ct >> 3; r < BKV; r += 8) {
+      for (int r = ct >> 3; r < BKV; r += kConvThreads / 8) {
         const uint4 x = *reinterpret_cast<const uint4 *>(base + L::KV_BYTES / 2 + r * 128 + j * 16);
         __syncwarp();
         uint4 a = make_uint4(0, 0, 0, 0), b = make_uint4(0, 0, 0, 0);
@@ -596,7 +607,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     }
   } else {
-    asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kRegsSoftmax));
+    asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(RegSplit<FP8>::softmax));
     // ------------------------------------------------------------ softmax
     const int h = warp >> 2, q = warp & 3;
     const int R = h * 128 + q * 32 + lane;              // unit row
