@@ -19,6 +19,11 @@ about 2^-17 relative; a tensor-core product then runs once per half):
   split-act    GEMM inputs split; queries and P single bf16; fp32 residual
   split-q      GEMM inputs and queries split; P single bf16; fp32 residual
   split-all    GEMM inputs, queries and P split; fp32 residual
+  split-qp     queries and P split, every GEMM input single bf16
+  split-qp-attn  queries, P and the attention-side GEMM inputs (the Q
+               projection's normalised input, the attention output) split
+  split-qp-mlp   queries, P and the MLP's GEMM inputs (the gate/up
+               projection's normalised input, the SwiGLU output) split
 
 The drift measured here is a property of the arithmetic and of the random
 model, not of any kernel; the full-pass tolerances of the parity tests are
@@ -75,7 +80,10 @@ def fp32(x):
     return x.astype(np.float32).astype(np.float64)
 
 
-# name -> (query rounding, GEMM-input rounding, P rounding, residual rounding)
+# name -> (query rounding, GEMM-input rounding, P rounding, residual rounding);
+# a GEMM-input entry may be a pair (attention-side inputs: normalised input of
+# the Q projection and the attention output; MLP inputs: normalised input of
+# gate/up and the SwiGLU output)
 VARIANTS = {
     "exact": (exact, exact, exact, exact),
     "queries": (bf16, exact, exact, exact),
@@ -84,11 +92,15 @@ VARIANTS = {
     "split-act": (bf16, split, bf16, fp32),
     "split-q": (split, split, bf16, fp32),
     "split-all": (split, split, split, fp32),
+    "split-qp": (split, bf16, split, fp32),                  # attention operands only
+    "split-qp-attn": (split, (split, bf16), split, fp32),    # + the attention-side GEMM inputs
+    "split-qp-mlp": (split, (bf16, split), split, fp32),     # + the MLP GEMM inputs
 }
 
 
 def layer(h, rows, pos, lw, k, v, n, shape, rounding):
     rq, ra, rp, rh = rounding
+    ra, rm = ra if isinstance(ra, tuple) else (ra, ra)   # attention-side, MLP GEMM inputs
     a = ra(R.rms_norm(h, lw["attn_norm"], shape.rms_eps))
     q = (a @ R.f64(lw["wq"]).T).reshape(len(rows), shape.n_q_heads, shape.head_dim)
     q = rq(R.rope(q, pos, shape.rope_theta))
@@ -97,8 +109,8 @@ def layer(h, rows, pos, lw, k, v, n, shape, rounding):
     else:
         o = ra(attention_rounded_p(q, k, v, rows, n, rp))
     h = rh(h + o.reshape(len(rows), -1) @ R.f64(lw["wo"]).T)
-    m = ra(R.rms_norm(h, lw["mlp_norm"], shape.rms_eps))
-    act = ra(R.silu(m @ R.f64(lw["w_gate"]).T) * (m @ R.f64(lw["w_up"]).T))
+    m = rm(R.rms_norm(h, lw["mlp_norm"], shape.rms_eps))
+    act = rm(R.silu(m @ R.f64(lw["w_gate"]).T) * (m @ R.f64(lw["w_up"]).T))
     return rh(h + act @ R.f64(lw["w_down"]).T)
 
 

@@ -132,3 +132,27 @@ def test_range_past_the_sequence_end_is_reported(pkg):
     cc.cc_score_rows(SMALL_GPU, w, cache, cc.SCORE_LOGIT, False, lo, hi, scores, ws)
     assert cc.cc_get_status() == cc.CC_ERR_DEVICE_ARG
     assert cc.cc_get_status() == cc.CC_OK
+
+
+@pytest.mark.parametrize("layout", ["e4m3", "paged", "head_major"])
+def test_rows_in_blocks_over_cache_layout_variants(pkg, layout):
+    """The same bit-for-bit equality over an e4m3 cache, a paged cache (a
+    shuffled pool of 256-slot pages with a block table) and a head-major
+    cache."""
+    import bench
+    from paper_2607_27600_gb300 import cc
+    shape = synth.WORKLOADS["qwen7b-table1-fast-4096"].shape
+    seq, cap = [4096, 2500], 4096
+    last = shape.n_layers - 1
+    w = synth.model_weights(shape, 51, device="cuda", layers=[last], with_embed=False)
+    c = synth.synthetic_cache(shape, seq, cap, 52, device="cuda")
+    if layout == "e4m3":
+        bench.to_e4m3_cache(c)
+    elif layout == "paged":
+        bench.to_paged_cache(c, 256, 53)
+    else:
+        for key in ("k", "v"):
+            c[key] = [x.permute(0, 2, 1, 3).contiguous() for x in c[key]]
+        c["kv_layout"] = 1
+    single, merged, parts = _single_and_sharded(pkg, shape, w, c, cc.SCORE_LOGIT, False, 3)
+    _check(single, merged, parts, seq)
