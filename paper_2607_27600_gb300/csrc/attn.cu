@@ -237,7 +237,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     return;
   }
 
-  if (threadIdx.x == 0) {
+  // The producer warp initialises the barriers and issues the Q load before
+  // the CTA-wide barrier, so the load's latency overlaps the TMEM allocation
+  // and the barrier.
+  if (warp == 8 && lane == 0) {
     mbar_init(q_full, 1);
     for (int s = 0; s < KST; ++s) {   // FP8: K/V stages are filled by the 64 converter threads
       mbar_init(&k_full[s], FP8 ? kConvThreads : 1);
@@ -265,6 +268,29 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     *abort_flag = 0;
     fence_barrier_init();
+    tma_prefetch_desc(&tmQ);
+    tma_prefetch_desc(&tmK);
+    tma_prefetch_desc(&tmV);
+    mbar_arrive_expect_tx(q_full, (SPLIT ? 2 : 1) * L::NH * 128 * G * P);
+    for (int hh = 0; hh < L::NH; ++hh)
+      tma_load_3d(smem + L::OFF_Q + hh * 256 * 128, &tmQ, q_full, hh * 64, g * G,
+                  (int)row_base + p0);
+    if constexpr (SPLIT)   // lo heads follow the hi heads in each row
+      for (int hh = 0; hh < L::NH; ++hh)
+        tma_load_3d(smem + L::OFF_QLO + hh * 256 * 128, &tmQ, q_full, hh * 64,
+                    p.n_q_heads + g * G, (int)row_base + p0);
+  }
+  // Rows P*G..255 of the Q tile exist when G does not divide 256: zero them
+  // (the Q load does not write them) so their S rows are exact zeros (finite,
+  // never NaN) and the softmax can treat every row of a tile alike (no
+  // per-row mask path); visible to the tensor cores after the barrier below.
+  if (warp == 8 && G * P < 256) {
+    for (int qt = 0; qt < (SPLIT ? 2 : 1); ++qt)
+      for (int hh = 0; hh < L::NH; ++hh)
+        for (int idx = G * P * 8 + lane; idx < 256 * 8; idx += 32)
+          reinterpret_cast<uint4 *>(smem + L::OFF_Q + qt * L::Q_BYTES + hh * 256 * 128)[idx] =
+              make_uint4(0, 0, 0, 0);
+    fence_proxy_async_smem();
   }
   if (warp == 9) tmem_alloc(tmem_slot, 512);
   tc_fence_before();
@@ -275,31 +301,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(RegSplit<FP8>::producer));
     if (warp == 8) {
     // ------------------------------------------------------------ producer
-    // Rows P*G..255 of the Q tile exist when G does not divide 256: zero
-    // them once so their S rows are exact zeros (finite, never NaN) and the
-    // softmax can treat every row of a tile alike (no per-row mask path).
-    if (G * P < 256) {
-      for (int qt = 0; qt < (SPLIT ? 2 : 1); ++qt)
-        for (int hh = 0; hh < L::NH; ++hh)
-          for (int idx = G * P * 8 + lane; idx < 256 * 8; idx += 32)
-            reinterpret_cast<uint4 *>(smem + L::OFF_Q + qt * L::Q_BYTES + hh * 256 * 128)[idx] =
-                make_uint4(0, 0, 0, 0);
-      fence_proxy_async_smem();
-      __syncwarp();
-    }
-    if (lane == 0) {
-      tma_prefetch_desc(&tmQ);
-      tma_prefetch_desc(&tmK);
-      tma_prefetch_desc(&tmV);
-      mbar_arrive_expect_tx(q_full, (SPLIT ? 2 : 1) * L::NH * 128 * G * P);
-      for (int hh = 0; hh < L::NH; ++hh)
-        tma_load_3d(smem + L::OFF_Q + hh * 256 * 128, &tmQ, q_full, hh * 64, g * G,
-                    (int)row_base + p0);
-      if constexpr (SPLIT)   // lo heads follow the hi heads in each row
-        for (int hh = 0; hh < L::NH; ++hh)
-          tma_load_3d(smem + L::OFF_QLO + hh * 256 * 128, &tmQ, q_full, hh * 64,
-                      p.n_q_heads + g * G, (int)row_base + p0);
-    }
+    // (the Q tile was requested before the CTA-wide barrier)
     if constexpr (L::IN_PLACE) {
       // fp8 tiles into the upper half of their own stage (converted in place)
       for (int it = 0; it < ntiles; ++it) {
