@@ -57,3 +57,42 @@ def test_fp8_cache_halves_the_kv_bytes_of_the_compaction():
     b16, b8 = bench.algorithmic_work(wl, 2)["compact"][1], bench.algorithmic_work(wl, 1)["compact"][1]
     kv = 2 * 40 * 2 * wl.shape.n_layers * wl.shape.n_kv_heads * wl.shape.head_dim
     assert b16 - b8 == kv
+
+
+def test_tensor_peak_is_sustained_for_long_timed_regions():
+    peaks = {"bf16_tflops": 1916.0, "bf16_tflops_sustained": 1732.6, "hbm_gbs": 6682.5}
+    assert bench.tensor_peak(peaks, 0.5) == (1916.0, "bf16 dense burst")
+    assert bench.tensor_peak(peaks, 6.0) == (1732.6, "bf16 dense sustained")
+    assert bench.tensor_peak({"bf16_tflops": 1900.0}, 6.0)[0] == 1900.0   # no sustained figure
+    # a 1 ms launch of 1.5 TFLOP: 1500 TFLOP/s against either peak
+    table = bench.kernel_table({"gemm_gateup": (2, 2.0)}, 2, {"gemm_gateup": ("tensor", 1.5e12)},
+                               peaks, timed_s=6.0)
+    e = table["gemm_gateup"]
+    assert e["achieved"] == 1500.0
+    assert e["frac"] == round(1500.0 / 1732.6, 4) and e["frac_of_burst"] == round(1500.0 / 1916.0, 4)
+
+
+def test_oracle_leg_samples_and_extrapolation():
+    """The oracle leg on the tiny workload (CPU tensors): the row sample is
+    uniform over all positions and inside every sequence, the layer sample of a
+    full pass truncates the model, and the extrapolated refresh time grows
+    linearly from the sampled rows to every row (per-call fixed cost once)."""
+    import numpy as np
+    wl = _tiny("full", [300, 129, 64], [75, 40, 16], n_layers=4)
+    w = synth.model_weights(wl.shape, 3)
+    cache = synth.synthetic_cache(wl.shape, wl.seq_lens, wl.cap, 3, with_h_last=False)
+    leg = bench.OracleLeg(wl, w, cache, "logit")
+    assert leg.shape.n_layers == 2 and leg.layers == [0, 1]
+    rows = leg.sample(leg.rows_large, seed=4)
+    assert sum(len(r) for r in rows) == leg.rows_large
+    for r, n in zip(rows, wl.seq_lens):
+        assert all(0 <= i < n for i in r) and r == sorted(set(r))
+    scores = np.random.default_rng(0).standard_normal((wl.batch, wl.cap)).astype(np.float32)
+    leg.fixed = 0.5          # a known fixed cost: the extrapolation is then checkable
+    measured, total, d = leg.step(scores, seed=5)
+    per_row = max(0.0, d["t_rows"] - 0.5) / d["rows"]
+    want = (wl.shape.n_layers / 2) * (0.5 + per_row * sum(wl.seq_lens)) + d["t_sel"] + d["t_compact"]
+    assert abs(total - want) <= 1e-9 * want
+    assert measured > 0
+    base = leg.cpu_baseline(scores)
+    assert base["kind"] == "oracle" and base["extrapolated"] and base["value"] > 0
