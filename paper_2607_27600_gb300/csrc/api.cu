@@ -12,6 +12,7 @@
 // logsumexp(final-norm(h) W_U^T) - z[x_i]      (log-prob mode, GEMM+LSE).
 #include <math.h>
 #include <stdio.h>
+#include <stdlib.h>
 
 #include <algorithm>
 #include <atomic>
@@ -343,11 +344,21 @@ cc_status gemm_setup(Gemm &g, int epi, const void *A, int K, const void *W, cons
                           ((epi == EPI_RESID_F32 || epi == EPI_RESID_LOGIT) && nk_total < 128) ||
                           epi == EPI_BF16;
   DevState *dev_info = nullptr;
-  if (narrowable && dev_state(&dev_info) &&
+  const bool have_dev = dev_state(&dev_info);
+  // CTA pairs: for launches of two waves or more of 128 x 256 tiles (a pair
+  // takes two of them at once).  CC_GEMM_PAIRS=0: never; =2: whenever the
+  // tiles are 256 columns wide (narrow problems keep wide tiles then)
+  const char *pairs_env = getenv("CC_GEMM_PAIRS");
+  const int pair_mode = !pairs_env ? 1 : pairs_env[0] == '0' ? 0 : pairs_env[0] == '2' ? 2 : 1;
+  if (narrowable && have_dev && pair_mode != 2 &&
       ((R_est + 127) / 128) * (uint64_t)((N + 255) / 256) < (uint64_t)dev_info->sms)
     bn = 128;
+  const bool pair = have_dev && epi != EPI_ARGMAX && (epi == EPI_SWIGLU || bn == 256) &&
+                    (pair_mode == 2 ||
+                     (pair_mode == 1 && ((R_est + 127) / 128) * (uint64_t)((N + bn - 1) / bn) >=
+                                            2 * (uint64_t)dev_info->sms));
   if (!tmap_rows(&g.a, A, R, a_split ? 2 * K : K, 128)) return tmap_fail();
-  if (!tmap_rows(&g.b, W, N, K, epi == EPI_SWIGLU ? 128 : bn)) return tmap_fail();
+  if (!tmap_rows(&g.b, W, N, K, epi == EPI_SWIGLU || pair ? 128 : bn)) return tmap_fail();
   if (epi == EPI_SWIGLU) {
     if (!tmap_rows(&g.b2, W2, N, K, 128)) return tmap_fail();
   } else {
@@ -387,6 +398,8 @@ cc_status gemm_setup(Gemm &g, int epi, const void *A, int K, const void *W, cons
   const double t1 = a_bytes + b_bytes * ((num_m + gm - 1) / gm);
   g.p.raster = t1 < 0.8 * t0 ? 1 : 0;
   g.p.group = g.p.raster == 0 ? gn : gm;
+  g.p.pair = pair ? 1 : 0;
+  if (pair && g.p.raster == 1) g.p.group = std::max(1, gm / 2);   // pairs of row tiles
   return CC_OK;
 }
 
@@ -403,8 +416,9 @@ cc_status gemm_setup_qkv(Gemm &g, const void *xn, const cc_model_cfg *c,
   cc_status s = gemm_setup(g, EPI_QKV, xn, d, lw.wq, nullptr, qd + 2 * kvd, batch, cap, seq_len,
                            status, false, rows_hint);
   if (s != CC_OK) return s;
-  if (!tmap_rows(&g.b, lw.wq, qd, d, 256) || !tmap_rows(&g.b2, lw.wk, kvd, d, 256) ||
-      !tmap_rows(&g.b3, lw.wv, kvd, d, 256))
+  const uint32_t box = g.p.pair ? 128 : 256;   // a pair's CTAs load half a tile each
+  if (!tmap_rows(&g.b, lw.wq, qd, d, box) || !tmap_rows(&g.b2, lw.wk, kvd, d, box) ||
+      !tmap_rows(&g.b3, lw.wv, kvd, d, box))
     return tmap_fail();
   g.p.n_q_tiles = qd / 256;
   g.p.n_k_tiles = kvd / 256;
@@ -423,7 +437,7 @@ cc_status gemm_setup_qkv(Gemm &g, const void *xn, const cc_model_cfg *c,
 // residual in order (flags in the caller's workspace, tagged per launch).
 void plan_k_splits(Gemm &g, int epi, int sms, unsigned *flags) {
   g.p.k_splits = 1;
-  if ((epi != EPI_RESID_F32 && epi != EPI_RESID_LOGIT) || !flags) return;
+  if ((epi != EPI_RESID_F32 && epi != EPI_RESID_LOGIT) || !flags || g.p.pair) return;
   const uint64_t tiles = ((g.rows_est + 127) / 128) * (uint64_t)g.p.n_tiles;
   const int nk_total = ((g.p.K + 63) / 64) * (g.p.a_split ? 2 : 1);
   if (tiles == 0 || tiles >= (uint64_t)sms || tiles > (uint64_t)kSplitFlags) return;

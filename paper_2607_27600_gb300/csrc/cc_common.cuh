@@ -68,14 +68,31 @@ CC_DEV bool mbar_try_wait(uint64_t *bar, uint32_t parity) {
   return ok != 0;
 }
 
+// As mbar_try_wait, with acquire at cluster scope: for a barrier that threads
+// of the other CTA of a cluster arrive on (mbar_arrive_cluster).
+CC_DEV bool mbar_try_wait_cluster(uint64_t *bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
 // Waits for the phase of `parity` to complete.  Gives up (returns false)
 // when *abort is set by another role of the CTA, or after kWaitLimitNs, in
-// which case it sets *abort and records CC_ERR_TIMEOUT.
+// which case it sets *abort and records CC_ERR_TIMEOUT.  CL: acquire at
+// cluster scope (arrivals from the other CTA of a pair).
+template <bool CL = false>
 CC_DEV bool mbar_wait(uint64_t *bar, uint32_t parity, volatile int *abort, unsigned *status) {
-  if (mbar_try_wait(bar, parity)) return true;
+  auto try_wait = [&]() { return CL ? mbar_try_wait_cluster(bar, parity) : mbar_try_wait(bar, parity); };
+  if (try_wait()) return true;
   uint64_t t0 = globaltimer();
   for (uint32_t it = 1;; ++it) {
-    if (mbar_try_wait(bar, parity)) return true;
+    if (try_wait()) return true;
     if ((it & 63u) == 0) {
       if (*abort) return false;
       if (globaltimer() - t0 > kWaitLimitNs) {
@@ -115,6 +132,18 @@ CC_DEV void tma_load_2d_hint(void *dst, const CUtensorMap *m, uint64_t *bar, int
       "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.L2::cache_hint"
       " [%0], [%1, {%3, %4}], [%2], %5;" ::"r"(smem_u32(dst)),
       "l"(reinterpret_cast<uint64_t>(m)), "r"(smem_u32(bar)), "r"(c0), "r"(c1), "l"(policy)
+      : "memory");
+}
+// 2-D tile load into this CTA's shared memory whose completion is counted
+// on the barrier at `bar_cl` (a shared::cluster address): with cta_group::2
+// that barrier may belong to the other CTA of the pair, so both CTAs' stage
+// loads complete on one barrier of CTA 0.
+CC_DEV void tma_load_2d_pair_hint(void *dst, const CUtensorMap *m, uint32_t bar_cl, int32_t c0,
+                                  int32_t c1, uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      ".L2::cache_hint [%0], [%1, {%3, %4}], [%2], %5;" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(m)), "r"(bar_cl), "r"(c0), "r"(c1), "l"(policy)
       : "memory");
 }
 // L2 policies: keep (evict last) for data read again soon, stream (evict first).
@@ -228,6 +257,73 @@ CC_DEV void umma_commit(uint64_t *bar) {
   asm volatile(
       "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
           smem_u32(bar))
+      : "memory");
+}
+
+// ---------------------------------------------------------------------------
+// CTA pairs: a cluster of two CTAs on two SMs sharing one tcgen05 product
+// (cta_group::2).  The pair's M = 256 product reads A rows 0-127 from the
+// shared memory of CTA 0 and rows 128-255 from CTA 1, B rows [0, N/2) from
+// CTA 0 and [N/2, N) from CTA 1 (both at the same shared-memory offsets), and
+// writes D rows 0-127 to the tensor memory of CTA 0 and 128-255 to CTA 1.
+// One thread of CTA 0 issues it; allocation and release of the tensor
+// memory are done by one warp of each CTA together.
+// ---------------------------------------------------------------------------
+CC_DEV uint32_t cluster_ctarank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+CC_DEV uint32_t cluster_nctarank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_nctarank;" : "=r"(r));
+  return r;
+}
+// Address in the shared::cluster window of the variable at `p` (this CTA's
+// shared memory) as laid out in CTA `rank` of the cluster.
+CC_DEV uint32_t cluster_addr(const void *p, uint32_t rank) {
+  uint32_t a;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(a) : "r"(smem_u32(p)), "r"(rank));
+  return a;
+}
+// Arrive on an mbarrier of another CTA of the cluster (release, cluster scope).
+CC_DEV void mbar_arrive_cluster(uint32_t cl_addr) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cl_addr)
+               : "memory");
+}
+// Every thread of every CTA of the cluster (release / acquire).
+CC_DEV void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\t"
+               "barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+CC_DEV void tmem_alloc_pair(uint32_t *dst, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                   smem_u32(dst)),
+               "r"(ncols)
+               : "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+}
+CC_DEV void tmem_dealloc_pair(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+               : "memory");
+}
+// The pair's D[tmem] (+)= A[smem desc] * B[smem desc]^T (kind::f16), issued
+// by CTA 0 for both CTAs.
+CC_DEV void umma_ss_pair(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                         uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+// Arrive on the mbarrier at `bar`'s offset in every CTA of `cta_mask` once
+// the pair products this thread issued so far complete.
+CC_DEV void umma_commit_pair(uint64_t *bar, uint16_t cta_mask) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
+      " [%0], %1;" ::"r"(smem_u32(bar)),
+      "h"(cta_mask)
       : "memory");
 }
 

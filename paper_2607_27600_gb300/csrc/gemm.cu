@@ -14,7 +14,13 @@
 //   warps 2..5  epilogue: tcgen05.ld of the accumulator (one row per thread)
 // Two 256-column accumulators in TMEM let the epilogue of one tile overlap
 // the main loop of the next.
+// Large launches run as CTA pairs (clusters of two, cta_group::2): one
+// M = 256, N = 256 product per pair, each CTA staging its own 128 A rows and
+// half of the B tile, so a CTA moves 32 KB instead of 48 KB through L2 and
+// shared memory per 128 x 256 x 64 block of its output.
 #include "gemm.cuh"
+
+#include <algorithm>
 
 namespace cc {
 
@@ -23,6 +29,9 @@ namespace {
 // BN: the widest column tile (256); a launch uses TBN = 256 or, for narrow
 // problems (less than one wave of 256-column tiles), 128.
 constexpr int BM = 128, BN = 256, BK = 64, ST = 4;
+// CTA pairs (one 256 x 256 product per pair, each CTA holding 128 A rows and
+// 128 B rows of a stage): 16 + 16 KB stages, six of them
+constexpr int ST_PAIR = 6;
 constexpr int A_BYTES = BM * BK * 2;   // 16 KB
 constexpr int B_BYTES = BN * BK * 2;   // 32 KB: shared-memory stage of the widest B tile
 constexpr int kThreads = 192;
@@ -33,8 +42,13 @@ constexpr int kMaxBatch = 1024;
 constexpr int kStageLd = 36;
 constexpr int kStageBytes = 4 * 32 * kStageLd * 4;   // the four epilogue warps
 constexpr size_t kPrefixBytes = ((kMaxBatch + 1) * sizeof(int) + 15) & ~size_t(15);
-constexpr size_t kSmemBytes = 1024 /*align slack*/ + ST * (A_BYTES + B_BYTES) + 256 +
-                              kPrefixBytes + kStageBytes;
+__host__ __device__ constexpr size_t stages(bool pair) { return pair ? ST_PAIR : ST; }
+__host__ __device__ constexpr size_t b_stage_bytes(bool pair) { return pair ? B_BYTES / 2 : B_BYTES; }
+__host__ __device__ constexpr size_t ring_bytes(bool pair) { return stages(pair) * (A_BYTES + b_stage_bytes(pair)); }
+__host__ __device__ constexpr size_t smem_bytes(bool pair) {
+  return 1024 /*align slack*/ + ring_bytes(pair) + 256 + kPrefixBytes + kStageBytes;
+}
+static_assert(smem_bytes(false) <= 232448 && smem_bytes(true) <= 232448, "shared memory");
 
 // RoPE'd bf16 store of one accumulator tile row: destination columns
 // [col0, col0 + TBN) of out (row stride ldo, n_dest columns in all), each tile
@@ -525,36 +539,58 @@ CC_DEV void tile_coords(const GemmParams &p, int t, int num_m, int &m, int &n) {
   }
 }
 
-template <int EPI, int TBN>
+// One CTA (PAIR false) or a CTA pair (PAIR true, a cluster of two) per SM
+// pair, persistent over the output tiles.  A pair computes 256-row tiles:
+// CTA r holds row tile 2 mp + r of pair row mp (rows of two consecutive
+// 128-row tiles, which may belong to different sequences) and B rows
+// [r TBN/2, (r+1) TBN/2) of the column tile; CTA 0 issues the pair's
+// products into both tensor memories and its commits release the stages
+// and accumulators of both CTAs.  Both CTAs' loads of a stage complete on
+// CTA 0's stage barrier (CTA 0 arms it with the bytes of both), and CTA 1's
+// epilogue warps release an accumulator by arriving on CTA 0's barrier.
+// (A relay thread in CTA 1 that waited for its own stage barrier and then
+// arrived on CTA 0's measured 3.4x slower on the gate/up shape: the
+// hand-over latency sat on every stage.)  K splits run on single CTAs only.
+template <int EPI, int TBN, bool PAIR>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                 const __grid_constant__ CUtensorMap tmB2, const __grid_constant__ CUtensorMap tmB3,
                 const __grid_constant__ GemmParams p) {
-  constexpr int TB_BYTES = TBN * BK * 2;   // B stage of this launch's tile width
+  constexpr int kSt = (int)stages(PAIR);
+  constexpr int TB_BYTES = TBN * BK * 2;                  // B tile of one product
+  constexpr int SB = PAIR ? TB_BYTES / 2 : TB_BYTES;       // B stage: this CTA's share
+  static_assert(!PAIR || TBN == BN, "CTA pairs use 256-column tiles");
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                               ~uintptr_t(1023));
   uint8_t *sA = smem;
-  uint8_t *sB = smem + ST * A_BYTES;
-  uint64_t *full = reinterpret_cast<uint64_t *>(sB + ST * B_BYTES);
-  uint64_t *empty = full + ST;
-  uint64_t *tfull = empty + ST;
+  uint8_t *sB = smem + kSt * A_BYTES;
+  uint64_t *full = reinterpret_cast<uint64_t *>(smem + ring_bytes(PAIR));
+  uint64_t *empty = full + kSt;
+  uint64_t *tfull = empty + kSt;
   uint64_t *tempty = tfull + 2;
   uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(tempty + 2);
   volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
-  int *prefix = reinterpret_cast<int *>(smem + ST * (A_BYTES + B_BYTES) + 256);
-  float *stage_all = reinterpret_cast<float *>(smem + ST * (A_BYTES + B_BYTES) + 256 + kPrefixBytes);
+  int *prefix = reinterpret_cast<int *>(smem + ring_bytes(PAIR) + 256);
+  float *stage_all = reinterpret_cast<float *>(smem + ring_bytes(PAIR) + 256 + kPrefixBytes);
   __shared__ int split_ok;   // K splits: the previous split of the tile has published
 
+  // a pair kernel launched without its cluster of two has no partner for
+  // the pair instructions: every CTA reports it and leaves before any
+  if (PAIR && cluster_nctarank() != 2) {
+    if (threadIdx.x == 0) set_status(p.status, CC_ERR_DEVICE_ARG);
+    return;
+  }
+  const uint32_t rank = PAIR ? cluster_ctarank() : 0;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
-    for (int s = 0; s < ST; ++s) {
-      mbar_init(&full[s], 1);
+    for (int s = 0; s < kSt; ++s) {
+      mbar_init(&full[s], 1);   // CTA 1 of a pair leaves its own unused
       mbar_init(&empty[s], 1);
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&tfull[a], 1);
-      mbar_init(&tempty[a], 4);
+      mbar_init(&tempty[a], PAIR ? 8 : 4);   // the epilogue warps (of both CTAs)
     }
     *abort_flag = 0;
     build_tile_prefix(p.seq_len, p.row_lo, p.batch, p.cap, BM, prefix, p.status);
@@ -566,19 +602,30 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (EPI == EPI_SWIGLU || EPI == EPI_QKV) tma_prefetch_desc(&tmB2);
     if (EPI == EPI_QKV) tma_prefetch_desc(&tmB3);
   }
-  if (warp == 1) tmem_alloc(tmem_slot, 512);
+  if (warp == 1) {
+    if constexpr (PAIR) tmem_alloc_pair(tmem_slot, 512);
+    else tmem_alloc(tmem_slot, 512);
+  }
   tc_fence_before();
   __syncthreads();
+  if constexpr (PAIR) cluster_sync();   // both CTAs' barriers exist before any remote arrival
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
   const int num_m = prefix[p.batch];
-  const int total = num_m * p.n_tiles;
+  const int num_mu = PAIR ? (num_m + 1) / 2 : num_m;   // row units: tiles or tile pairs
+  const int total = num_mu * p.n_tiles;
   const int nk = (p.K + BK - 1) / BK;           // k-blocks of one operand pass
   const int nk_total = p.a_split ? 2 * nk : nk;  // split A: the hi pass, then the lo pass
   // Work item = (tile, K split): the splits of a tile are consecutive items.
-  const int S = ((EPI == EPI_RESID_F32 || EPI == EPI_RESID_LOGIT) && p.k_splits > 1) ? p.k_splits
-                                                                                     : 1;
+  const int S = (!PAIR && (EPI == EPI_RESID_F32 || EPI == EPI_RESID_LOGIT) && p.k_splits > 1)
+                    ? p.k_splits
+                    : 1;
   const int total_items = total * S;
+  const int unit0 = PAIR ? (int)(blockIdx.x >> 1) : (int)blockIdx.x;
+  const int n_units = PAIR ? (int)(gridDim.x >> 1) : (int)gridDim.x;
+  // row tile of this CTA in row unit u (-1: past the last tile, the second
+  // CTA of an odd pair: it loads its B share only and stores nothing)
+  auto row_tile = [&](int u) { const int mt = PAIR ? 2 * u + (int)rank : u; return mt < num_m ? mt : -1; };
 
   if (warp == 0) {
     if (lane == 0) {  // ---------------- TMA producer
@@ -587,64 +634,89 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint64_t pol_b = p.raster == 0 ? keep : stream;
       int stage = 0;
       uint32_t phase = 0;
-      for (int item = blockIdx.x; item < total_items; item += gridDim.x) {
+      bool ok = true;
+      for (int item = unit0; ok && item < total_items; item += n_units) {
         const int tile = item / S, split = item - tile * S;
-        int mt, nt;
-        tile_coords(p, tile, num_m, mt, nt);
-        const int b = find_seq(prefix, p.batch, mt);
-        const int row0 = b * p.cap + (p.row_lo ? p.row_lo[b] : 0) + (mt - prefix[b]) * BM;
+        int mu, nt;
+        tile_coords(p, tile, num_mu, mu, nt);
+        const int mt = row_tile(mu);
+        int row0 = 0;
+        if (mt >= 0) {
+          const int b = find_seq(prefix, p.batch, mt);
+          row0 = b * p.cap + (p.row_lo ? p.row_lo[b] : 0) + (mt - prefix[b]) * BM;
+        }
         const int kb0 = split * nk_total / S, kb1 = (split + 1) * nk_total / S;
+        // a pair's second row tile exists (CTA 0 counts its A bytes)
+        const bool a1 = PAIR && 2 * mu + 1 < num_m;
         for (int kb = kb0; kb < kb1; ++kb) {
-          if (!mbar_wait(&empty[stage], phase ^ 1, abort_flag, p.status)) goto producer_done;
-          mbar_arrive_expect_tx(&full[stage], A_BYTES + TB_BYTES);
+          if (!(ok = mbar_wait(&empty[stage], phase ^ 1, abort_flag, p.status))) break;
+          if (!PAIR) mbar_arrive_expect_tx(&full[stage], A_BYTES + TB_BYTES);
+          else if (rank == 0) mbar_arrive_expect_tx(&full[stage], (a1 ? 2 : 1) * A_BYTES + TB_BYTES);
+          const uint32_t bar_cl = PAIR ? cluster_addr(&full[stage], 0) : 0;
+          auto load = [&](uint8_t *dst, const CUtensorMap *m, int c0, int c1, uint64_t pol) {
+            if constexpr (PAIR) tma_load_2d_pair_hint(dst, m, bar_cl, c0, c1, pol);
+            else tma_load_2d_hint(dst, m, &full[stage], c0, c1, pol);
+          };
           // A column block kb of [hi | lo] (hi and lo halves are K apart), B block kb mod nk
           const int ka = kb < nk ? kb * BK : p.K + (kb - nk) * BK;
           const int kw = (kb < nk ? kb : kb - nk) * BK;
-          tma_load_2d_hint(sA + stage * A_BYTES, &tmA, &full[stage], ka, row0, pol_a);
-          if constexpr (EPI == EPI_SWIGLU) {
-            tma_load_2d_hint(sB + stage * TB_BYTES, &tmB, &full[stage], kw, nt * 128, pol_b);
-            tma_load_2d_hint(sB + stage * TB_BYTES + TB_BYTES / 2, &tmB2, &full[stage], kw, nt * 128,
-                             pol_b);
+          if (mt >= 0) load(sA + stage * A_BYTES, &tmA, ka, row0, pol_a);
+          uint8_t *sb = sB + stage * SB;
+          if constexpr (EPI == EPI_SWIGLU) {   // gate rows, then up rows (CTA 0: gate, CTA 1: up)
+            if (!PAIR || rank == 0) load(sb, &tmB, kw, nt * 128, pol_b);
+            if (!PAIR || rank == 1) load(PAIR ? sb : sb + TB_BYTES / 2, &tmB2, kw, nt * 128, pol_b);
           } else if constexpr (EPI == EPI_QKV) {
-            const int nq = p.n_q_tiles, nk = p.n_k_tiles;
-            const CUtensorMap *m = nt < nq ? &tmB : (nt < nq + nk ? &tmB2 : &tmB3);
-            const int r0 = (nt < nq ? nt : (nt < nq + nk ? nt - nq : nt - nq - nk)) * TBN;
-            tma_load_2d_hint(sB + stage * TB_BYTES, m, &full[stage], kw, r0, pol_b);
+            const int nq = p.n_q_tiles, nkt = p.n_k_tiles;
+            const CUtensorMap *m = nt < nq ? &tmB : (nt < nq + nkt ? &tmB2 : &tmB3);
+            const int r0 = (nt < nq ? nt : (nt < nq + nkt ? nt - nq : nt - nq - nkt)) * TBN;
+            load(sb, m, kw, r0 + (int)rank * (TBN / 2), pol_b);
           } else {
-            tma_load_2d_hint(sB + stage * TB_BYTES, &tmB, &full[stage], kw, nt * TBN, pol_b);
+            load(sb, &tmB, kw, nt * TBN + (int)rank * (TBN / 2), pol_b);
           }
-          if (++stage == ST) { stage = 0; phase ^= 1; }
+          if (++stage == kSt) { stage = 0; phase ^= 1; }
         }
       }
-    producer_done:;
+      if (PAIR && ok) {
+        // every stage's last release (a commit of CTA 0) has landed before
+        // the CTA may leave
+        for (int i = 0; i < kSt; ++i) {
+          if (!mbar_wait(&empty[stage], phase ^ 1, abort_flag, p.status)) break;
+          if (++stage == kSt) { stage = 0; phase ^= 1; }
+        }
+      }
     }
   } else if (warp == 1) {
-    if (lane == 0) {  // ---------------- MMA issuer
-      constexpr uint32_t idesc = make_idesc_bf16(BM, TBN, 0, 0);
+    if (lane == 0 && rank == 0) {  // ---------------- MMA issuer (CTA 0 of a pair)
+      constexpr uint32_t idesc = make_idesc_bf16(PAIR ? 2 * BM : BM, TBN, 0, 0);
       const uint64_t a_desc0 = make_sdesc_sw128(smem_u32(sA), 16, 1024);
       const uint64_t b_desc0 = make_sdesc_sw128(smem_u32(sB), 16, 1024);
       int stage = 0, acc = 0;
       uint32_t phase = 0, acc_phase = 0;
-      for (int item = blockIdx.x; item < total_items; item += gridDim.x) {
+      for (int item = unit0; item < total_items; item += n_units) {
         const int split = item % S;
         const int kb0 = split * nk_total / S, kb1 = (split + 1) * nk_total / S;
-        if (!mbar_wait(&tempty[acc], acc_phase ^ 1, abort_flag, p.status)) break;
+        if (!mbar_wait<PAIR>(&tempty[acc], acc_phase ^ 1, abort_flag, p.status)) break;
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + acc * TBN;
         for (int kb = kb0; kb < kb1; ++kb) {
-          if (!mbar_wait(&full[stage], phase, abort_flag, p.status)) goto mma_done;
+          if (!mbar_wait<PAIR>(&full[stage], phase, abort_flag, p.status)) goto mma_done;
           tc_fence_after();
           // descriptors of this stage; a K step of 16 columns advances the
           // start-address field by 32 bytes (+2 in 16-byte units)
           const uint64_t ad = a_desc0 + (uint64_t)(stage * (A_BYTES >> 4));
-          const uint64_t bd = b_desc0 + (uint64_t)(stage * (TB_BYTES >> 4));
+          const uint64_t bd = b_desc0 + (uint64_t)(stage * (SB >> 4));
 #pragma unroll
-          for (int k = 0; k < BK / 16; ++k)
-            umma_ss(d_tmem, ad + 2 * k, bd + 2 * k, idesc, (kb != kb0 || k != 0) ? 1u : 0u);
-          umma_commit(&empty[stage]);
-          if (++stage == ST) { stage = 0; phase ^= 1; }
+          for (int k = 0; k < BK / 16; ++k) {
+            const uint32_t accum = (kb != kb0 || k != 0) ? 1u : 0u;
+            if constexpr (PAIR) umma_ss_pair(d_tmem, ad + 2 * k, bd + 2 * k, idesc, accum);
+            else umma_ss(d_tmem, ad + 2 * k, bd + 2 * k, idesc, accum);
+          }
+          if constexpr (PAIR) umma_commit_pair(&empty[stage], 0x3);
+          else umma_commit(&empty[stage]);
+          if (++stage == kSt) { stage = 0; phase ^= 1; }
         }
-        umma_commit(&tfull[acc]);
+        if constexpr (PAIR) umma_commit_pair(&tfull[acc], 0x3);
+        else umma_commit(&tfull[acc]);
         if (++acc == 2) { acc = 0; acc_phase ^= 1; }
       }
     mma_done:;
@@ -654,14 +726,19 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int r = q * 32 + lane;   // accumulator row of this thread
     int acc = 0;
     uint32_t acc_phase = 0;
-    for (int item = blockIdx.x; item < total_items; item += gridDim.x) {
+    for (int item = unit0; item < total_items; item += n_units) {
       const int tile = item / S, split = item - tile * S;
-      int mt, nt;
-      tile_coords(p, tile, num_m, mt, nt);
-      const int b = find_seq(prefix, p.batch, mt);
-      const int i = (p.row_lo ? p.row_lo[b] : 0) + (mt - prefix[b]) * BM + r;
-      const bool valid = i < (p.seq_len ? p.seq_len[b] : p.cap);
-      const int grow = b * p.cap + i;
+      int mu, nt;
+      tile_coords(p, tile, num_mu, mu, nt);
+      const int mt = row_tile(mu);
+      bool valid = false;
+      int grow = 0;
+      if (mt >= 0) {
+        const int b = find_seq(prefix, p.batch, mt);
+        const int i = (p.row_lo ? p.row_lo[b] : 0) + (mt - prefix[b]) * BM + r;
+        valid = i < (p.seq_len ? p.seq_len[b] : p.cap);
+        grow = b * p.cap + i;
+      }
       if (!mbar_wait(&tfull[acc], acc_phase, abort_flag, p.status)) break;
       tc_fence_after();
       const uint32_t tacc = tmem_base + acc * TBN + (uint32_t(q * 32) << 16);
@@ -669,7 +746,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // waits until split s-1 of the tile has published epoch * 16 + s.
       // Split s-1 is a lower work item, and every CTA takes its items in
       // increasing order, so the wait always ends (bounded all the same).
-      bool add = true;
+      bool add = mt >= 0;
       if (S > 1) {
         if (warp == 2 && lane == 0)
           split_ok = split == 0 || wait_value(&p.split_flags[tile], p.epoch * 16u + split, p.status);
@@ -688,47 +765,86 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
       __syncwarp();
-      if (lane == 0) mbar_arrive(&tempty[acc]);
+      if (lane == 0) {
+        if (PAIR && rank == 1) mbar_arrive_cluster(cluster_addr(&tempty[acc], 0));
+        else mbar_arrive(&tempty[acc]);
+      }
       if (++acc == 2) { acc = 0; acc_phase ^= 1; }
     }
   }
 
   tc_fence_before();
   __syncthreads();
+  if constexpr (PAIR) cluster_sync();   // the partner is done with this CTA's memories
   if (*abort_flag) __nanosleep(1000000);   // let copies still in flight land
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem_base, 512);
+    if constexpr (PAIR) tmem_dealloc_pair(tmem_base, 512);
+    else tmem_dealloc(tmem_base, 512);
   }
 }
 
-template <int EPI, int TBN>
+template <int EPI, int TBN, bool PAIR>
 cudaError_t launch_t(const CUtensorMap &a, const CUtensorMap &b, const CUtensorMap &b2,
                      const CUtensorMap &b3, const GemmParams &p, int grid, cudaStream_t stream) {
-  auto kern = gemm_kernel<EPI, TBN>;
+  auto kern = gemm_kernel<EPI, TBN, PAIR>;
   static bool attr_set[64] = {};
+  static int max_pairs[64] = {};   // co-resident CTA pairs (cluster occupancy)
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev < 64 && !attr_set[dev]) {
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)kSmemBytes);
+                                         (int)smem_bytes(PAIR));
     if (e != cudaSuccess) return e;
     attr_set[dev] = true;
   }
-  kern<<<grid, kThreads, kSmemBytes, stream>>>(a, b, b2, b3, p);
-  return cudaGetLastError();
+  if constexpr (!PAIR) {
+    kern<<<grid, kThreads, smem_bytes(false), stream>>>(a, b, b2, b3, p);
+    return cudaGetLastError();
+  } else {
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(2 * (unsigned)std::max(grid / 2, 1));
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = smem_bytes(true);
+    cfg.stream = stream;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int pairs = grid / 2;
+    if (dev < 64) {
+      if (max_pairs[dev] == 0) {
+        int n = 0;
+        cudaError_t e = cudaOccupancyMaxActiveClusters(&n, kern, &cfg);
+        if (e != cudaSuccess) return e;
+        max_pairs[dev] = std::max(n, 1);
+      }
+      pairs = std::min(pairs, max_pairs[dev]);
+    }
+    cfg.gridDim = dim3(2 * (unsigned)std::max(pairs, 1));
+    return cudaLaunchKernelEx(&cfg, kern, a, b, b2, b3, p);
+  }
 }
 
 // SwiGLU (gate and up halves), LSE and the fused q/k/v projections always
-// use 256-wide tiles; the others take p.block_n (128 or 256).
+// use 256-wide tiles; the others take p.block_n (128 or 256).  p.pair: CTA
+// pairs (256-wide tiles only; greedy decoding's argmax never pairs).
 template <int EPI>
 cudaError_t launch(const CUtensorMap &a, const CUtensorMap &b, const CUtensorMap &b2,
                    const CUtensorMap &b3, const GemmParams &p, int grid, cudaStream_t stream) {
-  if constexpr (EPI == EPI_SWIGLU || EPI == EPI_LSE || EPI == EPI_QKV) {
-    return launch_t<EPI, BN>(a, b, b2, b3, p, grid, stream);
+  constexpr bool kWide = EPI == EPI_SWIGLU || EPI == EPI_LSE || EPI == EPI_QKV;
+  if constexpr (EPI != EPI_ARGMAX) {
+    if (p.pair && (kWide || p.block_n == BN)) return launch_t<EPI, BN, true>(a, b, b2, b3, p, grid, stream);
+  }
+  if (p.pair) return cudaErrorInvalidValue;
+  if constexpr (kWide) {
+    return launch_t<EPI, BN, false>(a, b, b2, b3, p, grid, stream);
   } else {
-    if (p.block_n == 128) return launch_t<EPI, 128>(a, b, b2, b3, p, grid, stream);
-    return launch_t<EPI, BN>(a, b, b2, b3, p, grid, stream);
+    if (p.block_n == 128) return launch_t<EPI, 128, false>(a, b, b2, b3, p, grid, stream);
+    return launch_t<EPI, BN, false>(a, b, b2, b3, p, grid, stream);
   }
 }
 

@@ -63,6 +63,9 @@ struct GemmParams {
                            // (B kept in L2, A streamed per group); 1 = groups of `group`
                            // row tiles stay resident (A kept, B streamed per group)
   int group;
+  int pair;                // run as CTA pairs (256-column tiles, k_splits 1): the B tensor
+                           // maps' boxes are 128 rows (each CTA loads half of a tile);
+                           // raster 1 groups count pairs of row tiles
   int out_split;           // EPI_SWIGLU, EPI_QROPE (not into the cache): out rows are
                            // [hi | lo], lo at column offset N
   int k_splits;            // EPI_RESID_F32 / EPI_RESID_LOGIT only: K range split over
@@ -87,7 +90,7 @@ struct GemmParams {
 int gemm_block_n(int epi);
 int gemm_max_batch();
 // a: A rows x K (box 64 x 128); b (and b2 for SwiGLU, b2 and b3 for the fused
-// projections): weights N x K (box 64 x 256, or 64 x 128 for SwiGLU).
+// projections): weights N x K (box 64 x 256, or 64 x 128 for SwiGLU and for CTA pairs).
 // grid: persistent CTAs (one per SM).
 cudaError_t launch_gemm(int epi, const CUtensorMap &a, const CUtensorMap &b, const CUtensorMap &b2,
                         const CUtensorMap &b3, const GemmParams &p, int grid, cudaStream_t stream);
