@@ -629,9 +629,14 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 0) {
     if (lane == 0) {  // ---------------- TMA producer
+      // L2 policies: the resident operand evict-last, the streamed one
+      // evict-first; CTA pairs keep both evict-last (measured at the Llama-3-8B
+      // 16k launches: evict-first A made the pairs re-read it from DRAM,
+      // gate/up 4.3 -> 1.7 GB and 1.98 -> 1.92 ms, down 5.5 -> 3.5 GB and
+      // 1.09 -> 1.05 ms)
       const uint64_t keep = make_policy_evict_last(), stream = make_policy_evict_first();
-      const uint64_t pol_a = p.raster == 1 ? keep : stream;
-      const uint64_t pol_b = p.raster == 0 ? keep : stream;
+      const uint64_t pol_a = PAIR || p.raster == 1 ? keep : stream;
+      const uint64_t pol_b = PAIR || p.raster == 0 ? keep : stream;
       int stage = 0;
       uint32_t phase = 0;
       bool ok = true;
