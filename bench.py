@@ -409,11 +409,14 @@ def refresh_record(args, dist, wl, w, pristine, mode, steps, with_e2e=True, with
             cc.cc_h2o_accumulate(shape, cache, recent, kws)
             cc.cc_score_h2o(cache, recent, scores)
 
-    def step():
-        score()
+    def select_compact():
         cc.cc_select_keep(scores, cache.d["seq_len"], b, cap, budget, wl.n_sink, keep_idx,
                           keep_count)
         cc.cc_compact_kv(shape, cache, keep_idx, keep_count, cws)
+
+    def step():
+        score()
+        select_compact()
 
     def prepare():
         restore_cache(work, pristine)
@@ -461,8 +464,20 @@ def refresh_record(args, dist, wl, w, pristine, mode, steps, with_e2e=True, with
 
     e2e = None
     if with_e2e:
+        blocks = None
+        # the fast pass's rows scored block by block as their inputs land: one
+        # block per ~16k rows, at most 8 (ragged 32k batch, 81920 rows: 2.03 M
+        # positions/s end to end in one block, 2.34 M in 4, 2.31 M in 8, 2.14 M
+        # in 16; the 8k sequence: 2.75 M in one block, 2.29 M in 8)
+        nb = (args.e2e_blocks if args.e2e_blocks > 0 else
+              max(1, min(8, sum(wl.seq_lens) // 16384)))
+        if fast and scorer == "counter-causal" and row_shard is None and nb > 1:
+            blocks = {"n": nb, "select_compact": select_compact,
+                      "score": lambda lo, hi: cc.cc_score_rows(
+                          shape, weights, cache, mode | cc.SCORE_RANGE_ONLY, False, lo, hi,
+                          scores, ws)}
         e2e = e2e_leg(args, dist, wl, work, pristine, cache, step, keep_idx, keep_count, flush,
-                      stream, steps)
+                      stream, steps, blocks)
         if not (torch.equal(e2e.pop("keep_idx"), ref_idx) and
                 torch.equal(e2e.pop("keep_count"), ref_cnt)):
             raise SystemExit(f"{wl.name}: the end-to-end keep-set differs from the "
@@ -508,6 +523,9 @@ def refresh_record(args, dist, wl, w, pristine, mode, steps, with_e2e=True, with
                                      (e2e["ms"] * 1e-3), 1),
                       "unit": "positions/s", "h2d_bytes_per_step": e2e["h2d"],
                       "d2h_bytes_per_step": e2e["d2h"], "ms_per_step": round(e2e["ms"], 4)}
+        if e2e["blocks"] > 1:
+            rec["e2e"]["pipeline"] = (f"{e2e['blocks']} row blocks per sequence, uploaded from the "
+                                      "sequence ends backwards, each scored once it has landed")
     if (with_cpu and dist.world == 1 and not args.no_cpu_baseline and
             scorer == "counter-causal"):
         rec["cpu_baseline"] = OracleLeg(wl, w, pristine, args.score).cpu_baseline(
@@ -528,17 +546,41 @@ def roofline_of(table, dom, peaks, peak_src, timed_s, traffic):
                            f"lasts {SUSTAINED_AFTER_S:.0f} s or more, here {timed_s:.1f} s)"}
 
 
+def block_bounds(seq_lens, n_blocks, align=128):
+    """Starts of `n_blocks` row blocks of every sequence, [n_blocks + 1][batch]:
+    block k of sequence b is slots [bounds[k][b], bounds[k + 1][b]), about
+    n / n_blocks rows each; every interior start a multiple of `align` (128:
+    no key tile of a block's attention reaches below the block, so a block
+    scored before the earlier slots have landed never reads them)."""
+    out = []
+    for k in range(n_blocks + 1):
+        out.append([n if k == n_blocks else min(n, -(-(n * k // n_blocks) // align) * align)
+                    for n in seq_lens])
+    return out
+
+
 def e2e_leg(args, dist, wl, work, pristine, cache, step, keep_idx, keep_count, flush, stream,
-            steps):
+            steps, blocks=None):
     """The refresh through the public API with the step's inputs in pinned
-    host memory: H^(L-1) (fast pass), token ids, positions and lengths on the
-    compute stream; each scored layer's K/V on a copy stream that the library
-    waits on per layer (cc_kv_cache.kv_ready), so the uploads overlap the
-    kernels ahead of that layer's first K/V reader; the keep-set read back.
-    Copies and reads are inside the timed region."""
+    host memory: token ids, positions and lengths on the compute stream; the
+    scored rows' inputs (H^(L-1) in the fast pass, every scored layer's K/V)
+    on a copy stream, only each sequence's slots [0, n); the keep-set read
+    back.  Copies and reads are inside the timed region.
+    Full pass: the library waits per layer for that layer's K/V
+    (cc_kv_cache.kv_ready), so the uploads overlap the layers ahead of it.
+    Fast pass with `blocks` (n, score(lo, hi), select_compact): the rows are
+    uploaded in blocks from the sequence ends backwards and each block is
+    scored (cc_score_rows, CC_SCORE_RANGE_ONLY) once it has landed -- a row
+    attends only later slots, which arrived before it -- so the uploads
+    overlap the scoring; select and compaction follow.
+    Before every step the uploaded device tensors are overwritten with NaN
+    (outside the timed region): a block scored before its inputs landed
+    would change the keep-set, which the caller compares with the
+    device-resident step's."""
     dev = torch.device(f"cuda:{dist.local}")
     fast = wl.mode == "layer"
     b, cap = wl.batch, wl.cap
+    seq = list(wl.seq_lens)
     n_l = len(work["k"])
     kv_layers = [n_l - 1] if fast else list(range(n_l))
     host = {"h_last": pristine["h_last"].cpu().pin_memory() if fast else None,
@@ -547,39 +589,95 @@ def e2e_leg(args, dist, wl, work, pristine, cache, step, keep_idx, keep_count, f
             "seq_len": pristine["seq_len"].cpu().pin_memory(),
             "k": {l: pristine["k"][l].cpu().pin_memory() for l in kv_layers},
             "v": {l: pristine["v"][l].cpu().pin_memory() for l in kv_layers}}
+    for t in ([host["h_last"]] if fast else []) + list(host["k"].values()):
+        assert t.dim() >= 3 and t.shape[:2] == (b, cap), t.shape   # [batch, cap, ...]
+    nb = blocks["n"] if blocks else 1
+    bounds = block_bounds(seq, nb)
+    lo_host = torch.tensor(bounds[:-1], dtype=torch.int32).pin_memory()   # [nb][batch]
+    hi_host = torch.tensor(bounds[1:], dtype=torch.int32).pin_memory()
+    lo_dev = torch.empty_like(lo_host, device=dev)
+    hi_dev = torch.empty_like(hi_host, device=dev)
     out_idx = torch.empty(b, cap, dtype=torch.int32).pin_memory()
     out_cnt = torch.empty(b, dtype=torch.int32).pin_memory()
-    h2d = sum(t.numel() * t.element_size() for key in ("h_last", "tokens", "pos", "seq_len")
-              for t in [host[key]] if t is not None)
-    h2d += sum(t.numel() * t.element_size() for key in ("k", "v") for t in host[key].values())
+
+    def row_bytes(t):   # bytes of one slot of a [batch, cap, ...] tensor
+        return t[0, 0].numel() * t.element_size()
+
+    n_valid = sum(seq)
+    h2d = sum(host[key].numel() * host[key].element_size() for key in ("tokens", "pos", "seq_len"))
+    if fast:
+        h2d += n_valid * row_bytes(host["h_last"])
+    h2d += sum(n_valid * row_bytes(t) for key in ("k", "v") for t in host[key].values())
+    if blocks:
+        h2d += 2 * lo_host.numel() * 4
     d2h = out_idx.numel() * 4 + out_cnt.numel() * 4
     up = torch.cuda.Stream(dev)
     ready = [torch.cuda.Event() if l in kv_layers else None for l in range(n_l)]
     for e in ready:
         if e is not None:
             e.record(up)
+    landed = [torch.cuda.Event() for _ in range(nb)]
+
+    def upload_rows(k):
+        """Block k's rows of the uploaded tensors (on the copy stream)."""
+        for bi, n in enumerate(seq):
+            lo, hi = bounds[k][bi], bounds[k + 1][bi]
+            if hi <= lo:
+                continue
+            if fast:
+                work["h_last"][bi, lo:hi].copy_(host["h_last"][bi, lo:hi], non_blocking=True)
+            for l in kv_layers:
+                work["k"][l][bi, lo:hi].copy_(host["k"][l][bi, lo:hi], non_blocking=True)
+                work["v"][l][bi, lo:hi].copy_(host["v"][l][bi, lo:hi], non_blocking=True)
 
     def e2e_step():
         work["seq_len"].copy_(host["seq_len"], non_blocking=True)
         work["tokens"].copy_(host["tokens"], non_blocking=True)
         work["pos"].copy_(host["pos"], non_blocking=True)
-        if fast:
-            work["h_last"].copy_(host["h_last"], non_blocking=True)
         up.wait_stream(stream)
-        with torch.cuda.stream(up):
-            for l in kv_layers:
-                work["k"][l].copy_(host["k"][l], non_blocking=True)
-                work["v"][l].copy_(host["v"][l], non_blocking=True)
-                ready[l].record(up)
-        step()
+        if blocks:
+            lo_dev.copy_(lo_host, non_blocking=True)
+            hi_dev.copy_(hi_host, non_blocking=True)
+            with torch.cuda.stream(up):
+                for k in reversed(range(nb)):   # the sequence ends first
+                    upload_rows(k)
+                    landed[k].record(up)
+            for k in reversed(range(nb)):
+                stream.wait_event(landed[k])
+                blocks["score"](lo_dev[k], hi_dev[k])
+            blocks["select_compact"]()
+        else:
+            with torch.cuda.stream(up):
+                if fast:
+                    upload_rows(0)
+                for l in kv_layers:
+                    if not fast:
+                        for bi, n in enumerate(seq):
+                            work["k"][l][bi, :n].copy_(host["k"][l][bi, :n], non_blocking=True)
+                            work["v"][l][bi, :n].copy_(host["v"][l][bi, :n], non_blocking=True)
+                    ready[l].record(up)
+            if fast:
+                stream.wait_stream(up)
+            step()
         out_idx.copy_(keep_idx, non_blocking=True)
         out_cnt.copy_(keep_count, non_blocking=True)
 
-    cache.set_kv_ready(ready)
+    def poison(t):   # NaN in bf16 / fp32 tensors, the e4m3 NaN code in byte tensors
+        if t.dtype.is_floating_point:
+            t.fill_(float("nan"))
+        else:
+            t.fill_(0x7F)
+
+    cache.set_kv_ready(None if (fast or blocks) else ready)
     e2e_ms = []
     try:
         for _ in range(steps):
             restore_cache(work, pristine)   # the rest of the device-resident cache
+            if fast:
+                poison(work["h_last"])
+            for l in kv_layers:
+                poison(work["k"][l])
+                poison(work["v"][l])
             flush.fill_(1)
             torch.cuda.synchronize(dev)
             t0 = torch.cuda.Event(enable_timing=True)
@@ -596,7 +694,7 @@ def e2e_leg(args, dist, wl, work, pristine, cache, step, keep_idx, keep_count, f
     if status != cc.CC_OK:
         raise SystemExit(f"{wl.name}: device status after e2e: {cc.cc_status_str(status)}")
     return {"ms": dist.max(sum(e2e_ms) / len(e2e_ms)), "h2d": int(h2d), "d2h": int(d2h),
-            "keep_idx": out_idx.clone(), "keep_count": out_cnt.clone()}
+            "blocks": nb, "keep_idx": out_idx.clone(), "keep_count": out_cnt.clone()}
 
 
 def cycles_record(args, dist, wl, w, pristine, steps):
@@ -1381,6 +1479,9 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--precise", action="store_true",
                     help="time the precise mode (CC_SCORE_PRECISE) as the headline")
+    ap.add_argument("--e2e-blocks", type=int, default=0,
+                    help="fast pass end to end: row blocks uploaded and scored in turn (1: the "
+                         "whole input first; 0: one block per 16k rows, at most 8)")
     ap.add_argument("--no-records", action="store_true",
                     help="only the named workload (no precise-mode and other-workload records)")
     ap.add_argument("--synthetic-cache", action="store_true",

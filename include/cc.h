@@ -65,7 +65,12 @@ typedef enum {
    * depth by several percent; with it the 32-layer score stays within
    * ~1e-3.  With an e4m3 cache the attention operands are f16 and the
    * queries and P stay single. */
-  CC_SCORE_PRECISE = 0x100
+  CC_SCORE_PRECISE = 0x100,
+  /* Flag, OR-ed into the mode of cc_score_rows: the rows of the range are
+   * written and every other entry of scores (other rows, slots past the
+   * sequence ends) keeps its value, so that calls over disjoint ranges fill
+   * one buffer -- e.g. blocks of rows scored as their inputs arrive. */
+  CC_SCORE_RANGE_ONLY = 0x200
 } cc_score_mode;
 
 /* Element format of the cached keys and values.  The paper keeps the model's
@@ -230,7 +235,8 @@ cc_status cc_score_full(const cc_model_cfg *cfg, const cc_model_weights *w,
  * their scores (slot seq_len[b]-1 gets +inf when in range) and every other
  * entry of scores [batch][cap] gets -inf, so the element-wise maximum of the
  * ranks' buffers (one MAX all-reduce of batch * cap floats) is the whole
- * refresh's scores.  A row's score is bit-identical to the one
+ * refresh's scores; with CC_SCORE_RANGE_ONLY in mode the other entries are
+ * left as they are instead.  A row's score is bit-identical to the one
  * cc_score_layer / cc_score_full writes for it with the same cache and mode.
  * Same workspace as those calls.  row_lo and row_hi must both be null (every
  * row) or both be given. */

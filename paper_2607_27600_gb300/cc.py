@@ -27,6 +27,7 @@ STATUS_NAMES = {0: "CC_OK", 1: "CC_ERR_INVALID_ARG", 2: "CC_ERR_CUDA", 3: "CC_ER
 SCORE_LOGIT = 0
 SCORE_LOGPROB = 1
 SCORE_PRECISE = 0x100   # flag: hi + lo bf16 GEMM activations, queries and P (either pass)
+SCORE_RANGE_ONLY = 0x200   # flag (cc_score_rows): entries outside the row range keep their values
 
 
 class CCError(RuntimeError):
@@ -329,7 +330,7 @@ def cc_score_full(cfg, weights, cache, mode, scores, ws, stream=None):
 def cc_score_rows(cfg, weights, cache, mode, full: bool, row_lo, row_hi, scores, ws, stream=None):
     """Scores only rows [row_lo[b], row_hi[b]) of each sequence (device int32
     [batch] each, or both None for every row); every other entry of `scores`
-    gets -inf."""
+    gets -inf, or keeps its value with SCORE_RANGE_ONLY in `mode`."""
     code = load_library().cc_score_rows(
         ctypes.byref(_cfg(cfg)), ctypes.byref(weights.c), ctypes.byref(cache.c), int(mode),
         1 if full else 0, _dev_ptr(row_lo, "row_lo"), _dev_ptr(row_hi, "row_hi"),

@@ -894,7 +894,7 @@ cc_status check_score_args(const cc_model_cfg *c, const cc_model_weights *w, con
     return CC_ERR_INVALID_ARG;
   const int base_mode = mode & 0xFF;
   if ((base_mode != CC_SCORE_LOGIT && base_mode != CC_SCORE_LOGPROB) ||
-      (mode & ~(0xFF | CC_SCORE_PRECISE)))
+      (mode & ~(0xFF | CC_SCORE_PRECISE | CC_SCORE_RANGE_ONLY)))
     return CC_ERR_INVALID_ARG;
   if (kv->batch < 1 || kv->cap < 1 || !kv->seq_len || !kv->tokens || !kv->pos ||
       !kv_format_ok(c, kv))
@@ -923,7 +923,8 @@ cc_status check_score_args(const cc_model_cfg *c, const cc_model_weights *w, con
 // rng_lo / rng_hi (device [batch], or both null): score only the rows
 // [rng_lo[b], rng_hi[b]) of each sequence, each attending every later slot;
 // every row kernel then visits those rows alone and the head writes only
-// their scores (cc_score_rows).
+// their scores (cc_score_rows), -inf elsewhere unless the mode has
+// CC_SCORE_RANGE_ONLY (elsewhere untouched).
 cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_kv_cache *kv,
                     cc_score_mode mode, float *scores, void *ws, size_t ws_bytes, void *stream,
                     bool full, const int32_t *rng_lo = nullptr, const int32_t *rng_hi = nullptr) {
@@ -941,6 +942,7 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
   const bool split_q = split && kv->kv_format != CC_KV_E4M3;
   const ScoreWs L = score_layout(c, batch, cap, mode, split);
   const bool logit = (mode & 0xFF) == CC_SCORE_LOGIT;
+  const bool keep_outside = (mode & CC_SCORE_RANGE_ONLY) != 0;   // other entries untouched
   uint8_t *wsb = reinterpret_cast<uint8_t *>(ws);
   void *xn = wsb + L.xn, *q = wsb + L.q, *o = wsb + L.o, *act = wsb + L.act;
   float *h = reinterpret_cast<float *>(wsb + L.h);
@@ -1048,7 +1050,7 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
     TimedScope t(CC_KERNEL_HEAD_LOGIT, st);
     CC_TRY(launch_head_logit(reinterpret_cast<const float2 *>(wsb + L.hpart), n_htiles,
                              kv->tokens, scores, d, c->vocab, c->rms_eps, kv->seq_len, cap, rows,
-                             status, st, rng_lo, rng_hi));
+                             status, st, rng_lo, rng_hi, keep_outside));
   } else {
     {
       TimedScope t(CC_KERNEL_RMSNORM, st);
@@ -1069,7 +1071,7 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
     if ((s = run_gemm(gl, EPI_LSE, CC_KERNEL_GEMM_LMHEAD, dev->sms, st)) != CC_OK) return s;
     TimedScope t(CC_KERNEL_LSE_COMBINE, st);
     CC_TRY(launch_lse_combine(part, L.n_vtiles, zt, scores, kv->seq_len, cap, rows, st, rng_lo,
-                              rng_hi));
+                              rng_hi, keep_outside));
   }
   return CC_OK;
 }

@@ -279,14 +279,16 @@ __global__ void argmax_combine_kernel(const float2 *part, int n_tiles, const int
 __global__ void __launch_bounds__(kWarps * 32)
     head_logit_kernel(const float2 *part, int n_tiles, const int32_t *tokens, float *scores,
                       int d, int vocab, float eps, const int32_t *seq_len, int cap, int rows,
-                      unsigned *status, const int32_t *rng_lo, const int32_t *rng_hi) {
+                      unsigned *status, const int32_t *rng_lo, const int32_t *rng_hi,
+                      int keep_outside) {
   const int lane = threadIdx.x & 31;
   const int row = blockIdx.x * kWarps + (threadIdx.x >> 5);
   if (row >= rows) return;
   int i, n;
-  // rows outside the range (another rank's) and past the sequence end: -inf
+  // rows outside the range (another rank's) and past the sequence end: -inf,
+  // or left as they are (keep_outside)
   if (!in_score_range(rng_lo, rng_hi, cap, row) || !row_valid(seq_len, cap, row, i, n)) {
-    if (lane == 0) scores[row] = -INFINITY;
+    if (lane == 0 && !keep_outside) scores[row] = -INFINITY;
     return;
   }
   if (i == n - 1) {   // no future context: maximum surprise, always retained
@@ -311,14 +313,15 @@ __global__ void __launch_bounds__(kWarps * 32)
 __global__ void __launch_bounds__(kWarps * 32)
     lse_combine_kernel(const float2 *part, int n_tiles, const float *z_target, float *scores,
                        const int32_t *seq_len, int cap, int rows, const int32_t *rng_lo,
-                       const int32_t *rng_hi) {
+                       const int32_t *rng_hi, int keep_outside) {
   const int lane = threadIdx.x & 31;
   const int row = blockIdx.x * kWarps + (threadIdx.x >> 5);
   if (row >= rows) return;
   int i, n;
-  // rows outside the range (another rank's) and past the sequence end: -inf
+  // rows outside the range (another rank's) and past the sequence end: -inf,
+  // or left as they are (keep_outside)
   if (!in_score_range(rng_lo, rng_hi, cap, row) || !row_valid(seq_len, cap, row, i, n)) {
-    if (lane == 0) scores[row] = -INFINITY;
+    if (lane == 0 && !keep_outside) scores[row] = -INFINITY;
     return;
   }
   if (i == n - 1) {
@@ -403,20 +406,23 @@ cudaError_t launch_append_finish(int32_t *seq_len, const int32_t *row_hi, int ba
 cudaError_t launch_head_logit(const float2 *part, int n_tiles, const int32_t *tokens,
                               float *scores, int d, int vocab, float eps, const int32_t *seq_len,
                               int cap, int rows, unsigned *status, cudaStream_t st,
-                              const int32_t *rng_lo, const int32_t *rng_hi) {
+                              const int32_t *rng_lo, const int32_t *rng_hi, bool keep_outside) {
   if (rows <= 0) return cudaSuccess;
   head_logit_kernel<<<blocks_for(rows), kWarps * 32, 0, st>>>(part, n_tiles, tokens, scores, d,
                                                              vocab, eps, seq_len, cap, rows,
-                                                             status, rng_lo, rng_hi);
+                                                             status, rng_lo, rng_hi,
+                                                             keep_outside ? 1 : 0);
   return cudaGetLastError();
 }
 
 cudaError_t launch_lse_combine(const float2 *part, int n_tiles, const float *z_target,
                                float *scores, const int32_t *seq_len, int cap, int rows,
-                               cudaStream_t st, const int32_t *rng_lo, const int32_t *rng_hi) {
+                               cudaStream_t st, const int32_t *rng_lo, const int32_t *rng_hi,
+                               bool keep_outside) {
   if (rows <= 0) return cudaSuccess;
   lse_combine_kernel<<<blocks_for(rows), kWarps * 32, 0, st>>>(part, n_tiles, z_target, scores,
-                                                              seq_len, cap, rows, rng_lo, rng_hi);
+                                                              seq_len, cap, rows, rng_lo, rng_hi,
+                                                              keep_outside ? 1 : 0);
   return cudaGetLastError();
 }
 

@@ -38,15 +38,16 @@ cudaError_t launch_argmax_combine(const float2 *part, int n_tiles, const int32_t
 // partials part[row][n_tiles] = (sum h^2, sum h * gain * lm_head[tokens[row]])
 // of the fused down projection; +inf at the last slot.  rng_lo / rng_hi
 // (device [batch], or null): only slots [rng_lo[b], rng_hi[b]) are scored,
-// the others get -inf.
+// the others get -inf (keep_outside: keep their values).
 cudaError_t launch_head_logit(const float2 *part, int n_tiles, const int32_t *tokens,
                               float *scores, int d, int vocab, float eps, const int32_t *seq_len,
                               int cap, int rows, unsigned *status, cudaStream_t st,
-                              const int32_t *rng_lo = nullptr, const int32_t *rng_hi = nullptr);
+                              const int32_t *rng_lo = nullptr, const int32_t *rng_hi = nullptr,
+                              bool keep_outside = false);
 // scores[row] = logsumexp - z_target, +inf at the last slot (ranges as above)
 cudaError_t launch_lse_combine(const float2 *part, int n_tiles, const float *z_target,
                                float *scores, const int32_t *seq_len, int cap, int rows,
                                cudaStream_t st, const int32_t *rng_lo = nullptr,
-                               const int32_t *rng_hi = nullptr);
+                               const int32_t *rng_hi = nullptr, bool keep_outside = false);
 
 }  // namespace cc

@@ -96,3 +96,19 @@ def test_oracle_leg_samples_and_extrapolation():
     assert measured > 0
     base = leg.cpu_baseline(scores)
     assert base["kind"] == "oracle" and base["extrapolated"] and base["value"] > 0
+
+
+def test_e2e_row_blocks_cover_every_slot_once_on_key_tile_boundaries():
+    """The fast pass's end-to-end blocks: every slot [0, n) of a sequence in
+    exactly one block, none past n, every interior start a multiple of 128
+    (a block's attention then reads no key tile below its own start)."""
+    seq = [32768, 8192, 300, 129, 64, 1, 0]
+    for nb in (1, 2, 8, 16):
+        bounds = bench.block_bounds(seq, nb)
+        assert len(bounds) == nb + 1
+        assert bounds[0] == [0] * len(seq) and bounds[-1] == seq
+        for k in range(nb):
+            for b, n in enumerate(seq):
+                lo, hi = bounds[k][b], bounds[k + 1][b]
+                assert 0 <= lo <= hi <= n
+                assert lo % 128 == 0 or lo == n

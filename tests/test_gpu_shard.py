@@ -79,6 +79,39 @@ def test_small_ragged_batch_both_passes_and_modes(pkg, mode_name, full):
     _check(single, merged, parts, seq)
 
 
+@pytest.mark.parametrize("mode_name", ["logit", "logprob", "precise"])
+@pytest.mark.parametrize("full", [False, True])
+def test_range_only_blocks_fill_one_buffer(pkg, mode_name, full):
+    """CC_SCORE_RANGE_ONLY: blocks of rows scored from the sequence ends
+    backwards (the order in which a pipelined upload delivers them) into one
+    buffer give the single call's scores bit for bit; entries past the
+    sequence ends are never written."""
+    from paper_2607_27600_gb300 import cc
+    mode = {"logit": cc.SCORE_LOGIT, "logprob": cc.SCORE_LOGPROB,
+            "precise": cc.SCORE_LOGIT | cc.SCORE_PRECISE}[mode_name]
+    seq, cap = [300, 129, 1, 64, 0], 320
+    w_np = to_np(synth.model_weights(SMALL_GPU, 23, with_kv_proj=True))
+    c_np = causal_cache(SMALL_GPU, w_np, seq, cap, 24)
+    w, c = to_device(w_np), to_device(c_np)
+    weights, cache = pkg.Weights(w), pkg.Cache(c)
+    b = len(seq)
+    ws = cc.alloc_workspace(cc.cc_score_workspace_size(SMALL_GPU, b, cap, mode))
+    single = torch.empty(b, cap, dtype=torch.float32, device="cuda")
+    (cc.cc_score_full if full else cc.cc_score_layer)(SMALL_GPU, weights, cache, mode, single, ws)
+    filled = torch.full((b, cap), float("nan"), dtype=torch.float32, device="cuda")
+    n_blocks = 4
+    for k in reversed(range(n_blocks)):   # the last rows first
+        lo = torch.tensor([n * k // n_blocks for n in seq], dtype=torch.int32, device="cuda")
+        hi = torch.tensor([n * (k + 1) // n_blocks for n in seq], dtype=torch.int32, device="cuda")
+        cc.cc_score_rows(SMALL_GPU, weights, cache, mode | cc.SCORE_RANGE_ONLY, full, lo, hi,
+                         filled, ws)
+    assert cc.cc_get_status() == cc.CC_OK
+    s, f = single.cpu().numpy(), filled.cpu().numpy()
+    for i, n in enumerate(seq):
+        assert np.array_equal(f[i, :n].view(np.uint32), s[i, :n].view(np.uint32))
+        assert np.all(np.isnan(f[i, n:]))
+
+
 def test_sharded_refresh_keep_set_and_compaction_equal_the_single_call(pkg):
     """Two ranks' blocks, the merge, then select and compaction on a replica:
     the same keep-set and the same compacted cache as the unsharded refresh."""
