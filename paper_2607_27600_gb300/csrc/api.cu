@@ -959,11 +959,19 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
     CC_TRY(launch_embed(w->embed, kv->tokens, h, d, c->vocab, sl, cap, rows, status, st, rng_lo));
   }
   const int l0 = full ? 0 : c->n_layers - 1;
+  // per-column-tile partial sums of h^2 written by the residual GEMMs for the
+  // next RMSNorm (the O projection's for the MLP norm, the down projection's
+  // for the next layer's attention norm); each is read by the GEMM right
+  // after its writer, before the next writer runs
+  float *ss_part = reinterpret_cast<float *>(wsb + L.sspart);
+  int ss_tiles = 0;   // column tiles of the attention norm's partials (0: none)
   for (int l = l0; l < c->n_layers; ++l) {
     const cc_layer_weights &lw = w->layers[l];
     const bool first_from_bf16 = !full;   // fast mode: the layer input is H^(L-1) (bf16)
-    // xn = RMSNorm(h)
-    {
+    // xn = RMSNorm(h); after the first layer of the full pass the previous
+    // down projection's epilogue has written xn = h * g (unnormalised) and
+    // the partials, and the query projection scales its rows by 1 / rms(h)
+    if (ss_tiles == 0) {
       TimedScope t(CC_KERNEL_RMSNORM, st);
       CC_TRY(launch_rmsnorm(first_from_bf16 ? kv->h_last : (const void *)h, !first_from_bf16,
                             lw.attn_norm, xn, d, c->rms_eps, sl, cap, rows, split, st, rng_lo));
@@ -974,6 +982,12 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
                         split)) != CC_OK)
       return s;
     gq.p.row_lo = rng_lo;
+    if (ss_tiles > 0) {
+      gq.p.row_ss = ss_part;
+      gq.p.n_ss = ss_tiles;
+      gq.p.ss_d = d;
+      gq.p.eps = c->rms_eps;
+    }
     gq.p.out = q;
     gq.p.ldo = split_q ? 2 * qd : qd;
     gq.p.out_split = split_q ? 1 : 0;
@@ -1002,7 +1016,6 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
     // the post-attention RMSNorm fused across the two GEMMs: this epilogue
     // writes xn = h * g (unnormalised) and per-tile sums of h^2; the gate/up
     // epilogue scales its accumulators by 1 / rms(h)
-    float *ss_part = reinterpret_cast<float *>(wsb + L.sspart);
     go.p.norm_out = reinterpret_cast<__nv_bfloat16 *>(xn);
     go.p.norm_gain = reinterpret_cast<const __nv_bfloat16 *>(lw.mlp_norm);
     go.p.ld_norm = split ? 2 * d : d;
@@ -1041,6 +1054,15 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
       gd.p.vocab = c->vocab;
       gd.p.head_part = reinterpret_cast<float2 *>(wsb + L.hpart);
       n_htiles = gd.p.n_tiles;
+    }
+    ss_tiles = 0;
+    if (full && l + 1 < c->n_layers) {   // the next layer's attention RMSNorm, fused as above
+      gd.p.norm_out = reinterpret_cast<__nv_bfloat16 *>(xn);
+      gd.p.norm_gain = reinterpret_cast<const __nv_bfloat16 *>(w->layers[l + 1].attn_norm);
+      gd.p.ld_norm = split ? 2 * d : d;
+      gd.p.norm_split = split ? 1 : 0;
+      gd.p.ss_part = ss_part;
+      ss_tiles = gd.p.n_tiles;
     }
     plan_k_splits(gd, epi_d, dev->sms, flags);
     if ((s = run_gemm(gd, epi_d, CC_KERNEL_GEMM_DOWN, dev->sms, st)) != CC_OK) return s;

@@ -71,12 +71,24 @@ CC_DEV uint8_t *out_at(const GemmParams &p, uint8_t *base, long long orow, int l
   return base + ((size_t)orow * ldo + c) * EB;
 }
 
+// The RMSNorm scale 1 / rms(x) of A row `grow` when the A rows are
+// unnormalised (x * gain, with the per-column-tile partial sums of x^2 in
+// row_ss, summed in a fixed order), else 1.
+CC_DEV float row_rms_scale(const GemmParams &p, int grow, bool valid) {
+  if (!p.row_ss || !valid) return 1.f;
+  const float *pr = p.row_ss + (size_t)grow * p.n_ss;
+  float ss = 0.f;
+  for (int t = 0; t < p.n_ss; ++t) ss += pr[t];
+  return rsqrtf(ss / (float)p.ss_d + p.eps);
+}
+
 // lo_off > 0 (bf16 only): also the lo half of each value, bf16(y - hi), at
 // element offset lo_off of the row (the precise pass's [hi | lo] queries).
+// rs: scale of the accumulator (before the bias and the rotation).
 template <int TBN, bool F8 = false>
 CC_DEV void rope_store(const GemmParams &p, uint32_t tacc, int grow, long long orow, bool valid,
                        void *out_base, int ldo, const __nv_bfloat16 *bias, int col0, int n_dest,
-                       float qscale = 1.f, bool hm = false, int lo_off = 0) {
+                       float qscale = 1.f, bool hm = false, int lo_off = 0, float rs = 1.f) {
   const int half = p.head_dim >> 1;
   valid = valid && orow >= 0;
   const uint32_t pos = valid ? (uint32_t)p.pos[grow] : 0u;
@@ -109,10 +121,10 @@ CC_DEV void rope_store(const GemmParams &p, uint32_t tacc, int grow, long long o
         float c_a, s_a, c_b, s_b;
         rope_cs(pos, p.turns[c0 + k], c_a, s_a);
         rope_cs(pos, p.turns[c0 + k + 1], c_b, s_b);
-        float a1 = __uint_as_float(x1[k]) + bf16_lo(bb1[k / 2]);
-        float a2 = __uint_as_float(x2[k]) + bf16_lo(bb2[k / 2]);
-        float b1 = __uint_as_float(x1[k + 1]) + bf16_hi(bb1[k / 2]);
-        float b2 = __uint_as_float(x2[k + 1]) + bf16_hi(bb2[k / 2]);
+        float a1 = fmaf(__uint_as_float(x1[k]), rs, bf16_lo(bb1[k / 2]));
+        float a2 = fmaf(__uint_as_float(x2[k]), rs, bf16_lo(bb2[k / 2]));
+        float b1 = fmaf(__uint_as_float(x1[k + 1]), rs, bf16_hi(bb1[k / 2]));
+        float b2 = fmaf(__uint_as_float(x2[k + 1]), rs, bf16_hi(bb2[k / 2]));
         if constexpr (F8) {   // two codes per pair, four per word
           const uint32_t e1 = pack_e4m3x2((a1 * c_a - a2 * s_a) * qscale,
                                           (b1 * c_b - b2 * s_b) * qscale);
@@ -390,9 +402,9 @@ CC_DEV void epilogue_tile(const GemmParams &p, uint32_t tacc, int grow, bool val
     if (p.kv_fp8)
       rope_store<TBN, true>(p, tacc, grow, orow, valid, p.out, p.ldo, p.bias, tile_n0, p.N,
                             p.k_qscale, hm);
-    else
+    else   // with row_ss: the query projection of unnormalised rows (x * gain)
       rope_store<TBN>(p, tacc, grow, orow, valid, p.out, p.ldo, p.bias, tile_n0, p.N, 1.f, hm,
-                      p.out_split ? p.N : 0);
+                      p.out_split ? p.N : 0, row_rms_scale(p, grow, valid));
   } else if constexpr (EPI == EPI_BF16) {    // kv_fp8: the V rows of an e4m3 cache
     const long long orow = p.kv_dest ? cache_row(p, grow, valid) : grow;
     const bool hm = p.kv_dest && p.pg.head_major;
@@ -423,13 +435,7 @@ CC_DEV void epilogue_tile(const GemmParams &p, uint32_t tacc, int grow, bool val
   } else if constexpr (EPI == EPI_SWIGLU) {
     // columns [0,128) = gate rows nt*128.., [128,256) = up rows nt*128..
     __nv_bfloat16 *out = reinterpret_cast<__nv_bfloat16 *>(p.out) + (size_t)grow * p.ldo;
-    float rs = 1.f;   // the input row's RMSNorm scale (row_ss: A rows unnormalised)
-    if (p.row_ss && valid) {
-      const float *pr = p.row_ss + (size_t)grow * p.n_ss;
-      float ss = 0.f;
-      for (int t = 0; t < p.n_ss; ++t) ss += pr[t];
-      rs = rsqrtf(ss / (float)p.ss_d + p.eps);
-    }
+    const float rs = row_rms_scale(p, grow, valid);   // row_ss: A rows unnormalised
 #pragma unroll 1
     for (int c0 = 0; c0 < 128; c0 += 32) {
       uint32_t g[32], u[32];

@@ -51,9 +51,9 @@ struct GemmParams {
   const __nv_bfloat16 *norm_gain;
   int ld_norm, norm_split;
   float *ss_part;
-  // EPI_SWIGLU with row_ss: the A rows are unnormalised (as above); the
-  // accumulators are scaled by rsqrt(sum_t row_ss[row][t] / ss_d + eps),
-  // t < n_ss, before the activation
+  // EPI_SWIGLU / EPI_QROPE with row_ss: the A rows are unnormalised (as
+  // above); the accumulators are scaled by rsqrt(sum_t row_ss[row][t] / ss_d
+  // + eps), t < n_ss, before the activation (before the bias and RoPE)
   const float *row_ss;
   int n_ss, ss_d;
   float eps;
