@@ -271,6 +271,8 @@ def algorithmic_work(wl, kv_bytes=2):
         "compact": ("hbm", 2.0 * moved * (n_arrays_kv * kv_row + h_row + 8)),
         # at most 9 passes over the scores (up to 8 radix passes + the emit pass)
         "select": ("hbm", 9.0 * 4.0 * n_rows),
+        # an e4m3 layer's K and V codes read, their bf16 copies written (per launch)
+        "kv_dequant": ("hbm", n_rows * 2.0 * s.n_kv_heads * dh * 3.0),
     }
 
 
@@ -433,18 +435,21 @@ def refresh_record(args, dist, wl, w, pristine, mode, steps, with_e2e=True, with
     clocks = ClockSampler(dist.local)
     clocks.start()
     time.sleep(0.3)
-    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-          for _ in range(steps)]
+    # (a third event between the scoring and select: the scoring pass's own time)
+    ev = [tuple(torch.cuda.Event(enable_timing=True) for _ in range(3)) for _ in range(steps)]
     dist.barrier()
     torch.cuda.synchronize(dev)
     for i in range(steps):
         prepare()
         ev[i][0].record(stream)
-        step()
+        score()
+        ev[i][2].record(stream)
+        select_compact()
         ev[i][1].record(stream)
     torch.cuda.synchronize(dev)
     dist.barrier()
-    step_ms = [a.elapsed_time(bb) for a, bb in ev]
+    step_ms = [a.elapsed_time(bb) for a, bb, _ in ev]
+    score_ms = dist.max(sum(a.elapsed_time(c) for a, _, c in ev) / steps)
     ref_idx, ref_cnt = keep_idx.cpu(), keep_count.cpu()   # the last timed step's keep-set
     # per-kernel table: the same steps again with CUDA events around every
     # library launch (kept out of the timed steps above, whose launches they
@@ -500,6 +505,10 @@ def refresh_record(args, dist, wl, w, pristine, mode, steps, with_e2e=True, with
     rec = {
         "workload": wl.name, "value": round(value, 1), "unit": "positions/s",
         "ms_per_step": round(ms, 4), "steps": steps,
+        # the metric's other form: positions per second of the scoring pass alone
+        "score_only": {"value": round(positions * (1 if row_shard is not None else dist.world) /
+                                      (score_ms * 1e-3), 1),
+                       "unit": "positions/s", "ms": round(score_ms, 4)},
         "mode": ("precise: [hi | lo] bf16 pairs for activations, queries and P"
                  if precise else "bf16 operands, fp32 accumulation"),
         "pass": ("fast single-layer" if fast else f"full {shape.n_layers}-layer")
@@ -891,8 +900,8 @@ def suite_line(args, dist, wl, head, cache_src, records):
                                    f"rows, MAX all-reduce of the scores)" if args.shard == "rows"
                                    else f"replicas x{dist.world}")},
     }
-    for key in ("shard", "e2e", "gpu_launches", "roofline", "kernels", "tflops_per_step_achieved",
-                "clocks", "cpu_baseline", "cycles", "value_basis"):
+    for key in ("score_only", "shard", "e2e", "gpu_launches", "roofline", "kernels",
+                "tflops_per_step_achieved", "clocks", "cpu_baseline", "cycles", "value_basis"):
         if key in head:
             line[key] = head[key]
     if wl.paper_positions_per_s and args.scorer == "counter-causal":

@@ -63,8 +63,8 @@ typedef enum {
    * pass).  Weights, cached K/V and H^(L-1) are bf16 inputs and stay exact.
    * Without it a deep random-weight model drifts from the exact score over
    * depth by several percent; with it the 32-layer score stays within
-   * ~1e-3.  With an e4m3 cache the attention operands are f16 and the
-   * queries and P stay single. */
+   * ~1e-3.  An e4m3 cache's codes enter the attention as exact bf16
+   * values (the scales applied in fp32), so the same holds. */
   CC_SCORE_PRECISE = 0x100,
   /* Flag, OR-ed into the mode of cc_score_rows: the rows of the range are
    * written and every other entry of scores (other rows, slots past the
@@ -80,7 +80,10 @@ typedef enum {
  * scoring passes, the compaction, cc_append_chunk and cc_decode_step take
  * either format (appends write codes rounded to nearest, saturating at
  * +-448); the attention-based comparison scorers and
- * cc_counter_causal_attention take bf16 only (CC_ERR_UNSUPPORTED). */
+ * cc_counter_causal_attention take bf16 only (CC_ERR_UNSUPPORTED).  The
+ * scoring passes and the append attend over an exact bf16 copy of each
+ * layer's codes, made in the workspace's activation buffer (which needs
+ * 4 * Hkv * head_dim <= 2 * d_ff bytes per slot, else CC_ERR_UNSUPPORTED). */
 typedef enum {
   CC_KV_BF16 = 0,
   CC_KV_E4M3 = 1

@@ -148,7 +148,7 @@ _SIGS = {
     "cc_kernel_name": (ctypes.c_char_p, [ctypes.c_int32]),
     "cc_debug_withhold_compact_unit": (ctypes.c_int, [ctypes.c_int32]),
 }
-KERNEL_COUNT = 18
+KERNEL_COUNT = 19
 
 
 def library_path() -> str:

@@ -505,11 +505,38 @@ cc_status run_attention(const cc_model_cfg *c, const void *q, const void *k, con
                         cudaStream_t st, bool split = false, const int32_t *row_lo = nullptr,
                         int q_span = 0, const AttnPartials *parts = nullptr, int sms = 0,
                         KvFmt kvf = KvFmt(), bool q_split = false,
-                        const int32_t *range_lo = nullptr, const int32_t *range_hi = nullptr) {
+                        const int32_t *range_lo = nullptr, const int32_t *range_hi = nullptr,
+                        void *kv_scratch = nullptr, size_t kv_scratch_bytes = 0) {
   const int G = c->n_q_heads / c->n_kv_heads, dh = c->head_dim;
   const int P = attn_positions_per_unit(G);
   const uint64_t R = (uint64_t)batch * cap;
-  if (q_split && (row_lo || kvf.fp8)) return CC_ERR_UNSUPPORTED;
+  if (q_split && row_lo) return CC_ERR_UNSUPPORTED;
+  // one query row per sequence: the decode kernel, which reads either format
+  const long long units0 = (long long)batch * c->n_kv_heads *
+                           (((row_lo ? q_span : cap) + P - 1) / P);
+  const bool decode = row_lo && q_span == 1 && G <= kDecMaxG && parts && parts->o && parts->ml &&
+                      units0 <= kAttnMaxSplitSlots;
+  if (kvf.fp8 && !decode) {
+    // the tile attention over an e4m3 cache: the layer's codes as bf16 (exact)
+    // in a slot-major scratch, the scales kept folded into the softmax scale
+    // and the output normalisation
+    const size_t half = R * c->n_kv_heads * dh * 2;
+    if (!kv_scratch || kv_scratch_bytes < 2 * half) return CC_ERR_UNSUPPORTED;
+    __nv_bfloat16 *ks = reinterpret_cast<__nv_bfloat16 *>(kv_scratch);
+    __nv_bfloat16 *vs = reinterpret_cast<__nv_bfloat16 *>(reinterpret_cast<uint8_t *>(kv_scratch) + half);
+    {
+      TimedScope t(CC_KERNEL_KV_DEQUANT, st);
+      CC_TRY(launch_kv_to_bf16(reinterpret_cast<const uint8_t *>(k),
+                               reinterpret_cast<const uint8_t *>(v), kvf.pg, cap, c->n_kv_heads,
+                               dh, seq_len, batch, ks, vs, status, st));
+    }
+    k = ks;
+    v = vs;
+    kvf.fp8 = false;
+    kvf.pg = KvLayout{};
+    kvf.pg.hkv = c->n_kv_heads;
+    kvf.rows = R;
+  }
   CUtensorMap tq, tk, tv;
   {
     // q_split: rows [hi heads | lo heads], the map spans both (lo at head Hq + t)
@@ -523,21 +550,13 @@ cc_status run_attention(const cc_model_cfg *c, const void *q, const void *k, con
   const bool hm = kvf.pg.head_major != 0;
   // slot-major maps (dh, Hkv, rows), box (.., 1, 128 slots); head-major maps
   // (dh, cap, batch*Hkv), box (.., 128 slots, 1): the same shared-memory image
-  const int eb = kvf.fp8 ? 1 : 2;
+  // (the tile kernel's maps: bf16; an e4m3 cache reaches here only for the
+  // decode kernel, which reads the raw buffers)
   const uint64_t kv_dims[3] = {(uint64_t)dh, hm ? (uint64_t)cap : (uint64_t)c->n_kv_heads,
                                hm ? (uint64_t)batch * c->n_kv_heads : RK};
-  const uint64_t kv_strides[2] = {(uint64_t)dh * eb,
-                                  hm ? (uint64_t)cap * dh * eb : (uint64_t)c->n_kv_heads * dh * eb};
-  if (kvf.fp8) {   // e4m3 bytes, one unswizzled box per 128-key tile (converted in the kernel)
-    const uint64_t *dims = kv_dims;
-    const uint64_t *strides = kv_strides;
-    const uint32_t box[3] = {(uint32_t)dh, hm ? 128u : 1u, hm ? 1u : 128u};
-    if (!make_tmap(&tk, k, 3, dims, strides, box, CU_TENSOR_MAP_SWIZZLE_NONE,
-                   CU_TENSOR_MAP_DATA_TYPE_UINT8) ||
-        !make_tmap(&tv, v, 3, dims, strides, box, CU_TENSOR_MAP_SWIZZLE_NONE,
-                   CU_TENSOR_MAP_DATA_TYPE_UINT8))
-      return tmap_fail();
-  } else {
+  const uint64_t kv_strides[2] = {(uint64_t)dh * 2,
+                                  hm ? (uint64_t)cap * dh * 2 : (uint64_t)c->n_kv_heads * dh * 2};
+  if (!kvf.fp8) {
     const uint32_t box[3] = {64, hm ? 128u : 1u, hm ? 1u : 128u};
     if (!make_tmap(&tk, k, 3, kv_dims, kv_strides, box)) return tmap_fail();
     if (!make_tmap(&tv, v, 3, kv_dims, kv_strides, box)) return tmap_fail();
@@ -569,8 +588,7 @@ cc_status run_attention(const cc_model_cfg *c, const void *q, const void *k, con
   p.row_hi = row_lo ? nullptr : range_hi;
   p.q_span = row_lo ? q_span : cap;
   const long long units = attn_units(p);
-  if (row_lo && q_span == 1 && G <= kDecMaxG && parts && parts->o && parts->ml &&
-      units <= kAttnMaxSplitSlots) {   // one query row per sequence: the decode kernel
+  if (decode) {   // one query row per sequence: the decode kernel
     p.kv_splits = attn_decode_splits(units, cap, sms);
     p.part_o = parts->o;
     p.part_ml = parts->ml;
@@ -824,8 +842,10 @@ cc_status run_append(const cc_model_cfg *c, const cc_model_weights *w, const cc_
       if ((s = run_gemm(g, pj.epi, pj.kind, dev->sms, st)) != CC_OK) return s;
     }
     // o = attention of the chunk rows over the memory and the chunk (causal)
+    // (act is free until the MLP: an e4m3 layer's bf16 copy for the tile attention)
     if ((s = run_attention(c, q, kv->k[l], kv->v[l], o, hi, batch, cap, status, st, false, lo,
-                           max_count, &parts, dev->sms, kvf)) != CC_OK)
+                           max_count, &parts, dev->sms, kvf, false, nullptr, nullptr, act,
+                           (size_t)batch * cap * c->d_ff * 2)) != CC_OK)
       return s;
     // h += o Wo^T; xn = RMSNorm(h); act = SwiGLU; h += act Wd^T
     if (use_gemv) {
@@ -937,9 +957,9 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
   const int batch = kv->batch, cap = kv->cap, rows = batch * cap;
   const int d = c->d_model, qd = c->n_q_heads * c->head_dim, f = c->d_ff;
   const bool split = (mode & CC_SCORE_PRECISE) != 0;   // [hi | lo] GEMM activations
-  // [hi | lo] queries and attention probabilities too (a bf16 cache; with an
-  // e4m3 cache the attention's operands are f16 and the queries stay single)
-  const bool split_q = split && kv->kv_format != CC_KV_E4M3;
+  // [hi | lo] queries and attention probabilities too (an e4m3 cache's layers
+  // enter the attention as exact bf16 copies)
+  const bool split_q = split;
   const ScoreWs L = score_layout(c, batch, cap, mode, split);
   const bool logit = (mode & 0xFF) == CC_SCORE_LOGIT;
   const bool keep_outside = (mode & CC_SCORE_RANGE_ONLY) != 0;   // other entries untouched
@@ -998,9 +1018,11 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
     if ((s = run_gemm(gq, EPI_QROPE, CC_KERNEL_GEMM_QROPE, dev->sms, st)) != CC_OK) return s;
     // O = counter-causal attention
     CC_TRY(wait_kv_ready(kv, l, l + 1, st));
+    // (act is free until the MLP: an e4m3 layer's bf16 copy for the tile attention)
     if ((s = run_attention(c, q, kv->k[l], kv->v[l], o, kv->seq_len, batch, cap, status, st,
                            split, nullptr, 0, nullptr, 0, kv_fmt(c, kv, l), split_q, rng_lo,
-                           rng_hi)) != CC_OK)
+                           rng_hi, act, (size_t)batch * cap * c->d_ff * 2 * (split ? 2 : 1))) !=
+        CC_OK)
       return s;
     // h = h + O Wo^T  (fast mode: h = H^(L-1) + O Wo^T)
     Gemm go;
@@ -1684,7 +1706,7 @@ const char *cc_kernel_name(int32_t kind) {
   static const char *names[CC_KERNEL_COUNT] = {
       "rmsnorm", "embed", "gemm_qrope", "attention", "gemm_oproj", "gemm_gateup", "gemm_down",
       "head_logit", "gemm_lmhead", "lse_combine", "select", "compact", "other",
-      "gemm_kv", "attention_causal", "append", "gemm_qkv", "keyattn"};
+      "gemm_kv", "attention_causal", "append", "gemm_qkv", "keyattn", "kv_dequant"};
   return (kind >= 0 && kind < CC_KERNEL_COUNT) ? names[kind] : "unknown";
 }
 

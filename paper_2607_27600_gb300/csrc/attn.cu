@@ -25,12 +25,9 @@
 //   warp 10           tcgen05.mma issuer of M-half 1
 //   warp 11           idle (completes the third warpgroup)
 //
-// With an e4m3 cache (FP8) warp 9 issues both halves' products and warps 10
-// and 11 convert: Q bf16 -> f16 once, then every K and V tile from the fp8
-// staging buffer (TMA, unswizzled) into the 128-byte-swizzled f16 stage the
-// MMA reads, zeroing V rows past the sequence end; the MMAs then run on f16
-// operands (Q, K, V and P all f16: e4m3 -> f16 is exact), the K scale folded
-// into the softmax scale and the V scale into the output normalisation.
+// An e4m3 cache reaches this kernel as an exact bf16 copy of the layer's
+// codes (made by the caller), its K scale folded into the softmax scale and
+// its V scale into the output normalisation.
 //
 // SPLIT (the precise scoring pass over a bf16 cache): the queries arrive as
 // bf16 pairs hi + lo (hi = bf16(q), lo = bf16(q - hi)), so S = Q_hi K^T +
@@ -49,18 +46,16 @@ namespace cc {
 namespace {
 
 constexpr int BKV = 128;        // keys per tile
-constexpr bool kFp8TwoIssuers = false;  // e4m3 cache: one issuer, two converter warps (measured: turn-taking issuers with one converter warp are slower, 1.13 vs 0.65 ms at 8k)
 constexpr int KST = 2;          // K and V pipeline stages
 constexpr int kThreads = 384;   // 3 warpgroups: softmax 0, softmax 1, producer/MMA
 // Register split after launch (setmaxnreg): the block is launched with 168
 // registers per thread (64512 in all); the producer/MMA warpgroup gives some
-// up and the two softmax warpgroups take them: bf16 operands 224 / 56, an
-// e4m3 cache (whose converters run in the third warpgroup) 208 / 88 -- the
-// splits at which each variant compiles without (or, split operands, with the
-// fewest) spills; 2 * 128 * softmax + 128 * producer <= 384 * 168.
+// up and the two softmax warpgroups take them (224 / 56: the split at which
+// the kernel compiles without spills, the split-operand variant with the
+// fewest); 2 * 128 * softmax + 128 * producer <= 384 * 168.
 constexpr int kRegsLaunch = 168;
-template <bool FP8> struct RegSplit {
-  static constexpr int softmax = FP8 ? 208 : 224, producer = FP8 ? 88 : 56;
+struct RegSplit {
+  static constexpr int softmax = 224, producer = 56;
   static_assert(2 * 128 * softmax + 128 * producer <= kThreads * kRegsLaunch,
                 "register split exceeds the launch allocation");
 };
@@ -75,42 +70,28 @@ CC_DEV float fast_exp2(float x) {
 }
 
 
-template <int DH, bool FP8 = false, bool SPLIT = false>
+template <int DH, bool SPLIT = false>
 struct AttnSmem {
   static constexpr int NH = DH / 64;                 // 64-element (128-byte) column halves
   static constexpr int Q_BYTES = NH * 256 * 128;     // 256 rows
   static constexpr int KV_BYTES = NH * BKV * 128;    // one K (or V) tile (2-byte elements)
   // V stages: one when the second (lo) Q tile of SPLIT leaves no room for two
   static constexpr int KSTV = (SPLIT && DH == 128) ? 1 : KST;
-  // FP8, head_dim 128: the fp8 tile lands in the upper half of its own f16
-  // stage and is expanded in place (no staging); head_dim 64: one staging
-  // buffer per K and V
-  static constexpr bool IN_PLACE = FP8 && DH == 128;
-  static constexpr int FP8_TILE = BKV * DH;            // bytes of one fp8 K (or V) tile
-  static constexpr int STG_BYTES = (FP8 && !IN_PLACE) ? FP8_TILE : 0;
   static constexpr int OFF_Q = 0;
   static constexpr int OFF_QLO = OFF_Q + Q_BYTES;          // SPLIT: the lo tile of Q
   static constexpr int OFF_K = OFF_QLO + (SPLIT ? Q_BYTES : 0);
   static constexpr int OFF_V = OFF_K + KST * KV_BYTES;
-  static constexpr int OFF_STG = OFF_V + KSTV * KV_BYTES;  // [K, V] staging (FP8)
-  static constexpr int OFF_BAR = OFF_STG + 2 * STG_BYTES;
+  static constexpr int OFF_BAR = OFF_V + KSTV * KV_BYTES;
   static constexpr int BYTES = OFF_BAR + 256 + 1024;   // barriers + alignment slack
   static_assert(BYTES <= 232448, "shared memory of a CTA exceeds 227 KB");
-  static_assert(!(SPLIT && FP8), "split queries take bf16 K/V operands");
 };
 
-// e4m3 pair (low 16 bits) -> f16 pair, exact; bf16 pair -> f16 pair; f16 pack.
+// e4m3 pair (low 16 bits) -> f16 pair, exact (the decode kernel's e4m3 cache).
 CC_DEV uint32_t e4m3x2_to_f16x2(uint32_t two) {
   uint32_t r;
   asm("cvt.rn.f16x2.e4m3x2 %0, %1;" : "=r"(r) : "h"((unsigned short)(two & 0xFFFFu)));
   return r;
 }
-CC_DEV uint32_t pack_f16x2(float lo, float hi) {
-  uint32_t r;
-  asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
-  return r;
-}
-CC_DEV uint32_t bf16x2_to_f16x2(uint32_t w) { return pack_f16x2(bf16_lo(w), bf16_hi(w)); }
 
 // Work unit `unit_id` -> (sequence b, KV head g, positions p0..p_last).
 // Counter-causal rows run over [row_lo, row_hi) when a range is given (keys
@@ -152,16 +133,11 @@ CC_DEV UnitInfo decode_unit(const AttnParams &p, int unit_id, bool causal) {
   return u;
 }
 
-template <int DH, bool CAUSAL, bool FP8, bool SPLIT>
+template <int DH, bool CAUSAL, bool SPLIT>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                 const __grid_constant__ CUtensorMap tmV, const __grid_constant__ AttnParams p) {
-  using L = AttnSmem<DH, FP8, SPLIT>;
-  // two turn-taking issuers (warps 9, 10); with an e4m3 cache warp 11 alone
-  // converts (kFp8TwoIssuers), else warp 9 issues both halves and warps 10-11 convert
-  constexpr bool kTwoIssuers = !FP8 || kFp8TwoIssuers;
-  constexpr int kConvWarp0 = kTwoIssuers ? 11 : 10;            // FP8: first converter warp
-  constexpr int kConvThreads = (12 - kConvWarp0) * 32;
+  using L = AttnSmem<DH, SPLIT>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                               ~uintptr_t(1023));
@@ -175,12 +151,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t *s_ready = v_fixed + 1;         // [2]
   uint64_t *p_ready = s_ready + 2;         // [2] (keys 0..63 of P when split)
   uint64_t *o_done = p_ready + 2;          // [2]
-  uint64_t *stg_full = o_done + 2;         // [2] FP8: fp8 K / V tile in the staging buffer
-  uint64_t *stg_empty = stg_full + 2;      // [2] FP8: staging converted (free)
-  uint64_t *q_conv = stg_empty + 2;        // FP8: Q converted to f16
-  uint64_t *k_load = q_conv + 1;           // [KST] FP8 in place: fp8 K tile in stage s
-  uint64_t *v_load = k_load + KST;         // [KST] FP8 in place: fp8 V tile in stage s
-  uint64_t *turn = v_load + KST;           // [2] two issuers: issuer h may issue its next burst
+  uint64_t *turn = o_done + 2;             // [2] two issuers: issuer h may issue its next burst
   uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(turn + 2);
   volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
 
@@ -242,24 +213,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   // and the barrier.
   if (warp == 8 && lane == 0) {
     mbar_init(q_full, 1);
-    for (int s = 0; s < KST; ++s) {   // FP8: K/V stages are filled by the 64 converter threads
-      mbar_init(&k_full[s], FP8 ? kConvThreads : 1);
-      mbar_init(&k_empty[s], kTwoIssuers ? 2 : 1);   // one commit per MMA issuer
-      mbar_init(&v_full[s], FP8 ? kConvThreads : 1);
-      mbar_init(&v_empty[s], kTwoIssuers ? 2 : 1);
+    for (int s = 0; s < KST; ++s) {
+      mbar_init(&k_full[s], 1);
+      mbar_init(&k_empty[s], 2);   // one commit per MMA issuer
+      mbar_init(&v_full[s], 1);
+      mbar_init(&v_empty[s], 2);
     }
     mbar_init(v_fixed, 1);
-    if (FP8) {
-      for (int i = 0; i < 2; ++i) {
-        mbar_init(&stg_full[i], 1);
-        mbar_init(&stg_empty[i], kConvThreads);
-      }
-      mbar_init(q_conv, kConvThreads);
-      for (int s = 0; s < KST; ++s) {
-        mbar_init(&k_load[s], 1);
-        mbar_init(&v_load[s], 1);
-      }
-    }
     for (int h = 0; h < 2; ++h) {
       mbar_init(&turn[h], 1);
       mbar_init(&s_ready[h], 1);
@@ -298,63 +258,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   if (warp >= 8) {
-    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(RegSplit<FP8>::producer));
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(RegSplit::producer));
     if (warp == 8) {
     // ------------------------------------------------------------ producer
     // (the Q tile was requested before the CTA-wide barrier)
-    if constexpr (L::IN_PLACE) {
-      // fp8 tiles into the upper half of their own stage (converted in place)
-      for (int it = 0; it < ntiles; ++it) {
-        const int t = t_hi - it, s = it % KST;
-        const uint32_t ph = (it / KST) & 1;
-        const int krow = tile_row(t);
-        // TMA coordinates after the head_dim one: (KV head, row), or head-major (slot, b*Hkv + g)
-        const int kc1 = p.pg.head_major ? t * BKV : g;
-        const int kc2 = p.pg.head_major ? b * p.n_kv_heads + g : krow;
-        int ok = 1;
-        if (lane == 0) {
-          ok = mbar_wait(&k_empty[s], ph ^ 1, abort_flag, p.status);
-          if (ok) {
-            mbar_arrive_expect_tx(&k_load[s], L::FP8_TILE);
-            tma_load_3d(smem + L::OFF_K + s * L::KV_BYTES + L::KV_BYTES / 2, &tmK, &k_load[s], 0,
-                        kc1, kc2);
-            ok = mbar_wait(&v_empty[s], ph ^ 1, abort_flag, p.status);
-          }
-          if (ok) {
-            mbar_arrive_expect_tx(&v_load[s], L::FP8_TILE);
-            tma_load_3d(smem + L::OFF_V + s * L::KV_BYTES + L::KV_BYTES / 2, &tmV, &v_load[s], 0,
-                        kc1, kc2);
-          }
-        }
-        ok = __shfl_sync(0xFFFFFFFFu, ok, 0);
-        if (!ok) break;
-      }
-    } else if constexpr (FP8) {
-      // fp8 tiles into the one staging buffer; the converters fill the stages
-      for (int it = 0; it < ntiles; ++it) {
-        const int t = t_hi - it;
-        const uint32_t sp = it & 1;
-        const int krow = tile_row(t);
-        // TMA coordinates after the head_dim one: (KV head, row), or head-major (slot, b*Hkv + g)
-        const int kc1 = p.pg.head_major ? t * BKV : g;
-        const int kc2 = p.pg.head_major ? b * p.n_kv_heads + g : krow;
-        int ok = 1;
-        if (lane == 0) {
-          ok = mbar_wait(&stg_empty[0], sp ^ 1, abort_flag, p.status);
-          if (ok) {
-            mbar_arrive_expect_tx(&stg_full[0], L::STG_BYTES);
-            tma_load_3d(smem + L::OFF_STG, &tmK, &stg_full[0], 0, kc1, kc2);
-            ok = mbar_wait(&stg_empty[1], sp ^ 1, abort_flag, p.status);
-          }
-          if (ok) {
-            mbar_arrive_expect_tx(&stg_full[1], L::STG_BYTES);
-            tma_load_3d(smem + L::OFF_STG + L::STG_BYTES, &tmV, &stg_full[1], 0, kc1, kc2);
-          }
-        }
-        ok = __shfl_sync(0xFFFFFFFFu, ok, 0);
-        if (!ok) break;
-      }
-    } else {
+    {
       for (int it = 0; it < ntiles; ++it) {
         const int t = t_hi - it, s = it % KST;   // key tiles from the sequence end downwards
         const uint32_t ph = (it / KST) & 1;
@@ -398,10 +306,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
     }
-    } else if (warp == 9 || (kTwoIssuers && warp == 10)) {
+    } else if (warp == 9 || warp == 10) {
     // ------------------------------------------------------------ MMA issuers
-    // One issuing thread per M-half (warp 9: half 0, warp 10: half 1), or
-    // warp 9 for both halves with an e4m3 cache (warps 10-11 convert).  An
+    // One issuing thread per M-half (warp 9: half 0, warp 10: half 1).  An
     // issuing thread blocks while the tensor pipe's short queue is full, so a
     // lone issuer leaves the pipe idle during its own barrier waits between
     // bursts.  Two issuers take turns: a burst is one half's products for
@@ -414,12 +321,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     // (PV(t) before QK(t+1): P lives in S's columns), so every result is
     // deterministic.
     if (lane == 0) {
-      const int h_lo = kTwoIssuers ? warp - 9 : 0, h_hi = kTwoIssuers ? warp - 9 : 1;
-      // FP8: every operand (Q, K, V, P) is f16; otherwise every operand is bf16
-      constexpr uint32_t idesc_qk =
-          FP8 ? make_idesc_f16(128, BKV, 0, 0) : make_idesc_bf16(128, BKV, 0, 0);
-      constexpr uint32_t idesc_pv =
-          FP8 ? make_idesc_f16(128, DH, 0, 1) : make_idesc_bf16(128, DH, 0, 1);
+      const int h_lo = warp - 9, h_hi = warp - 9;   // this issuer's M-half
+      constexpr uint32_t idesc_qk = make_idesc_bf16(128, BKV, 0, 0);   // every operand bf16
+      constexpr uint32_t idesc_pv = make_idesc_bf16(128, DH, 0, 1);
       // Shared-memory descriptors built once; a K step only advances the
       // start-address field (16-byte units): +2 per 16 columns of a 128-byte
       // row (Q, K), +128 per 16 keys of V.
@@ -464,15 +368,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       // burst (half 0 opens; half 1's burst kb follows half 0's burst kb)
       int kb = 0;
       auto take_turn = [&]() -> bool {
-        if (!kTwoIssuers) return true;
         if (h_lo == 0) return kb == 0 || mbar_wait(&turn[0], (kb - 1) & 1, abort_flag, p.status);
         return mbar_wait(&turn[1], kb & 1, abort_flag, p.status);
       };
       auto pass_turn = [&]() {
-        if (kTwoIssuers) mbar_arrive(&turn[1 - h_lo]);
+        mbar_arrive(&turn[1 - h_lo]);
         ++kb;
       };
-      bool ok = mbar_wait(FP8 ? q_conv : q_full, 0, abort_flag, p.status);
+      bool ok = mbar_wait(q_full, 0, abort_flag, p.status);
       if (ok) ok = mbar_wait(&k_full[0], 0, abort_flag, p.status);
       if (ok) ok = take_turn();
       if (ok) {
@@ -487,7 +390,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int t = t_hi - it, s = it % L::KSTV;   // V stage
         const uint32_t ph = (it / L::KSTV) & 1;
         if (!(ok = mbar_wait(&v_full[s], ph, abort_flag, p.status))) break;
-        if (!FP8 && t == t_top && n - t * BKV < BKV)
+        if (t == t_top && n - t * BKV < BKV)
           if (!(ok = mbar_wait(v_fixed, 0, abort_flag, p.status))) break;
         for (int h = h_lo; h <= h_hi; ++h) {
           if (!(ok = mbar_wait(&p_ready[h], it & 1, abort_flag, p.status))) break;
@@ -518,98 +421,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
     }
-    } else if (FP8 && warp >= kConvWarp0) {
-    // ------------------------------------------------------------ converters (FP8)
-    const int ct = threadIdx.x - kConvWarp0 * 32;   // 0 .. kConvThreads - 1
-    bool ok = mbar_wait(q_full, 0, abort_flag, p.status);
-    if (ok) {   // Q bf16 -> f16 in place (same layout, element by element)
-      uint4 *qv = reinterpret_cast<uint4 *>(smem + L::OFF_Q);
-      for (int i = ct; i < L::Q_BYTES / 16; i += kConvThreads) {
-        uint4 x = qv[i];
-        x.x = bf16x2_to_f16x2(x.x);
-        x.y = bf16x2_to_f16x2(x.y);
-        x.z = bf16x2_to_f16x2(x.z);
-        x.w = bf16x2_to_f16x2(x.w);
-        qv[i] = x;
-      }
-      fence_proxy_async_smem();
-      mbar_arrive(q_conv);
-    }
-    // fp8 [BKV][DH] (row r, 8 elements at column 8j) -> f16 stage: 128-byte
-    // rows per 64-column half, 16-byte chunk c of row r at chunk c ^ (r & 7)
-    // (the TMA's 128-byte swizzle); rows >= zero_from are written as zeros
-    auto convert = [&](const uint8_t *src, uint8_t *dst, int zero_from) {
-      for (int i = ct; i < BKV * L::NH * 8; i += kConvThreads) {
-        const int r = i / (L::NH * 8), rem = i - r * (L::NH * 8), hh = rem >> 3, c = rem & 7;
-        uint4 o = make_uint4(0, 0, 0, 0);
-        if (r < zero_from) {
-          const uint2 x = *reinterpret_cast<const uint2 *>(src + r * DH + hh * 64 + c * 8);
-          o.x = e4m3x2_to_f16x2(x.x);
-          o.y = e4m3x2_to_f16x2(x.x >> 16);
-          o.z = e4m3x2_to_f16x2(x.y);
-          o.w = e4m3x2_to_f16x2(x.y >> 16);
-        }
-        *reinterpret_cast<uint4 *>(dst + hh * BKV * 128 + r * 128 + ((c ^ (r & 7)) << 4)) = o;
-      }
-      fence_proxy_async_smem();
-    };
-    // head_dim 128 in place: the fp8 tile sits in the stage's upper 16 KB
-    // (row r = 128 bytes at 16K + 128 r); 8 lanes own a row, lane j its bytes
-    // 16j..16j+15 (dims 16j..16j+15).  The f16 row r of the upper column
-    // half occupies exactly the bytes of fp8 row r, so the 8 lanes read the
-    // whole row before any of them writes (syncwarp); rows are split between
-    // the two warps, so no other warp touches them.
-    auto convert_in_place = [&](uint8_t *base, int zero_from) {
-      const int j = ct & 7;
-      const int hh = j >> 2, c = (j & 3) * 2;
-      for (int r = ct >> 3; r < BKV; r += kConvThreads / 8) {
-        const uint4 x = *reinterpret_cast<const uint4 *>(base + L::KV_BYTES / 2 + r * 128 + j * 16);
-        __syncwarp();
-        uint4 a = make_uint4(0, 0, 0, 0), b = make_uint4(0, 0, 0, 0);
-        if (r < zero_from) {
-          a = make_uint4(e4m3x2_to_f16x2(x.x), e4m3x2_to_f16x2(x.x >> 16), e4m3x2_to_f16x2(x.y),
-                         e4m3x2_to_f16x2(x.y >> 16));
-          b = make_uint4(e4m3x2_to_f16x2(x.z), e4m3x2_to_f16x2(x.z >> 16), e4m3x2_to_f16x2(x.w),
-                         e4m3x2_to_f16x2(x.w >> 16));
-        }
-        uint8_t *row = base + hh * BKV * 128 + r * 128;
-        *reinterpret_cast<uint4 *>(row + ((c ^ (r & 7)) << 4)) = a;
-        *reinterpret_cast<uint4 *>(row + (((c + 1) ^ (r & 7)) << 4)) = b;
-      }
-      fence_proxy_async_smem();
-    };
-    if constexpr (L::IN_PLACE) {
-      for (int it = 0; ok && it < ntiles; ++it) {
-        const int t = t_hi - it, s = it % KST;
-        const uint32_t ph = (it / KST) & 1;
-        if (!(ok = mbar_wait(&k_load[s], ph, abort_flag, p.status))) break;
-        convert_in_place(smem + L::OFF_K + s * L::KV_BYTES, BKV);
-        mbar_arrive(&k_full[s]);
-        if (!(ok = mbar_wait(&v_load[s], ph, abort_flag, p.status))) break;
-        const int keep = (t == t_top && n - t * BKV < BKV) ? n - t * BKV : BKV;
-        convert_in_place(smem + L::OFF_V + s * L::KV_BYTES, keep);
-        mbar_arrive(&v_full[s]);
-      }
-    }
-    for (int it = 0; !L::IN_PLACE && ok && it < ntiles; ++it) {
-      const int t = t_hi - it, s = it % KST;
-      const uint32_t ph = (it / KST) & 1, sp = it & 1;
-      if (!(ok = mbar_wait(&stg_full[0], sp, abort_flag, p.status))) break;
-      if (!(ok = mbar_wait(&k_empty[s], ph ^ 1, abort_flag, p.status))) break;
-      convert(smem + L::OFF_STG, smem + L::OFF_K + s * L::KV_BYTES, BKV);
-      mbar_arrive(&stg_empty[0]);
-      mbar_arrive(&k_full[s]);
-      if (!(ok = mbar_wait(&stg_full[1], sp, abort_flag, p.status))) break;
-      if (!(ok = mbar_wait(&v_empty[s], ph ^ 1, abort_flag, p.status))) break;
-      // V rows past the sequence end may hold any bits (0 * NaN would poison O)
-      const int keep = (t == t_top && n - t * BKV < BKV) ? n - t * BKV : BKV;
-      convert(smem + L::OFF_STG + L::STG_BYTES, smem + L::OFF_V + s * L::KV_BYTES, keep);
-      mbar_arrive(&stg_empty[1]);
-      mbar_arrive(&v_full[s]);
-    }
     }
   } else {
-    asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(RegSplit<FP8>::softmax));
+    asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(RegSplit::softmax));
     // ------------------------------------------------------------ softmax
     const int h = warp >> 2, q = warp & 3;
     const int R = h * 128 + q * 32 + lane;              // unit row
@@ -697,7 +511,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           const float2 y = __ffma2_rn(make_float2(__uint_as_float(sr[c0 + k]),
                                                   __uint_as_float(sr[c0 + k + 1])), sl2v, nmv);
           const float2 e = make_float2(fast_exp2(y.x), fast_exp2(y.y));
-          pk[k / 2] = FP8 ? pack_f16x2(e.x, e.y) : pack_bf16x2(e.x, e.y);
+          pk[k / 2] = pack_bf16x2(e.x, e.y);
           if constexpr (SPLIT)   // P_lo = bf16(p - P_hi)
             pl[k / 2] = pack_bf16x2(e.x - bf16_lo(pk[k / 2]), e.y - bf16_hi(pk[k / 2]));
           lsum = __fadd2_rn(lsum, e);
@@ -832,11 +646,11 @@ __global__ void attn_combine_kernel(const __grid_constant__ AttnParams p) {
   if (p.out_lo > 0) dst[p.out_lo] = __float2bfloat16_rn(v - __bfloat162float(hi));
 }
 
-template <int DH, bool CAUSAL, bool FP8, bool SPLIT = false>
+template <int DH, bool CAUSAL, bool SPLIT = false>
 cudaError_t launch_dh(const CUtensorMap &q, const CUtensorMap &k, const CUtensorMap &v,
                       const AttnParams &p, cudaStream_t stream) {
-  using L = AttnSmem<DH, FP8, SPLIT>;
-  auto kern = attn_kernel<DH, CAUSAL, FP8, SPLIT>;
+  using L = AttnSmem<DH, SPLIT>;
+  auto kern = attn_kernel<DH, CAUSAL, SPLIT>;
   static bool attr_set[64] = {};
   int dev = 0;
   cudaGetDevice(&dev);
@@ -1175,25 +989,17 @@ cudaError_t launch_attention_decode(const AttnParams &p, cudaStream_t stream) {
 
 cudaError_t launch_attention(const CUtensorMap &q, const CUtensorMap &k, const CUtensorMap &v,
                              const AttnParams &p, cudaStream_t stream) {
-  const bool f8 = p.kv_fp8 != 0;
+  // an e4m3 cache reaches the tile kernel as a bf16 copy (the caller's)
+  if (p.kv_fp8) return cudaErrorInvalidValue;
   if (p.causal) {
-    if (p.head_dim == 128)
-      return f8 ? launch_dh<128, true, true>(q, k, v, p, stream)
-                : launch_dh<128, true, false>(q, k, v, p, stream);
-    if (p.head_dim == 64)
-      return f8 ? launch_dh<64, true, true>(q, k, v, p, stream)
-                : launch_dh<64, true, false>(q, k, v, p, stream);
-  } else if (p.q_split) {   // the precise scoring pass: bf16 cache only
-    if (f8) return cudaErrorInvalidValue;
-    if (p.head_dim == 128) return launch_dh<128, false, false, true>(q, k, v, p, stream);
-    if (p.head_dim == 64) return launch_dh<64, false, false, true>(q, k, v, p, stream);
+    if (p.head_dim == 128) return launch_dh<128, true>(q, k, v, p, stream);
+    if (p.head_dim == 64) return launch_dh<64, true>(q, k, v, p, stream);
+  } else if (p.q_split) {   // the precise scoring pass
+    if (p.head_dim == 128) return launch_dh<128, false, true>(q, k, v, p, stream);
+    if (p.head_dim == 64) return launch_dh<64, false, true>(q, k, v, p, stream);
   } else {
-    if (p.head_dim == 128)
-      return f8 ? launch_dh<128, false, true>(q, k, v, p, stream)
-                : launch_dh<128, false, false>(q, k, v, p, stream);
-    if (p.head_dim == 64)
-      return f8 ? launch_dh<64, false, true>(q, k, v, p, stream)
-                : launch_dh<64, false, false>(q, k, v, p, stream);
+    if (p.head_dim == 128) return launch_dh<128, false>(q, k, v, p, stream);
+    if (p.head_dim == 64) return launch_dh<64, false>(q, k, v, p, stream);
   }
   return cudaErrorInvalidValue;
 }

@@ -31,8 +31,9 @@ struct AttnParams {
   float2 *part_ml;          // kv_splits > 1: [unit][split][256 rows] (reference max, row sum)
   const __nv_bfloat16 *q;   // decode kernel: Q [rows][Hq][dh]
   const void *k, *v;        // decode kernel: cache [rows][Hkv][dh] (bf16, or e4m3 bytes)
-  int kv_fp8;               // K/V are e4m3 codes: the tile kernel converts them to f16 in
-                            // shared memory; the K scale is folded into scale_log2
+  int kv_fp8;               // decode kernel: K/V are e4m3 codes (the tile kernel takes bf16
+                            // only: an e4m3 layer arrives as a bf16 copy of its codes); the
+                            // K scale is folded into scale_log2 either way
   float v_scale;            // output = v_scale * (P V) / l (1 for a bf16 cache)
   KvLayout pg;              // paged K/V (pg.table nullptr: slot-major)
   int kv_rows;              // rows of the K/V tensor maps (a coordinate there reads zeros)
@@ -47,9 +48,7 @@ int attn_positions_per_unit(int group);
 long long attn_units(const AttnParams &p);
 constexpr int kAttnPartRowFloats = 256;   // rows of a unit (times head_dim + 2 floats each)
 // q: 3-D map over Q [rows][Hq][dh] (q_split: [rows][2 Hq][dh]), box {64, group, P}; k, v: 3-D maps over
-// the cache [batch*cap][Hkv][dh], box {64, 1, 128}; all 128-byte swizzled.
-// With kv_fp8: k, v are byte maps over the e4m3 cache, box {dh, 1, 128},
-// unswizzled.
+// the cache [batch*cap][Hkv][dh] (bf16), box {64, 1, 128}; all 128-byte swizzled.
 cudaError_t launch_attention(const CUtensorMap &q, const CUtensorMap &k, const CUtensorMap &v,
                              const AttnParams &p, cudaStream_t stream);
 // Causal attention of one query row per sequence (q_span == 1, group <=

@@ -397,6 +397,66 @@ cudaError_t launch_argmax_combine(const float2 *part, int n_tiles, const int32_t
   return cudaGetLastError();
 }
 
+// e4m3 K/V codes of one layer -> bf16 (exact: every e4m3 value is a bf16
+// value), into slot-major rows b * cap + i, i < seq_end[b], from a slot-major,
+// paged or head-major cache.  One thread converts 16 codes of K and of V.
+// A paged row outside the pool is reported and skipped.
+__global__ void __launch_bounds__(256)
+    kv_to_bf16_kernel(const uint8_t *k, const uint8_t *v, KvLayout pg, int cap, int hkv, int dh,
+                      const int32_t *seq_end, int batch, __nv_bfloat16 *ko, __nv_bfloat16 *vo,
+                      unsigned *status) {
+  const int chunks = hkv * dh / 16;   // 16-code chunks of one slot
+  const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= (long long)batch * cap * chunks) return;
+  const long long row = idx / chunks;
+  const int c = (int)(idx - row * chunks);
+  const int b = (int)(row / cap), i = (int)(row - (long long)b * cap);
+  if (i >= seq_end[b]) return;
+  const int h = c * 16 / dh, e = c * 16 - h * dh;
+  long long src;
+  if (pg.head_major) {
+    src = (((long long)b * hkv + h) * cap + i) * dh + e;
+  } else {
+    const long long r = kv_row(pg, cap, b, i);
+    if (r < 0) {
+      set_status(status, CC_ERR_DEVICE_ARG);
+      return;
+    }
+    src = (r * hkv + h) * dh + e;
+  }
+  const size_t dst = (size_t)row * hkv * dh + (size_t)h * dh + e;
+  auto convert = [](const uint8_t *in, __nv_bfloat16 *out) {
+    const uint4 x = *reinterpret_cast<const uint4 *>(in);
+    const uint32_t w[4] = {x.x, x.y, x.z, x.w};
+    uint32_t o[8];
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+#pragma unroll
+      for (int hf = 0; hf < 2; ++hf) {   // two codes -> f16 pair (exact) -> bf16 pair (exact)
+        uint32_t f2;
+        asm("cvt.rn.f16x2.e4m3x2 %0, %1;" : "=r"(f2) : "h"((unsigned short)(w[j] >> (16 * hf))));
+        const float2 f = __half22float2(*reinterpret_cast<const __half2 *>(&f2));
+        o[j * 2 + hf] = pack_bf16x2(f.x, f.y);
+      }
+    uint4 *d = reinterpret_cast<uint4 *>(out);
+    d[0] = make_uint4(o[0], o[1], o[2], o[3]);
+    d[1] = make_uint4(o[4], o[5], o[6], o[7]);
+  };
+  convert(k + src, ko + dst);
+  convert(v + src, vo + dst);
+}
+
+cudaError_t launch_kv_to_bf16(const uint8_t *k, const uint8_t *v, const KvLayout &pg, int cap,
+                              int hkv, int dh, const int32_t *seq_end, int batch,
+                              __nv_bfloat16 *k_out, __nv_bfloat16 *v_out, unsigned *status,
+                              cudaStream_t st) {
+  const long long n = (long long)batch * cap * (hkv * dh / 16);
+  if (n <= 0) return cudaSuccess;
+  kv_to_bf16_kernel<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(k, v, pg, cap, hkv, dh, seq_end,
+                                                                 batch, k_out, v_out, status);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_append_finish(int32_t *seq_len, const int32_t *row_hi, int batch,
                                  cudaStream_t st) {
   append_finish_kernel<<<(batch + 255) / 256, 256, 0, st>>>(seq_len, row_hi, batch);

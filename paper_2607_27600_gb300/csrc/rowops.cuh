@@ -27,6 +27,12 @@ cudaError_t launch_append_prepare(const int32_t *seq_len, const int32_t *count,
                                   int32_t *tokens, int32_t *pos, int32_t *row_lo, int32_t *row_hi,
                                   int batch, int cap, unsigned *status, cudaStream_t st);
 // seq_len = row_hi
+// One layer of an e4m3 cache as bf16 (exact), slot-major [batch * cap][hkv][dh]
+// for the slots i < seq_end[b] (dh a multiple of 16).
+cudaError_t launch_kv_to_bf16(const uint8_t *k, const uint8_t *v, const KvLayout &pg, int cap,
+                              int hkv, int dh, const int32_t *seq_end, int batch,
+                              __nv_bfloat16 *k_out, __nv_bfloat16 *v_out, unsigned *status,
+                              cudaStream_t st);
 cudaError_t launch_append_finish(int32_t *seq_len, const int32_t *row_hi, int batch,
                                  cudaStream_t st);
 // next[b] = first column of the largest logit over the (max, column) tile
