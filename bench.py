@@ -932,7 +932,7 @@ def read_traffic(kernel, workload):
 # the CUDA sources each kernel kind is built from (its own file, its header,
 # the shared PTX wrappers)
 KERNEL_SOURCES = {
-    "gemm": ["gemm.cu", "gemm.cuh", "cc_common.cuh"],
+    "gemm": ["gemm.cu", "gemm.cuh", "cc_common.cuh", "api.cu"],   # api.cu: the tile order
     "attention": ["attn.cu", "attn.cuh", "cc_common.cuh"],
     "compact": ["compact.cu", "compact.cuh", "cc_common.cuh"],
     "select": ["select.cu", "select.cuh", "cc_common.cuh"],

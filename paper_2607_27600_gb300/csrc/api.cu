@@ -375,8 +375,9 @@ cc_status gemm_setup(Gemm &g, int epi, const void *A, int K, const void *W, cons
   g.p.n_tiles = (N + bn - 1) / bn;
   g.p.status = status;
   g.p.a_split = a_split ? 1 : 0;
-  // Tile order for L2 reuse: keep a slab of <= ~40 MB of one operand resident
-  // (evict-last) while the other streams past (evict-first).  Weight slabs
+  // Tile order for L2 reuse: keep a slab of one operand resident (evict-last;
+  // budget below) while the other streams past (evict-first; CTA pairs keep
+  // both evict-last).  Weight slabs
   // resident (raster 0) is the default: a group's tiles of one activation row
   // tile run on consecutive CTAs, so the streamed row tile is read from DRAM
   // about once per group, and on the Llama-3-8B projections (K = 4096 and
@@ -384,8 +385,19 @@ cc_status gemm_setup(Gemm &g, int epi, const void *A, int K, const void *W, cons
   // even where a count of whole-slab re-reads favoured the latter by up to
   // 16 %.  The activation-resident order is taken only when that count is
   // below 0.8x (an LM head whose weight is far larger than L2).
-  const double budget = 40.0 * (1 << 20);
   const uint64_t R_used = R_est;
+  // The slab budget: 40 MB, or 60 MB for an fp32-output GEMM whose streamed
+  // activations outweigh its output (the down projection: each group of
+  // resident weight tiles re-reads the activations).  Measured at the Llama-3-8B 16k launches (DRAM bytes read
+  // per launch, 20 / 30 / 40 / 60 / 80 MB): the down projection (470 MB of
+  // activations, 268 MB fp32 output) 5.5 / 3.6 / 3.8 / 2.6 / 3.2 GB, 1.06 ms
+  // at 60 against 1.10 at 40; gate/up (134 MB in, 470 MB out) 3.2 / 2.4 /
+  // 2.3 / 2.8 / 5.1 GB.
+  const bool f32_out = epi == EPI_F32 || epi == EPI_RESID_BF16 || epi == EPI_RESID_F32 ||
+                       epi == EPI_RESID_LOGIT;
+  const double act_bytes = (double)R_used * K * (a_split ? 2.0 : 1.0) * 2;
+  const double out_bytes = (double)R_used * N * (f32_out ? 4.0 : 2.0);
+  const double budget = (f32_out && act_bytes > out_bytes ? 60.0 : 40.0) * (1 << 20);
   g.rows_est = R_used;
   const int num_m = (int)((R_used + 127) / 128), num_n = g.p.n_tiles;
   const double k_a = (a_split ? 2.0 : 1.0) * K;
