@@ -115,3 +115,43 @@ def test_binding_structs_match_the_header(name):
     member the library reads)."""
     from paper_2607_27600_gb300 import cc
     assert [f[0] for f in getattr(cc, name)._fields_] == _header_struct_fields(name)
+
+
+def header_enums():
+    """name -> value of every enumerator the public headers define."""
+    vals = {}
+    for h in os.listdir(os.path.join(ROOT, "include")):
+        if not h.endswith(".h"):
+            continue
+        src = re.sub(r"/\*.*?\*/", "", open(os.path.join(ROOT, "include", h)).read(), flags=re.S)
+        for body in re.findall(r"typedef\s+enum\s*\{(.*?)\}", src, flags=re.S):
+            nxt = 0
+            for item in body.split(","):
+                item = item.strip()
+                if not item:
+                    continue
+                name, _, val = item.partition("=")
+                nxt = int(val.strip(), 0) if val.strip() else nxt
+                vals[name.strip()] = nxt
+                nxt += 1
+    return vals
+
+
+def test_binding_constants_match_the_headers(lib):
+    from paper_2607_27600_gb300 import cc
+    e = header_enums()
+    pairs = {"CC_OK": cc.CC_OK, "CC_ERR_INVALID_ARG": cc.CC_ERR_INVALID_ARG,
+             "CC_ERR_CUDA": cc.CC_ERR_CUDA, "CC_ERR_BUDGET": cc.CC_ERR_BUDGET,
+             "CC_ERR_WORKSPACE": cc.CC_ERR_WORKSPACE, "CC_ERR_TIMEOUT": cc.CC_ERR_TIMEOUT,
+             "CC_ERR_UNSUPPORTED": cc.CC_ERR_UNSUPPORTED, "CC_ERR_DEVICE_ARG": cc.CC_ERR_DEVICE_ARG,
+             "CC_SCORE_LOGIT": cc.SCORE_LOGIT, "CC_SCORE_LOGPROB": cc.SCORE_LOGPROB,
+             "CC_SCORE_PRECISE": cc.SCORE_PRECISE, "CC_SCORE_RANGE_ONLY": cc.SCORE_RANGE_ONLY,
+             "CC_KV_BF16": cc.KV_BF16, "CC_KV_E4M3": cc.KV_E4M3,
+             "CC_KV_SLOT_MAJOR": cc.KV_SLOT_MAJOR, "CC_KV_HEAD_MAJOR": cc.KV_HEAD_MAJOR,
+             "CC_KERNEL_COUNT": cc.KERNEL_COUNT}
+    for name, val in pairs.items():
+        assert e[name] == val, (name, e[name], val)
+    # every profiled kernel kind has its own name in the library
+    names = [lib.cc_kernel_name(k).decode() for k in range(cc.KERNEL_COUNT)]
+    assert len(set(names)) == cc.KERNEL_COUNT and "unknown" not in names
+    assert lib.cc_kernel_name(cc.KERNEL_COUNT).decode() == "unknown"
