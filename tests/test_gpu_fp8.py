@@ -103,6 +103,22 @@ def test_fp8_scores_small_ragged(cc, full):
         assert np.abs(bf[fin] - want[fin]).max() > 0
 
 
+@pytest.mark.parametrize("full", [False, True])
+def test_fp8_precise_mode_small_ragged(cc, full):
+    """CC_SCORE_PRECISE over an e4m3 cache: each layer's codes reach the
+    attention as an exact bf16 copy, so the queries and P are split there as
+    over a bf16 cache, and the scores stay within 2e-3 of the oracle's on the
+    dequantised cache (an order of magnitude inside the default mode's bar)."""
+    seq, cap = [300, 129, 1, 64], 320
+    w_np = to_np(synth.model_weights(SMALL_GPU, 73, with_kv_proj=True))
+    c_np = causal_cache(SMALL_GPU, w_np, seq, cap, 73)
+    on, dev = fp8_views(c_np)
+    want = (oracle.score_full if full else oracle.score_layer)(SMALL_GPU, w_np, on)
+    got, _ = _score(cc, SMALL_GPU, w_np, dev, cc.SCORE_LOGIT | cc.SCORE_PRECISE, full)
+    err = rel_err(got, want)
+    assert err < TOL and err < 2e-3, err
+
+
 @pytest.mark.parametrize("name", ["llama", "qwen"])
 def test_fp8_fast_scores_model_shapes(cc, name):
     """Last-layer refresh at Llama-3-8B (G = 4) and Qwen2.5-7B (G = 7) layer
