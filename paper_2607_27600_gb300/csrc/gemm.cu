@@ -545,10 +545,10 @@ CC_DEV void tile_coords(const GemmParams &p, int t, int num_m, int &m, int &n) {
   }
 }
 
-// One CTA (PAIR false) or a CTA pair (PAIR true, a cluster of two) per SM
-// pair, persistent over the output tiles.  A pair computes 256-row tiles:
-// CTA r holds row tile 2 mp + r of pair row mp (rows of two consecutive
-// 128-row tiles, which may belong to different sequences) and B rows
+// One CTA per SM (PAIR false) or a CTA pair per two SMs (PAIR true, a
+// cluster of two), persistent over the output tiles.  A pair computes
+// 256-row tiles: CTA r holds row tile 2 mu + r of row unit mu (two
+// consecutive 128-row tiles, which may belong to different sequences) and B rows
 // [r TBN/2, (r+1) TBN/2) of the column tile; CTA 0 issues the pair's
 // products into both tensor memories and its commits release the stages
 // and accumulators of both CTAs.  Both CTAs' loads of a stage complete on
