@@ -46,6 +46,8 @@ test_append_after_compaction_then_score = append_tests.test_append_after_compact
 test_append_llama_shape_chunk_over_long_memory = (
     append_tests.test_append_llama_shape_chunk_over_long_memory)
 test_fp8_append_llama_fused_projection = fp8_tests.test_fp8_append_llama_fused_projection
+test_fp8_scores_small_ragged = fp8_tests.test_fp8_scores_small_ragged
+test_fp8_precise_mode_small_ragged = fp8_tests.test_fp8_precise_mode_small_ragged
 test_paged_append_matches_slot_major = paged_tests.test_paged_append_matches_slot_major
 
 

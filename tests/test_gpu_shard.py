@@ -189,3 +189,42 @@ def test_rows_in_blocks_over_cache_layout_variants(pkg, layout):
         c["kv_layout"] = 1
     single, merged, parts = _single_and_sharded(pkg, shape, w, c, cc.SCORE_LOGIT, False, 3)
     _check(single, merged, parts, seq)
+
+
+@pytest.mark.parametrize("layout", ["e4m3", "paged", "head_major"])
+def test_range_only_blocks_over_cache_layout_variants(pkg, layout):
+    """CC_SCORE_RANGE_ONLY blocks (the sequence ends first) over an e4m3, a
+    paged and a head-major cache: one buffer, the single call's scores bit
+    for bit (an e4m3 layer is copied to bf16 for each block's attention)."""
+    import bench
+    from paper_2607_27600_gb300 import cc
+    shape = synth.WORKLOADS["qwen7b-table1-fast-4096"].shape
+    seq, cap = [4096, 2500], 4096
+    last = shape.n_layers - 1
+    w = synth.model_weights(shape, 61, device="cuda", layers=[last], with_embed=False)
+    c = synth.synthetic_cache(shape, seq, cap, 62, device="cuda")
+    if layout == "e4m3":
+        bench.to_e4m3_cache(c)
+    elif layout == "paged":
+        bench.to_paged_cache(c, 256, 63)
+    else:
+        for key in ("k", "v"):
+            c[key] = [x.permute(0, 2, 1, 3).contiguous() for x in c[key]]
+        c["kv_layout"] = 1
+    weights, cache = pkg.Weights(w), pkg.Cache(c)
+    b = len(seq)
+    mode = cc.SCORE_LOGIT
+    ws = cc.alloc_workspace(cc.cc_score_workspace_size(shape, b, cap, mode))
+    single = torch.empty(b, cap, dtype=torch.float32, device="cuda")
+    cc.cc_score_layer(shape, weights, cache, mode, single, ws)
+    filled = torch.full((b, cap), float("nan"), dtype=torch.float32, device="cuda")
+    bounds = bench.block_bounds(seq, 3)
+    for k in reversed(range(3)):
+        lo = torch.tensor(bounds[k], dtype=torch.int32, device="cuda")
+        hi = torch.tensor(bounds[k + 1], dtype=torch.int32, device="cuda")
+        cc.cc_score_rows(shape, weights, cache, mode | cc.SCORE_RANGE_ONLY, False, lo, hi, filled, ws)
+    assert cc.cc_get_status() == cc.CC_OK
+    s, f = single.cpu().numpy(), filled.cpu().numpy()
+    for i, n in enumerate(seq):
+        assert np.array_equal(f[i, :n].view(np.uint32), s[i, :n].view(np.uint32))
+        assert np.all(np.isnan(f[i, n:]))
