@@ -271,8 +271,9 @@ def algorithmic_work(wl, kv_bytes=2):
         "compact": ("hbm", 2.0 * moved * (n_arrays_kv * kv_row + h_row + 8)),
         # at most 9 passes over the scores (up to 8 radix passes + the emit pass)
         "select": ("hbm", 9.0 * 4.0 * n_rows),
-        # an e4m3 layer's K and V codes read, their bf16 copies written (per launch)
-        "kv_dequant": ("hbm", n_rows * 2.0 * s.n_kv_heads * dh * 3.0),
+        # a layer's K and V read (e4m3 codes, or bf16 in the fp16 operand mode)
+        # and their 2-byte copies written (per launch)
+        "kv_dequant": ("hbm", n_rows * 2.0 * s.n_kv_heads * dh * (kv_bytes + 2.0)),
     }
 
 
@@ -372,7 +373,10 @@ def refresh_record(args, dist, wl, w, pristine, mode, steps, with_e2e=True, with
     shape = wl.shape
     fast = wl.mode == "layer"
     work = clone_cache(pristine)
-    weights, cache = pkg.Weights(w), pkg.Cache(work)
+    f16 = bool(mode & cc.SCORE_F16)
+    # fp16 operand mode: the layer matrices converted once (model preparation,
+    # outside the timed steps)
+    weights, cache = pkg.Weights(cc.f16_weights(w) if f16 else w), pkg.Cache(work)
     b, cap = wl.batch, wl.cap
     scores = torch.empty(b, cap, dtype=torch.float32, device=dev)
     keep_idx = torch.empty(b, cap, dtype=torch.int32, device=dev)
@@ -497,7 +501,7 @@ def refresh_record(args, dist, wl, w, pristine, mode, steps, with_e2e=True, with
     table = kernel_table(kernels, steps, work_tbl, peaks, timed_s)
     dom = max(kernels.items(), key=lambda kv: kv[1][1])[0]
     precise = bool(mode & cc.SCORE_PRECISE)
-    traffic = None if precise else read_traffic(dom, wl.name)
+    traffic = None if precise else read_traffic(dom, wl.name, "f16" if f16 else "bf16")
     roof = roofline_of(table, dom, peaks, peak_src, timed_s, traffic)
     # replicas: every rank refreshes its own copy (weak scaling); row shards:
     # the ranks share one refresh (strong scaling)
@@ -509,8 +513,9 @@ def refresh_record(args, dist, wl, w, pristine, mode, steps, with_e2e=True, with
         "score_only": {"value": round(positions * (1 if row_shard is not None else dist.world) /
                                       (score_ms * 1e-3), 1),
                        "unit": "positions/s", "ms": round(score_ms, 4)},
-        "mode": ("precise: [hi | lo] bf16 pairs for activations, queries and P"
-                 if precise else "bf16 operands, fp32 accumulation"),
+        "mode": ("precise: [hi | lo] bf16 pairs for activations, queries and P" if precise else
+                 "fp16 operands (layer weights converted once; K/V copied per layer), fp32 "
+                 "accumulation" if f16 else "bf16 operands, fp32 accumulation"),
         "pass": ("fast single-layer" if fast else f"full {shape.n_layers}-layer")
         if scorer == "counter-causal" else
         {"recency": "position", "importance": "last-layer key attention",
@@ -519,6 +524,7 @@ def refresh_record(args, dist, wl, w, pristine, mode, steps, with_e2e=True, with
                                      if scorer == "counter-causal" else None),
         "step_tflop": round(step_flops(wl) / 1e12, 3) if scorer == "counter-causal" else None,
         "gpu_launches": int(sum(c for c, _ in kernels.values())),
+        "dtype": "f16" if f16 else "bf16",
         "roofline": roof, "kernels": table, "clocks": clk,
     }
     if row_shard is not None:
@@ -527,6 +533,9 @@ def refresh_record(args, dist, wl, w, pristine, mode, steps, with_e2e=True, with
     if precise:
         rec["roofline"]["note"] = ("algorithmic FLOPs of the pass; the precise mode issues each "
                                    "product once per operand half (about twice these FLOPs)")
+    if f16 and rec["roofline"].get("bound") == "tensor":
+        rec["roofline"]["peak_source"] += ("; fp16 operands: the nominal dense fp16 rate equals "
+                                           "the bf16 one, so the measured bf16 peak applies")
     if e2e is not None:
         rec["e2e"] = {"value": round(positions * (1 if row_shard is not None else dist.world) /
                                      (e2e["ms"] * 1e-3), 1),
@@ -829,7 +838,8 @@ def cycles_record(args, dist, wl, w, pristine, steps):
 def run_suite(args, dist):
     """The default bench line: the headline workload (the full-model pass over
     all 32 layers of the Llama-3-8B shape, the largest single-GPU workload
-    with a full pass) plus, in the same line, its precise mode, the ragged
+    with a full pass, fp16 operands unless --bf16 or --precise) plus, in the
+    same line, the same pass in the other two operand modes, the ragged
     32k single-layer batch and the long-context refresh cycles."""
     import paper_2607_27600_gb300 as pkg
     from paper_2607_27600_gb300 import cc
@@ -843,8 +853,14 @@ def run_suite(args, dist):
                                  shape=dataclasses.replace(wl.shape, n_layers=args.layers))
         args.no_records = True
     mode = cc.SCORE_LOGPROB if args.score == "logprob" else cc.SCORE_LOGIT
+    if args.precise and args.bf16:
+        raise SystemExit("--precise and --bf16 are two modes: pick one")
+    # the refresh's operand mode: fp16 (the fastest mode that holds the full
+    # pass to the stated tolerance) unless --bf16 or --precise asks otherwise
     if args.precise:
         mode |= cc.SCORE_PRECISE
+    elif not args.bf16 and args.scorer == "counter-causal":
+        mode |= cc.SCORE_F16
     if wl.cycles > 1 and args.scorer == "counter-causal" and not args.single_cycle:
         (w, pristine), cache_src = bench_inputs(args, wl, dev)
         rec = cycles_record(args, dist, wl, w, pristine, args.steps)
@@ -854,10 +870,13 @@ def run_suite(args, dist):
     records = {}
     if not args.no_records and args.scorer == "counter-causal" and dist.world >= 1:
         sub = min(args.steps, 10)
-        if not args.precise:
-            records[wl.name + "/precise"] = refresh_record(
-                args, dist, wl, w, pristine, mode | cc.SCORE_PRECISE, sub, with_e2e=False,
-                with_cpu=False)
+        # the pass in the other two operand modes
+        base = mode & ~(cc.SCORE_PRECISE | cc.SCORE_F16)
+        for tag, m in (("bf16", base), ("f16", base | cc.SCORE_F16),
+                       ("precise", base | cc.SCORE_PRECISE)):
+            if m != mode:
+                records[f"{wl.name}/{tag}"] = refresh_record(
+                    args, dist, wl, w, pristine, m, sub, with_e2e=False, with_cpu=False)
         if args.workload == synth.HEADLINE:
             del w, pristine
             torch.cuda.empty_cache()
@@ -883,7 +902,7 @@ def suite_line(args, dist, wl, head, cache_src, records):
         "value": head["value"], "unit": "positions/s", "n_gpus": dist.world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": head.get("ms_per_step"),
         "higher_is_better": True, "scaling": "strong" if args.shard == "rows" else "weak",
-        "vs_baseline": vs_baseline, "dtype": "bf16",
+        "vs_baseline": vs_baseline, "dtype": head.get("dtype", "bf16"),
         "data": f"synthetic (seeded random-init weights N(0,0.02); cache: {cache_src})",
         "config": {"workload": wl.name, "scorer": args.scorer,
                    "kv_cache": ("e4m3 (per-layer scales)" if args.kv_fp8 else "bf16") +
@@ -912,8 +931,9 @@ def suite_line(args, dist, wl, head, cache_src, records):
     return line
 
 
-def read_traffic(kernel, workload):
-    """DRAM bytes per launch from a committed ncu summary, when it matches the
+def read_traffic(kernel, workload, operands="bf16"):
+    """DRAM bytes per launch from a committed ncu summary, when it was taken
+    in the same operand mode (an entry without "operands" is bf16) on the
     current sources of that kernel; else None."""
     p = os.path.join(ROOT, "profiles", "dram_traffic.json")
     if not os.path.exists(p):
@@ -923,6 +943,8 @@ def read_traffic(kernel, workload):
             tbl = json.load(f)
         e = tbl.get(workload, {}).get(kernel)
         if not e or e.get("sources_sha") != kernel_digest(kernel):
+            return None
+        if e.get("operands", "bf16") != operands:
             return None
         return e.get("bytes_per_launch")
     except Exception:
@@ -1317,6 +1339,7 @@ def run_append(args, dist):
                 "h2d_bytes_per_step": int(host_tok.numel() * 4 + 4), "d2h_bytes_per_step": 4,
                 "ms_per_step": round(e2e_ms, 4)},
         "gpu_launches": int(sum(c for c, _ in kernels.values())),
+        "dtype": "f16" if f16 else "bf16",
         "roofline": {"kernel": dom, "bound": d.get("bound"), "achieved": d.get("achieved"),
                      "peak": peaks["bf16_tflops"] if d.get("bound") == "tensor" else peaks["hbm_gbs"],
                      "unit": d.get("unit"), "frac": d.get("frac"), "traffic": None,
@@ -1443,6 +1466,7 @@ def run_decode(args, dist):
                 "h2d_bytes_per_step": 4 * B, "d2h_bytes_per_step": 4 * B,
                 "ms_per_step": round(e2e_ms, 4)},
         "gpu_launches": int(sum(c for c, _ in kernels.values())),
+        "dtype": "f16" if f16 else "bf16",
         "roofline": {"kernel": dom, "bound": dd.get("bound"), "achieved": dd.get("achieved"),
                      "peak": peaks["hbm_gbs"], "unit": dd.get("unit"), "frac": dd.get("frac"),
                      "traffic": None, "peak_source": f"{peak_src} (HBM copy)"},
@@ -1488,6 +1512,9 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--precise", action="store_true",
                     help="time the precise mode (CC_SCORE_PRECISE) as the headline")
+    ap.add_argument("--bf16", action="store_true",
+                    help="time the bf16 operand mode (the library's default) as the headline "
+                         "instead of the fp16 one (CC_SCORE_F16)")
     ap.add_argument("--e2e-blocks", type=int, default=0,
                     help="fast pass end to end: row blocks uploaded and scored in turn (1: the "
                          "whole input first; 0: one block per 16k rows, at most 8)")

@@ -45,7 +45,9 @@ typedef enum {
   CC_ERR_WORKSPACE = 4,    /* workspace smaller than *_workspace_size              */
   CC_ERR_TIMEOUT = 5,      /* device: an internal wait gave up (kernel returned)   */
   CC_ERR_UNSUPPORTED = 6,  /* shape outside what the kernels implement             */
-  CC_ERR_DEVICE_ARG = 7    /* device: seq_len/keep_count outside [0, cap]          */
+  CC_ERR_DEVICE_ARG = 7,   /* device: seq_len/keep_count outside [0, cap]          */
+  CC_ERR_RANGE = 8         /* device: a value written as an fp16 operand (mode
+                              CC_SCORE_F16, cc_bf16_to_f16) exceeded 65504         */
 } cc_status;
 
 /* Score definition.  Sec. 3.1 takes the logit of the row's own token x_i as
@@ -70,7 +72,26 @@ typedef enum {
    * written and every other entry of scores (other rows, slots past the
    * sequence ends) keeps its value, so that calls over disjoint ranges fill
    * one buffer -- e.g. blocks of rows scored as their inputs arrive. */
-  CC_SCORE_RANGE_ONLY = 0x200
+  CC_SCORE_RANGE_ONLY = 0x200,
+  /* Flag, OR-ed into the mode, either pass (not with CC_SCORE_PRECISE): every
+   * tensor-core operand of the layers in fp16 instead of bf16 -- one value,
+   * not a pair, so the pass costs what the default one does.  fp16 keeps 11
+   * significant bits to bf16's 8, so each rounding is 8x smaller, and it
+   * represents every bf16 value of magnitude in [2^-14, 65504] exactly:
+   *   - wq, wo, w_gate, w_up and w_down of layers[] are fp16 here (same
+   *     shapes; cc_bf16_to_f16 converts the bf16 weights once);
+   *   - the cached K/V (bf16 or e4m3) are copied to fp16 per layer in the
+   *     workspace's activation buffer (needs 4 * Hkv * head_dim <= 2 * d_ff
+   *     bytes per slot, else CC_ERR_UNSUPPORTED);
+   *   - the queries, the attention probabilities and the GEMM activations
+   *     (normalised inputs, attention output, SwiGLU output) are written as
+   *     fp16; a finite value above 65504 in magnitude is reported on the
+   *     device as CC_ERR_RANGE (use the bf16 modes for such a model);
+   *   - the gains, biases, embedding, lm_head, H^(L-1) and the head (final
+   *     norm, logit or log-prob) stay as in the default mode.
+   * On a deep random-weight model the 32-layer score stays within ~2e-2 of
+   * the exact one, where single bf16 operands drift by several percent. */
+  CC_SCORE_F16 = 0x400
 } cc_score_mode;
 
 /* Element format of the cached keys and values.  The paper keeps the model's
@@ -223,6 +244,16 @@ cc_status cc_score_layer(const cc_model_cfg *cfg, const cc_model_weights *w,
 cc_status cc_score_full(const cc_model_cfg *cfg, const cc_model_weights *w,
                         const cc_kv_cache *cache, cc_score_mode mode, float *scores,
                         void *ws, size_t ws_bytes, void *stream);
+
+/* cc_bf16_to_f16 -- dst[i] = fp16(src[i]) for i < n: the weight matrices of
+ * mode CC_SCORE_F16, converted once before the scoring calls.  Exact for
+ * magnitudes in [2^-14, 65504] (and zero); smaller ones round to the nearest
+ * multiple of 2^-24 (ties to even); a larger finite value becomes +-inf and
+ * is reported as CC_ERR_RANGE on the device (cc_get_status).  NaN and inf
+ * pass through.  src, dst: device, 16-byte aligned, not overlapping; n a
+ * multiple of 8 (else CC_ERR_INVALID_ARG); n = 0 does nothing.  Async on
+ * `stream`. */
+cc_status cc_bf16_to_f16(const void *src, void *dst, size_t n, void *stream);
 
 /* ---- one refresh sharded over several GPUs by query rows ----------------------
  * Given the cache, a row's score depends only on its own input (token or

@@ -21,13 +21,15 @@ CC_ERR_WORKSPACE = 4
 CC_ERR_TIMEOUT = 5
 CC_ERR_UNSUPPORTED = 6
 CC_ERR_DEVICE_ARG = 7
+CC_ERR_RANGE = 8
 STATUS_NAMES = {0: "CC_OK", 1: "CC_ERR_INVALID_ARG", 2: "CC_ERR_CUDA", 3: "CC_ERR_BUDGET",
                 4: "CC_ERR_WORKSPACE", 5: "CC_ERR_TIMEOUT", 6: "CC_ERR_UNSUPPORTED",
-                7: "CC_ERR_DEVICE_ARG"}
+                7: "CC_ERR_DEVICE_ARG", 8: "CC_ERR_RANGE"}
 SCORE_LOGIT = 0
 SCORE_LOGPROB = 1
 SCORE_PRECISE = 0x100   # flag: hi + lo bf16 GEMM activations, queries and P (either pass)
 SCORE_RANGE_ONLY = 0x200   # flag (cc_score_rows): entries outside the row range keep their values
+SCORE_F16 = 0x400   # flag: fp16 tensor-core operands (the layer weights passed as fp16)
 
 
 class CCError(RuntimeError):
@@ -132,6 +134,8 @@ _SIGS = {
     "cc_graph_end": (ctypes.c_int, [ctypes.c_void_p, ctypes.POINTER(ctypes.c_void_p)]),
     "cc_graph_launch": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p]),
     "cc_graph_destroy": (ctypes.c_int, [ctypes.c_void_p]),
+    "cc_bf16_to_f16": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_size_t,
+                                      ctypes.c_void_p]),
     "cc_get_status": (ctypes.c_int, [ctypes.c_void_p]),
     "cc_status_str": (ctypes.c_char_p, [ctypes.c_int]),
     "cc_last_error": (ctypes.c_char_p, []),
@@ -235,6 +239,27 @@ class Weights:
                                   _dev_ptr(w["lm_head"], "lm_head"), self._layers)
 
 
+F16_MATRICES = ("wq", "wo", "w_gate", "w_up", "w_down")   # what SCORE_F16 reads as fp16
+
+
+def f16_weights(w: dict, stream=None) -> dict:
+    """The weights dict of Weights with the layer matrices that SCORE_F16
+    reads (F16_MATRICES) converted to fp16 by cc_bf16_to_f16; every other
+    entry is shared with `w`."""
+    out = dict(w)
+    out["layers"] = []
+    for lw in w["layers"]:
+        if lw is None:
+            out["layers"].append(None)
+            continue
+        nl = dict(lw)
+        for f in F16_MATRICES:
+            nl[f] = torch.empty(lw[f].shape, dtype=torch.float16, device=lw[f].device)
+            cc_bf16_to_f16(lw[f], nl[f], stream)
+        out["layers"].append(nl)
+    return out
+
+
 class Cache:
     """cc_kv_cache over a dict of CUDA tensors (k[l], v[l] bf16 [B, cap, Hkv, dh],
     or e4m3 codes (uint8) when the dict holds "kv_scale": per layer the (K, V)
@@ -325,6 +350,16 @@ def cc_score_layer(cfg, weights, cache, mode, scores, ws, stream=None):
 
 def cc_score_full(cfg, weights, cache, mode, scores, ws, stream=None):
     _score("cc_score_full", cfg, weights, cache, mode, scores, ws, stream)
+
+
+def cc_bf16_to_f16(src, dst, stream=None):
+    """dst (fp16) = src (bf16), element by element (same number of elements,
+    a multiple of 8): the layer weights of SCORE_F16."""
+    if src.dtype != torch.bfloat16 or dst.dtype != torch.float16 or src.numel() != dst.numel():
+        raise ValueError("cc_bf16_to_f16: src bf16 and dst fp16 of one size")
+    code = load_library().cc_bf16_to_f16(_dev_ptr(src, "src"), _dev_ptr(dst, "dst"), src.numel(),
+                                         _stream(stream))
+    _check(code, "cc_bf16_to_f16")
 
 
 def cc_score_rows(cfg, weights, cache, mode, full: bool, row_lo, row_hi, scores, ws, stream=None):

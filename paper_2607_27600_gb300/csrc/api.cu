@@ -518,29 +518,33 @@ cc_status run_attention(const cc_model_cfg *c, const void *q, const void *k, con
                         int q_span = 0, const AttnPartials *parts = nullptr, int sms = 0,
                         KvFmt kvf = KvFmt(), bool q_split = false,
                         const int32_t *range_lo = nullptr, const int32_t *range_hi = nullptr,
-                        void *kv_scratch = nullptr, size_t kv_scratch_bytes = 0) {
+                        void *kv_scratch = nullptr, size_t kv_scratch_bytes = 0,
+                        bool f16 = false) {
   const int G = c->n_q_heads / c->n_kv_heads, dh = c->head_dim;
   const int P = attn_positions_per_unit(G);
   const uint64_t R = (uint64_t)batch * cap;
   if (q_split && row_lo) return CC_ERR_UNSUPPORTED;
+  // fp16 operands (q and out fp16): the counter-causal pass with single operands
+  if (f16 && (row_lo || split || q_split)) return CC_ERR_UNSUPPORTED;
   // one query row per sequence: the decode kernel, which reads either format
   const long long units0 = (long long)batch * c->n_kv_heads *
                            (((row_lo ? q_span : cap) + P - 1) / P);
   const bool decode = row_lo && q_span == 1 && G <= kDecMaxG && parts && parts->o && parts->ml &&
                       units0 <= kAttnMaxSplitSlots;
-  if (kvf.fp8 && !decode) {
-    // the tile attention over an e4m3 cache: the layer's codes as bf16 (exact)
-    // in a slot-major scratch, the scales kept folded into the softmax scale
-    // and the output normalisation
+  if ((kvf.fp8 || f16) && !decode) {
+    // the tile attention over an e4m3 cache, or with fp16 operands: the
+    // layer's elements as bf16 or fp16 values (exact) in a slot-major scratch;
+    // an e4m3 cache's scales stay folded into the softmax scale and the output
+    // normalisation
     const size_t half = R * c->n_kv_heads * dh * 2;
     if (!kv_scratch || kv_scratch_bytes < 2 * half) return CC_ERR_UNSUPPORTED;
-    __nv_bfloat16 *ks = reinterpret_cast<__nv_bfloat16 *>(kv_scratch);
-    __nv_bfloat16 *vs = reinterpret_cast<__nv_bfloat16 *>(reinterpret_cast<uint8_t *>(kv_scratch) + half);
+    uint8_t *ks = reinterpret_cast<uint8_t *>(kv_scratch);
+    uint8_t *vs = ks + half;
     {
       TimedScope t(CC_KERNEL_KV_DEQUANT, st);
-      CC_TRY(launch_kv_to_bf16(reinterpret_cast<const uint8_t *>(k),
-                               reinterpret_cast<const uint8_t *>(v), kvf.pg, cap, c->n_kv_heads,
-                               dh, seq_len, batch, ks, vs, status, st));
+      CC_TRY(launch_kv_copy(reinterpret_cast<const uint8_t *>(k),
+                            reinterpret_cast<const uint8_t *>(v), kvf.fp8, f16, kvf.pg, cap,
+                            c->n_kv_heads, dh, seq_len, batch, ks, vs, status, st));
     }
     k = ks;
     v = vs;
@@ -590,6 +594,7 @@ cc_status run_attention(const cc_model_cfg *c, const void *q, const void *k, con
   // scale; O = v_scale * P . codes, applied with the normalisation
   p.scale_log2 = (float)(1.4426950408889634 / sqrt((double)dh) * kvf.k_scale);
   p.kv_fp8 = kvf.fp8 ? 1 : 0;
+  p.f16 = f16 ? 1 : 0;
   p.v_scale = kvf.v_scale;
   p.pg = kvf.pg;
   p.kv_rows = (int)RK;
@@ -926,7 +931,8 @@ cc_status check_score_args(const cc_model_cfg *c, const cc_model_weights *w, con
     return CC_ERR_INVALID_ARG;
   const int base_mode = mode & 0xFF;
   if ((base_mode != CC_SCORE_LOGIT && base_mode != CC_SCORE_LOGPROB) ||
-      (mode & ~(0xFF | CC_SCORE_PRECISE | CC_SCORE_RANGE_ONLY)))
+      (mode & ~(0xFF | CC_SCORE_PRECISE | CC_SCORE_RANGE_ONLY | CC_SCORE_F16)) ||
+      ((mode & CC_SCORE_PRECISE) && (mode & CC_SCORE_F16)))
     return CC_ERR_INVALID_ARG;
   if (kv->batch < 1 || kv->cap < 1 || !kv->seq_len || !kv->tokens || !kv->pos ||
       !kv_format_ok(c, kv))
@@ -972,6 +978,10 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
   // [hi | lo] queries and attention probabilities too (an e4m3 cache's layers
   // enter the attention as exact bf16 copies)
   const bool split_q = split;
+  // fp16 operands: the layer weights (the caller's), K/V (copied per layer),
+  // the queries, P and the GEMM activations; the tensor maps are the same
+  // (a tile copy moves 2-byte elements unchanged)
+  const bool f16 = (mode & CC_SCORE_F16) != 0;
   const ScoreWs L = score_layout(c, batch, cap, mode, split);
   const bool logit = (mode & 0xFF) == CC_SCORE_LOGIT;
   const bool keep_outside = (mode & CC_SCORE_RANGE_ONLY) != 0;   // other entries untouched
@@ -1006,7 +1016,8 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
     if (ss_tiles == 0) {
       TimedScope t(CC_KERNEL_RMSNORM, st);
       CC_TRY(launch_rmsnorm(first_from_bf16 ? kv->h_last : (const void *)h, !first_from_bf16,
-                            lw.attn_norm, xn, d, c->rms_eps, sl, cap, rows, split, st, rng_lo));
+                            lw.attn_norm, xn, d, c->rms_eps, sl, cap, rows, split, st, rng_lo, 0,
+                            f16, status));
     }
     // Q = RoPE(xn Wq^T)
     Gemm gq;
@@ -1023,6 +1034,7 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
     gq.p.out = q;
     gq.p.ldo = split_q ? 2 * qd : qd;
     gq.p.out_split = split_q ? 1 : 0;
+    gq.p.ab_f16 = gq.p.out_f16 = f16 ? 1 : 0;
     gq.p.pos = kv->pos;
     gq.p.bias = reinterpret_cast<const __nv_bfloat16 *>(lw.bq);
     gq.p.head_dim = c->head_dim;
@@ -1033,8 +1045,8 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
     // (act is free until the MLP: an e4m3 layer's bf16 copy for the tile attention)
     if ((s = run_attention(c, q, kv->k[l], kv->v[l], o, kv->seq_len, batch, cap, status, st,
                            split, nullptr, 0, nullptr, 0, kv_fmt(c, kv, l), split_q, rng_lo,
-                           rng_hi, act, (size_t)batch * cap * c->d_ff * 2 * (split ? 2 : 1))) !=
-        CC_OK)
+                           rng_hi, act, (size_t)batch * cap * c->d_ff * 2 * (split ? 2 : 1),
+                           f16)) != CC_OK)
       return s;
     // h = h + O Wo^T  (fast mode: h = H^(L-1) + O Wo^T)
     Gemm go;
@@ -1055,6 +1067,7 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
     go.p.ld_norm = split ? 2 * d : d;
     go.p.norm_split = split ? 1 : 0;
     go.p.ss_part = ss_part;
+    go.p.ab_f16 = go.p.out_f16 = f16 ? 1 : 0;
     plan_k_splits(go, epi_o, dev->sms, flags);
     if ((s = run_gemm(go, epi_o, CC_KERNEL_GEMM_OPROJ, dev->sms, st)) != CC_OK) return s;
     // act = silu(xn Wg^T / rms(h)) * (xn Wu^T / rms(h))
@@ -1070,6 +1083,7 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
     gu.p.n_ss = go.p.n_tiles;
     gu.p.ss_d = d;
     gu.p.eps = c->rms_eps;
+    gu.p.ab_f16 = gu.p.out_f16 = f16 ? 1 : 0;
     if ((s = run_gemm(gu, EPI_SWIGLU, CC_KERNEL_GEMM_GATEUP, dev->sms, st)) != CC_OK) return s;
     // h = h + act Wd^T; in logit mode the last layer's add is fused with the
     // head: per column tile, partial sums of h^2 and of h * g . W_U[x_i]
@@ -1081,6 +1095,7 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
     gd.p.row_lo = rng_lo;
     gd.p.out = h;
     gd.p.ldo = d;
+    gd.p.ab_f16 = gd.p.out_f16 = f16 ? 1 : 0;   // out_f16: the next layer's norm input
     if (epi_d == EPI_RESID_LOGIT) {
       gd.p.tokens = kv->tokens;
       gd.p.head_gain = reinterpret_cast<const __nv_bfloat16 *>(w->final_norm);
@@ -1434,6 +1449,19 @@ cc_status cc_score_full(const cc_model_cfg *cfg, const cc_model_weights *w,
   return run_score(cfg, w, cache, mode, scores, ws, ws_bytes, stream, true);
 }
 
+cc_status cc_bf16_to_f16(const void *src, void *dst, size_t n, void *stream) {
+  if (n == 0) return CC_OK;
+  if (!src || !dst || n % 8 || !aligned16(src) || !aligned16(dst)) return CC_ERR_INVALID_ARG;
+  const uintptr_t a = reinterpret_cast<uintptr_t>(src), b = reinterpret_cast<uintptr_t>(dst);
+  if (a < b + 2 * n && b < a + 2 * n) return CC_ERR_INVALID_ARG;   // overlapping
+  DevState *dev;
+  if (!dev_state(&dev)) return device_fail();
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  TimedScope t(CC_KERNEL_OTHER, st);
+  CC_TRY(launch_bf16_to_f16(src, dst, n, dev->sms, dev->status, st));
+  return CC_OK;
+}
+
 cc_status cc_score_rows(const cc_model_cfg *cfg, const cc_model_weights *w,
                         const cc_kv_cache *cache, cc_score_mode mode, int32_t full,
                         const int32_t *row_lo, const int32_t *row_hi, float *scores, void *ws,
@@ -1563,6 +1591,7 @@ const char *cc_status_str(cc_status s) {
     case CC_ERR_TIMEOUT: return "device wait timed out";
     case CC_ERR_UNSUPPORTED: return "unsupported shape";
     case CC_ERR_DEVICE_ARG: return "device-side argument out of range";
+    case CC_ERR_RANGE: return "value outside the fp16 range";
   }
   return "unknown status";
 }

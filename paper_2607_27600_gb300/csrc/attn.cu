@@ -38,6 +38,12 @@
 // tile costs 64 KB of shared memory at head_dim 128; the V ring then has one
 // stage.
 //
+// F16 (the fp16 operand mode of the scoring pass): Q, K and V arrive as fp16
+// (K and V as the caller's fp16 copy of the layer), P is written to TMEM as
+// fp16 and O is stored as fp16; both products then run with fp16 operands
+// (kind::f16 takes one type for A and B).  P <= 2^8 and |O| <= max |V|, so
+// neither can leave the fp16 range.
+//
 // TMEM columns: S0 [0,128)  S1 [128,256)  O0 [256,256+DH)  O1 [256+DH, 256+2DH)
 #include "attn.cuh"
 
@@ -133,7 +139,7 @@ CC_DEV UnitInfo decode_unit(const AttnParams &p, int unit_id, bool causal) {
   return u;
 }
 
-template <int DH, bool CAUSAL, bool SPLIT>
+template <int DH, bool CAUSAL, bool SPLIT, bool F16>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                 const __grid_constant__ CUtensorMap tmV, const __grid_constant__ AttnParams p) {
@@ -322,8 +328,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     // deterministic.
     if (lane == 0) {
       const int h_lo = warp - 9, h_hi = warp - 9;   // this issuer's M-half
-      constexpr uint32_t idesc_qk = make_idesc_bf16(128, BKV, 0, 0);   // every operand bf16
-      constexpr uint32_t idesc_pv = make_idesc_bf16(128, DH, 0, 1);
+      // every operand bf16 (fp16 with F16)
+      constexpr uint32_t idesc_qk = F16 ? make_idesc_f16(128, BKV, 0, 0) : make_idesc_bf16(128, BKV, 0, 0);
+      constexpr uint32_t idesc_pv = F16 ? make_idesc_f16(128, DH, 0, 1) : make_idesc_bf16(128, DH, 0, 1);
       // Shared-memory descriptors built once; a K step only advances the
       // start-address field (16-byte units): +2 per 16 columns of a 128-byte
       // row (Q, K), +128 per 16 keys of V.
@@ -511,7 +518,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           const float2 y = __ffma2_rn(make_float2(__uint_as_float(sr[c0 + k]),
                                                   __uint_as_float(sr[c0 + k + 1])), sl2v, nmv);
           const float2 e = make_float2(fast_exp2(y.x), fast_exp2(y.y));
-          pk[k / 2] = pack_bf16x2(e.x, e.y);
+          pk[k / 2] = F16 ? pack_f16x2(e.x, e.y) : pack_bf16x2(e.x, e.y);
           if constexpr (SPLIT)   // P_lo = bf16(p - P_hi)
             pl[k / 2] = pack_bf16x2(e.x - bf16_lo(pk[k / 2]), e.y - bf16_hi(pk[k / 2]));
           lsum = __fadd2_rn(lsum, e);
@@ -556,7 +563,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         uint32_t pk[16];
 #pragma unroll
         for (int k = 0; k < 32; k += 2)
-          pk[k / 2] = pack_bf16x2(__uint_as_float(o[k]) * inv, __uint_as_float(o[k + 1]) * inv);
+          pk[k / 2] = F16 ? pack_f16x2(__uint_as_float(o[k]) * inv, __uint_as_float(o[k + 1]) * inv)
+                          : pack_bf16x2(__uint_as_float(o[k]) * inv, __uint_as_float(o[k + 1]) * inv);
         if (store) {
           uint4 *d = reinterpret_cast<uint4 *>(dst + c);
 #pragma unroll
@@ -641,16 +649,21 @@ __global__ void attn_combine_kernel(const __grid_constant__ AttnParams p) {
   const float v = l > 0.f ? o * p.v_scale / l : 0.f;
   __nv_bfloat16 *dst = p.out + ((size_t)u.b * p.cap + pos) * p.out_ld +
                        (size_t)(u.g * G + hl) * p.head_dim + d;
+  if (p.f16) {   // fp16 operand mode: O as fp16 (the same 2 bytes)
+    const __half hf = __float2half_rn(v);
+    *dst = *reinterpret_cast<const __nv_bfloat16 *>(&hf);
+    return;
+  }
   const __nv_bfloat16 hi = __float2bfloat16_rn(v);
   *dst = hi;
   if (p.out_lo > 0) dst[p.out_lo] = __float2bfloat16_rn(v - __bfloat162float(hi));
 }
 
-template <int DH, bool CAUSAL, bool SPLIT = false>
+template <int DH, bool CAUSAL, bool SPLIT = false, bool F16 = false>
 cudaError_t launch_dh(const CUtensorMap &q, const CUtensorMap &k, const CUtensorMap &v,
                       const AttnParams &p, cudaStream_t stream) {
   using L = AttnSmem<DH, SPLIT>;
-  auto kern = attn_kernel<DH, CAUSAL, SPLIT>;
+  auto kern = attn_kernel<DH, CAUSAL, SPLIT, F16>;
   static bool attr_set[64] = {};
   int dev = 0;
   cudaGetDevice(&dev);
@@ -989,8 +1002,14 @@ cudaError_t launch_attention_decode(const AttnParams &p, cudaStream_t stream) {
 
 cudaError_t launch_attention(const CUtensorMap &q, const CUtensorMap &k, const CUtensorMap &v,
                              const AttnParams &p, cudaStream_t stream) {
-  // an e4m3 cache reaches the tile kernel as a bf16 copy (the caller's)
+  // an e4m3 cache reaches the tile kernel as a bf16 (or fp16) copy (the caller's)
   if (p.kv_fp8) return cudaErrorInvalidValue;
+  if (p.f16) {   // the fp16 operand scoring pass: counter-causal, single operands
+    if (p.causal || p.q_split || p.out_lo > 0) return cudaErrorInvalidValue;
+    if (p.head_dim == 128) return launch_dh<128, false, false, true>(q, k, v, p, stream);
+    if (p.head_dim == 64) return launch_dh<64, false, false, true>(q, k, v, p, stream);
+    return cudaErrorInvalidValue;
+  }
   if (p.causal) {
     if (p.head_dim == 128) return launch_dh<128, true>(q, k, v, p, stream);
     if (p.head_dim == 64) return launch_dh<64, true>(q, k, v, p, stream);

@@ -35,6 +35,8 @@ struct AttnParams {
                             // only: an e4m3 layer arrives as a bf16 copy of its codes); the
                             // K scale is folded into scale_log2 either way
   float v_scale;            // output = v_scale * (P V) / l (1 for a bf16 cache)
+  int f16;                  // tile kernel, counter-causal, no split: Q, K, V, P and the
+                            // output are fp16 (the fp16 operand mode of the scoring pass)
   KvLayout pg;              // paged K/V (pg.table nullptr: slot-major)
   int kv_rows;              // rows of the K/V tensor maps (a coordinate there reads zeros)
   unsigned *status;

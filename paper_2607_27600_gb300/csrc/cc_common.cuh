@@ -420,6 +420,31 @@ CC_DEV uint32_t pack_bf16x2(float lo, float hi) {
 }
 CC_DEV float bf16_lo(uint32_t v) { return __uint_as_float(v << 16); }
 CC_DEV float bf16_hi(uint32_t v) { return __uint_as_float(v & 0xFFFF0000u); }
+CC_DEV uint32_t pack_f16x2(float lo, float hi) {
+  __half2 v = __floats2half2_rn(lo, hi);
+  return *reinterpret_cast<uint32_t *>(&v);
+}
+
+// Largest finite fp16 value.  The fp16 operand mode (CC_SCORE_F16) reports
+// a value written as an fp16 operand whose magnitude exceeds it.
+constexpr float kF16Max = 65504.f;
+
+// A finite value that fp16 cannot hold (its magnitude above kF16Max).
+CC_DEV bool f16_overflow(float x) {
+  const float a = fabsf(x);
+  return a > kF16Max && a < INFINITY;
+}
+
+// Two activations as the next tensor-core product reads them: a bf16 pair,
+// or an fp16 pair (f16), recording in `over` a finite magnitude above
+// kF16Max (infinities and NaN pass through unflagged).
+CC_DEV uint32_t pack_act2(float lo, float hi, bool f16, bool &over) {
+  if (f16) {
+    over |= f16_overflow(lo) || f16_overflow(hi);
+    return pack_f16x2(lo, hi);
+  }
+  return pack_bf16x2(lo, hi);
+}
 
 // K/V layout.  Paged K/V: the pool row of logical slot i of sequence b.  Pages hold `page`
 // slots (a multiple of 128, so a key tile never straddles two pages); the

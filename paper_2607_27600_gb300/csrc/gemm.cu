@@ -84,7 +84,8 @@ CC_DEV float row_rms_scale(const GemmParams &p, int grow, bool valid) {
 
 // lo_off > 0 (bf16 only): also the lo half of each value, bf16(y - hi), at
 // element offset lo_off of the row (the precise pass's [hi | lo] queries).
-// rs: scale of the accumulator (before the bias and the rotation).
+// rs: scale of the accumulator (before the bias and the rotation).  With
+// p.out_f16 (not F8, lo_off 0) the values are written as fp16.
 template <int TBN, bool F8 = false>
 CC_DEV void rope_store(const GemmParams &p, uint32_t tacc, int grow, long long orow, bool valid,
                        void *out_base, int ldo, const __nv_bfloat16 *bias, int col0, int n_dest,
@@ -116,6 +117,7 @@ CC_DEV void rope_store(const GemmParams &p, uint32_t tacc, int grow, long long o
       }
       uint32_t o1[16], o2[16];
       [[maybe_unused]] uint32_t l1[16], l2[16];
+      [[maybe_unused]] bool over = false;
 #pragma unroll
       for (int k = 0; k < 32; k += 2) {
         float c_a, s_a, c_b, s_b;
@@ -140,12 +142,14 @@ CC_DEV void rope_store(const GemmParams &p, uint32_t tacc, int grow, long long o
         } else {
           const float y1a = a1 * c_a - a2 * s_a, y1b = b1 * c_b - b2 * s_b;
           const float y2a = a2 * c_a + a1 * s_a, y2b = b2 * c_b + b1 * s_b;
-          o1[k / 2] = pack_bf16x2(y1a, y1b);
-          o2[k / 2] = pack_bf16x2(y2a, y2b);
+          o1[k / 2] = pack_act2(y1a, y1b, p.out_f16, over);
+          o2[k / 2] = pack_act2(y2a, y2b, p.out_f16, over);
           l1[k / 2] = pack_bf16x2(y1a - bf16_lo(o1[k / 2]), y1b - bf16_hi(o1[k / 2]));
           l2[k / 2] = pack_bf16x2(y2a - bf16_lo(o2[k / 2]), y2b - bf16_hi(o2[k / 2]));
         }
       }
+      if constexpr (!F8)
+        if (over) set_status(p.status, CC_ERR_RANGE);
       constexpr int EB = F8 ? 1 : 2;
       uint4 *d1 = reinterpret_cast<uint4 *>(out_at<EB>(p, base, orow, ldo, hm, grow, col));
       uint4 *d2 = reinterpret_cast<uint4 *>(out_at<EB>(p, base, orow, ldo, hm, grow, col + half));
@@ -307,7 +311,8 @@ CC_DEV void logit_partials(const GemmParams &p, uint32_t tacc, int grow, bool va
 
 // fp32 outputs (EPI_F32, EPI_RESID_*), through the staging tile: out = acc
 // (+ bf16 resid, or += for RESID_F32); with norm_out (last K split) also
-// bf16(out * norm_gain) (and the lo part) and the tile's partial sum of out^2.
+// bf16(out * norm_gain) (and the lo part; fp16 instead with out_f16) and the
+// tile's partial sum of out^2.
 template <int EPI, int TBN>
 CC_DEV void f32_epilogue(const GemmParams &p, uint32_t tacc, int grow, bool valid, int nt,
                          int tile_n0, bool last, float *stage) {
@@ -363,7 +368,10 @@ CC_DEV void f32_epilogue(const GemmParams &p, uint32_t tacc, int grow, bool vali
         ss[i] = fmaf(a[i].w, a[i].w, ss[i]);
         const float y0 = a[i].x * g4[0], y1 = a[i].y * g4[1], y2 = a[i].z * g4[2],
                     y3 = a[i].w * g4[3];
-        const uint32_t h0 = pack_bf16x2(y0, y1), h1 = pack_bf16x2(y2, y3);
+        bool over = false;
+        const uint32_t h0 = pack_act2(y0, y1, p.out_f16, over),
+                       h1 = pack_act2(y2, y3, p.out_f16, over);
+        if (over) set_status(p.status, CC_ERR_RANGE);
         __nv_bfloat16 *dn = p.norm_out + row * p.ld_norm + col + cq;
         *reinterpret_cast<uint2 *>(dn) = make_uint2(h0, h1);
         if (p.norm_split)   // lo = y * gain - hi, at column offset N
@@ -449,8 +457,10 @@ CC_DEV void epilogue_tile(const GemmParams &p, uint32_t tacc, int grow, bool val
       for (int k = 0; k < 32; ++k)
         y[k] = silu(__uint_as_float(g[k]) * rs) * (__uint_as_float(u[k]) * rs);
       uint32_t o[16];
+      bool over = false;
 #pragma unroll
-      for (int k = 0; k < 32; k += 2) o[k / 2] = pack_bf16x2(y[k], y[k + 1]);
+      for (int k = 0; k < 32; k += 2) o[k / 2] = pack_act2(y[k], y[k + 1], p.out_f16, over);
+      if (over) set_status(p.status, CC_ERR_RANGE);
       uint4 *d = reinterpret_cast<uint4 *>(out + col);
 #pragma unroll
       for (int v = 0; v < 4; ++v) d[v] = make_uint4(o[v * 4], o[v * 4 + 1], o[v * 4 + 2], o[v * 4 + 3]);
@@ -698,7 +708,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp == 1) {
     if (lane == 0 && rank == 0) {  // ---------------- MMA issuer (CTA 0 of a pair)
-      constexpr uint32_t idesc = make_idesc_bf16(PAIR ? 2 * BM : BM, TBN, 0, 0);
+      const uint32_t idesc = p.ab_f16 ? make_idesc_f16(PAIR ? 2 * BM : BM, TBN, 0, 0)
+                                      : make_idesc_bf16(PAIR ? 2 * BM : BM, TBN, 0, 0);
       const uint64_t a_desc0 = make_sdesc_sw128(smem_u32(sA), 16, 1024);
       const uint64_t b_desc0 = make_sdesc_sw128(smem_u32(sB), 16, 1024);
       int stage = 0, acc = 0;

@@ -68,6 +68,10 @@ struct GemmParams {
                            // raster 1 groups count pairs of row tiles
   int out_split;           // EPI_SWIGLU, EPI_QROPE (not into the cache): out rows are
                            // [hi | lo], lo at column offset N
+  int ab_f16;              // A and W are fp16 (else bf16): the fp16 operand mode
+  int out_f16;             // the activations written for the next product (EPI_SWIGLU and
+                           // EPI_QROPE out, norm_out) are fp16 (not with the splits); a
+                           // value above 65504 in magnitude sets CC_ERR_RANGE in status
   int k_splits;            // EPI_RESID_F32 / EPI_RESID_LOGIT only: K range split over
                            // k_splits work items per tile (< one wave of tiles); the splits
                            // add into out in order (EPI_RESID_LOGIT: the last one takes the

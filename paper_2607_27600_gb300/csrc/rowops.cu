@@ -5,6 +5,8 @@
 // One warp per cache row, rows = b*cap + i; rows with i >= seq_len[b] are
 // skipped (the heads write -inf there).  All are HBM-bound streams with
 // 16-byte vector accesses.
+#include <algorithm>
+
 #include "rowops.cuh"
 
 namespace cc {
@@ -99,19 +101,20 @@ CC_DEV float row_inv_rms(const void *row, int d, float eps, int lane) {
   return rsqrtf(ss / (float)d + eps);
 }
 
-// Elements [e, e+8) of the normalised row: bf16(f * inv * gain), and with
-// split the remainder at column offset d.
+// Elements [e, e+8) of the normalised row: bf16(f * inv * gain) (fp16 with
+// f16, a magnitude above kF16Max recorded in `over`), and with split the
+// remainder at column offset d.
 CC_DEV void store_norm8(__nv_bfloat16 *o, int d, int e, const float *f, const uint4 &g, float inv,
-                        int split) {
+                        int split, bool f16, bool &over) {
   float gf[8], y[8];
   unpack8(g, gf);
 #pragma unroll
   for (int k = 0; k < 8; ++k) y[k] = f[k] * inv * gf[k];
   uint4 v;
-  v.x = pack_bf16x2(y[0], y[1]);
-  v.y = pack_bf16x2(y[2], y[3]);
-  v.z = pack_bf16x2(y[4], y[5]);
-  v.w = pack_bf16x2(y[6], y[7]);
+  v.x = pack_act2(y[0], y[1], f16, over);
+  v.y = pack_act2(y[2], y[3], f16, over);
+  v.z = pack_act2(y[4], y[5], f16, over);
+  v.w = pack_act2(y[6], y[7], f16, over);
   *reinterpret_cast<uint4 *>(o + e) = v;
   if (split) {
     uint4 lo;
@@ -124,12 +127,13 @@ CC_DEV void store_norm8(__nv_bfloat16 *o, int d, int e, const float *f, const ui
 }
 
 // out (bf16) = x * gain / rms(x).  split: the row holds [hi | lo] (2d values),
-// hi = bf16(y), lo = bf16(y - hi), so hi + lo carries y to ~2^-17.
+// hi = bf16(y), lo = bf16(y - hi), so hi + lo carries y to ~2^-17.  f16: out
+// is fp16 instead (not with split); a value above kF16Max is reported.
 template <bool IN_F32>
 __global__ void __launch_bounds__(kWarps * 32)
     rmsnorm_kernel(const void *x, const __nv_bfloat16 *gain, __nv_bfloat16 *out, int d, float eps,
                    const int32_t *seq_len, const int32_t *row_lo, int cap, int rows, int span,
-                   int split) {
+                   int split, int f16, unsigned *status) {
   const int lane = threadIdx.x & 31;
   int row;
   if (!warp_row(seq_len, row_lo, cap, rows, span, blockIdx.x * kWarps + (threadIdx.x >> 5), row))
@@ -138,6 +142,7 @@ __global__ void __launch_bounds__(kWarps * 32)
   const void *xr = reinterpret_cast<const uint8_t *>(x) + (size_t)row * d * es;
   const float inv = row_inv_rms<IN_F32>(xr, d, eps, lane);
   __nv_bfloat16 *o = out + (size_t)row * d * (split ? 2 : 1);
+  bool over = false;
   int e = lane * 8;
   for (; e + 3 * 256 < d; e += 4 * 256) {
     float f[4][8];
@@ -148,13 +153,14 @@ __global__ void __launch_bounds__(kWarps * 32)
       g[u] = *reinterpret_cast<const uint4 *>(gain + e + u * 256);
     }
 #pragma unroll
-    for (int u = 0; u < 4; ++u) store_norm8(o, d, e + u * 256, f[u], g[u], inv, split);
+    for (int u = 0; u < 4; ++u) store_norm8(o, d, e + u * 256, f[u], g[u], inv, split, f16, over);
   }
   for (; e < d; e += 256) {
     float f[8];
     load8<IN_F32>(xr, e, f);
-    store_norm8(o, d, e, f, *reinterpret_cast<const uint4 *>(gain + e), inv, split);
+    store_norm8(o, d, e, f, *reinterpret_cast<const uint4 *>(gain + e), inv, split, f16, over);
   }
+  if (over) set_status(status, CC_ERR_RANGE);
 }
 
 // h (fp32) = embed[tokens[row]]
@@ -349,17 +355,19 @@ int warps_for(int rows, int cap, int span, const int32_t *row_lo) {
 
 cudaError_t launch_rmsnorm(const void *x, bool x_f32, const void *gain, void *out, int d, float eps,
                            const int32_t *seq_len, int cap, int rows, bool split, cudaStream_t st,
-                           const int32_t *row_lo, int span) {
+                           const int32_t *row_lo, int span, bool f16, unsigned *status) {
   if (rows <= 0) return cudaSuccess;
+  if (split && f16) return cudaErrorInvalidValue;
   auto *g = reinterpret_cast<const __nv_bfloat16 *>(gain);
   auto *o = reinterpret_cast<__nv_bfloat16 *>(out);
   const unsigned blocks = blocks_for(warps_for(rows, cap, span, row_lo));
   if (x_f32)
     rmsnorm_kernel<true><<<blocks, kWarps * 32, 0, st>>>(x, g, o, d, eps, seq_len, row_lo, cap, rows,
-                                                          span, split ? 1 : 0);
+                                                          span, split ? 1 : 0, f16 ? 1 : 0, status);
   else
     rmsnorm_kernel<false><<<blocks, kWarps * 32, 0, st>>>(x, g, o, d, eps, seq_len, row_lo, cap,
-                                                           rows, span, split ? 1 : 0);
+                                                           rows, span, split ? 1 : 0, f16 ? 1 : 0,
+                                                           status);
   return cudaGetLastError();
 }
 
@@ -397,15 +405,20 @@ cudaError_t launch_argmax_combine(const float2 *part, int n_tiles, const int32_t
   return cudaGetLastError();
 }
 
-// e4m3 K/V codes of one layer -> bf16 (exact: every e4m3 value is a bf16
-// value), into slot-major rows b * cap + i, i < seq_end[b], from a slot-major,
-// paged or head-major cache.  One thread converts 16 codes of K and of V.
-// A paged row outside the pool is reported and skipped.
+namespace {
+
+// One layer's K/V as a slot-major copy for the tile attention: e4m3 codes ->
+// bf16 or fp16 (exact: every e4m3 value is both), or bf16 -> fp16 (exact for
+// magnitudes in [2^-14, 65504]; a larger one is reported), into rows
+// b * cap + i, i < seq_end[b], from a slot-major, paged or head-major cache.
+// One thread converts 16 elements of K and of V.  A paged row outside the
+// pool is reported and skipped.
+template <bool IN_FP8, bool OUT_F16>
 __global__ void __launch_bounds__(256)
-    kv_to_bf16_kernel(const uint8_t *k, const uint8_t *v, KvLayout pg, int cap, int hkv, int dh,
-                      const int32_t *seq_end, int batch, __nv_bfloat16 *ko, __nv_bfloat16 *vo,
-                      unsigned *status) {
-  const int chunks = hkv * dh / 16;   // 16-code chunks of one slot
+    kv_copy_kernel(const uint8_t *k, const uint8_t *v, KvLayout pg, int cap, int hkv, int dh,
+                   const int32_t *seq_end, int batch, uint16_t *ko, uint16_t *vo,
+                   unsigned *status) {
+  const int chunks = hkv * dh / 16;   // 16-element chunks of one slot
   const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
   if (idx >= (long long)batch * cap * chunks) return;
   const long long row = idx / chunks;
@@ -425,35 +438,89 @@ __global__ void __launch_bounds__(256)
     src = (r * hkv + h) * dh + e;
   }
   const size_t dst = (size_t)row * hkv * dh + (size_t)h * dh + e;
-  auto convert = [](const uint8_t *in, __nv_bfloat16 *out) {
-    const uint4 x = *reinterpret_cast<const uint4 *>(in);
-    const uint32_t w[4] = {x.x, x.y, x.z, x.w};
+  bool over = false;
+  auto convert = [&over](const uint8_t *in, uint16_t *out) {
     uint32_t o[8];
+    if constexpr (IN_FP8) {
+      const uint4 x = *reinterpret_cast<const uint4 *>(in);
+      const uint32_t w[4] = {x.x, x.y, x.z, x.w};
 #pragma unroll
-    for (int j = 0; j < 4; ++j)
+      for (int j = 0; j < 4; ++j)
 #pragma unroll
-      for (int hf = 0; hf < 2; ++hf) {   // two codes -> f16 pair (exact) -> bf16 pair (exact)
-        uint32_t f2;
-        asm("cvt.rn.f16x2.e4m3x2 %0, %1;" : "=r"(f2) : "h"((unsigned short)(w[j] >> (16 * hf))));
-        const float2 f = __half22float2(*reinterpret_cast<const __half2 *>(&f2));
-        o[j * 2 + hf] = pack_bf16x2(f.x, f.y);
-      }
+        for (int hf = 0; hf < 2; ++hf) {   // two codes -> f16 pair (exact) [-> bf16 pair (exact)]
+          uint32_t f2;
+          asm("cvt.rn.f16x2.e4m3x2 %0, %1;" : "=r"(f2) : "h"((unsigned short)(w[j] >> (16 * hf))));
+          if constexpr (OUT_F16) {
+            o[j * 2 + hf] = f2;
+          } else {
+            const float2 f = __half22float2(*reinterpret_cast<const __half2 *>(&f2));
+            o[j * 2 + hf] = pack_bf16x2(f.x, f.y);
+          }
+        }
+    } else {   // bf16 -> fp16
+      const uint4 *x = reinterpret_cast<const uint4 *>(in);
+      const uint4 a = x[0], bq = x[1];
+      const uint32_t w[8] = {a.x, a.y, a.z, a.w, bq.x, bq.y, bq.z, bq.w};
+#pragma unroll
+      for (int j = 0; j < 8; ++j) o[j] = pack_act2(bf16_lo(w[j]), bf16_hi(w[j]), true, over);
+    }
     uint4 *d = reinterpret_cast<uint4 *>(out);
     d[0] = make_uint4(o[0], o[1], o[2], o[3]);
     d[1] = make_uint4(o[4], o[5], o[6], o[7]);
   };
-  convert(k + src, ko + dst);
-  convert(v + src, vo + dst);
+  constexpr int EB = IN_FP8 ? 1 : 2;   // input bytes per element
+  convert(k + src * EB, ko + dst);
+  convert(v + src * EB, vo + dst);
+  if (over) set_status(status, CC_ERR_RANGE);
 }
 
-cudaError_t launch_kv_to_bf16(const uint8_t *k, const uint8_t *v, const KvLayout &pg, int cap,
-                              int hkv, int dh, const int32_t *seq_end, int batch,
-                              __nv_bfloat16 *k_out, __nv_bfloat16 *v_out, unsigned *status,
-                              cudaStream_t st) {
+// dst (fp16) = src (bf16), 8 values per thread and step (grid-stride).
+__global__ void __launch_bounds__(256)
+    bf16_to_f16_kernel(const uint4 *src, uint4 *dst, size_t n8, unsigned *status) {
+  bool over = false;
+  for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < n8;
+       i += (size_t)gridDim.x * blockDim.x) {
+    const uint4 x = src[i];
+    dst[i] = make_uint4(pack_act2(bf16_lo(x.x), bf16_hi(x.x), true, over),
+                        pack_act2(bf16_lo(x.y), bf16_hi(x.y), true, over),
+                        pack_act2(bf16_lo(x.z), bf16_hi(x.z), true, over),
+                        pack_act2(bf16_lo(x.w), bf16_hi(x.w), true, over));
+  }
+  if (over) set_status(status, CC_ERR_RANGE);
+}
+
+}  // namespace
+
+cudaError_t launch_kv_copy(const uint8_t *k, const uint8_t *v, bool in_fp8, bool out_f16,
+                           const KvLayout &pg, int cap, int hkv, int dh, const int32_t *seq_end,
+                           int batch, void *k_out, void *v_out, unsigned *status,
+                           cudaStream_t st) {
   const long long n = (long long)batch * cap * (hkv * dh / 16);
   if (n <= 0) return cudaSuccess;
-  kv_to_bf16_kernel<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(k, v, pg, cap, hkv, dh, seq_end,
-                                                                 batch, k_out, v_out, status);
+  if (!in_fp8 && !out_f16) return cudaErrorInvalidValue;   // bf16 -> bf16: no copy needed
+  auto *ko = reinterpret_cast<uint16_t *>(k_out);
+  auto *vo = reinterpret_cast<uint16_t *>(v_out);
+  const unsigned blocks = (unsigned)((n + 255) / 256);
+  if (in_fp8 && out_f16)
+    kv_copy_kernel<true, true><<<blocks, 256, 0, st>>>(k, v, pg, cap, hkv, dh, seq_end, batch, ko,
+                                                       vo, status);
+  else if (in_fp8)
+    kv_copy_kernel<true, false><<<blocks, 256, 0, st>>>(k, v, pg, cap, hkv, dh, seq_end, batch, ko,
+                                                        vo, status);
+  else
+    kv_copy_kernel<false, true><<<blocks, 256, 0, st>>>(k, v, pg, cap, hkv, dh, seq_end, batch, ko,
+                                                        vo, status);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_bf16_to_f16(const void *src, void *dst, size_t n, int sms, unsigned *status,
+                               cudaStream_t st) {
+  const size_t n8 = n / 8;
+  if (n8 == 0) return cudaSuccess;
+  const size_t want = (n8 + 255) / 256;
+  const unsigned blocks = (unsigned)std::min<size_t>(want, (size_t)sms * 8);
+  bf16_to_f16_kernel<<<blocks, 256, 0, st>>>(reinterpret_cast<const uint4 *>(src),
+                                             reinterpret_cast<uint4 *>(dst), n8, status);
   return cudaGetLastError();
 }
 

@@ -9,9 +9,12 @@ namespace cc {
 // Row kernels visit rows b*cap + i with row_lo[b] <= i < seq_len[b] (row_lo
 // null: from 0).  span > 0 (with row_lo): seq_len[b] - row_lo[b] <= span, and
 // the launch has batch * span warps instead of one per cache row.
+// f16: out is fp16 [rows][d] instead (not with split); a value above 65504 in
+// magnitude sets CC_ERR_RANGE in status.
 cudaError_t launch_rmsnorm(const void *x, bool x_f32, const void *gain, void *out, int d, float eps,
                            const int32_t *seq_len, int cap, int rows, bool split, cudaStream_t st,
-                           const int32_t *row_lo = nullptr, int span = 0);
+                           const int32_t *row_lo = nullptr, int span = 0, bool f16 = false,
+                           unsigned *status = nullptr);
 // h fp32 [rows][d] = embed[tokens[row]]
 cudaError_t launch_embed(const void *embed, const int32_t *tokens, float *h, int d, int vocab,
                          const int32_t *seq_len, int cap, int rows, unsigned *status,
@@ -27,12 +30,19 @@ cudaError_t launch_append_prepare(const int32_t *seq_len, const int32_t *count,
                                   int32_t *tokens, int32_t *pos, int32_t *row_lo, int32_t *row_hi,
                                   int batch, int cap, unsigned *status, cudaStream_t st);
 // seq_len = row_hi
-// One layer of an e4m3 cache as bf16 (exact), slot-major [batch * cap][hkv][dh]
-// for the slots i < seq_end[b] (dh a multiple of 16).
-cudaError_t launch_kv_to_bf16(const uint8_t *k, const uint8_t *v, const KvLayout &pg, int cap,
-                              int hkv, int dh, const int32_t *seq_end, int batch,
-                              __nv_bfloat16 *k_out, __nv_bfloat16 *v_out, unsigned *status,
-                              cudaStream_t st);
+// One layer of the cache copied for the tile attention, slot-major
+// [batch * cap][hkv][dh] for the slots i < seq_end[b] (dh a multiple of 16):
+// e4m3 codes (in_fp8) as bf16 or fp16 (out_f16) values, exact either way, or
+// bf16 as fp16 (exact for magnitudes in [2^-14, 65504]; a larger one sets
+// CC_ERR_RANGE).  bf16 to bf16 is refused (cudaErrorInvalidValue).
+cudaError_t launch_kv_copy(const uint8_t *k, const uint8_t *v, bool in_fp8, bool out_f16,
+                           const KvLayout &pg, int cap, int hkv, int dh, const int32_t *seq_end,
+                           int batch, void *k_out, void *v_out, unsigned *status,
+                           cudaStream_t st);
+// dst (fp16) = src (bf16) for n elements (n a multiple of 8, both 16-byte
+// aligned); a finite value above 65504 in magnitude sets CC_ERR_RANGE.
+cudaError_t launch_bf16_to_f16(const void *src, void *dst, size_t n, int sms, unsigned *status,
+                               cudaStream_t st);
 cudaError_t launch_append_finish(int32_t *seq_len, const int32_t *row_hi, int batch,
                                  cudaStream_t st);
 // next[b] = first column of the largest logit over the (max, column) tile

@@ -24,6 +24,8 @@ about 2^-17 relative; a tensor-core product then runs once per half):
                projection's normalised input, the attention output) split
   split-qp-mlp   queries, P and the MLP's GEMM inputs (the gate/up
                projection's normalised input, the SwiGLU output) split
+  fp16-pass    every rounding point of `bf16-pass` in fp16 instead, with the
+               weights and cached K/V converted to fp16 as well
 
 The drift measured here is a property of the arithmetic and of the random
 model, not of any kernel; the full-pass tolerances of the parity tests are
@@ -58,6 +60,12 @@ def split(x):
 
 def exact(x):
     return x
+
+
+def f16(x):
+    """Round to the nearest fp16 value (ties to even; subnormals below
+    2^-14), kept in fp64."""
+    return np.asarray(x, np.float64).astype(np.float32).astype(np.float16).astype(np.float64)
 
 
 def attention_rounded_p(q, k, v, rows, n, rp):
@@ -95,11 +103,19 @@ VARIANTS = {
     "split-qp": (split, bf16, split, fp32),                  # attention operands only
     "split-qp-attn": (split, (split, bf16), split, fp32),    # + the attention-side GEMM inputs
     "split-qp-mlp": (split, (bf16, split), split, fp32),     # + the MLP GEMM inputs
+    # every tensor-core operand in fp16: the bf16 weights and cached K/V
+    # converted (exact but for magnitudes below 2^-14), the activations,
+    # queries and P rounded to fp16
+    "fp16-pass": (f16, f16, f16, fp32, f16),
 }
 
 
 def layer(h, rows, pos, lw, k, v, n, shape, rounding):
-    rq, ra, rp, rh = rounding
+    rq, ra, rp, rh = rounding[:4]
+    if len(rounding) > 4:   # the weights and the cached K/V as the tensor cores see them
+        rw = rounding[4]
+        lw = {name: rw(w) for name, w in lw.items()}
+        k, v = rw(k), rw(v)
     ra, rm = ra if isinstance(ra, tuple) else (ra, ra)   # attention-side, MLP GEMM inputs
     a = ra(R.rms_norm(h, lw["attn_norm"], shape.rms_eps))
     q = (a @ R.f64(lw["wq"]).T).reshape(len(rows), shape.n_q_heads, shape.head_dim)

@@ -5,7 +5,8 @@ columns wide (CC_GEMM_PAIRS=2), so that the small seeded workloads the
 oracle checks row by row reach it too: odd row-tile counts (the second CTA
 of the last pair stores nothing), pairs whose two row tiles belong to
 different sequences, ragged column counts and every epilogue of the refresh
-(Sec. 3.1), of the append and of the fused q/k/v projections.  The
+(Sec. 3.1) in bf16 and fp16 operands, of the append and of the fused q/k/v
+projections.  The
 full-size parity tests run the default choice, which pairs the large
 launches."""
 import os
@@ -16,6 +17,7 @@ import torch
 
 import synth
 import tests.test_gpu_append as append_tests
+import tests.test_gpu_f16 as f16_tests
 import tests.test_gpu_fp8 as fp8_tests
 import tests.test_gpu_kernels as kernel_tests
 import tests.test_gpu_paged as paged_tests
@@ -49,6 +51,8 @@ test_fp8_append_llama_fused_projection = fp8_tests.test_fp8_append_llama_fused_p
 test_fp8_scores_small_ragged = fp8_tests.test_fp8_scores_small_ragged
 test_fp8_precise_mode_small_ragged = fp8_tests.test_fp8_precise_mode_small_ragged
 test_paged_append_matches_slot_major = paged_tests.test_paged_append_matches_slot_major
+test_tiny_f16_mode_all_rows = f16_tests.test_tiny_f16_mode_all_rows
+test_small_two_layer_f16_ragged = f16_tests.test_small_two_layer_f16_ragged
 
 
 def _linear(cc, x, w):
