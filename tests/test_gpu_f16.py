@@ -214,3 +214,42 @@ def test_f16_mode_rejects_the_precise_flag(cc, tiny):
     with pytest.raises(cc.CCError) as e:
         cc.cc_score_layer(wl.shape, weights, cache, mode, scores, ws)
     assert e.value.code == cc.CC_ERR_INVALID_ARG
+
+
+@pytest.mark.parametrize("layout", ["paged", "head_major", "e4m3_paged"])
+def test_f16_cache_layouts_match_slot_major(cc, layout):
+    """Qwen2.5-7B last layer (G = 7, head_dim 128), two sequences of 4096 and
+    2500 slots: the fp16 mode over a paged, a head-major and a paged e4m3
+    cache (each layer's K/V copied to fp16 through the block table or by
+    head) writes the slot-major cache's scores bit for bit; the slot-major
+    scores match the oracle on sampled rows within 2e-3."""
+    import bench
+    import paper_2607_27600_gb300 as pkg
+    from tests.test_gpu_fullsize import host_view, sample
+    shape = synth.WORKLOADS["qwen7b-table1-fast-4096"].shape
+    seq, cap = [4096, 2500], 4096
+    last = shape.n_layers - 1
+    w = synth.model_weights(shape, 81, device="cuda", layers=[last], with_embed=False)
+    c = synth.synthetic_cache(shape, seq, cap, 82, device="cuda")
+    if layout == "e4m3_paged":
+        bench.to_e4m3_cache(c)
+    weights = pkg.Weights(cc.f16_weights(w))
+    mode = cc.SCORE_LOGIT | cc.SCORE_F16
+    ref = _score(cc, shape, weights, pkg.Cache(dict(c)), mode, False)
+    if layout == "head_major":
+        for key in ("k", "v"):
+            c[key] = [None if x is None else x.permute(0, 2, 1, 3).contiguous() for x in c[key]]
+        c["kv_layout"] = 1
+    else:
+        bench.to_paged_cache(c, 256, 83)
+    got = _score(cc, shape, weights, pkg.Cache(c), mode, False)
+    for i, n in enumerate(seq):
+        assert torch.equal(got[i, :n].view(torch.int32), ref[i, :n].view(torch.int32)), i
+    if layout == "head_major":   # the oracle once, on the slot-major draw
+        c = synth.synthetic_cache(shape, seq, cap, 82, device="cuda")
+        wn, cn = host_view(w, c)
+        rows = sample(seq, 24, seed=84)
+        want = oracle.score_layer(shape, wn, cn, rows=rows)
+        r = ref.cpu().numpy()
+        err = max(rel_err(r[i, rw], want[i, rw]) for i, rw in enumerate(rows))
+        assert err < TOL and err < 2e-3, err
