@@ -218,43 +218,13 @@ def test_full_pass_32_layers_sampled_rows(pkg):
     assert check_rows(default, want, rows) < DEFAULT_FULL32_TOL
 
 
-def test_headline_keep_set_full_oracle(pkg):
-    """llama8b-layer-8k end to end: every row scored by the oracle; the GPU
-    keep-set is identical where the oracle's boundary gap exceeds the
-    tolerance, else overlaps >= 99.5 %; the GPU select equals the oracle's
-    select on the same fp32 scores exactly."""
+def _gpu_keep(pkg, wl, w, c, mode):
+    """GPU scores of the whole batch in `mode` and the GPU keep-set on them,
+    which must equal the oracle's select on the same fp32 scores exactly."""
     from paper_2607_27600_gb300 import cc
-    wl = synth.WORKLOADS["llama8b-layer-8k"]
-    w, c = workload_inputs(wl)
-    got = gpu_scores(pkg, wl.shape, w, c, cc.SCORE_LOGIT, full=False)
-    wn, cn = host_view(w, c)
-    want = oracle.score_layer(wl.shape, wn, cn)
-    assert rel_err(got, want) < TOL
-    b, cap = c["tokens"].shape
-    idx = torch.empty(b, cap, dtype=torch.int32, device="cuda")
-    cnt = torch.empty(b, dtype=torch.int32, device="cuda")
-    cc.cc_select_keep(torch.from_numpy(got).cuda(), c["seq_len"], b, cap,
-                      torch.tensor(wl.budgets, dtype=torch.int32, device="cuda"), 0, idx, cnt)
-    gi, gc = idx.cpu().numpy(), cnt.cpu().numpy()
-    oi, oc = oracle.select_keep(got, wl.seq_lens, wl.budgets)
-    assert np.array_equal(gc, oc) and np.array_equal(gi[0, :oc[0]], oi[0, :oc[0]])
-    wi, wc = oracle.select_keep(want.astype(np.float32), wl.seq_lens, wl.budgets)
-    ok, det = keep_set_ok(gi, gc, wi, wc, want, wl.seq_lens, wl.budgets)
-    assert ok, det
-
-
-def test_ragged_batch_keep_set_per_sequence_budget(pkg):
-    """llama8b-layer-32k-ragged (Algorithm DoMemRefresh per sequence, budgets
-    25 % of each length): the whole batch scored and selected on the GPU in
-    one call each, as bench.py times it; the 8192-slot sequence's keep-set
-    (budget 2048) checked against the oracle's scores of every one of its
-    rows: identical where the boundary gap exceeds the tolerance, else >= 99.5 %
-    overlap with near-tie swaps only; the other sequences' keep-sets equal the
-    oracle's select on the GPU's own scores."""
-    from paper_2607_27600_gb300 import cc
-    wl = synth.WORKLOADS["llama8b-layer-32k-ragged"]
-    w, c = workload_inputs(wl)
-    got = gpu_scores(pkg, wl.shape, w, c, cc.SCORE_LOGIT, full=False)
+    if mode & cc.SCORE_F16:
+        w = cc.f16_weights(w)
+    got = gpu_scores(pkg, wl.shape, w, c, mode, full=False)
     b, cap = c["tokens"].shape
     idx = torch.empty(b, cap, dtype=torch.int32, device="cuda")
     cnt = torch.empty(b, dtype=torch.int32, device="cuda")
@@ -266,16 +236,52 @@ def test_ragged_batch_keep_set_per_sequence_budget(pkg):
     assert np.array_equal(gc, oc)
     for s_ in range(b):
         assert np.array_equal(gi[s_, :oc[s_]], oi[s_, :oc[s_]]), s_
+    return got, gi, gc
+
+
+def test_headline_keep_set_full_oracle(pkg):
+    """llama8b-layer-8k end to end, with bf16 and with fp16 operands: every
+    row scored by the oracle; the GPU keep-set is identical where the
+    oracle's boundary gap exceeds the tolerance, else overlaps >= 99.5 %; the
+    GPU select equals the oracle's select on the same fp32 scores exactly."""
+    from paper_2607_27600_gb300 import cc
+    wl = synth.WORKLOADS["llama8b-layer-8k"]
+    w, c = workload_inputs(wl)
+    runs = [_gpu_keep(pkg, wl, w, c, m) for m in (cc.SCORE_LOGIT, cc.SCORE_LOGIT | cc.SCORE_F16)]
+    wn, cn = host_view(w, c)
+    want = oracle.score_layer(wl.shape, wn, cn)
+    wi, wc = oracle.select_keep(want.astype(np.float32), wl.seq_lens, wl.budgets)
+    for got, gi, gc in runs:
+        assert rel_err(got, want) < TOL
+        ok, det = keep_set_ok(gi, gc, wi, wc, want, wl.seq_lens, wl.budgets)
+        assert ok, det
+
+
+def test_ragged_batch_keep_set_per_sequence_budget(pkg):
+    """llama8b-layer-32k-ragged (Algorithm DoMemRefresh per sequence, budgets
+    25 % of each length), with bf16 and with fp16 operands: the whole batch
+    scored and selected on the GPU in one call each, as bench.py times it;
+    the 8192-slot sequence's keep-set (budget 2048) checked against the
+    oracle's scores of every one of its rows: identical where the boundary
+    gap exceeds the tolerance, else >= 99.5 % overlap with near-tie swaps
+    only; every sequence's keep-set equals the oracle's select on the GPU's
+    own scores."""
+    from paper_2607_27600_gb300 import cc
+    wl = synth.WORKLOADS["llama8b-layer-32k-ragged"]
+    w, c = workload_inputs(wl)
+    b = c["tokens"].shape[0]
+    runs = [_gpu_keep(pkg, wl, w, c, m) for m in (cc.SCORE_LOGIT, cc.SCORE_LOGIT | cc.SCORE_F16)]
     seq = int(np.argmin(wl.seq_lens))               # the 8192-slot sequence
     n = wl.seq_lens[seq]
     wn, cn = host_view(w, c)
     rows = [np.arange(n) if s_ == seq else np.array([], np.int64) for s_ in range(b)]
     want = oracle.score_layer(wl.shape, wn, cn, rows=rows)
-    assert rel_err(got[seq, :n], want[seq, :n]) < TOL
     wi, wc = oracle.select_keep(want[seq:seq + 1].astype(np.float32), [n], [wl.budgets[seq]])
-    ok, det = keep_set_ok(gi[seq:seq + 1], gc[seq:seq + 1], wi, wc, want[seq:seq + 1], [n],
-                          [wl.budgets[seq]])
-    assert ok, det
+    for got, gi, gc in runs:
+        assert rel_err(got[seq, :n], want[seq, :n]) < TOL
+        ok, det = keep_set_ok(gi[seq:seq + 1], gc[seq:seq + 1], wi, wc, want[seq:seq + 1], [n],
+                              [wl.budgets[seq]])
+        assert ok, det
 
 
 def seeded_keep(n, budget, seed):
