@@ -335,7 +335,21 @@ def cc_score_workspace_size(cfg, batch: int, cap: int, mode: int = SCORE_LOGIT) 
     return int(load_library().cc_score_workspace_size(ctypes.byref(_cfg(cfg)), batch, cap, mode))
 
 
+def _check_operand_type(weights, mode):
+    """The layer matrices must be fp16 exactly when the mode has SCORE_F16
+    (the library reads the same pointers as bf16 otherwise)."""
+    want = torch.float16 if int(mode) & SCORE_F16 else torch.bfloat16
+    for l, lw in enumerate(weights.w["layers"]):
+        if lw is None:
+            continue
+        for f in F16_MATRICES:
+            if lw[f].dtype != want:
+                raise ValueError(f"layers[{l}].{f} is {lw[f].dtype}; this mode reads {want} "
+                                 "(f16_weights converts the matrices for SCORE_F16)")
+
+
 def _score(fn, cfg, weights: Weights, cache: Cache, mode, scores, ws, stream):
+    _check_operand_type(weights, mode)
     c = _cfg(cfg)
     code = getattr(load_library(), fn)(ctypes.byref(c), ctypes.byref(weights.c),
                                        ctypes.byref(cache.c), int(mode),
@@ -366,6 +380,7 @@ def cc_score_rows(cfg, weights, cache, mode, full: bool, row_lo, row_hi, scores,
     """Scores only rows [row_lo[b], row_hi[b]) of each sequence (device int32
     [batch] each, or both None for every row); every other entry of `scores`
     gets -inf, or keeps its value with SCORE_RANGE_ONLY in `mode`."""
+    _check_operand_type(weights, mode)
     code = load_library().cc_score_rows(
         ctypes.byref(_cfg(cfg)), ctypes.byref(weights.c), ctypes.byref(cache.c), int(mode),
         1 if full else 0, _dev_ptr(row_lo, "row_lo"), _dev_ptr(row_hi, "row_hi"),

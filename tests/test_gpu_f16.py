@@ -253,3 +253,22 @@ def test_f16_cache_layouts_match_slot_major(cc, layout):
         r = ref.cpu().numpy()
         err = max(rel_err(r[i, rw], want[i, rw]) for i, rw in enumerate(rows))
         assert err < TOL and err < 2e-3, err
+
+
+def test_binding_refuses_weights_of_the_other_operand_type(cc, tiny):
+    """The C ABI reads the same weight pointers as fp16 or bf16 by the mode;
+    the binding checks the tensors' dtype against it before the call."""
+    import paper_2607_27600_gb300 as pkg
+    wl, w_np, c_np = tiny
+    w_dev, c_dev = to_device(w_np), to_device(c_np)
+    b, cap = c_np["tokens"].shape
+    scores = torch.empty(b, cap, dtype=torch.float32, device="cuda")
+    ws = cc.alloc_workspace(cc.cc_score_workspace_size(wl.shape, b, cap, cc.SCORE_LOGIT))
+    cases = ((pkg.Weights(w_dev), cc.SCORE_LOGIT | cc.SCORE_F16),
+             (pkg.Weights(cc.f16_weights(w_dev)), cc.SCORE_LOGIT))
+    for weights, mode in cases:
+        with pytest.raises(ValueError):
+            cc.cc_score_layer(wl.shape, weights, pkg.Cache(c_dev), mode, scores, ws)
+        with pytest.raises(ValueError):
+            cc.cc_score_rows(wl.shape, weights, pkg.Cache(c_dev), mode, False, None, None, scores, ws)
+    assert cc.cc_get_status() == cc.CC_OK
