@@ -35,7 +35,8 @@ typedef enum {
   CC_KERNEL_APPEND = 15,     /* append bookkeeping: tokens, positions, H^(L-1)    */
   CC_KERNEL_GEMM_QKV = 16,   /* fused q/k/v projections (+ RoPE) of the append    */
   CC_KERNEL_KEYATTN = 17,    /* comparison scorers: attention received per key    */
-  CC_KERNEL_KV_DEQUANT = 18, /* a layer of an e4m3 cache as bf16 (tile attention) */
+  CC_KERNEL_KV_DEQUANT = 18, /* a layer's K/V copied for the tile attention: e4m3
+                                as bf16 or fp16, bf16 as fp16 (CC_SCORE_F16)        */
   CC_KERNEL_COUNT = 19
 } cc_kernel_kind;
 
