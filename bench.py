@@ -962,16 +962,30 @@ KERNEL_SOURCES = {
 }
 
 
-def kernel_digest(kernel):
-    """Hash of the sources of one kernel kind (e.g. gemm_gateup -> gemm.cu, ...)."""
+def code_tokens(text):
+    """C/CUDA source without its comments and with runs of whitespace
+    collapsed: what a change must touch to change the compiled code."""
+    import re
+    text = re.sub(r"/\*.*?\*/", " ", text, flags=re.S)
+    text = re.sub(r"//[^\n]*", " ", text)
+    return " ".join(text.split())
+
+
+def kernel_digest(kernel, read=None):
+    """Hash of the code (comments and layout ignored) of the sources of one
+    kernel kind (e.g. gemm_gateup -> gemm.cu, ...); `read(name)` returns a
+    source's text (default: the file under csrc/)."""
     import hashlib
     fam = ("gemm" if kernel.startswith("gemm") else "attention" if kernel.startswith("attention")
            else kernel if kernel in KERNEL_SOURCES else "rowops")
-    h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2607_27600_gb300", "csrc")
+    if read is None:
+        def read(name):
+            with open(os.path.join(csrc, name), encoding="utf-8") as fh:
+                return fh.read()
+    h = hashlib.sha256()
     for f in KERNEL_SOURCES[fam]:
-        with open(os.path.join(csrc, f), "rb") as fh:
-            h.update(f.encode() + fh.read())
+        h.update((f + "\n" + code_tokens(read(f))).encode())
     return h.hexdigest()[:16]
 
 

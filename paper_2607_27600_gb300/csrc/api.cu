@@ -1042,7 +1042,8 @@ cc_status run_score(const cc_model_cfg *c, const cc_model_weights *w, const cc_k
     if ((s = run_gemm(gq, EPI_QROPE, CC_KERNEL_GEMM_QROPE, dev->sms, st)) != CC_OK) return s;
     // O = counter-causal attention
     CC_TRY(wait_kv_ready(kv, l, l + 1, st));
-    // (act is free until the MLP: an e4m3 layer's bf16 copy for the tile attention)
+    // (act is free until the MLP: the layer's bf16 copy of an e4m3 cache, or its
+    // fp16 copy with fp16 operands, for the tile attention)
     if ((s = run_attention(c, q, kv->k[l], kv->v[l], o, kv->seq_len, batch, cap, status, st,
                            split, nullptr, 0, nullptr, 0, kv_fmt(c, kv, l), split_q, rng_lo,
                            rng_hi, act, (size_t)batch * cap * c->d_ff * 2 * (split ? 2 : 1),

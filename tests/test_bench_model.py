@@ -112,3 +112,16 @@ def test_e2e_row_blocks_cover_every_slot_once_on_key_tile_boundaries():
                 lo, hi = bounds[k][b], bounds[k + 1][b]
                 assert 0 <= lo <= hi <= n
                 assert lo % 128 == 0 or lo == n
+
+
+def test_kernel_digest_ignores_comments_not_code():
+    """The DRAM-traffic record stays valid through comment and layout edits
+    of a kernel's sources and goes stale on any code edit."""
+    import bench
+    src = {"gemm.cu": "int a = 1; // one\n/* block\n comment */ int b = a  +  2;\n",
+           "gemm.cuh": "", "cc_common.cuh": "", "api.cu": ""}
+    base = bench.kernel_digest("gemm_gateup", read=lambda f: src[f])
+    src["gemm.cu"] = "int a = 1;   // the first\nint b = a + 2; /* sum */\n"
+    assert bench.kernel_digest("gemm_gateup", read=lambda f: src[f]) == base
+    src["gemm.cu"] = "int a = 1;\nint b = a + 3;\n"
+    assert bench.kernel_digest("gemm_gateup", read=lambda f: src[f]) != base
