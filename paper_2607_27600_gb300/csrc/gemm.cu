@@ -30,7 +30,8 @@ namespace {
 // problems (less than one wave of 256-column tiles), 128.
 constexpr int BM = 128, BN = 256, BK = 64, ST = 4;
 // CTA pairs (one 256 x 256 product per pair, each CTA holding 128 A rows and
-// 128 B rows of a stage): 16 + 16 KB stages, six of them
+// 128 B rows of a k-block): 16 + 16 KB ring slots, six of them, which the
+// kernel fills and drains two per barrier stage
 constexpr int ST_PAIR = 6;
 constexpr int A_BYTES = BM * BK * 2;   // 16 KB
 constexpr int B_BYTES = BN * BK * 2;   // 32 KB: shared-memory stage of the widest B tile
