@@ -650,6 +650,13 @@ AppendWs append_layout(const cc_model_cfg *c, int batch, int cap) {
   return w;
 }
 
+// The tile attention over an e4m3 cache, or with fp16 operands, reads a
+// 2-byte copy of the layer's K and V made in the activation buffer: whether
+// it fits in `act_bytes` per slot.
+bool kv_copy_fits(const cc_model_cfg *c, uint64_t act_bytes) {
+  return 4ull * c->n_kv_heads * c->head_dim <= act_bytes;
+}
+
 cc_status check_append_args(const cc_model_cfg *c, const cc_model_weights *w,
                             const cc_kv_cache *kv, const int32_t *tokens_in,
                             const int32_t *count, int max_count, void *ws, size_t ws_bytes) {
@@ -663,6 +670,11 @@ cc_status check_append_args(const cc_model_cfg *c, const cc_model_weights *w,
     return CC_ERR_INVALID_ARG;
   if (kv->batch > gemm_max_batch()) return CC_ERR_UNSUPPORTED;
   if ((uint64_t)kv->batch * kv->cap >= (1ull << 31)) return CC_ERR_UNSUPPORTED;
+  // an e4m3 layer copied for the tile attention (chunks, or query groups the
+  // decode kernel does not take), checked before anything is enqueued
+  const bool tile_attn = max_count != 1 || c->n_q_heads / c->n_kv_heads > kDecMaxG;
+  if (kv->kv_format == CC_KV_E4M3 && tile_attn && !kv_copy_fits(c, 2ull * c->d_ff))
+    return CC_ERR_UNSUPPORTED;
   for (int l = 0; l < c->n_layers; ++l) {
     const cc_layer_weights &lw = w->layers[l];
     const void *ptrs[] = {lw.attn_norm, lw.wq, lw.wk, lw.wv, lw.wo, lw.mlp_norm, lw.w_gate,
@@ -939,6 +951,11 @@ cc_status check_score_args(const cc_model_cfg *c, const cc_model_weights *w, con
     return CC_ERR_INVALID_ARG;
   if (kv->batch > gemm_max_batch()) return CC_ERR_UNSUPPORTED;
   if ((uint64_t)kv->batch * kv->cap >= (1ull << 31)) return CC_ERR_UNSUPPORTED;
+  // the per-layer K/V copy of an e4m3 cache or of the fp16 mode, checked
+  // before anything is enqueued
+  if ((kv->kv_format == CC_KV_E4M3 || (mode & CC_SCORE_F16)) &&
+      !kv_copy_fits(c, 2ull * c->d_ff * ((mode & CC_SCORE_PRECISE) ? 2 : 1)))
+    return CC_ERR_UNSUPPORTED;
   if (full && !w->embed) return CC_ERR_INVALID_ARG;
   if (!full && !kv->h_last) return CC_ERR_INVALID_ARG;
   const int l0 = full ? 0 : c->n_layers - 1;

@@ -272,3 +272,32 @@ def test_binding_refuses_weights_of_the_other_operand_type(cc, tiny):
         with pytest.raises(ValueError):
             cc.cc_score_rows(wl.shape, weights, pkg.Cache(c_dev), mode, False, None, None, scores, ws)
     assert cc.cc_get_status() == cc.CC_OK
+
+
+def test_kv_copy_that_does_not_fit_is_refused_before_any_launch(cc):
+    """The per-layer K/V copy (fp16 mode, or an e4m3 cache) lives in the
+    activation buffer, 2 * d_ff bytes per slot: a shape whose K and V need
+    more (8 KV heads of 128 against d_ff 1024) is refused with
+    CC_ERR_UNSUPPORTED before anything is enqueued; the bf16 mode over the
+    bf16 cache takes it."""
+    import bench
+    import paper_2607_27600_gb300 as pkg
+    from synth.configs import ModelShape
+    shape = ModelShape(n_layers=1, d_model=256, n_q_heads=8, n_kv_heads=8, head_dim=128,
+                       d_ff=1024, vocab=1000, rope_theta=1e4, rms_eps=1e-5)
+    w = synth.model_weights(shape, 91, device="cuda")
+    c = synth.synthetic_cache(shape, [100], 128, 92, device="cuda")
+    c8 = bench.to_e4m3_cache(synth.synthetic_cache(shape, [100], 128, 92, device="cuda"))
+    ws = cc.alloc_workspace(cc.cc_score_workspace_size(shape, 1, 128, cc.SCORE_LOGIT))
+    cases = ((cc.f16_weights(w), c, cc.SCORE_LOGIT | cc.SCORE_F16),
+             (w, c8, cc.SCORE_LOGIT))
+    for weights, cache, mode in cases:
+        scores = torch.full((1, 128), float("nan"), device="cuda")
+        with pytest.raises(cc.CCError) as e:
+            cc.cc_score_layer(shape, pkg.Weights(weights), pkg.Cache(cache), mode, scores, ws)
+        assert e.value.code == cc.CC_ERR_UNSUPPORTED
+        assert torch.isnan(scores).all()   # nothing ran
+    assert cc.cc_get_status() == cc.CC_OK
+    scores = torch.empty(1, 128, device="cuda")
+    cc.cc_score_layer(shape, pkg.Weights(w), pkg.Cache(c), cc.SCORE_LOGIT, scores, ws)
+    assert cc.cc_get_status() == cc.CC_OK
