@@ -155,3 +155,34 @@ def test_binding_constants_match_the_headers(lib):
     names = [lib.cc_kernel_name(k).decode() for k in range(cc.KERNEL_COUNT)]
     assert len(set(names)) == cc.KERNEL_COUNT and "unknown" not in names
     assert lib.cc_kernel_name(cc.KERNEL_COUNT).decode() == "unknown"
+
+
+def test_bf16_to_f16_argument_checks_without_device(lib):
+    """cc_bf16_to_f16 refuses null, misaligned, overlapping and non-multiple-
+    of-8 arguments on the host (nothing reaches a device); n = 0 is a no-op."""
+    from paper_2607_27600_gb300 import cc
+    assert lib.cc_bf16_to_f16(None, None, 0, None) == cc.CC_OK
+    assert lib.cc_bf16_to_f16(None, None, 8, None) == cc.CC_ERR_INVALID_ARG
+    base = 1 << 20   # addresses only: none is dereferenced on these paths
+    assert lib.cc_bf16_to_f16(base, base + 4096, 12, None) == cc.CC_ERR_INVALID_ARG   # n % 8
+    assert lib.cc_bf16_to_f16(base + 2, base + 4096, 8, None) == cc.CC_ERR_INVALID_ARG  # align
+    assert lib.cc_bf16_to_f16(base, base + 16, 16, None) == cc.CC_ERR_INVALID_ARG     # overlap
+
+
+def test_binding_operand_type_check_without_device():
+    """The binding's dtype check of the layer matrices against the operand
+    mode (host logic: the CUDA tensors only carry the dtype)."""
+    import types
+
+    import torch
+    from paper_2607_27600_gb300 import cc
+    layer = {f: torch.zeros(8, 8, dtype=torch.bfloat16) for f in cc.F16_MATRICES}
+    w = types.SimpleNamespace(w={"layers": [None, layer]})
+    cc._check_operand_type(w, cc.SCORE_LOGIT)
+    cc._check_operand_type(w, cc.SCORE_LOGPROB | cc.SCORE_PRECISE)
+    with pytest.raises(ValueError):
+        cc._check_operand_type(w, cc.SCORE_LOGIT | cc.SCORE_F16)
+    w16 = types.SimpleNamespace(w={"layers": [{f: t.half() for f, t in layer.items()}]})
+    cc._check_operand_type(w16, cc.SCORE_LOGIT | cc.SCORE_F16)
+    with pytest.raises(ValueError):
+        cc._check_operand_type(w16, cc.SCORE_LOGIT)
