@@ -5,6 +5,10 @@ A step = one refresh of one synthetic cache: counter-causal scores of every
 cached position (fast single-layer approximation, or the full L-layer pass),
 keep-set selection at the budget, in-place compaction of every layer's K/V,
 H^(L-1), tokens and positions.  Metric: scored KV positions per second.
+The scoring pass runs with fp16 tensor-core operands (CC_SCORE_F16: the
+fastest mode that holds the full 32-layer pass to the stated tolerance; the
+layer weights are converted once before the timed steps) unless --bf16 or
+--precise names another operand mode.
 
     python bench.py [--gpus N --steps K --warmup W] [--workload NAME] [--impl reference]
 
